@@ -1,0 +1,218 @@
+/*
+ * dpo_oracle.c -- plain CPU oracle of the one-step-delayed AdamW step with
+ * update-level Error Feedback (arXiv 2606.30634).
+ *
+ * TEST INFRASTRUCTURE. Loaded only by the tests, the package smoke check and
+ * the benchmark's CPU-baseline leg; the product library never uses it.
+ *
+ * The code follows the paper's statement step by step, one element at a
+ * time, in double precision, with no fusion or reordering: see the header
+ * for the passages each step comes from. The element loop may run on several
+ * OpenMP threads; every element is independent, so the result does not depend
+ * on the thread count. Sums run in a fixed order.
+ */
+#include "dpo_oracle.h"
+
+#include <math.h>
+#include <stddef.h>
+#include <stdlib.h>
+#include <string.h>
+
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+int oracle_num_threads(void)
+{
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+/* bf16: 8 significant bits, the exponent range of fp32. Round half to even
+ * on the value's own ulp; below 2^-126 the ulp is fixed at 2^-133. */
+static double round_bf16(double x)
+{
+    if (isnan(x) || isinf(x) || x == 0.0)
+        return x;
+    int e;
+    (void)frexp(fabs(x), &e);          /* |x| = f * 2^e, f in [0.5, 1) */
+    if (e < -125)
+        e = -125;                      /* subnormal range: ulp 2^-133 */
+    double q = ldexp(fabs(x), 8 - e);  /* |x| in units of one bf16 ulp */
+    q = nearbyint(q);                  /* default mode: ties to even */
+    double r = ldexp(q, e - 8);
+    if (r >= 0x1p128)
+        r = INFINITY;
+    return copysign(r, x);
+}
+
+double oracle_round(double x, int store)
+{
+    switch (store) {
+    case ORACLE_F32:
+        return (double)(float)x;
+    case ORACLE_BF16:
+        return round_bf16(x);
+    default:
+        return x;
+    }
+}
+
+void oracle_round_n(int64_t n, const double *in, double *out, int store)
+{
+    for (int64_t i = 0; i < n; ++i)
+        out[i] = oracle_round(in[i], store);
+}
+
+int oracle_step(int64_t n, int64_t k, const oracle_hparams *hp,
+                const double *g, double clip_scale, const uint8_t *wd_on,
+                double *x, double *m, double *v, double *u_prev,
+                double *stash, double *param)
+{
+    if (n < 0 || k < 1 || hp == NULL || (n > 0 && (g == NULL || x == NULL)))
+        return -1;
+    if (hp->rule == ORACLE_RULE_ADAMW && n > 0 && (m == NULL || v == NULL))
+        return -1;
+    if (hp->delay == 1 && n > 0 && stash == NULL)
+        return -1;
+
+    /* Error Feedback is active for delayed training with an EF buffer; the
+     * lambda-scaled form reduces to the standard rule at lambda = 0. */
+    const int use_ef = (hp->delay == 1 && u_prev != NULL);
+    /* Alg. 1: the standard rule is used for t <= 1 even under EF; call k is
+     * iteration t = k. */
+    const int ef_now = use_ef && k >= 2;
+    const double lam = hp->ef_lambda;
+
+    /* Bias corrections of Adam at the k-th gradient. */
+    const double bc1 = 1.0 - pow(hp->beta1, (double)k);
+    const double bc2 = 1.0 - pow(hp->beta2, (double)k);
+
+#pragma omp parallel for schedule(static)
+    for (int64_t i = 0; i < n; ++i) {
+        const double gi = clip_scale * g[i];
+        const double wd = (wd_on == NULL || wd_on[i]) ? hp->weight_decay : 0.0;
+        const double xt = x[i];
+
+        /* Update the optimizer statistics with g_{t-1} and form u_{t-1}. */
+        double u;
+        if (hp->rule == ORACLE_RULE_ADAMW) {
+            const double mi = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;
+            const double vi = hp->beta2 * v[i] + (1.0 - hp->beta2) * gi * gi;
+            const double m_hat = mi / bc1;
+            const double v_hat = vi / bc2;
+            u = hp->lr * (m_hat / (sqrt(v_hat) + hp->eps) + wd * xt);
+            m[i] = oracle_round(mi, hp->x_store);
+            v[i] = oracle_round(vi, hp->x_store);
+        } else {
+            u = hp->lr * (gi + wd * xt);
+        }
+
+        /* Apply it: standard delayed rule, or the EF correction. */
+        double xn;
+        if (!ef_now)
+            xn = xt - u;
+        else
+            xn = xt - u - lam * (u - u_prev[i]);
+
+        if (use_ef)
+            u_prev[i] = oracle_round(u, hp->x_store);
+        /* The stash keeps the pre-update weights x_t: the version the next
+         * gradient is evaluated at (one step behind the latest). */
+        if (hp->delay == 1)
+            stash[i] = oracle_round(xt, hp->stash_store);
+        x[i] = oracle_round(xn, hp->x_store);
+        if (param != NULL)
+            param[i] = oracle_round(x[i], hp->param_store);
+    }
+    return 0;
+}
+
+#define ORACLE_SUM_BLOCK 65536
+
+/* Fixed-order sum of squares: per-block sums (blocks may run on different
+ * threads), then the block sums added left to right. */
+#define DEFINE_SQNORM(NAME, T, WIDEN)                                       \
+    double NAME(int64_t n, const T *g)                                      \
+    {                                                                       \
+        if (n <= 0)                                                         \
+            return 0.0;                                                     \
+        const int64_t nb = (n + ORACLE_SUM_BLOCK - 1) / ORACLE_SUM_BLOCK;   \
+        double total = 0.0;                                                 \
+        double *part = (double *)malloc(sizeof(double) * (size_t)nb);       \
+        if (part == NULL)                                                   \
+            return NAN;                                                     \
+        _Pragma("omp parallel for schedule(static)")                        \
+        for (int64_t b = 0; b < nb; ++b) {                                  \
+            const int64_t lo = b * ORACLE_SUM_BLOCK;                        \
+            const int64_t hi = lo + ORACLE_SUM_BLOCK < n ? lo + ORACLE_SUM_BLOCK : n; \
+            double s = 0.0;                                                 \
+            for (int64_t i = lo; i < hi; ++i) {                             \
+                const double gi = WIDEN(g[i]);                              \
+                s += gi * gi;                                               \
+            }                                                               \
+            part[b] = s;                                                    \
+        }                                                                   \
+        for (int64_t b = 0; b < nb; ++b)                                    \
+            total += part[b];                                               \
+        free(part);                                                         \
+        return total;                                                       \
+    }
+
+static double widen_f64(double g) { return g; }
+static double widen_f32(float g) { return (double)g; }
+/* A bf16 bit pattern is the upper half of the fp32 with the same value. */
+static double widen_bf16(uint16_t bits)
+{
+    uint32_t w = (uint32_t)bits << 16;
+    float f;
+    memcpy(&f, &w, sizeof f);
+    return (double)f;
+}
+
+DEFINE_SQNORM(oracle_sqnorm, double, widen_f64)
+DEFINE_SQNORM(oracle_sqnorm_f32, float, widen_f32)
+DEFINE_SQNORM(oracle_sqnorm_bf16, uint16_t, widen_bf16)
+
+/* Global-norm clipping (App. E.1 uses a threshold of 1.0): the coefficient
+ * is clamped at 1 and 1e-6 is added to the norm. */
+double oracle_clip_coef(double sqnorm, double max_norm)
+{
+    if (!(max_norm > 0.0))
+        return 1.0;
+    const double coef = max_norm / (sqrt(sqnorm) + 1e-6);
+    return coef < 1.0 ? coef : 1.0;
+}
+
+double oracle_quadratic(int64_t n, const double *a, const double *wstar,
+                        const double *w, const double *noise, int store,
+                        double *grad_out)
+{
+    if (n <= 0)
+        return 0.0;
+    const int64_t nb = (n + ORACLE_SUM_BLOCK - 1) / ORACLE_SUM_BLOCK;
+    double *part = (double *)malloc(sizeof(double) * (size_t)nb);
+    if (part == NULL)
+        return NAN;
+#pragma omp parallel for schedule(static)
+    for (int64_t b = 0; b < nb; ++b) {
+        const int64_t lo = b * ORACLE_SUM_BLOCK;
+        const int64_t hi = lo + ORACLE_SUM_BLOCK < n ? lo + ORACLE_SUM_BLOCK : n;
+        double s = 0.0;
+        for (int64_t i = lo; i < hi; ++i) {
+            const double d = w[i] - wstar[i];
+            if (grad_out != NULL)
+                grad_out[i] = oracle_round(a[i] * d + (noise ? noise[i] : 0.0), store);
+            s += a[i] * d * d;
+        }
+        part[b] = s;
+    }
+    double total = 0.0;
+    for (int64_t b = 0; b < nb; ++b)
+        total += part[b];
+    free(part);
+    return 0.5 * total;
+}

@@ -1,0 +1,117 @@
+/*
+ * dpo_oracle.h -- plain CPU oracle of the one-step-delayed optimizer step.
+ *
+ * TEST INFRASTRUCTURE. Only the tests, the package smoke check and the CPU
+ * baseline leg of the benchmark load this library. The product library
+ * (libdpo) never links, loads or calls it, and the two share no code.
+ *
+ * Method (arXiv 2606.30634, "One-Step Gradient Delay is Not a Barrier for
+ * Large-Scale Asynchronous Pipeline Parallel LLM Pretraining"):
+ *   Alg. 1 (Delayed Gradient Update), Sec. 2: at iteration t the optimizer
+ *     statistics are updated with the stale gradient g_{t-1}, the step
+ *     u_{t-1}(g_{t-1}) is formed, and
+ *        x_{t+1} = x_t - u_{t-1}                       (standard, or t <= 1)
+ *        x_{t+1} = x_t - 2 u_{t-1} + u_{t-2}           (Error Feedback)
+ *   Eq. (1), Sec. 3.2: the Error-Feedback update above.
+ *   App. A.4 (Error Feedback Coefficient Ablation): the lambda-scaled form
+ *        x_{t+1} = x_t - u_{t-1} - lambda (u_{t-1} - u_{t-2}),
+ *     lambda = 0 standard delayed training, lambda = 1 Eq. (1).
+ *   u is AdamW with beta = (0.9, 0.95) (Sec. 2.1), EMA convention
+ *     m_t = beta m_{t-1} + (1 - beta) g_t (Sec. 2.2), decoupled weight decay
+ *     on the current iterate x_t (Alg. 2: U_{t-1} = eta (O_{t-1} + lambda X_t)),
+ *     and global gradient-norm clipping at 1.0 (Sec. 2, App. E.1).
+ *
+ * Every arithmetic operation is done in double. After each step every state
+ * buffer is rounded to its storage format (double: no rounding; fp32; bf16
+ * round-to-nearest-even from the fp32 master), exactly as a GPU holding the
+ * same buffers in those formats would store them.
+ */
+#ifndef DPO_ORACLE_H
+#define DPO_ORACLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Storage formats of the state buffers. */
+enum { ORACLE_F64 = 0, ORACLE_F32 = 1, ORACLE_BF16 = 2 };
+
+/* Update rules u. ADAMW is the method's optimizer. SGD (u = lr * g) exists
+ * only so that tests can check the delay/EF driver of Alg. 1 apart from Adam. */
+enum { ORACLE_RULE_ADAMW = 0, ORACLE_RULE_SGD = 1 };
+
+typedef struct {
+    double lr;            /* learning rate eta of the call */
+    double beta1, beta2;  /* EMA coefficients of m and v */
+    double eps;           /* added to sqrt(v_hat) */
+    double weight_decay;  /* decoupled decay coefficient */
+    double ef_lambda;     /* lambda of the EF correction; 0 = standard */
+    int delay;            /* 1 = one-step-delayed (Alg. 1), 0 = synchronous */
+    int rule;             /* ORACLE_RULE_* */
+    int x_store;          /* storage of master x, m, v and u_prev (F64 or F32) */
+    int stash_store;      /* storage of the stash (F64, F32 or BF16) */
+    int param_store;      /* storage of the latest-weights copy (F64, F32, BF16) */
+} oracle_hparams;
+
+/*
+ * One call of the delayed step over n elements (one flat tensor or the
+ * concatenation of several; the step is elementwise).
+ *
+ *   k          number of stale gradients consumed including this one (>= 1);
+ *              the first call is Alg. 1 iteration t = 1, because t = 0 only
+ *              sets x_1 = x_0 (u_{-1} = 0).
+ *   g          the gradient evaluated at the stash (the stale weights), as
+ *              doubles holding values of the gradient storage format.
+ *   clip_scale multiplier applied to g (1 when clipping is off), from
+ *              oracle_clip_coef().
+ *   wd_on      per-element 0/1 mask for weight decay, or NULL (decay on all).
+ *   x, m, v    master weights and Adam moments, updated in place.
+ *   u_prev     EF buffer, holding u_{t-2} on entry and u_{t-1} on return.
+ *              NULL selects the standard delayed rule (no Error Feedback);
+ *              with a buffer and delay == 1 the lambda-scaled EF rule runs
+ *              (lambda = 0 then gives the standard result).
+ *   stash      receives x_t, the weights the next gradient is evaluated at;
+ *              may be NULL when delay == 0 (the latest weights are read).
+ *   param      receives the new latest weights x_{t+1}, or NULL.
+ *
+ * Returns 0, or -1 on an invalid argument.
+ */
+int oracle_step(int64_t n, int64_t k, const oracle_hparams *hp,
+                const double *g, double clip_scale, const uint8_t *wd_on,
+                double *x, double *m, double *v, double *u_prev,
+                double *stash, double *param);
+
+/* Sum of g_i^2 in double over n elements (fixed order: blocks of 65536
+ * elements summed left to right, block sums added left to right). */
+double oracle_sqnorm(int64_t n, const double *g);
+
+/* Same, with the gradient given as bf16 bit patterns or as fp32 values. */
+double oracle_sqnorm_bf16(int64_t n, const uint16_t *g_bits);
+double oracle_sqnorm_f32(int64_t n, const float *g);
+
+/* Clip coefficient min(1, max_norm / (sqrt(sqnorm) + 1e-6)); 1 when
+ * max_norm <= 0 (clipping off). */
+double oracle_clip_coef(double sqnorm, double max_norm);
+
+/* Number of threads the element loops use (OpenMP), 1 without OpenMP. */
+int oracle_num_threads(void);
+
+/* Round a value to a storage format (ORACLE_F64 / F32 / BF16). */
+double oracle_round(double x, int store);
+/* out[i] = oracle_round(in[i], store) for i < n (in and out may alias). */
+void oracle_round_n(int64_t n, const double *in, double *out, int store);
+
+/* Quadratic workload f(w) = 1/2 sum a_i (w_i - w*_i)^2 (the noisy diagonal
+ * quadratic used to emulate delayed training):
+ *   grad_i = a_i (w_i - wstar_i) + noise_i, rounded to `store`;
+ *   returns the loss 1/2 sum a_i (w_i - wstar_i)^2 at w. */
+double oracle_quadratic(int64_t n, const double *a, const double *wstar,
+                        const double *w, const double *noise, int store,
+                        double *grad_out);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* DPO_ORACLE_H */

@@ -1,0 +1,25 @@
+import os
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+
+def pytest_configure(config):
+    config.addinivalue_line(
+        "markers", "gpu: needs a CUDA GPU (sm_103a); run with -m gpu")
+    config.addinivalue_line(
+        "markers", "slow: full-size parity case (minutes)")
+
+
+@pytest.fixture(scope="session")
+def cuda_device():
+    """The GPU the parity tests run on; a GPU test without one is an error,
+    not a skip."""
+    import torch
+    if not torch.cuda.is_available():
+        pytest.fail("GPU test collected on a machine without CUDA")
+    return torch.device("cuda:0")

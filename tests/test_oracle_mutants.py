@@ -1,0 +1,77 @@
+"""The oracle's pins catch plausible mistakes.
+
+Each case copies ``oracle/dpo_oracle.c``, plants one mistake in the copy (a
+dropped term, a wrong sign or index, swapped operands, a misread passage),
+builds it into a temporary library, and runs ``test_oracle_pins.py`` against
+that build. Every planted mistake must make at least one pin fail. Nothing
+here touches the committed oracle or any GPU.
+"""
+from __future__ import annotations
+
+import os
+import subprocess
+import sys
+from concurrent.futures import ThreadPoolExecutor
+
+import pytest
+
+from oracle import build as oracle_build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+# (name, text in dpo_oracle.c, replacement)
+MUTANTS = [
+    ("decay_on_stale_copy", "hp->eps) + wd * xt)",
+     "hp->eps) + wd * (stash != NULL ? stash[i] : xt))"),
+    ("eps_inside_sqrt", "(sqrt(v_hat) + hp->eps)", "sqrt(v_hat + hp->eps)"),
+    ("ef_sign_flipped", "xn = xt - u - lam * (u - u_prev[i]);",
+     "xn = xt - u + lam * (u - u_prev[i]);"),
+    ("ef_at_first_update", "use_ef && k >= 2", "use_ef && k >= 1"),
+    ("bias_correction_index", "pow(hp->beta1, (double)k)", "pow(hp->beta1, (double)(k + 1))"),
+    ("no_bias_correction_m", "const double m_hat = mi / bc1;", "const double m_hat = mi;"),
+    ("stash_holds_new_weights", "stash[i] = oracle_round(xt, hp->stash_store);",
+     "stash[i] = oracle_round(xn, hp->stash_store);"),
+    ("v_from_momentum", "(1.0 - hp->beta2) * gi * gi", "(1.0 - hp->beta2) * gi * mi"),
+    ("ema_roles_swapped", "hp->beta1 * m[i] + (1.0 - hp->beta1) * gi",
+     "(1.0 - hp->beta1) * m[i] + hp->beta1 * gi"),
+    ("ef_stores_displacement", "u_prev[i] = oracle_round(u, hp->x_store);",
+     "u_prev[i] = oracle_round(xt - xn, hp->x_store);"),
+    ("clip_not_applied", "const double gi = clip_scale * g[i];", "const double gi = g[i];"),
+    ("clip_no_epsilon", "(sqrt(sqnorm) + 1e-6)", "sqrt(sqnorm)"),
+    ("bf16_ties_away", "q = nearbyint(q);", "q = round(q);"),
+    ("bf16_subnormal_quantum", "if (e < -125)\n        e = -125;", "if (e < -126)\n        e = -126;"),
+    ("decay_ignores_mask", "(wd_on == NULL || wd_on[i])", "(1)"),
+]
+
+
+def _build_mutant(tmp_path, name, old, new):
+    src = open(oracle_build.SRC).read()
+    assert src.count(old) == 1, f"mutation site for {name} not unique"
+    path = tmp_path / f"{name}.c"
+    path.write_text(src.replace(old, new))
+    return oracle_build.build(force=True, src=str(path),
+                              out=str(tmp_path / f"lib{name}.so"))
+
+
+def _run_pins(lib_path):
+    env = dict(os.environ, DPO_ORACLE_LIB=lib_path, OMP_NUM_THREADS="1")
+    r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
+                        os.path.join(ROOT, "tests", "test_oracle_pins.py")],
+                       cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+    return r.returncode, r.stdout[-600:]
+
+
+def test_every_planted_mistake_fails_a_pin(tmp_path):
+    libs = [(name, _build_mutant(tmp_path, name, old, new)) for name, old, new in MUTANTS]
+    with ThreadPoolExecutor(max_workers=min(8, os.cpu_count() or 1)) as ex:
+        results = list(ex.map(lambda nl: (nl[0],) + _run_pins(nl[1]), libs))
+    survivors = [(n, out) for n, rc, out in results if rc == 0]
+    assert not survivors, f"mistakes no pin caught: {[n for n, _ in survivors]}"
+    # exit code 1 = tests failed (not a collection or usage error)
+    assert all(rc == 1 for _, rc, _ in results), results
+
+
+def test_unmutated_copy_passes(tmp_path):
+    lib = _build_mutant(tmp_path, "identity", "int oracle_step(", "int oracle_step(")
+    rc, out = _run_pins(lib)
+    assert rc == 0, out

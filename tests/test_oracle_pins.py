@@ -1,0 +1,444 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+None of these compares the oracle with itself: each expected value comes from
+a library routine (torch.optim.AdamW, torch's bf16 cast), exact rational
+arithmetic on a worked example, a closed-form trajectory, or an invariant that
+the update rule implies. ``test_oracle_mutants.py`` plants single mistakes in
+a copy of the oracle and checks that these pins catch each one.
+
+Paper passages (arXiv 2606.30634): Alg. 1 (delayed update, standard rule for
+t <= 1), Eq. (1) of Sec. 3.2 (Error Feedback), App. A.4 (lambda-scaled EF),
+App. B.1 (SAPipe weight prediction has EF's displacement), Alg. 2 (decay on
+X_t), Sec. 2.1 / App. E.1 (AdamW beta = (0.9, 0.95), wd 0.1, clip 1.0).
+"""
+from __future__ import annotations
+
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from oracle import BF16, F32, F64, HParams
+
+pytestmark = pytest.mark.filterwarnings("ignore::DeprecationWarning")
+
+
+@pytest.fixture
+def lib():
+    """The oracle under test: the default build, or (when DPO_ORACLE_LIB
+    names one) a build with a planted mistake from test_oracle_mutants."""
+    path = os.environ.get("DPO_ORACLE_LIB")
+    return oracle.load(path) if path else oracle.load()
+
+
+# ---------------------------------------------------------------- P1 ------
+# Delay-free application of the AdamW rule equals torch.optim.AdamW.
+
+def _torch_adamw_run(x0s, grads, hp: HParams, lrs, max_norm=0.0):
+    ps = [torch.nn.Parameter(torch.tensor(x, dtype=torch.float64)) for x in x0s]
+    opt = torch.optim.AdamW(ps, lr=lrs[0], betas=(hp.beta1, hp.beta2),
+                            eps=hp.eps, weight_decay=hp.weight_decay,
+                            foreach=False, fused=False)
+    traj = []
+    for gs, lr in zip(grads, lrs):
+        for p, g in zip(ps, gs):
+            p.grad = torch.tensor(g, dtype=torch.float64)
+        if max_norm > 0:
+            torch.nn.utils.clip_grad_norm_(ps, max_norm)
+        for group in opt.param_groups:
+            group["lr"] = lr
+        opt.step()
+        traj.append(np.concatenate([p.detach().numpy().ravel() for p in ps]))
+    return traj
+
+
+def _oracle_run(lib, x0s, grads, hp: HParams, lrs, ef=False):
+    o = oracle.DelayedOptimizer(x0s, hp, ef=ef, x_store=F64, stash_store=F64,
+                                lib=lib)
+    traj = []
+    for gs, lr in zip(grads, lrs):
+        o.step(np.concatenate([np.ravel(g) for g in gs]), lr=lr)
+        traj.append(o.x.copy())
+    return traj, o
+
+
+def _rel(a, b):
+    return np.max(np.abs(a - b) / np.maximum(np.abs(b), 1e-300))
+
+
+@pytest.mark.parametrize("delay", [0, 1])
+@pytest.mark.parametrize("max_norm", [0.0, 1.0])
+def test_p1_matches_torch_adamw(lib, delay, max_norm):
+    """Applying the given gradient sequence, the oracle's weights equal
+    torch.optim.AdamW's (delay changes only where gradients are evaluated,
+    not the arithmetic of the update). Includes clipping at 1.0 against
+    torch.nn.utils.clip_grad_norm_ and a changing learning rate."""
+    rng = np.random.default_rng(7)
+    shapes = [(5, 3), (7,), (1,)]
+    x0s = [rng.normal(0, 0.5, s) for s in shapes]
+    grads = [[rng.normal(0, 0.7, s) for s in shapes] for _ in range(12)]
+    lrs = [1e-2 * (1 + 0.1 * i) for i in range(12)]
+    hp = HParams(lr=lrs[0], beta1=0.9, beta2=0.95, eps=1e-8, weight_decay=0.1,
+                 max_grad_norm=max_norm, delay=delay)
+    ref = _torch_adamw_run(x0s, grads, hp, lrs, max_norm)
+    got, _ = _oracle_run(lib, x0s, grads, hp, lrs)
+    for r, g in zip(ref, got):
+        assert _rel(g, r) < 1e-12
+
+
+def test_p1_other_betas_and_eps(lib):
+    """Same pin away from the paper's constants, so a swapped beta or a
+    misplaced eps cannot hide behind them."""
+    rng = np.random.default_rng(11)
+    x0s = [rng.normal(0, 1, (9,))]
+    grads = [[rng.normal(0, 1e-3, (9,))] for _ in range(6)]
+    hp = HParams(lr=0.05, beta1=0.5, beta2=0.7, eps=1e-3, weight_decay=0.3,
+                 delay=0)
+    lrs = [0.05] * 6
+    ref = _torch_adamw_run(x0s, grads, hp, lrs)
+    got, _ = _oracle_run(lib, x0s, grads, hp, lrs)
+    for r, g in zip(ref, got):
+        assert _rel(g, r) < 1e-12
+
+
+# ---------------------------------------------------------------- P2 ------
+# Hand-worked example: scalar x0 = 1, beta = (0.9, 0.95), lr = 0.1, stale
+# gradients 2, 1, -0.5. By hand:
+#   k=1: m = 0.2,   v = 0.2,    1-b1^k = 0.1,   1-b2^k = 0.05     -> m_hat = 2, v_hat = 4
+#   k=2: m = 0.28,  v = 0.24,   1-b1^k = 0.19,  1-b2^k = 0.0975
+#   k=3: m = 0.202, v = 0.2405, 1-b1^k = 0.271, 1-b2^k = 0.142625
+# Alg. 1 uses the standard rule at the first update in both modes; EF then
+# applies x - 2u + u_prev (Eq. (1)).
+
+_HAND_MV = [(0.2, 0.2, 0.1, 0.05), (0.28, 0.24, 0.19, 0.0975),
+            (0.202, 0.2405, 0.271, 0.142625)]
+
+
+@pytest.mark.parametrize("ef", [False, True])
+def test_p2_hand_steps_no_decay(lib, ef):
+    """eps = 0, wd = 0: u1 = lr sign(g) = 0.1 (Adam's first step)."""
+    u1 = 0.1
+    u2 = 0.1 * (0.28 / 0.19) / math.sqrt(0.24 / 0.0975)
+    u3 = 0.1 * (0.202 / 0.271) / math.sqrt(0.2405 / 0.142625)
+    if ef:
+        x = [1 - u1, 1 - u1 - 2 * u2 + u1]
+        x.append(x[1] - 2 * u3 + u2)
+    else:
+        x = [1 - u1, 1 - u1 - u2, 1 - u1 - u2 - u3]
+    assert abs(u2 - 0.0939293068293407) < 1e-15   # worked by hand
+    hp = HParams(lr=0.1, beta1=0.9, beta2=0.95, eps=0.0, weight_decay=0.0,
+                 ef_lambda=1.0 if ef else 0.0)
+    o = oracle.DelayedOptimizer([np.array([1.0])], hp, ef=ef, x_store=F64,
+                                stash_store=F64, lib=lib)
+    for k, (g, u) in enumerate(zip([2.0, 1.0, -0.5], [u1, u2, u3])):
+        w, tag = o.read_weights("stale")
+        o.step(np.array([g]), tag=tag)
+        mk, vk, _, _ = _HAND_MV[k]
+        assert o.m[0] == pytest.approx(mk, rel=1e-15)
+        assert o.v[0] == pytest.approx(vk, rel=1e-15)
+        assert o.x[0] == pytest.approx(x[k], rel=1e-14)
+        if ef:
+            assert o.u_prev[0] == pytest.approx(u, rel=1e-14)
+
+
+@pytest.mark.parametrize("ef", [False, True])
+def test_p2_hand_steps_with_decay(lib, ef):
+    """wd = 0.1, eps = 1e-8: the decay term acts on the current master x_t
+    (Alg. 2), not on the stale copy the gradient was evaluated at."""
+    x1 = 1.0 - 0.1 * (2.0 / (2.0 + 1e-8) + 0.1 * 1.0)
+    u1 = 1.0 - x1
+    u2 = 0.1 * ((0.28 / 0.19) / (math.sqrt(0.24 / 0.0975) + 1e-8) + 0.1 * x1)
+    x2 = x1 - 2 * u2 + u1 if ef else x1 - u2
+    u3 = 0.1 * ((0.202 / 0.271) / (math.sqrt(0.2405 / 0.142625) + 1e-8) + 0.1 * x2)
+    x3 = x2 - 2 * u3 + u2 if ef else x2 - u3
+    hp = HParams(lr=0.1, beta1=0.9, beta2=0.95, eps=1e-8, weight_decay=0.1,
+                 ef_lambda=1.0 if ef else 0.0)
+    o = oracle.DelayedOptimizer([np.array([1.0])], hp, ef=ef, x_store=F64,
+                                stash_store=F64, lib=lib)
+    for g, xk in zip([2.0, 1.0, -0.5], [x1, x2, x3]):
+        o.step(np.array([g]), tag=o.read_weights()[1])
+        assert o.x[0] == pytest.approx(xk, rel=1e-14)
+
+
+# ---------------------------------------------------------------- P3 ------
+
+@pytest.mark.parametrize("ef", [False, True])
+@pytest.mark.parametrize("c", [0.3, -2.0, 3e-9])
+def test_p3_constant_gradient_no_decay(lib, ef, c):
+    """Constant gradient c, wd = 0: m_hat = c and v_hat = c^2 at every step,
+    so u = lr c / (|c| + eps) and x_n = x_0 - n u in both modes (EF is the
+    identity for a constant update: -2u + u = -u)."""
+    lr, eps, n = 1e-2, 1e-8, 40
+    hp = HParams(lr=lr, eps=eps, weight_decay=0.0, ef_lambda=1.0 if ef else 0.0)
+    o = oracle.DelayedOptimizer([np.array([0.7])], hp, ef=ef, x_store=F64,
+                                stash_store=F64, lib=lib)
+    u = lr * c / (abs(c) + eps)
+    for i in range(1, n + 1):
+        o.step(np.array([c]))
+        assert o.x[0] == pytest.approx(0.7 - i * u, rel=1e-12, abs=1e-14)
+
+
+def _linear_recurrence_closed_form(coeffs, init, n):
+    """Closed form of e_{j+1} = sum_i coeffs[i] e_{j-i} from the roots of its
+    characteristic polynomial (distinct roots), fitted to ``init``."""
+    order = len(coeffs)
+    poly = np.concatenate([[1.0], -np.asarray(coeffs, dtype=float)])
+    roots = np.roots(poly)
+    V = np.array([[r ** j for r in roots] for j in range(order)], dtype=complex)
+    amp = np.linalg.solve(V, np.asarray(init[:order], dtype=complex))
+    return np.array([np.real(np.sum(amp * roots ** j)) for j in range(n)])
+
+
+@pytest.mark.parametrize("ef", [False, True])
+def test_p3_constant_gradient_with_decay(lib, ef):
+    """Constant c, wd > 0, a = lr wd, s = c/(|c|+eps), fixed point
+    x* = -s/wd. Standard: e_{n+1} = (1-a) e_n. EF: e_1 = (1-a) e_0 (first
+    update is standard), then e_{n+1} = (1-2a) e_n + a e_{n-1}; its closed
+    form comes from the roots of r^2 - (1-2a) r - a."""
+    lr, wd, eps, c, x0, n = 0.05, 0.4, 1e-8, 0.8, 1.5, 60
+    a = lr * wd
+    s = c / (abs(c) + eps)
+    xstar = -s / wd
+    e0 = x0 - xstar
+    if ef:
+        e = _linear_recurrence_closed_form([1 - 2 * a, a], [e0, (1 - a) * e0], n + 1)
+    else:
+        e = np.array([e0 * (1 - a) ** j for j in range(n + 1)])
+    hp = HParams(lr=lr, eps=eps, weight_decay=wd, ef_lambda=1.0 if ef else 0.0)
+    o = oracle.DelayedOptimizer([np.array([x0])], hp, ef=ef, x_store=F64,
+                                stash_store=F64, lib=lib)
+    for j in range(1, n + 1):
+        o.step(np.array([c]))
+        assert o.x[0] - xstar == pytest.approx(e[j], rel=1e-10, abs=1e-12)
+
+
+def test_p3_sign_regime_switch_is_one_call_late(lib):
+    """beta1 = beta2 = 0, eps = 0, wd = 0: u = lr sign(g). On the quadratic
+    a/2 (x - x*)^2 started above x*, x_n = x_0 - n lr while the gradient is
+    positive. The gradient is evaluated at the stash, one version behind, so
+    the first upward step comes exactly one call later than without delay."""
+    lr, x0, xstar, a = 0.1, 1.0, 0.53, 2.0
+
+    def run(delay):
+        hp = HParams(lr=lr, beta1=0.0, beta2=0.0, eps=0.0, weight_decay=0.0,
+                     delay=delay)
+        o = oracle.DelayedOptimizer([np.array([x0])], hp, x_store=F64,
+                                    stash_store=F64, lib=lib)
+        xs = [x0]
+        for _ in range(12):
+            w, tag = o.read_weights("stale")
+            g, _ = oracle.quadratic([a], [xstar], w, None, F64, lib=lib)
+            o.step(g, tag=tag)
+            xs.append(o.x[0])
+        return np.array(xs)
+
+    sync, delayed = run(0), run(1)
+    flip = lambda xs: int(np.argmax(np.diff(xs) > 0)) + 1
+    # Without delay the gradient at x_{n-1} turns negative once x_{n-1} < x*.
+    k_sync = next(k for k in range(1, 20) if x0 - (k - 1) * lr < xstar)
+    assert flip(sync) == k_sync
+    assert flip(delayed) == k_sync + 1
+    for xs, kf in ((sync, k_sync), (delayed, k_sync + 1)):
+        np.testing.assert_allclose(xs[:kf], x0 - lr * np.arange(kf), rtol=0, atol=1e-14)
+
+
+@pytest.mark.parametrize("ef", [False, True])
+def test_p3_sgd_driver_closed_form(lib, ef):
+    """Alg. 1 driver with the test-only rule u = eta g on f = a/2 x^2, so
+    g_{t-1} = a x_{t-1}. Standard: x_{t+1} = x_t - eta a x_{t-1}, roots of
+    r^2 - r + eta a. EF: x_{t+1} = x_t - 2 eta a x_{t-1} + eta a x_{t-2},
+    roots of r^3 - r^2 + 2 eta a r - eta a. Initial values x_0 = x_1 and
+    x_2 = (1 - eta a) x_0 (the first update is standard)."""
+    eta, a, x0, n = 0.3, 0.25, 1.0, 50
+    q = eta * a
+    if ef:
+        e = _linear_recurrence_closed_form([1.0, -2 * q, q], [x0, x0, (1 - q) * x0], n + 2)
+    else:
+        e = _linear_recurrence_closed_form([1.0, -q], [x0, x0], n + 2)
+    hp = HParams(lr=eta, weight_decay=0.0, rule=oracle.RULE_SGD,
+                 ef_lambda=1.0 if ef else 0.0)
+    o = oracle.DelayedOptimizer([np.array([x0])], hp, ef=ef, x_store=F64,
+                                stash_store=F64, lib=lib)
+    for t in range(1, n + 1):
+        w, tag = o.read_weights("stale")
+        g, _ = oracle.quadratic([a], [0.0], w, None, F64, lib=lib)
+        o.step(g, tag=tag)
+        # after call t the master holds x_{t+1}
+        assert o.x[0] == pytest.approx(e[t + 1], rel=1e-11, abs=1e-13)
+
+
+# ---------------------------------------------------------------- P4 ------
+
+def _random_run(lib, ef, lam, steps, store, n=257, seed=3, wd_on=None,
+                shapes=None, perm=None, stash_store=None):
+    rng = np.random.default_rng(seed)
+    shapes = shapes or [n]
+    x0 = rng.normal(0, 0.02, sum(shapes))
+    grads = [rng.normal(0, 1e-3, sum(shapes)) for _ in range(steps)]
+    if store == F32:
+        x0 = x0.astype(np.float32).astype(np.float64)
+        grads = [g.astype(np.float32).astype(np.float64) for g in grads]
+    if perm is not None:
+        x0 = x0[perm]
+        grads = [g[perm] for g in grads]
+    parts = np.split(x0, np.cumsum(shapes)[:-1])
+    hp = HParams(lr=3e-4, ef_lambda=lam)
+    o = oracle.DelayedOptimizer(parts, hp, ef=ef, x_store=store,
+                                stash_store=stash_store or store,
+                                param_store=BF16 if store == F32 else None,
+                                wd_on=wd_on, lib=lib)
+    hist = []
+    for g in grads:
+        o.step(g, tag=o.read_weights()[1])
+        hist.append(dict(x=o.x.copy(), u=None if o.u_prev is None else o.u_prev.copy(),
+                         stash=o.stash.copy(),
+                         param=None if o.param is None else o.param.copy()))
+    return o, hist
+
+
+def test_p4a_ef_lambda_zero_is_standard_bitwise(lib):
+    """App. A.4: lambda = 0 recovers standard delayed training."""
+    _, h_std = _random_run(lib, ef=False, lam=0.0, steps=8, store=F32)
+    _, h_ef0 = _random_run(lib, ef=True, lam=0.0, steps=8, store=F32)
+    for a, b in zip(h_std, h_ef0):
+        assert np.array_equal(a["x"], b["x"])
+        assert np.array_equal(a["param"], b["param"])
+
+
+@pytest.mark.parametrize("lam", [1.0, 0.5, 2.0])
+def test_p4b_sapipe_restatement(lib, lam):
+    """App. B.1: with p_t = x_t + lambda u_{t-2}, EF is the standard
+    recursion p_{t+1} = p_t - u_{t-1}, and x_{t+1} = p_t - (1+lambda) u_{t-1}
+    (for lambda = 1 these are SAPipe-WP's prediction points, whose
+    displacement is Eq. (1)'s). Holds from the second update on."""
+    o, hist = _random_run(lib, ef=True, lam=lam, steps=10, store=F64)
+    # hist[j] is the state after call k = j + 1: x_{k+1} and u_{k-1}.
+    for t in range(1, len(hist)):
+        p_t = hist[t - 1]["x"] + lam * hist[t - 1]["u"]
+        u = hist[t]["u"]
+        p_next = hist[t]["x"] + lam * u
+        np.testing.assert_allclose(p_next, p_t - u, rtol=1e-12, atol=1e-17)
+        np.testing.assert_allclose(hist[t]["x"], p_t - (1 + lam) * u,
+                                   rtol=1e-12, atol=1e-17)
+
+
+def test_p4c_version_lag(lib):
+    """Sec. 2 / Alg. 1: the gradient consumed at call k was evaluated at
+    x_{k-1}, the stash; the stash after each call is the previous master
+    (bitwise the previous bf16 weights when the stash is bf16)."""
+    o, hist = _random_run(lib, ef=True, lam=1.0, steps=6, store=F32,
+                          stash_store=BF16)
+    for t in range(1, len(hist)):
+        assert np.array_equal(hist[t]["stash"], hist[t - 1]["param"])
+    o2, hist2 = _random_run(lib, ef=False, lam=0.0, steps=6, store=F32)
+    for t in range(1, len(hist2)):
+        assert np.array_equal(hist2[t]["stash"], hist2[t - 1]["x"])
+    # evaluating the gradient at the latest weights instead is rejected
+    latest_tag = o.read_weights("latest")[1]
+    with pytest.raises(oracle.StaleVersionError):
+        o.step(np.zeros(o.x.size), tag=latest_tag)
+    assert o.read_weights("stale")[1] == o.k and latest_tag == o.k + 1
+
+
+@pytest.mark.parametrize("lam", [0.0, 1.0, 3.0])
+def test_p4d_displacement_bound(lib, lam):
+    """|x_{t+1} - x_t| <= (1 + 2|lambda|) max(|u_{t-1}|, |u_{t-2}|) per
+    element (the step-size bound used in App. D's proofs, for tau = 1)."""
+    o, hist = _random_run(lib, ef=True, lam=lam, steps=8, store=F64)
+    for t in range(1, len(hist)):
+        d = np.abs(hist[t]["x"] - hist[t - 1]["x"])
+        bound = (1 + 2 * abs(lam)) * np.maximum(np.abs(hist[t]["u"]), np.abs(hist[t - 1]["u"]))
+        assert np.all(d <= bound * (1 + 1e-12) + 1e-300)
+
+
+def test_p4e_permutation_and_split_invariance(lib):
+    """The step is elementwise: permuting elements or splitting them into
+    tensors differently leaves every value unchanged (clipping off)."""
+    n = 300
+    perm = np.random.default_rng(0).permutation(n)
+    _, h_a = _random_run(lib, ef=True, lam=1.0, steps=5, store=F32, n=n)
+    _, h_b = _random_run(lib, ef=True, lam=1.0, steps=5, store=F32, n=n,
+                         perm=perm)
+    _, h_c = _random_run(lib, ef=True, lam=1.0, steps=5, store=F32,
+                         shapes=[1, 150, 7, 142])
+    for a, b, c in zip(h_a, h_b, h_c):
+        assert np.array_equal(a["x"][perm], b["x"])
+        assert np.array_equal(a["x"], c["x"])
+
+
+def test_weight_decay_mask(lib):
+    """A tensor with decay switched off takes the wd = 0 update."""
+    rng = np.random.default_rng(5)
+    x0 = [rng.normal(0, 1, 4), rng.normal(0, 1, 3)]
+    g = rng.normal(0, 1, 7)
+    hp = HParams(lr=0.01, weight_decay=0.5)
+    o = oracle.DelayedOptimizer(x0, hp, x_store=F64, stash_store=F64,
+                                wd_on=[True, False], lib=lib)
+    o.step(g)
+    ref_on = _torch_adamw_run([x0[0]], [[g[:4]]], hp, [0.01])[0]
+    ref_off = _torch_adamw_run([x0[1]], [[g[4:]]],
+                               HParams(lr=0.01, weight_decay=0.0), [0.01])[0]
+    assert _rel(o.x[:4], ref_on) < 1e-13
+    assert _rel(o.x[4:], ref_off) < 1e-13
+
+
+# ------------------------------------------------------------- storage ----
+
+def test_bf16_rounding_matches_torch(lib):
+    """The oracle's own bf16 rounding equals torch's fp32 -> bf16 cast
+    (round to nearest even) on ties, subnormals, overflow and random values."""
+    rng = np.random.default_rng(1)
+    vals = [rng.normal(0, s, 4000).astype(np.float32) for s in (1e-3, 1.0, 1e30)]
+    bits = np.arange(0, 1 << 16, 7, dtype=np.uint32)
+    ties = ((bits << 16) | 0x8000).view(np.float32)      # exactly halfway
+    near = ((bits << 16) | 0x7FFF).view(np.float32)
+    tiny = (np.arange(1, 3000, dtype=np.uint32)).view(np.float32)  # subnormals
+    big = np.array([3.3895e38, 3.39e38, -3.4028235e38, 65504.0], np.float32)
+    x = np.concatenate(vals + [ties, near, tiny, big])
+    x = x[np.isfinite(x)]
+    ref = torch.from_numpy(x).to(torch.bfloat16).to(torch.float64).numpy()
+    got = oracle.round_to(x.astype(np.float64), BF16, lib=lib)
+    np.testing.assert_array_equal(got, ref)
+
+
+def test_f32_rounding_matches_numpy(lib):
+    x = np.random.default_rng(2).normal(0, 1, 1000) * 10.0 ** np.random.default_rng(3).integers(-40, 38, 1000)
+    np.testing.assert_array_equal(oracle.round_to(x, F32, lib=lib),
+                                  x.astype(np.float32).astype(np.float64))
+
+
+def test_sqnorm_and_clip(lib):
+    rng = np.random.default_rng(4)
+    g = rng.normal(0, 1, 200_001)
+    ref = math.fsum(v * v for v in g)
+    assert oracle.sqnorm(g, lib=lib) == pytest.approx(ref, rel=1e-13)
+    g32 = g.astype(np.float32)
+    assert oracle.sqnorm_f32(g32, lib=lib) == pytest.approx(
+        math.fsum(float(v) ** 2 for v in g32), rel=1e-13)
+    gb = torch.from_numpy(g32).to(torch.bfloat16)
+    bits = gb.view(torch.int16).numpy().view(np.uint16)
+    assert oracle.sqnorm_bf16(bits, lib=lib) == pytest.approx(
+        math.fsum(float(v) ** 2 for v in gb.double().numpy()), rel=1e-13)
+    assert oracle.clip_coef(4.0, 1.0, lib=lib) == pytest.approx(1.0 / (2.0 + 1e-6), rel=1e-15)
+    assert oracle.clip_coef(0.25, 1.0, lib=lib) == 1.0
+    assert oracle.clip_coef(4.0, 0.0, lib=lib) == 1.0
+
+
+def test_quadratic_gradient_is_loss_derivative(lib):
+    """grad = d loss / dw (central differences) when the noise is zero."""
+    rng = np.random.default_rng(6)
+    n = 20
+    a = np.exp(rng.uniform(np.log(1e-3), 0, n))
+    ws, w = rng.normal(0, 1, n), rng.normal(0, 1, n)
+    g, loss = oracle.quadratic(a, ws, w, None, F64, lib=lib)
+    h = 1e-6
+    for i in range(n):
+        e = np.zeros(n)
+        e[i] = h
+        lp = oracle.quadratic(a, ws, w + e, None, F64, lib=lib)[1]
+        lm = oracle.quadratic(a, ws, w - e, None, F64, lib=lib)[1]
+        assert g[i] == pytest.approx((lp - lm) / (2 * h), rel=1e-6, abs=1e-9)
+    assert loss == pytest.approx(0.5 * np.sum(a * (w - ws) ** 2), rel=1e-14)
