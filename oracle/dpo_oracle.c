@@ -178,13 +178,14 @@ DEFINE_SQNORM(oracle_sqnorm_f32, float, widen_f32)
 DEFINE_SQNORM(oracle_sqnorm_bf16, uint16_t, widen_bf16)
 
 /* Global-norm clipping (App. E.1 uses a threshold of 1.0): the coefficient
- * is clamped at 1 and 1e-6 is added to the norm. */
+ * is clamped at 1 and 1e-6 is added to the norm. A NaN norm is not clamped,
+ * so NaN reaches every element, as torch.nn.utils.clip_grad_norm_ does. */
 double oracle_clip_coef(double sqnorm, double max_norm)
 {
     if (!(max_norm > 0.0))
         return 1.0;
     const double coef = max_norm / (sqrt(sqnorm) + 1e-6);
-    return coef < 1.0 ? coef : 1.0;
+    return coef > 1.0 ? 1.0 : coef;   /* a NaN norm gives a NaN coefficient */
 }
 
 double oracle_quadratic(int64_t n, const double *a, const double *wstar,

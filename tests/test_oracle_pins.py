@@ -427,6 +427,18 @@ def test_sqnorm_and_clip(lib):
     assert oracle.clip_coef(4.0, 0.0, lib=lib) == 1.0
 
 
+def test_clip_nonfinite_norm_like_torch(lib):
+    """A NaN gradient makes every clipped element NaN and an infinite norm
+    zeroes the finite ones, as torch.nn.utils.clip_grad_norm_ does."""
+    for bad in (float("nan"), float("inf")):
+        g = np.array([0.5, bad, -2.0])
+        p = torch.nn.Parameter(torch.zeros(3, dtype=torch.float64))
+        p.grad = torch.tensor(g)
+        torch.nn.utils.clip_grad_norm_([p], 1.0)
+        coef = oracle.clip_coef(oracle.sqnorm(g, lib=lib), 1.0, lib=lib)
+        np.testing.assert_array_equal(coef * g, p.grad.numpy())
+
+
 def test_quadratic_gradient_is_loss_derivative(lib):
     """grad = d loss / dw (central differences) when the noise is zero."""
     rng = np.random.default_rng(6)
