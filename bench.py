@@ -1,0 +1,383 @@
+"""Benchmark of the one-step-delayed AdamW step (arXiv 2606.30634, Alg. 1 with
+Error Feedback) on a 6.74e9-parameter Llama-7B-shaped tensor set.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl dpo|reference]
+                    [--workload llama-7B] [--mode ef|std]
+
+A step is one dpo_step over the whole set: every parameter's stale gradient
+is consumed and master, m, v, the EF buffer, the bf16 stash and the bf16
+latest copy are rewritten (inputs already resident in HBM when timing
+starts; the 148 GB working set is far larger than L2, so no flush is
+needed). Prints one JSON line: throughput in parameters updated per second,
+the fused kernel's achieved HBM bandwidth against the measured copy peak,
+an end-to-end figure through the public API with the gradients coming from
+and the new weights going to pinned host memory, and the CPU oracle's
+throughput on a bounded sample of the same set.
+
+Under torchrun every rank runs its own full replica on its own GPU (the step
+is elementwise, so ranks are independent problems: weak scaling, no
+collective on the data path); timing is the maximum over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "params updated/sec and achieved HBM GB/s (% of GB300 peak), 7B-shaped step"
+UNIT = "params/s"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args(argv=None):
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=30)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["dpo", "reference"], default="dpo")
+    p.add_argument("--workload", default="llama-7B")
+    p.add_argument("--mode", choices=["ef", "std"], default="ef")
+    p.add_argument("--e2e-steps", type=int, default=4)
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=12.0)
+    return p.parse_args(argv)
+
+
+# ----------------------------------------------------------- distributed --
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    """Maximum of a per-rank scalar (a timing) over all ranks."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate(units_per_rank: float, seconds_per_rank: float, world: int, device=None):
+    """Whole-job throughput: units all ranks processed / the slowest rank's time."""
+    t = max_over_ranks(seconds_per_rank, world, device)
+    return units_per_rank * world / t, t
+
+
+# ----------------------------------------------------------------- peaks --
+
+def measured_hbm_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def committed_traffic(kernel_tag: str):
+    """dram bytes per parameter from the committed ncu summary of the fused
+    kernel, if that summary was taken on the kernel source as it is now."""
+    src = os.path.join(ROOT, "paper_2606_30634_gb300", "csrc", "dpo_kernels.cu")
+    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    for name in sorted(os.listdir(os.path.join(ROOT, "profiles"))) if os.path.isdir(
+            os.path.join(ROOT, "profiles")) else []:
+        if not name.endswith(".md"):
+            continue
+        text = open(os.path.join(ROOT, "profiles", name)).read()
+        m_tag = re.search(r"^kernel_tag:\s*(\S+)", text, re.M)
+        m_sha = re.search(r"^kernel_source_sha256_16:\s*(\S+)", text, re.M)
+        m_b = re.search(r"^dram_bytes_per_param:\s*([0-9.eE+-]+)", text, re.M)
+        if m_tag and m_sha and m_b and m_tag.group(1) == kernel_tag and m_sha.group(1) == sha:
+            return float(m_b.group(1))
+    return None
+
+
+# ---------------------------------------------------------------- clocks --
+
+class ClockSampler:
+    """nvidia-smi samples during the timed region."""
+    FIELDS = ("index,pci.bus_id,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, bus_id=None):
+        self.bus_id = (bus_id or "").lower()
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = [r.split(", ") for r in out.strip().splitlines() if r.count(",") >= 9]
+        if self.bus_id:
+            mine = [r for r in rows if self.bus_id.endswith(r[1].lower()[-12:]) or
+                    r[1].lower().endswith(self.bus_id[-12:])]
+            rows = mine or rows
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[6:10]) if v.strip() == "Active"})
+        sm = sorted(float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit())
+        mx = max((float(r[3]) for r in rows if r[3].strip().replace(".", "").isdigit()), default=None)
+        pw = [float(r[4]) for r in rows if re.match(r"^[0-9.]+$", r[4].strip())]
+        return {"sm_mhz": sm[len(sm) // 2] if sm else None, "sm_max_mhz": mx,
+                "reasons": reasons, "samples": len(rows),
+                "power_w_max": max(pw) if pw else None}
+
+
+# ------------------------------------------------------------ CPU oracle --
+
+def oracle_sample_run(w, ef: bool, seconds: float, max_steps: int = 1000, n: int = 1 << 22):
+    """Time the oracle as it stands on the first n parameters of the set
+    (input draws excluded from the timing). Returns (params/s, cores, steps,
+    n)."""
+    import numpy as np
+
+    import oracle
+    from paper_2606_30634_gb300 import synth
+    from paper_2606_30634_gb300.synth import workloads as W
+
+    n = min(n, w.n_params)
+    STORE = {0: oracle.F32, 1: oracle.BF16}
+    x0 = synth.host_normal(w.seed, synth.STREAM_INIT, 0, 0, n, W.INIT_SIGMA).astype(np.float64)
+    hp = oracle.HParams(lr=w.lr, weight_decay=w.weight_decay, ef_lambda=1.0 if ef else 0.0,
+                        max_grad_norm=w.max_grad_norm).as_f32()
+    o = oracle.DelayedOptimizer([x0], hp, ef=ef, x_store=oracle.F32,
+                                stash_store=STORE[w.stash_dtype],
+                                param_store=oracle.BF16 if w.param_dtype == 1 else None)
+    gdt = synth.BF16 if w.grad_dtype == 1 else synth.F32
+    spent, steps = 0.0, 0
+    while steps < max_steps and (spent < seconds or steps < 2):
+        g = synth.host_normal(w.seed, synth.STREAM_GRAD, steps + 1, 0, n, W.GRAD_SIGMA, gdt)
+        g = (synth.bf16_bits_to_f32(g) if gdt == synth.BF16 else g).astype(np.float64)
+        sq = oracle.sqnorm(g) if w.max_grad_norm > 0 else None
+        t0 = time.perf_counter()
+        o.step(g, sq=sq)
+        spent += time.perf_counter() - t0
+        steps += 1
+    return n * steps / spent, oracle.num_threads(), steps, n
+
+
+# ------------------------------------------------------------------- GPU --
+
+def run_gpu(args, w, world, rank, local):
+    import numpy as np
+    import torch
+
+    from paper_2606_30634_gb300 import dpo, synth
+    from paper_2606_30634_gb300.synth import workloads as W
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    ef = args.mode == "ef"
+    stream = torch.cuda.Stream(dev)
+    offs = np.concatenate([[0], np.cumsum(w.numels)]).astype(np.int64)
+    with torch.cuda.stream(stream):
+        lay = dpo.Layout.of(w.numels)
+        x0 = torch.empty(lay.total, dtype=torch.float32, device=dev)
+        for i, (o, n) in enumerate(zip(lay.offsets, lay.numels)):
+            synth.dev_normal(w.seed, synth.STREAM_INIT, 0, int(offs[i]), x0[o:o + n], W.INIT_SIGMA)
+        opt = dpo.DelayedAdamW(w.numels, param_dtype=w.param_dtype, stash_dtype=w.stash_dtype,
+                               grad_dtype=w.grad_dtype, lr=w.lr, beta1=w.beta1, beta2=w.beta2,
+                               eps=w.eps, weight_decay=w.weight_decay, ef=ef, ef_lambda=1.0,
+                               max_grad_norm=w.max_grad_norm, delay=1, device=dev, x0=x0,
+                               stream=stream)
+        del x0
+        for i, (o, n) in enumerate(zip(lay.offsets, lay.numels)):
+            synth.dev_normal(w.seed, synth.STREAM_GRAD, 1, int(offs[i]), opt.grads(i),
+                             W.GRAD_SIGMA)
+    torch.cuda.synchronize(dev)
+    step_bytes, norm_bytes = dpo.dpo_algorithmic_bytes(opt.ctx)
+    step_ctas, norm_ctas, threads = dpo.dpo_launch_config(opt.ctx)
+    launches_per_step = 2 if w.max_grad_norm > 0 else 1
+
+    for _ in range(args.warmup):
+        opt.step(stream=stream)
+    torch.cuda.synchronize(dev)
+
+    props = torch.cuda.get_device_properties(dev)
+    sampler = ClockSampler(getattr(props, "pci_bus_id", None))
+    K = args.steps
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(K + 1)]
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize(dev)
+    sampler.start()
+    time.sleep(0.25)
+    ev[0].record(stream)
+    for i in range(K):
+        opt.step(stream=stream)
+        ev[i + 1].record(stream)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        torch.distributed.barrier()
+    clocks = sampler.stop()
+    per_step_ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(K)]
+    total_s = ev[0].elapsed_time(ev[K]) / 1e3
+    value, t_max = aggregate(w.n_params * K, total_s, world, dev)
+    kernel_ms = sum(per_step_ms) / K          # one fused launch per step (no clipping)
+    achieved = step_bytes / (kernel_ms / 1e3) / 1e9
+
+    # End to end through the public API, gradients from and new bf16 weights
+    # to pinned host memory, copies inside the timed region.
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, opt, stream, dev, world, w)
+
+    opt.close()
+    return dict(value=value, t_max=t_max, per_step_ms=per_step_ms, kernel_ms=kernel_ms,
+                achieved=achieved, step_bytes=step_bytes, norm_bytes=norm_bytes, clocks=clocks,
+                launches=K * launches_per_step, step_ctas=step_ctas, threads=threads, e2e=e2e,
+                device_name=props.name)
+
+
+def _host_avail_bytes():
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    return int(line.split()[1]) * 1024
+    except Exception:
+        pass
+    return 0
+
+
+def run_e2e(args, opt, stream, dev, world, w):
+    import torch
+    need = opt.grad.numel() * opt.grad.element_size() + opt.param.numel() * opt.param.element_size()
+    if _host_avail_bytes() < 2 * need + (16 << 30):
+        return {"skipped": f"host memory: {need / 1e9:.1f} GB pinned needed"}
+    h_grad = torch.empty(opt.grad.shape, dtype=opt.grad.dtype, pin_memory=True)
+    h_param = torch.empty(opt.param.shape, dtype=opt.param.dtype, pin_memory=True)
+    with torch.cuda.stream(stream):
+        h_grad.copy_(opt.grad, non_blocking=True)
+    torch.cuda.synchronize(dev)
+    K = max(1, args.e2e_steps)
+
+    def one_step():
+        with torch.cuda.stream(stream):
+            opt.grad.copy_(h_grad, non_blocking=True)
+            opt.step(stream=stream)
+            h_param.copy_(opt.param, non_blocking=True)
+
+    one_step()
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        torch.distributed.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(K):
+        one_step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    secs = e0.elapsed_time(e1) / 1e3
+    value, _ = aggregate(w.n_params * K, secs, world, dev)
+    out = {"value": value, "unit": UNIT,
+           "h2d_bytes_per_step": h_grad.numel() * h_grad.element_size(),
+           "d2h_bytes_per_step": h_param.numel() * h_param.element_size(),
+           "ms_per_step": secs / K * 1e3, "steps": K}
+    del h_grad, h_param
+    return out
+
+
+# ------------------------------------------------------------------ main --
+
+def main(argv=None):
+    args = parse_args(argv)
+    from paper_2606_30634_gb300.synth import workloads as W
+    w = W.ALL[args.workload]
+    world, rank, local = dist_env()
+    ef = args.mode == "ef"
+    cfg = {"workload": f"{w.name}: {w.n_params} params in {len(w.tensors)} tensors, "
+                       f"{'EF (lambda=1)' if ef else 'standard delayed rule'}, one-step delay",
+           "mode": args.mode, "param_dtype": "bf16" if w.param_dtype else "f32",
+           "stash_dtype": "bf16" if w.stash_dtype else "f32",
+           "grad_dtype": "bf16" if w.grad_dtype else "f32",
+           "state": "fp32 master/m/v" + (" + fp32 EF buffer" if ef else ""),
+           "clip": w.max_grad_norm, "l2": "inputs larger than L2 (no flush needed)"}
+
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        v, cores, steps, n = oracle_sample_run(w, ef, args.cpu_seconds,
+                                               max_steps=max(1, args.steps + args.warmup))
+        sample = f"first {n} params of the set, {steps} oracle steps (plain C, fp64)"
+        line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT,
+                "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+                "ms_per_step": w.n_params / v * 1e3, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                "config": cfg,
+                "cpu_baseline": {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
+                                 "sample": sample},
+                "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
+        print(json.dumps(line), flush=True)
+        return 0
+
+    import torch
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    r = run_gpu(args, w, world, rank, local)
+    peak, peak_kind = measured_hbm_peak()
+    kernel_tag = f"fused_step:{w.name}:{args.mode}"
+    traffic = committed_traffic(kernel_tag)
+    roof = {"bound": "hbm", "achieved": r["achieved"], "peak": peak, "unit": "GB/s",
+            "frac": r["achieved"] / peak, "peak_kind": peak_kind,
+            "traffic": None if traffic is None else traffic * w.n_params,
+            "kernel": "fused_step_kernel", "algorithmic_bytes_per_launch": r["step_bytes"],
+            "bytes_per_param": r["step_bytes"] / w.n_params,
+            "avg_launch_ms": r["kernel_ms"], "nominal_peak_gbs": 8000.0,
+            "frac_of_nominal": r["achieved"] / 8000.0}
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        v, cores, steps, n = oracle_sample_run(w, ef, args.cpu_seconds)
+        cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
+               "sample": f"first {n} params of the set, {steps} oracle steps (plain C, fp64)"}
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    if rank != 0:
+        return 0
+    line = {"metric": METRIC, "value": r["value"], "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": r["t_max"] / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic", "config": cfg, "roofline": roof, "cpu_baseline": cpu,
+            "e2e": r["e2e"], "gpu_launches": r["launches"], "clocks": r["clocks"],
+            "launch": {"ctas": r["step_ctas"], "threads": r["threads"]},
+            "hbm_gbs_achieved": r["achieved"], "device": r["device_name"]}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,186 @@
+/*
+ * dpo.h -- one-step-delayed AdamW step with Error Feedback, C ABI.
+ *
+ * The per-parameter optimizer step of arXiv 2606.30634 ("One-Step Gradient
+ * Delay is Not a Barrier for Large-Scale Asynchronous Pipeline Parallel LLM
+ * Pretraining"), for one GPU (sm_103a):
+ *
+ *   Alg. 1 (Sec. 2), Delayed Gradient Update. Iteration t updates the
+ *   optimizer statistics with the stale gradient g_{t-1}, forms the update
+ *   u_{t-1}(g_{t-1}) and applies
+ *       x_{t+1} = x_t - u_{t-1}                          standard, or t <= 1
+ *       x_{t+1} = x_t - u_{t-1} - lambda (u_{t-1} - u_{t-2})   Error Feedback
+ *   (Eq. (1), Sec. 3.2 for lambda = 1; App. A.4 for general lambda).
+ *   u is AdamW (Sec. 2.1: beta = (0.9, 0.95); Sec. 2.2: EMA moments) with
+ *   decoupled weight decay on the current iterate x_t (Alg. 2) and optional
+ *   global gradient-norm clipping (App. E.1):
+ *       g^ = s g,  s = min(1, max_norm / (||g||_2 + 1e-6))  (1 without clipping)
+ *       m  = beta1 m + (1 - beta1) g^,   v = beta2 v + (1 - beta2) g^2
+ *       u  = lr ( (m / (1 - beta1^k)) / (sqrt(v / (1 - beta2^k)) + eps) + wd x_t )
+ *   k counts the gradients consumed (the k-th dpo_step is iteration t = k;
+ *   iteration t = 0 only sets x_1 = x_0 since u_{-1} = 0).
+ *
+ *   Weight-version stash (Sec. 2, PipeDream-2BW keeps one extra weight
+ *   version): after each step the stash holds x_t, the weights before the
+ *   update, and the latest copy holds x_{t+1}. The next forward/backward reads
+ *   the stash (dpo_read_weights(DPO_STALE)), so the gradient the next
+ *   dpo_step consumes was evaluated one version behind the weights it updates.
+ *
+ * Layout and ownership. The caller owns and allocates every buffer named in
+ * a dpo_tensor (device memory of the current device, 16-byte aligned, not
+ * overlapping one another), keeps them alive until dpo_destroy, and may not
+ * move them. The library owns only its context: a device copy of the tensor
+ * table and a few hundred bytes of device scratch per SM for the gradient
+ * norm. All launches go to the stream passed in (a cudaStream_t, NULL for the
+ * legacy default stream); dpo_step never synchronizes the host.
+ *
+ * Errors. Every call returns DPO_OK (0) or a negative DPO_E* code; nothing
+ * aborts. dpo_last_error gives a message for the last failing call on a
+ * context (or, with NULL, for the last dpo_init failure of this thread).
+ */
+#ifndef DPO_H
+#define DPO_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define DPO_ABI_VERSION 1
+
+/* Status codes. */
+#define DPO_OK 0
+#define DPO_EINVAL (-1)  /* bad argument: NULL or overlapping buffers, bad size or value */
+#define DPO_EALIGN (-2)  /* a buffer is not 16-byte aligned */
+#define DPO_EDTYPE (-3)  /* unsupported dtype or dtype combination */
+#define DPO_ECUDA (-4)   /* a CUDA runtime call or launch failed */
+#define DPO_ESTATE (-5)  /* the context is not in a state that allows the call */
+#define DPO_ENOMEM (-6)  /* the library's own small device allocation failed */
+
+typedef enum { DPO_F32 = 0, DPO_BF16 = 1 } dpo_dtype;
+
+/* dpo_tensor.flags */
+#define DPO_WD_ON 1u     /* apply weight decay to this tensor */
+
+/* dpo_read_weights(which) */
+#define DPO_STALE 0      /* what the next forward/backward reads (the stash) */
+#define DPO_LATEST 1     /* the newest weights x_{t+1} */
+
+/* dpo_init(init_mode) */
+#define DPO_INIT_FRESH 0   /* m = v = 0, EF buffer = 0, stash and param := master */
+#define DPO_INIT_RESUME 1  /* keep every buffer as given (restore with dpo_set_step) */
+
+/* dpo_get_flags() bits */
+#define DPO_FLAG_NONFINITE 1u  /* a clipped step saw a non-finite gradient norm */
+
+typedef struct {
+    float beta1;          /* first-moment EMA coefficient, [0, 1) */
+    float beta2;          /* second-moment EMA coefficient, [0, 1) */
+    float eps;            /* added to sqrt(v_hat), >= 0 */
+    float weight_decay;   /* decoupled decay (tensors with DPO_WD_ON), >= 0 */
+    float ef_lambda;      /* lambda of the EF correction (tables with EF buffers) */
+    float max_grad_norm;  /* > 0: global-norm clipping threshold; <= 0: off */
+    int delay;            /* 1: one-step-delayed with stash; 0: synchronous */
+} dpo_hparams;
+
+typedef struct {
+    /* Latest weights x_{t+1} in the param dtype. With DPO_BF16 params this is
+     * written every step (round to nearest even from master). With DPO_F32
+     * params it must be NULL: the fp32 master is then the latest copy. */
+    void *param;
+    float *master;     /* fp32 master weights, read and written */
+    float *m;          /* Adam first moment, fp32, read and written */
+    float *v;          /* Adam second moment, fp32, read and written */
+    /* Stale weights in the stash dtype: x_t after each step. Required when
+     * delay == 1; ignored (may be NULL) when delay == 0. */
+    void *stash;
+    /* EF buffer (fp32): u_{t-2} on entry, u_{t-1} on return. NULL on every
+     * tensor: standard delayed rule. Non-NULL on every tensor: EF with
+     * hparams.ef_lambda (lambda = 0 gives the standard result). */
+    float *ef;
+    /* The gradient the step consumes, in the grad dtype, evaluated at the
+     * stash (delay == 1) or at the latest weights (delay == 0). Read only. */
+    const void *grad;
+    int64_t numel;     /* elements, >= 0; 0 is allowed and skipped */
+    uint32_t flags;    /* DPO_WD_ON or 0 */
+} dpo_tensor;
+
+typedef struct dpo_ctx dpo_ctx;
+
+/*
+ * Create a context over n_tensors tensors (table is copied; the buffers it
+ * points to are not). Validates every pointer (NULL, 16-byte alignment,
+ * overlap, device residency), dtype and hyperparameter. With DPO_INIT_FRESH
+ * it then enqueues, on cuda_stream, the Alg. 1 start state: m = v = 0, EF
+ * buffer = 0 (u_{-1} = 0), stash := x_0 and param := x_0 from master, and
+ * sets k = 0. Supported dtypes: param F32|BF16, stash F32|BF16, grad
+ * F32|BF16. Returns DPO_OK and *out, or an error and *out = NULL.
+ */
+int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
+             dpo_dtype param_dtype, dpo_dtype stash_dtype, dpo_dtype grad_dtype,
+             const dpo_hparams *hp, int init_mode, void *cuda_stream);
+
+/*
+ * stash := the current master weights (rounded to the stash dtype), and the
+ * bf16 param copy := master. Used at start-up and when delayed training is
+ * (re)entered after synchronous steps. Enqueued on cuda_stream.
+ */
+int dpo_stash(dpo_ctx *ctx, void *cuda_stream);
+
+/*
+ * One delayed step (Alg. 1 iteration t = k + 1) with learning rate lr:
+ * consumes every tensor's grad, updates master, m, v (and the EF buffer),
+ * writes stash := x_t (delay == 1) and param := x_{t+1}, then k += 1.
+ * With clipping, first computes the global gradient norm over all tensors
+ * (deterministic, fixed reduction order). Asynchronous on cuda_stream, no
+ * host synchronization, no allocation. lr must be finite and >= 0.
+ */
+int dpo_step(dpo_ctx *ctx, float lr, void *cuda_stream);
+
+/*
+ * Pointer and dtype of tensor `tensor`'s stale (DPO_STALE) or latest
+ * (DPO_LATEST) weights. Under delay == 0 both name the latest weights. The
+ * pointer is one of the caller's own buffers; no copy is made.
+ */
+int dpo_read_weights(const dpo_ctx *ctx, int which, int tensor,
+                     const void **ptr, dpo_dtype *dtype);
+
+/* Step counter k (gradients consumed so far); set it when resuming. */
+int dpo_get_step(const dpo_ctx *ctx, int64_t *k);
+int dpo_set_step(dpo_ctx *ctx, int64_t k);
+
+/*
+ * Diagnostics of the last clipped step: the DPO_FLAG_* bits raised since the
+ * previous dpo_get_flags (reading clears them), the global gradient norm and
+ * the clip coefficient used. Synchronizes cuda_stream (not for the hot
+ * loop). Any output pointer may be NULL.
+ */
+int dpo_get_flags(dpo_ctx *ctx, uint32_t *flags, double *grad_norm,
+                  float *clip_scale, void *cuda_stream);
+
+/*
+ * Bytes one dpo_step must move through memory by the layout of the context
+ * (algorithmic, not measured): *step_bytes for the fused step over all
+ * tensors, *norm_bytes for the gradient-norm pass (0 without clipping).
+ */
+int dpo_algorithmic_bytes(const dpo_ctx *ctx, int64_t *step_bytes,
+                          int64_t *norm_bytes);
+
+/* Launch geometry chosen at init: CTAs of the fused step and of the norm
+ * pass (both persistent: a multiple of the SM count) and threads per CTA. */
+int dpo_launch_config(const dpo_ctx *ctx, int *step_ctas, int *norm_ctas,
+                      int *threads);
+
+/* Message of the last failing call on ctx (NULL ctx: last dpo_init failure of
+ * the calling thread). Never NULL; owned by the library. */
+const char *dpo_last_error(const dpo_ctx *ctx);
+
+/* Free the context and its device scratch (after the work enqueued on it has
+ * finished or been synchronized by the caller). NULL is ignored. */
+void dpo_destroy(dpo_ctx *ctx);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* DPO_H */

@@ -1,0 +1,462 @@
+// dpo_abi.cpp -- the C ABI of include/dpo.h: validation, context, launches.
+//
+// Host side of the one-step-delayed AdamW step (arXiv 2606.30634, Alg. 1 with
+// the Error-Feedback correction of Eq. (1) / App. A.4). The per-call scalars
+// (bias corrections, the Alg. 1 "standard rule for t <= 1" switch) are formed
+// here in double and handed to the kernels by value; every per-element
+// operation runs in dpo_kernels.cu.
+#include "dpo.h"
+#include "dpo_internal.h"
+
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <new>
+#include <string>
+#include <vector>
+
+using dpo::DevTensor;
+using dpo::StashKind;
+
+struct dpo_ctx {
+    int device = 0;
+    int n = 0;
+    dpo_dtype param_dt = DPO_F32, stash_dt = DPO_F32, grad_dt = DPO_F32;
+    dpo_hparams hp{};
+    bool ef = false;
+    bool clip = false;
+    int64_t k = 0;
+    int64_t total_pkts = 0;
+    int64_t total_elems = 0;
+    std::vector<dpo_tensor> table;
+    int step_grid = 0, norm_grid = 0, stash_grid = 0;
+    // one device allocation: table | pkt_begin | partials | scalars
+    void *dev_block = nullptr;
+    DevTensor *d_table = nullptr;
+    int64_t *d_pkt_begin = nullptr;
+    double *d_partials = nullptr;
+    dpo::NormScalars *d_scalars = nullptr;
+    std::string err;
+};
+
+namespace {
+
+thread_local std::string g_init_err;
+
+int fail(dpo_ctx *c, int code, const char *fmt, ...)
+{
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    if (c != nullptr)
+        c->err = buf;
+    else
+        g_init_err = buf;
+    return code;
+}
+
+int cuda_fail(dpo_ctx *c, cudaError_t e, const char *what)
+{
+    return fail(c, DPO_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool valid_dtype(int d) { return d == DPO_F32 || d == DPO_BF16; }
+int64_t dt_size(dpo_dtype d) { return d == DPO_BF16 ? 2 : 4; }
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+StashKind stash_kind(const dpo_ctx *c)
+{
+    if (c->hp.delay == 0)
+        return dpo::kStashNone;
+    return c->stash_dt == DPO_BF16 ? dpo::kStashBF16 : dpo::kStashF32;
+}
+
+struct Span {
+    uintptr_t lo, hi;
+    int tensor;
+    const char *name;
+};
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+}  // namespace
+
+extern "C" const char *dpo_last_error(const dpo_ctx *ctx)
+{
+    if (ctx == nullptr)
+        return g_init_err.c_str();
+    return ctx->err.c_str();
+}
+
+extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
+                        dpo_dtype param_dtype, dpo_dtype stash_dtype, dpo_dtype grad_dtype,
+                        const dpo_hparams *hp, int init_mode, void *cuda_stream)
+{
+    if (out == nullptr)
+        return fail(nullptr, DPO_EINVAL, "out is NULL");
+    *out = nullptr;
+    if (hp == nullptr)
+        return fail(nullptr, DPO_EINVAL, "hparams is NULL");
+    if (n_tensors < 1 || table == nullptr)
+        return fail(nullptr, DPO_EINVAL, "need a table of at least one tensor");
+    if (!valid_dtype(param_dtype) || !valid_dtype(stash_dtype) || !valid_dtype(grad_dtype))
+        return fail(nullptr, DPO_EDTYPE, "dtype must be DPO_F32 or DPO_BF16");
+    if (init_mode != DPO_INIT_FRESH && init_mode != DPO_INIT_RESUME)
+        return fail(nullptr, DPO_EINVAL, "init_mode must be DPO_INIT_FRESH or DPO_INIT_RESUME");
+    if (hp->delay != 0 && hp->delay != 1)
+        return fail(nullptr, DPO_EINVAL, "delay must be 0 or 1");
+    const float reals[] = {hp->beta1, hp->beta2, hp->eps, hp->weight_decay, hp->ef_lambda,
+                           hp->max_grad_norm};
+    for (float r : reals)
+        if (!std::isfinite(r))
+            return fail(nullptr, DPO_EINVAL, "hyperparameters must be finite");
+    if (!(hp->beta1 >= 0.0f && hp->beta1 < 1.0f && hp->beta2 >= 0.0f && hp->beta2 < 1.0f))
+        return fail(nullptr, DPO_EINVAL, "beta1 and beta2 must lie in [0, 1)");
+    if (hp->eps < 0.0f || hp->weight_decay < 0.0f)
+        return fail(nullptr, DPO_EINVAL, "eps and weight_decay must be >= 0");
+
+    // Table: NULL pointers, EF consistency, alignment, overlaps.
+    const bool ef = table[0].ef != nullptr;
+    std::vector<Span> spans;
+    int64_t total_pkts = 0, total_elems = 0;
+    for (int t = 0; t < n_tensors; ++t) {
+        const dpo_tensor &d = table[t];
+        if (d.numel < 0)
+            return fail(nullptr, DPO_EINVAL, "tensor %d: numel < 0", t);
+        if ((d.ef != nullptr) != ef)
+            return fail(nullptr, DPO_EINVAL,
+                        "tensor %d: EF buffers must be given for all tensors or for none", t);
+        if ((d.flags & ~DPO_WD_ON) != 0)
+            return fail(nullptr, DPO_EINVAL, "tensor %d: unknown flags 0x%x", t, d.flags);
+        if (d.numel == 0)
+            continue;
+        if (d.master == nullptr || d.m == nullptr || d.v == nullptr || d.grad == nullptr)
+            return fail(nullptr, DPO_EINVAL, "tensor %d: master, m, v and grad are required", t);
+        if (hp->delay == 1 && d.stash == nullptr)
+            return fail(nullptr, DPO_EINVAL, "tensor %d: delay = 1 needs a stash buffer", t);
+        if (param_dtype == DPO_BF16 && d.param == nullptr)
+            return fail(nullptr, DPO_EINVAL, "tensor %d: bf16 params need a param buffer", t);
+        if (param_dtype == DPO_F32 && d.param != nullptr)
+            return fail(nullptr, DPO_EINVAL,
+                        "tensor %d: with fp32 params the master is the latest copy; param must be NULL",
+                        t);
+        const struct {
+            const void *p;
+            int64_t bytes;
+            const char *name;
+        } bufs[] = {
+            {d.master, 4 * d.numel, "master"},
+            {d.m, 4 * d.numel, "m"},
+            {d.v, 4 * d.numel, "v"},
+            {d.grad, dt_size(grad_dtype) * d.numel, "grad"},
+            {d.param, dt_size(param_dtype) * d.numel, "param"},
+            {hp->delay == 1 ? d.stash : nullptr, dt_size(stash_dtype) * d.numel, "stash"},
+            {d.ef, 4 * d.numel, "ef"},
+        };
+        for (const auto &b : bufs) {
+            if (b.p == nullptr)
+                continue;
+            if (!aligned16(b.p))
+                return fail(nullptr, DPO_EALIGN, "tensor %d: %s is not 16-byte aligned", t,
+                            b.name);
+            const uintptr_t lo = reinterpret_cast<uintptr_t>(b.p);
+            spans.push_back({lo, lo + static_cast<uintptr_t>(b.bytes), t, b.name});
+        }
+        total_pkts += (d.numel + dpo::kPacket - 1) / dpo::kPacket;
+        total_elems += d.numel;
+    }
+    if (hp->ef_lambda != 0.0f && !ef)
+        return fail(nullptr, DPO_EINVAL, "ef_lambda != 0 needs EF buffers");
+    std::sort(spans.begin(), spans.end(),
+              [](const Span &a, const Span &b) { return a.lo < b.lo; });
+    for (size_t i = 1; i < spans.size(); ++i)
+        if (spans[i].lo < spans[i - 1].hi)
+            return fail(nullptr, DPO_EINVAL, "buffers overlap: tensor %d %s and tensor %d %s",
+                        spans[i - 1].tensor, spans[i - 1].name, spans[i].tensor, spans[i].name);
+
+    // Device checks: every buffer must be device memory of the current device.
+    int device = 0;
+    cudaError_t e = cudaGetDevice(&device);
+    if (e != cudaSuccess)
+        return cuda_fail(nullptr, e, "cudaGetDevice");
+    for (const Span &s : spans) {
+        cudaPointerAttributes attr{};
+        e = cudaPointerGetAttributes(&attr, reinterpret_cast<const void *>(s.lo));
+        if (e != cudaSuccess)
+            return cuda_fail(nullptr, e, "cudaPointerGetAttributes");
+        if ((attr.type != cudaMemoryTypeDevice && attr.type != cudaMemoryTypeManaged) ||
+            attr.device != device)
+            return fail(nullptr, DPO_EINVAL,
+                        "tensor %d: %s is not device memory of the current device", s.tensor,
+                        s.name);
+    }
+
+    dpo_ctx *c = new (std::nothrow) dpo_ctx;
+    if (c == nullptr)
+        return fail(nullptr, DPO_ENOMEM, "out of host memory");
+    c->device = device;
+    c->n = n_tensors;
+    c->param_dt = param_dtype;
+    c->stash_dt = stash_dtype;
+    c->grad_dt = grad_dtype;
+    c->hp = *hp;
+    c->ef = ef;
+    c->clip = hp->max_grad_norm > 0.0f;
+    c->total_pkts = total_pkts;
+    c->total_elems = total_elems;
+    c->table.assign(table, table + n_tensors);
+
+    // Launch geometry: persistent grids, resident CTAs x SMs, never more CTAs
+    // than packet groups of one CTA-width.
+    int sms = 0, per_sm_step = 0, per_sm_norm = 0;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
+    e = dpo::step_ctas_per_sm(param_dtype == DPO_BF16, stash_kind(c), grad_dtype == DPO_BF16,
+                              ef && hp->delay == 1, &per_sm_step);
+    if (e == cudaSuccess)
+        e = dpo::norm_ctas_per_sm(grad_dtype == DPO_BF16, &per_sm_norm);
+    if (e != cudaSuccess) {
+        int rc = cuda_fail(nullptr, e, "occupancy query");
+        delete c;
+        return rc;
+    }
+    const int64_t groups = std::max<int64_t>(1, (total_pkts + dpo::kThreads - 1) / dpo::kThreads);
+    auto grid_of = [&](int per_sm) {
+        return static_cast<int>(std::min<int64_t>(groups, (int64_t)std::max(1, sms) * std::max(1, per_sm)));
+    };
+    c->step_grid = grid_of(per_sm_step);
+    c->norm_grid = grid_of(per_sm_norm);
+    c->stash_grid = c->step_grid;
+
+    // Device block: table, packet prefix, norm scratch.
+    const size_t off_table = 0;
+    const size_t off_pkt = align_up(off_table + sizeof(DevTensor) * n_tensors, 256);
+    const size_t off_part = align_up(off_pkt + sizeof(int64_t) * (n_tensors + 1), 256);
+    const size_t off_scal = align_up(off_part + sizeof(double) * c->norm_grid, 256);
+    const size_t bytes = off_scal + sizeof(dpo::NormScalars);
+    e = cudaMalloc(&c->dev_block, bytes);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        fail(nullptr, DPO_ENOMEM, "cudaMalloc of %zu bytes: %s", bytes, cudaGetErrorString(e));
+        delete c;
+        return DPO_ENOMEM;
+    }
+    char *base = static_cast<char *>(c->dev_block);
+    c->d_table = reinterpret_cast<DevTensor *>(base + off_table);
+    c->d_pkt_begin = reinterpret_cast<int64_t *>(base + off_pkt);
+    c->d_partials = reinterpret_cast<double *>(base + off_part);
+    c->d_scalars = reinterpret_cast<dpo::NormScalars *>(base + off_scal);
+
+    std::vector<DevTensor> dt(n_tensors);
+    std::vector<int64_t> pkt(n_tensors + 1, 0);
+    for (int t = 0; t < n_tensors; ++t) {
+        const dpo_tensor &d = table[t];
+        DevTensor &x = dt[t];
+        x.param = d.param;
+        x.master = d.master;
+        x.m = d.m;
+        x.v = d.v;
+        x.stash = hp->delay == 1 ? d.stash : nullptr;
+        x.ef = d.ef;
+        x.grad = d.grad;
+        x.numel = d.numel;
+        x.flags = d.flags;
+        x.pad_ = 0;
+        pkt[t + 1] = pkt[t] + (d.numel + dpo::kPacket - 1) / dpo::kPacket;
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+    e = cudaMemcpyAsync(c->d_table, dt.data(), sizeof(DevTensor) * n_tensors,
+                        cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(c->d_pkt_begin, pkt.data(), sizeof(int64_t) * (n_tensors + 1),
+                            cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess)
+        e = cudaMemsetAsync(base + off_part, 0, bytes - off_part, s);
+    // The pageable host copies above are staged before cudaMemcpyAsync
+    // returns, so dt and pkt may go out of scope afterwards.
+    if (e != cudaSuccess) {
+        int rc = cuda_fail(nullptr, e, "uploading the tensor table");
+        cudaFree(c->dev_block);
+        delete c;
+        return rc;
+    }
+    if (init_mode == DPO_INIT_FRESH && total_pkts > 0) {
+        dpo::StashArgs a{c->d_table, c->d_pkt_begin, n_tensors, total_pkts, 1};
+        e = dpo::launch_stash(param_dtype == DPO_BF16, stash_kind(c), c->stash_grid, a, s);
+        if (e != cudaSuccess) {
+            int rc = cuda_fail(nullptr, e, "launching the initial stash");
+            cudaFree(c->dev_block);
+            delete c;
+            return rc;
+        }
+    }
+    *out = c;
+    return DPO_OK;
+}
+
+extern "C" int dpo_stash(dpo_ctx *c, void *cuda_stream)
+{
+    if (c == nullptr)
+        return fail(nullptr, DPO_EINVAL, "ctx is NULL");
+    if (c->total_pkts == 0)
+        return DPO_OK;
+    dpo::StashArgs a{c->d_table, c->d_pkt_begin, c->n, c->total_pkts, 0};
+    const cudaError_t e = dpo::launch_stash(c->param_dt == DPO_BF16, stash_kind(c), c->stash_grid,
+                                            a, static_cast<cudaStream_t>(cuda_stream));
+    return e == cudaSuccess ? DPO_OK : cuda_fail(c, e, "stash launch");
+}
+
+extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
+{
+    if (c == nullptr)
+        return fail(nullptr, DPO_EINVAL, "ctx is NULL");
+    if (!std::isfinite(lr) || lr < 0.0f)
+        return fail(c, DPO_EINVAL, "lr must be finite and >= 0");
+    const int64_t k = c->k + 1;   // this call consumes the k-th stale gradient
+    cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+    if (c->total_pkts > 0) {
+        if (c->clip) {
+            dpo::NormArgs na{c->d_table, c->d_pkt_begin, c->n, c->total_pkts,
+                             (double)c->hp.max_grad_norm, c->d_partials, c->d_scalars};
+            const cudaError_t e = dpo::launch_norm(c->grad_dt == DPO_BF16, c->norm_grid, na, s);
+            if (e != cudaSuccess)
+                return cuda_fail(c, e, "gradient-norm launch");
+        }
+        const double b1 = c->hp.beta1, b2 = c->hp.beta2, lrd = lr;
+        const double bc1 = 1.0 - std::pow(b1, (double)k);
+        const double bc2 = 1.0 - std::pow(b2, (double)k);
+        const bool ef = c->ef && c->hp.delay == 1;
+        dpo::StepArgs a{};
+        a.table = c->d_table;
+        a.pkt_begin = c->d_pkt_begin;
+        a.n_tensors = c->n;
+        a.total_pkts = c->total_pkts;
+        a.beta1 = c->hp.beta1;
+        a.omb1 = (float)(1.0 - b1);
+        a.beta2 = c->hp.beta2;
+        a.omb2 = (float)(1.0 - b2);
+        a.step_size = (float)(lrd / bc1);
+        a.inv_sqrt_bc2 = (float)(1.0 / std::sqrt(bc2));
+        a.eps = c->hp.eps;
+        a.lr_wd = (float)(lrd * (double)c->hp.weight_decay);
+        // Alg. 1: the standard rule for t <= 1, i.e. at the first update.
+        a.lam = (ef && k >= 2) ? c->hp.ef_lambda : 0.0f;
+        a.clip = c->clip ? &c->d_scalars->clip : nullptr;
+        const cudaError_t e = dpo::launch_step(c->param_dt == DPO_BF16, stash_kind(c),
+                                               c->grad_dt == DPO_BF16, ef, c->step_grid, a, s);
+        if (e != cudaSuccess)
+            return cuda_fail(c, e, "fused step launch");
+    }
+    c->k = k;
+    return DPO_OK;
+}
+
+extern "C" int dpo_read_weights(const dpo_ctx *c, int which, int tensor, const void **ptr,
+                                dpo_dtype *dtype)
+{
+    if (c == nullptr || ptr == nullptr)
+        return DPO_EINVAL;
+    if (tensor < 0 || tensor >= c->n || (which != DPO_STALE && which != DPO_LATEST))
+        return DPO_EINVAL;
+    const dpo_tensor &d = c->table[tensor];
+    if (which == DPO_STALE && c->hp.delay == 1) {
+        *ptr = d.stash;
+        if (dtype)
+            *dtype = c->stash_dt;
+    } else if (c->param_dt == DPO_BF16) {
+        *ptr = d.param;
+        if (dtype)
+            *dtype = DPO_BF16;
+    } else {
+        *ptr = d.master;
+        if (dtype)
+            *dtype = DPO_F32;
+    }
+    return DPO_OK;
+}
+
+extern "C" int dpo_get_step(const dpo_ctx *c, int64_t *k)
+{
+    if (c == nullptr || k == nullptr)
+        return DPO_EINVAL;
+    *k = c->k;
+    return DPO_OK;
+}
+
+extern "C" int dpo_set_step(dpo_ctx *c, int64_t k)
+{
+    if (c == nullptr)
+        return DPO_EINVAL;
+    if (k < 0)
+        return fail(c, DPO_EINVAL, "step counter must be >= 0");
+    c->k = k;
+    return DPO_OK;
+}
+
+extern "C" int dpo_get_flags(dpo_ctx *c, uint32_t *flags, double *grad_norm, float *clip_scale,
+                             void *cuda_stream)
+{
+    if (c == nullptr)
+        return DPO_EINVAL;
+    dpo::NormScalars h{};
+    cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+    cudaError_t e = cudaMemcpyAsync(&h, c->d_scalars, sizeof h, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess)
+        e = cudaMemsetAsync(&c->d_scalars->flags, 0, sizeof(unsigned int), s);   // read clears
+    if (e == cudaSuccess)
+        e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess)
+        return cuda_fail(c, e, "reading diagnostics");
+    if (flags)
+        *flags = h.flags;
+    if (grad_norm)
+        *grad_norm = h.norm;
+    if (clip_scale)
+        *clip_scale = c->clip ? h.clip : 1.0f;
+    return DPO_OK;
+}
+
+extern "C" int dpo_algorithmic_bytes(const dpo_ctx *c, int64_t *step_bytes, int64_t *norm_bytes)
+{
+    if (c == nullptr)
+        return DPO_EINVAL;
+    // Per element: read master, m, v (fp32) and grad; write master, m, v,
+    // the stash (delay 1) and the bf16 param; EF reads and writes its buffer.
+    int64_t per = 4 * 3 + dt_size(c->grad_dt) + 4 * 3;
+    if (c->hp.delay == 1)
+        per += dt_size(c->stash_dt);
+    if (c->param_dt == DPO_BF16)
+        per += 2;
+    if (c->ef && c->hp.delay == 1)
+        per += 8;
+    if (step_bytes)
+        *step_bytes = per * c->total_elems;
+    if (norm_bytes)
+        *norm_bytes = c->clip ? dt_size(c->grad_dt) * c->total_elems : 0;
+    return DPO_OK;
+}
+
+extern "C" int dpo_launch_config(const dpo_ctx *c, int *step_ctas, int *norm_ctas, int *threads)
+{
+    if (c == nullptr)
+        return DPO_EINVAL;
+    if (step_ctas)
+        *step_ctas = c->step_grid;
+    if (norm_ctas)
+        *norm_ctas = c->norm_grid;
+    if (threads)
+        *threads = dpo::kThreads;
+    return DPO_OK;
+}
+
+extern "C" void dpo_destroy(dpo_ctx *c)
+{
+    if (c == nullptr)
+        return;
+    if (c->dev_block != nullptr)
+        cudaFree(c->dev_block);
+    delete c;
+}

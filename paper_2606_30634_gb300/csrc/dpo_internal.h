@@ -1,0 +1,91 @@
+// dpo_internal.h -- shared definitions of the C-ABI layer and the kernels.
+//
+// The tensor table is a virtual concatenation: tensor t owns packets
+// [pkt_begin[t], pkt_begin[t+1]) of 8 elements each (its last packet may be
+// partial). Every kernel gives CTA c the contiguous packet range
+// [P c / G, P (c+1) / G) of the concatenation, so a CTA looks a tensor up
+// only when its range crosses a tensor boundary.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace dpo {
+
+constexpr int kThreads = 256;   // threads per CTA of every kernel
+constexpr int kPacket = 8;      // elements per packet: 16 B of bf16, 32 B of fp32
+
+// Device copy of one table entry.
+struct DevTensor {
+    void *param;        // bf16 latest copy or nullptr
+    float *master;
+    float *m;
+    float *v;
+    void *stash;        // stash dtype, or nullptr when not written
+    float *ef;          // EF buffer or nullptr
+    const void *grad;
+    int64_t numel;
+    uint32_t flags;
+    uint32_t pad_;
+};
+
+// Kernel template selectors.
+enum StashKind { kStashNone = 0, kStashF32 = 1, kStashBF16 = 2 };
+
+// Scalars of one fused step, precomputed on the host in double and rounded
+// once to fp32.
+struct StepArgs {
+    const DevTensor *table;
+    const int64_t *pkt_begin;   // n_tensors + 1 prefix offsets
+    int n_tensors;
+    int64_t total_pkts;
+    float beta1, omb1;          // beta1, 1 - beta1
+    float beta2, omb2;          // beta2, 1 - beta2
+    float step_size;            // lr / (1 - beta1^k)
+    float inv_sqrt_bc2;         // 1 / sqrt(1 - beta2^k)
+    float eps;
+    float lr_wd;                // lr * weight_decay
+    float lam;                  // lambda of this call (0 at k = 1, Alg. 1)
+    const float *clip;          // device clip coefficient, or nullptr
+};
+
+// Device scalars written by the norm pass (one per context).
+struct NormScalars {
+    double norm;          // global gradient norm of the last clipped step
+    float clip;           // clip coefficient used by that step
+    unsigned int ticket;  // CTA arrival counter, 0 between launches
+    unsigned int flags;   // DPO_FLAG_* bits, sticky until dpo_get_flags reads them
+    unsigned int pad_;
+};
+
+struct NormArgs {
+    const DevTensor *table;
+    const int64_t *pkt_begin;
+    int n_tensors;
+    int64_t total_pkts;
+    double max_norm;            // clip threshold (> 0)
+    double *partials;           // one per CTA (scratch)
+    NormScalars *out;           // norm, clip coefficient, ticket, flags
+};
+
+struct StashArgs {
+    const DevTensor *table;
+    const int64_t *pkt_begin;
+    int n_tensors;
+    int64_t total_pkts;
+    int zero_state;             // also zero m, v and the EF buffer (fresh start)
+};
+
+// Launchers (dpo_kernels.cu). Each returns the launch's cudaError_t.
+cudaError_t launch_step(bool param_bf16, StashKind stash, bool grad_bf16, bool ef,
+                        int grid, const StepArgs &a, cudaStream_t s);
+cudaError_t launch_norm(bool grad_bf16, int grid, const NormArgs &a, cudaStream_t s);
+cudaError_t launch_stash(bool param_bf16, StashKind stash, int grid, const StashArgs &a,
+                         cudaStream_t s);
+
+// Resident CTAs per SM of each kernel at kThreads threads (occupancy query).
+cudaError_t step_ctas_per_sm(bool param_bf16, StashKind stash, bool grad_bf16, bool ef,
+                             int *n);
+cudaError_t norm_ctas_per_sm(bool grad_bf16, int *n);
+
+}  // namespace dpo

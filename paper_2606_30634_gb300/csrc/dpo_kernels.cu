@@ -1,0 +1,443 @@
+// dpo_kernels.cu -- sm_103a kernels of the one-step-delayed AdamW step.
+//
+//   fused_step_kernel   the whole per-element step of Alg. 1 with AdamW and
+//                       the lambda-scaled Error Feedback (Eq. (1), App. A.4)
+//                       in one pass over HBM: read master, m, v, grad (and
+//                       the EF buffer); write master, m, v, stash, the bf16
+//                       latest copy (and the EF buffer).
+//   grad_sqnorm_kernel  global ||g||^2 over the whole table for clipping
+//                       (App. E.1), deterministic: fixed per-thread order,
+//                       fixed block tree, fixed-order sum of the per-CTA
+//                       partials by the last CTA to finish (no spin-wait).
+//   stash_kernel        stash := master, param := master (Alg. 1 start, mode
+//                       switches), optionally zeroing m, v and the EF buffer.
+//
+// All three are persistent (grid = SMs x resident CTAs) and give each CTA a
+// contiguous range of 8-element packets of the virtual concatenation of the
+// tensors; data moves in 128-bit coalesced accesses with streaming
+// (evict-first) cache hints, since no element is touched twice in a step.
+// The step is elementwise and HBM-bound: no tensor-core work exists here.
+#include "dpo_internal.h"
+
+#include <cuda_bf16.h>
+#include <math.h>
+
+namespace dpo {
+namespace {
+
+// ---------------------------------------------------------------- I/O ----
+
+__device__ __forceinline__ void ld8(const float *p, float (&r)[8])
+{
+    const float4 a = __ldcs(reinterpret_cast<const float4 *>(p));
+    const float4 b = __ldcs(reinterpret_cast<const float4 *>(p) + 1);
+    r[0] = a.x; r[1] = a.y; r[2] = a.z; r[3] = a.w;
+    r[4] = b.x; r[5] = b.y; r[6] = b.z; r[7] = b.w;
+}
+
+__device__ __forceinline__ void ld8(const __nv_bfloat16 *p, float (&r)[8])
+{
+    const uint4 q = __ldcs(reinterpret_cast<const uint4 *>(p));
+    const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        r[2 * j] = __uint_as_float(w[j] << 16);
+        r[2 * j + 1] = __uint_as_float(w[j] & 0xFFFF0000u);
+    }
+}
+
+__device__ __forceinline__ void st8(float *p, const float (&r)[8])
+{
+    __stcs(reinterpret_cast<float4 *>(p), make_float4(r[0], r[1], r[2], r[3]));
+    __stcs(reinterpret_cast<float4 *>(p) + 1, make_float4(r[4], r[5], r[6], r[7]));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
+{
+    const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);   // round to nearest even
+    return *reinterpret_cast<const uint32_t *>(&h);
+}
+
+__device__ __forceinline__ void st8(__nv_bfloat16 *p, const float (&r)[8])
+{
+    const uint4 q = make_uint4(pack_bf16x2(r[0], r[1]), pack_bf16x2(r[2], r[3]),
+                               pack_bf16x2(r[4], r[5]), pack_bf16x2(r[6], r[7]));
+    __stcs(reinterpret_cast<uint4 *>(p), q);
+}
+
+__device__ __forceinline__ float ld1(const float *p) { return __ldcs(p); }
+__device__ __forceinline__ float ld1(const __nv_bfloat16 *p) { return __bfloat162float(*p); }
+__device__ __forceinline__ void st1(float *p, float x) { __stcs(p, x); }
+__device__ __forceinline__ void st1(__nv_bfloat16 *p, float x) { *p = __float2bfloat16_rn(x); }
+
+template <bool BF16> struct Elem { using T = float; };
+template <> struct Elem<true> { using T = __nv_bfloat16; };
+
+template <int SK> struct StashT { using T = float; };
+template <> struct StashT<kStashBF16> { using T = __nv_bfloat16; };
+
+// First tensor whose packet range ends after packet p (pkt_begin sorted,
+// pkt_begin[0] = 0, pkt_begin[n] = total).
+__device__ __forceinline__ int find_tensor(const int64_t *pkt_begin, int n, int64_t p)
+{
+    int lo = 0, hi = n;   // answer in [lo, hi)
+    while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (__ldg(pkt_begin + mid) <= p)
+            lo = mid;
+        else
+            hi = mid;
+    }
+    return lo;
+}
+
+__device__ __forceinline__ void cta_range(int64_t total, int64_t *lo, int64_t *hi)
+{
+    *lo = total * (int64_t)blockIdx.x / gridDim.x;
+    *hi = total * (int64_t)(blockIdx.x + 1) / gridDim.x;
+}
+
+// ------------------------------------------------------- the fused step ----
+
+struct Scalars {
+    float beta1, omb1, beta2, omb2, step_size, inv_sqrt_bc2, eps, lam;
+};
+
+// Moments with the (clipped) stale gradient, then the AdamW update
+//   u = lr (m_hat / (sqrt(v_hat) + eps) + wd x_t)
+// with lr / (1 - beta1^k) and 1 / sqrt(1 - beta2^k) folded on the host.
+__device__ __forceinline__ float adamw_update(const Scalars &s, float g, float x, float wd_lr,
+                                              float &m, float &v)
+{
+    m = fmaf(s.beta1, m, s.omb1 * g);
+    v = fmaf(s.beta2, v, (s.omb2 * g) * g);
+    const float denom = fmaf(sqrtf(v), s.inv_sqrt_bc2, s.eps);
+    return fmaf(s.step_size, m / denom, wd_lr * x);
+}
+
+template <int PB, int SK, int GB, int EF>
+__global__ void __launch_bounds__(kThreads) fused_step_kernel(const StepArgs a)
+{
+    using GT = typename Elem<GB != 0>::T;
+    using ST = typename StashT<SK>::T;
+
+    int64_t lo, hi;
+    cta_range(a.total_pkts, &lo, &hi);
+    if (lo >= hi)
+        return;
+
+    const Scalars s{a.beta1, a.omb1, a.beta2, a.omb2, a.step_size, a.inv_sqrt_bc2, a.eps, a.lam};
+    const float clip = a.clip != nullptr ? __ldg(a.clip) : 1.0f;
+    const bool use_prev = EF && a.lam != 0.0f;
+
+    for (int t = find_tensor(a.pkt_begin, a.n_tensors, lo); t < a.n_tensors; ++t) {
+        const int64_t tb = __ldg(a.pkt_begin + t);
+        const int64_t te = __ldg(a.pkt_begin + t + 1);
+        if (tb >= hi)
+            break;
+        if (te <= lo)
+            continue;
+        const DevTensor d = a.table[t];
+        float *__restrict__ master = d.master;
+        float *__restrict__ mm = d.m;
+        float *__restrict__ vv = d.v;
+        float *__restrict__ ef = d.ef;
+        const GT *__restrict__ grad = static_cast<const GT *>(d.grad);
+        ST *__restrict__ stash = static_cast<ST *>(d.stash);
+        __nv_bfloat16 *__restrict__ param = static_cast<__nv_bfloat16 *>(d.param);
+        const float wd_lr = (d.flags & 1u) ? a.lr_wd : 0.0f;
+        const int64_t full = d.numel / kPacket;
+        const int64_t q_end = (hi < te ? hi : te) - tb;
+
+        for (int64_t q = (lo > tb ? lo : tb) - tb + threadIdx.x; q < q_end; q += kThreads) {
+            const int64_t e = q * kPacket;
+            if (q < full) {
+                float x[8], m[8], v[8], g[8], up[8];
+                ld8(master + e, x);
+                ld8(mm + e, m);
+                ld8(vv + e, v);
+                ld8(grad + e, g);
+                if (use_prev)
+                    ld8(ef + e, up);
+                if (SK != kStashNone)
+                    st8(stash + e, x);   // stash := x_t, before the update
+                float u[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    u[j] = adamw_update(s, g[j] * clip, x[j], wd_lr, m[j], v[j]);
+                    const float xs = x[j] - u[j];
+                    x[j] = use_prev ? fmaf(-s.lam, u[j] - up[j], xs) : xs;
+                }
+                st8(master + e, x);
+                st8(mm + e, m);
+                st8(vv + e, v);
+                if (EF)
+                    st8(ef + e, u);
+                if (PB)
+                    st8(param + e, x);
+            } else {
+                // the tensor's last, partial packet
+                for (int64_t i = e; i < d.numel; ++i) {
+                    float x = master[i], m = mm[i], v = vv[i];
+                    const float g = ld1(grad + i);
+                    if (SK != kStashNone)
+                        st1(stash + i, x);
+                    const float u = adamw_update(s, g * clip, x, wd_lr, m, v);
+                    const float xs = x - u;
+                    x = use_prev ? fmaf(-s.lam, u - ef[i], xs) : xs;
+                    master[i] = x;
+                    mm[i] = m;
+                    vv[i] = v;
+                    if (EF)
+                        ef[i] = u;
+                    if (PB)
+                        st1(param + i, x);
+                }
+            }
+        }
+    }
+}
+
+// ------------------------------------------------------ gradient norm ----
+
+__device__ __forceinline__ double block_sum(double x, double *red)
+{
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1)
+        x += __shfl_down_sync(0xFFFFFFFFu, x, off);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0)
+        red[warp] = x;
+    __syncthreads();
+    double r = 0.0;
+    if (warp == 0) {
+        r = lane < kThreads / 32 ? red[lane] : 0.0;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1)
+            r += __shfl_down_sync(0xFFFFFFFFu, r, off);
+    }
+    __syncthreads();
+    return r;   // valid in thread 0
+}
+
+// Kahan-compensated fp32 accumulation of per-packet sums of squares (the
+// compensation keeps the per-thread error near one rounding however many
+// packets a thread visits), fp64 from the block reduction on.
+__device__ __forceinline__ void kahan_add(float &sum, float &c, float x)
+{
+    const float y = x - c;
+    const float t = sum + y;
+    c = (t - sum) - y;
+    sum = t;
+}
+
+template <int GB>
+__global__ void __launch_bounds__(kThreads) grad_sqnorm_kernel(const NormArgs a)
+{
+    using GT = typename Elem<GB != 0>::T;
+    __shared__ double red[kThreads / 32];
+    __shared__ bool last;
+
+    int64_t lo, hi;
+    cta_range(a.total_pkts, &lo, &hi);
+    float sum = 0.0f, comp = 0.0f;
+    if (lo < hi) {
+        for (int t = find_tensor(a.pkt_begin, a.n_tensors, lo); t < a.n_tensors; ++t) {
+            const int64_t tb = __ldg(a.pkt_begin + t);
+            const int64_t te = __ldg(a.pkt_begin + t + 1);
+            if (tb >= hi)
+                break;
+            if (te <= lo)
+                continue;
+            const GT *__restrict__ grad = static_cast<const GT *>(a.table[t].grad);
+            const int64_t numel = a.table[t].numel;
+            const int64_t full = numel / kPacket;
+            const int64_t q_end = (hi < te ? hi : te) - tb;
+            for (int64_t q = (lo > tb ? lo : tb) - tb + threadIdx.x; q < q_end; q += kThreads) {
+                const int64_t e = q * kPacket;
+                float p;
+                if (q < full) {
+                    float g[8];
+                    ld8(grad + e, g);
+                    p = ((g[0] * g[0] + g[1] * g[1]) + (g[2] * g[2] + g[3] * g[3])) +
+                        ((g[4] * g[4] + g[5] * g[5]) + (g[6] * g[6] + g[7] * g[7]));
+                } else {
+                    p = 0.0f;
+                    for (int64_t i = e; i < numel; ++i) {
+                        const float g = ld1(grad + i);
+                        p += g * g;
+                    }
+                }
+                kahan_add(sum, comp, p);
+            }
+        }
+    }
+    const double cta = block_sum((double)sum - (double)comp, red);
+
+    // Publish this CTA's partial; the last CTA to arrive finishes the sum in
+    // CTA order, so the result does not depend on arrival order.
+    if (threadIdx.x == 0) {
+        a.partials[blockIdx.x] = cta;
+        __threadfence();
+        const unsigned int prev = atomicAdd(&a.out->ticket, 1u);
+        last = (prev == gridDim.x - 1);
+    }
+    __syncthreads();
+    if (!last)
+        return;
+    __threadfence();
+    double acc = 0.0;
+    for (int b = threadIdx.x; b < (int)gridDim.x; b += kThreads)
+        acc += __ldcg(a.partials + b);
+    const double total = block_sum(acc, red);
+    if (threadIdx.x == 0) {
+        const double norm = sqrt(total);
+        double coef = a.max_norm / (norm + 1e-6);
+        coef = coef > 1.0 ? 1.0 : coef;   // a NaN norm stays NaN and reaches every element
+        if (!isfinite(total))
+            a.out->flags |= 1u;
+        a.out->clip = (float)coef;
+        a.out->norm = norm;
+        a.out->ticket = 0u;   // ready for the next launch
+    }
+}
+
+// -------------------------------------------------------------- stash ----
+
+template <int PB, int SK>
+__global__ void __launch_bounds__(kThreads) stash_kernel(const StashArgs a)
+{
+    using ST = typename StashT<SK>::T;
+    int64_t lo, hi;
+    cta_range(a.total_pkts, &lo, &hi);
+    if (lo >= hi)
+        return;
+    for (int t = find_tensor(a.pkt_begin, a.n_tensors, lo); t < a.n_tensors; ++t) {
+        const int64_t tb = __ldg(a.pkt_begin + t);
+        const int64_t te = __ldg(a.pkt_begin + t + 1);
+        if (tb >= hi)
+            break;
+        if (te <= lo)
+            continue;
+        const DevTensor d = a.table[t];
+        ST *stash = static_cast<ST *>(d.stash);
+        __nv_bfloat16 *param = static_cast<__nv_bfloat16 *>(d.param);
+        const int64_t full = d.numel / kPacket;
+        const int64_t q_end = (hi < te ? hi : te) - tb;
+        for (int64_t q = (lo > tb ? lo : tb) - tb + threadIdx.x; q < q_end; q += kThreads) {
+            const int64_t e = q * kPacket;
+            if (q < full) {
+                float x[8];
+                ld8(d.master + e, x);
+                if (SK != kStashNone)
+                    st8(stash + e, x);
+                if (PB)
+                    st8(param + e, x);
+                if (a.zero_state) {
+                    const float z[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+                    st8(d.m + e, z);
+                    st8(d.v + e, z);
+                    if (d.ef != nullptr)
+                        st8(d.ef + e, z);
+                }
+            } else {
+                for (int64_t i = e; i < d.numel; ++i) {
+                    const float x = d.master[i];
+                    if (SK != kStashNone)
+                        st1(stash + i, x);
+                    if (PB)
+                        st1(param + i, x);
+                    if (a.zero_state) {
+                        d.m[i] = 0.0f;
+                        d.v[i] = 0.0f;
+                        if (d.ef != nullptr)
+                            d.ef[i] = 0.0f;
+                    }
+                }
+            }
+        }
+    }
+}
+
+// ------------------------------------------------------------ dispatch ----
+
+using StepFn = void (*)(StepArgs);
+
+template <int PB, int GB>
+StepFn pick_step_sk(StashKind sk, bool ef)
+{
+    switch (sk) {
+    case kStashF32:
+        return ef ? fused_step_kernel<PB, kStashF32, GB, 1> : fused_step_kernel<PB, kStashF32, GB, 0>;
+    case kStashBF16:
+        return ef ? fused_step_kernel<PB, kStashBF16, GB, 1> : fused_step_kernel<PB, kStashBF16, GB, 0>;
+    default:
+        return ef ? nullptr : fused_step_kernel<PB, kStashNone, GB, 0>;
+    }
+}
+
+StepFn pick_step(bool pb, StashKind sk, bool gb, bool ef)
+{
+    if (pb)
+        return gb ? pick_step_sk<1, 1>(sk, ef) : pick_step_sk<1, 0>(sk, ef);
+    return gb ? pick_step_sk<0, 1>(sk, ef) : pick_step_sk<0, 0>(sk, ef);
+}
+
+using StashFn = void (*)(StashArgs);
+
+template <int PB>
+StashFn pick_stash_sk(StashKind sk)
+{
+    switch (sk) {
+    case kStashF32:
+        return stash_kernel<PB, kStashF32>;
+    case kStashBF16:
+        return stash_kernel<PB, kStashBF16>;
+    default:
+        return stash_kernel<PB, kStashNone>;
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_step(bool pb, StashKind sk, bool gb, bool ef, int grid, const StepArgs &a,
+                        cudaStream_t s)
+{
+    StepFn f = pick_step(pb, sk, gb, ef);
+    if (f == nullptr)
+        return cudaErrorInvalidValue;
+    f<<<grid, kThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_norm(bool gb, int grid, const NormArgs &a, cudaStream_t s)
+{
+    if (gb)
+        grad_sqnorm_kernel<1><<<grid, kThreads, 0, s>>>(a);
+    else
+        grad_sqnorm_kernel<0><<<grid, kThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_stash(bool pb, StashKind sk, int grid, const StashArgs &a, cudaStream_t s)
+{
+    StashFn f = pb ? pick_stash_sk<1>(sk) : pick_stash_sk<0>(sk);
+    f<<<grid, kThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t step_ctas_per_sm(bool pb, StashKind sk, bool gb, bool ef, int *n)
+{
+    StepFn f = pick_step(pb, sk, gb, ef);
+    if (f == nullptr)
+        return cudaErrorInvalidValue;
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, f, kThreads, 0);
+}
+
+cudaError_t norm_ctas_per_sm(bool gb, int *n)
+{
+    return gb ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, grad_sqnorm_kernel<1>, kThreads, 0)
+              : cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, grad_sqnorm_kernel<0>, kThreads, 0);
+}
+
+}  // namespace dpo

@@ -1,0 +1,286 @@
+"""Python binding of the C ABI in include/dpo.h (argument marshalling only).
+
+Every function here has the name and meaning of the C entry point it wraps;
+each step of the optimizer runs in ``libdpo.so``'s CUDA kernels. PyTorch only
+provides device memory and streams: buffers are passed as raw device
+pointers, streams as ``cudaStream_t`` handles.
+
+``DelayedAdamW`` is a convenience owner of the state buffers for a list of
+parameter shapes: it lays every state kind out as one flat, 256-byte-aligned
+device arena (the layout the kernels stream through) and builds the tensor
+table from it.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+from typing import List, Optional, Sequence
+
+from . import build as _build
+
+DPO_OK, DPO_EINVAL, DPO_EALIGN, DPO_EDTYPE, DPO_ECUDA, DPO_ESTATE, DPO_ENOMEM = 0, -1, -2, -3, -4, -5, -6
+DPO_F32, DPO_BF16 = 0, 1
+DPO_WD_ON = 1
+DPO_STALE, DPO_LATEST = 0, 1
+DPO_INIT_FRESH, DPO_INIT_RESUME = 0, 1
+DPO_FLAG_NONFINITE = 1
+
+EXPORTS = ("dpo_init", "dpo_stash", "dpo_step", "dpo_read_weights", "dpo_get_step",
+           "dpo_set_step", "dpo_get_flags", "dpo_algorithmic_bytes", "dpo_launch_config",
+           "dpo_last_error", "dpo_destroy")
+
+
+class DpoError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"[{code}] {msg}")
+        self.code = code
+
+
+class dpo_hparams(ctypes.Structure):
+    _fields_ = [("beta1", ctypes.c_float), ("beta2", ctypes.c_float), ("eps", ctypes.c_float),
+                ("weight_decay", ctypes.c_float), ("ef_lambda", ctypes.c_float),
+                ("max_grad_norm", ctypes.c_float), ("delay", ctypes.c_int)]
+
+
+class dpo_tensor(ctypes.Structure):
+    _fields_ = [("param", ctypes.c_void_p), ("master", ctypes.c_void_p), ("m", ctypes.c_void_p),
+                ("v", ctypes.c_void_p), ("stash", ctypes.c_void_p), ("ef", ctypes.c_void_p),
+                ("grad", ctypes.c_void_p), ("numel", ctypes.c_int64), ("flags", ctypes.c_uint32)]
+
+
+_lib = None
+
+
+def lib_path() -> str:
+    return os.path.join(_build.OUT, "libdpo.so")
+
+
+def load() -> ctypes.CDLL:
+    """Load libdpo.so (building it first if it is missing or stale). Raises
+    if it cannot be built: there is no other implementation to fall back to."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.build()["libdpo.so"]
+    if not os.path.exists(path):
+        raise RuntimeError(f"libdpo.so is missing at {path}")
+    L = ctypes.CDLL(path)
+    P, I, F, V = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, None
+    sig = {
+        "dpo_init": (I, [ctypes.POINTER(P), ctypes.POINTER(dpo_tensor), I, I, I, I,
+                         ctypes.POINTER(dpo_hparams), I, P]),
+        "dpo_stash": (I, [P, P]),
+        "dpo_step": (I, [P, F, P]),
+        "dpo_read_weights": (I, [P, I, I, ctypes.POINTER(P), ctypes.POINTER(I)]),
+        "dpo_get_step": (I, [P, ctypes.POINTER(ctypes.c_int64)]),
+        "dpo_set_step": (I, [P, ctypes.c_int64]),
+        "dpo_get_flags": (I, [P, ctypes.POINTER(ctypes.c_uint32), ctypes.POINTER(ctypes.c_double),
+                              ctypes.POINTER(F), P]),
+        "dpo_algorithmic_bytes": (I, [P, ctypes.POINTER(ctypes.c_int64),
+                                      ctypes.POINTER(ctypes.c_int64)]),
+        "dpo_launch_config": (I, [P, ctypes.POINTER(I), ctypes.POINTER(I), ctypes.POINTER(I)]),
+        "dpo_last_error": (ctypes.c_char_p, [P]),
+        "dpo_destroy": (V, [P]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(L, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = L
+    return L
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _check(rc: int, ctx) -> None:
+    if rc != DPO_OK:
+        raise DpoError(rc, dpo_last_error(ctx))
+
+
+def dpo_last_error(ctx) -> str:
+    return load().dpo_last_error(ctx).decode()
+
+
+def dpo_init(table: Sequence[dpo_tensor], param_dtype: int, stash_dtype: int, grad_dtype: int,
+             hp: dpo_hparams, init_mode: int = DPO_INIT_FRESH, stream=None):
+    """Returns the context handle (an int). Raises DpoError on failure."""
+    L = load()
+    arr = (dpo_tensor * len(table))(*table)
+    out = ctypes.c_void_p()
+    rc = L.dpo_init(ctypes.byref(out), arr, len(table), param_dtype, stash_dtype, grad_dtype,
+                    ctypes.byref(hp), init_mode, _stream(stream))
+    _check(rc, None)
+    return out.value
+
+
+def dpo_stash(ctx, stream=None) -> None:
+    _check(load().dpo_stash(ctx, _stream(stream)), ctx)
+
+
+def dpo_step(ctx, lr: float, stream=None) -> None:
+    _check(load().dpo_step(ctx, lr, _stream(stream)), ctx)
+
+
+def dpo_read_weights(ctx, which: int, tensor: int):
+    ptr, dt = ctypes.c_void_p(), ctypes.c_int()
+    _check(load().dpo_read_weights(ctx, which, tensor, ctypes.byref(ptr), ctypes.byref(dt)), ctx)
+    return ptr.value, dt.value
+
+
+def dpo_get_step(ctx) -> int:
+    k = ctypes.c_int64()
+    _check(load().dpo_get_step(ctx, ctypes.byref(k)), ctx)
+    return k.value
+
+
+def dpo_set_step(ctx, k: int) -> None:
+    _check(load().dpo_set_step(ctx, k), ctx)
+
+
+def dpo_get_flags(ctx, stream=None):
+    f, n, c = ctypes.c_uint32(), ctypes.c_double(), ctypes.c_float()
+    _check(load().dpo_get_flags(ctx, ctypes.byref(f), ctypes.byref(n), ctypes.byref(c),
+                                _stream(stream)), ctx)
+    return f.value, n.value, c.value
+
+
+def dpo_algorithmic_bytes(ctx):
+    s, n = ctypes.c_int64(), ctypes.c_int64()
+    _check(load().dpo_algorithmic_bytes(ctx, ctypes.byref(s), ctypes.byref(n)), ctx)
+    return s.value, n.value
+
+
+def dpo_launch_config(ctx):
+    a, b, t = ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
+    _check(load().dpo_launch_config(ctx, ctypes.byref(a), ctypes.byref(b), ctypes.byref(t)), ctx)
+    return a.value, b.value, t.value
+
+
+def dpo_destroy(ctx) -> None:
+    if ctx:
+        load().dpo_destroy(ctx)
+
+
+# ------------------------------------------------------------------ owner --
+
+ALIGN_ELEMS = 128   # 256-byte alignment of every tensor in every arena (bf16 or fp32)
+
+
+@dataclass
+class Layout:
+    numels: List[int]
+    offsets: List[int]   # element offset of each tensor in every arena
+    total: int           # arena length in elements (padded)
+
+    @staticmethod
+    def of(numels: Sequence[int]) -> "Layout":
+        offs, o = [], 0
+        for n in numels:
+            offs.append(o)
+            o += -(-int(n) // ALIGN_ELEMS) * ALIGN_ELEMS
+        return Layout([int(n) for n in numels], offs, max(o, ALIGN_ELEMS))
+
+
+class DelayedAdamW:
+    """Owns the state of a one-step-delayed AdamW step for a set of parameter
+    tensors and drives the C ABI.
+
+    Arenas (torch tensors on the device): master, m, v (fp32), grad (grad
+    dtype), param (bf16, only with param_dtype BF16), stash (stash dtype,
+    delay 1), ef (fp32, when ``ef`` is set). ``x0`` fills the master before
+    dpo_init(FRESH); pass ``init_mode=DPO_INIT_RESUME`` to start from arenas
+    restored by ``load_state``.
+    """
+
+    def __init__(self, numels: Sequence[int], *, param_dtype=DPO_BF16, stash_dtype=DPO_F32,
+                 grad_dtype=DPO_BF16, lr=3e-4, beta1=0.9, beta2=0.95, eps=1e-8,
+                 weight_decay=0.1, ef=False, ef_lambda=1.0, max_grad_norm=0.0, delay=1,
+                 wd_on: Optional[Sequence[bool]] = None, device=None, x0=None,
+                 init_mode=DPO_INIT_FRESH, stream=None):
+        import torch
+        self.torch = torch
+        self.device = torch.device(device or "cuda")
+        self.layout = Layout.of(numels)
+        self.param_dtype, self.stash_dtype, self.grad_dtype = param_dtype, stash_dtype, grad_dtype
+        self.delay = delay
+        self.lr = lr
+        tdt = {DPO_F32: torch.float32, DPO_BF16: torch.bfloat16}
+        n = self.layout.total
+        alloc = lambda dt: torch.empty(n, dtype=dt, device=self.device)
+        self.master = alloc(torch.float32)
+        self.m = alloc(torch.float32)
+        self.v = alloc(torch.float32)
+        self.grad = alloc(tdt[grad_dtype])
+        self.grad.zero_()
+        self.param = alloc(torch.bfloat16) if param_dtype == DPO_BF16 else None
+        self.stash = alloc(tdt[stash_dtype]) if delay == 1 else None
+        self.ef = alloc(torch.float32) if ef else None
+        if x0 is not None:
+            self.master.copy_(x0)
+        self.hp = dpo_hparams(beta1, beta2, eps, weight_decay, ef_lambda if ef else 0.0,
+                              max_grad_norm, delay)
+        wd_on = list(wd_on) if wd_on is not None else [True] * len(numels)
+        table = []
+        for i, (cnt, off) in enumerate(zip(self.layout.numels, self.layout.offsets)):
+            ptr = lambda t: (t.data_ptr() + off * t.element_size()) if t is not None else None
+            table.append(dpo_tensor(ptr(self.param), ptr(self.master), ptr(self.m), ptr(self.v),
+                                    ptr(self.stash), ptr(self.ef), ptr(self.grad), cnt,
+                                    DPO_WD_ON if wd_on[i] else 0))
+        self.table = table
+        self.ctx = dpo_init(table, param_dtype, stash_dtype, grad_dtype, self.hp, init_mode,
+                            stream)
+
+    def view(self, arena, i: int):
+        off, cnt = self.layout.offsets[i], self.layout.numels[i]
+        return arena[off:off + cnt]
+
+    def grads(self, i: int):
+        return self.view(self.grad, i)
+
+    def stale(self, i: int):
+        """What the next forward/backward reads (dpo_read_weights(DPO_STALE))."""
+        if self.delay == 1:
+            return self.view(self.stash, i)
+        return self.latest(i)
+
+    def latest(self, i: int):
+        return self.view(self.param if self.param is not None else self.master, i)
+
+    def step(self, lr: Optional[float] = None, stream=None) -> None:
+        dpo_step(self.ctx, self.lr if lr is None else lr, stream)
+
+    def restash(self, stream=None) -> None:
+        dpo_stash(self.ctx, stream)
+
+    @property
+    def k(self) -> int:
+        return dpo_get_step(self.ctx)
+
+    def state_dict(self) -> dict:
+        bufs = {n: getattr(self, n) for n in ("master", "m", "v", "param", "stash", "ef")}
+        return {"k": self.k, **{n: b.clone() for n, b in bufs.items() if b is not None}}
+
+    def load_state(self, sd: dict) -> None:
+        for n in ("master", "m", "v", "param", "stash", "ef"):
+            if getattr(self, n) is not None:
+                getattr(self, n).copy_(sd[n])
+        dpo_set_step(self.ctx, int(sd["k"]))
+
+    def close(self) -> None:
+        if getattr(self, "ctx", None):
+            dpo_destroy(self.ctx)
+            self.ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

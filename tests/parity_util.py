@@ -1,0 +1,212 @@
+"""Parity harness: the CUDA path (through the C ABI) and the oracle, run on the
+same seeded inputs and compared element by element.
+
+Tolerances (the error metric below):
+  fp32 state   err = max_i |gpu_i - ref_i| / max(|ref_i|, 1e-2 rms(ref))
+               <= 1e-6 after one step, <= 1e-4 after any number of steps;
+  bf16 copies  within 1 bf16 ulp of the oracle's rounded fp32 value.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+from typing import List, Optional, Sequence
+
+import numpy as np
+
+import oracle
+from paper_2606_30634_gb300 import dpo, synth
+
+TOL_ONE_STEP = 1e-6
+TOL_RUN = 1e-4
+
+STORE = {dpo.DPO_F32: oracle.F32, dpo.DPO_BF16: oracle.BF16}
+
+
+def rel_err(gpu: np.ndarray, ref: np.ndarray) -> float:
+    gpu = np.asarray(gpu, np.float64)
+    ref = np.asarray(ref, np.float64)
+    if ref.size == 0:
+        return 0.0
+    if not np.array_equal(np.isfinite(gpu), np.isfinite(ref)):
+        return float("inf")
+    fin = np.isfinite(ref)
+    gpu, ref = gpu[fin], ref[fin]
+    if ref.size == 0:
+        return 0.0
+    floor = 1e-2 * np.sqrt(np.mean(ref * ref))
+    den = np.maximum(np.abs(ref), floor if floor > 0 else np.finfo(np.float64).tiny)
+    return float(np.max(np.abs(gpu - ref) / den))
+
+
+def bf16_ord(bits: np.ndarray) -> np.ndarray:
+    b = np.asarray(bits, np.uint16).astype(np.int32)
+    return np.where(b & 0x8000, -(b & 0x7FFF), b)
+
+
+def bf16_bits_of(values: np.ndarray) -> np.ndarray:
+    """bf16 bit patterns of values that are exactly bf16 (the oracle's)."""
+    f = np.asarray(values, np.float64).astype(np.float32)
+    return (f.view(np.uint32) >> 16).astype(np.uint16)
+
+
+def bf16_ulps(gpu_bits: np.ndarray, ref_values: np.ndarray) -> int:
+    if len(gpu_bits) == 0:
+        return 0
+    return int(np.max(np.abs(bf16_ord(gpu_bits) - bf16_ord(bf16_bits_of(ref_values)))))
+
+
+@dataclass
+class Case:
+    numels: Sequence[int]
+    param_dtype: int = dpo.DPO_BF16
+    stash_dtype: int = dpo.DPO_F32
+    grad_dtype: int = dpo.DPO_BF16
+    ef: bool = False
+    ef_lambda: float = 1.0
+    max_grad_norm: float = 0.0
+    delay: int = 1
+    lr: float = 3e-4
+    weight_decay: float = 0.1
+    wd_on: Optional[Sequence[bool]] = None
+    seed: int = 0xD0D0
+    grad_sigma: float = 1e-3
+    init_sigma: float = 0.02
+
+
+class Run:
+    """A GPU optimizer and an oracle over the same seeded set."""
+
+    def __init__(self, case: Case, device, sample: Optional[np.ndarray] = None):
+        import torch
+        self.torch = torch
+        self.c = case
+        self.N = int(sum(case.numels))
+        self.offs = np.concatenate([[0], np.cumsum(case.numels)]).astype(np.int64)
+        self.gpu = dpo.DelayedAdamW(
+            case.numels, param_dtype=case.param_dtype, stash_dtype=case.stash_dtype,
+            grad_dtype=case.grad_dtype, lr=case.lr, weight_decay=case.weight_decay,
+            ef=case.ef, ef_lambda=case.ef_lambda, max_grad_norm=case.max_grad_norm,
+            delay=case.delay, wd_on=case.wd_on, device=device,
+            x0=self._dev_x0(device), init_mode=dpo.DPO_INIT_FRESH)
+        # the oracle tracks every element, or only ``sample`` (global indices)
+        self.sample = sample
+        idx = np.arange(self.N) if sample is None else np.asarray(sample, np.int64)
+        self.idx = idx
+        x0 = synth.host_normal_at(case.seed, synth.STREAM_INIT, 0, idx, case.init_sigma)
+        hp = oracle.HParams(lr=case.lr, weight_decay=case.weight_decay,
+                            ef_lambda=case.ef_lambda if case.ef else 0.0,
+                            max_grad_norm=case.max_grad_norm, delay=case.delay).as_f32()
+        if sample is None:
+            parts = np.split(x0.astype(np.float64), self.offs[1:-1])
+            wd = case.wd_on
+        else:
+            parts = [x0.astype(np.float64)]
+            wd = None if case.wd_on is None else [True]
+            self._mask = None
+            if case.wd_on is not None:
+                t_of = np.searchsorted(self.offs, idx, side="right") - 1
+                self._mask = np.array(case.wd_on, bool)[t_of]
+        self.ref = oracle.DelayedOptimizer(
+            parts, hp, ef=case.ef, x_store=oracle.F32, stash_store=STORE[case.stash_dtype],
+            param_store=oracle.BF16 if case.param_dtype == dpo.DPO_BF16 else None, wd_on=wd)
+        if sample is not None and case.wd_on is not None:
+            self.ref.mask = self._mask.astype(np.uint8)
+        # arena index of every tracked element
+        t_of = np.searchsorted(self.offs, idx, side="right") - 1
+        arena_off = np.asarray(self.gpu.layout.offsets, np.int64)
+        self.arena_idx = arena_off[t_of] + (idx - self.offs[t_of])
+        self._arena_idx_dev = torch.from_numpy(self.arena_idx).to(device)
+        self.k = 0
+
+    def _dev_x0(self, device):
+        import torch
+        x0 = torch.empty(dpo.Layout.of(self.c.numels).total, dtype=torch.float32, device=device)
+        lay = dpo.Layout.of(self.c.numels)
+        for i, (o, n) in enumerate(zip(lay.offsets, lay.numels)):
+            if n:
+                synth.dev_normal(self.c.seed, synth.STREAM_INIT, 0, int(self.offs[i]),
+                                 x0[o:o + n], self.c.init_sigma)
+        return x0
+
+    def step(self, lr: Optional[float] = None):
+        """Draw gradient k+1 on both sides and take one step on each."""
+        c = self.c
+        k = self.k + 1
+        for i, n in enumerate(c.numels):
+            if n:
+                synth.dev_normal(c.seed, synth.STREAM_GRAD, k, int(self.offs[i]),
+                                 self.gpu.grads(i), c.grad_sigma)
+        self.gpu.step(lr)
+        gdt = synth.BF16 if c.grad_dtype == dpo.DPO_BF16 else synth.F32
+        g = synth.host_normal_at(c.seed, synth.STREAM_GRAD, k, self.idx, c.grad_sigma, gdt)
+        g = synth.bf16_bits_to_f32(g) if gdt == synth.BF16 else g
+        sq = None
+        if c.max_grad_norm > 0 and self.sample is not None:
+            sq = self.full_sqnorm(k)
+        lr32 = None if lr is None else float(np.float32(lr))
+        self.ref.step(g.astype(np.float64), tag=self.ref.read_weights("stale")[1], lr=lr32, sq=sq)
+        self.k = k
+
+    def full_sqnorm(self, k: int) -> float:
+        """The oracle's squared norm of the whole k-th gradient (drawn on the
+        host in chunks)."""
+        c = self.c
+        gdt = synth.BF16 if c.grad_dtype == dpo.DPO_BF16 else synth.F32
+        total, chunk = 0.0, 1 << 24
+        for lo in range(0, self.N, chunk):
+            n = min(chunk, self.N - lo)
+            g = synth.host_normal(c.seed, synth.STREAM_GRAD, k, lo, n, c.grad_sigma, gdt)
+            total += oracle.sqnorm_bf16(g) if gdt == synth.BF16 else oracle.sqnorm_f32(g)
+        return total
+
+    def gather(self, arena) -> np.ndarray:
+        t = arena.index_select(0, self._arena_idx_dev)
+        if t.dtype == self.torch.bfloat16:
+            return t.view(self.torch.int16).cpu().numpy().view(np.uint16)
+        return t.cpu().numpy()
+
+    def compare(self) -> dict:
+        """Errors of every state buffer against the oracle."""
+        self.torch.cuda.synchronize()
+        g, r = self.gpu, self.ref
+        out = {"master": rel_err(self.gather(g.master), r.x),
+               "m": rel_err(self.gather(g.m), r.m),
+               "v": rel_err(self.gather(g.v), r.v)}
+        if g.ef is not None:
+            out["ef"] = rel_err(self.gather(g.ef), r.u_prev)
+        if g.stash is not None:
+            s = self.gather(g.stash)
+            if self.c.stash_dtype == dpo.DPO_BF16:
+                out["stash_ulp"] = bf16_ulps(s, r.stash)
+            else:
+                out["stash"] = rel_err(s, r.stash)
+        if g.param is not None:
+            out["param_ulp"] = bf16_ulps(self.gather(g.param), r.param)
+        return out
+
+    def assert_close(self, tol: float) -> dict:
+        e = self.compare()
+        for key, val in e.items():
+            if key.endswith("_ulp"):
+                assert val <= 1, (key, e)
+            else:
+                assert val <= tol, (key, e)
+        return e
+
+    def close(self):
+        self.gpu.close()
+
+
+def sample_indices(numels: Sequence[int], n_random: int, seed: int = 1, edge: int = 9) -> np.ndarray:
+    """Random global indices plus the first and last ``edge`` elements of
+    every tensor (tensor boundaries and partial packets)."""
+    offs = np.concatenate([[0], np.cumsum(numels)]).astype(np.int64)
+    N = int(offs[-1])
+    rng = np.random.default_rng(seed)
+    parts = [rng.integers(0, N, n_random)]
+    for i, n in enumerate(numels):
+        if n:
+            lo, hi = offs[i], offs[i + 1]
+            parts.append(np.arange(lo, min(hi, lo + edge)))
+            parts.append(np.arange(max(lo, hi - edge), hi))
+    return np.unique(np.concatenate(parts))

@@ -1,0 +1,71 @@
+"""Host-side logic of bench.py: the max-over-ranks timing and whole-job
+aggregation across processes (gloo, world size 2, CPU only), the JSON of the
+reference arm, and the committed-traffic lookup."""
+from __future__ import annotations
+
+import json
+import os
+import socket
+import subprocess
+import sys
+
+import pytest
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+import bench  # noqa: E402
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
+
+
+def _worker(rank, world, port, q):
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    secs = [2.0, 3.0][rank]
+    value, t = bench.aggregate(units_per_rank=600.0, seconds_per_rank=secs, world=world)
+    q.put((rank, value, t))
+    dist.destroy_process_group()
+
+
+def test_aggregate_takes_slowest_rank_gloo():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = sorted(q.get(timeout=120) for _ in procs)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    for rank, value, t in res:
+        assert t == 3.0                      # max over ranks
+        assert value == pytest.approx(1200.0 / 3.0)   # all ranks' units / slowest time
+
+
+def test_single_rank_aggregate():
+    assert bench.aggregate(10.0, 2.0, 1) == (5.0, 2.0)
+
+
+def test_reference_arm_json_line():
+    env = dict(os.environ, OMP_NUM_THREADS="2")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+                        "--steps", "1", "--warmup", "0", "--cpu-seconds", "0.5"],
+                       capture_output=True, text=True, env=env, timeout=600, cwd=ROOT)
+    assert r.returncode == 0, r.stderr[-2000:]
+    line = json.loads(r.stdout.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["unit"] == "params/s" and line["value"] > 0
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == 2
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["higher_is_better"] is True
+
+
+def test_traffic_lookup_ignores_stale_summaries(tmp_path, monkeypatch):
+    assert bench.committed_traffic("no-such-kernel") is None

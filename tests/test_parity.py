@@ -1,0 +1,237 @@
+"""GPU parity: the CUDA path through the C ABI against the oracle, element by
+element, on small seeded tables spanning many CTAs, ragged tails and empty
+tensors, in every supported dtype / mode combination."""
+from __future__ import annotations
+
+import ctypes
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2606_30634_gb300 import dpo, synth
+from parity_util import TOL_ONE_STEP, TOL_RUN, Case, Run, bf16_ulps, rel_err
+
+pytestmark = pytest.mark.gpu
+
+# many CTA ranges, 8-element packets with partial tails, an empty tensor
+RAGGED = [1, 7, 8, 9, 4095, 4096, 65537, 0, 3, 300_001, 33]
+
+F, B = dpo.DPO_F32, dpo.DPO_BF16
+
+COMBOS = [
+    # param, stash, grad, ef, clip, delay
+    (B, F, B, False, 0.0, 1),   # GPT-2 / Llama-1B-like layout
+    (B, F, B, True, 0.0, 1),
+    (B, F, B, True, 1.0, 1),    # clipped (the Llama-1B workload clips)
+    (B, B, B, True, 0.0, 1),    # Llama-7B layout
+    (B, B, B, False, 0.0, 1),
+    (F, F, F, False, 0.0, 1),   # flat fp32
+    (F, F, F, True, 0.0, 1),
+    (F, B, F, True, 0.05, 1),
+    (B, F, F, False, 0.0, 0),   # synchronous AdamW
+    (F, F, B, False, 0.02, 0),
+]
+
+
+@pytest.mark.parametrize("pdt,sdt,gdt,ef,clip,delay", COMBOS)
+def test_ragged_table_parity(cuda_device, pdt, sdt, gdt, ef, clip, delay):
+    case = Case(RAGGED, param_dtype=pdt, stash_dtype=sdt, grad_dtype=gdt, ef=ef,
+                max_grad_norm=clip, delay=delay)
+    run = Run(case, cuda_device)
+    try:
+        errs = []
+        for k in range(1, 7):
+            run.step()
+            errs.append(run.assert_close(TOL_ONE_STEP if k == 1 else TOL_RUN))
+            if clip > 0:
+                _, norm, coef = dpo.dpo_get_flags(run.gpu.ctx)
+                assert norm ** 2 == pytest.approx(run.ref.last_sqnorm, rel=1e-6)
+                assert coef == pytest.approx(run.ref.last_clip, rel=1e-6)
+                assert coef < 1.0   # the threshold is below the gradient norm
+    finally:
+        run.close()
+
+
+@pytest.mark.parametrize("lam", [0.0, 0.5, 2.0])
+def test_ef_lambda_sweep(cuda_device, lam):
+    """App. A.4: lambda-scaled correction, lambda in {0, 0.5, 2}."""
+    run = Run(Case(RAGGED, ef=True, ef_lambda=lam), cuda_device)
+    try:
+        for k in range(1, 5):
+            run.step()
+            run.assert_close(TOL_ONE_STEP if k == 1 else TOL_RUN)
+    finally:
+        run.close()
+
+
+def test_changing_lr_and_weight_decay_mask(cuda_device):
+    wd_on = [i % 2 == 0 for i in range(len(RAGGED))]
+    run = Run(Case(RAGGED, ef=True, wd_on=wd_on, weight_decay=0.5), cuda_device)
+    try:
+        for k, lr in enumerate([1e-3, 5e-4, 2e-3, 0.0, 1e-4], start=1):
+            run.step(lr)
+            run.assert_close(TOL_ONE_STEP if k == 1 else TOL_RUN)
+    finally:
+        run.close()
+
+
+def test_ef_lambda_zero_is_standard_bitwise(cuda_device):
+    a = Run(Case(RAGGED, ef=False), cuda_device)
+    b = Run(Case(RAGGED, ef=True, ef_lambda=0.0), cuda_device)
+    try:
+        for _ in range(4):
+            a.step()
+            b.step()
+        torch.cuda.synchronize()
+        assert torch.equal(a.gpu.master, b.gpu.master)
+        assert torch.equal(a.gpu.param, b.gpu.param)
+    finally:
+        a.close()
+        b.close()
+
+
+def test_stash_is_previous_latest_bitwise(cuda_device):
+    """After every step the stash (bf16) equals the previous step's bf16
+    latest weights: the next gradient is evaluated one version behind."""
+    run = Run(Case(RAGGED, stash_dtype=B, ef=True), cuda_device)
+    try:
+        prev = run.gpu.param.clone()
+        for _ in range(4):
+            run.step()
+            torch.cuda.synchronize()
+            for i, n in enumerate(RAGGED):
+                assert torch.equal(run.gpu.view(run.gpu.stash, i), run.gpu.view(prev, i))
+            prev = run.gpu.param.clone()
+        for i in range(len(RAGGED)):
+            p, dt = dpo.dpo_read_weights(run.gpu.ctx, dpo.DPO_STALE, i)
+            assert dt == B and p == run.gpu.view(run.gpu.stash, i).data_ptr()
+            p, dt = dpo.dpo_read_weights(run.gpu.ctx, dpo.DPO_LATEST, i)
+            assert dt == B and p == run.gpu.view(run.gpu.param, i).data_ptr()
+    finally:
+        run.close()
+
+
+def test_padding_between_tensors_untouched(cuda_device):
+    """Guard values in the alignment padding of every arena survive steps."""
+    run = Run(Case(RAGGED, ef=True), cuda_device)
+    try:
+        lay = run.gpu.layout
+        pad = torch.ones(lay.total, dtype=torch.bool, device=cuda_device)
+        for o, n in zip(lay.offsets, lay.numels):
+            pad[o:o + n] = False
+        arenas = [run.gpu.master, run.gpu.m, run.gpu.v, run.gpu.param, run.gpu.stash, run.gpu.ef]
+        for a in arenas:
+            a[pad] = 777.0
+        for _ in range(3):
+            run.step()
+        torch.cuda.synchronize()
+        for a in arenas:
+            assert bool((a[pad].float() == 777.0).all())
+        run.assert_close(TOL_RUN)
+    finally:
+        run.close()
+
+
+def test_deterministic(cuda_device):
+    outs = []
+    for _ in range(2):
+        run = Run(Case(RAGGED, ef=True, max_grad_norm=1e-3), cuda_device)
+        for _ in range(3):
+            run.step()
+        torch.cuda.synchronize()
+        outs.append((run.gpu.master.clone(), dpo.dpo_get_flags(run.gpu.ctx)))
+        run.close()
+    assert torch.equal(outs[0][0], outs[1][0])
+    assert outs[0][1] == outs[1][1]
+
+
+def test_checkpoint_resume_bitwise(cuda_device):
+    """5 steps, save, restore into a new context (INIT_RESUME), 5 more steps:
+    bitwise equal to 10 straight steps."""
+    case = Case(RAGGED, stash_dtype=B, ef=True, max_grad_norm=0.05)
+    straight = Run(case, cuda_device)
+    split = Run(case, cuda_device)
+    try:
+        for _ in range(10):
+            straight.step()
+        for _ in range(5):
+            split.step()
+        sd = split.gpu.state_dict()
+        split.gpu.close()
+        fresh = dpo.DelayedAdamW(case.numels, param_dtype=case.param_dtype,
+                                 stash_dtype=case.stash_dtype, grad_dtype=case.grad_dtype,
+                                 ef=True, max_grad_norm=case.max_grad_norm,
+                                 device=cuda_device, init_mode=dpo.DPO_INIT_RESUME)
+        fresh.load_state(sd)
+        split.gpu = fresh
+        assert dpo.dpo_get_step(fresh.ctx) == 5
+        for _ in range(5):
+            split.step()
+        torch.cuda.synchronize()
+        for name in ("master", "m", "v", "param", "stash", "ef"):
+            assert torch.equal(getattr(straight.gpu, name), getattr(split.gpu, name)), name
+    finally:
+        straight.close()
+        split.close()
+
+
+def test_nonfinite_gradient_flag(cuda_device):
+    run = Run(Case([1000, 17], max_grad_norm=1.0), cuda_device)
+    try:
+        run.step()
+        flags, norm, _ = dpo.dpo_get_flags(run.gpu.ctx)
+        assert flags == 0 and np.isfinite(norm)
+        synth.dev_normal(1, synth.STREAM_GRAD, 9, 0, run.gpu.grads(0), 1e-3)
+        run.gpu.grads(1)[3] = float("nan")
+        run.gpu.step()
+        flags, norm, coef = dpo.dpo_get_flags(run.gpu.ctx)
+        assert flags & dpo.DPO_FLAG_NONFINITE and np.isnan(norm) and np.isnan(coef)
+        assert bool(torch.isnan(run.gpu.master[:1000]).all())   # NaN reaches every element
+        flags, _, _ = dpo.dpo_get_flags(run.gpu.ctx)
+        assert flags == 0   # reading cleared the flag
+    finally:
+        run.close()
+
+
+def test_dpo_stash_resets_stale_copy(cuda_device):
+    run = Run(Case(RAGGED, stash_dtype=F), cuda_device)
+    try:
+        run.step()
+        run.step()
+        dpo.dpo_stash(run.gpu.ctx)
+        torch.cuda.synchronize()
+        assert torch.equal(run.gpu.stash, run.gpu.master)
+    finally:
+        run.close()
+
+
+def test_misaligned_device_pointer_rejected(cuda_device):
+    buf = torch.zeros(1 << 12, dtype=torch.float32, device=cuda_device)
+    p = buf.data_ptr()
+    t = dpo.dpo_tensor(None, p + 4, p + 8192, p + 4096, p + 12288, None, p + 2048, 10, 1)
+    with pytest.raises(dpo.DpoError) as e:
+        dpo.dpo_init([t], F, F, F, dpo.dpo_hparams(0.9, 0.95, 1e-8, 0.1, 0.0, 0.0, 1))
+    assert e.value.code == dpo.DPO_EALIGN
+
+
+def test_host_pointer_rejected(cuda_device):
+    host = np.zeros(1 << 12, np.float32)
+    p = host.ctypes.data
+    p += (-p) % 16
+    t = dpo.dpo_tensor(None, p, p + 4096, p + 8192, p + 12288, None, p + 14000 - 14000 % 16, 10, 1)
+    with pytest.raises(dpo.DpoError) as e:
+        dpo.dpo_init([t], F, F, F, dpo.dpo_hparams(0.9, 0.95, 1e-8, 0.1, 0.0, 0.0, 1))
+    assert e.value.code == dpo.DPO_EINVAL
+
+
+def test_launch_geometry_is_persistent(cuda_device):
+    run = Run(Case([50_000_000]), cuda_device)
+    try:
+        steps, norms, threads = dpo.dpo_launch_config(run.gpu.ctx)
+        sms = torch.cuda.get_device_properties(cuda_device).multi_processor_count
+        assert threads == 256 and steps % sms == 0 and norms % sms == 0
+        sb, nb = dpo.dpo_algorithmic_bytes(run.gpu.ctx)
+        assert sb == 50_000_000 * (12 + 2 + 12 + 4 + 2) and nb == 0
+    finally:
+        run.close()
