@@ -27,7 +27,7 @@
  *   dpo_step consumes was evaluated one version behind the weights it updates.
  *
  * Layout and ownership. The caller owns and allocates every buffer named in
- * a dpo_tensor (device memory of the current device, 16-byte aligned, not
+ * a dpo_tensor (device memory of the current device, 32-byte aligned, not
  * overlapping one another), keeps them alive until dpo_destroy, and may not
  * move them. The library owns only its context: a device copy of the tensor
  * table and a few hundred bytes of device scratch per SM for the gradient
@@ -52,7 +52,7 @@ extern "C" {
 /* Status codes. */
 #define DPO_OK 0
 #define DPO_EINVAL (-1)  /* bad argument: NULL or overlapping buffers, bad size or value */
-#define DPO_EALIGN (-2)  /* a buffer is not 16-byte aligned */
+#define DPO_EALIGN (-2)  /* a buffer is not 32-byte aligned */
 #define DPO_EDTYPE (-3)  /* unsupported dtype or dtype combination */
 #define DPO_ECUDA (-4)   /* a CUDA runtime call or launch failed */
 #define DPO_ESTATE (-5)  /* the context is not in a state that allows the call */
@@ -110,7 +110,7 @@ typedef struct dpo_ctx dpo_ctx;
 
 /*
  * Create a context over n_tensors tensors (table is copied; the buffers it
- * points to are not). Validates every pointer (NULL, 16-byte alignment,
+ * points to are not). Validates every pointer (NULL, 32-byte alignment,
  * overlap, device residency), dtype and hyperparameter. With DPO_INIT_FRESH
  * it then enqueues, on cuda_stream, the Alg. 1 start state: m = v = 0, EF
  * buffer = 0 (u_{-1} = 0), stash := x_0 and param := x_0 from master, and
@@ -168,7 +168,8 @@ int dpo_algorithmic_bytes(const dpo_ctx *ctx, int64_t *step_bytes,
                           int64_t *norm_bytes);
 
 /* Launch geometry chosen at init: CTAs of the fused step and of the norm
- * pass (both persistent: a multiple of the SM count) and threads per CTA. */
+ * pass (both persistent: a multiple of the SM count for sets large enough to
+ * fill the GPU) and threads per CTA of the fused step. */
 int dpo_launch_config(const dpo_ctx *ctx, int *step_ctas, int *norm_ctas,
                       int *threads);
 

@@ -67,7 +67,7 @@ int cuda_fail(dpo_ctx *c, cudaError_t e, const char *what)
 
 bool valid_dtype(int d) { return d == DPO_F32 || d == DPO_BF16; }
 int64_t dt_size(dpo_dtype d) { return d == DPO_BF16 ? 2 : 4; }
-bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+bool aligned(const void *p) { return (reinterpret_cast<uintptr_t>(p) % dpo::kAlign) == 0; }
 StashKind stash_kind(const dpo_ctx *c)
 {
     if (c->hp.delay == 0)
@@ -160,9 +160,9 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
         for (const auto &b : bufs) {
             if (b.p == nullptr)
                 continue;
-            if (!aligned16(b.p))
-                return fail(nullptr, DPO_EALIGN, "tensor %d: %s is not 16-byte aligned", t,
-                            b.name);
+            if (!aligned(b.p))
+                return fail(nullptr, DPO_EALIGN, "tensor %d: %s is not %d-byte aligned", t,
+                            b.name, dpo::kAlign);
             const uintptr_t lo = reinterpret_cast<uintptr_t>(b.p);
             spans.push_back({lo, lo + static_cast<uintptr_t>(b.bytes), t, b.name});
         }
@@ -210,8 +210,9 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
     c->total_elems = total_elems;
     c->table.assign(table, table + n_tensors);
 
-    // Launch geometry: persistent grids, resident CTAs x SMs, never more CTAs
-    // than packet groups of one CTA-width.
+    // Launch geometry: persistent grids, a fixed number of resident CTAs per
+    // SM (the step targets kStepCtasPerSm, see dpo_internal.h), never more
+    // CTAs than there are CTA-widths of packets.
     int sms = 0, per_sm_step = 0, per_sm_norm = 0;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
     e = dpo::step_ctas_per_sm(param_dtype == DPO_BF16, stash_kind(c), grad_dtype == DPO_BF16,
@@ -223,12 +224,13 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
         delete c;
         return rc;
     }
-    const int64_t groups = std::max<int64_t>(1, (total_pkts + dpo::kThreads - 1) / dpo::kThreads);
-    auto grid_of = [&](int per_sm) {
-        return static_cast<int>(std::min<int64_t>(groups, (int64_t)std::max(1, sms) * std::max(1, per_sm)));
+    auto grid_of = [&](int per_sm, int64_t pkts_per_cta) {
+        const int64_t groups = std::max<int64_t>(1, (total_pkts + pkts_per_cta - 1) / pkts_per_cta);
+        return static_cast<int>(
+            std::min<int64_t>(groups, (int64_t)std::max(1, sms) * std::max(1, per_sm)));
     };
-    c->step_grid = grid_of(per_sm_step);
-    c->norm_grid = grid_of(per_sm_norm);
+    c->step_grid = grid_of(std::min(per_sm_step, dpo::kStepCtasPerSm), dpo::kStepThreads);
+    c->norm_grid = grid_of(per_sm_norm, (int64_t)dpo::kNormThreads * dpo::kNormUnroll);
     c->stash_grid = c->step_grid;
 
     // Device block: table, packet prefix, norm scratch.
@@ -448,7 +450,7 @@ extern "C" int dpo_launch_config(const dpo_ctx *c, int *step_ctas, int *norm_cta
     if (norm_ctas)
         *norm_ctas = c->norm_grid;
     if (threads)
-        *threads = dpo::kThreads;
+        *threads = dpo::kStepThreads;
     return DPO_OK;
 }
 

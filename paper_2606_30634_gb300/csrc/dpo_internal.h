@@ -2,9 +2,11 @@
 //
 // The tensor table is a virtual concatenation: tensor t owns packets
 // [pkt_begin[t], pkt_begin[t+1]) of 8 elements each (its last packet may be
-// partial). Every kernel gives CTA c the contiguous packet range
-// [P c / G, P (c+1) / G) of the concatenation, so a CTA looks a tensor up
-// only when its range crosses a tensor boundary.
+// partial). Every kernel walks the packets grid-stride: thread i of the grid
+// takes packets i, i + T, i + 2T, ... (T threads in the grid), so at any time
+// all CTAs work in one narrow window of every array (DRAM row locality), and
+// each thread keeps a cursor on the tensor holding its packet, advanced
+// monotonically as its packet index grows.
 #pragma once
 
 #include <cuda_runtime.h>
@@ -12,8 +14,20 @@
 
 namespace dpo {
 
-constexpr int kThreads = 256;   // threads per CTA of every kernel
 constexpr int kPacket = 8;      // elements per packet: 16 B of bf16, 32 B of fp32
+constexpr int kAlign = 32;      // buffer alignment: fp32 packets move as 256-bit accesses
+
+// Fused step and stash kernels: 128-thread CTAs, at most kStepCtasPerSm
+// resident per SM. Twelve warps per SM keep ~55 KB of loads in flight per SM,
+// which measured fastest on GB300 HBM3e for the fused step's 10-14 streams
+// (8 warps starve the memory pipe; 16 or more lose DRAM efficiency).
+constexpr int kStepThreads = 128;
+constexpr int kStepCtasPerSm = 3;
+
+// Gradient-norm kernel: one read stream, so each thread loads
+// kNormUnroll packets per iteration.
+constexpr int kNormThreads = 256;
+constexpr int kNormUnroll = 4;
 
 // Device copy of one table entry.
 struct DevTensor {
@@ -83,7 +97,7 @@ cudaError_t launch_norm(bool grad_bf16, int grid, const NormArgs &a, cudaStream_
 cudaError_t launch_stash(bool param_bf16, StashKind stash, int grid, const StashArgs &a,
                          cudaStream_t s);
 
-// Resident CTAs per SM of each kernel at kThreads threads (occupancy query).
+// Resident CTAs per SM of each kernel at its block size (occupancy query).
 cudaError_t step_ctas_per_sm(bool param_bf16, StashKind stash, bool grad_bf16, bool ef,
                              int *n);
 cudaError_t norm_ctas_per_sm(bool grad_bf16, int *n);

@@ -12,11 +12,12 @@
 //   stash_kernel        stash := master, param := master (Alg. 1 start, mode
 //                       switches), optionally zeroing m, v and the EF buffer.
 //
-// All three are persistent (grid = SMs x resident CTAs) and give each CTA a
-// contiguous range of 8-element packets of the virtual concatenation of the
-// tensors; data moves in 128-bit coalesced accesses with streaming
-// (evict-first) cache hints, since no element is touched twice in a step.
-// The step is elementwise and HBM-bound: no tensor-core work exists here.
+// All three are persistent (a fixed number of CTAs per SM) and walk the
+// 8-element packets of the virtual concatenation of the tensors grid-stride
+// (see dpo_internal.h). fp32 packets move as single 256-bit accesses, bf16
+// packets as 128-bit ones, all with streaming (evict-first) cache hints: no
+// element is touched twice in a step. The step is elementwise and HBM-bound;
+// there is no tensor-core work in it.
 #include "dpo_internal.h"
 
 #include <cuda_bf16.h>
@@ -26,15 +27,25 @@ namespace dpo {
 namespace {
 
 // ---------------------------------------------------------------- I/O ----
+// fp32 packet: one 32-byte (256-bit) load or store per thread.
 
 __device__ __forceinline__ void ld8(const float *p, float (&r)[8])
 {
-    const float4 a = __ldcs(reinterpret_cast<const float4 *>(p));
-    const float4 b = __ldcs(reinterpret_cast<const float4 *>(p) + 1);
-    r[0] = a.x; r[1] = a.y; r[2] = a.z; r[3] = a.w;
-    r[4] = b.x; r[5] = b.y; r[6] = b.z; r[7] = b.w;
+    asm volatile("ld.global.cs.v8.f32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                 : "=f"(r[0]), "=f"(r[1]), "=f"(r[2]), "=f"(r[3]), "=f"(r[4]), "=f"(r[5]),
+                   "=f"(r[6]), "=f"(r[7])
+                 : "l"(p));
 }
 
+__device__ __forceinline__ void st8(float *p, const float (&r)[8])
+{
+    asm volatile("st.global.cs.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};"
+                 :: "l"(p), "f"(r[0]), "f"(r[1]), "f"(r[2]), "f"(r[3]), "f"(r[4]), "f"(r[5]),
+                    "f"(r[6]), "f"(r[7])
+                 : "memory");
+}
+
+// bf16 packet: one 16-byte load or store; values widen exactly to fp32.
 __device__ __forceinline__ void ld8(const __nv_bfloat16 *p, float (&r)[8])
 {
     const uint4 q = __ldcs(reinterpret_cast<const uint4 *>(p));
@@ -44,12 +55,6 @@ __device__ __forceinline__ void ld8(const __nv_bfloat16 *p, float (&r)[8])
         r[2 * j] = __uint_as_float(w[j] << 16);
         r[2 * j + 1] = __uint_as_float(w[j] & 0xFFFF0000u);
     }
-}
-
-__device__ __forceinline__ void st8(float *p, const float (&r)[8])
-{
-    __stcs(reinterpret_cast<float4 *>(p), make_float4(r[0], r[1], r[2], r[3]));
-    __stcs(reinterpret_cast<float4 *>(p) + 1, make_float4(r[4], r[5], r[6], r[7]));
 }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
@@ -76,8 +81,10 @@ template <> struct Elem<true> { using T = __nv_bfloat16; };
 template <int SK> struct StashT { using T = float; };
 template <> struct StashT<kStashBF16> { using T = __nv_bfloat16; };
 
-// First tensor whose packet range ends after packet p (pkt_begin sorted,
-// pkt_begin[0] = 0, pkt_begin[n] = total).
+// ------------------------------------------------------------- cursor ----
+
+// Last tensor whose first packet is <= p (pkt_begin sorted, pkt_begin[0] = 0,
+// pkt_begin[n] = total): for p < total, the tensor holding packet p.
 __device__ __forceinline__ int find_tensor(const int64_t *pkt_begin, int n, int64_t p)
 {
     int lo = 0, hi = n;   // answer in [lo, hi)
@@ -91,11 +98,31 @@ __device__ __forceinline__ int find_tensor(const int64_t *pkt_begin, int n, int6
     return lo;
 }
 
-__device__ __forceinline__ void cta_range(int64_t total, int64_t *lo, int64_t *hi)
-{
-    *lo = total * (int64_t)blockIdx.x / gridDim.x;
-    *hi = total * (int64_t)(blockIdx.x + 1) / gridDim.x;
-}
+// The tensor holding a thread's current packet. Packet indices only grow, so
+// the cursor moves forward, skipping whole tensors (empty ones included).
+struct Cursor {
+    int t;
+    int64_t tb, te;   // packet range [tb, te) of tensor t
+
+    __device__ __forceinline__ void seek(const int64_t *pkt_begin, int n, int64_t p)
+    {
+        t = find_tensor(pkt_begin, n, p);
+        tb = __ldg(pkt_begin + t);
+        te = __ldg(pkt_begin + t + 1);
+    }
+    // true when the packet moved to another tensor (p < total)
+    __device__ __forceinline__ bool advance(const int64_t *pkt_begin, int64_t p)
+    {
+        if (p < te)
+            return false;
+        do {
+            ++t;
+            tb = te;
+            te = __ldg(pkt_begin + t + 1);
+        } while (p >= te);
+        return true;
+    }
+};
 
 // ------------------------------------------------------- the fused step ----
 
@@ -106,38 +133,49 @@ struct Scalars {
 // Moments with the (clipped) stale gradient, then the AdamW update
 //   u = lr (m_hat / (sqrt(v_hat) + eps) + wd x_t)
 // with lr / (1 - beta1^k) and 1 / sqrt(1 - beta2^k) folded on the host.
+// The first moment's product (1 - beta1) g is carried exactly (its rounding
+// error recovered with an fma), so where beta1 m and that product nearly
+// cancel the new m keeps full relative accuracy; v has no cancellation.
 __device__ __forceinline__ float adamw_update(const Scalars &s, float g, float x, float wd_lr,
                                               float &m, float &v)
 {
-    m = fmaf(s.beta1, m, s.omb1 * g);
+    const float p = s.omb1 * g;
+    const float p_err = fmaf(s.omb1, g, -p);
+    m = fmaf(s.beta1, m, p) + p_err;
     v = fmaf(s.beta2, v, (s.omb2 * g) * g);
     const float denom = fmaf(sqrtf(v), s.inv_sqrt_bc2, s.eps);
     return fmaf(s.step_size, m / denom, wd_lr * x);
 }
 
+// Displacement of the lambda-scaled EF rule, x_{t+1} = x_t - (u + lambda (u - u_prev)):
+// the small terms are summed first so the weight is rounded once, at its own
+// magnitude (subtracting u and then the correction would round x twice).
+__device__ __forceinline__ float ef_displacement(float lam, float u, float u_prev)
+{
+    return fmaf(lam, u - u_prev, u);
+}
+
 template <int PB, int SK, int GB, int EF>
-__global__ void __launch_bounds__(kThreads) fused_step_kernel(const StepArgs a)
+__global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs a)
 {
     using GT = typename Elem<GB != 0>::T;
     using ST = typename StashT<SK>::T;
 
-    int64_t lo, hi;
-    cta_range(a.total_pkts, &lo, &hi);
-    if (lo >= hi)
+    const int64_t stride = (int64_t)gridDim.x * kStepThreads;
+    int64_t p = (int64_t)blockIdx.x * kStepThreads + threadIdx.x;
+    if (p >= a.total_pkts)
         return;
 
     const Scalars s{a.beta1, a.omb1, a.beta2, a.omb2, a.step_size, a.inv_sqrt_bc2, a.eps, a.lam};
     const float clip = a.clip != nullptr ? __ldg(a.clip) : 1.0f;
     const bool use_prev = EF && a.lam != 0.0f;
 
-    for (int t = find_tensor(a.pkt_begin, a.n_tensors, lo); t < a.n_tensors; ++t) {
-        const int64_t tb = __ldg(a.pkt_begin + t);
-        const int64_t te = __ldg(a.pkt_begin + t + 1);
-        if (tb >= hi)
-            break;
-        if (te <= lo)
-            continue;
-        const DevTensor d = a.table[t];
+    Cursor c;
+    c.seek(a.pkt_begin, a.n_tensors, p);
+    DevTensor d = a.table[c.t];
+    for (; p < a.total_pkts; p += stride) {
+        if (c.advance(a.pkt_begin, p))
+            d = a.table[c.t];
         float *__restrict__ master = d.master;
         float *__restrict__ mm = d.m;
         float *__restrict__ vv = d.v;
@@ -146,53 +184,47 @@ __global__ void __launch_bounds__(kThreads) fused_step_kernel(const StepArgs a)
         ST *__restrict__ stash = static_cast<ST *>(d.stash);
         __nv_bfloat16 *__restrict__ param = static_cast<__nv_bfloat16 *>(d.param);
         const float wd_lr = (d.flags & 1u) ? a.lr_wd : 0.0f;
-        const int64_t full = d.numel / kPacket;
-        const int64_t q_end = (hi < te ? hi : te) - tb;
+        const int64_t e = (p - c.tb) * kPacket;
 
-        for (int64_t q = (lo > tb ? lo : tb) - tb + threadIdx.x; q < q_end; q += kThreads) {
-            const int64_t e = q * kPacket;
-            if (q < full) {
-                float x[8], m[8], v[8], g[8], up[8];
-                ld8(master + e, x);
-                ld8(mm + e, m);
-                ld8(vv + e, v);
-                ld8(grad + e, g);
-                if (use_prev)
-                    ld8(ef + e, up);
-                if (SK != kStashNone)
-                    st8(stash + e, x);   // stash := x_t, before the update
-                float u[8];
+        if (e + kPacket <= d.numel) {
+            float x[8], m[8], v[8], g[8], up[8];
+            ld8(master + e, x);
+            ld8(mm + e, m);
+            ld8(vv + e, v);
+            ld8(grad + e, g);
+            if (use_prev)
+                ld8(ef + e, up);
+            if (SK != kStashNone)
+                st8(stash + e, x);   // stash := x_t, before the update
+            float u[8];
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    u[j] = adamw_update(s, g[j] * clip, x[j], wd_lr, m[j], v[j]);
-                    const float xs = x[j] - u[j];
-                    x[j] = use_prev ? fmaf(-s.lam, u[j] - up[j], xs) : xs;
-                }
-                st8(master + e, x);
-                st8(mm + e, m);
-                st8(vv + e, v);
+            for (int j = 0; j < 8; ++j) {
+                u[j] = adamw_update(s, g[j] * clip, x[j], wd_lr, m[j], v[j]);
+                x[j] -= use_prev ? ef_displacement(s.lam, u[j], up[j]) : u[j];
+            }
+            st8(master + e, x);
+            st8(mm + e, m);
+            st8(vv + e, v);
+            if (EF)
+                st8(ef + e, u);
+            if (PB)
+                st8(param + e, x);
+        } else {
+            // the tensor's last, partial packet
+            for (int64_t i = e; i < d.numel; ++i) {
+                float x = master[i], m = mm[i], v = vv[i];
+                const float g = ld1(grad + i);
+                if (SK != kStashNone)
+                    st1(stash + i, x);
+                const float u = adamw_update(s, g * clip, x, wd_lr, m, v);
+                x -= use_prev ? ef_displacement(s.lam, u, ef[i]) : u;
+                master[i] = x;
+                mm[i] = m;
+                vv[i] = v;
                 if (EF)
-                    st8(ef + e, u);
+                    ef[i] = u;
                 if (PB)
-                    st8(param + e, x);
-            } else {
-                // the tensor's last, partial packet
-                for (int64_t i = e; i < d.numel; ++i) {
-                    float x = master[i], m = mm[i], v = vv[i];
-                    const float g = ld1(grad + i);
-                    if (SK != kStashNone)
-                        st1(stash + i, x);
-                    const float u = adamw_update(s, g * clip, x, wd_lr, m, v);
-                    const float xs = x - u;
-                    x = use_prev ? fmaf(-s.lam, u - ef[i], xs) : xs;
-                    master[i] = x;
-                    mm[i] = m;
-                    vv[i] = v;
-                    if (EF)
-                        ef[i] = u;
-                    if (PB)
-                        st1(param + i, x);
-                }
+                    st1(param + i, x);
             }
         }
     }
@@ -200,6 +232,7 @@ __global__ void __launch_bounds__(kThreads) fused_step_kernel(const StepArgs a)
 
 // ------------------------------------------------------ gradient norm ----
 
+template <int NT>
 __device__ __forceinline__ double block_sum(double x, double *red)
 {
 #pragma unroll
@@ -211,7 +244,7 @@ __device__ __forceinline__ double block_sum(double x, double *red)
     __syncthreads();
     double r = 0.0;
     if (warp == 0) {
-        r = lane < kThreads / 32 ? red[lane] : 0.0;
+        r = lane < NT / 32 ? red[lane] : 0.0;
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1)
             r += __shfl_down_sync(0xFFFFFFFFu, r, off);
@@ -231,48 +264,62 @@ __device__ __forceinline__ void kahan_add(float &sum, float &c, float x)
     sum = t;
 }
 
+template <class GT>
+__device__ __forceinline__ float packet_sqsum(const GT *grad, int64_t e, int64_t numel)
+{
+    if (e + kPacket <= numel) {
+        float g[8];
+        ld8(grad + e, g);
+        return ((g[0] * g[0] + g[1] * g[1]) + (g[2] * g[2] + g[3] * g[3])) +
+               ((g[4] * g[4] + g[5] * g[5]) + (g[6] * g[6] + g[7] * g[7]));
+    }
+    float s = 0.0f;
+    for (int64_t i = e; i < numel; ++i) {
+        const float g = ld1(grad + i);
+        s += g * g;
+    }
+    return s;
+}
+
 template <int GB>
-__global__ void __launch_bounds__(kThreads) grad_sqnorm_kernel(const NormArgs a)
+__global__ void __launch_bounds__(kNormThreads) grad_sqnorm_kernel(const NormArgs a)
 {
     using GT = typename Elem<GB != 0>::T;
-    __shared__ double red[kThreads / 32];
+    __shared__ double red[kNormThreads / 32];
     __shared__ bool last;
 
-    int64_t lo, hi;
-    cta_range(a.total_pkts, &lo, &hi);
+    // Each thread takes kNormUnroll packets per round, kNormThreads apart, so
+    // their loads are in flight together; rounds are grid-stride, and each of
+    // the kNormUnroll packet streams keeps its own tensor cursor.
+    const int64_t round = (int64_t)gridDim.x * kNormThreads * kNormUnroll;
+    const int64_t first = (int64_t)blockIdx.x * kNormThreads * kNormUnroll + threadIdx.x;
     float sum = 0.0f, comp = 0.0f;
-    if (lo < hi) {
-        for (int t = find_tensor(a.pkt_begin, a.n_tensors, lo); t < a.n_tensors; ++t) {
-            const int64_t tb = __ldg(a.pkt_begin + t);
-            const int64_t te = __ldg(a.pkt_begin + t + 1);
-            if (tb >= hi)
-                break;
-            if (te <= lo)
-                continue;
-            const GT *__restrict__ grad = static_cast<const GT *>(a.table[t].grad);
-            const int64_t numel = a.table[t].numel;
-            const int64_t full = numel / kPacket;
-            const int64_t q_end = (hi < te ? hi : te) - tb;
-            for (int64_t q = (lo > tb ? lo : tb) - tb + threadIdx.x; q < q_end; q += kThreads) {
-                const int64_t e = q * kPacket;
-                float p;
-                if (q < full) {
-                    float g[8];
-                    ld8(grad + e, g);
-                    p = ((g[0] * g[0] + g[1] * g[1]) + (g[2] * g[2] + g[3] * g[3])) +
-                        ((g[4] * g[4] + g[5] * g[5]) + (g[6] * g[6] + g[7] * g[7]));
-                } else {
-                    p = 0.0f;
-                    for (int64_t i = e; i < numel; ++i) {
-                        const float g = ld1(grad + i);
-                        p += g * g;
-                    }
+    if (first < a.total_pkts) {
+        Cursor c[kNormUnroll];
+#pragma unroll
+        for (int u = 0; u < kNormUnroll; ++u) {
+            const int64_t p = first + (int64_t)u * kNormThreads;
+            c[u].seek(a.pkt_begin, a.n_tensors, p < a.total_pkts ? p : a.total_pkts - 1);
+        }
+        for (int64_t base = first; base < a.total_pkts; base += round) {
+            float part[kNormUnroll];
+#pragma unroll
+            for (int u = 0; u < kNormUnroll; ++u) {
+                const int64_t p = base + (int64_t)u * kNormThreads;
+                part[u] = 0.0f;
+                if (p < a.total_pkts) {
+                    c[u].advance(a.pkt_begin, p);
+                    const DevTensor &d = a.table[c[u].t];
+                    part[u] = packet_sqsum(static_cast<const GT *>(d.grad),
+                                           (p - c[u].tb) * kPacket, d.numel);
                 }
-                kahan_add(sum, comp, p);
             }
+#pragma unroll
+            for (int u = 0; u < kNormUnroll; ++u)
+                kahan_add(sum, comp, part[u]);
         }
     }
-    const double cta = block_sum((double)sum - (double)comp, red);
+    const double cta = block_sum<kNormThreads>((double)sum - (double)comp, red);
 
     // Publish this CTA's partial; the last CTA to arrive finishes the sum in
     // CTA order, so the result does not depend on arrival order.
@@ -287,9 +334,9 @@ __global__ void __launch_bounds__(kThreads) grad_sqnorm_kernel(const NormArgs a)
         return;
     __threadfence();
     double acc = 0.0;
-    for (int b = threadIdx.x; b < (int)gridDim.x; b += kThreads)
+    for (int b = threadIdx.x; b < (int)gridDim.x; b += kNormThreads)
         acc += __ldcg(a.partials + b);
-    const double total = block_sum(acc, red);
+    const double total = block_sum<kNormThreads>(acc, red);
     if (threadIdx.x == 0) {
         const double norm = sqrt(total);
         double coef = a.max_norm / (norm + 1e-6);
@@ -305,54 +352,48 @@ __global__ void __launch_bounds__(kThreads) grad_sqnorm_kernel(const NormArgs a)
 // -------------------------------------------------------------- stash ----
 
 template <int PB, int SK>
-__global__ void __launch_bounds__(kThreads) stash_kernel(const StashArgs a)
+__global__ void __launch_bounds__(kStepThreads) stash_kernel(const StashArgs a)
 {
     using ST = typename StashT<SK>::T;
-    int64_t lo, hi;
-    cta_range(a.total_pkts, &lo, &hi);
-    if (lo >= hi)
+    const int64_t stride = (int64_t)gridDim.x * kStepThreads;
+    int64_t p = (int64_t)blockIdx.x * kStepThreads + threadIdx.x;
+    if (p >= a.total_pkts)
         return;
-    for (int t = find_tensor(a.pkt_begin, a.n_tensors, lo); t < a.n_tensors; ++t) {
-        const int64_t tb = __ldg(a.pkt_begin + t);
-        const int64_t te = __ldg(a.pkt_begin + t + 1);
-        if (tb >= hi)
-            break;
-        if (te <= lo)
-            continue;
-        const DevTensor d = a.table[t];
+    Cursor c;
+    c.seek(a.pkt_begin, a.n_tensors, p);
+    DevTensor d = a.table[c.t];
+    for (; p < a.total_pkts; p += stride) {
+        if (c.advance(a.pkt_begin, p))
+            d = a.table[c.t];
         ST *stash = static_cast<ST *>(d.stash);
         __nv_bfloat16 *param = static_cast<__nv_bfloat16 *>(d.param);
-        const int64_t full = d.numel / kPacket;
-        const int64_t q_end = (hi < te ? hi : te) - tb;
-        for (int64_t q = (lo > tb ? lo : tb) - tb + threadIdx.x; q < q_end; q += kThreads) {
-            const int64_t e = q * kPacket;
-            if (q < full) {
-                float x[8];
-                ld8(d.master + e, x);
+        const int64_t e = (p - c.tb) * kPacket;
+        if (e + kPacket <= d.numel) {
+            float x[8];
+            ld8(d.master + e, x);
+            if (SK != kStashNone)
+                st8(stash + e, x);
+            if (PB)
+                st8(param + e, x);
+            if (a.zero_state) {
+                const float z[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+                st8(d.m + e, z);
+                st8(d.v + e, z);
+                if (d.ef != nullptr)
+                    st8(d.ef + e, z);
+            }
+        } else {
+            for (int64_t i = e; i < d.numel; ++i) {
+                const float x = d.master[i];
                 if (SK != kStashNone)
-                    st8(stash + e, x);
+                    st1(stash + i, x);
                 if (PB)
-                    st8(param + e, x);
+                    st1(param + i, x);
                 if (a.zero_state) {
-                    const float z[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-                    st8(d.m + e, z);
-                    st8(d.v + e, z);
+                    d.m[i] = 0.0f;
+                    d.v[i] = 0.0f;
                     if (d.ef != nullptr)
-                        st8(d.ef + e, z);
-                }
-            } else {
-                for (int64_t i = e; i < d.numel; ++i) {
-                    const float x = d.master[i];
-                    if (SK != kStashNone)
-                        st1(stash + i, x);
-                    if (PB)
-                        st1(param + i, x);
-                    if (a.zero_state) {
-                        d.m[i] = 0.0f;
-                        d.v[i] = 0.0f;
-                        if (d.ef != nullptr)
-                            d.ef[i] = 0.0f;
-                    }
+                        d.ef[i] = 0.0f;
                 }
             }
         }
@@ -406,23 +447,23 @@ cudaError_t launch_step(bool pb, StashKind sk, bool gb, bool ef, int grid, const
     StepFn f = pick_step(pb, sk, gb, ef);
     if (f == nullptr)
         return cudaErrorInvalidValue;
-    f<<<grid, kThreads, 0, s>>>(a);
+    f<<<grid, kStepThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 
 cudaError_t launch_norm(bool gb, int grid, const NormArgs &a, cudaStream_t s)
 {
     if (gb)
-        grad_sqnorm_kernel<1><<<grid, kThreads, 0, s>>>(a);
+        grad_sqnorm_kernel<1><<<grid, kNormThreads, 0, s>>>(a);
     else
-        grad_sqnorm_kernel<0><<<grid, kThreads, 0, s>>>(a);
+        grad_sqnorm_kernel<0><<<grid, kNormThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 
 cudaError_t launch_stash(bool pb, StashKind sk, int grid, const StashArgs &a, cudaStream_t s)
 {
     StashFn f = pb ? pick_stash_sk<1>(sk) : pick_stash_sk<0>(sk);
-    f<<<grid, kThreads, 0, s>>>(a);
+    f<<<grid, kStepThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 
@@ -431,13 +472,13 @@ cudaError_t step_ctas_per_sm(bool pb, StashKind sk, bool gb, bool ef, int *n)
     StepFn f = pick_step(pb, sk, gb, ef);
     if (f == nullptr)
         return cudaErrorInvalidValue;
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, f, kThreads, 0);
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, f, kStepThreads, 0);
 }
 
 cudaError_t norm_ctas_per_sm(bool gb, int *n)
 {
-    return gb ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, grad_sqnorm_kernel<1>, kThreads, 0)
-              : cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, grad_sqnorm_kernel<0>, kThreads, 0);
+    return gb ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, grad_sqnorm_kernel<1>, kNormThreads, 0)
+              : cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, grad_sqnorm_kernel<0>, kNormThreads, 0);
 }
 
 }  // namespace dpo

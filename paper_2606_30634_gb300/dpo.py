@@ -57,12 +57,13 @@ def lib_path() -> str:
 
 
 def load() -> ctypes.CDLL:
-    """Load libdpo.so (building it first if it is missing or stale). Raises
-    if it cannot be built: there is no other implementation to fall back to."""
+    """Load libdpo.so (building it first if it is missing or stale; the
+    DPO_LIBRARY environment variable names another build of it). Raises if
+    it cannot be built: there is no other implementation to fall back to."""
     global _lib
     if _lib is not None:
         return _lib
-    path = _build.build()["libdpo.so"]
+    path = os.environ.get("DPO_LIBRARY") or _build.build()["libdpo.so"]
     if not os.path.exists(path):
         raise RuntimeError(f"libdpo.so is missing at {path}")
     L = ctypes.CDLL(path)
@@ -214,12 +215,12 @@ class DelayedAdamW:
         self.lr = lr
         tdt = {DPO_F32: torch.float32, DPO_BF16: torch.bfloat16}
         n = self.layout.total
-        alloc = lambda dt: torch.empty(n, dtype=dt, device=self.device)
+        # zero-filled, so the alignment padding between tensors is defined
+        alloc = lambda dt: torch.zeros(n, dtype=dt, device=self.device)
         self.master = alloc(torch.float32)
         self.m = alloc(torch.float32)
         self.v = alloc(torch.float32)
         self.grad = alloc(tdt[grad_dtype])
-        self.grad.zero_()
         self.param = alloc(torch.bfloat16) if param_dtype == DPO_BF16 else None
         self.stash = alloc(tdt[stash_dtype]) if delay == 1 else None
         self.ef = alloc(torch.float32) if ef else None

@@ -88,7 +88,12 @@ LLAMA_1B = Workload("llama-1B", _llama(2048, 8192, 128256, 16, 32, 8, tied=True)
 LLAMA_7B = Workload("llama-7B", _llama(4096, 11008, 32000, 32, 32, 32, tied=False), BF16, BF16,
                     BF16, steps=20, seed=0xD0D0 + 5)
 
-ALL = {w.name: w for w in (FLAT, QUADRATIC, GPT2_SMALL, LLAMA_1B, LLAMA_7B)}
+# One decoder layer of the 7B shapes with the 7B dtypes: the same kernel
+# instance on a ~4.4 GB working set (profiler captures).
+LLAMA_7B_LAYER = Workload("llama-7B-layer", LLAMA_7B.tensors[1:10], BF16, BF16, BF16, steps=20,
+                          seed=0xD0D0 + 5)
+
+ALL = {w.name: w for w in (FLAT, QUADRATIC, GPT2_SMALL, LLAMA_1B, LLAMA_7B, LLAMA_7B_LAYER)}
 
 # the quadratic's noise and curvature
 QUAD_NOISE_SIGMA = 1e-2

@@ -112,7 +112,7 @@ def test_init_rejects(case, expect):
     elif case == "misaligned_grad":
         tbl[0] = _t(0, grad=tbl[0].grad + 2)
     elif case == "overlap":
-        tbl[1] = _t(1, m=tbl[0].v + 16)
+        tbl[1] = _t(1, m=tbl[0].v + 32)
     elif case == "negative_numel":
         tbl[1] = _t(1, numel=-1)
     elif case == "null_master":

@@ -23,7 +23,7 @@ COMBOS = [
     # param, stash, grad, ef, clip, delay
     (B, F, B, False, 0.0, 1),   # GPT-2 / Llama-1B-like layout
     (B, F, B, True, 0.0, 1),
-    (B, F, B, True, 1.0, 1),    # clipped (the Llama-1B workload clips)
+    (B, F, B, True, 0.3, 1),    # clipped (the norm of this table is ~0.6)
     (B, B, B, True, 0.0, 1),    # Llama-7B layout
     (B, B, B, False, 0.0, 1),
     (F, F, F, False, 0.0, 1),   # flat fp32
@@ -66,12 +66,15 @@ def test_ef_lambda_sweep(cuda_device, lam):
 
 
 def test_changing_lr_and_weight_decay_mask(cuda_device):
+    """Learning rate changing every call (the schedule is host-side), decay
+    on every other tensor. The fp32 update x - u carries an absolute error of
+    a few ulps of u, so the one-step bar, set for lr = 3e-4, scales with lr."""
     wd_on = [i % 2 == 0 for i in range(len(RAGGED))]
     run = Run(Case(RAGGED, ef=True, wd_on=wd_on, weight_decay=0.5), cuda_device)
     try:
         for k, lr in enumerate([1e-3, 5e-4, 2e-3, 0.0, 1e-4], start=1):
             run.step(lr)
-            run.assert_close(TOL_ONE_STEP if k == 1 else TOL_RUN)
+            run.assert_close(TOL_ONE_STEP * lr / 3e-4 if k == 1 else TOL_RUN)
     finally:
         run.close()
 
@@ -104,6 +107,8 @@ def test_stash_is_previous_latest_bitwise(cuda_device):
                 assert torch.equal(run.gpu.view(run.gpu.stash, i), run.gpu.view(prev, i))
             prev = run.gpu.param.clone()
         for i in range(len(RAGGED)):
+            if RAGGED[i] == 0:
+                continue   # torch gives empty views a null data_ptr
             p, dt = dpo.dpo_read_weights(run.gpu.ctx, dpo.DPO_STALE, i)
             assert dt == B and p == run.gpu.view(run.gpu.stash, i).data_ptr()
             p, dt = dpo.dpo_read_weights(run.gpu.ctx, dpo.DPO_LATEST, i)
@@ -122,12 +127,12 @@ def test_padding_between_tensors_untouched(cuda_device):
             pad[o:o + n] = False
         arenas = [run.gpu.master, run.gpu.m, run.gpu.v, run.gpu.param, run.gpu.stash, run.gpu.ef]
         for a in arenas:
-            a[pad] = 777.0
+            a[pad] = -3.5   # exact in bf16 and fp32
         for _ in range(3):
             run.step()
         torch.cuda.synchronize()
         for a in arenas:
-            assert bool((a[pad].float() == 777.0).all())
+            assert bool((a[pad].float() == -3.5).all())
         run.assert_close(TOL_RUN)
     finally:
         run.close()
@@ -218,8 +223,8 @@ def test_misaligned_device_pointer_rejected(cuda_device):
 def test_host_pointer_rejected(cuda_device):
     host = np.zeros(1 << 12, np.float32)
     p = host.ctypes.data
-    p += (-p) % 16
-    t = dpo.dpo_tensor(None, p, p + 4096, p + 8192, p + 12288, None, p + 14000 - 14000 % 16, 10, 1)
+    p += (-p) % 32
+    t = dpo.dpo_tensor(None, p, p + 4096, p + 8192, p + 12288, None, p + 13824, 10, 1)
     with pytest.raises(dpo.DpoError) as e:
         dpo.dpo_init([t], F, F, F, dpo.dpo_hparams(0.9, 0.95, 1e-8, 0.1, 0.0, 0.0, 1))
     assert e.value.code == dpo.DPO_EINVAL
@@ -230,7 +235,7 @@ def test_launch_geometry_is_persistent(cuda_device):
     try:
         steps, norms, threads = dpo.dpo_launch_config(run.gpu.ctx)
         sms = torch.cuda.get_device_properties(cuda_device).multi_processor_count
-        assert threads == 256 and steps % sms == 0 and norms % sms == 0
+        assert threads == 128 and steps == 3 * sms and norms % sms == 0
         sb, nb = dpo.dpo_algorithmic_bytes(run.gpu.ctx)
         assert sb == 50_000_000 * (12 + 2 + 12 + 4 + 2) and nb == 0
     finally:
