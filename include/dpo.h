@@ -173,6 +173,46 @@ int dpo_algorithmic_bytes(const dpo_ctx *ctx, int64_t *step_bytes,
 int dpo_launch_config(const dpo_ctx *ctx, int *step_ctas, int *norm_ctas,
                       int *threads);
 
+/*
+ * Gradient norm without device allocation.
+ *
+ * The paper has no counterpart to this entry point; it serves callers that
+ * cannot call cudaMalloc. A training framework whose caching allocator has
+ * already reserved the GPU's memory cannot let a library take more behind
+ * its back, and a latency-critical loop cannot take the device-wide
+ * synchronization cudaMalloc and cudaFree may imply; dpo_init allocates a
+ * small device block, so such callers use this instead. It computes what
+ * the clipped dpo_step computes before its update, for one contiguous
+ * gradient buffer: the global L2 norm (deterministic: fixed chunking and
+ * summation order) and the clip coefficient min(1, max_grad_norm /
+ * (norm + 1e-6)) (1 when max_grad_norm <= 0; NaN when the norm is NaN).
+ *
+ *   grad          device buffer of numel gradients (grad_dtype F32 or BF16),
+ *                 32-byte aligned; 0 <= numel <= DPO_NOALLOC_MAX_NUMEL.
+ *   norm_out      device pointer, receives the norm (double, 8-byte aligned).
+ *   clip_out      device pointer, receives the coefficient (float).
+ *
+ * Its scratch is a fixed file-scope device array of
+ * DPO_NOALLOC_MAX_CHUNKS partial sums (128 KiB), one per chunk of
+ * DPO_NOALLOC_CHUNK_ELEMS elements; every GPU that loads the library holds
+ * it until the process exits. Larger inputs are rejected with DPO_EINVAL.
+ * The call allocates nothing: it enqueues one small memset (clearing the
+ * scratch's counter, which must start at zero) and one kernel on
+ * cuda_stream. The first call on each device looks up the scratch array's
+ * device address (cudaGetSymbolAddress) with that device current; make that
+ * first call before any stream capture. All calls share the scratch array,
+ * which keeps the last call's contents, so calls whose kernels overlap on the
+ * GPU (different streams or host threads on one device) race on it.
+ * Returns DPO_OK, DPO_EINVAL, DPO_EALIGN, DPO_EDTYPE or DPO_ECUDA.
+ */
+#define DPO_NOALLOC_CHUNK_ELEMS (1 << 20)
+#define DPO_NOALLOC_MAX_CHUNKS 16384
+#define DPO_NOALLOC_MAX_NUMEL ((int64_t)DPO_NOALLOC_MAX_CHUNKS * DPO_NOALLOC_CHUNK_ELEMS)
+
+int dpo_grad_norm_noalloc(const void *grad, int64_t numel, dpo_dtype grad_dtype,
+                          float max_grad_norm, double *norm_out, float *clip_out,
+                          void *cuda_stream);
+
 /* Message of the last failing call on ctx (NULL ctx: last dpo_init failure of
  * the calling thread). Never NULL; owned by the library. */
 const char *dpo_last_error(const dpo_ctx *ctx);

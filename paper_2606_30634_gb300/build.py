@@ -29,7 +29,7 @@ COMMON = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O3,-fop
 
 LIBS = {
     "libdpo.so": {
-        "sources": ["csrc/dpo_kernels.cu", "csrc/dpo_abi.cpp"],
+        "sources": ["csrc/dpo_kernels.cu", "csrc/dpo_abi.cpp", "csrc/dpo_noalloc.cu"],
         "headers": ["csrc/dpo_internal.h", "../include/dpo.h"],
         "includes": ["csrc"],
         "ptxas_v": ["csrc/dpo_kernels.cu"],

@@ -28,7 +28,11 @@ DPO_FLAG_NONFINITE = 1
 
 EXPORTS = ("dpo_init", "dpo_stash", "dpo_step", "dpo_read_weights", "dpo_get_step",
            "dpo_set_step", "dpo_get_flags", "dpo_algorithmic_bytes", "dpo_launch_config",
-           "dpo_last_error", "dpo_destroy")
+           "dpo_last_error", "dpo_destroy", "dpo_grad_norm_noalloc")
+
+DPO_NOALLOC_CHUNK_ELEMS = 1 << 20
+DPO_NOALLOC_MAX_CHUNKS = 16384
+DPO_NOALLOC_MAX_NUMEL = DPO_NOALLOC_MAX_CHUNKS * DPO_NOALLOC_CHUNK_ELEMS
 
 
 class DpoError(RuntimeError):
@@ -83,6 +87,7 @@ def load() -> ctypes.CDLL:
         "dpo_launch_config": (I, [P, ctypes.POINTER(I), ctypes.POINTER(I), ctypes.POINTER(I)]),
         "dpo_last_error": (ctypes.c_char_p, [P]),
         "dpo_destroy": (V, [P]),
+        "dpo_grad_norm_noalloc": (I, [P, ctypes.c_int64, I, F, P, P, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -168,6 +173,19 @@ def dpo_launch_config(ctx):
 def dpo_destroy(ctx) -> None:
     if ctx:
         load().dpo_destroy(ctx)
+
+
+def dpo_grad_norm_noalloc(grad, numel: int, grad_dtype: int, max_grad_norm: float, norm_out,
+                          clip_out, stream=None) -> None:
+    """Norm and clip coefficient of one contiguous device gradient buffer,
+    with no device allocation (scratch in a fixed device array; see
+    include/dpo.h for its limit and sharing rules). ``grad``, ``norm_out``
+    (float64) and ``clip_out`` (float32) are device pointers or tensors."""
+    ptr = lambda t: t if isinstance(t, int) or t is None else t.data_ptr()
+    rc = load().dpo_grad_norm_noalloc(ptr(grad), numel, grad_dtype, max_grad_norm,
+                                      ptr(norm_out), ptr(clip_out), _stream(stream))
+    if rc != DPO_OK:
+        raise DpoError(rc, "dpo_grad_norm_noalloc rejected its arguments or failed")
 
 
 # ------------------------------------------------------------------ owner --
