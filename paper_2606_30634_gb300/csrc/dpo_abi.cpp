@@ -211,8 +211,10 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
     c->table.assign(table, table + n_tensors);
 
     // Launch geometry: persistent grids, a fixed number of resident CTAs per
-    // SM (the step targets kStepCtasPerSm, see dpo_internal.h), never more
-    // CTAs than there are CTA-widths of packets.
+    // SM, never more CTAs than there are CTA-widths of packets. The step's
+    // CTAs per SM put about kStepInflightPerSm bytes of loads in flight per SM
+    // (see dpo_internal.h): bytes loaded per packet = master, m, v, grad and,
+    // with EF, the EF buffer.
     int sms = 0, per_sm_step = 0, per_sm_norm = 0;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
     e = dpo::step_ctas_per_sm(param_dtype == DPO_BF16, stash_kind(c), grad_dtype == DPO_BF16,
@@ -229,7 +231,12 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
         return static_cast<int>(
             std::min<int64_t>(groups, (int64_t)std::max(1, sms) * std::max(1, per_sm)));
     };
-    c->step_grid = grid_of(std::min(per_sm_step, dpo::kStepCtasPerSm), dpo::kStepThreads);
+    const bool ef_active = ef && hp->delay == 1;
+    const int64_t load_bytes = dpo::kPacket * (12 + dt_size(grad_dtype) + (ef_active ? 4 : 0));
+    const int want_per_sm = std::max<int>(
+        1, (int)((dpo::kStepInflightPerSm + load_bytes * dpo::kStepThreads / 2) /
+                 (load_bytes * dpo::kStepThreads)));
+    c->step_grid = grid_of(std::min(per_sm_step, want_per_sm), dpo::kStepThreads);
     c->norm_grid = grid_of(per_sm_norm, (int64_t)dpo::kNormThreads * dpo::kNormUnroll);
     c->stash_grid = c->step_grid;
 

@@ -17,12 +17,14 @@ namespace dpo {
 constexpr int kPacket = 8;      // elements per packet: 16 B of bf16, 32 B of fp32
 constexpr int kAlign = 32;      // buffer alignment: fp32 packets move as 256-bit accesses
 
-// Fused step and stash kernels: 128-thread CTAs, at most kStepCtasPerSm
-// resident per SM. Twelve warps per SM keep ~55 KB of loads in flight per SM,
-// which measured fastest on GB300 HBM3e for the fused step's 10-14 streams
-// (8 warps starve the memory pipe; 16 or more lose DRAM efficiency).
+// Fused step and stash kernels: 128-thread CTAs. The number resident per SM
+// is chosen so that about kStepInflightPerSm bytes of loads are in flight per
+// SM (one packet per thread): measured on GB300 HBM3e, fewer starve the
+// memory pipe and more lose DRAM efficiency. That is 3 CTAs (12 warps) for
+// the EF layouts (144-160 B of loads per packet) and 4 CTAs (16 warps) for
+// the standard rule (112-128 B).
 constexpr int kStepThreads = 128;
-constexpr int kStepCtasPerSm = 3;
+constexpr int kStepInflightPerSm = 56 * 1024;
 
 // Gradient-norm kernel: one read stream, so each thread loads
 // kNormUnroll packets per iteration.

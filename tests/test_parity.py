@@ -235,7 +235,7 @@ def test_launch_geometry_is_persistent(cuda_device):
     try:
         steps, norms, threads = dpo.dpo_launch_config(run.gpu.ctx)
         sms = torch.cuda.get_device_properties(cuda_device).multi_processor_count
-        assert threads == 128 and steps == 3 * sms and norms % sms == 0
+        assert threads == 128 and steps == 4 * sms and norms % sms == 0   # standard rule: 4 CTAs/SM
         sb, nb = dpo.dpo_algorithmic_bytes(run.gpu.ctx)
         assert sb == 50_000_000 * (12 + 2 + 12 + 4 + 2) and nb == 0
     finally:
