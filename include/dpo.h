@@ -27,9 +27,16 @@
  *   dpo_step consumes was evaluated one version behind the weights it updates.
  *
  * Layout and ownership. The caller owns and allocates every buffer named in
- * a dpo_tensor (device memory of the current device, 32-byte aligned, not
- * overlapping one another), keeps them alive until dpo_destroy, and may not
- * move them. The library owns only its context: a device copy of the tensor
+ * a dpo_tensor (32-byte aligned, not overlapping one another), keeps them
+ * alive until dpo_destroy, and may not move them. The optimizer state
+ * (master, m, v, stash, EF buffer) is device memory of the current device.
+ * grad and param may be device memory too, or host memory the GPU addresses
+ * directly: pinned memory mapped at the same address (cudaHostAlloc), or
+ * pageable memory on a device with pageable-memory access (NVLink-C2C
+ * systems). The fused kernel then reads the gradients from and writes the new
+ * weights to host memory itself, over the host link, with no staging copy;
+ * the step is then bound by that link (2 B per parameter each way for bf16).
+ * The host must not touch those buffers while a step is in flight. The library owns only its context: a device copy of the tensor
  * table and a few hundred bytes of device scratch per SM for the gradient
  * norm. All launches go to the stream passed in (a cudaStream_t, NULL for the
  * legacy default stream); dpo_step never synchronizes the host.
@@ -111,7 +118,7 @@ typedef struct dpo_ctx dpo_ctx;
 /*
  * Create a context over n_tensors tensors (table is copied; the buffers it
  * points to are not). Validates every pointer (NULL, 32-byte alignment,
- * overlap, device residency), dtype and hyperparameter. With DPO_INIT_FRESH
+ * overlap, residency as above), dtype and hyperparameter. With DPO_INIT_FRESH
  * it then enqueues, on cuda_stream, the Alg. 1 start state: m = v = 0, EF
  * buffer = 0 (u_{-1} = 0), stash := x_0 and param := x_0 from master, and
  * sets k = 0. Supported dtypes: param F32|BF16, stash F32|BF16, grad

@@ -28,6 +28,7 @@ struct dpo_ctx {
     dpo_hparams hp{};
     bool ef = false;
     bool clip = false;
+    bool host_io = false;   // grad or param in host memory
     int64_t k = 0;
     int64_t total_pkts = 0;
     int64_t total_elems = 0;
@@ -79,6 +80,7 @@ struct Span {
     uintptr_t lo, hi;
     int tensor;
     const char *name;
+    bool host_ok;   // grad and param may live in host memory the GPU can address
 };
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -148,14 +150,15 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
             const void *p;
             int64_t bytes;
             const char *name;
+            bool host_ok;
         } bufs[] = {
-            {d.master, 4 * d.numel, "master"},
-            {d.m, 4 * d.numel, "m"},
-            {d.v, 4 * d.numel, "v"},
-            {d.grad, dt_size(grad_dtype) * d.numel, "grad"},
-            {d.param, dt_size(param_dtype) * d.numel, "param"},
-            {hp->delay == 1 ? d.stash : nullptr, dt_size(stash_dtype) * d.numel, "stash"},
-            {d.ef, 4 * d.numel, "ef"},
+            {d.master, 4 * d.numel, "master", false},
+            {d.m, 4 * d.numel, "m", false},
+            {d.v, 4 * d.numel, "v", false},
+            {d.grad, dt_size(grad_dtype) * d.numel, "grad", true},
+            {d.param, dt_size(param_dtype) * d.numel, "param", true},
+            {hp->delay == 1 ? d.stash : nullptr, dt_size(stash_dtype) * d.numel, "stash", false},
+            {d.ef, 4 * d.numel, "ef", false},
         };
         for (const auto &b : bufs) {
             if (b.p == nullptr)
@@ -164,7 +167,7 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
                 return fail(nullptr, DPO_EALIGN, "tensor %d: %s is not %d-byte aligned", t,
                             b.name, dpo::kAlign);
             const uintptr_t lo = reinterpret_cast<uintptr_t>(b.p);
-            spans.push_back({lo, lo + static_cast<uintptr_t>(b.bytes), t, b.name});
+            spans.push_back({lo, lo + static_cast<uintptr_t>(b.bytes), t, b.name, b.host_ok});
         }
         total_pkts += (d.numel + dpo::kPacket - 1) / dpo::kPacket;
         total_elems += d.numel;
@@ -178,21 +181,40 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
             return fail(nullptr, DPO_EINVAL, "buffers overlap: tensor %d %s and tensor %d %s",
                         spans[i - 1].tensor, spans[i - 1].name, spans[i].tensor, spans[i].name);
 
-    // Device checks: every buffer must be device memory of the current device.
+    // Residency: the optimizer state must be device memory of the current
+    // device. grad and param may instead be host memory the GPU addresses
+    // directly (pinned and mapped at the same address, or pageable memory on
+    // a device with pageable-memory access, e.g. over NVLink-C2C); the fused
+    // kernel then reads the gradients and writes the new weights across the
+    // host link itself.
     int device = 0;
     cudaError_t e = cudaGetDevice(&device);
     if (e != cudaSuccess)
         return cuda_fail(nullptr, e, "cudaGetDevice");
+    int pageable_ok = 0;
+    cudaDeviceGetAttribute(&pageable_ok, cudaDevAttrPageableMemoryAccess, device);
+    bool host_io = false;
     for (const Span &s : spans) {
         cudaPointerAttributes attr{};
-        e = cudaPointerGetAttributes(&attr, reinterpret_cast<const void *>(s.lo));
+        const void *ptr = reinterpret_cast<const void *>(s.lo);
+        e = cudaPointerGetAttributes(&attr, ptr);
         if (e != cudaSuccess)
             return cuda_fail(nullptr, e, "cudaPointerGetAttributes");
-        if ((attr.type != cudaMemoryTypeDevice && attr.type != cudaMemoryTypeManaged) ||
-            attr.device != device)
-            return fail(nullptr, DPO_EINVAL,
-                        "tensor %d: %s is not device memory of the current device", s.tensor,
-                        s.name);
+        const bool on_device = (attr.type == cudaMemoryTypeDevice ||
+                                attr.type == cudaMemoryTypeManaged) && attr.device == device;
+        const bool host_mapped = attr.type == cudaMemoryTypeHost && attr.devicePointer == ptr;
+        const bool host_pageable = attr.type == cudaMemoryTypeUnregistered && pageable_ok;
+        if (on_device)
+            continue;
+        if (s.host_ok && (host_mapped || host_pageable)) {
+            host_io = true;
+            continue;
+        }
+        return fail(nullptr, DPO_EINVAL,
+                    s.host_ok ? "tensor %d: %s is neither device memory of the current device "
+                                "nor host memory this device can address"
+                              : "tensor %d: %s is not device memory of the current device",
+                    s.tensor, s.name);
     }
 
     dpo_ctx *c = new (std::nothrow) dpo_ctx;
@@ -208,6 +230,7 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
     c->clip = hp->max_grad_norm > 0.0f;
     c->total_pkts = total_pkts;
     c->total_elems = total_elems;
+    c->host_io = host_io;
     c->table.assign(table, table + n_tensors);
 
     // Launch geometry: persistent grids, a fixed number of resident CTAs per

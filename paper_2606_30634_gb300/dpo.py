@@ -216,14 +216,16 @@ class DelayedAdamW:
     dtype), param (bf16, only with param_dtype BF16), stash (stash dtype,
     delay 1), ef (fp32, when ``ef`` is set). ``x0`` fills the master before
     dpo_init(FRESH); pass ``init_mode=DPO_INIT_RESUME`` to start from arenas
-    restored by ``load_state``.
+    restored by ``load_state``. With ``host_grad`` / ``host_param`` the grad /
+    param arenas are pinned host memory instead, which the fused kernel reads
+    and writes across the host link (see include/dpo.h).
     """
 
     def __init__(self, numels: Sequence[int], *, param_dtype=DPO_BF16, stash_dtype=DPO_F32,
                  grad_dtype=DPO_BF16, lr=3e-4, beta1=0.9, beta2=0.95, eps=1e-8,
                  weight_decay=0.1, ef=False, ef_lambda=1.0, max_grad_norm=0.0, delay=1,
                  wd_on: Optional[Sequence[bool]] = None, device=None, x0=None,
-                 init_mode=DPO_INIT_FRESH, stream=None):
+                 init_mode=DPO_INIT_FRESH, stream=None, host_grad=False, host_param=False):
         import torch
         self.torch = torch
         self.device = torch.device(device or "cuda")
@@ -235,27 +237,51 @@ class DelayedAdamW:
         n = self.layout.total
         # zero-filled, so the alignment padding between tensors is defined
         alloc = lambda dt: torch.zeros(n, dtype=dt, device=self.device)
+        host_alloc = lambda dt: torch.zeros(n, dtype=dt, pin_memory=True)
         self.master = alloc(torch.float32)
         self.m = alloc(torch.float32)
         self.v = alloc(torch.float32)
-        self.grad = alloc(tdt[grad_dtype])
-        self.param = alloc(torch.bfloat16) if param_dtype == DPO_BF16 else None
+        self.grad = (host_alloc if host_grad else alloc)(tdt[grad_dtype])
+        self.param = ((host_alloc if host_param else alloc)(torch.bfloat16)
+                      if param_dtype == DPO_BF16 else None)
         self.stash = alloc(tdt[stash_dtype]) if delay == 1 else None
         self.ef = alloc(torch.float32) if ef else None
         if x0 is not None:
             self.master.copy_(x0)
         self.hp = dpo_hparams(beta1, beta2, eps, weight_decay, ef_lambda if ef else 0.0,
                               max_grad_norm, delay)
-        wd_on = list(wd_on) if wd_on is not None else [True] * len(numels)
+        self.wd_on = list(wd_on) if wd_on is not None else [True] * len(numels)
+        self.ctx = None
+        self._init(init_mode, stream)
+
+    def _init(self, init_mode, stream) -> None:
         table = []
         for i, (cnt, off) in enumerate(zip(self.layout.numels, self.layout.offsets)):
             ptr = lambda t: (t.data_ptr() + off * t.element_size()) if t is not None else None
             table.append(dpo_tensor(ptr(self.param), ptr(self.master), ptr(self.m), ptr(self.v),
                                     ptr(self.stash), ptr(self.ef), ptr(self.grad), cnt,
-                                    DPO_WD_ON if wd_on[i] else 0))
+                                    DPO_WD_ON if self.wd_on[i] else 0))
         self.table = table
-        self.ctx = dpo_init(table, param_dtype, stash_dtype, grad_dtype, self.hp, init_mode,
-                            stream)
+        self.ctx = dpo_init(table, self.param_dtype, self.stash_dtype, self.grad_dtype, self.hp,
+                            init_mode, stream)
+
+    def use_host_io(self, grad: bool = True, param: bool = True, stream=None) -> None:
+        """Move the grad and/or bf16 param arenas to pinned host memory (their
+        contents copied) and rebuild the context over them, keeping the step
+        counter and all device state: from then on each step reads its
+        gradients from and writes its new weights to host memory directly."""
+        torch = self.torch
+        k = self.k
+        torch.cuda.synchronize(self.device)
+        dpo_destroy(self.ctx)
+        self.ctx = None
+        to_host = lambda t: torch.empty(t.shape, dtype=t.dtype, pin_memory=True).copy_(t)
+        if grad and self.grad.is_cuda:
+            self.grad = to_host(self.grad)
+        if param and self.param is not None and self.param.is_cuda:
+            self.param = to_host(self.param)
+        self._init(DPO_INIT_RESUME, stream)
+        dpo_set_step(self.ctx, k)
 
     def view(self, arena, i: int):
         off, cnt = self.layout.offsets[i], self.layout.numels[i]

@@ -121,6 +121,8 @@ class Case:
     seed: int = 0xD0D0
     grad_sigma: float = 1e-3
     init_sigma: float = 0.02
+    host_grad: bool = False     # grad arena in pinned host memory
+    host_param: bool = False    # bf16 param arena in pinned host memory
 
 
 class Run:
@@ -137,7 +139,8 @@ class Run:
             grad_dtype=case.grad_dtype, lr=case.lr, weight_decay=case.weight_decay,
             ef=case.ef, ef_lambda=case.ef_lambda, max_grad_norm=case.max_grad_norm,
             delay=case.delay, wd_on=case.wd_on, device=device,
-            x0=self._dev_x0(device), init_mode=dpo.DPO_INIT_FRESH)
+            x0=self._dev_x0(device), init_mode=dpo.DPO_INIT_FRESH,
+            host_grad=case.host_grad, host_param=case.host_param)
         # the oracle tracks every element, or only ``sample`` (global indices)
         self.sample = sample
         idx = np.arange(self.N) if sample is None else np.asarray(sample, np.int64)
@@ -165,7 +168,8 @@ class Run:
         t_of = np.searchsorted(self.offs, idx, side="right") - 1
         arena_off = np.asarray(self.gpu.layout.offsets, np.int64)
         self.arena_idx = arena_off[t_of] + (idx - self.offs[t_of])
-        self._arena_idx_dev = torch.from_numpy(self.arena_idx).to(device)
+        self._arena_idx_cpu = torch.from_numpy(self.arena_idx)
+        self._arena_idx_dev = self._arena_idx_cpu.to(device)
         self.k = 0
 
     def _dev_x0(self, device):
@@ -210,7 +214,7 @@ class Run:
         return total
 
     def gather(self, arena) -> np.ndarray:
-        t = arena.index_select(0, self._arena_idx_dev)
+        t = arena.index_select(0, self._arena_idx_dev if arena.is_cuda else self._arena_idx_cpu)
         if t.dtype == self.torch.bfloat16:
             return t.view(self.torch.int16).cpu().numpy().view(np.uint16)
         return t.cpu().numpy()

@@ -240,3 +240,43 @@ def test_launch_geometry_is_persistent(cuda_device):
         assert sb == 50_000_000 * (12 + 2 + 12 + 4 + 2) and nb == 0
     finally:
         run.close()
+
+
+@pytest.mark.parametrize("host_grad,host_param", [(True, True), (True, False), (False, True)])
+def test_host_io_parity(cuda_device, host_grad, host_param):
+    """Gradients read from and/or bf16 weights written to pinned host memory
+    by the fused kernel itself (no staging copy): same results."""
+    run = Run(Case(RAGGED, stash_dtype=B, ef=True, max_grad_norm=0.3, host_grad=host_grad,
+                   host_param=host_param), cuda_device)
+    try:
+        assert run.gpu.grad.is_cuda != host_grad and run.gpu.param.is_cuda != host_param
+        for k in range(1, 5):
+            run.step()
+            run.assert_close(TOL_ONE_STEP if k == 1 else TOL_RUN)
+        p, _ = dpo.dpo_read_weights(run.gpu.ctx, dpo.DPO_LATEST, 0)
+        assert p == run.gpu.view(run.gpu.param, 0).data_ptr()
+    finally:
+        run.close()
+
+
+def test_switch_to_host_io_continues_bitwise(cuda_device):
+    """use_host_io() mid-run rebuilds the context over host arenas (RESUME,
+    same step counter): the run continues exactly as the device-only one."""
+    case = Case(RAGGED, stash_dtype=B, ef=True)
+    a, b = Run(case, cuda_device), Run(case, cuda_device)
+    try:
+        for _ in range(3):
+            a.step()
+            b.step()
+        b.gpu.use_host_io()
+        assert not b.gpu.grad.is_cuda and not b.gpu.param.is_cuda
+        for _ in range(3):
+            a.step()
+            b.step()
+        torch.cuda.synchronize()
+        assert torch.equal(a.gpu.master, b.gpu.master)
+        assert torch.equal(a.gpu.param.cpu(), b.gpu.param)
+        assert dpo.dpo_get_step(b.gpu.ctx) == 6
+    finally:
+        a.close()
+        b.close()
