@@ -41,6 +41,7 @@ from . import build as _build
 
 F64, F32, BF16 = 0, 1, 2
 RULE_ADAMW, RULE_SGD = 0, 1
+CORR_EF, CORR_SAPIPE_SAME, CORR_SAPIPE_UPDATED = 0, 1, 2
 STORE_NAMES = {"f64": F64, "f32": F32, "bf16": BF16}
 
 _lib = None
@@ -56,6 +57,7 @@ class _HParams(ctypes.Structure):
         ("ef_lambda", ctypes.c_double),
         ("delay", ctypes.c_int),
         ("rule", ctypes.c_int),
+        ("correction", ctypes.c_int),
         ("x_store", ctypes.c_int),
         ("stash_store", ctypes.c_int),
         ("param_store", ctypes.c_int),
@@ -175,6 +177,7 @@ class HParams:
     max_grad_norm: float = 0.0
     delay: int = 1
     rule: int = RULE_ADAMW
+    correction: int = CORR_EF
 
     def as_f32(self) -> "HParams":
         """The same settings with every real rounded to fp32: the exact
@@ -182,7 +185,7 @@ class HParams:
         r = lambda v: float(np.float32(v))
         return HParams(r(self.lr), r(self.beta1), r(self.beta2), r(self.eps),
                        r(self.weight_decay), r(self.ef_lambda),
-                       r(self.max_grad_norm), self.delay, self.rule)
+                       r(self.max_grad_norm), self.delay, self.rule, self.correction)
 
 
 class StaleVersionError(AssertionError):
@@ -265,7 +268,7 @@ class DelayedOptimizer:
         self.last_clip = clip
         hp = _HParams(lr if lr is not None else self.hp.lr, self.hp.beta1,
                       self.hp.beta2, self.hp.eps, self.hp.weight_decay,
-                      self.hp.ef_lambda, self.hp.delay, self.hp.rule,
+                      self.hp.ef_lambda, self.hp.delay, self.hp.rule, self.hp.correction,
                       self.x_store, self.stash_store,
                       self.param_store if self.param_store is not None else F64)
         rc = self.lib.oracle_step(

@@ -79,17 +79,27 @@ int oracle_step(int64_t n, int64_t k, const oracle_hparams *hp,
     if (hp->delay == 1 && n > 0 && stash == NULL)
         return -1;
 
-    /* Error Feedback is active for delayed training with an EF buffer; the
-     * lambda-scaled form reduces to the standard rule at lambda = 0. */
+    /* A staleness correction is active for delayed training with an
+     * update-history buffer; the lambda-scaled EF form reduces to the
+     * standard rule at lambda = 0. */
     const int use_ef = (hp->delay == 1 && u_prev != NULL);
+    const int corr = use_ef ? hp->correction : ORACLE_CORR_EF;
+    if (corr != ORACLE_CORR_EF && corr != ORACLE_CORR_SAPIPE_SAME &&
+        corr != ORACLE_CORR_SAPIPE_UPDATED)
+        return -1;
+    if (corr == ORACLE_CORR_SAPIPE_UPDATED && hp->rule != ORACLE_RULE_ADAMW)
+        return -1;
     /* Alg. 1: the standard rule is used for t <= 1 even under EF; call k is
      * iteration t = k. */
-    const int ef_now = use_ef && k >= 2;
+    const int ef_now = use_ef && corr == ORACLE_CORR_EF && k >= 2;
     const double lam = hp->ef_lambda;
 
-    /* Bias corrections of Adam at the k-th gradient. */
+    /* Bias corrections of Adam at the k-th gradient, and at the (k+1)-th for
+     * the SAPipe updated-state prediction. */
     const double bc1 = 1.0 - pow(hp->beta1, (double)k);
     const double bc2 = 1.0 - pow(hp->beta2, (double)k);
+    const double bc1_next = 1.0 - pow(hp->beta1, (double)(k + 1));
+    const double bc2_next = 1.0 - pow(hp->beta2, (double)(k + 1));
 
 #pragma omp parallel for schedule(static)
     for (int64_t i = 0; i < n; ++i) {
@@ -98,10 +108,10 @@ int oracle_step(int64_t n, int64_t k, const oracle_hparams *hp,
         const double xt = x[i];
 
         /* Update the optimizer statistics with g_{t-1} and form u_{t-1}. */
-        double u;
+        double u, mi = 0.0, vi = 0.0;
         if (hp->rule == ORACLE_RULE_ADAMW) {
-            const double mi = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;
-            const double vi = hp->beta2 * v[i] + (1.0 - hp->beta2) * gi * gi;
+            mi = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;
+            vi = hp->beta2 * v[i] + (1.0 - hp->beta2) * gi * gi;
             const double m_hat = mi / bc1;
             const double v_hat = vi / bc2;
             u = hp->lr * (m_hat / (sqrt(v_hat) + hp->eps) + wd * xt);
@@ -118,12 +128,30 @@ int oracle_step(int64_t n, int64_t k, const oracle_hparams *hp,
         else
             xn = xt - u - lam * (u - u_prev[i]);
 
-        if (use_ef)
-            u_prev[i] = oracle_round(u, hp->x_store);
-        /* The stash keeps the pre-update weights x_t: the version the next
-         * gradient is evaluated at (one step behind the latest). */
-        if (hp->delay == 1)
-            stash[i] = oracle_round(xt, hp->stash_store);
+        /* The stash: the weights the next gradient is evaluated at. Under
+         * EF (and the standard rule) that is the pre-update x_t, one step
+         * behind the latest; under SAPipe-WP it is the prediction made at the
+         * previous step, x_t - u_prev, a weight in the master's format
+         * rounded to the stash format. */
+        if (hp->delay == 1) {
+            if (corr == ORACLE_CORR_EF)
+                stash[i] = oracle_round(xt, hp->stash_store);
+            else
+                stash[i] = oracle_round(oracle_round(xt - u_prev[i], hp->x_store),
+                                        hp->stash_store);
+        }
+        if (use_ef) {
+            double hist = u;
+            if (corr == ORACLE_CORR_SAPIPE_UPDATED) {
+                /* The optimizer step once more on g_{t-1}, from the state the
+                 * real update left, at the next time index, decaying x_{t+1}. */
+                const double m2 = hp->beta1 * mi + (1.0 - hp->beta1) * gi;
+                const double v2 = hp->beta2 * vi + (1.0 - hp->beta2) * gi * gi;
+                hist = hp->lr * ((m2 / bc1_next) / (sqrt(v2 / bc2_next) + hp->eps) +
+                                 wd * oracle_round(xn, hp->x_store));
+            }
+            u_prev[i] = oracle_round(hist, hp->x_store);
+        }
         x[i] = oracle_round(xn, hp->x_store);
         if (param != NULL)
             param[i] = oracle_round(x[i], hp->param_store);

@@ -42,6 +42,23 @@ enum { ORACLE_F64 = 0, ORACLE_F32 = 1, ORACLE_BF16 = 2 };
  * only so that tests can check the delay/EF driver of Alg. 1 apart from Adam. */
 enum { ORACLE_RULE_ADAMW = 0, ORACLE_RULE_SGD = 1 };
 
+/* Staleness correction applied when an update-history buffer is given
+ * (u_prev != NULL) under delay == 1:
+ *   EF             Eq. (1) / App. A.4: x_{t+1} = x_t - u - lambda (u - u_prev);
+ *                  the stash receives x_t.
+ *   SAPIPE_SAME    App. B.1, SAPipe-WP with the same optimizer state: the
+ *                  weights follow the standard rule x_{t+1} = x_t - u, and the
+ *                  next forward/backward reads the prediction made at the
+ *                  previous step, x~_t = x_t - u_{t-2} (the stash). u_prev
+ *                  then holds u.
+ *   SAPIPE_UPDATED App. B.1, SAPipe-WP with the updated state: as SAPIPE_SAME,
+ *                  but the prediction update is the AdamW step at the next
+ *                  time index on the same gradient, from the state after the
+ *                  real update (a temporary second blend of g into m and v,
+ *                  bias corrections at k + 1, decay on x_{t+1}); u_prev holds
+ *                  that prediction update. */
+enum { ORACLE_CORR_EF = 0, ORACLE_CORR_SAPIPE_SAME = 1, ORACLE_CORR_SAPIPE_UPDATED = 2 };
+
 typedef struct {
     double lr;            /* learning rate eta of the call */
     double beta1, beta2;  /* EMA coefficients of m and v */
@@ -50,6 +67,7 @@ typedef struct {
     double ef_lambda;     /* lambda of the EF correction; 0 = standard */
     int delay;            /* 1 = one-step-delayed (Alg. 1), 0 = synchronous */
     int rule;             /* ORACLE_RULE_* */
+    int correction;       /* ORACLE_CORR_*, used when u_prev != NULL and delay == 1 */
     int x_store;          /* storage of master x, m, v and u_prev (F64 or F32) */
     int stash_store;      /* storage of the stash (F64, F32 or BF16) */
     int param_store;      /* storage of the latest-weights copy (F64, F32, BF16) */
@@ -68,12 +86,14 @@ typedef struct {
  *              oracle_clip_coef().
  *   wd_on      per-element 0/1 mask for weight decay, or NULL (decay on all).
  *   x, m, v    master weights and Adam moments, updated in place.
- *   u_prev     EF buffer, holding u_{t-2} on entry and u_{t-1} on return.
- *              NULL selects the standard delayed rule (no Error Feedback);
- *              with a buffer and delay == 1 the lambda-scaled EF rule runs
- *              (lambda = 0 then gives the standard result).
- *   stash      receives x_t, the weights the next gradient is evaluated at;
- *              may be NULL when delay == 0 (the latest weights are read).
+ *   u_prev     update-history buffer: u_{t-2} on entry and u_{t-1} on return
+ *              (SAPIPE_UPDATED: the prediction updates). NULL selects the
+ *              standard delayed rule; with a buffer and delay == 1 the
+ *              correction hp->correction runs (EF with lambda = 0 gives the
+ *              standard result).
+ *   stash      receives the weights the next gradient is evaluated at: x_t,
+ *              or the SAPipe prediction point; may be NULL when delay == 0
+ *              (the latest weights are read).
  *   param      receives the new latest weights x_{t+1}, or NULL.
  *
  * Returns 0, or -1 on an invalid argument.

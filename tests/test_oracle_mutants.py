@@ -26,21 +26,28 @@ MUTANTS = [
     ("eps_inside_sqrt", "(sqrt(v_hat) + hp->eps)", "sqrt(v_hat + hp->eps)"),
     ("ef_sign_flipped", "xn = xt - u - lam * (u - u_prev[i]);",
      "xn = xt - u + lam * (u - u_prev[i]);"),
-    ("ef_at_first_update", "use_ef && k >= 2", "use_ef && k >= 1"),
+    ("ef_at_first_update", "corr == ORACLE_CORR_EF && k >= 2", "corr == ORACLE_CORR_EF && k >= 1"),
     ("bias_correction_index", "pow(hp->beta1, (double)k)", "pow(hp->beta1, (double)(k + 1))"),
     ("no_bias_correction_m", "const double m_hat = mi / bc1;", "const double m_hat = mi;"),
     ("stash_holds_new_weights", "stash[i] = oracle_round(xt, hp->stash_store);",
      "stash[i] = oracle_round(xn, hp->stash_store);"),
-    ("v_from_momentum", "(1.0 - hp->beta2) * gi * gi", "(1.0 - hp->beta2) * gi * mi"),
+    ("v_from_momentum", "vi = hp->beta2 * v[i] + (1.0 - hp->beta2) * gi * gi",
+     "vi = hp->beta2 * v[i] + (1.0 - hp->beta2) * gi * mi"),
     ("ema_roles_swapped", "hp->beta1 * m[i] + (1.0 - hp->beta1) * gi",
      "(1.0 - hp->beta1) * m[i] + hp->beta1 * gi"),
-    ("ef_stores_displacement", "u_prev[i] = oracle_round(u, hp->x_store);",
-     "u_prev[i] = oracle_round(xt - xn, hp->x_store);"),
+    ("ef_stores_displacement", "double hist = u;", "double hist = xt - xn;"),
     ("clip_not_applied", "const double gi = clip_scale * g[i];", "const double gi = g[i];"),
     ("clip_no_epsilon", "(sqrt(sqnorm) + 1e-6)", "sqrt(sqnorm)"),
     ("bf16_ties_away", "q = nearbyint(q);", "q = round(q);"),
     ("bf16_subnormal_quantum", "if (e < -125)\n        e = -125;", "if (e < -126)\n        e = -126;"),
     ("decay_ignores_mask", "(wd_on == NULL || wd_on[i])", "(1)"),
+    ("sapipe_predicts_with_current_update", "oracle_round(xt - u_prev[i], hp->x_store)",
+     "oracle_round(xt - u, hp->x_store)"),
+    ("sapipe_updated_bias_index", "bc1_next = 1.0 - pow(hp->beta1, (double)(k + 1))",
+     "bc1_next = 1.0 - pow(hp->beta1, (double)k)"),
+    ("sapipe_updated_decays_old_weights", "wd * oracle_round(xn, hp->x_store)", "wd * xt"),
+    ("sapipe_updated_no_second_blend", "hp->beta1 * mi + (1.0 - hp->beta1) * gi;",
+     "mi;"),
 ]
 
 

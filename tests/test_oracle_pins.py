@@ -454,3 +454,108 @@ def test_quadratic_gradient_is_loss_derivative(lib):
         lm = oracle.quadratic(a, ws, w - e, None, F64, lib=lib)[1]
         assert g[i] == pytest.approx((lp - lm) / (2 * h), rel=1e-6, abs=1e-9)
     assert loss == pytest.approx(0.5 * np.sum(a * (w - ws) ** 2), rel=1e-14)
+
+
+# ------------------------------------------------------- SAPipe-WP (App. B.1)
+
+def _fixed_grad_run(lib, correction, steps=8, wd=0.1, ef=True, lam=1.0, beta=(0.9, 0.95),
+                    eps=1e-8, n=64, seed=21):
+    rng = np.random.default_rng(seed)
+    x0 = rng.normal(0, 0.5, n)
+    grads = [rng.normal(0, 1.0, n) for _ in range(steps)]
+    hp = HParams(lr=0.01, beta1=beta[0], beta2=beta[1], eps=eps, weight_decay=wd,
+                 ef_lambda=lam, correction=correction)
+    o = oracle.DelayedOptimizer([x0], hp, ef=ef, x_store=F64, stash_store=F64, lib=lib)
+    hist = []
+    for g in grads:
+        o.step(g, tag=o.read_weights()[1])
+        hist.append(dict(x=o.x.copy(), stash=o.stash.copy(), u=o.u_prev.copy() if ef else None,
+                         m=o.m.copy(), v=o.v.copy()))
+    return hist, grads, x0, hp
+
+
+def test_sapipe_same_weights_follow_the_standard_rule(lib):
+    """SAPipe-WP changes only where the next gradient is evaluated: the
+    weights take the standard delayed update, bitwise."""
+    h_sp, _, _, _ = _fixed_grad_run(lib, oracle.CORR_SAPIPE_SAME)
+    h_std, _, _, _ = _fixed_grad_run(lib, oracle.CORR_EF, ef=False)
+    for a, b in zip(h_sp, h_std):
+        assert np.array_equal(a["x"], b["x"])
+
+
+def test_sapipe_same_prediction_points_move_like_ef(lib):
+    """App. B.1: the displacement between consecutive SAPipe prediction points
+    is -2 u(g_{t-1}) + u(g_{t-2}), Eq. (1)'s. Checked against the identity and
+    against an EF run's weight displacement on the same gradient sequence
+    (wd = 0, so both runs form the same updates)."""
+    h_sp, _, _, _ = _fixed_grad_run(lib, oracle.CORR_SAPIPE_SAME, wd=0.0)
+    h_ef, _, _, _ = _fixed_grad_run(lib, oracle.CORR_EF, wd=0.0)
+    for j in range(1, len(h_sp)):
+        u_prev = h_sp[j - 1]["u"]
+        u_prev2 = h_sp[j - 2]["u"] if j >= 2 else 0.0
+        d_stash = h_sp[j]["stash"] - h_sp[j - 1]["stash"]
+        np.testing.assert_allclose(d_stash, -2 * u_prev + u_prev2, rtol=1e-11, atol=1e-15)
+        if j >= 2:   # the EF weights take the same displacement one call earlier
+            d_ef = h_ef[j - 1]["x"] - h_ef[j - 2]["x"]
+            np.testing.assert_allclose(d_stash, d_ef, rtol=1e-11, atol=1e-15)
+
+
+def test_sapipe_updated_prediction_is_adamw_stepped_again(lib):
+    """The updated-state prediction update is what torch.optim.AdamW applies
+    when stepped once more on the same gradient from the state its real step
+    left (then discarded)."""
+    hist, grads, x0, hp = _fixed_grad_run(lib, oracle.CORR_SAPIPE_UPDATED)
+    p = torch.nn.Parameter(torch.tensor(x0))
+    opt = torch.optim.AdamW([p], lr=hp.lr, betas=(hp.beta1, hp.beta2), eps=hp.eps,
+                            weight_decay=hp.weight_decay, foreach=False, fused=False)
+    for k, g in enumerate(grads):
+        p.grad = torch.tensor(g)
+        opt.step()
+        np.testing.assert_allclose(p.detach().numpy(), hist[k]["x"], rtol=1e-12)
+        # prediction: one more step on the same gradient from a copy of the state
+        q = torch.nn.Parameter(p.detach().clone())
+        opt2 = torch.optim.AdamW([q], lr=hp.lr, betas=(hp.beta1, hp.beta2), eps=hp.eps,
+                                 weight_decay=hp.weight_decay, foreach=False, fused=False)
+        st = opt.state[p]
+        opt2.state[q] = {"step": st["step"].clone(), "exp_avg": st["exp_avg"].clone(),
+                         "exp_avg_sq": st["exp_avg_sq"].clone()}
+        q.grad = torch.tensor(g)
+        opt2.step()
+        u_pred = p.detach().numpy() - q.detach().numpy()
+        np.testing.assert_allclose(hist[k]["u"], u_pred, rtol=1e-10, atol=1e-16)
+        # the next forward reads the previous prediction point
+        if k >= 1:
+            np.testing.assert_allclose(hist[k]["stash"], hist[k - 1]["x"] - hist[k - 1]["u"],
+                                       rtol=1e-13)
+
+
+def test_sapipe_updated_equals_same_when_adam_is_memoryless(lib):
+    """beta1 = beta2 = 0, eps = 0, wd = 0: every Adam update is lr sign(g),
+    so recomputing it from the updated state changes nothing."""
+    kw = dict(wd=0.0, beta=(0.0, 0.0), eps=0.0)
+    h_u, _, _, _ = _fixed_grad_run(lib, oracle.CORR_SAPIPE_UPDATED, **kw)
+    h_s, _, _, _ = _fixed_grad_run(lib, oracle.CORR_SAPIPE_SAME, **kw)
+    for a, b in zip(h_u, h_s):
+        for key in ("x", "stash", "u"):
+            assert np.array_equal(a[key], b[key])
+
+
+def test_sapipe_updated_hand_steps(lib):
+    """x0 = 1, beta = (0.9, 0.95), eps = 0, wd = 0, lr = 0.1, gradients 2, 1.
+    Call 1: m = 0.2, v = 0.2, u = 0.1; prediction from m' = 0.38, v' = 0.39
+    at k = 2 (1 - b1^2 = 0.19, 1 - b2^2 = 0.0975): m_hat = 2, v_hat = 4, so 0.1.
+    Call 2: stash = x_2 - 0.1 = 0.8; u = 0.1 (0.28/0.19) / sqrt(0.24/0.0975);
+    prediction from m' = 0.352, v' = 0.278 at k = 3 (0.271, 0.142625)."""
+    hp = HParams(lr=0.1, beta1=0.9, beta2=0.95, eps=0.0, weight_decay=0.0,
+                 correction=oracle.CORR_SAPIPE_UPDATED)
+    o = oracle.DelayedOptimizer([np.array([1.0])], hp, ef=True, x_store=F64, stash_store=F64,
+                                lib=lib)
+    o.step(np.array([2.0]), tag=o.read_weights()[1])
+    assert o.stash[0] == 1.0 and o.x[0] == pytest.approx(0.9, rel=1e-15)
+    assert o.u_prev[0] == pytest.approx(0.1, rel=1e-15)
+    o.step(np.array([1.0]), tag=o.read_weights()[1])
+    assert o.stash[0] == pytest.approx(0.8, rel=1e-15)
+    u2 = 0.1 * (0.28 / 0.19) / math.sqrt(0.24 / 0.0975)
+    assert o.x[0] == pytest.approx(0.9 - u2, rel=1e-14)
+    assert o.u_prev[0] == pytest.approx(0.1 * (0.352 / 0.271) / math.sqrt(0.278 / 0.142625),
+                                        rel=1e-14)
