@@ -45,7 +45,8 @@ def parse_args(argv=None):
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=["dpo", "reference"], default="dpo")
     p.add_argument("--workload", default="llama-7B")
-    p.add_argument("--mode", choices=["ef", "std"], default="ef")
+    p.add_argument("--mode", choices=["ef", "std", "sapipe-same", "sapipe-updated"],
+                   default="ef")
     p.add_argument("--e2e-steps", type=int, default=4)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -154,9 +155,20 @@ class ClockSampler:
                 "power_w_max": max(pw) if pw else None}
 
 
+# ----------------------------------------------------------------- modes --
+
+# mode -> (update-history buffer, correction, description)
+MODES = {
+    "ef": (True, 0, "EF (lambda=1)"),
+    "std": (False, 0, "standard delayed rule"),
+    "sapipe-same": (True, 1, "SAPipe-WP prediction, same optimizer state"),
+    "sapipe-updated": (True, 2, "SAPipe-WP prediction, updated optimizer state"),
+}
+
+
 # ------------------------------------------------------------ CPU oracle --
 
-def oracle_sample_run(w, ef: bool, seconds: float, max_steps: int = 1000, n: int = 1 << 22):
+def oracle_sample_run(w, mode: str, seconds: float, max_steps: int = 1000, n: int = 1 << 22):
     """Time the oracle as it stands on the first n parameters of the set
     (input draws excluded from the timing). Returns (params/s, cores, steps,
     n)."""
@@ -168,9 +180,11 @@ def oracle_sample_run(w, ef: bool, seconds: float, max_steps: int = 1000, n: int
 
     n = min(n, w.n_params)
     STORE = {0: oracle.F32, 1: oracle.BF16}
+    ef, corr, _ = MODES[mode]
     x0 = synth.host_normal(w.seed, synth.STREAM_INIT, 0, 0, n, W.INIT_SIGMA).astype(np.float64)
-    hp = oracle.HParams(lr=w.lr, weight_decay=w.weight_decay, ef_lambda=1.0 if ef else 0.0,
-                        max_grad_norm=w.max_grad_norm).as_f32()
+    hp = oracle.HParams(lr=w.lr, weight_decay=w.weight_decay,
+                        ef_lambda=1.0 if ef and corr == 0 else 0.0,
+                        max_grad_norm=w.max_grad_norm, correction=corr).as_f32()
     o = oracle.DelayedOptimizer([x0], hp, ef=ef, x_store=oracle.F32,
                                 stash_store=STORE[w.stash_dtype],
                                 param_store=oracle.BF16 if w.param_dtype == 1 else None)
@@ -198,7 +212,7 @@ def run_gpu(args, w, world, rank, local):
 
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
-    ef = args.mode == "ef"
+    ef, corr, _ = MODES[args.mode]
     stream = torch.cuda.Stream(dev)
     offs = np.concatenate([[0], np.cumsum(w.numels)]).astype(np.int64)
     with torch.cuda.stream(stream):
@@ -210,7 +224,7 @@ def run_gpu(args, w, world, rank, local):
                                grad_dtype=w.grad_dtype, lr=w.lr, beta1=w.beta1, beta2=w.beta2,
                                eps=w.eps, weight_decay=w.weight_decay, ef=ef, ef_lambda=1.0,
                                max_grad_norm=w.max_grad_norm, delay=1, device=dev, x0=x0,
-                               stream=stream)
+                               stream=stream, correction=corr)
         del x0
         for i, (o, n) in enumerate(zip(lay.offsets, lay.numels)):
             synth.dev_normal(w.seed, synth.STREAM_GRAD, 1, int(offs[i]), opt.grads(i),
@@ -339,19 +353,19 @@ def main(argv=None):
     from paper_2606_30634_gb300.synth import workloads as W
     w = W.ALL[args.workload]
     world, rank, local = dist_env()
-    ef = args.mode == "ef"
+    ef, _, what = MODES[args.mode]
     cfg = {"workload": f"{w.name}: {w.n_params} params in {len(w.tensors)} tensors, "
-                       f"{'EF (lambda=1)' if ef else 'standard delayed rule'}, one-step delay",
+                       f"{what}, one-step delay",
            "mode": args.mode, "param_dtype": "bf16" if w.param_dtype else "f32",
            "stash_dtype": "bf16" if w.stash_dtype else "f32",
            "grad_dtype": "bf16" if w.grad_dtype else "f32",
-           "state": "fp32 master/m/v" + (" + fp32 EF buffer" if ef else ""),
+           "state": "fp32 master/m/v" + (" + fp32 update-history buffer" if ef else ""),
            "clip": w.max_grad_norm, "l2": "inputs larger than L2 (no flush needed)"}
 
     if args.impl == "reference":
         if rank != 0:
             return 0
-        v, cores, steps, n = oracle_sample_run(w, ef, args.cpu_seconds,
+        v, cores, steps, n = oracle_sample_run(w, args.mode, args.cpu_seconds,
                                                max_steps=max(1, args.steps + args.warmup))
         sample = f"first {n} params of the set, {steps} oracle steps (plain C, fp64)"
         line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT,
@@ -385,7 +399,7 @@ def main(argv=None):
             "frac_of_nominal": r["achieved"] / 8000.0}
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        v, cores, steps, n = oracle_sample_run(w, ef, args.cpu_seconds)
+        v, cores, steps, n = oracle_sample_run(w, args.mode, args.cpu_seconds)
         cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
                "sample": f"first {n} params of the set, {steps} oracle steps (plain C, fp64)"}
     if world > 1:

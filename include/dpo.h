@@ -81,6 +81,26 @@ typedef enum { DPO_F32 = 0, DPO_BF16 = 1 } dpo_dtype;
 /* dpo_get_flags() bits */
 #define DPO_FLAG_NONFINITE 1u  /* a clipped step saw a non-finite gradient norm */
 
+/* dpo_hparams.correction: the staleness correction run when the table has
+ * update-history (EF) buffers and delay == 1.
+ *   DPO_CORR_EF              Eq. (1) / App. A.4: x_{t+1} = x_t - u - lambda (u - u_prev);
+ *                            the stash receives x_t.
+ *   DPO_CORR_SAPIPE_SAME     App. B.1, SAPipe-WP weight prediction with the same
+ *                            optimizer state: the weights take the standard rule
+ *                            x_{t+1} = x_t - u, and the stash (what the next
+ *                            forward/backward reads) receives the prediction made
+ *                            at the previous step, x_t - u_prev; the buffer then
+ *                            holds u.
+ *   DPO_CORR_SAPIPE_UPDATED  App. B.1 with the updated state: as above, but the
+ *                            buffer holds the prediction update: the AdamW step
+ *                            at the next time index on the same gradient, from
+ *                            the state the real update left (moments blended
+ *                            with g once more, bias corrections at k + 1, decay
+ *                            on x_{t+1}), not kept in m and v. */
+#define DPO_CORR_EF 0
+#define DPO_CORR_SAPIPE_SAME 1
+#define DPO_CORR_SAPIPE_UPDATED 2
+
 typedef struct {
     float beta1;          /* first-moment EMA coefficient, [0, 1) */
     float beta2;          /* second-moment EMA coefficient, [0, 1) */
@@ -89,6 +109,7 @@ typedef struct {
     float ef_lambda;      /* lambda of the EF correction (tables with EF buffers) */
     float max_grad_norm;  /* > 0: global-norm clipping threshold; <= 0: off */
     int delay;            /* 1: one-step-delayed with stash; 0: synchronous */
+    int correction;       /* DPO_CORR_* (tables with EF buffers, delay == 1) */
 } dpo_hparams;
 
 typedef struct {
@@ -102,9 +123,10 @@ typedef struct {
     /* Stale weights in the stash dtype: x_t after each step. Required when
      * delay == 1; ignored (may be NULL) when delay == 0. */
     void *stash;
-    /* EF buffer (fp32): u_{t-2} on entry, u_{t-1} on return. NULL on every
-     * tensor: standard delayed rule. Non-NULL on every tensor: EF with
-     * hparams.ef_lambda (lambda = 0 gives the standard result). */
+    /* Update-history (EF) buffer (fp32): u_{t-2} on entry, u_{t-1} on return
+     * (the prediction update under DPO_CORR_SAPIPE_UPDATED). NULL on every
+     * tensor: standard delayed rule. Non-NULL on every tensor: the correction
+     * hparams.correction (EF with lambda = 0 gives the standard result). */
     float *ef;
     /* The gradient the step consumes, in the grad dtype, evaluated at the
      * stash (delay == 1) or at the latest weights (delay == 0). Read only. */

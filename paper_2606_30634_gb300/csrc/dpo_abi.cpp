@@ -76,6 +76,20 @@ StashKind stash_kind(const dpo_ctx *c)
     return c->stash_dt == DPO_BF16 ? dpo::kStashBF16 : dpo::kStashF32;
 }
 
+dpo::Correction correction_kind(bool ef, const dpo_hparams &hp)
+{
+    if (!ef || hp.delay != 1)
+        return dpo::kCorrNone;
+    switch (hp.correction) {
+    case DPO_CORR_SAPIPE_SAME:
+        return dpo::kCorrSapipeSame;
+    case DPO_CORR_SAPIPE_UPDATED:
+        return dpo::kCorrSapipeUpdated;
+    default:
+        return dpo::kCorrEF;
+    }
+}
+
 struct Span {
     uintptr_t lo, hi;
     int tensor;
@@ -120,6 +134,9 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
         return fail(nullptr, DPO_EINVAL, "beta1 and beta2 must lie in [0, 1)");
     if (hp->eps < 0.0f || hp->weight_decay < 0.0f)
         return fail(nullptr, DPO_EINVAL, "eps and weight_decay must be >= 0");
+    if (hp->correction != DPO_CORR_EF && hp->correction != DPO_CORR_SAPIPE_SAME &&
+        hp->correction != DPO_CORR_SAPIPE_UPDATED)
+        return fail(nullptr, DPO_EINVAL, "correction must be one of DPO_CORR_*");
 
     // Table: NULL pointers, EF consistency, alignment, overlaps.
     const bool ef = table[0].ef != nullptr;
@@ -241,7 +258,7 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
     int sms = 0, per_sm_step = 0, per_sm_norm = 0;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
     e = dpo::step_ctas_per_sm(param_dtype == DPO_BF16, stash_kind(c), grad_dtype == DPO_BF16,
-                              ef && hp->delay == 1, &per_sm_step);
+                              correction_kind(ef, *hp), &per_sm_step);
     if (e == cudaSuccess)
         e = dpo::norm_ctas_per_sm(grad_dtype == DPO_BF16, &per_sm_norm);
     if (e != cudaSuccess) {
@@ -360,7 +377,7 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
         const double b1 = c->hp.beta1, b2 = c->hp.beta2, lrd = lr;
         const double bc1 = 1.0 - std::pow(b1, (double)k);
         const double bc2 = 1.0 - std::pow(b2, (double)k);
-        const bool ef = c->ef && c->hp.delay == 1;
+        const dpo::Correction corr = correction_kind(c->ef, c->hp);
         dpo::StepArgs a{};
         a.table = c->d_table;
         a.pkt_begin = c->d_pkt_begin;
@@ -375,10 +392,12 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
         a.eps = c->hp.eps;
         a.lr_wd = (float)(lrd * (double)c->hp.weight_decay);
         // Alg. 1: the standard rule for t <= 1, i.e. at the first update.
-        a.lam = (ef && k >= 2) ? c->hp.ef_lambda : 0.0f;
+        a.lam = (corr == dpo::kCorrEF && k >= 2) ? c->hp.ef_lambda : 0.0f;
+        a.step_size_next = (float)(lrd / (1.0 - std::pow(b1, (double)(k + 1))));
+        a.inv_sqrt_bc2_next = (float)(1.0 / std::sqrt(1.0 - std::pow(b2, (double)(k + 1))));
         a.clip = c->clip ? &c->d_scalars->clip : nullptr;
         const cudaError_t e = dpo::launch_step(c->param_dt == DPO_BF16, stash_kind(c),
-                                               c->grad_dt == DPO_BF16, ef, c->step_grid, a, s);
+                                               c->grad_dt == DPO_BF16, corr, c->step_grid, a, s);
         if (e != cudaSuccess)
             return cuda_fail(c, e, "fused step launch");
     }

@@ -47,6 +47,9 @@ struct DevTensor {
 
 // Kernel template selectors.
 enum StashKind { kStashNone = 0, kStashF32 = 1, kStashBF16 = 2 };
+// Staleness correction of a delayed step (the DPO_CORR_* of include/dpo.h, or
+// none when the table has no update-history buffers).
+enum Correction { kCorrNone = 0, kCorrEF = 1, kCorrSapipeSame = 2, kCorrSapipeUpdated = 3 };
 
 // Scalars of one fused step, precomputed on the host in double and rounded
 // once to fp32.
@@ -62,6 +65,8 @@ struct StepArgs {
     float eps;
     float lr_wd;                // lr * weight_decay
     float lam;                  // lambda of this call (0 at k = 1, Alg. 1)
+    float step_size_next;       // lr / (1 - beta1^(k+1))       (SAPipe updated state)
+    float inv_sqrt_bc2_next;    // 1 / sqrt(1 - beta2^(k+1))    (SAPipe updated state)
     const float *clip;          // device clip coefficient, or nullptr
 };
 
@@ -93,14 +98,14 @@ struct StashArgs {
 };
 
 // Launchers (dpo_kernels.cu). Each returns the launch's cudaError_t.
-cudaError_t launch_step(bool param_bf16, StashKind stash, bool grad_bf16, bool ef,
+cudaError_t launch_step(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr,
                         int grid, const StepArgs &a, cudaStream_t s);
 cudaError_t launch_norm(bool grad_bf16, int grid, const NormArgs &a, cudaStream_t s);
 cudaError_t launch_stash(bool param_bf16, StashKind stash, int grid, const StashArgs &a,
                          cudaStream_t s);
 
 // Resident CTAs per SM of each kernel at its block size (occupancy query).
-cudaError_t step_ctas_per_sm(bool param_bf16, StashKind stash, bool grad_bf16, bool ef,
+cudaError_t step_ctas_per_sm(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr,
                              int *n);
 cudaError_t norm_ctas_per_sm(bool grad_bf16, int *n);
 

@@ -1,10 +1,11 @@
 // dpo_kernels.cu -- sm_103a kernels of the one-step-delayed AdamW step.
 //
-//   fused_step_kernel   the whole per-element step of Alg. 1 with AdamW and
-//                       the lambda-scaled Error Feedback (Eq. (1), App. A.4)
-//                       in one pass over HBM: read master, m, v, grad (and
-//                       the EF buffer); write master, m, v, stash, the bf16
-//                       latest copy (and the EF buffer).
+//   fused_step_kernel   the whole per-element step of Alg. 1 with AdamW and a
+//                       staleness correction (lambda-scaled Error Feedback,
+//                       Eq. (1) / App. A.4, or SAPipe-WP weight prediction,
+//                       App. B.1) in one pass over HBM: read master, m, v,
+//                       grad (and the update-history buffer); write master,
+//                       m, v, stash, the bf16 latest copy (and the buffer).
 //   grad_sqnorm_kernel  global ||g||^2 over the whole table for clipping
 //                       (App. E.1), deterministic: fixed per-thread order,
 //                       fixed block tree, fixed-order sum of the per-CTA
@@ -128,6 +129,7 @@ struct Cursor {
 
 struct Scalars {
     float beta1, omb1, beta2, omb2, step_size, inv_sqrt_bc2, eps, lam;
+    float step_size_next, inv_sqrt_bc2_next;
 };
 
 // Moments with the (clipped) stale gradient, then the AdamW update
@@ -147,6 +149,20 @@ __device__ __forceinline__ float adamw_update(const Scalars &s, float g, float x
     return fmaf(s.step_size, m / denom, wd_lr * x);
 }
 
+// SAPipe-WP with the updated state (App. B.1): the AdamW update at the next
+// time index on the same gradient g, from the moments m, v the real update
+// left (blended with g once more into temporaries), decaying x_{t+1}.
+__device__ __forceinline__ float adamw_prediction(const Scalars &s, float g, float x_next,
+                                                  float wd_lr, float m, float v)
+{
+    const float p = s.omb1 * g;
+    const float p_err = fmaf(s.omb1, g, -p);
+    const float m2 = fmaf(s.beta1, m, p) + p_err;
+    const float v2 = fmaf(s.beta2, v, (s.omb2 * g) * g);
+    const float denom = fmaf(sqrtf(v2), s.inv_sqrt_bc2_next, s.eps);
+    return fmaf(s.step_size_next, m2 / denom, wd_lr * x_next);
+}
+
 // Displacement of the lambda-scaled EF rule, x_{t+1} = x_t - (u + lambda (u - u_prev)):
 // the small terms are summed first so the weight is rounded once, at its own
 // magnitude (subtracting u and then the correction would round x twice).
@@ -155,20 +171,28 @@ __device__ __forceinline__ float ef_displacement(float lam, float u, float u_pre
     return fmaf(lam, u - u_prev, u);
 }
 
-template <int PB, int SK, int GB, int EF>
+// CORR is a Correction: kCorrNone (standard rule, no history buffer),
+// kCorrEF (lambda-scaled EF; the buffer is read only when lambda != 0),
+// kCorrSapipeSame / kCorrSapipeUpdated (the stash receives the prediction
+// point x_t - u_prev; the weights take the standard rule).
+template <int PB, int SK, int GB, int CORR>
 __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs a)
 {
     using GT = typename Elem<GB != 0>::T;
     using ST = typename StashT<SK>::T;
+    constexpr bool kHist = CORR != kCorrNone;
+    constexpr bool kSapipe = CORR == kCorrSapipeSame || CORR == kCorrSapipeUpdated;
 
     const int64_t stride = (int64_t)gridDim.x * kStepThreads;
     int64_t p = (int64_t)blockIdx.x * kStepThreads + threadIdx.x;
     if (p >= a.total_pkts)
         return;
 
-    const Scalars s{a.beta1, a.omb1, a.beta2, a.omb2, a.step_size, a.inv_sqrt_bc2, a.eps, a.lam};
+    const Scalars s{a.beta1, a.omb1, a.beta2, a.omb2, a.step_size, a.inv_sqrt_bc2, a.eps, a.lam,
+                    a.step_size_next, a.inv_sqrt_bc2_next};
     const float clip = a.clip != nullptr ? __ldg(a.clip) : 1.0f;
-    const bool use_prev = EF && a.lam != 0.0f;
+    const bool use_prev = kSapipe || (CORR == kCorrEF && a.lam != 0.0f);
+    const bool ef_now = CORR == kCorrEF && a.lam != 0.0f;
 
     Cursor c;
     c.seek(a.pkt_begin, a.n_tensors, p);
@@ -194,18 +218,30 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
             ld8(grad + e, g);
             if (use_prev)
                 ld8(ef + e, up);
-            if (SK != kStashNone)
-                st8(stash + e, x);   // stash := x_t, before the update
+            if (SK != kStashNone) {
+                if (kSapipe) {   // stash := the prediction point x_t - u_prev
+                    float xp[8];
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        xp[j] = x[j] - up[j];
+                    st8(stash + e, xp);
+                } else {
+                    st8(stash + e, x);   // stash := x_t, before the update
+                }
+            }
             float u[8];
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
-                u[j] = adamw_update(s, g[j] * clip, x[j], wd_lr, m[j], v[j]);
-                x[j] -= use_prev ? ef_displacement(s.lam, u[j], up[j]) : u[j];
+                const float gc = g[j] * clip;
+                u[j] = adamw_update(s, gc, x[j], wd_lr, m[j], v[j]);
+                x[j] -= ef_now ? ef_displacement(s.lam, u[j], up[j]) : u[j];
+                if (CORR == kCorrSapipeUpdated)
+                    u[j] = adamw_prediction(s, gc, x[j], wd_lr, m[j], v[j]);
             }
             st8(master + e, x);
             st8(mm + e, m);
             st8(vv + e, v);
-            if (EF)
+            if (kHist)
                 st8(ef + e, u);
             if (PB)
                 st8(param + e, x);
@@ -213,15 +249,18 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
             // the tensor's last, partial packet
             for (int64_t i = e; i < d.numel; ++i) {
                 float x = master[i], m = mm[i], v = vv[i];
-                const float g = ld1(grad + i);
+                const float g = ld1(grad + i) * clip;
+                const float up = use_prev ? ef[i] : 0.0f;
                 if (SK != kStashNone)
-                    st1(stash + i, x);
-                const float u = adamw_update(s, g * clip, x, wd_lr, m, v);
-                x -= use_prev ? ef_displacement(s.lam, u, ef[i]) : u;
+                    st1(stash + i, kSapipe ? x - up : x);
+                float u = adamw_update(s, g, x, wd_lr, m, v);
+                x -= ef_now ? ef_displacement(s.lam, u, up) : u;
+                if (CORR == kCorrSapipeUpdated)
+                    u = adamw_prediction(s, g, x, wd_lr, m, v);
                 master[i] = x;
                 mm[i] = m;
                 vv[i] = v;
-                if (EF)
+                if (kHist)
                     ef[i] = u;
                 if (PB)
                     st1(param + i, x);
@@ -404,24 +443,40 @@ __global__ void __launch_bounds__(kStepThreads) stash_kernel(const StashArgs a)
 
 using StepFn = void (*)(StepArgs);
 
+template <int PB, int SK, int GB>
+StepFn pick_step_corr(Correction corr)
+{
+    switch (corr) {
+    case kCorrNone:
+        return fused_step_kernel<PB, SK, GB, kCorrNone>;
+    case kCorrEF:
+        return fused_step_kernel<PB, SK, GB, kCorrEF>;
+    case kCorrSapipeSame:
+        return fused_step_kernel<PB, SK, GB, kCorrSapipeSame>;
+    case kCorrSapipeUpdated:
+        return fused_step_kernel<PB, SK, GB, kCorrSapipeUpdated>;
+    }
+    return nullptr;
+}
+
 template <int PB, int GB>
-StepFn pick_step_sk(StashKind sk, bool ef)
+StepFn pick_step_sk(StashKind sk, Correction corr)
 {
     switch (sk) {
     case kStashF32:
-        return ef ? fused_step_kernel<PB, kStashF32, GB, 1> : fused_step_kernel<PB, kStashF32, GB, 0>;
+        return pick_step_corr<PB, kStashF32, GB>(corr);
     case kStashBF16:
-        return ef ? fused_step_kernel<PB, kStashBF16, GB, 1> : fused_step_kernel<PB, kStashBF16, GB, 0>;
-    default:
-        return ef ? nullptr : fused_step_kernel<PB, kStashNone, GB, 0>;
+        return pick_step_corr<PB, kStashBF16, GB>(corr);
+    default:   // synchronous: no stash, no correction
+        return corr == kCorrNone ? fused_step_kernel<PB, kStashNone, GB, kCorrNone> : nullptr;
     }
 }
 
-StepFn pick_step(bool pb, StashKind sk, bool gb, bool ef)
+StepFn pick_step(bool pb, StashKind sk, bool gb, Correction corr)
 {
     if (pb)
-        return gb ? pick_step_sk<1, 1>(sk, ef) : pick_step_sk<1, 0>(sk, ef);
-    return gb ? pick_step_sk<0, 1>(sk, ef) : pick_step_sk<0, 0>(sk, ef);
+        return gb ? pick_step_sk<1, 1>(sk, corr) : pick_step_sk<1, 0>(sk, corr);
+    return gb ? pick_step_sk<0, 1>(sk, corr) : pick_step_sk<0, 0>(sk, corr);
 }
 
 using StashFn = void (*)(StashArgs);
@@ -441,10 +496,10 @@ StashFn pick_stash_sk(StashKind sk)
 
 }  // namespace
 
-cudaError_t launch_step(bool pb, StashKind sk, bool gb, bool ef, int grid, const StepArgs &a,
-                        cudaStream_t s)
+cudaError_t launch_step(bool pb, StashKind sk, bool gb, Correction corr, int grid,
+                        const StepArgs &a, cudaStream_t s)
 {
-    StepFn f = pick_step(pb, sk, gb, ef);
+    StepFn f = pick_step(pb, sk, gb, corr);
     if (f == nullptr)
         return cudaErrorInvalidValue;
     f<<<grid, kStepThreads, 0, s>>>(a);
@@ -467,9 +522,9 @@ cudaError_t launch_stash(bool pb, StashKind sk, int grid, const StashArgs &a, cu
     return cudaGetLastError();
 }
 
-cudaError_t step_ctas_per_sm(bool pb, StashKind sk, bool gb, bool ef, int *n)
+cudaError_t step_ctas_per_sm(bool pb, StashKind sk, bool gb, Correction corr, int *n)
 {
-    StepFn f = pick_step(pb, sk, gb, ef);
+    StepFn f = pick_step(pb, sk, gb, corr);
     if (f == nullptr)
         return cudaErrorInvalidValue;
     return cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, f, kStepThreads, 0);

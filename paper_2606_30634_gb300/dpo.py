@@ -25,6 +25,7 @@ DPO_WD_ON = 1
 DPO_STALE, DPO_LATEST = 0, 1
 DPO_INIT_FRESH, DPO_INIT_RESUME = 0, 1
 DPO_FLAG_NONFINITE = 1
+DPO_CORR_EF, DPO_CORR_SAPIPE_SAME, DPO_CORR_SAPIPE_UPDATED = 0, 1, 2
 
 EXPORTS = ("dpo_init", "dpo_stash", "dpo_step", "dpo_read_weights", "dpo_get_step",
            "dpo_set_step", "dpo_get_flags", "dpo_algorithmic_bytes", "dpo_launch_config",
@@ -44,7 +45,8 @@ class DpoError(RuntimeError):
 class dpo_hparams(ctypes.Structure):
     _fields_ = [("beta1", ctypes.c_float), ("beta2", ctypes.c_float), ("eps", ctypes.c_float),
                 ("weight_decay", ctypes.c_float), ("ef_lambda", ctypes.c_float),
-                ("max_grad_norm", ctypes.c_float), ("delay", ctypes.c_int)]
+                ("max_grad_norm", ctypes.c_float), ("delay", ctypes.c_int),
+                ("correction", ctypes.c_int)]
 
 
 class dpo_tensor(ctypes.Structure):
@@ -216,7 +218,8 @@ class DelayedAdamW:
     dtype), param (bf16, only with param_dtype BF16), stash (stash dtype,
     delay 1), ef (fp32, when ``ef`` is set). ``x0`` fills the master before
     dpo_init(FRESH); pass ``init_mode=DPO_INIT_RESUME`` to start from arenas
-    restored by ``load_state``. With ``host_grad`` / ``host_param`` the grad /
+    restored by ``load_state``. ``ef`` allocates the update-history buffer the
+    staleness ``correction`` (DPO_CORR_*) uses. With ``host_grad`` / ``host_param`` the grad /
     param arenas are pinned host memory instead, which the fused kernel reads
     and writes across the host link (see include/dpo.h).
     """
@@ -225,7 +228,8 @@ class DelayedAdamW:
                  grad_dtype=DPO_BF16, lr=3e-4, beta1=0.9, beta2=0.95, eps=1e-8,
                  weight_decay=0.1, ef=False, ef_lambda=1.0, max_grad_norm=0.0, delay=1,
                  wd_on: Optional[Sequence[bool]] = None, device=None, x0=None,
-                 init_mode=DPO_INIT_FRESH, stream=None, host_grad=False, host_param=False):
+                 init_mode=DPO_INIT_FRESH, stream=None, host_grad=False, host_param=False,
+                 correction=DPO_CORR_EF):
         import torch
         self.torch = torch
         self.device = torch.device(device or "cuda")
@@ -249,7 +253,7 @@ class DelayedAdamW:
         if x0 is not None:
             self.master.copy_(x0)
         self.hp = dpo_hparams(beta1, beta2, eps, weight_decay, ef_lambda if ef else 0.0,
-                              max_grad_norm, delay)
+                              max_grad_norm, delay, correction)
         self.wd_on = list(wd_on) if wd_on is not None else [True] * len(numels)
         self.ctx = None
         self._init(init_mode, stream)

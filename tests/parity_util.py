@@ -121,6 +121,7 @@ class Case:
     seed: int = 0xD0D0
     grad_sigma: float = 1e-3
     init_sigma: float = 0.02
+    correction: int = dpo.DPO_CORR_EF   # with ef: EF, SAPipe same / updated state
     host_grad: bool = False     # grad arena in pinned host memory
     host_param: bool = False    # bf16 param arena in pinned host memory
 
@@ -140,7 +141,7 @@ class Run:
             ef=case.ef, ef_lambda=case.ef_lambda, max_grad_norm=case.max_grad_norm,
             delay=case.delay, wd_on=case.wd_on, device=device,
             x0=self._dev_x0(device), init_mode=dpo.DPO_INIT_FRESH,
-            host_grad=case.host_grad, host_param=case.host_param)
+            host_grad=case.host_grad, host_param=case.host_param, correction=case.correction)
         # the oracle tracks every element, or only ``sample`` (global indices)
         self.sample = sample
         idx = np.arange(self.N) if sample is None else np.asarray(sample, np.int64)
@@ -148,7 +149,8 @@ class Run:
         x0 = synth.host_normal_at(case.seed, synth.STREAM_INIT, 0, idx, case.init_sigma)
         hp = oracle.HParams(lr=case.lr, weight_decay=case.weight_decay,
                             ef_lambda=case.ef_lambda if case.ef else 0.0,
-                            max_grad_norm=case.max_grad_norm, delay=case.delay).as_f32()
+                            max_grad_norm=case.max_grad_norm, delay=case.delay,
+                            correction=case.correction).as_f32()
         if sample is None:
             parts = np.split(x0.astype(np.float64), self.offs[1:-1])
             wd = case.wd_on

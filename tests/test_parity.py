@@ -280,3 +280,36 @@ def test_switch_to_host_io_continues_bitwise(cuda_device):
     finally:
         a.close()
         b.close()
+
+
+SP_SAME, SP_UPD = dpo.DPO_CORR_SAPIPE_SAME, dpo.DPO_CORR_SAPIPE_UPDATED
+
+
+@pytest.mark.parametrize("corr", [SP_SAME, SP_UPD])
+@pytest.mark.parametrize("pdt,sdt,gdt,clip", [(B, B, B, 0.0), (B, F, B, 0.3), (F, F, F, 0.0)])
+def test_sapipe_parity(cuda_device, corr, pdt, sdt, gdt, clip):
+    """App. B.1 SAPipe-WP prediction (same / updated optimizer state): the
+    stash receives the prediction point, the weights the standard rule."""
+    run = Run(Case(RAGGED, param_dtype=pdt, stash_dtype=sdt, grad_dtype=gdt, ef=True,
+                   correction=corr, max_grad_norm=clip), cuda_device)
+    try:
+        for k in range(1, 7):
+            run.step()
+            run.assert_close(TOL_ONE_STEP if k == 1 else TOL_RUN)
+    finally:
+        run.close()
+
+
+def test_sapipe_same_weights_equal_standard_rule_bitwise(cuda_device):
+    a = Run(Case(RAGGED, ef=False), cuda_device)
+    b = Run(Case(RAGGED, ef=True, correction=SP_SAME), cuda_device)
+    try:
+        for _ in range(4):
+            a.step()
+            b.step()
+        torch.cuda.synchronize()
+        assert torch.equal(a.gpu.master, b.gpu.master)
+        assert not torch.equal(a.gpu.stash, b.gpu.stash)   # prediction points differ
+    finally:
+        a.close()
+        b.close()

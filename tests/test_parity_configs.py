@@ -34,11 +34,11 @@ pytestmark = pytest.mark.gpu
 FULL = os.environ.get("DPO_FULL_RUNS", "0") == "1"
 
 
-def _case(w: W.Workload, ef: bool) -> Case:
+def _case(w: W.Workload, ef: bool, correction: int = dpo.DPO_CORR_EF) -> Case:
     return Case(w.numels, param_dtype=w.param_dtype, stash_dtype=w.stash_dtype,
                 grad_dtype=w.grad_dtype, ef=ef, max_grad_norm=w.max_grad_norm, lr=w.lr,
                 weight_decay=w.weight_decay, seed=w.seed, grad_sigma=W.GRAD_SIGMA,
-                init_sigma=W.INIT_SIGMA)
+                init_sigma=W.INIT_SIGMA, correction=correction)
 
 
 def _free():
@@ -149,6 +149,29 @@ def test_llama_7b(cuda_device, ef):
     master/m/v (and EF buffer): ~148 GB resident with EF."""
     w = W.LLAMA_7B
     run = Run(_case(w, ef), cuda_device, sample=sample_indices(w.numels, 1_000_000))
+    try:
+        _run_steps(run, w.steps, check_every=5)
+    finally:
+        run.close()
+        _free()
+
+
+@pytest.mark.parametrize("corr", [dpo.DPO_CORR_SAPIPE_SAME, dpo.DPO_CORR_SAPIPE_UPDATED])
+def test_gpt2_small_sapipe(cuda_device, corr):
+    """SAPipe-WP prediction (App. B.1) on the 124M set, 100 steps."""
+    w = W.GPT2_SMALL
+    run = Run(_case(w, True, corr), cuda_device, sample=sample_indices(w.numels, 1_000_000))
+    try:
+        _run_steps(run, w.steps, check_every=10)
+    finally:
+        run.close()
+        _free()
+
+
+def test_llama_7b_sapipe_updated(cuda_device):
+    w = W.LLAMA_7B
+    run = Run(_case(w, True, dpo.DPO_CORR_SAPIPE_UPDATED), cuda_device,
+              sample=sample_indices(w.numels, 1_000_000))
     try:
         _run_steps(run, w.steps, check_every=5)
     finally:
