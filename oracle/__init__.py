@@ -79,9 +79,9 @@ def load(path: Optional[str] = None):
     lib = ctypes.CDLL(path)
     lib.oracle_step.restype = ctypes.c_int
     lib.oracle_step.argtypes = [
-        ctypes.c_int64, ctypes.c_int64, ctypes.POINTER(_HParams), _dp,
-        ctypes.c_double, ctypes.POINTER(ctypes.c_uint8), _dp, _dp, _dp, _dp,
-        _dp, _dp]
+        ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, ctypes.POINTER(_HParams), _dp,
+        ctypes.c_double, ctypes.POINTER(ctypes.c_uint8), ctypes.POINTER(ctypes.c_uint8),
+        _dp, _dp, _dp, _dp, _dp, _dp]
     lib.oracle_sqnorm.restype = ctypes.c_double
     lib.oracle_sqnorm.argtypes = [ctypes.c_int64, _dp]
     lib.oracle_sqnorm_f32.restype = ctypes.c_double
@@ -197,12 +197,20 @@ class DelayedOptimizer:
     """Alg. 1 with AdamW (or the test-only SGD rule) over a set of tensors.
 
     The tensors are kept concatenated (the step is elementwise; only the clip
-    norm spans them). Version tags follow Alg. 1's iterate index: after
-    construction the stash holds x_0 (tag 0) and the master holds
-    x_1 = x_0 (tag 1, iteration t = 0 applies u_{-1} = 0); after call k the
-    master holds x_{k+1} and the stash x_k. With delay = 1 the gradient
-    consumed by call k must be evaluated at the stash (tag k - 1); with
-    delay = 0 it must be evaluated at the latest weights.
+    norm spans them). Version tags follow Alg. 1's iterate index: with delay
+    from the start, after construction the stash holds x_0 (tag 0) and the
+    master holds x_1 = x_0 (tag 1, iteration t = 0 applies u_{-1} = 0); after
+    call k the master holds x_{k+1} and the stash x_k. With delay = 1 the
+    gradient consumed by a call must be evaluated at the stale view (the
+    stash, or the latest weights for tensors trained synchronously); with
+    delay = 0 at the latest weights.
+
+    ``delayed`` marks per tensor whether it takes delayed updates (default
+    all): WPipe (App. B.2) delays half the model, the LM-head ablation
+    (App. A.9) keeps the head synchronous. ``set_delay`` switches the whole
+    run between synchronous and delayed training (synchronous start and
+    cooldown, Sec. 3.1): entering delayed training stashes the current
+    weights and restarts Alg. 1 (u_{-1} = 0, standard rule at its first call).
     """
     x0: Sequence[np.ndarray]
     hp: HParams = field(default_factory=HParams)
@@ -213,6 +221,7 @@ class DelayedOptimizer:
     grad_store: int = F32
     wd_on: Optional[Sequence[bool]] = None
     lib: object = None
+    delayed: Optional[Sequence[bool]] = None
 
     def __post_init__(self):
         self.lib = self.lib or load()
@@ -225,29 +234,51 @@ class DelayedOptimizer:
         self.m = np.zeros(n)
         self.v = np.zeros(n)
         self.u_prev = np.zeros(n) if self.ef else None
-        self.stash = (round_to(self.x, self.stash_store, self.lib)
-                      if self.hp.delay == 1 else None)
+        self.stash = round_to(self.x, self.stash_store, self.lib)
         self.param = (round_to(self.x, self.param_store, self.lib)
                       if self.param_store is not None else None)
-        if self.wd_on is None:
-            self.mask = None
-        else:
-            self.mask = np.concatenate([
-                np.full(s, 1 if on else 0, np.uint8)
-                for s, on in zip(self.sizes, self.wd_on)]) if n else np.zeros(0, np.uint8)
+        self.mask = self._tensor_mask(self.wd_on, n)
+        self.delay_mask = self._tensor_mask(self.delayed, n)
+        self.delay = self.hp.delay
         self.k = 0
-        self.latest_tag = 1 if self.hp.delay == 1 else 0
+        self.t = 0   # Alg. 1 iteration within the current delayed phase
+        self.latest_tag = 1 if self.delay == 1 else 0
         self.stash_tag = 0
         self.last_clip = 1.0
         self.last_sqnorm = 0.0
 
+    def _tensor_mask(self, flags, n):
+        if flags is None:
+            return None
+        if not n:
+            return np.zeros(0, np.uint8)
+        return np.concatenate([np.full(s, 1 if on else 0, np.uint8)
+                               for s, on in zip(self.sizes, flags)])
+
     def read_weights(self, which: str = "stale"):
-        """(weights, tag): the stale stash (what the next forward/backward
-        reads under delay = 1) or the latest weights."""
-        if which == "stale" and self.hp.delay == 1:
-            return self.stash, self.stash_tag
+        """(weights, tag): the stale view (what the next forward/backward
+        reads under delay = 1: the stash, with the latest weights for
+        synchronously trained tensors) or the latest weights."""
         latest = self.param if self.param is not None else self.x
+        if which == "stale" and self.delay == 1:
+            if self.delay_mask is None:
+                return self.stash, self.stash_tag
+            return np.where(self.delay_mask == 1, self.stash, latest), self.stash_tag
         return latest, self.latest_tag
+
+    def set_delay(self, delay: int) -> None:
+        """Switch between synchronous (0) and one-step-delayed (1) training.
+        Entering delayed training stashes the current weights and zeroes the
+        update history: Alg. 1 restarts there."""
+        if delay == self.delay:
+            return
+        if delay == 1:
+            self.stash = round_to(self.x, self.stash_store, self.lib)
+            if self.u_prev is not None:
+                self.u_prev[:] = 0.0
+            self.t = 0
+            self.stash_tag = self.latest_tag
+        self.delay = delay
 
     def step(self, g, tag: Optional[int] = None, lr: Optional[float] = None,
              sq: Optional[float] = None) -> None:
@@ -256,11 +287,13 @@ class DelayedOptimizer:
         given); ``sq``: the gradient's squared norm when ``g`` covers only a
         sample of the elements (clipping needs the full norm)."""
         g = _f64(g).ravel()
-        expected = self.stash_tag if self.hp.delay == 1 else self.latest_tag
+        expected = self.stash_tag if self.delay == 1 else self.latest_tag
         if tag is not None and tag != expected:
             raise StaleVersionError(
                 f"gradient from version {tag}, Alg. 1 needs version {expected}")
         self.k += 1
+        if self.delay == 1:
+            self.t += 1
         if sq is None:
             sq = float(self.lib.oracle_sqnorm(g.size, _ptr(g)))
         self.last_sqnorm = sq
@@ -268,16 +301,17 @@ class DelayedOptimizer:
         self.last_clip = clip
         hp = _HParams(lr if lr is not None else self.hp.lr, self.hp.beta1,
                       self.hp.beta2, self.hp.eps, self.hp.weight_decay,
-                      self.hp.ef_lambda, self.hp.delay, self.hp.rule, self.hp.correction,
+                      self.hp.ef_lambda, self.delay, self.hp.rule, self.hp.correction,
                       self.x_store, self.stash_store,
                       self.param_store if self.param_store is not None else F64)
         rc = self.lib.oracle_step(
-            g.size, self.k, ctypes.byref(hp), _ptr(g), clip,
-            _ptr(self.mask, ctypes.c_uint8), _ptr(self.x), _ptr(self.m),
-            _ptr(self.v), _ptr(self.u_prev), _ptr(self.stash), _ptr(self.param))
+            g.size, self.k, max(self.t, 1), ctypes.byref(hp), _ptr(g), clip,
+            _ptr(self.mask, ctypes.c_uint8), _ptr(self.delay_mask, ctypes.c_uint8),
+            _ptr(self.x), _ptr(self.m), _ptr(self.v), _ptr(self.u_prev), _ptr(self.stash),
+            _ptr(self.param))
         if rc != 0:
             raise ValueError("oracle_step rejected its arguments")
-        if self.hp.delay == 1:
+        if self.delay == 1:
             self.stash_tag = self.latest_tag
         self.latest_tag += 1
 

@@ -67,12 +67,12 @@ void oracle_round_n(int64_t n, const double *in, double *out, int store)
         out[i] = oracle_round(in[i], store);
 }
 
-int oracle_step(int64_t n, int64_t k, const oracle_hparams *hp,
+int oracle_step(int64_t n, int64_t k, int64_t t, const oracle_hparams *hp,
                 const double *g, double clip_scale, const uint8_t *wd_on,
-                double *x, double *m, double *v, double *u_prev,
-                double *stash, double *param)
+                const uint8_t *delay_on, double *x, double *m, double *v,
+                double *u_prev, double *stash, double *param)
 {
-    if (n < 0 || k < 1 || hp == NULL || (n > 0 && (g == NULL || x == NULL)))
+    if (n < 0 || k < 1 || t < 1 || hp == NULL || (n > 0 && (g == NULL || x == NULL)))
         return -1;
     if (hp->rule == ORACLE_RULE_ADAMW && n > 0 && (m == NULL || v == NULL))
         return -1;
@@ -89,9 +89,8 @@ int oracle_step(int64_t n, int64_t k, const oracle_hparams *hp,
         return -1;
     if (corr == ORACLE_CORR_SAPIPE_UPDATED && hp->rule != ORACLE_RULE_ADAMW)
         return -1;
-    /* Alg. 1: the standard rule is used for t <= 1 even under EF; call k is
-     * iteration t = k. */
-    const int ef_now = use_ef && corr == ORACLE_CORR_EF && k >= 2;
+    /* Alg. 1: the standard rule is used for t <= 1 even under EF. */
+    const int ef_now = use_ef && corr == ORACLE_CORR_EF && t >= 2;
     const double lam = hp->ef_lambda;
 
     /* Bias corrections of Adam at the k-th gradient, and at the (k+1)-th for
@@ -106,6 +105,10 @@ int oracle_step(int64_t n, int64_t k, const oracle_hparams *hp,
         const double gi = clip_scale * g[i];
         const double wd = (wd_on == NULL || wd_on[i]) ? hp->weight_decay : 0.0;
         const double xt = x[i];
+        /* An element of a synchronously trained tensor: no stash, no
+         * correction, its history untouched. */
+        const int delayed = hp->delay == 1 && (delay_on == NULL || delay_on[i]);
+        const int hist_i = use_ef && delayed;
 
         /* Update the optimizer statistics with g_{t-1} and form u_{t-1}. */
         double u, mi = 0.0, vi = 0.0;
@@ -123,7 +126,7 @@ int oracle_step(int64_t n, int64_t k, const oracle_hparams *hp,
 
         /* Apply it: standard delayed rule, or the EF correction. */
         double xn;
-        if (!ef_now)
+        if (!(ef_now && delayed))
             xn = xt - u;
         else
             xn = xt - u - lam * (u - u_prev[i]);
@@ -133,14 +136,14 @@ int oracle_step(int64_t n, int64_t k, const oracle_hparams *hp,
          * behind the latest; under SAPipe-WP it is the prediction made at the
          * previous step, x_t - u_prev, a weight in the master's format
          * rounded to the stash format. */
-        if (hp->delay == 1) {
+        if (delayed) {
             if (corr == ORACLE_CORR_EF)
                 stash[i] = oracle_round(xt, hp->stash_store);
             else
                 stash[i] = oracle_round(oracle_round(xt - u_prev[i], hp->x_store),
                                         hp->stash_store);
         }
-        if (use_ef) {
+        if (hist_i) {
             double hist = u;
             if (corr == ORACLE_CORR_SAPIPE_UPDATED) {
                 /* The optimizer step once more on g_{t-1}, from the state the

@@ -77,14 +77,23 @@ typedef struct {
  * One call of the delayed step over n elements (one flat tensor or the
  * concatenation of several; the step is elementwise).
  *
- *   k          number of stale gradients consumed including this one (>= 1);
- *              the first call is Alg. 1 iteration t = 1, because t = 0 only
- *              sets x_1 = x_0 (u_{-1} = 0).
+ *   k          number of gradients consumed including this one (>= 1): the
+ *              index of Adam's bias corrections.
+ *   t          Alg. 1 iteration of this call within the current delayed
+ *              phase (>= 1): t = k when training is delayed from the start;
+ *              after a switch from synchronous to delayed training Alg. 1
+ *              restarts, its first delayed call being t = 1 (t = 0 only sets
+ *              x_1 = x_0, u_{-1} = 0). The EF correction applies from t = 2.
  *   g          the gradient evaluated at the stash (the stale weights), as
  *              doubles holding values of the gradient storage format.
  *   clip_scale multiplier applied to g (1 when clipping is off), from
  *              oracle_clip_coef().
  *   wd_on      per-element 0/1 mask for weight decay, or NULL (decay on all).
+ *   delay_on   per-element 0/1 mask under delay == 1: 0 marks elements of a
+ *              tensor trained synchronously (its gradient evaluated at the
+ *              latest weights: no stash, no correction, history untouched), as
+ *              in WPipe (App. B.2) or a synchronous LM head (App. A.9); NULL
+ *              means every element is delayed.
  *   x, m, v    master weights and Adam moments, updated in place.
  *   u_prev     update-history buffer: u_{t-2} on entry and u_{t-1} on return
  *              (SAPIPE_UPDATED: the prediction updates). NULL selects the
@@ -98,10 +107,10 @@ typedef struct {
  *
  * Returns 0, or -1 on an invalid argument.
  */
-int oracle_step(int64_t n, int64_t k, const oracle_hparams *hp,
+int oracle_step(int64_t n, int64_t k, int64_t t, const oracle_hparams *hp,
                 const double *g, double clip_scale, const uint8_t *wd_on,
-                double *x, double *m, double *v, double *u_prev,
-                double *stash, double *param);
+                const uint8_t *delay_on, double *x, double *m, double *v,
+                double *u_prev, double *stash, double *param);
 
 /* Sum of g_i^2 in double over n elements (fixed order: blocks of 65536
  * elements summed left to right, block sums added left to right). */

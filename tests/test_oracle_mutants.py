@@ -26,7 +26,7 @@ MUTANTS = [
     ("eps_inside_sqrt", "(sqrt(v_hat) + hp->eps)", "sqrt(v_hat + hp->eps)"),
     ("ef_sign_flipped", "xn = xt - u - lam * (u - u_prev[i]);",
      "xn = xt - u + lam * (u - u_prev[i]);"),
-    ("ef_at_first_update", "corr == ORACLE_CORR_EF && k >= 2", "corr == ORACLE_CORR_EF && k >= 1"),
+    ("ef_at_first_update", "corr == ORACLE_CORR_EF && t >= 2", "corr == ORACLE_CORR_EF && t >= 1"),
     ("bias_correction_index", "pow(hp->beta1, (double)k)", "pow(hp->beta1, (double)(k + 1))"),
     ("no_bias_correction_m", "const double m_hat = mi / bc1;", "const double m_hat = mi;"),
     ("stash_holds_new_weights", "stash[i] = oracle_round(xt, hp->stash_store);",
@@ -48,6 +48,9 @@ MUTANTS = [
     ("sapipe_updated_decays_old_weights", "wd * oracle_round(xn, hp->x_store)", "wd * xt"),
     ("sapipe_updated_no_second_blend", "hp->beta1 * mi + (1.0 - hp->beta1) * gi;",
      "mi;"),
+    ("delay_mask_ignored", "(delay_on == NULL || delay_on[i])", "(1)"),
+    ("ef_restart_counts_all_steps", "corr == ORACLE_CORR_EF && t >= 2",
+     "corr == ORACLE_CORR_EF && k >= 2"),
 ]
 
 

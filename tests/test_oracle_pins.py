@@ -559,3 +559,101 @@ def test_sapipe_updated_hand_steps(lib):
     assert o.x[0] == pytest.approx(0.9 - u2, rel=1e-14)
     assert o.u_prev[0] == pytest.approx(0.1 * (0.352 / 0.271) / math.sqrt(0.278 / 0.142625),
                                         rel=1e-14)
+
+
+# ------------------------------- per-tensor delay and mode switches (Sec. 3.1,
+# App. A.9 synchronous LM head, App. B.2 WPipe)
+
+def _sgd_quadratic_run(lib, a, x0, steps, ef=False, delayed=None, schedule=None, eta=0.3):
+    """Alg. 1 driver, SGD rule, on f = sum a_i/2 x_i^2; ``schedule[c]`` is the
+    delay mode to switch to before call c (1-based)."""
+    hp = HParams(lr=eta, weight_decay=0.0, rule=oracle.RULE_SGD, ef_lambda=1.0 if ef else 0.0,
+                 delay=(schedule or {}).get(0, 1))
+    o = oracle.DelayedOptimizer([np.array([v]) for v in x0], hp, ef=ef, x_store=F64,
+                                stash_store=F64, delayed=delayed, lib=lib)
+    xs = [o.x.copy()]
+    for c in range(1, steps + 1):
+        if schedule and c in schedule:
+            o.set_delay(schedule[c])
+        w, tag = o.read_weights("stale")
+        g, _ = oracle.quadratic(a, [0.0] * len(a), w, None, F64, lib=lib)
+        o.step(g, tag=tag)
+        xs.append(o.x.copy())
+    return np.array(xs)
+
+
+def _alg1_closed_form(q, x_start, n, ef):
+    """Alg. 1 from x_0 = x_1 = x_start with u = eta g on a/2 x^2 (q = eta a):
+    element j of the result is x_j."""
+    if ef:
+        return _linear_recurrence_closed_form([1.0, -2 * q, q],
+                                              [x_start, x_start, (1 - q) * x_start], n)
+    return _linear_recurrence_closed_form([1.0, -q], [x_start, x_start], n)
+
+
+def test_per_tensor_delay_sync_and_delayed_side_by_side(lib):
+    """One run, two tensors: the synchronous one decays geometrically,
+    x_{t+1} = (1 - q) x_t, the delayed one follows Alg. 1's recurrence."""
+    a, x0, n, eta = [0.25, 0.5], [1.0, -2.0], 30, 0.3
+    xs = _sgd_quadratic_run(lib, a, x0, n, delayed=[True, False], eta=eta)
+    q0, q1 = eta * a[0], eta * a[1]
+    e0 = _alg1_closed_form(q0, x0[0], n + 2, ef=False)
+    for c in range(1, n + 1):
+        assert xs[c][0] == pytest.approx(e0[c + 1], rel=1e-11, abs=1e-13)
+        assert xs[c][1] == pytest.approx(x0[1] * (1 - q1) ** c, rel=1e-11, abs=1e-13)
+
+
+@pytest.mark.parametrize("ef", [False, True])
+def test_synchronous_start_then_delay(lib, ef):
+    """S synchronous steps, then delayed training (Sec. 3.1): geometric
+    decay, then Alg. 1 restarted from the switch point (its first delayed
+    call uses the standard rule even under EF)."""
+    a, x0, S, n, eta = [0.25], [1.0], 5, 25, 0.3
+    q = eta * a[0]
+    xs = _sgd_quadratic_run(lib, a, x0, S + n, ef=ef, schedule={0: 0, S + 1: 1}, eta=eta)
+    for c in range(1, S + 1):
+        assert xs[c][0] == pytest.approx((1 - q) ** c, rel=1e-12)
+    xS = (1 - q) ** S
+    e = _alg1_closed_form(q, xS, n + 2, ef)
+    for j in range(1, n + 1):   # call S + j leaves x_{j+1} of the restarted run
+        assert xs[S + j][0] == pytest.approx(e[j + 1], rel=1e-10, abs=1e-13)
+
+
+@pytest.mark.parametrize("ef", [False, True])
+def test_synchronous_cooldown(lib, ef):
+    """Delayed training, then synchronous from call D + 1 (App. A.10): Alg. 1,
+    then geometric decay from the weights reached."""
+    a, x0, D, n, eta = [0.25], [1.0], 12, 10, 0.3
+    q = eta * a[0]
+    xs = _sgd_quadratic_run(lib, a, x0, D + n, ef=ef, schedule={D + 1: 0}, eta=eta)
+    e = _alg1_closed_form(q, x0[0], D + 2, ef)
+    for c in range(1, D + 1):
+        assert xs[c][0] == pytest.approx(e[c + 1], rel=1e-10, abs=1e-13)
+    for j in range(1, n + 1):
+        assert xs[D + j][0] == pytest.approx(xs[D][0] * (1 - q) ** j, rel=1e-11, abs=1e-14)
+
+
+def test_per_tensor_delay_is_elementwise(lib):
+    """With fixed gradients, a mixed table equals, tensor by tensor, an
+    all-delayed run and an all-synchronous run (bitwise)."""
+    rng = np.random.default_rng(8)
+    sizes = [13, 7, 21]
+    x0 = [rng.normal(0, 0.5, s) for s in sizes]
+    grads = [rng.normal(0, 1.0, sum(sizes)) for _ in range(6)]
+
+    def run(delayed, delay):
+        hp = HParams(lr=0.01, ef_lambda=1.0, delay=delay)
+        o = oracle.DelayedOptimizer(x0, hp, ef=True, x_store=F32, stash_store=F32,
+                                    delayed=delayed, lib=lib)
+        for g in grads:
+            o.step(g)
+        return o
+
+    mixed = run([True, False, True], 1)
+    all_d, all_s = run(None, 1), run(None, 0)
+    for i, ref in ((0, all_d), (1, all_s), (2, all_d)):
+        for name in ("x", "m", "v"):
+            assert np.array_equal(mixed.tensor(name, i), ref.tensor(name, i))
+    assert np.array_equal(mixed.tensor("stash", 0), all_d.tensor("stash", 0))
+    assert np.array_equal(mixed.tensor("u_prev", 2), all_d.tensor("u_prev", 2))
+    assert np.array_equal(mixed.tensor("u_prev", 1), np.zeros(7))   # history untouched
