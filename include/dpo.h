@@ -69,6 +69,11 @@ typedef enum { DPO_F32 = 0, DPO_BF16 = 1 } dpo_dtype;
 
 /* dpo_tensor.flags */
 #define DPO_WD_ON 1u     /* apply weight decay to this tensor */
+#define DPO_SYNC 2u      /* train this tensor synchronously even while the run is
+                          * delayed: its gradient is evaluated at the latest
+                          * weights, no stash is written and no correction runs
+                          * (WPipe's second half, App. B.2; the synchronous LM
+                          * head of App. A.9) */
 
 /* dpo_read_weights(which) */
 #define DPO_STALE 0      /* what the next forward/backward reads (the stash) */
@@ -120,8 +125,10 @@ typedef struct {
     float *master;     /* fp32 master weights, read and written */
     float *m;          /* Adam first moment, fp32, read and written */
     float *v;          /* Adam second moment, fp32, read and written */
-    /* Stale weights in the stash dtype: x_t after each step. Required when
-     * delay == 1; ignored (may be NULL) when delay == 0. */
+    /* Stale weights in the stash dtype: x_t after each step (the SAPipe
+     * prediction point under those corrections). Required for tensors without
+     * DPO_SYNC when delay == 1; with delay == 0 it may be NULL, and giving it
+     * lets dpo_set_delay switch the run to delayed training later. */
     void *stash;
     /* Update-history (EF) buffer (fp32): u_{t-2} on entry, u_{t-1} on return
      * (the prediction update under DPO_CORR_SAPIPE_UPDATED). NULL on every
@@ -168,9 +175,24 @@ int dpo_stash(dpo_ctx *ctx, void *cuda_stream);
 int dpo_step(dpo_ctx *ctx, float lr, void *cuda_stream);
 
 /*
+ * Switch the run between synchronous (delay = 0) and one-step-delayed
+ * (delay = 1) training: synchronous start and synchronous cooldown (Sec. 3.1,
+ * App. A.10). Entering delayed training enqueues stash := master for every
+ * delayed tensor and zeroes the update-history buffers, so Alg. 1 restarts at
+ * the next dpo_step: the gradient it consumes is evaluated at the stash (the
+ * current weights), its update uses the standard rule, and EF applies from the
+ * following call. Needs stash buffers for every tensor without DPO_SYNC
+ * (DPO_ESTATE otherwise). Leaving it takes effect at the next dpo_step, whose
+ * gradient must then be evaluated at the latest weights. No host
+ * synchronization.
+ */
+int dpo_set_delay(dpo_ctx *ctx, int delay, void *cuda_stream);
+
+/*
  * Pointer and dtype of tensor `tensor`'s stale (DPO_STALE) or latest
- * (DPO_LATEST) weights. Under delay == 0 both name the latest weights. The
- * pointer is one of the caller's own buffers; no copy is made.
+ * (DPO_LATEST) weights. Under delay == 0, and for DPO_SYNC tensors, both name
+ * the latest weights. The pointer is one of the caller's own buffers; no copy
+ * is made.
  */
 int dpo_read_weights(const dpo_ctx *ctx, int which, int tensor,
                      const void **ptr, dpo_dtype *dtype);

@@ -29,10 +29,14 @@ struct dpo_ctx {
     bool ef = false;
     bool clip = false;
     bool host_io = false;   // grad or param in host memory
+    bool has_stash = false; // some tensor has a stash buffer
+    bool can_delay = false; // every tensor without DPO_SYNC has one
     int64_t k = 0;
+    int64_t phase_k0 = 0;   // k when the current delayed phase began
     int64_t total_pkts = 0;
     int64_t total_elems = 0;
     std::vector<dpo_tensor> table;
+    int sms = 0;
     int step_grid = 0, norm_grid = 0, stash_grid = 0;
     // one device allocation: table | pkt_begin | partials | scalars
     void *dev_block = nullptr;
@@ -69,9 +73,18 @@ int cuda_fail(dpo_ctx *c, cudaError_t e, const char *what)
 bool valid_dtype(int d) { return d == DPO_F32 || d == DPO_BF16; }
 int64_t dt_size(dpo_dtype d) { return d == DPO_BF16 ? 2 : 4; }
 bool aligned(const void *p) { return (reinterpret_cast<uintptr_t>(p) % dpo::kAlign) == 0; }
+// Stash kind of the fused step: none while the run is synchronous.
 StashKind stash_kind(const dpo_ctx *c)
 {
     if (c->hp.delay == 0)
+        return dpo::kStashNone;
+    return c->stash_dt == DPO_BF16 ? dpo::kStashBF16 : dpo::kStashF32;
+}
+
+// Stash kind of the stash kernel: the buffers' dtype whenever they exist.
+StashKind stash_buffer_kind(const dpo_ctx *c)
+{
+    if (!c->has_stash)
         return dpo::kStashNone;
     return c->stash_dt == DPO_BF16 ? dpo::kStashBF16 : dpo::kStashF32;
 }
@@ -98,6 +111,39 @@ struct Span {
 };
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+int grid_of(const dpo_ctx *c, int per_sm, int64_t pkts_per_cta)
+{
+    const int64_t groups = std::max<int64_t>(1, (c->total_pkts + pkts_per_cta - 1) / pkts_per_cta);
+    return static_cast<int>(
+        std::min<int64_t>(groups, (int64_t)std::max(1, c->sms) * std::max(1, per_sm)));
+}
+
+// Grid of the fused step for the context's current mode. Its CTAs per SM put
+// about kStepInflightPerSm bytes of loads in flight per SM (see
+// dpo_internal.h): bytes loaded per packet = master, m, v, grad and, under a
+// correction, the update-history buffer.
+int set_step_grid(dpo_ctx *c)
+{
+    const dpo::Correction corr = correction_kind(c->ef, c->hp);
+    int per_sm = 0;
+    const cudaError_t e = dpo::step_ctas_per_sm(c->param_dt == DPO_BF16, stash_kind(c),
+                                                c->grad_dt == DPO_BF16, corr, &per_sm);
+    if (e != cudaSuccess)
+        return cuda_fail(c, e, "occupancy query");
+    const int64_t load_bytes =
+        dpo::kPacket * (12 + dt_size(c->grad_dt) + (corr != dpo::kCorrNone ? 4 : 0));
+    int want = std::max<int>(1, (int)((dpo::kStepInflightPerSm + load_bytes * dpo::kStepThreads / 2) /
+                                      (load_bytes * dpo::kStepThreads)));
+    // The SAPipe updated-state prediction evaluates AdamW twice per element,
+    // so each thread spends longer between its loads: one more CTA per SM
+    // keeps the same bytes in flight (measured: 3 CTAs 89%, 4 CTAs 98% of the
+    // copy peak on the 7B set).
+    if (corr == dpo::kCorrSapipeUpdated)
+        want += 1;
+    c->step_grid = grid_of(c, std::min(per_sm, want), dpo::kStepThreads);
+    return DPO_OK;
+}
 
 }  // namespace
 
@@ -140,6 +186,7 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
 
     // Table: NULL pointers, EF consistency, alignment, overlaps.
     const bool ef = table[0].ef != nullptr;
+    bool has_stash = false, can_delay = true;
     std::vector<Span> spans;
     int64_t total_pkts = 0, total_elems = 0;
     for (int t = 0; t < n_tensors; ++t) {
@@ -149,14 +196,18 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
         if ((d.ef != nullptr) != ef)
             return fail(nullptr, DPO_EINVAL,
                         "tensor %d: EF buffers must be given for all tensors or for none", t);
-        if ((d.flags & ~DPO_WD_ON) != 0)
+        if ((d.flags & ~(DPO_WD_ON | DPO_SYNC)) != 0)
             return fail(nullptr, DPO_EINVAL, "tensor %d: unknown flags 0x%x", t, d.flags);
         if (d.numel == 0)
             continue;
         if (d.master == nullptr || d.m == nullptr || d.v == nullptr || d.grad == nullptr)
             return fail(nullptr, DPO_EINVAL, "tensor %d: master, m, v and grad are required", t);
-        if (hp->delay == 1 && d.stash == nullptr)
+        if (hp->delay == 1 && d.stash == nullptr && !(d.flags & DPO_SYNC))
             return fail(nullptr, DPO_EINVAL, "tensor %d: delay = 1 needs a stash buffer", t);
+        if (d.stash != nullptr)
+            has_stash = true;
+        else if (!(d.flags & DPO_SYNC))
+            can_delay = false;
         if (param_dtype == DPO_BF16 && d.param == nullptr)
             return fail(nullptr, DPO_EINVAL, "tensor %d: bf16 params need a param buffer", t);
         if (param_dtype == DPO_F32 && d.param != nullptr)
@@ -174,7 +225,7 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
             {d.v, 4 * d.numel, "v", false},
             {d.grad, dt_size(grad_dtype) * d.numel, "grad", true},
             {d.param, dt_size(param_dtype) * d.numel, "param", true},
-            {hp->delay == 1 ? d.stash : nullptr, dt_size(stash_dtype) * d.numel, "stash", false},
+            {d.stash, dt_size(stash_dtype) * d.numel, "stash", false},
             {d.ef, 4 * d.numel, "ef", false},
         };
         for (const auto &b : bufs) {
@@ -248,42 +299,27 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
     c->total_pkts = total_pkts;
     c->total_elems = total_elems;
     c->host_io = host_io;
+    c->has_stash = has_stash;
+    c->can_delay = can_delay && has_stash;
     c->table.assign(table, table + n_tensors);
 
     // Launch geometry: persistent grids, a fixed number of resident CTAs per
-    // SM, never more CTAs than there are CTA-widths of packets. The step's
-    // CTAs per SM put about kStepInflightPerSm bytes of loads in flight per SM
-    // (see dpo_internal.h): bytes loaded per packet = master, m, v, grad and,
-    // with EF, the EF buffer.
-    int sms = 0, per_sm_step = 0, per_sm_norm = 0;
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
-    e = dpo::step_ctas_per_sm(param_dtype == DPO_BF16, stash_kind(c), grad_dtype == DPO_BF16,
-                              correction_kind(ef, *hp), &per_sm_step);
-    if (e == cudaSuccess)
-        e = dpo::norm_ctas_per_sm(grad_dtype == DPO_BF16, &per_sm_norm);
+    // SM, never more CTAs than there are CTA-widths of packets (set_step_grid
+    // for the fused step).
+    int per_sm_norm = 0;
+    cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, device);
+    e = dpo::norm_ctas_per_sm(grad_dtype == DPO_BF16, &per_sm_norm);
     if (e != cudaSuccess) {
         int rc = cuda_fail(nullptr, e, "occupancy query");
         delete c;
         return rc;
     }
-    auto grid_of = [&](int per_sm, int64_t pkts_per_cta) {
-        const int64_t groups = std::max<int64_t>(1, (total_pkts + pkts_per_cta - 1) / pkts_per_cta);
-        return static_cast<int>(
-            std::min<int64_t>(groups, (int64_t)std::max(1, sms) * std::max(1, per_sm)));
-    };
-    const bool ef_active = ef && hp->delay == 1;
-    const int64_t load_bytes = dpo::kPacket * (12 + dt_size(grad_dtype) + (ef_active ? 4 : 0));
-    int want_per_sm = std::max<int>(
-        1, (int)((dpo::kStepInflightPerSm + load_bytes * dpo::kStepThreads / 2) /
-                 (load_bytes * dpo::kStepThreads)));
-    // The SAPipe updated-state prediction evaluates AdamW twice per element,
-    // so each thread spends longer between its loads: one more CTA per SM
-    // keeps the same bytes in flight (measured: 3 CTAs 89%, 4 CTAs 98% of the
-    // copy peak on the 7B set).
-    if (correction_kind(ef, *hp) == dpo::kCorrSapipeUpdated)
-        want_per_sm += 1;
-    c->step_grid = grid_of(std::min(per_sm_step, want_per_sm), dpo::kStepThreads);
-    c->norm_grid = grid_of(per_sm_norm, (int64_t)dpo::kNormThreads * dpo::kNormUnroll);
+    if (set_step_grid(c) != DPO_OK) {
+        g_init_err = c->err;
+        delete c;
+        return DPO_ECUDA;
+    }
+    c->norm_grid = grid_of(c, per_sm_norm, (int64_t)dpo::kNormThreads * dpo::kNormUnroll);
     c->stash_grid = c->step_grid;
 
     // Device block: table, packet prefix, norm scratch.
@@ -314,7 +350,7 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
         x.master = d.master;
         x.m = d.m;
         x.v = d.v;
-        x.stash = hp->delay == 1 ? d.stash : nullptr;
+        x.stash = d.stash;
         x.ef = d.ef;
         x.grad = d.grad;
         x.numel = d.numel;
@@ -339,8 +375,9 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
         return rc;
     }
     if (init_mode == DPO_INIT_FRESH && total_pkts > 0) {
-        dpo::StashArgs a{c->d_table, c->d_pkt_begin, n_tensors, total_pkts, 1};
-        e = dpo::launch_stash(param_dtype == DPO_BF16, stash_kind(c), c->stash_grid, a, s);
+        dpo::StashArgs a{c->d_table, c->d_pkt_begin, n_tensors, total_pkts, 1, 1};
+        e = dpo::launch_stash(param_dtype == DPO_BF16, stash_buffer_kind(c), c->stash_grid, a,
+                              s);
         if (e != cudaSuccess) {
             int rc = cuda_fail(nullptr, e, "launching the initial stash");
             cudaFree(c->dev_block);
@@ -358,10 +395,39 @@ extern "C" int dpo_stash(dpo_ctx *c, void *cuda_stream)
         return fail(nullptr, DPO_EINVAL, "ctx is NULL");
     if (c->total_pkts == 0)
         return DPO_OK;
-    dpo::StashArgs a{c->d_table, c->d_pkt_begin, c->n, c->total_pkts, 0};
-    const cudaError_t e = dpo::launch_stash(c->param_dt == DPO_BF16, stash_kind(c), c->stash_grid,
-                                            a, static_cast<cudaStream_t>(cuda_stream));
+    dpo::StashArgs a{c->d_table, c->d_pkt_begin, c->n, c->total_pkts, 0, 0};
+    const cudaError_t e = dpo::launch_stash(c->param_dt == DPO_BF16, stash_buffer_kind(c),
+                                            c->stash_grid, a,
+                                            static_cast<cudaStream_t>(cuda_stream));
     return e == cudaSuccess ? DPO_OK : cuda_fail(c, e, "stash launch");
+}
+
+extern "C" int dpo_set_delay(dpo_ctx *c, int delay, void *cuda_stream)
+{
+    if (c == nullptr)
+        return fail(nullptr, DPO_EINVAL, "ctx is NULL");
+    if (delay != 0 && delay != 1)
+        return fail(c, DPO_EINVAL, "delay must be 0 or 1");
+    if (delay == c->hp.delay)
+        return DPO_OK;
+    if (delay == 1) {
+        if (!c->can_delay)
+            return fail(c, DPO_ESTATE,
+                        "delayed training needs a stash buffer for every tensor without DPO_SYNC");
+        if (c->total_pkts > 0) {
+            // stash := the current weights, update history := 0: Alg. 1 restarts
+            dpo::StashArgs a{c->d_table, c->d_pkt_begin, c->n, c->total_pkts, 0, 1};
+            const cudaError_t e =
+                dpo::launch_stash(c->param_dt == DPO_BF16, stash_buffer_kind(c), c->stash_grid, a,
+                                  static_cast<cudaStream_t>(cuda_stream));
+            if (e != cudaSuccess)
+                return cuda_fail(c, e, "stash launch");
+        }
+        c->phase_k0 = c->k;
+    }
+    c->hp.delay = delay;
+    const int rc = set_step_grid(c);
+    return rc;
 }
 
 extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
@@ -370,7 +436,8 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
         return fail(nullptr, DPO_EINVAL, "ctx is NULL");
     if (!std::isfinite(lr) || lr < 0.0f)
         return fail(c, DPO_EINVAL, "lr must be finite and >= 0");
-    const int64_t k = c->k + 1;   // this call consumes the k-th stale gradient
+    const int64_t k = c->k + 1;        // this call consumes the k-th gradient
+    const int64_t t = k - c->phase_k0; // Alg. 1 iteration within the delayed phase
     cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
     if (c->total_pkts > 0) {
         if (c->clip) {
@@ -398,7 +465,7 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
         a.eps = c->hp.eps;
         a.lr_wd = (float)(lrd * (double)c->hp.weight_decay);
         // Alg. 1: the standard rule for t <= 1, i.e. at the first update.
-        a.lam = (corr == dpo::kCorrEF && k >= 2) ? c->hp.ef_lambda : 0.0f;
+        a.lam = (corr == dpo::kCorrEF && t >= 2) ? c->hp.ef_lambda : 0.0f;
         a.step_size_next = (float)(lrd / (1.0 - std::pow(b1, (double)(k + 1))));
         a.inv_sqrt_bc2_next = (float)(1.0 / std::sqrt(1.0 - std::pow(b2, (double)(k + 1))));
         a.clip = c->clip ? &c->d_scalars->clip : nullptr;
@@ -419,7 +486,7 @@ extern "C" int dpo_read_weights(const dpo_ctx *c, int which, int tensor, const v
     if (tensor < 0 || tensor >= c->n || (which != DPO_STALE && which != DPO_LATEST))
         return DPO_EINVAL;
     const dpo_tensor &d = c->table[tensor];
-    if (which == DPO_STALE && c->hp.delay == 1) {
+    if (which == DPO_STALE && c->hp.delay == 1 && !(d.flags & DPO_SYNC)) {
         *ptr = d.stash;
         if (dtype)
             *dtype = c->stash_dt;
@@ -480,17 +547,17 @@ extern "C" int dpo_algorithmic_bytes(const dpo_ctx *c, int64_t *step_bytes, int6
 {
     if (c == nullptr)
         return DPO_EINVAL;
-    // Per element: read master, m, v (fp32) and grad; write master, m, v,
-    // the stash (delay 1) and the bf16 param; EF reads and writes its buffer.
-    int64_t per = 4 * 3 + dt_size(c->grad_dt) + 4 * 3;
-    if (c->hp.delay == 1)
-        per += dt_size(c->stash_dt);
-    if (c->param_dt == DPO_BF16)
-        per += 2;
-    if (c->ef && c->hp.delay == 1)
-        per += 8;
+    // Per element: read master, m, v (fp32) and grad; write master, m, v and
+    // the bf16 param; a delayed tensor also writes its stash, and under a
+    // correction reads and writes its update-history buffer.
+    const int64_t base = 4 * 3 + dt_size(c->grad_dt) + 4 * 3 + (c->param_dt == DPO_BF16 ? 2 : 0);
+    const int64_t delayed_extra =
+        c->hp.delay == 1 ? dt_size(c->stash_dt) + (c->ef ? 8 : 0) : 0;
+    int64_t total = 0;
+    for (const dpo_tensor &d : c->table)
+        total += d.numel * (base + ((d.flags & DPO_SYNC) ? 0 : delayed_extra));
     if (step_bytes)
-        *step_bytes = per * c->total_elems;
+        *step_bytes = total;
     if (norm_bytes)
         *norm_bytes = c->clip ? dt_size(c->grad_dt) * c->total_elems : 0;
     return DPO_OK;

@@ -15,6 +15,8 @@
 namespace dpo {
 
 constexpr int kPacket = 8;      // elements per packet: 16 B of bf16, 32 B of fp32
+constexpr uint32_t kFlagWd = 1u;    // DPO_WD_ON
+constexpr uint32_t kFlagSync = 2u;  // DPO_SYNC
 constexpr int kAlign = 32;      // buffer alignment: fp32 packets move as 256-bit accesses
 
 // Fused step and stash kernels: 128-thread CTAs. The number resident per SM
@@ -95,6 +97,7 @@ struct StashArgs {
     int n_tensors;
     int64_t total_pkts;
     int zero_state;             // also zero m, v and the EF buffer (fresh start)
+    int zero_hist;              // also zero the EF buffer (delayed training restarts)
 };
 
 // Launchers (dpo_kernels.cu). Each returns the launch's cudaError_t.

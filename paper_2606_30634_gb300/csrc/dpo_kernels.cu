@@ -10,8 +10,9 @@
 //                       (App. E.1), deterministic: fixed per-thread order,
 //                       fixed block tree, fixed-order sum of the per-CTA
 //                       partials by the last CTA to finish (no spin-wait).
-//   stash_kernel        stash := master, param := master (Alg. 1 start, mode
-//                       switches), optionally zeroing m, v and the EF buffer.
+//   stash_kernel        stash := master (tensors without DPO_SYNC), param :=
+//                       master (Alg. 1 start, switches into delayed training),
+//                       optionally zeroing m, v and / or the EF buffer.
 //
 // All three are persistent (a fixed number of CTAs per SM) and walk the
 // 8-element packets of the virtual concatenation of the tensors grid-stride
@@ -207,7 +208,12 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
         const GT *__restrict__ grad = static_cast<const GT *>(d.grad);
         ST *__restrict__ stash = static_cast<ST *>(d.stash);
         __nv_bfloat16 *__restrict__ param = static_cast<__nv_bfloat16 *>(d.param);
-        const float wd_lr = (d.flags & 1u) ? a.lr_wd : 0.0f;
+        const float wd_lr = (d.flags & kFlagWd) ? a.lr_wd : 0.0f;
+        // A DPO_SYNC tensor takes the standard update with no stash and no
+        // correction even while the run is delayed.
+        const bool dly = SK != kStashNone && !(d.flags & kFlagSync);
+        const bool prev_t = dly && use_prev;
+        const bool efn_t = dly && ef_now;
         const int64_t e = (p - c.tb) * kPacket;
 
         if (e + kPacket <= d.numel) {
@@ -216,9 +222,9 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
             ld8(mm + e, m);
             ld8(vv + e, v);
             ld8(grad + e, g);
-            if (use_prev)
+            if (prev_t)
                 ld8(ef + e, up);
-            if (SK != kStashNone) {
+            if (dly) {
                 if (kSapipe) {   // stash := the prediction point x_t - u_prev
                     float xp[8];
 #pragma unroll
@@ -234,14 +240,14 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
             for (int j = 0; j < 8; ++j) {
                 const float gc = g[j] * clip;
                 u[j] = adamw_update(s, gc, x[j], wd_lr, m[j], v[j]);
-                x[j] -= ef_now ? ef_displacement(s.lam, u[j], up[j]) : u[j];
+                x[j] -= efn_t ? ef_displacement(s.lam, u[j], up[j]) : u[j];
                 if (CORR == kCorrSapipeUpdated)
                     u[j] = adamw_prediction(s, gc, x[j], wd_lr, m[j], v[j]);
             }
             st8(master + e, x);
             st8(mm + e, m);
             st8(vv + e, v);
-            if (kHist)
+            if (kHist && dly)
                 st8(ef + e, u);
             if (PB)
                 st8(param + e, x);
@@ -250,17 +256,17 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
             for (int64_t i = e; i < d.numel; ++i) {
                 float x = master[i], m = mm[i], v = vv[i];
                 const float g = ld1(grad + i) * clip;
-                const float up = use_prev ? ef[i] : 0.0f;
-                if (SK != kStashNone)
+                const float up = prev_t ? ef[i] : 0.0f;
+                if (dly)
                     st1(stash + i, kSapipe ? x - up : x);
                 float u = adamw_update(s, g, x, wd_lr, m, v);
-                x -= ef_now ? ef_displacement(s.lam, u, up) : u;
+                x -= efn_t ? ef_displacement(s.lam, u, up) : u;
                 if (CORR == kCorrSapipeUpdated)
                     u = adamw_prediction(s, g, x, wd_lr, m, v);
                 master[i] = x;
                 mm[i] = m;
                 vv[i] = v;
-                if (kHist)
+                if (kHist && dly)
                     ef[i] = u;
                 if (PB)
                     st1(param + i, x);
@@ -406,34 +412,36 @@ __global__ void __launch_bounds__(kStepThreads) stash_kernel(const StashArgs a)
             d = a.table[c.t];
         ST *stash = static_cast<ST *>(d.stash);
         __nv_bfloat16 *param = static_cast<__nv_bfloat16 *>(d.param);
+        const bool do_stash = SK != kStashNone && stash != nullptr && !(d.flags & kFlagSync);
+        const bool zero_ef = d.ef != nullptr && (a.zero_state || a.zero_hist);
         const int64_t e = (p - c.tb) * kPacket;
         if (e + kPacket <= d.numel) {
             float x[8];
+            const float z[8] = {0, 0, 0, 0, 0, 0, 0, 0};
             ld8(d.master + e, x);
-            if (SK != kStashNone)
+            if (do_stash)
                 st8(stash + e, x);
             if (PB)
                 st8(param + e, x);
             if (a.zero_state) {
-                const float z[8] = {0, 0, 0, 0, 0, 0, 0, 0};
                 st8(d.m + e, z);
                 st8(d.v + e, z);
-                if (d.ef != nullptr)
-                    st8(d.ef + e, z);
             }
+            if (zero_ef)
+                st8(d.ef + e, z);
         } else {
             for (int64_t i = e; i < d.numel; ++i) {
                 const float x = d.master[i];
-                if (SK != kStashNone)
+                if (do_stash)
                     st1(stash + i, x);
                 if (PB)
                     st1(param + i, x);
                 if (a.zero_state) {
                     d.m[i] = 0.0f;
                     d.v[i] = 0.0f;
-                    if (d.ef != nullptr)
-                        d.ef[i] = 0.0f;
                 }
+                if (zero_ef)
+                    d.ef[i] = 0.0f;
             }
         }
     }

@@ -22,6 +22,7 @@ from . import build as _build
 DPO_OK, DPO_EINVAL, DPO_EALIGN, DPO_EDTYPE, DPO_ECUDA, DPO_ESTATE, DPO_ENOMEM = 0, -1, -2, -3, -4, -5, -6
 DPO_F32, DPO_BF16 = 0, 1
 DPO_WD_ON = 1
+DPO_SYNC = 2
 DPO_STALE, DPO_LATEST = 0, 1
 DPO_INIT_FRESH, DPO_INIT_RESUME = 0, 1
 DPO_FLAG_NONFINITE = 1
@@ -29,7 +30,7 @@ DPO_CORR_EF, DPO_CORR_SAPIPE_SAME, DPO_CORR_SAPIPE_UPDATED = 0, 1, 2
 
 EXPORTS = ("dpo_init", "dpo_stash", "dpo_step", "dpo_read_weights", "dpo_get_step",
            "dpo_set_step", "dpo_get_flags", "dpo_algorithmic_bytes", "dpo_launch_config",
-           "dpo_last_error", "dpo_destroy", "dpo_grad_norm_noalloc")
+           "dpo_last_error", "dpo_destroy", "dpo_grad_norm_noalloc", "dpo_set_delay")
 
 DPO_NOALLOC_CHUNK_ELEMS = 1 << 20
 DPO_NOALLOC_MAX_CHUNKS = 16384
@@ -78,6 +79,7 @@ def load() -> ctypes.CDLL:
         "dpo_init": (I, [ctypes.POINTER(P), ctypes.POINTER(dpo_tensor), I, I, I, I,
                          ctypes.POINTER(dpo_hparams), I, P]),
         "dpo_stash": (I, [P, P]),
+        "dpo_set_delay": (I, [P, I, P]),
         "dpo_step": (I, [P, F, P]),
         "dpo_read_weights": (I, [P, I, I, ctypes.POINTER(P), ctypes.POINTER(I)]),
         "dpo_get_step": (I, [P, ctypes.POINTER(ctypes.c_int64)]),
@@ -131,6 +133,10 @@ def dpo_init(table: Sequence[dpo_tensor], param_dtype: int, stash_dtype: int, gr
 
 def dpo_stash(ctx, stream=None) -> None:
     _check(load().dpo_stash(ctx, _stream(stream)), ctx)
+
+
+def dpo_set_delay(ctx, delay: int, stream=None) -> None:
+    _check(load().dpo_set_delay(ctx, delay, _stream(stream)), ctx)
 
 
 def dpo_step(ctx, lr: float, stream=None) -> None:
@@ -229,7 +235,8 @@ class DelayedAdamW:
                  weight_decay=0.1, ef=False, ef_lambda=1.0, max_grad_norm=0.0, delay=1,
                  wd_on: Optional[Sequence[bool]] = None, device=None, x0=None,
                  init_mode=DPO_INIT_FRESH, stream=None, host_grad=False, host_param=False,
-                 correction=DPO_CORR_EF):
+                 correction=DPO_CORR_EF, sync: Optional[Sequence[bool]] = None,
+                 keep_stash: Optional[bool] = None):
         import torch
         self.torch = torch
         self.device = torch.device(device or "cuda")
@@ -248,13 +255,15 @@ class DelayedAdamW:
         self.grad = (host_alloc if host_grad else alloc)(tdt[grad_dtype])
         self.param = ((host_alloc if host_param else alloc)(torch.bfloat16)
                       if param_dtype == DPO_BF16 else None)
-        self.stash = alloc(tdt[stash_dtype]) if delay == 1 else None
+        keep_stash = delay == 1 if keep_stash is None else keep_stash
+        self.stash = alloc(tdt[stash_dtype]) if keep_stash else None
         self.ef = alloc(torch.float32) if ef else None
         if x0 is not None:
             self.master.copy_(x0)
         self.hp = dpo_hparams(beta1, beta2, eps, weight_decay, ef_lambda if ef else 0.0,
                               max_grad_norm, delay, correction)
         self.wd_on = list(wd_on) if wd_on is not None else [True] * len(numels)
+        self.sync = list(sync) if sync is not None else [False] * len(numels)
         self.ctx = None
         self._init(init_mode, stream)
 
@@ -262,9 +271,9 @@ class DelayedAdamW:
         table = []
         for i, (cnt, off) in enumerate(zip(self.layout.numels, self.layout.offsets)):
             ptr = lambda t: (t.data_ptr() + off * t.element_size()) if t is not None else None
+            flags = (DPO_WD_ON if self.wd_on[i] else 0) | (DPO_SYNC if self.sync[i] else 0)
             table.append(dpo_tensor(ptr(self.param), ptr(self.master), ptr(self.m), ptr(self.v),
-                                    ptr(self.stash), ptr(self.ef), ptr(self.grad), cnt,
-                                    DPO_WD_ON if self.wd_on[i] else 0))
+                                    ptr(self.stash), ptr(self.ef), ptr(self.grad), cnt, flags))
         self.table = table
         self.ctx = dpo_init(table, self.param_dtype, self.stash_dtype, self.grad_dtype, self.hp,
                             init_mode, stream)
@@ -296,9 +305,15 @@ class DelayedAdamW:
 
     def stale(self, i: int):
         """What the next forward/backward reads (dpo_read_weights(DPO_STALE))."""
-        if self.delay == 1:
+        if self.delay == 1 and not self.sync[i]:
             return self.view(self.stash, i)
         return self.latest(i)
+
+    def set_delay(self, delay: int, stream=None) -> None:
+        """Switch between synchronous and delayed training (dpo_set_delay)."""
+        dpo_set_delay(self.ctx, delay, stream)
+        self.delay = delay
+        self.hp.delay = delay
 
     def latest(self, i: int):
         return self.view(self.param if self.param is not None else self.master, i)

@@ -122,6 +122,8 @@ class Case:
     grad_sigma: float = 1e-3
     init_sigma: float = 0.02
     correction: int = dpo.DPO_CORR_EF   # with ef: EF, SAPipe same / updated state
+    sync: Optional[Sequence[bool]] = None      # per tensor: trained synchronously
+    schedule: Optional[dict] = None            # call k -> delay mode switched to before it
     host_grad: bool = False     # grad arena in pinned host memory
     host_param: bool = False    # bf16 param arena in pinned host memory
 
@@ -141,7 +143,8 @@ class Run:
             ef=case.ef, ef_lambda=case.ef_lambda, max_grad_norm=case.max_grad_norm,
             delay=case.delay, wd_on=case.wd_on, device=device,
             x0=self._dev_x0(device), init_mode=dpo.DPO_INIT_FRESH,
-            host_grad=case.host_grad, host_param=case.host_param, correction=case.correction)
+            host_grad=case.host_grad, host_param=case.host_param, correction=case.correction,
+            sync=case.sync, keep_stash=True)
         # the oracle tracks every element, or only ``sample`` (global indices)
         self.sample = sample
         idx = np.arange(self.N) if sample is None else np.asarray(sample, np.int64)
@@ -161,11 +164,20 @@ class Run:
             if case.wd_on is not None:
                 t_of = np.searchsorted(self.offs, idx, side="right") - 1
                 self._mask = np.array(case.wd_on, bool)[t_of]
+        delayed = None if case.sync is None else [not s_ for s_ in case.sync]
+        if sample is not None and delayed is not None:
+            delayed = [True]
         self.ref = oracle.DelayedOptimizer(
             parts, hp, ef=case.ef, x_store=oracle.F32, stash_store=STORE[case.stash_dtype],
-            param_store=oracle.BF16 if case.param_dtype == dpo.DPO_BF16 else None, wd_on=wd)
+            param_store=oracle.BF16 if case.param_dtype == dpo.DPO_BF16 else None, wd_on=wd,
+            delayed=delayed)
         if sample is not None and case.wd_on is not None:
             self.ref.mask = self._mask.astype(np.uint8)
+        t_of_s = np.searchsorted(self.offs, idx, side="right") - 1
+        self.sync_mask = (np.zeros(idx.size, bool) if case.sync is None
+                          else np.array(case.sync, bool)[t_of_s])
+        if sample is not None and case.sync is not None:
+            self.ref.delay_mask = (~self.sync_mask).astype(np.uint8)
         # arena index of every tracked element
         t_of = np.searchsorted(self.offs, idx, side="right") - 1
         arena_off = np.asarray(self.gpu.layout.offsets, np.int64)
@@ -188,6 +200,9 @@ class Run:
         """Draw gradient k+1 on both sides and take one step on each."""
         c = self.c
         k = self.k + 1
+        if c.schedule and k in c.schedule:
+            self.gpu.set_delay(c.schedule[k])
+            self.ref.set_delay(c.schedule[k])
         for i, n in enumerate(c.numels):
             if n:
                 synth.dev_normal(c.seed, synth.STREAM_GRAD, k, int(self.offs[i]),
@@ -229,16 +244,24 @@ class Run:
                "m": rel_err(self.gather(g.m), r.m),
                "v": rel_err(self.gather(g.v), r.v)}
         if g.ef is not None:
+            # the update history of a synchronously trained tensor stays
+            # untouched (zero on both sides); the metric's floor is taken over
+            # the delayed tensors' history, where it carries values
             e = self.gather(g.ef)
-            out["ef"] = rel_err(e, r.u_prev)
-            out["ef_norm"] = norm_err(e, r.u_prev)
+            keep = ~self.sync_mask
+            out["ef"] = rel_err(e[keep], r.u_prev[keep])
+            out["ef_norm"] = norm_err(e[keep], r.u_prev[keep])
+            if (~keep).any():
+                out["ef_sync_absdiff"] = float(np.max(np.abs(e[~keep] - r.u_prev[~keep])))
         if g.stash is not None:
-            s = self.gather(g.stash)
+            # the stash of a synchronously trained tensor is never read
+            keep = ~self.sync_mask
+            s, rs = self.gather(g.stash)[keep], r.stash[keep]
             if self.c.stash_dtype == dpo.DPO_BF16:
-                out["stash_ulp"] = bf16_ulps(s, r.stash)
-                out["stash_raw_ulp"] = bf16_raw_ulps(s, r.stash)
+                out["stash_ulp"] = bf16_ulps(s, rs)
+                out["stash_raw_ulp"] = bf16_raw_ulps(s, rs)
             else:
-                out["stash"] = rel_err(s, r.stash)
+                out["stash"] = rel_err(s, rs)
         if g.param is not None:
             p = self.gather(g.param)
             out["param_ulp"] = bf16_ulps(p, r.param)
@@ -257,6 +280,8 @@ class Run:
                 continue
             if key in normwise:
                 assert e[key + "_norm"] <= tol, (key, e)
+            elif key.endswith("_absdiff"):
+                assert val == 0.0, (key, e)
             elif key.endswith("_ulp"):
                 assert val <= 1.0, (key, e)
             else:

@@ -313,3 +313,75 @@ def test_sapipe_same_weights_equal_standard_rule_bitwise(cuda_device):
     finally:
         a.close()
         b.close()
+
+
+HALF = [i >= len(RAGGED) // 2 for i in range(len(RAGGED))]   # WPipe: second half synchronous
+
+
+@pytest.mark.parametrize("ef,corr", [(False, dpo.DPO_CORR_EF), (True, dpo.DPO_CORR_EF),
+                                     (True, SP_SAME), (True, SP_UPD)])
+def test_wpipe_half_synchronous_parity(cuda_device, ef, corr):
+    """App. B.2 WPipe: the second half of the model trains synchronously (no
+    stash, no correction), the first half one-step delayed."""
+    run = Run(Case(RAGGED, stash_dtype=B, ef=ef, correction=corr, sync=HALF,
+                   max_grad_norm=0.3), cuda_device)
+    try:
+        for k in range(1, 7):
+            run.step()
+            run.assert_close(TOL_ONE_STEP if k == 1 else TOL_RUN)
+        for i, sy in enumerate(HALF):
+            if RAGGED[i] == 0:
+                continue
+            p, _ = dpo.dpo_read_weights(run.gpu.ctx, dpo.DPO_STALE, i)
+            ref = run.gpu.view(run.gpu.param if sy else run.gpu.stash, i)
+            assert p == ref.data_ptr()
+    finally:
+        run.close()
+
+
+def test_synchronous_lm_head_parity(cuda_device):
+    """App. A.9: the last tensor (the LM head) synchronous, the rest delayed with EF."""
+    sync = [False] * (len(RAGGED) - 1) + [True]
+    run = Run(Case(RAGGED, ef=True, sync=sync), cuda_device)
+    try:
+        for k in range(1, 6):
+            run.step()
+            run.assert_close(TOL_ONE_STEP if k == 1 else TOL_RUN)
+    finally:
+        run.close()
+
+
+@pytest.mark.parametrize("ef,corr", [(True, dpo.DPO_CORR_EF), (True, SP_UPD), (False, 0)])
+def test_synchronous_start_then_delayed(cuda_device, ef, corr):
+    """Sec. 3.1 synchronous start: calls 1-3 synchronous, then delayed; Alg. 1
+    restarts at the switch (standard rule at its first delayed call)."""
+    run = Run(Case(RAGGED, stash_dtype=B, ef=ef, correction=corr, delay=0, schedule={4: 1}),
+              cuda_device)
+    try:
+        for k in range(1, 9):
+            run.step()
+            run.assert_close(TOL_ONE_STEP if k == 1 else TOL_RUN)
+            assert run.gpu.delay == (1 if k >= 4 else 0)
+    finally:
+        run.close()
+
+
+def test_synchronous_cooldown(cuda_device):
+    """App. A.10: delayed with EF for 5 calls, then synchronous."""
+    run = Run(Case(RAGGED, ef=True, schedule={6: 0}), cuda_device)
+    try:
+        for k in range(1, 10):
+            run.step()
+            run.assert_close(TOL_ONE_STEP if k == 1 else TOL_RUN)
+    finally:
+        run.close()
+
+
+def test_set_delay_needs_stash_buffers(cuda_device):
+    opt = dpo.DelayedAdamW([1000, 24], delay=0, keep_stash=False, device=cuda_device)
+    try:
+        with pytest.raises(dpo.DpoError) as e:
+            opt.set_delay(1)
+        assert e.value.code == dpo.DPO_ESTATE
+    finally:
+        opt.close()
