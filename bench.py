@@ -47,6 +47,8 @@ def parse_args(argv=None):
     p.add_argument("--workload", default="llama-7B")
     p.add_argument("--mode", choices=["ef", "std", "sapipe-same", "sapipe-updated"],
                    default="ef")
+    p.add_argument("--wpipe", action="store_true",
+                   help="train the second half of the tensor list synchronously (App. B.2)")
     p.add_argument("--e2e-steps", type=int, default=4)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -166,6 +168,13 @@ MODES = {
 }
 
 
+def wpipe_sync(w, args):
+    """Per-tensor DPO_SYNC flags: the second half of the tensor list under
+    --wpipe (WPipe trains the second half of the model without delay)."""
+    n = len(w.tensors)
+    return [args.wpipe and i >= n // 2 for i in range(n)]
+
+
 # ------------------------------------------------------------ CPU oracle --
 
 def oracle_sample_run(w, mode: str, seconds: float, max_steps: int = 1000, n: int = 1 << 22):
@@ -224,7 +233,7 @@ def run_gpu(args, w, world, rank, local):
                                grad_dtype=w.grad_dtype, lr=w.lr, beta1=w.beta1, beta2=w.beta2,
                                eps=w.eps, weight_decay=w.weight_decay, ef=ef, ef_lambda=1.0,
                                max_grad_norm=w.max_grad_norm, delay=1, device=dev, x0=x0,
-                               stream=stream, correction=corr)
+                               stream=stream, correction=corr, sync=wpipe_sync(w, args))
         del x0
         for i, (o, n) in enumerate(zip(lay.offsets, lay.numels)):
             synth.dev_normal(w.seed, synth.STREAM_GRAD, 1, int(offs[i]), opt.grads(i),
@@ -360,7 +369,8 @@ def main(argv=None):
            "stash_dtype": "bf16" if w.stash_dtype else "f32",
            "grad_dtype": "bf16" if w.grad_dtype else "f32",
            "state": "fp32 master/m/v" + (" + fp32 update-history buffer" if ef else ""),
-           "clip": w.max_grad_norm, "l2": "inputs larger than L2 (no flush needed)"}
+           "clip": w.max_grad_norm, "l2": "inputs larger than L2 (no flush needed)",
+           "wpipe": bool(args.wpipe)}
 
     if args.impl == "reference":
         if rank != 0:
