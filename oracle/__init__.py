@@ -40,7 +40,7 @@ import numpy as np
 from . import build as _build
 
 F64, F32, BF16 = 0, 1, 2
-RULE_ADAMW, RULE_SGD = 0, 1
+RULE_ADAMW, RULE_SGD, RULE_NADAM, RULE_LION, RULE_ADAN = 0, 1, 2, 3, 4
 CORR_EF, CORR_SAPIPE_SAME, CORR_SAPIPE_UPDATED = 0, 1, 2
 STORE_NAMES = {"f64": F64, "f32": F32, "bf16": BF16}
 
@@ -55,6 +55,9 @@ class _HParams(ctypes.Structure):
         ("eps", ctypes.c_double),
         ("weight_decay", ctypes.c_double),
         ("ef_lambda", ctypes.c_double),
+        ("beta3", ctypes.c_double),
+        ("momentum_decay", ctypes.c_double),
+        ("dc_lambda", ctypes.c_double),
         ("delay", ctypes.c_int),
         ("rule", ctypes.c_int),
         ("correction", ctypes.c_int),
@@ -81,7 +84,7 @@ def load(path: Optional[str] = None):
     lib.oracle_step.argtypes = [
         ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, ctypes.POINTER(_HParams), _dp,
         ctypes.c_double, ctypes.POINTER(ctypes.c_uint8), ctypes.POINTER(ctypes.c_uint8),
-        _dp, _dp, _dp, _dp, _dp, _dp]
+        _dp, _dp, _dp, _dp, _dp, _dp, _dp, _dp]
     lib.oracle_sqnorm.restype = ctypes.c_double
     lib.oracle_sqnorm.argtypes = [ctypes.c_int64, _dp]
     lib.oracle_sqnorm_f32.restype = ctypes.c_double
@@ -178,6 +181,9 @@ class HParams:
     delay: int = 1
     rule: int = RULE_ADAMW
     correction: int = CORR_EF
+    beta3: float = 0.99
+    momentum_decay: float = 0.004
+    dc_lambda: float = 0.0
 
     def as_f32(self) -> "HParams":
         """The same settings with every real rounded to fp32: the exact
@@ -185,7 +191,8 @@ class HParams:
         r = lambda v: float(np.float32(v))
         return HParams(r(self.lr), r(self.beta1), r(self.beta2), r(self.eps),
                        r(self.weight_decay), r(self.ef_lambda),
-                       r(self.max_grad_norm), self.delay, self.rule, self.correction)
+                       r(self.max_grad_norm), self.delay, self.rule, self.correction,
+                       r(self.beta3), r(self.momentum_decay), r(self.dc_lambda))
 
 
 class StaleVersionError(AssertionError):
@@ -233,6 +240,9 @@ class DelayedOptimizer:
         self.x = round_to(flat, self.x_store, self.lib)
         self.m = np.zeros(n)
         self.v = np.zeros(n)
+        adan = self.hp.rule == RULE_ADAN
+        self.n3 = np.zeros(n) if adan else None
+        self.g_prev = np.zeros(n) if adan else None
         self.u_prev = np.zeros(n) if self.ef else None
         self.stash = round_to(self.x, self.stash_store, self.lib)
         self.param = (round_to(self.x, self.param_store, self.lib)
@@ -301,14 +311,15 @@ class DelayedOptimizer:
         self.last_clip = clip
         hp = _HParams(lr if lr is not None else self.hp.lr, self.hp.beta1,
                       self.hp.beta2, self.hp.eps, self.hp.weight_decay,
-                      self.hp.ef_lambda, self.delay, self.hp.rule, self.hp.correction,
+                      self.hp.ef_lambda, self.hp.beta3, self.hp.momentum_decay,
+                      self.hp.dc_lambda, self.delay, self.hp.rule, self.hp.correction,
                       self.x_store, self.stash_store,
                       self.param_store if self.param_store is not None else F64)
         rc = self.lib.oracle_step(
             g.size, self.k, max(self.t, 1), ctypes.byref(hp), _ptr(g), clip,
             _ptr(self.mask, ctypes.c_uint8), _ptr(self.delay_mask, ctypes.c_uint8),
             _ptr(self.x), _ptr(self.m), _ptr(self.v), _ptr(self.u_prev), _ptr(self.stash),
-            _ptr(self.param))
+            _ptr(self.param), _ptr(self.n3), _ptr(self.g_prev))
         if rc != 0:
             raise ValueError("oracle_step rejected its arguments")
         if self.delay == 1:

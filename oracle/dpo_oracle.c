@@ -70,11 +70,20 @@ void oracle_round_n(int64_t n, const double *in, double *out, int store)
 int oracle_step(int64_t n, int64_t k, int64_t t, const oracle_hparams *hp,
                 const double *g, double clip_scale, const uint8_t *wd_on,
                 const uint8_t *delay_on, double *x, double *m, double *v,
-                double *u_prev, double *stash, double *param)
+                double *u_prev, double *stash, double *param, double *n3,
+                double *g_prev)
 {
     if (n < 0 || k < 1 || t < 1 || hp == NULL || (n > 0 && (g == NULL || x == NULL)))
         return -1;
-    if (hp->rule == ORACLE_RULE_ADAMW && n > 0 && (m == NULL || v == NULL))
+    const int rule = hp->rule;
+    if (rule < ORACLE_RULE_ADAMW || rule > ORACLE_RULE_ADAN)
+        return -1;
+    if (rule != ORACLE_RULE_SGD && n > 0 && m == NULL)
+        return -1;
+    if ((rule == ORACLE_RULE_ADAMW || rule == ORACLE_RULE_NADAM || rule == ORACLE_RULE_ADAN) &&
+        n > 0 && v == NULL)
+        return -1;
+    if (rule == ORACLE_RULE_ADAN && n > 0 && (n3 == NULL || g_prev == NULL))
         return -1;
     if (hp->delay == 1 && n > 0 && stash == NULL)
         return -1;
@@ -99,20 +108,35 @@ int oracle_step(int64_t n, int64_t k, int64_t t, const oracle_hparams *hp,
     const double bc2 = 1.0 - pow(hp->beta2, (double)k);
     const double bc1_next = 1.0 - pow(hp->beta1, (double)(k + 1));
     const double bc2_next = 1.0 - pow(hp->beta2, (double)(k + 1));
+    const double bc3 = 1.0 - pow(hp->beta3, (double)k);
+
+    /* NAdam's momentum schedule mu_i = beta1 (1 - 0.5 * 0.96^(i psi)) and its
+     * running products up to k and k + 1. */
+    double mu_prod = 1.0;
+    for (int64_t i = 1; i <= k; ++i)
+        mu_prod *= hp->beta1 * (1.0 - 0.5 * pow(0.96, (double)i * hp->momentum_decay));
+    const double mu_k = hp->beta1 * (1.0 - 0.5 * pow(0.96, (double)k * hp->momentum_decay));
+    const double mu_next =
+        hp->beta1 * (1.0 - 0.5 * pow(0.96, (double)(k + 1) * hp->momentum_decay));
+    const double mu_prod_next = mu_prod * mu_next;
 
 #pragma omp parallel for schedule(static)
     for (int64_t i = 0; i < n; ++i) {
-        const double gi = clip_scale * g[i];
         const double wd = (wd_on == NULL || wd_on[i]) ? hp->weight_decay : 0.0;
         const double xt = x[i];
         /* An element of a synchronously trained tensor: no stash, no
          * correction, its history untouched. */
         const int delayed = hp->delay == 1 && (delay_on == NULL || delay_on[i]);
         const int hist_i = use_ef && delayed;
+        double gi = clip_scale * g[i];
+        /* DC-ASGD: first-order Taylor compensation of the stale gradient,
+         * with the stash still holding the weights it was evaluated at. */
+        if (hp->dc_lambda != 0.0 && delayed)
+            gi = gi + hp->dc_lambda * gi * gi * (xt - stash[i]);
 
         /* Update the optimizer statistics with g_{t-1} and form u_{t-1}. */
         double u, mi = 0.0, vi = 0.0;
-        if (hp->rule == ORACLE_RULE_ADAMW) {
+        if (rule == ORACLE_RULE_ADAMW) {
             mi = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;
             vi = hp->beta2 * v[i] + (1.0 - hp->beta2) * gi * gi;
             const double m_hat = mi / bc1;
@@ -120,6 +144,31 @@ int oracle_step(int64_t n, int64_t k, int64_t t, const oracle_hparams *hp,
             u = hp->lr * (m_hat / (sqrt(v_hat) + hp->eps) + wd * xt);
             m[i] = oracle_round(mi, hp->x_store);
             v[i] = oracle_round(vi, hp->x_store);
+        } else if (rule == ORACLE_RULE_NADAM) {
+            mi = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;
+            vi = hp->beta2 * v[i] + (1.0 - hp->beta2) * gi * gi;
+            const double d = sqrt(vi / bc2) + hp->eps;
+            u = hp->lr * ((1.0 - mu_k) / (1.0 - mu_prod) * gi / d +
+                          mu_next / (1.0 - mu_prod_next) * mi / d + wd * xt);
+            m[i] = oracle_round(mi, hp->x_store);
+            v[i] = oracle_round(vi, hp->x_store);
+        } else if (rule == ORACLE_RULE_LION) {
+            const double c = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;
+            const double sgn = c > 0.0 ? 1.0 : (c < 0.0 ? -1.0 : 0.0);
+            u = hp->lr * (sgn + wd * xt);
+            m[i] = oracle_round(hp->beta2 * m[i] + (1.0 - hp->beta2) * gi, hp->x_store);
+        } else if (rule == ORACLE_RULE_ADAN) {
+            const double diff = k == 1 ? 0.0 : gi - g_prev[i];
+            mi = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;
+            vi = hp->beta2 * v[i] + (1.0 - hp->beta2) * diff;
+            const double w = gi + hp->beta2 * diff;
+            const double ni = hp->beta3 * n3[i] + (1.0 - hp->beta3) * w * w;
+            const double d = sqrt(ni / bc3) + hp->eps;
+            u = hp->lr * ((mi / bc1 + hp->beta2 * vi / bc2) / d + wd * xt);
+            m[i] = oracle_round(mi, hp->x_store);
+            v[i] = oracle_round(vi, hp->x_store);
+            n3[i] = oracle_round(ni, hp->x_store);
+            g_prev[i] = oracle_round(gi, hp->x_store);
         } else {
             u = hp->lr * (gi + wd * xt);
         }

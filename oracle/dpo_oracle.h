@@ -38,9 +38,33 @@ extern "C" {
 /* Storage formats of the state buffers. */
 enum { ORACLE_F64 = 0, ORACLE_F32 = 1, ORACLE_BF16 = 2 };
 
-/* Update rules u. ADAMW is the method's optimizer. SGD (u = lr * g) exists
- * only so that tests can check the delay/EF driver of Alg. 1 apart from Adam. */
-enum { ORACLE_RULE_ADAMW = 0, ORACLE_RULE_SGD = 1 };
+/* Update rules u. ADAMW is the optimizer of the hot path. SGD (u = lr g)
+ * exists only so that tests can check the delay/EF driver of Alg. 1 apart
+ * from Adam. NADAM, LION and ADAN are the other elementwise optimizers the
+ * paper benchmarks under one-step delay (Sec. 2.2, Tab. main_results); the
+ * paper cites them without restating them, so each follows its published
+ * form, with decoupled weight decay on the current iterate as for AdamW:
+ *   NADAM  Dozat 2016, as torch.optim.NAdam with decoupled_weight_decay:
+ *          momentum schedule mu_k = beta1 (1 - 0.5 * 0.96^(k psi)),
+ *          u = lr ( (1 - mu_k) / (1 - prod_{i<=k} mu_i) g / d
+ *               + mu_{k+1} / (1 - prod_{i<=k+1} mu_i) m / d + wd x ),
+ *          d = sqrt(v / (1 - beta2^k)) + eps.
+ *   LION   Chen et al. 2023: c = beta1 m + (1 - beta1) g,
+ *          u = lr (sign(c) + wd x), then m = beta2 m + (1 - beta2) g
+ *          (v unused).
+ *   ADAN   Xie et al. 2022, in its authors' distributed form: with
+ *          diff = g - g_prev (0 at the first gradient),
+ *          m = beta1 m + (1 - beta1) g, v = beta2 v + (1 - beta2) diff,
+ *          n = beta3 n + (1 - beta3) (g + beta2 diff)^2,
+ *          u = lr ( (m / (1 - beta1^k) + beta2 v / (1 - beta2^k))
+ *                   / (sqrt(n / (1 - beta3^k)) + eps) + wd x ), g_prev = g. */
+enum {
+    ORACLE_RULE_ADAMW = 0,
+    ORACLE_RULE_SGD = 1,
+    ORACLE_RULE_NADAM = 2,
+    ORACLE_RULE_LION = 3,
+    ORACLE_RULE_ADAN = 4
+};
 
 /* Staleness correction applied when an update-history buffer is given
  * (u_prev != NULL) under delay == 1:
@@ -65,6 +89,9 @@ typedef struct {
     double eps;           /* added to sqrt(v_hat) */
     double weight_decay;  /* decoupled decay coefficient */
     double ef_lambda;     /* lambda of the EF correction; 0 = standard */
+    double beta3;         /* ADAN: EMA coefficient of n */
+    double momentum_decay;/* NADAM: psi of the momentum schedule */
+    double dc_lambda;     /* DC-ASGD compensation strength (Sec. 3.1); 0 = off */
     int delay;            /* 1 = one-step-delayed (Alg. 1), 0 = synchronous */
     int rule;             /* ORACLE_RULE_* */
     int correction;       /* ORACLE_CORR_*, used when u_prev != NULL and delay == 1 */
@@ -86,6 +113,10 @@ typedef struct {
  *              x_1 = x_0, u_{-1} = 0). The EF correction applies from t = 2.
  *   g          the gradient evaluated at the stash (the stale weights), as
  *              doubles holding values of the gradient storage format.
+ *              With dc_lambda != 0 and delay == 1 it is first corrected by
+ *              DC-ASGD's Taylor term (Zheng et al. 2017; Sec. 3.1):
+ *              g~ = g + dc_lambda g^2 (x_t - stash), the stash holding the
+ *              weights the gradient was evaluated at (after clipping).
  *   clip_scale multiplier applied to g (1 when clipping is off), from
  *              oracle_clip_coef().
  *   wd_on      per-element 0/1 mask for weight decay, or NULL (decay on all).
@@ -104,13 +135,16 @@ typedef struct {
  *              or the SAPipe prediction point; may be NULL when delay == 0
  *              (the latest weights are read).
  *   param      receives the new latest weights x_{t+1}, or NULL.
+ *   n, g_prev  ADAN's third moment and previous (corrected) gradient; NULL
+ *              for the other rules.
  *
  * Returns 0, or -1 on an invalid argument.
  */
 int oracle_step(int64_t n, int64_t k, int64_t t, const oracle_hparams *hp,
                 const double *g, double clip_scale, const uint8_t *wd_on,
                 const uint8_t *delay_on, double *x, double *m, double *v,
-                double *u_prev, double *stash, double *param);
+                double *u_prev, double *stash, double *param, double *n3,
+                double *g_prev);
 
 /* Sum of g_i^2 in double over n elements (fixed order: blocks of 65536
  * elements summed left to right, block sums added left to right). */

@@ -31,12 +31,12 @@ MUTANTS = [
     ("no_bias_correction_m", "const double m_hat = mi / bc1;", "const double m_hat = mi;"),
     ("stash_holds_new_weights", "stash[i] = oracle_round(xt, hp->stash_store);",
      "stash[i] = oracle_round(xn, hp->stash_store);"),
-    ("v_from_momentum", "vi = hp->beta2 * v[i] + (1.0 - hp->beta2) * gi * gi",
-     "vi = hp->beta2 * v[i] + (1.0 - hp->beta2) * gi * mi"),
-    ("ema_roles_swapped", "hp->beta1 * m[i] + (1.0 - hp->beta1) * gi",
-     "(1.0 - hp->beta1) * m[i] + hp->beta1 * gi"),
+    ("v_from_momentum", "if (rule == ORACLE_RULE_ADAMW) {\n            mi = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;\n            vi = hp->beta2 * v[i] + (1.0 - hp->beta2) * gi * gi;",
+     "if (rule == ORACLE_RULE_ADAMW) {\n            mi = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;\n            vi = hp->beta2 * v[i] + (1.0 - hp->beta2) * gi * mi;"),
+    ("ema_roles_swapped", "if (rule == ORACLE_RULE_ADAMW) {\n            mi = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;\n            vi = hp->beta2 * v[i] + (1.0 - hp->beta2) * gi * gi;",
+     "if (rule == ORACLE_RULE_ADAMW) {\n            mi = (1.0 - hp->beta1) * m[i] + hp->beta1 * gi;\n            vi = hp->beta2 * v[i] + (1.0 - hp->beta2) * gi * gi;"),
     ("ef_stores_displacement", "double hist = u;", "double hist = xt - xn;"),
-    ("clip_not_applied", "const double gi = clip_scale * g[i];", "const double gi = g[i];"),
+    ("clip_not_applied", "double gi = clip_scale * g[i];", "double gi = g[i];"),
     ("clip_no_epsilon", "(sqrt(sqnorm) + 1e-6)", "sqrt(sqnorm)"),
     ("bf16_ties_away", "q = nearbyint(q);", "q = round(q);"),
     ("bf16_subnormal_quantum", "if (e < -125)\n        e = -125;", "if (e < -126)\n        e = -126;"),
@@ -51,6 +51,13 @@ MUTANTS = [
     ("delay_mask_ignored", "(delay_on == NULL || delay_on[i])", "(1)"),
     ("ef_restart_counts_all_steps", "corr == ORACLE_CORR_EF && t >= 2",
      "corr == ORACLE_CORR_EF && k >= 2"),
+    ("nadam_next_mu_index", "pow(0.96, (double)(k + 1) * hp->momentum_decay)",
+     "pow(0.96, (double)k * hp->momentum_decay)"),
+    ("lion_roles_swapped", "oracle_round(hp->beta2 * m[i] + (1.0 - hp->beta2) * gi, hp->x_store)",
+     "oracle_round(hp->beta1 * m[i] + (1.0 - hp->beta1) * gi, hp->x_store)"),
+    ("adan_diff_sign", "gi - g_prev[i]", "g_prev[i] - gi"),
+    ("adan_no_lookahead", "gi + hp->beta2 * diff", "gi"),
+    ("dc_sign", "(xt - stash[i])", "(stash[i] - xt)"),
 ]
 
 

@@ -657,3 +657,142 @@ def test_per_tensor_delay_is_elementwise(lib):
     assert np.array_equal(mixed.tensor("stash", 0), all_d.tensor("stash", 0))
     assert np.array_equal(mixed.tensor("u_prev", 2), all_d.tensor("u_prev", 2))
     assert np.array_equal(mixed.tensor("u_prev", 1), np.zeros(7))   # history untouched
+
+
+# ------------------- other elementwise optimizers under delay (Tab. main_results)
+
+@pytest.fixture
+def f64_default():
+    """torch keeps NAdam's running product of mu in the default scalar dtype:
+    make it fp64 for the duration of a test."""
+    prev = torch.get_default_dtype()
+    torch.set_default_dtype(torch.float64)
+    try:
+        yield
+    finally:
+        torch.set_default_dtype(prev)
+
+
+@pytest.mark.parametrize("delay", [0, 1])
+@pytest.mark.parametrize("psi", [0.004, 0.02])
+def test_nadam_matches_torch(lib, f64_default, delay, psi):
+    """NAdam = torch.optim.NAdam with decoupled weight decay, including its
+    momentum schedule mu_k = beta1 (1 - 0.5 * 0.96^(k psi)), changing lr."""
+    rng = np.random.default_rng(12)
+    shapes = [(4, 3), (5,)]
+    x0s = [rng.normal(0, 0.5, s) for s in shapes]
+    grads = [[rng.normal(0, 0.7, s) for s in shapes] for _ in range(10)]
+    lrs = [2e-2 * (1 + 0.05 * i) for i in range(10)]
+    ps = [torch.nn.Parameter(torch.tensor(x)) for x in x0s]
+    opt = torch.optim.NAdam(ps, lr=lrs[0], betas=(0.9, 0.95), eps=1e-8, weight_decay=0.1,
+                            momentum_decay=psi, decoupled_weight_decay=True, foreach=False)
+    hp = HParams(lr=lrs[0], weight_decay=0.1, delay=delay, rule=oracle.RULE_NADAM,
+                 momentum_decay=psi)
+    o = oracle.DelayedOptimizer(x0s, hp, x_store=F64, stash_store=F64, lib=lib)
+    for gs, lr in zip(grads, lrs):
+        for p, g in zip(ps, gs):
+            p.grad = torch.tensor(g)
+        for group in opt.param_groups:
+            group["lr"] = lr
+        opt.step()
+        o.step(np.concatenate([g.ravel() for g in gs]), lr=lr)
+        ref = np.concatenate([p.detach().numpy().ravel() for p in ps])
+        assert _rel(o.x, ref) < 1e-12
+
+
+def test_lion_hand_steps(lib):
+    """Lion, beta = (0.9, 0.99), lr = 0.1, wd = 0, gradients 2, -1, 0.05:
+    c1 = 0.1*2 = 0.2 (+), m1 = 0.01*2 = 0.02;
+    c2 = 0.9*0.02 + 0.1*(-1) = -0.082 (-), m2 = 0.99*0.02 + 0.01*(-1) = 0.0098;
+    c3 = 0.9*0.0098 + 0.1*0.05 = 0.01382 (+). With the coefficients' roles
+    swapped the second step would move up, not down."""
+    hp = HParams(lr=0.1, beta1=0.9, beta2=0.99, weight_decay=0.0, rule=oracle.RULE_LION)
+    o = oracle.DelayedOptimizer([np.array([1.0])], hp, x_store=F64, stash_store=F64, lib=lib)
+    xs = []
+    for g in (2.0, -1.0, 0.05):
+        o.step(np.array([g]), tag=o.read_weights()[1])
+        xs.append(o.x[0])
+    assert xs == pytest.approx([0.9, 1.0, 0.9], abs=1e-15)
+    assert o.m[0] == pytest.approx(0.99 * 0.0098 + 0.01 * 0.05, rel=1e-14)
+
+
+def test_lion_moves_every_weight_by_exactly_lr(lib):
+    """A sign update: |x_{t+1} - (1 - lr wd) x_t| = lr for every element
+    whose interpolation c is non-zero, whatever the gradient scale."""
+    rng = np.random.default_rng(13)
+    x0 = rng.normal(0, 1, 200)
+    hp = HParams(lr=3e-3, beta1=0.9, beta2=0.99, weight_decay=0.5, rule=oracle.RULE_LION)
+    o = oracle.DelayedOptimizer([x0], hp, x_store=F64, stash_store=F64, lib=lib)
+    for s in (1e-6, 1.0, 1e3):
+        x = o.x.copy()
+        o.step(rng.normal(0, s, 200))
+        np.testing.assert_allclose(np.abs(o.x - (1 - 3e-3 * 0.5) * x), 3e-3, rtol=1e-12)
+
+
+def test_adan_first_step_is_adams(lib):
+    """At the first gradient diff = 0 and the bias-corrected moments are g and
+    g^2: Adan's update is Adam's first step lr (g / (|g| + eps) + wd x)."""
+    rng = np.random.default_rng(14)
+    x0, g = rng.normal(0, 1, 50), rng.normal(0, 1, 50)
+    hp = HParams(lr=0.01, beta1=0.98, beta2=0.92, beta3=0.99, eps=1e-8, weight_decay=0.1,
+                 rule=oracle.RULE_ADAN)
+    o = oracle.DelayedOptimizer([x0], hp, x_store=F64, stash_store=F64, lib=lib)
+    o.step(g)
+    np.testing.assert_allclose(o.x, x0 - 0.01 * (g / (np.abs(g) + 1e-8) + 0.1 * x0), rtol=1e-13)
+
+
+def test_adan_constant_gradient_closed_form(lib):
+    """Constant gradient c: diff = 0, so u = lr (c / (|c| + eps) + wd x) and
+    x_n - x* = (x_0 - x*) (1 - lr wd)^n with x* = -c / ((|c| + eps) wd)."""
+    lr, wd, eps, c, x0 = 0.05, 0.4, 1e-8, -0.7, 1.5
+    xstar = -(c / (abs(c) + eps)) / wd
+    hp = HParams(lr=lr, beta1=0.98, beta2=0.92, beta3=0.99, eps=eps, weight_decay=wd,
+                 rule=oracle.RULE_ADAN)
+    o = oracle.DelayedOptimizer([np.array([x0])], hp, x_store=F64, stash_store=F64, lib=lib)
+    for j in range(1, 40):
+        o.step(np.array([c]))
+        assert o.x[0] - xstar == pytest.approx((x0 - xstar) * (1 - lr * wd) ** j, rel=1e-10)
+
+
+def test_adan_hand_steps(lib):
+    """beta = (0.98, 0.92, 0.99), eps = 0, wd = 0, lr = 0.1, gradients 2, 1.
+    Step 1: u = 0.1 (Adam's first step). Step 2: diff = -1, m = 0.0592,
+    v = -0.08, w = 1 - 0.92 = 0.08, n = 0.99*0.04 + 0.01*0.0064 = 0.039664;
+    u = 0.1 (0.0592/0.0396 - 0.92*0.08/0.1536) / sqrt(0.039664/0.0199)."""
+    hp = HParams(lr=0.1, beta1=0.98, beta2=0.92, beta3=0.99, eps=0.0, weight_decay=0.0,
+                 rule=oracle.RULE_ADAN)
+    o = oracle.DelayedOptimizer([np.array([1.0])], hp, x_store=F64, stash_store=F64, lib=lib)
+    o.step(np.array([2.0]), tag=o.read_weights()[1])
+    assert o.x[0] == pytest.approx(0.9, rel=1e-14)
+    o.step(np.array([1.0]), tag=o.read_weights()[1])
+    u2 = 0.1 * (0.0592 / 0.0396 - 0.92 * 0.08 / 0.1536) / math.sqrt(0.039664 / 0.0199)
+    assert o.x[0] == pytest.approx(0.9 - u2, rel=1e-13)
+    assert o.v[0] == pytest.approx(-0.08, rel=1e-14)
+    assert o.n3[0] == pytest.approx(0.039664, rel=1e-14)
+
+
+def test_dc_asgd_compensation(lib):
+    """DC-ASGD (Sec. 3.1): g~ = g + lambda g^2 (x_t - x_stale), the stale
+    weights being the stash the gradient came from. With beta1 = 0 the first
+    moment is exactly g~. At the first call the stash equals x_t (no
+    correction); lambda = 0 is the plain rule bitwise."""
+    lam = 50.0
+    hp = HParams(lr=0.1, beta1=0.0, beta2=0.95, eps=1e-8, weight_decay=0.0, dc_lambda=lam)
+    o = oracle.DelayedOptimizer([np.array([1.0])], hp, x_store=F64, stash_store=F64, lib=lib)
+    o.step(np.array([2.0]), tag=o.read_weights()[1])
+    assert o.m[0] == 2.0
+    x2, x1 = o.x[0], o.stash[0]
+    o.step(np.array([1.0]), tag=o.read_weights()[1])
+    assert o.m[0] == pytest.approx(1.0 + lam * 1.0 * (x2 - x1), rel=1e-14)
+    assert x1 == 1.0 and x2 < 1.0
+    # lambda = 0: identical to the plain rule
+    rng = np.random.default_rng(15)
+    x0, grads = rng.normal(0, 1, 30), [rng.normal(0, 1, 30) for _ in range(5)]
+    runs = []
+    for dl in (0.0, None):
+        o = oracle.DelayedOptimizer([x0], HParams(lr=0.01, dc_lambda=dl or 0.0), x_store=F32,
+                                    stash_store=F32, lib=lib)
+        for g in grads:
+            o.step(g)
+        runs.append(o.x.copy())
+    assert np.array_equal(runs[0], runs[1])
