@@ -47,6 +47,9 @@ def parse_args(argv=None):
     p.add_argument("--workload", default="llama-7B")
     p.add_argument("--mode", choices=["ef", "std", "sapipe-same", "sapipe-updated"],
                    default="ef")
+    p.add_argument("--optimizer", choices=["adamw", "nadam", "lion", "adan"], default="adamw")
+    p.add_argument("--dc-lambda", type=float, default=0.0,
+                   help="DC-ASGD compensation strength (Sec. 3.1); 0: off")
     p.add_argument("--wpipe", action="store_true",
                    help="train the second half of the tensor list synchronously (App. B.2)")
     p.add_argument("--e2e-steps", type=int, default=4)
@@ -93,11 +96,23 @@ def measured_hbm_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+def kernel_source_sha() -> str:
+    """First 16 hex digits of the sha256 over the device sources (every .cu
+    and .cuh under csrc/, in name order): a summary taken on other sources
+    describes another kernel."""
+    csrc = os.path.join(ROOT, "paper_2606_30634_gb300", "csrc")
+    h = hashlib.sha256()
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh")):
+            h.update(name.encode() + b"\0")
+            h.update(open(os.path.join(csrc, name), "rb").read())
+    return h.hexdigest()[:16]
+
+
 def committed_traffic(kernel_tag: str):
     """dram bytes per parameter from the committed ncu summary of the fused
     kernel, if that summary was taken on the kernel source as it is now."""
-    src = os.path.join(ROOT, "paper_2606_30634_gb300", "csrc", "dpo_kernels.cu")
-    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    sha = kernel_source_sha()
     for name in sorted(os.listdir(os.path.join(ROOT, "profiles"))) if os.path.isdir(
             os.path.join(ROOT, "profiles")) else []:
         if not name.endswith(".md"):
@@ -168,6 +183,19 @@ MODES = {
 }
 
 
+def rule_settings(args) -> dict:
+    """Update rule and its settings (the paper's where it gives them: Lion
+    lr 5e-4, wd 0.5, App. E.1; Adan's usual betas)."""
+    from paper_2606_30634_gb300 import dpo
+    base = {"adamw": dict(optimizer=dpo.DPO_OPT_ADAMW),
+            "nadam": dict(optimizer=dpo.DPO_OPT_NADAM, momentum_decay=0.004),
+            "lion": dict(optimizer=dpo.DPO_OPT_LION, beta1=0.9, beta2=0.99, lr=5e-4,
+                         weight_decay=0.5),
+            "adan": dict(optimizer=dpo.DPO_OPT_ADAN, beta1=0.98, beta2=0.92, beta3=0.99),
+            }[args.optimizer]
+    return dict(base, dc_lambda=args.dc_lambda)
+
+
 def wpipe_sync(w, args):
     """Per-tensor DPO_SYNC flags: the second half of the tensor list under
     --wpipe (WPipe trains the second half of the model without delay)."""
@@ -177,7 +205,8 @@ def wpipe_sync(w, args):
 
 # ------------------------------------------------------------ CPU oracle --
 
-def oracle_sample_run(w, mode: str, seconds: float, max_steps: int = 1000, n: int = 1 << 22):
+def oracle_sample_run(w, mode: str, seconds: float, max_steps: int = 1000, n: int = 1 << 22,
+                      rule: dict = None):
     """Time the oracle as it stands on the first n parameters of the set
     (input draws excluded from the timing). Returns (params/s, cores, steps,
     n)."""
@@ -191,9 +220,14 @@ def oracle_sample_run(w, mode: str, seconds: float, max_steps: int = 1000, n: in
     STORE = {0: oracle.F32, 1: oracle.BF16}
     ef, corr, _ = MODES[mode]
     x0 = synth.host_normal(w.seed, synth.STREAM_INIT, 0, 0, n, W.INIT_SIGMA).astype(np.float64)
-    hp = oracle.HParams(lr=w.lr, weight_decay=w.weight_decay,
-                        ef_lambda=1.0 if ef and corr == 0 else 0.0,
-                        max_grad_norm=w.max_grad_norm, correction=corr).as_f32()
+    rule = dict(rule or {})
+    opt = rule.pop("optimizer", 0)
+    rule.setdefault("lr", w.lr)
+    rule.setdefault("weight_decay", w.weight_decay)
+    hp = oracle.HParams(ef_lambda=1.0 if ef and corr == 0 else 0.0,
+                        max_grad_norm=w.max_grad_norm, correction=corr,
+                        rule={0: oracle.RULE_ADAMW, 1: oracle.RULE_NADAM, 2: oracle.RULE_LION,
+                              3: oracle.RULE_ADAN}[opt], **rule).as_f32()
     o = oracle.DelayedOptimizer([x0], hp, ef=ef, x_store=oracle.F32,
                                 stash_store=STORE[w.stash_dtype],
                                 param_store=oracle.BF16 if w.param_dtype == 1 else None)
@@ -229,11 +263,13 @@ def run_gpu(args, w, world, rank, local):
         x0 = torch.empty(lay.total, dtype=torch.float32, device=dev)
         for i, (o, n) in enumerate(zip(lay.offsets, lay.numels)):
             synth.dev_normal(w.seed, synth.STREAM_INIT, 0, int(offs[i]), x0[o:o + n], W.INIT_SIGMA)
+        kw = dict(lr=w.lr, beta1=w.beta1, beta2=w.beta2, eps=w.eps,
+                  weight_decay=w.weight_decay)
+        kw.update(rule_settings(args))
         opt = dpo.DelayedAdamW(w.numels, param_dtype=w.param_dtype, stash_dtype=w.stash_dtype,
-                               grad_dtype=w.grad_dtype, lr=w.lr, beta1=w.beta1, beta2=w.beta2,
-                               eps=w.eps, weight_decay=w.weight_decay, ef=ef, ef_lambda=1.0,
+                               grad_dtype=w.grad_dtype, ef=ef, ef_lambda=1.0,
                                max_grad_norm=w.max_grad_norm, delay=1, device=dev, x0=x0,
-                               stream=stream, correction=corr, sync=wpipe_sync(w, args))
+                               stream=stream, correction=corr, sync=wpipe_sync(w, args), **kw)
         del x0
         for i, (o, n) in enumerate(zip(lay.offsets, lay.numels)):
             synth.dev_normal(w.seed, synth.STREAM_GRAD, 1, int(offs[i]), opt.grads(i),
@@ -370,13 +406,15 @@ def main(argv=None):
            "grad_dtype": "bf16" if w.grad_dtype else "f32",
            "state": "fp32 master/m/v" + (" + fp32 update-history buffer" if ef else ""),
            "clip": w.max_grad_norm, "l2": "inputs larger than L2 (no flush needed)",
-           "wpipe": bool(args.wpipe)}
+           "wpipe": bool(args.wpipe), "optimizer": args.optimizer,
+           "dc_lambda": args.dc_lambda}
 
     if args.impl == "reference":
         if rank != 0:
             return 0
         v, cores, steps, n = oracle_sample_run(w, args.mode, args.cpu_seconds,
-                                               max_steps=max(1, args.steps + args.warmup))
+                                               max_steps=max(1, args.steps + args.warmup),
+                                               rule=rule_settings(args))
         sample = f"first {n} params of the set, {steps} oracle steps (plain C, fp64)"
         line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT,
                 "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
@@ -409,7 +447,8 @@ def main(argv=None):
             "frac_of_nominal": r["achieved"] / 8000.0}
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        v, cores, steps, n = oracle_sample_run(w, args.mode, args.cpu_seconds)
+        v, cores, steps, n = oracle_sample_run(w, args.mode, args.cpu_seconds,
+                                               rule=rule_settings(args))
         cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
                "sample": f"first {n} params of the set, {steps} oracle steps (plain C, fp64)"}
     if world > 1:

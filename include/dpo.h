@@ -106,6 +106,29 @@ typedef enum { DPO_F32 = 0, DPO_BF16 = 1 } dpo_dtype;
 #define DPO_CORR_SAPIPE_SAME 1
 #define DPO_CORR_SAPIPE_UPDATED 2
 
+/* dpo_hparams.optimizer: the update rule u. AdamW is the hot path's; the
+ * others are the elementwise optimizers the paper also benchmarks under
+ * one-step delay (Sec. 2.2, Tab. main_results), in their published forms with
+ * decoupled weight decay on x_t:
+ *   DPO_OPT_ADAMW  as above.
+ *   DPO_OPT_NADAM  Dozat 2016 (as torch.optim.NAdam, decoupled decay):
+ *                  mu_k = beta1 (1 - 0.5 * 0.96^(k momentum_decay)),
+ *                  u = lr ((1-mu_k)/(1-prod_{i<=k} mu_i) g/d
+ *                      + mu_{k+1}/(1-prod_{i<=k+1} mu_i) m/d + wd x_t),
+ *                  d = sqrt(v / (1 - beta2^k)) + eps.
+ *   DPO_OPT_LION   Chen et al. 2023: u = lr (sign(beta1 m + (1-beta1) g) + wd x_t),
+ *                  m = beta2 m + (1 - beta2) g; v is not used (may be NULL).
+ *   DPO_OPT_ADAN   Xie et al. 2022 (its authors' distributed form): diff = g - g_prev
+ *                  (0 at the first gradient), m = beta1 m + (1-beta1) g,
+ *                  v = beta2 v + (1-beta2) diff, n = beta3 n + (1-beta3)(g + beta2 diff)^2,
+ *                  u = lr ((m/(1-beta1^k) + beta2 v/(1-beta2^k)) / (sqrt(n/(1-beta3^k)) + eps)
+ *                      + wd x_t); needs the n and grad_prev buffers.
+ * DPO_CORR_SAPIPE_UPDATED is defined for AdamW only. */
+#define DPO_OPT_ADAMW 0
+#define DPO_OPT_NADAM 1
+#define DPO_OPT_LION 2
+#define DPO_OPT_ADAN 3
+
 typedef struct {
     float beta1;          /* first-moment EMA coefficient, [0, 1) */
     float beta2;          /* second-moment EMA coefficient, [0, 1) */
@@ -115,6 +138,13 @@ typedef struct {
     float max_grad_norm;  /* > 0: global-norm clipping threshold; <= 0: off */
     int delay;            /* 1: one-step-delayed with stash; 0: synchronous */
     int correction;       /* DPO_CORR_* (tables with EF buffers, delay == 1) */
+    int optimizer;        /* DPO_OPT_* */
+    float beta3;          /* DPO_OPT_ADAN: EMA coefficient of n, [0, 1) */
+    float momentum_decay; /* DPO_OPT_NADAM: psi of the momentum schedule, >= 0 */
+    /* DC-ASGD (Sec. 3.1): when != 0, delayed tensors' gradients are first
+     * compensated, g~ = g + dc_lambda g^2 (x_t - stash), the stash holding the
+     * weights the gradient was evaluated at (after clipping). */
+    float dc_lambda;
 } dpo_hparams;
 
 typedef struct {
@@ -124,7 +154,8 @@ typedef struct {
     void *param;
     float *master;     /* fp32 master weights, read and written */
     float *m;          /* Adam first moment, fp32, read and written */
-    float *v;          /* Adam second moment, fp32, read and written */
+    float *v;          /* second moment, fp32, read and written (Adan: the averaged
+                        * gradient difference; Lion: unused, may be NULL) */
     /* Stale weights in the stash dtype: x_t after each step (the SAPipe
      * prediction point under those corrections). Required for tensors without
      * DPO_SYNC when delay == 1; with delay == 0 it may be NULL, and giving it
@@ -138,6 +169,8 @@ typedef struct {
     /* The gradient the step consumes, in the grad dtype, evaluated at the
      * stash (delay == 1) or at the latest weights (delay == 0). Read only. */
     const void *grad;
+    float *n;          /* DPO_OPT_ADAN: third moment (fp32), else NULL */
+    float *grad_prev;  /* DPO_OPT_ADAN: previous corrected gradient (fp32), else NULL */
     int64_t numel;     /* elements, >= 0; 0 is allowed and skipped */
     uint32_t flags;    /* DPO_WD_ON or 0 */
 } dpo_tensor;

@@ -29,10 +29,13 @@ COMMON = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O3,-fop
 
 LIBS = {
     "libdpo.so": {
-        "sources": ["csrc/dpo_kernels.cu", "csrc/dpo_abi.cpp", "csrc/dpo_noalloc.cu"],
-        "headers": ["csrc/dpo_internal.h", "../include/dpo.h"],
+        "sources": ["csrc/dpo_kernels.cu", "csrc/dpo_step_adamw.cu", "csrc/dpo_step_nadam.cu",
+                    "csrc/dpo_step_lion.cu", "csrc/dpo_step_adan.cu", "csrc/dpo_abi.cpp",
+                    "csrc/dpo_noalloc.cu"],
+        "headers": ["csrc/dpo_internal.h", "csrc/dpo_device.cuh", "csrc/dpo_step.cuh",
+                    "../include/dpo.h"],
         "includes": ["csrc"],
-        "ptxas_v": ["csrc/dpo_kernels.cu"],
+        "ptxas_v": ["csrc/dpo_step_adamw.cu"],
     },
     "libdpo_synth.so": {
         "sources": ["synth/synth.cu"],

@@ -33,6 +33,7 @@ struct dpo_ctx {
     bool can_delay = false; // every tensor without DPO_SYNC has one
     int64_t k = 0;
     int64_t phase_k0 = 0;   // k when the current delayed phase began
+    double mu_prod = 1.0;   // NAdam: prod_{i<=k} mu_i
     int64_t total_pkts = 0;
     int64_t total_elems = 0;
     std::vector<dpo_tensor> table;
@@ -72,6 +73,26 @@ int cuda_fail(dpo_ctx *c, cudaError_t e, const char *what)
 
 bool valid_dtype(int d) { return d == DPO_F32 || d == DPO_BF16; }
 int64_t dt_size(dpo_dtype d) { return d == DPO_BF16 ? 2 : 4; }
+
+// NAdam's momentum schedule mu_i = beta1 (1 - 0.5 * 0.96^(i psi)).
+double nadam_mu(const dpo_hparams &hp, int64_t i)
+{
+    return (double)hp.beta1 * (1.0 - 0.5 * std::pow(0.96, (double)i * (double)hp.momentum_decay));
+}
+
+// fp32 state streams of a rule besides master: m, v (not Lion), n and
+// grad_prev (Adan).
+int rule_state_streams(int opt)
+{
+    switch (opt) {
+    case DPO_OPT_LION:
+        return 1;
+    case DPO_OPT_ADAN:
+        return 4;
+    default:
+        return 2;
+    }
+}
 bool aligned(const void *p) { return (reinterpret_cast<uintptr_t>(p) % dpo::kAlign) == 0; }
 // Stash kind of the fused step: none while the run is synchronous.
 StashKind stash_kind(const dpo_ctx *c)
@@ -127,12 +148,18 @@ int set_step_grid(dpo_ctx *c)
 {
     const dpo::Correction corr = correction_kind(c->ef, c->hp);
     int per_sm = 0;
-    const cudaError_t e = dpo::step_ctas_per_sm(c->param_dt == DPO_BF16, stash_kind(c),
-                                                c->grad_dt == DPO_BF16, corr, &per_sm);
+    const cudaError_t e = dpo::step_ctas_per_sm(
+        static_cast<dpo::Optimizer>(c->hp.optimizer), c->param_dt == DPO_BF16, stash_kind(c),
+        c->grad_dt == DPO_BF16, corr, &per_sm);
     if (e != cudaSuccess)
         return cuda_fail(c, e, "occupancy query");
+    // bytes loaded per packet: master, the rule's state, grad, the history
+    // buffer under a correction, the stash under DC-ASGD
+    const bool delayed = c->hp.delay == 1;
     const int64_t load_bytes =
-        dpo::kPacket * (12 + dt_size(c->grad_dt) + (corr != dpo::kCorrNone ? 4 : 0));
+        dpo::kPacket * (4 + 4 * rule_state_streams(c->hp.optimizer) + dt_size(c->grad_dt) +
+                        (corr != dpo::kCorrNone ? 4 : 0) +
+                        (delayed && c->hp.dc_lambda != 0.0f ? dt_size(c->stash_dt) : 0));
     int want = std::max<int>(1, (int)((dpo::kStepInflightPerSm + load_bytes * dpo::kStepThreads / 2) /
                                       (load_bytes * dpo::kStepThreads)));
     // The SAPipe updated-state prediction evaluates AdamW twice per element,
@@ -183,6 +210,17 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
     if (hp->correction != DPO_CORR_EF && hp->correction != DPO_CORR_SAPIPE_SAME &&
         hp->correction != DPO_CORR_SAPIPE_UPDATED)
         return fail(nullptr, DPO_EINVAL, "correction must be one of DPO_CORR_*");
+    if (hp->optimizer < DPO_OPT_ADAMW || hp->optimizer > DPO_OPT_ADAN)
+        return fail(nullptr, DPO_EINVAL, "optimizer must be one of DPO_OPT_*");
+    if (!std::isfinite(hp->beta3) || !std::isfinite(hp->momentum_decay) ||
+        !std::isfinite(hp->dc_lambda))
+        return fail(nullptr, DPO_EINVAL, "hyperparameters must be finite");
+    if (hp->optimizer == DPO_OPT_ADAN && !(hp->beta3 >= 0.0f && hp->beta3 < 1.0f))
+        return fail(nullptr, DPO_EINVAL, "beta3 must lie in [0, 1)");
+    if (hp->optimizer == DPO_OPT_NADAM && hp->momentum_decay < 0.0f)
+        return fail(nullptr, DPO_EINVAL, "momentum_decay must be >= 0");
+    if (hp->correction == DPO_CORR_SAPIPE_UPDATED && hp->optimizer != DPO_OPT_ADAMW)
+        return fail(nullptr, DPO_EINVAL, "the SAPipe updated-state prediction is defined for AdamW");
 
     // Table: NULL pointers, EF consistency, alignment, overlaps.
     const bool ef = table[0].ef != nullptr;
@@ -200,8 +238,11 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
             return fail(nullptr, DPO_EINVAL, "tensor %d: unknown flags 0x%x", t, d.flags);
         if (d.numel == 0)
             continue;
-        if (d.master == nullptr || d.m == nullptr || d.v == nullptr || d.grad == nullptr)
+        if (d.master == nullptr || d.m == nullptr || d.grad == nullptr ||
+            (d.v == nullptr && hp->optimizer != DPO_OPT_LION))
             return fail(nullptr, DPO_EINVAL, "tensor %d: master, m, v and grad are required", t);
+        if (hp->optimizer == DPO_OPT_ADAN && (d.n == nullptr || d.grad_prev == nullptr))
+            return fail(nullptr, DPO_EINVAL, "tensor %d: Adan needs the n and grad_prev buffers", t);
         if (hp->delay == 1 && d.stash == nullptr && !(d.flags & DPO_SYNC))
             return fail(nullptr, DPO_EINVAL, "tensor %d: delay = 1 needs a stash buffer", t);
         if (d.stash != nullptr)
@@ -222,7 +263,10 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
         } bufs[] = {
             {d.master, 4 * d.numel, "master", false},
             {d.m, 4 * d.numel, "m", false},
-            {d.v, 4 * d.numel, "v", false},
+            {hp->optimizer == DPO_OPT_LION ? nullptr : d.v, 4 * d.numel, "v", false},
+            {hp->optimizer == DPO_OPT_ADAN ? d.n : nullptr, 4 * d.numel, "n", false},
+            {hp->optimizer == DPO_OPT_ADAN ? d.grad_prev : nullptr, 4 * d.numel, "grad_prev",
+             false},
             {d.grad, dt_size(grad_dtype) * d.numel, "grad", true},
             {d.param, dt_size(param_dtype) * d.numel, "param", true},
             {d.stash, dt_size(stash_dtype) * d.numel, "stash", false},
@@ -353,6 +397,9 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
         x.stash = d.stash;
         x.ef = d.ef;
         x.grad = d.grad;
+        x.v = hp->optimizer == DPO_OPT_LION ? nullptr : d.v;
+        x.n = hp->optimizer == DPO_OPT_ADAN ? d.n : nullptr;
+        x.grad_prev = hp->optimizer == DPO_OPT_ADAN ? d.grad_prev : nullptr;
         x.numel = d.numel;
         x.flags = d.flags;
         x.pad_ = 0;
@@ -447,7 +494,7 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
             if (e != cudaSuccess)
                 return cuda_fail(c, e, "gradient-norm launch");
         }
-        const double b1 = c->hp.beta1, b2 = c->hp.beta2, lrd = lr;
+        const double b1 = c->hp.beta1, b2 = c->hp.beta2, b3 = c->hp.beta3, lrd = lr;
         const double bc1 = 1.0 - std::pow(b1, (double)k);
         const double bc2 = 1.0 - std::pow(b2, (double)k);
         const dpo::Correction corr = correction_kind(c->ef, c->hp);
@@ -468,12 +515,25 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
         a.lam = (corr == dpo::kCorrEF && t >= 2) ? c->hp.ef_lambda : 0.0f;
         a.step_size_next = (float)(lrd / (1.0 - std::pow(b1, (double)(k + 1))));
         a.inv_sqrt_bc2_next = (float)(1.0 / std::sqrt(1.0 - std::pow(b2, (double)(k + 1))));
+        a.lr = lr;
+        const double mu_k = nadam_mu(c->hp, k), mu_next = nadam_mu(c->hp, k + 1);
+        const double mu_prod = c->mu_prod * mu_k;
+        a.nadam_cg = (float)(lrd * (1.0 - mu_k) / (1.0 - mu_prod));
+        a.nadam_cm = (float)(lrd * mu_next / (1.0 - mu_prod * mu_next));
+        a.beta3 = c->hp.beta3;
+        a.omb3 = (float)(1.0 - b3);
+        a.inv_sqrt_bc3 = (float)(1.0 / std::sqrt(1.0 - std::pow(b3, (double)k)));
+        a.adan_c2 = (float)(lrd * b2 / bc2);
+        a.first = k == 1;
+        a.dc_lambda = c->hp.delay == 1 ? c->hp.dc_lambda : 0.0f;
         a.clip = c->clip ? &c->d_scalars->clip : nullptr;
-        const cudaError_t e = dpo::launch_step(c->param_dt == DPO_BF16, stash_kind(c),
+        const cudaError_t e = dpo::launch_step(static_cast<dpo::Optimizer>(c->hp.optimizer),
+                                               c->param_dt == DPO_BF16, stash_kind(c),
                                                c->grad_dt == DPO_BF16, corr, c->step_grid, a, s);
         if (e != cudaSuccess)
             return cuda_fail(c, e, "fused step launch");
     }
+    c->mu_prod *= nadam_mu(c->hp, k);
     c->k = k;
     return DPO_OK;
 }
@@ -517,6 +577,9 @@ extern "C" int dpo_set_step(dpo_ctx *c, int64_t k)
     if (k < 0)
         return fail(c, DPO_EINVAL, "step counter must be >= 0");
     c->k = k;
+    c->mu_prod = 1.0;   // NAdam's running product, rebuilt for the restored counter
+    for (int64_t i = 1; i <= k; ++i)
+        c->mu_prod *= nadam_mu(c->hp, i);
     return DPO_OK;
 }
 
@@ -550,9 +613,12 @@ extern "C" int dpo_algorithmic_bytes(const dpo_ctx *c, int64_t *step_bytes, int6
     // Per element: read master, m, v (fp32) and grad; write master, m, v and
     // the bf16 param; a delayed tensor also writes its stash, and under a
     // correction reads and writes its update-history buffer.
-    const int64_t base = 4 * 3 + dt_size(c->grad_dt) + 4 * 3 + (c->param_dt == DPO_BF16 ? 2 : 0);
+    const int64_t base = 8 * (1 + rule_state_streams(c->hp.optimizer)) + dt_size(c->grad_dt) +
+                         (c->param_dt == DPO_BF16 ? 2 : 0);
     const int64_t delayed_extra =
-        c->hp.delay == 1 ? dt_size(c->stash_dt) + (c->ef ? 8 : 0) : 0;
+        c->hp.delay == 1 ? dt_size(c->stash_dt) * (c->hp.dc_lambda != 0.0f ? 2 : 1) +
+                               (c->ef ? 8 : 0)
+                         : 0;
     int64_t total = 0;
     for (const dpo_tensor &d : c->table)
         total += d.numel * (base + ((d.flags & DPO_SYNC) ? 0 : delayed_extra));

@@ -38,10 +38,12 @@ struct DevTensor {
     void *param;        // bf16 latest copy or nullptr
     float *master;
     float *m;
-    float *v;
+    float *v;           // second moment (Adan: the averaged gradient difference)
     void *stash;        // stash dtype, or nullptr when not written
-    float *ef;          // EF buffer or nullptr
+    float *ef;          // update-history buffer or nullptr
     const void *grad;
+    float *n;           // Adan: third moment, else nullptr
+    float *grad_prev;   // Adan: previous (corrected) gradient, else nullptr
     int64_t numel;
     uint32_t flags;
     uint32_t pad_;
@@ -52,6 +54,8 @@ enum StashKind { kStashNone = 0, kStashF32 = 1, kStashBF16 = 2 };
 // Staleness correction of a delayed step (the DPO_CORR_* of include/dpo.h, or
 // none when the table has no update-history buffers).
 enum Correction { kCorrNone = 0, kCorrEF = 1, kCorrSapipeSame = 2, kCorrSapipeUpdated = 3 };
+// Update rule (the DPO_OPT_* of include/dpo.h).
+enum Optimizer { kOptAdamW = 0, kOptNAdam = 1, kOptLion = 2, kOptAdan = 3 };
 
 // Scalars of one fused step, precomputed on the host in double and rounded
 // once to fp32.
@@ -69,6 +73,13 @@ struct StepArgs {
     float lam;                  // lambda of this call (0 at k = 1, Alg. 1)
     float step_size_next;       // lr / (1 - beta1^(k+1))       (SAPipe updated state)
     float inv_sqrt_bc2_next;    // 1 / sqrt(1 - beta2^(k+1))    (SAPipe updated state)
+    float lr;                   // Lion: size of the sign step
+    float nadam_cg, nadam_cm;   // NAdam: lr (1-mu_k)/(1-prod mu), lr mu_{k+1}/(1-prod' mu)
+    float beta3, omb3;          // Adan: beta3, 1 - beta3
+    float inv_sqrt_bc3;         // Adan: 1 / sqrt(1 - beta3^k)
+    float adan_c2;              // Adan: lr beta2 / (1 - beta2^k)
+    int first;                  // Adan: k == 1 (the gradient difference is 0)
+    float dc_lambda;            // DC-ASGD strength (0: off)
     const float *clip;          // device clip coefficient, or nullptr
 };
 
@@ -100,16 +111,25 @@ struct StashArgs {
     int zero_hist;              // also zero the EF buffer (delayed training restarts)
 };
 
+// The fused-step kernel instance for a layout, correction and rule (one
+// translation unit per rule, dpo_step_<rule>.cu); nullptr when that
+// combination is not provided.
+using StepFn = void (*)(StepArgs);
+StepFn pick_step_adamw(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr);
+StepFn pick_step_nadam(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr);
+StepFn pick_step_lion(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr);
+StepFn pick_step_adan(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr);
+
 // Launchers (dpo_kernels.cu). Each returns the launch's cudaError_t.
-cudaError_t launch_step(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr,
-                        int grid, const StepArgs &a, cudaStream_t s);
+cudaError_t launch_step(Optimizer opt, bool param_bf16, StashKind stash, bool grad_bf16,
+                        Correction corr, int grid, const StepArgs &a, cudaStream_t s);
 cudaError_t launch_norm(bool grad_bf16, int grid, const NormArgs &a, cudaStream_t s);
 cudaError_t launch_stash(bool param_bf16, StashKind stash, int grid, const StashArgs &a,
                          cudaStream_t s);
 
 // Resident CTAs per SM of each kernel at its block size (occupancy query).
-cudaError_t step_ctas_per_sm(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr,
-                             int *n);
+cudaError_t step_ctas_per_sm(Optimizer opt, bool param_bf16, StashKind stash, bool grad_bf16,
+                             Correction corr, int *n);
 cudaError_t norm_ctas_per_sm(bool grad_bf16, int *n);
 
 }  // namespace dpo

@@ -1,0 +1,12 @@
+// dpo_step_nadam.cu -- fused-step kernel instances for one update rule (see
+// dpo_step.cuh); one translation unit per rule so they compile in parallel.
+#include "dpo_step.cuh"
+
+namespace dpo {
+
+StepFn pick_step_nadam(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr)
+{
+    return pick_step<kOptNAdam>(param_bf16, stash, grad_bf16, corr);
+}
+
+}  // namespace dpo

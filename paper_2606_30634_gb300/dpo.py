@@ -27,6 +27,7 @@ DPO_STALE, DPO_LATEST = 0, 1
 DPO_INIT_FRESH, DPO_INIT_RESUME = 0, 1
 DPO_FLAG_NONFINITE = 1
 DPO_CORR_EF, DPO_CORR_SAPIPE_SAME, DPO_CORR_SAPIPE_UPDATED = 0, 1, 2
+DPO_OPT_ADAMW, DPO_OPT_NADAM, DPO_OPT_LION, DPO_OPT_ADAN = 0, 1, 2, 3
 
 EXPORTS = ("dpo_init", "dpo_stash", "dpo_step", "dpo_read_weights", "dpo_get_step",
            "dpo_set_step", "dpo_get_flags", "dpo_algorithmic_bytes", "dpo_launch_config",
@@ -47,13 +48,16 @@ class dpo_hparams(ctypes.Structure):
     _fields_ = [("beta1", ctypes.c_float), ("beta2", ctypes.c_float), ("eps", ctypes.c_float),
                 ("weight_decay", ctypes.c_float), ("ef_lambda", ctypes.c_float),
                 ("max_grad_norm", ctypes.c_float), ("delay", ctypes.c_int),
-                ("correction", ctypes.c_int)]
+                ("correction", ctypes.c_int), ("optimizer", ctypes.c_int),
+                ("beta3", ctypes.c_float), ("momentum_decay", ctypes.c_float),
+                ("dc_lambda", ctypes.c_float)]
 
 
 class dpo_tensor(ctypes.Structure):
     _fields_ = [("param", ctypes.c_void_p), ("master", ctypes.c_void_p), ("m", ctypes.c_void_p),
                 ("v", ctypes.c_void_p), ("stash", ctypes.c_void_p), ("ef", ctypes.c_void_p),
-                ("grad", ctypes.c_void_p), ("numel", ctypes.c_int64), ("flags", ctypes.c_uint32)]
+                ("grad", ctypes.c_void_p), ("n", ctypes.c_void_p), ("grad_prev", ctypes.c_void_p),
+                ("numel", ctypes.c_int64), ("flags", ctypes.c_uint32)]
 
 
 _lib = None
@@ -199,6 +203,7 @@ def dpo_grad_norm_noalloc(grad, numel: int, grad_dtype: int, max_grad_norm: floa
 # ------------------------------------------------------------------ owner --
 
 ALIGN_ELEMS = 128   # 256-byte alignment of every tensor in every arena (bf16 or fp32)
+STATE_BUFFERS = ("master", "m", "v", "n", "grad_prev", "param", "stash", "ef")
 
 
 @dataclass
@@ -217,8 +222,9 @@ class Layout:
 
 
 class DelayedAdamW:
-    """Owns the state of a one-step-delayed AdamW step for a set of parameter
-    tensors and drives the C ABI.
+    """Owns the state of a one-step-delayed optimizer step (AdamW by default;
+    ``optimizer`` selects NAdam, Lion or Adan) for a set of parameter tensors
+    and drives the C ABI.
 
     Arenas (torch tensors on the device): master, m, v (fp32), grad (grad
     dtype), param (bf16, only with param_dtype BF16), stash (stash dtype,
@@ -236,7 +242,8 @@ class DelayedAdamW:
                  wd_on: Optional[Sequence[bool]] = None, device=None, x0=None,
                  init_mode=DPO_INIT_FRESH, stream=None, host_grad=False, host_param=False,
                  correction=DPO_CORR_EF, sync: Optional[Sequence[bool]] = None,
-                 keep_stash: Optional[bool] = None):
+                 keep_stash: Optional[bool] = None, optimizer=DPO_OPT_ADAMW, beta3=0.99,
+                 momentum_decay=0.004, dc_lambda=0.0):
         import torch
         self.torch = torch
         self.device = torch.device(device or "cuda")
@@ -251,7 +258,9 @@ class DelayedAdamW:
         host_alloc = lambda dt: torch.zeros(n, dtype=dt, pin_memory=True)
         self.master = alloc(torch.float32)
         self.m = alloc(torch.float32)
-        self.v = alloc(torch.float32)
+        self.v = alloc(torch.float32) if optimizer != DPO_OPT_LION else None
+        self.n = alloc(torch.float32) if optimizer == DPO_OPT_ADAN else None
+        self.grad_prev = alloc(torch.float32) if optimizer == DPO_OPT_ADAN else None
         self.grad = (host_alloc if host_grad else alloc)(tdt[grad_dtype])
         self.param = ((host_alloc if host_param else alloc)(torch.bfloat16)
                       if param_dtype == DPO_BF16 else None)
@@ -261,7 +270,8 @@ class DelayedAdamW:
         if x0 is not None:
             self.master.copy_(x0)
         self.hp = dpo_hparams(beta1, beta2, eps, weight_decay, ef_lambda if ef else 0.0,
-                              max_grad_norm, delay, correction)
+                              max_grad_norm, delay, correction, optimizer, beta3,
+                              momentum_decay, dc_lambda)
         self.wd_on = list(wd_on) if wd_on is not None else [True] * len(numels)
         self.sync = list(sync) if sync is not None else [False] * len(numels)
         self.ctx = None
@@ -273,7 +283,8 @@ class DelayedAdamW:
             ptr = lambda t: (t.data_ptr() + off * t.element_size()) if t is not None else None
             flags = (DPO_WD_ON if self.wd_on[i] else 0) | (DPO_SYNC if self.sync[i] else 0)
             table.append(dpo_tensor(ptr(self.param), ptr(self.master), ptr(self.m), ptr(self.v),
-                                    ptr(self.stash), ptr(self.ef), ptr(self.grad), cnt, flags))
+                                    ptr(self.stash), ptr(self.ef), ptr(self.grad), ptr(self.n),
+                                    ptr(self.grad_prev), cnt, flags))
         self.table = table
         self.ctx = dpo_init(table, self.param_dtype, self.stash_dtype, self.grad_dtype, self.hp,
                             init_mode, stream)
@@ -329,11 +340,11 @@ class DelayedAdamW:
         return dpo_get_step(self.ctx)
 
     def state_dict(self) -> dict:
-        bufs = {n: getattr(self, n) for n in ("master", "m", "v", "param", "stash", "ef")}
+        bufs = {n: getattr(self, n) for n in STATE_BUFFERS}
         return {"k": self.k, **{n: b.clone() for n, b in bufs.items() if b is not None}}
 
     def load_state(self, sd: dict) -> None:
-        for n in ("master", "m", "v", "param", "stash", "ef"):
+        for n in STATE_BUFFERS:
             if getattr(self, n) is not None:
                 getattr(self, n).copy_(sd[n])
         dpo_set_step(self.ctx, int(sd["k"]))

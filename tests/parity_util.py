@@ -36,6 +36,8 @@ TOL_ONE_STEP = 1e-6
 TOL_RUN = 1e-4
 
 STORE = {dpo.DPO_F32: oracle.F32, dpo.DPO_BF16: oracle.BF16}
+RULE = {dpo.DPO_OPT_ADAMW: oracle.RULE_ADAMW, dpo.DPO_OPT_NADAM: oracle.RULE_NADAM,
+        dpo.DPO_OPT_LION: oracle.RULE_LION, dpo.DPO_OPT_ADAN: oracle.RULE_ADAN}
 
 
 def rel_err(gpu: np.ndarray, ref: np.ndarray) -> float:
@@ -122,6 +124,12 @@ class Case:
     grad_sigma: float = 1e-3
     init_sigma: float = 0.02
     correction: int = dpo.DPO_CORR_EF   # with ef: EF, SAPipe same / updated state
+    optimizer: int = dpo.DPO_OPT_ADAMW
+    beta1: float = 0.9
+    beta2: float = 0.95
+    beta3: float = 0.99
+    momentum_decay: float = 0.004
+    dc_lambda: float = 0.0
     sync: Optional[Sequence[bool]] = None      # per tensor: trained synchronously
     schedule: Optional[dict] = None            # call k -> delay mode switched to before it
     host_grad: bool = False     # grad arena in pinned host memory
@@ -144,16 +152,21 @@ class Run:
             delay=case.delay, wd_on=case.wd_on, device=device,
             x0=self._dev_x0(device), init_mode=dpo.DPO_INIT_FRESH,
             host_grad=case.host_grad, host_param=case.host_param, correction=case.correction,
-            sync=case.sync, keep_stash=True)
+            sync=case.sync, keep_stash=True, optimizer=case.optimizer, beta1=case.beta1,
+            beta2=case.beta2, beta3=case.beta3, momentum_decay=case.momentum_decay,
+            dc_lambda=case.dc_lambda)
         # the oracle tracks every element, or only ``sample`` (global indices)
         self.sample = sample
         idx = np.arange(self.N) if sample is None else np.asarray(sample, np.int64)
         self.idx = idx
         x0 = synth.host_normal_at(case.seed, synth.STREAM_INIT, 0, idx, case.init_sigma)
-        hp = oracle.HParams(lr=case.lr, weight_decay=case.weight_decay,
+        hp = oracle.HParams(lr=case.lr, beta1=case.beta1, beta2=case.beta2,
+                            weight_decay=case.weight_decay,
                             ef_lambda=case.ef_lambda if case.ef else 0.0,
                             max_grad_norm=case.max_grad_norm, delay=case.delay,
-                            correction=case.correction).as_f32()
+                            correction=case.correction, rule=RULE[case.optimizer],
+                            beta3=case.beta3, momentum_decay=case.momentum_decay,
+                            dc_lambda=case.dc_lambda).as_f32()
         if sample is None:
             parts = np.split(x0.astype(np.float64), self.offs[1:-1])
             wd = case.wd_on
@@ -236,26 +249,45 @@ class Run:
             return t.view(self.torch.int16).cpu().numpy().view(np.uint16)
         return t.cpu().numpy()
 
-    def compare(self) -> dict:
-        """Errors of every state buffer against the oracle."""
+    def input_mismatch(self) -> np.ndarray:
+        """Tracked elements whose master or stash differ bitwise between the
+        GPU and the oracle (inputs of the next step)."""
+        self.torch.cuda.synchronize()
+        bad = self.gather(self.gpu.master).astype(np.float64) != self.ref.x
+        if self.gpu.stash is not None:
+            s = self.gather(self.gpu.stash)
+            if self.c.stash_dtype == dpo.DPO_BF16:
+                s = synth.bf16_bits_to_f32(s)
+            bad |= s.astype(np.float64) != self.ref.stash
+        return bad
+
+    def compare(self, mask: Optional[np.ndarray] = None) -> dict:
+        """Errors of every state buffer against the oracle (over the tracked
+        elements, or those ``mask`` selects)."""
         self.torch.cuda.synchronize()
         g, r = self.gpu, self.ref
-        out = {"master": rel_err(self.gather(g.master), r.x),
-               "m": rel_err(self.gather(g.m), r.m),
-               "v": rel_err(self.gather(g.v), r.v)}
+        sel = np.ones(self.idx.size, bool) if mask is None else mask
+        out = {"master": rel_err(self.gather(g.master)[sel], r.x[sel]),
+               "m": rel_err(self.gather(g.m)[sel], r.m[sel])}
+        if g.v is not None:
+            out["v"] = rel_err(self.gather(g.v)[sel], r.v[sel])
+        if g.n is not None:
+            out["n"] = rel_err(self.gather(g.n)[sel], r.n3[sel])
+            out["grad_prev"] = rel_err(self.gather(g.grad_prev)[sel], r.g_prev[sel])
         if g.ef is not None:
             # the update history of a synchronously trained tensor stays
             # untouched (zero on both sides); the metric's floor is taken over
             # the delayed tensors' history, where it carries values
             e = self.gather(g.ef)
-            keep = ~self.sync_mask
+            keep = ~self.sync_mask & sel
             out["ef"] = rel_err(e[keep], r.u_prev[keep])
             out["ef_norm"] = norm_err(e[keep], r.u_prev[keep])
-            if (~keep).any():
-                out["ef_sync_absdiff"] = float(np.max(np.abs(e[~keep] - r.u_prev[~keep])))
+            sync_sel = self.sync_mask & sel
+            if sync_sel.any():
+                out["ef_sync_absdiff"] = float(np.max(np.abs(e[sync_sel] - r.u_prev[sync_sel])))
         if g.stash is not None:
             # the stash of a synchronously trained tensor is never read
-            keep = ~self.sync_mask
+            keep = ~self.sync_mask & sel
             s, rs = self.gather(g.stash)[keep], r.stash[keep]
             if self.c.stash_dtype == dpo.DPO_BF16:
                 out["stash_ulp"] = bf16_ulps(s, rs)
@@ -263,13 +295,14 @@ class Run:
             else:
                 out["stash"] = rel_err(s, rs)
         if g.param is not None:
-            p = self.gather(g.param)
-            out["param_ulp"] = bf16_ulps(p, r.param)
-            out["param_raw_ulp"] = bf16_raw_ulps(p, r.param)
+            p = self.gather(g.param)[sel]
+            out["param_ulp"] = bf16_ulps(p, r.param[sel])
+            out["param_raw_ulp"] = bf16_raw_ulps(p, r.param[sel])
         return out
 
-    def assert_close(self, tol: float, normwise: Sequence[str] = ()) -> dict:
-        e = self.compare()
+    def assert_close(self, tol: float, normwise: Sequence[str] = (),
+                     mask: Optional[np.ndarray] = None) -> dict:
+        e = self.compare(mask)
         log = os.environ.get("DPO_PARITY_LOG")
         if log:
             with open(log, "a") as f:

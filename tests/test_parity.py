@@ -10,6 +10,7 @@ import pytest
 import torch
 
 from paper_2606_30634_gb300 import dpo, synth
+import oracle
 from parity_util import TOL_ONE_STEP, TOL_RUN, Case, Run, bf16_ulps, rel_err
 
 pytestmark = pytest.mark.gpu
@@ -214,7 +215,8 @@ def test_dpo_stash_resets_stale_copy(cuda_device):
 def test_misaligned_device_pointer_rejected(cuda_device):
     buf = torch.zeros(1 << 12, dtype=torch.float32, device=cuda_device)
     p = buf.data_ptr()
-    t = dpo.dpo_tensor(None, p + 4, p + 8192, p + 4096, p + 12288, None, p + 2048, 10, 1)
+    t = dpo.dpo_tensor(param=None, master=p + 4, m=p + 8192, v=p + 4096, stash=p + 12288,
+                       ef=None, grad=p + 2048, numel=10, flags=1)
     with pytest.raises(dpo.DpoError) as e:
         dpo.dpo_init([t], F, F, F, dpo.dpo_hparams(0.9, 0.95, 1e-8, 0.1, 0.0, 0.0, 1))
     assert e.value.code == dpo.DPO_EALIGN
@@ -224,7 +226,8 @@ def test_host_pointer_rejected(cuda_device):
     host = np.zeros(1 << 12, np.float32)
     p = host.ctypes.data
     p += (-p) % 32
-    t = dpo.dpo_tensor(None, p, p + 4096, p + 8192, p + 12288, None, p + 13824, 10, 1)
+    t = dpo.dpo_tensor(param=None, master=p, m=p + 4096, v=p + 8192, stash=p + 12288, ef=None,
+                       grad=p + 13824, numel=10, flags=1)
     with pytest.raises(dpo.DpoError) as e:
         dpo.dpo_init([t], F, F, F, dpo.dpo_hparams(0.9, 0.95, 1e-8, 0.1, 0.0, 0.0, 1))
     assert e.value.code == dpo.DPO_EINVAL
@@ -385,3 +388,105 @@ def test_set_delay_needs_stash_buffers(cuda_device):
         assert e.value.code == dpo.DPO_ESTATE
     finally:
         opt.close()
+
+
+# ---------------- other elementwise optimizers under delay (Tab. main_results)
+# with the paper's settings where it gives them (Lion: lr 5e-4, wd 0.5, App. E.1)
+
+RULES = {
+    "nadam": dict(optimizer=dpo.DPO_OPT_NADAM, momentum_decay=0.004),
+    "lion": dict(optimizer=dpo.DPO_OPT_LION, beta1=0.9, beta2=0.99, lr=5e-4, weight_decay=0.5),
+    "adan": dict(optimizer=dpo.DPO_OPT_ADAN, beta1=0.98, beta2=0.92, beta3=0.99),
+}
+
+
+@pytest.mark.parametrize("rule", sorted(RULES))
+@pytest.mark.parametrize("ef,corr", [(False, dpo.DPO_CORR_EF), (True, dpo.DPO_CORR_EF),
+                                     (True, SP_SAME)])
+@pytest.mark.parametrize("pdt,sdt,gdt", [(B, B, B), (B, F, B), (F, F, F)])
+def test_rule_parity(cuda_device, rule, ef, corr, pdt, sdt, gdt):
+    run = Run(Case(RAGGED, param_dtype=pdt, stash_dtype=sdt, grad_dtype=gdt, ef=ef,
+                   correction=corr, max_grad_norm=0.3, **RULES[rule]), cuda_device)
+    try:
+        for k in range(1, 7):
+            run.step()
+            run.assert_close(TOL_ONE_STEP if k == 1 else TOL_RUN)
+    finally:
+        run.close()
+
+
+def test_dc_asgd_parity_multistep(cuda_device):
+    """DC-ASGD's Taylor compensation (Sec. 3.1) with EF over six steps, at
+    lambda = 1e4 with an fp32 stash. The term multiplies x_t - stash by
+    lambda g^2, so at larger lambda (the paper sweeps up to 1e8) a one-rounding
+    difference between the two sides' master or stash, allowed by the fp32
+    and bf16 bars, is amplified into the gradient: there the step is checked
+    on identical inputs instead (next test)."""
+    run = Run(Case(RAGGED, stash_dtype=F, ef=True, dc_lambda=1e4), cuda_device)
+    try:
+        for k in range(1, 7):
+            run.step()
+            run.assert_close(TOL_ONE_STEP if k == 1 else TOL_RUN)
+    finally:
+        run.close()
+
+
+@pytest.mark.parametrize("dc", [1e4, 1e6, 1e8])
+@pytest.mark.parametrize("sdt", [B, F])
+def test_dc_asgd_step_on_identical_inputs(cuda_device, dc, sdt):
+    """One DC-ASGD + EF step from a state both sides hold bit for bit, k = 1
+    done. The stash x_s ~ N(0, 0.02^2) is held in the stash dtype, the master
+    is x_s + sign(g)|N(0, (3e-4)^2)| in fp32, so the compensation term
+    lambda g^2 (x - x_s) has the sign of g and g + lambda g^2 (x - x_s) never
+    cancels: where it cancels the compensated gradient keeps only the digits
+    fp32 leaves and the Adam step near g~ = 0 amplifies them, which no fp32
+    implementation matches to the one-step bar. Every buffer within that bar."""
+    numels, seed = RAGGED, 0xDC
+    N = sum(numels)
+    gb = synth.host_normal(seed, synth.STREAM_GRAD, 2, 0, N, 1e-3, synth.BF16)
+    g = synth.bf16_bits_to_f32(gb).astype(np.float64)
+    xs = synth.host_normal(seed, synth.STREAM_INIT, 0, 0, N, 0.02).astype(np.float32)
+    if sdt == B:
+        xs = torch.from_numpy(xs).to(torch.bfloat16).float().numpy()
+    off = np.abs(synth.host_normal(seed, 7, 0, 0, N, 3e-4)).astype(np.float32)
+    x = (xs + np.sign(g).astype(np.float32) * off).astype(np.float32)
+    # the construction holds after fp32 rounding: no offset opposes its gradient
+    assert np.all(np.sign(x.astype(np.float64) - xs) * np.sign(g) >= 0)
+    opt = dpo.DelayedAdamW(numels, stash_dtype=sdt, ef=True, dc_lambda=dc, device=cuda_device,
+                           init_mode=dpo.DPO_INIT_RESUME)
+    try:
+        offs = np.concatenate([[0], np.cumsum(numels)])
+        for i, n in enumerate(numels):
+            if n:
+                sl = slice(int(offs[i]), int(offs[i + 1]))
+                opt.view(opt.master, i).copy_(torch.from_numpy(x[sl]))
+                opt.view(opt.stash, i).copy_(torch.from_numpy(xs[sl]))
+                opt.grads(i).copy_(torch.from_numpy(gb[sl].view(np.int16)).view(torch.bfloat16))
+        dpo.dpo_set_step(opt.ctx, 1)
+        opt.step()
+        hp = oracle.HParams(lr=3e-4, ef_lambda=1.0, dc_lambda=dc).as_f32()
+        ref = oracle.DelayedOptimizer([x.astype(np.float64)], hp, ef=True, x_store=oracle.F32,
+                                      stash_store=oracle.BF16 if sdt == B else oracle.F32,
+                                      param_store=oracle.BF16)
+        ref.stash[:] = xs
+        ref.k, ref.t = 1, 1
+        ref.step(synth.bf16_bits_to_f32(gb).astype(np.float64))
+        torch.cuda.synchronize()
+        cat = lambda a: torch.cat([opt.view(a, i) for i in range(len(numels))])
+        assert rel_err(cat(opt.master).cpu().numpy(), ref.x) <= TOL_ONE_STEP
+        assert rel_err(cat(opt.m).cpu().numpy(), ref.m) <= TOL_ONE_STEP
+        assert rel_err(cat(opt.v).cpu().numpy(), ref.v) <= TOL_ONE_STEP
+        assert rel_err(cat(opt.ef).cpu().numpy(), ref.u_prev) <= TOL_ONE_STEP
+        p = cat(opt.param).view(torch.int16).cpu().numpy().view(np.uint16)
+        assert bf16_ulps(p, ref.param) <= 1.0
+        # the compensation mattered: it moved the first moment away from (1 - beta1) g
+        assert np.max(np.abs(ref.m - 0.1 * g)) > 1e-3 * np.max(np.abs(0.1 * g))
+    finally:
+        opt.close()
+
+
+def test_sapipe_updated_state_needs_adamw(cuda_device):
+    with pytest.raises(dpo.DpoError) as e:
+        dpo.DelayedAdamW([100], ef=True, correction=SP_UPD, optimizer=dpo.DPO_OPT_LION,
+                         device=cuda_device)
+    assert e.value.code == dpo.DPO_EINVAL
