@@ -140,34 +140,49 @@ int grid_of(const dpo_ctx *c, int per_sm, int64_t pkts_per_cta)
         std::min<int64_t>(groups, (int64_t)std::max(1, c->sms) * std::max(1, per_sm)));
 }
 
-// Grid of the fused step for the context's current mode. Its CTAs per SM put
-// about kStepInflightPerSm bytes of loads in flight per SM (see
-// dpo_internal.h): bytes loaded per packet = master, m, v, grad and, under a
-// correction, the update-history buffer.
+// Whether the fused step compensates gradients with DC-ASGD in the current
+// mode (delayed training with a stash and a non-zero strength).
+bool dc_on(const dpo_ctx *c)
+{
+    return stash_kind(c) != dpo::kStashNone && c->hp.dc_lambda != 0.0f;
+}
+
+// Grid of the fused step for the context's current mode: 128-thread CTAs,
+// a measured number of them per SM. On the 7B-shaped bf16 set (GB300, 20
+// timed steps per point, 2 to 8 CTAs per SM tried) the best were:
+//                      standard rule   with an update history (EF, SAPipe)
+//   AdamW, NAdam, Lion       4                     3
+//   Adan                     3                     3
+//   SAPipe updated state     -                     4
+// Three CTAs where packets also carry the history buffer keep about 55 KiB
+// of loads in flight per SM; the standard rule loads less per packet and
+// wants a fourth; Adan's two extra state streams make three enough; the
+// SAPipe prediction's second Adam evaluation spaces the loads out and wants
+// four. A table whose tensors mostly skip the history (DPO_SYNC, as WPipe's
+// synchronous half) takes the standard rule's figure (measured: 4 CTAs 96.2%,
+// 3 CTAs 93.7% of the copy peak with half the tensors synchronous).
 int set_step_grid(dpo_ctx *c)
 {
     const dpo::Correction corr = correction_kind(c->ef, c->hp);
     int per_sm = 0;
     const cudaError_t e = dpo::step_ctas_per_sm(
         static_cast<dpo::Optimizer>(c->hp.optimizer), c->param_dt == DPO_BF16, stash_kind(c),
-        c->grad_dt == DPO_BF16, corr, &per_sm);
+        c->grad_dt == DPO_BF16, corr, dc_on(c), &per_sm);
     if (e != cudaSuccess)
         return cuda_fail(c, e, "occupancy query");
-    // bytes loaded per packet: master, the rule's state, grad, the history
-    // buffer under a correction, the stash under DC-ASGD
-    const bool delayed = c->hp.delay == 1;
-    const int64_t load_bytes =
-        dpo::kPacket * (4 + 4 * rule_state_streams(c->hp.optimizer) + dt_size(c->grad_dt) +
-                        (corr != dpo::kCorrNone ? 4 : 0) +
-                        (delayed && c->hp.dc_lambda != 0.0f ? dt_size(c->stash_dt) : 0));
-    int want = std::max<int>(1, (int)((dpo::kStepInflightPerSm + load_bytes * dpo::kStepThreads / 2) /
-                                      (load_bytes * dpo::kStepThreads)));
-    // The SAPipe updated-state prediction evaluates AdamW twice per element,
-    // so each thread spends longer between its loads: one more CTA per SM
-    // keeps the same bytes in flight (measured: 3 CTAs 89%, 4 CTAs 98% of the
-    // copy peak on the 7B set).
+    int64_t hist_elems = 0;
+    if (corr != dpo::kCorrNone)
+        for (const dpo_tensor &t : c->table)
+            if (!(t.flags & DPO_SYNC))
+                hist_elems += t.numel;
+    const bool mostly_hist = 4 * hist_elems >= 3 * c->total_elems && hist_elems > 0;
+    int want;
     if (corr == dpo::kCorrSapipeUpdated)
-        want += 1;
+        want = 4;
+    else if (c->hp.optimizer == DPO_OPT_ADAN)
+        want = 3;
+    else
+        want = mostly_hist ? 3 : 4;
     c->step_grid = grid_of(c, std::min(per_sm, want), dpo::kStepThreads);
     return DPO_OK;
 }
@@ -529,7 +544,8 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
         a.clip = c->clip ? &c->d_scalars->clip : nullptr;
         const cudaError_t e = dpo::launch_step(static_cast<dpo::Optimizer>(c->hp.optimizer),
                                                c->param_dt == DPO_BF16, stash_kind(c),
-                                               c->grad_dt == DPO_BF16, corr, c->step_grid, a, s);
+                                               c->grad_dt == DPO_BF16, corr, dc_on(c),
+                                               c->step_grid, a, s);
         if (e != cudaSuccess)
             return cuda_fail(c, e, "fused step launch");
     }

@@ -19,14 +19,10 @@ constexpr uint32_t kFlagWd = 1u;    // DPO_WD_ON
 constexpr uint32_t kFlagSync = 2u;  // DPO_SYNC
 constexpr int kAlign = 32;      // buffer alignment: fp32 packets move as 256-bit accesses
 
-// Fused step and stash kernels: 128-thread CTAs. The number resident per SM
-// is chosen so that about kStepInflightPerSm bytes of loads are in flight per
-// SM (one packet per thread): measured on GB300 HBM3e, fewer starve the
-// memory pipe and more lose DRAM efficiency. That is 3 CTAs (12 warps) for
-// the EF layouts (144-160 B of loads per packet) and 4 CTAs (16 warps) for
-// the standard rule (112-128 B).
+// Fused step and stash kernels: 128-thread CTAs, 3 or 4 resident per SM
+// (the measured table in set_step_grid, dpo_abi.cpp): enough loads in flight
+// to keep HBM3e busy, not so many that DRAM efficiency drops.
 constexpr int kStepThreads = 128;
-constexpr int kStepInflightPerSm = 56 * 1024;
 
 // Gradient-norm kernel: one read stream, so each thread loads
 // kNormUnroll packets per iteration.
@@ -111,25 +107,29 @@ struct StashArgs {
     int zero_hist;              // also zero the EF buffer (delayed training restarts)
 };
 
-// The fused-step kernel instance for a layout, correction and rule (one
-// translation unit per rule, dpo_step_<rule>.cu); nullptr when that
-// combination is not provided.
+// The fused-step kernel instance for a layout, correction, rule and DC-ASGD
+// setting (one translation unit per rule, dpo_step_<rule>.cu); nullptr when
+// that combination is not provided.
 using StepFn = void (*)(StepArgs);
-StepFn pick_step_adamw(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr);
-StepFn pick_step_nadam(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr);
-StepFn pick_step_lion(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr);
-StepFn pick_step_adan(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr);
+StepFn pick_step_adamw(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr,
+                       bool dc);
+StepFn pick_step_nadam(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr,
+                       bool dc);
+StepFn pick_step_lion(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr,
+                      bool dc);
+StepFn pick_step_adan(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr,
+                      bool dc);
 
 // Launchers (dpo_kernels.cu). Each returns the launch's cudaError_t.
 cudaError_t launch_step(Optimizer opt, bool param_bf16, StashKind stash, bool grad_bf16,
-                        Correction corr, int grid, const StepArgs &a, cudaStream_t s);
+                        Correction corr, bool dc, int grid, const StepArgs &a, cudaStream_t s);
 cudaError_t launch_norm(bool grad_bf16, int grid, const NormArgs &a, cudaStream_t s);
 cudaError_t launch_stash(bool param_bf16, StashKind stash, int grid, const StashArgs &a,
                          cudaStream_t s);
 
 // Resident CTAs per SM of each kernel at its block size (occupancy query).
 cudaError_t step_ctas_per_sm(Optimizer opt, bool param_bf16, StashKind stash, bool grad_bf16,
-                             Correction corr, int *n);
+                             Correction corr, bool dc, int *n);
 cudaError_t norm_ctas_per_sm(bool grad_bf16, int *n);
 
 }  // namespace dpo

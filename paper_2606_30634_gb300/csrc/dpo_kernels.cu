@@ -225,25 +225,26 @@ StashFn pick_stash_sk(StashKind sk)
 
 }  // namespace
 
-static StepFn pick_step_for(Optimizer opt, bool pb, StashKind sk, bool gb, Correction corr)
+static StepFn pick_step_for(Optimizer opt, bool pb, StashKind sk, bool gb, Correction corr,
+                            bool dc)
 {
     switch (opt) {
     case kOptAdamW:
-        return pick_step_adamw(pb, sk, gb, corr);
+        return pick_step_adamw(pb, sk, gb, corr, dc);
     case kOptNAdam:
-        return pick_step_nadam(pb, sk, gb, corr);
+        return pick_step_nadam(pb, sk, gb, corr, dc);
     case kOptLion:
-        return pick_step_lion(pb, sk, gb, corr);
+        return pick_step_lion(pb, sk, gb, corr, dc);
     case kOptAdan:
-        return pick_step_adan(pb, sk, gb, corr);
+        return pick_step_adan(pb, sk, gb, corr, dc);
     }
     return nullptr;
 }
 
-cudaError_t launch_step(Optimizer opt, bool pb, StashKind sk, bool gb, Correction corr, int grid,
-                        const StepArgs &a, cudaStream_t s)
+cudaError_t launch_step(Optimizer opt, bool pb, StashKind sk, bool gb, Correction corr, bool dc,
+                        int grid, const StepArgs &a, cudaStream_t s)
 {
-    StepFn f = pick_step_for(opt, pb, sk, gb, corr);
+    StepFn f = pick_step_for(opt, pb, sk, gb, corr, dc);
     if (f == nullptr)
         return cudaErrorInvalidValue;
     f<<<grid, kStepThreads, 0, s>>>(a);
@@ -267,9 +268,9 @@ cudaError_t launch_stash(bool pb, StashKind sk, int grid, const StashArgs &a, cu
 }
 
 cudaError_t step_ctas_per_sm(Optimizer opt, bool pb, StashKind sk, bool gb, Correction corr,
-                             int *n)
+                             bool dc, int *n)
 {
-    StepFn f = pick_step_for(opt, pb, sk, gb, corr);
+    StepFn f = pick_step_for(opt, pb, sk, gb, corr, dc);
     if (f == nullptr)
         return cudaErrorInvalidValue;
     return cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, f, kStepThreads, 0);

@@ -105,7 +105,9 @@ __device__ __forceinline__ float dc_compensate(float lambda, float g, float x, f
 // kCorrEF (lambda-scaled EF; the buffer is read only when lambda != 0),
 // kCorrSapipeSame / kCorrSapipeUpdated (the stash receives the prediction
 // point x_t - u_prev; the weights take the standard rule). OPT is the rule.
-template <int PB, int SK, int GB, int CORR, int OPT>
+// DC selects the DC-ASGD compensation of delayed tensors (instances with a
+// stash only); without it the kernel holds no registers for the stash read.
+template <int PB, int SK, int GB, int CORR, int OPT, int DC>
 __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs a)
 {
     using GT = typename Elem<GB != 0>::T;
@@ -149,7 +151,7 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
         const bool dly = SK != kStashNone && !(d.flags & kFlagSync);
         const bool prev_t = dly && use_prev;
         const bool efn_t = dly && ef_now;
-        const bool dc_t = dly && dc != 0.0f;
+        const bool dc_t = DC && dly;
         const int64_t e = (p - c.tb) * kPacket;
 
         if (e + kPacket <= d.numel) {
@@ -236,43 +238,45 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
 
 // ------------------------------------------------------------ dispatch ----
 
-template <int PB, int SK, int GB, int OPT>
+template <int PB, int SK, int GB, int OPT, int DC>
 StepFn pick_step_corr(Correction corr)
 {
     switch (corr) {
     case kCorrNone:
-        return fused_step_kernel<PB, SK, GB, kCorrNone, OPT>;
+        return fused_step_kernel<PB, SK, GB, kCorrNone, OPT, DC>;
     case kCorrEF:
-        return SK == kStashNone ? nullptr : fused_step_kernel<PB, SK, GB, kCorrEF, OPT>;
+        return fused_step_kernel<PB, SK, GB, kCorrEF, OPT, DC>;
     case kCorrSapipeSame:
-        return SK == kStashNone ? nullptr : fused_step_kernel<PB, SK, GB, kCorrSapipeSame, OPT>;
+        return fused_step_kernel<PB, SK, GB, kCorrSapipeSame, OPT, DC>;
     case kCorrSapipeUpdated:   // the prediction step is defined for AdamW
-        return SK == kStashNone || OPT != kOptAdamW
-                   ? nullptr
-                   : fused_step_kernel<PB, SK, GB, kCorrSapipeUpdated, OPT>;
+        return OPT != kOptAdamW ? nullptr
+                                : fused_step_kernel<PB, SK, GB, kCorrSapipeUpdated, OPT, DC>;
     }
     return nullptr;
 }
 
 template <int PB, int GB, int OPT>
-StepFn pick_step_sk(StashKind sk, Correction corr)
+StepFn pick_step_sk(StashKind sk, Correction corr, bool dc)
 {
     switch (sk) {
     case kStashF32:
-        return pick_step_corr<PB, kStashF32, GB, OPT>(corr);
+        return dc ? pick_step_corr<PB, kStashF32, GB, OPT, 1>(corr)
+                  : pick_step_corr<PB, kStashF32, GB, OPT, 0>(corr);
     case kStashBF16:
-        return pick_step_corr<PB, kStashBF16, GB, OPT>(corr);
-    default:   // synchronous: no stash, no correction
-        return corr == kCorrNone ? pick_step_corr<PB, kStashNone, GB, OPT>(corr) : nullptr;
+        return dc ? pick_step_corr<PB, kStashBF16, GB, OPT, 1>(corr)
+                  : pick_step_corr<PB, kStashBF16, GB, OPT, 0>(corr);
+    default:   // synchronous: no stash, no correction, no compensation
+        return corr == kCorrNone && !dc ? fused_step_kernel<PB, kStashNone, GB, kCorrNone, OPT, 0>
+                                        : nullptr;
     }
 }
 
 template <int OPT>
-StepFn pick_step(bool pb, StashKind sk, bool gb, Correction corr)
+StepFn pick_step(bool pb, StashKind sk, bool gb, Correction corr, bool dc)
 {
     if (pb)
-        return gb ? pick_step_sk<1, 1, OPT>(sk, corr) : pick_step_sk<1, 0, OPT>(sk, corr);
-    return gb ? pick_step_sk<0, 1, OPT>(sk, corr) : pick_step_sk<0, 0, OPT>(sk, corr);
+        return gb ? pick_step_sk<1, 1, OPT>(sk, corr, dc) : pick_step_sk<1, 0, OPT>(sk, corr, dc);
+    return gb ? pick_step_sk<0, 1, OPT>(sk, corr, dc) : pick_step_sk<0, 0, OPT>(sk, corr, dc);
 }
 
 }  // namespace

@@ -4,9 +4,10 @@
 
 namespace dpo {
 
-StepFn pick_step_lion(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr)
+StepFn pick_step_lion(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr,
+                       bool dc)
 {
-    return pick_step<kOptLion>(param_bf16, stash, grad_bf16, corr);
+    return pick_step<kOptLion>(param_bf16, stash, grad_bf16, corr, dc);
 }
 
 }  // namespace dpo
