@@ -102,6 +102,14 @@ def load(path: Optional[str] = None):
     lib.oracle_quadratic.restype = ctypes.c_double
     lib.oracle_quadratic.argtypes = [ctypes.c_int64, _dp, _dp, _dp, _dp,
                                      ctypes.c_int, _dp]
+    lib.oracle_newton_schulz.restype = ctypes.c_int
+    lib.oracle_newton_schulz.argtypes = [ctypes.c_int64, ctypes.c_int64, _dp, ctypes.c_double,
+                                         ctypes.c_double, ctypes.c_double, ctypes.c_double,
+                                         ctypes.c_int, ctypes.c_int, _dp]
+    lib.oracle_muon_step.restype = ctypes.c_int
+    lib.oracle_muon_step.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
+                                     ctypes.c_void_p, _dp, ctypes.c_double, _dp, _dp, _dp, _dp,
+                                     _dp, _dp]
     if default:
         _lib = lib
     return lib

@@ -297,3 +297,126 @@ double oracle_quadratic(int64_t n, const double *a, const double *wstar,
     free(part);
     return 0.5 * total;
 }
+
+/* ------------------------------------------------------------- Muon ---- */
+
+/* C (r x q) = P (r x s) Q (s x q), all row-major, exact products summed in
+ * double, k in increasing order. */
+static void matmul(int64_t r, int64_t s, int64_t q, const double *P, const double *Q, double *C)
+{
+#pragma omp parallel for schedule(static)
+    for (int64_t i = 0; i < r; ++i) {
+        for (int64_t j = 0; j < q; ++j)
+            C[i * q + j] = 0.0;
+        for (int64_t l = 0; l < s; ++l) {
+            const double p = P[i * s + l];
+            for (int64_t j = 0; j < q; ++j)
+                C[i * q + j] += p * Q[l * q + j];
+        }
+    }
+}
+
+int oracle_newton_schulz(int64_t rows, int64_t cols, const double *M, double eps, double a,
+                         double b, double c, int steps, int store, double *O)
+{
+    if (rows < 0 || cols < 0 || steps < 0 || (rows * cols > 0 && (M == NULL || O == NULL)))
+        return -1;
+    if (rows == 0 || cols == 0)
+        return 0;
+    /* Work on the orientation with the smaller Gram matrix: X is r x w. */
+    const int tall = rows > cols;
+    const int64_t r = tall ? cols : rows, w = tall ? rows : cols;
+    double *X = (double *)malloc(sizeof(double) * (size_t)(r * w));
+    double *Xt = (double *)malloc(sizeof(double) * (size_t)(w * r));
+    double *A = (double *)malloc(sizeof(double) * (size_t)(r * r));
+    double *AA = (double *)malloc(sizeof(double) * (size_t)(r * r));
+    double *BX = (double *)malloc(sizeof(double) * (size_t)(r * w));
+    if (!X || !Xt || !A || !AA || !BX) {
+        free(X); free(Xt); free(A); free(AA); free(BX);
+        return -1;
+    }
+    for (int64_t i = 0; i < r; ++i)
+        for (int64_t j = 0; j < w; ++j)
+            X[i * w + j] = tall ? M[j * cols + i] : M[i * cols + j];
+    double ss = 0.0;
+    for (int64_t i = 0; i < r * w; ++i)
+        ss += X[i] * X[i];
+    const double scale = 1.0 / (sqrt(ss) + eps);
+    for (int64_t i = 0; i < r * w; ++i)
+        X[i] = oracle_round(X[i] * scale, store);
+
+    for (int s = 0; s < steps; ++s) {
+        /* A = X X^T */
+        for (int64_t i = 0; i < r; ++i)
+            for (int64_t j = 0; j < w; ++j)
+                Xt[j * r + i] = X[i * w + j];
+        matmul(r, w, r, X, Xt, A);
+        oracle_round_n(r * r, A, A, store);
+        /* B = b A + c A A (B kept in AA) */
+        matmul(r, r, r, A, A, AA);
+        for (int64_t i = 0; i < r * r; ++i)
+            AA[i] = oracle_round(b * A[i] + c * AA[i], store);
+        /* X <- a X + B X */
+        matmul(r, r, w, AA, X, BX);
+        for (int64_t i = 0; i < r * w; ++i)
+            X[i] = oracle_round(a * X[i] + BX[i], store);
+    }
+    for (int64_t i = 0; i < r; ++i)
+        for (int64_t j = 0; j < w; ++j) {
+            if (tall)
+                O[j * cols + i] = X[i * w + j];
+            else
+                O[i * cols + j] = X[i * w + j];
+        }
+    free(X); free(Xt); free(A); free(AA); free(BX);
+    return 0;
+}
+
+int oracle_muon_step(int64_t rows, int64_t cols, int64_t t, const oracle_muon_hparams *hp,
+                     const double *g, double clip_scale, double *x, double *mom,
+                     double *u_prev, double *stash, double *param, double *o_out)
+{
+    const int64_t n = rows * cols;
+    if (rows < 0 || cols < 0 || t < 1 || hp == NULL ||
+        (n > 0 && (g == NULL || x == NULL || mom == NULL)))
+        return -1;
+    if (hp->delay == 1 && n > 0 && stash == NULL)
+        return -1;
+    if (n == 0)
+        return 0;
+    double *O = (double *)malloc(sizeof(double) * (size_t)n);
+    if (O == NULL)
+        return -1;
+
+    /* Momentum of the stale gradient G_{t-1}. */
+    for (int64_t i = 0; i < n; ++i)
+        mom[i] = oracle_round(hp->momentum * mom[i] + (1.0 - hp->momentum) * (clip_scale * g[i]),
+                              hp->x_store);
+    if (oracle_newton_schulz(rows, cols, mom, hp->ns_eps, hp->ns_a, hp->ns_b, hp->ns_c,
+                             hp->ns_steps, hp->ns_store, O) != 0) {
+        free(O);
+        return -1;
+    }
+    const double s = hp->rms_scale > 0.0
+                         ? hp->rms_scale * sqrt((double)(rows > cols ? rows : cols))
+                         : 1.0;
+    const int use_ef = hp->delay == 1 && u_prev != NULL;
+    /* Alg. 1 / Alg. 2: the standard rule at t <= 1, EF from t = 2. */
+    const int ef_now = use_ef && t >= 2;
+    for (int64_t i = 0; i < n; ++i) {
+        const double xt = x[i];
+        const double u = hp->lr * (s * O[i] + hp->weight_decay * xt);
+        const double xn = ef_now ? xt - u - hp->ef_lambda * (u - u_prev[i]) : xt - u;
+        if (hp->delay == 1)   /* the weights the next gradient is evaluated at */
+            stash[i] = oracle_round(x[i], hp->stash_store);
+        if (use_ef)
+            u_prev[i] = oracle_round(u, hp->x_store);
+        x[i] = oracle_round(xn, hp->x_store);
+        if (param != NULL)
+            param[i] = oracle_round(x[i], hp->param_store);
+    }
+    if (o_out != NULL)
+        memcpy(o_out, O, sizeof(double) * (size_t)n);
+    free(O);
+    return 0;
+}

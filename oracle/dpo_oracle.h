@@ -174,6 +174,65 @@ double oracle_quadratic(int64_t n, const double *a, const double *wstar,
                         const double *w, const double *noise, int store,
                         double *grad_out);
 
+/*
+ * Delayed Muon (Alg. 2, Sec. 4), one weight matrix at a time.
+ *
+ * Per call, with G the (clipped) stale gradient of a rows x cols matrix:
+ *   M <- mu M + (1 - mu) G                 momentum as an EMA (Sec. 2.2's
+ *                                          convention for the momentum decay
+ *                                          mu; Alg. 2 prints the two weights
+ *                                          the other way round)
+ *   O  = NewtonSchulz(M)                   oracle_newton_schulz below
+ *   U  = lr (s O + wd X_t),  s = rms_scale sqrt(max(rows, cols)) when
+ *        rms_scale > 0 (update RMS 0.2, Sec. 2.1, as Liu et al. 2025 scale
+ *        it), else s = 1 (Alg. 2 as printed)
+ *   X_{t+1} = X_t - U - lambda_eff (U - U_prev)   (Alg. 2 with EF is
+ *        lambda = 1: X_t - 2 U_{t-1} + U_{t-2}; lambda_eff = 0 at t = 1)
+ * The stash receives X_t and the history buffer U, exactly as oracle_step
+ * does for the elementwise rules.
+ */
+typedef struct {
+    double lr;             /* eta of the call */
+    double momentum;       /* mu */
+    double weight_decay;   /* decay on X_t (Alg. 2) */
+    double ef_lambda;      /* lambda of the EF correction; 0 = standard */
+    double ns_a, ns_b, ns_c;  /* coefficients of the quintic iteration */
+    int ns_steps;          /* iterations */
+    double ns_eps;         /* added to ||M||_F before normalising */
+    double rms_scale;      /* see above; 0 = no scaling */
+    int ns_store;          /* storage of every Newton-Schulz matrix: F64 or BF16 */
+    int delay;             /* 1 = one-step-delayed, 0 = synchronous */
+    int x_store;           /* storage of X, M and U_prev (F64 or F32) */
+    int stash_store;       /* storage of the stash */
+    int param_store;       /* storage of the latest-weights copy */
+} oracle_muon_hparams;
+
+/*
+ * Newton-Schulz orthogonalisation of a rows x cols matrix M (row-major), the
+ * quintic iteration of Jordan et al. 2024 that Muon uses:
+ *   X_0 = M / (||M||_F + eps), taken as its transpose when rows > cols so
+ *         that the Gram matrix is the smaller one;
+ *   A   = X X^T,  B = b A + c A A,  X <- a X + B X     (`steps` times);
+ *   O   = X (transposed back when rows > cols).
+ * store = ORACLE_BF16 rounds X_0 and every A, B and X to bf16 when it is
+ * formed (each from exact products of its rounded inputs), which is how the
+ * iteration runs in bf16 on tensor cores; ORACLE_F64 keeps them exact.
+ * Writes O (rows x cols). Returns 0, or -1 on bad arguments or no memory.
+ */
+int oracle_newton_schulz(int64_t rows, int64_t cols, const double *M, double eps, double a,
+                         double b, double c, int steps, int store, double *O);
+
+/*
+ * One call of delayed Muon on one matrix (see above). t is the Alg. 1
+ * iteration within the current delayed phase (>= 1). x, mom are updated in
+ * place; u_prev (history, or NULL for the standard rule), stash (needed when
+ * delay == 1) and param (or NULL) as in oracle_step. o_out, when not NULL,
+ * receives the Newton-Schulz output O. Returns 0, or -1 on bad arguments.
+ */
+int oracle_muon_step(int64_t rows, int64_t cols, int64_t t, const oracle_muon_hparams *hp,
+                     const double *g, double clip_scale, double *x, double *mom,
+                     double *u_prev, double *stash, double *param, double *o_out);
+
 #ifdef __cplusplus
 }
 #endif

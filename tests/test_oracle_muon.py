@@ -1,0 +1,208 @@
+"""Pins of the delayed-Muon oracle (Alg. 2) against facts outside it.
+
+* Newton-Schulz is a matrix polynomial in M M^T times M, so on M = U S V^T
+  it acts on each singular value alone: O = U p^s(S / (||M||_F + eps)) V^T
+  with p(x) = a x + b x^3 + c x^5 iterated s times. The singular vectors come
+  from numpy's SVD (a library routine); the scalar recursion is one line.
+* On a diagonal matrix every iterate stays diagonal, so the bf16 iteration
+  is a scalar recursion with one bf16 rounding per formed quantity.
+* The Muon step is checked by hand on small cases: the update scale, the
+  momentum's weighting, decay on the current weights, and Alg. 2's EF line
+  X_{t+1} = X_t - 2 U_{t-1} + U_{t-2}.
+"""
+from __future__ import annotations
+
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from oracle import muon
+from oracle.muon import NS_COEFFS, DelayedMuon, MuonHParams, newton_schulz
+
+F64, F32, BF16 = oracle.F64, oracle.F32, oracle.BF16
+A_, B_, C_ = NS_COEFFS
+
+
+@pytest.fixture(scope="module")
+def lib():
+    path = os.environ.get("DPO_ORACLE_LIB")
+    return oracle.load(path) if path else oracle.load()
+
+
+def p_iter(x, steps):
+    for _ in range(steps):
+        x = A_ * x + B_ * x ** 3 + C_ * x ** 5
+    return x
+
+
+def with_singular_values(rng, rows, cols, s):
+    u, _ = np.linalg.qr(rng.normal(size=(rows, rows)))
+    v, _ = np.linalg.qr(rng.normal(size=(cols, cols)))
+    r = min(rows, cols)
+    return u[:, :r] @ np.diag(s) @ v[:, :r].T, u[:, :r], v[:, :r]
+
+
+@pytest.mark.parametrize("rows,cols", [(5, 9), (9, 5), (7, 7), (1, 6), (6, 1)])
+@pytest.mark.parametrize("steps", [1, 2, 5])
+def test_ns_acts_on_singular_values(lib, rows, cols, steps):
+    rng = np.random.default_rng(rows * 100 + cols + steps)
+    s = np.sort(rng.uniform(0.05, 3.0, min(rows, cols)))[::-1]
+    M, u, v = with_singular_values(rng, rows, cols, s)
+    eps = 1e-7
+    expect = u @ np.diag(p_iter(s / (np.linalg.norm(s) + eps), steps)) @ v.T
+    O = newton_schulz(M, steps=steps, store=F64, eps=eps, lib=lib)
+    assert O.shape == (rows, cols)
+    assert np.max(np.abs(O - expect)) < 1e-12
+
+
+def test_ns_rank_one(lib):
+    """M = 4 u v^T: normalised, its one singular value is 4 / (4 + eps)."""
+    u = np.array([3.0, 4.0]) / 5.0
+    v = np.array([1.0, 2.0, 2.0]) / 3.0
+    M = 4.0 * np.outer(u, v)
+    O = newton_schulz(M, steps=5, store=F64, eps=1e-7, lib=lib)
+    np.testing.assert_allclose(O, p_iter(4.0 / (4.0 + 1e-7), 5) * np.outer(u, v), rtol=1e-13)
+
+
+def test_ns_zero_steps_is_normalisation(lib):
+    M = np.arange(12.0).reshape(3, 4) - 5.0
+    O = newton_schulz(M, steps=0, store=F64, eps=1e-7, lib=lib)
+    np.testing.assert_allclose(O, M / (math.sqrt(np.sum(M * M)) + 1e-7), rtol=1e-15)
+
+
+@pytest.mark.parametrize("store", [F64, BF16])
+def test_ns_transpose(lib, store):
+    """NS(M^T) = NS(M)^T exactly: both run on the same wide orientation."""
+    M = np.random.default_rng(3).normal(size=(6, 11))
+    O = newton_schulz(M, store=store, lib=lib)
+    Ot = newton_schulz(M.T.copy(), store=store, lib=lib)
+    assert np.array_equal(Ot, O.T)
+
+
+@pytest.mark.parametrize("rows,cols", [(4, 4), (4, 7), (7, 4)])
+def test_ns_bf16_on_diagonal(lib, rows, cols):
+    """A diagonal M stays diagonal: each entry follows x0 = bf(d / (||d|| +
+    eps)), then A = bf(x^2), B = bf(b A + c A^2), x = bf(a x + B x)."""
+    d = np.array([1.7, -0.3, 0.021, 0.9])
+    M = np.zeros((rows, cols))
+    for i in range(4):
+        M[i, i] = d[i]
+    bf = lambda z: oracle.round_to(np.asarray(z, np.float64), BF16, lib)
+    x = bf(d / (math.sqrt(np.sum(d * d)) + 1e-7))
+    for _ in range(5):
+        a = bf(x * x)
+        b = bf(B_ * a + C_ * (a * a))
+        x = bf(A_ * x + b * x)
+    O = newton_schulz(M, steps=5, store=BF16, eps=1e-7, lib=lib)
+    expect = np.zeros((rows, cols))
+    for i in range(4):
+        expect[i, i] = x[i]
+    assert np.array_equal(O, expect)
+    # and the result differs from the exact iteration (rounding happened)
+    assert not np.array_equal(O, newton_schulz(M, steps=5, store=F64, eps=1e-7, lib=lib))
+
+
+def test_ns_bf16_iterates_are_bf16(lib):
+    M = np.random.default_rng(4).normal(size=(8, 20))
+    O = newton_schulz(M, store=BF16, lib=lib)
+    assert np.array_equal(O, oracle.round_to(O, BF16, lib))
+
+
+# ----------------------------------------------------------------- step ----
+
+def _hp(**kw):
+    base = dict(lr=0.01, momentum=0.95, weight_decay=0.1, ns_store=F64, delay=1)
+    base.update(kw)
+    return MuonHParams(**base)
+
+
+def test_muon_first_step_by_hand(lib):
+    """First call: M = (1 - mu) g, whose normalisation removes (1 - mu) (up
+    to eps); U = lr (0.2 sqrt(max(rows, cols)) O + wd X_0); standard rule."""
+    rng = np.random.default_rng(5)
+    x0 = rng.normal(size=(4, 9))
+    s = np.array([2.0, 1.0, 0.5, 0.1])
+    g, u, v = with_singular_values(rng, 4, 9, s)
+    hp = _hp(ns_eps=0.0)
+    opt = DelayedMuon([x0], hp, ef=True, x_store=F64, stash_store=F64, param_store=F64, lib=lib)
+    opt.step([g])
+    O = u @ np.diag(p_iter(s / np.linalg.norm(s), 5)) @ v.T
+    U = 0.01 * (0.2 * 3.0 * O + 0.1 * x0)
+    np.testing.assert_allclose(opt.mom[0], 0.05 * g, rtol=1e-14, atol=1e-16)
+    np.testing.assert_allclose(opt.x[0], x0 - U, rtol=1e-12, atol=1e-14)
+    np.testing.assert_allclose(opt.u_prev[0], U, rtol=1e-12, atol=1e-14)
+    assert np.array_equal(opt.stash[0], x0)
+    assert np.array_equal(opt.param[0], opt.x[0])
+
+
+def test_muon_scale_uses_the_larger_dimension(lib):
+    """Zero decay: U = lr * 0.2 sqrt(max(rows, cols)) O, for both shapes."""
+    for shape in [(4, 25), (25, 4)]:
+        rng = np.random.default_rng(6)
+        g = rng.normal(size=shape)
+        opt = DelayedMuon([np.zeros(shape)], _hp(weight_decay=0.0), x_store=F64,
+                          stash_store=F64, lib=lib)
+        opt.step([g])
+        O = newton_schulz(0.05 * g, store=F64, lib=lib)
+        np.testing.assert_allclose(-opt.x[0], 0.01 * 0.2 * 5.0 * O, rtol=1e-13, atol=1e-16)
+
+
+def test_muon_momentum_weights_the_history(lib):
+    """With no Newton-Schulz steps O = M / ||M||: after gradients g1, g2 the
+    direction is that of mu g1 + g2 (Sec. 2.2's EMA), not (1 - mu) g1 + g2."""
+    rng = np.random.default_rng(7)
+    g1, g2 = rng.normal(size=(3, 5)), rng.normal(size=(3, 5))
+    opt = DelayedMuon([np.zeros((3, 5))], _hp(weight_decay=0.0, ns_steps=0, ns_eps=0.0,
+                                              rms_scale=0.0), x_store=F64, stash_store=F64,
+                      lib=lib)
+    opt.step([g1])
+    x1 = opt.x[0].copy()
+    opt.step([g2])
+    d = 0.95 * g1 + g2
+    np.testing.assert_allclose(x1 - opt.x[0], 0.01 * d / np.linalg.norm(d), rtol=1e-12)
+
+
+def test_muon_decay_acts_on_current_weights(lib):
+    """Zero gradients give O = 0, so each call scales X_t by (1 - lr wd);
+    under delay the stash lags one version and is not what decays."""
+    x0 = np.random.default_rng(8).normal(size=(3, 4))
+    opt = DelayedMuon([x0], _hp(lr=0.1, weight_decay=0.5), x_store=F64, stash_store=F64,
+                      lib=lib)
+    for k in range(1, 5):
+        opt.step([np.zeros((3, 4))])
+        np.testing.assert_allclose(opt.x[0], (1 - 0.05) ** k * x0, rtol=1e-14)
+
+
+def test_muon_ef_is_algorithm_2(lib):
+    """EF with lambda = 1: X_2 = X_1 - U_0 (standard rule at t = 1), then
+    X_{t+1} = X_t - 2 U_{t-1} + U_{t-2}, with U_{t-1} = lr (s O + wd X_t)
+    rebuilt from the Newton-Schulz outputs; the stash holds X_t."""
+    rng = np.random.default_rng(9)
+    x0 = rng.normal(size=(5, 3))
+    opt = DelayedMuon([x0], _hp(ef_lambda=1.0), ef=True, x_store=F64, stash_store=F64, lib=lib)
+    xs, us = [x0.copy()], []
+    for k in range(5):
+        xt = opt.x[0].copy()
+        opt.step([rng.normal(size=(5, 3))])
+        us.append(0.01 * (0.2 * math.sqrt(5) * opt.o[0] + 0.1 * xt))
+        assert np.array_equal(opt.stash[0], xt)
+        if k == 0:
+            np.testing.assert_allclose(opt.x[0], xt - us[0], rtol=1e-14)
+        else:
+            np.testing.assert_allclose(opt.x[0], xt - 2 * us[k] + us[k - 1], rtol=1e-13)
+        xs.append(opt.x[0].copy())
+
+
+def test_muon_empty_and_clip(lib):
+    """A 0 x n matrix is a no-op; clipping scales the gradient before the
+    momentum (global norm over all matrices)."""
+    opt = DelayedMuon([np.zeros((0, 4)), np.ones((2, 2))],
+                      _hp(max_grad_norm=1.0, ns_steps=0, ns_eps=0.0, rms_scale=0.0,
+                          weight_decay=0.0), x_store=F64, stash_store=F64, lib=lib)
+    g = np.full((2, 2), 3.0)   # norm 6
+    opt.step([np.zeros((0, 4)), g])
+    assert opt.last_clip == pytest.approx(1.0 / (6.0 + 1e-6), rel=1e-15)
+    np.testing.assert_allclose(opt.mom[1], 0.05 * g * opt.last_clip, rtol=1e-15)

@@ -2,8 +2,8 @@
 
 Each case copies ``oracle/dpo_oracle.c``, plants one mistake in the copy (a
 dropped term, a wrong sign or index, swapped operands, a misread passage),
-builds it into a temporary library, and runs ``test_oracle_pins.py`` against
-that build. Every planted mistake must make at least one pin fail. Nothing
+builds it into a temporary library, and runs ``test_oracle_pins.py`` and
+``test_oracle_muon.py`` against that build. Every planted mistake must make at least one pin fail. Nothing
 here touches the committed oracle or any GPU.
 """
 from __future__ import annotations
@@ -58,6 +58,28 @@ MUTANTS = [
     ("adan_diff_sign", "gi - g_prev[i]", "g_prev[i] - gi"),
     ("adan_no_lookahead", "gi + hp->beta2 * diff", "gi"),
     ("dc_sign", "(xt - stash[i])", "(stash[i] - xt)"),
+    # delayed Muon (Alg. 2) and its Newton-Schulz iteration
+    ("ns_coefficient_roles", "AA[i] = oracle_round(b * A[i] + c * AA[i], store);",
+     "AA[i] = oracle_round(c * A[i] + b * AA[i], store);"),
+    ("ns_drops_linear_term", "X[i] = oracle_round(a * X[i] + BX[i], store);",
+     "X[i] = oracle_round(BX[i], store);"),
+    ("ns_norm_squared", "const double scale = 1.0 / (sqrt(ss) + eps);",
+     "const double scale = 1.0 / (ss + eps);"),
+    ("ns_bf16_skips_b", "AA[i] = oracle_round(b * A[i] + c * AA[i], store);",
+     "AA[i] = b * A[i] + c * AA[i];"),
+    ("ns_output_not_transposed_back", "O[j * cols + i] = X[i * w + j];",
+     "O[i * rows + j] = X[i * w + j];"),
+    ("muon_momentum_roles",
+     "hp->momentum * mom[i] + (1.0 - hp->momentum) * (clip_scale * g[i])",
+     "(1.0 - hp->momentum) * mom[i] + hp->momentum * (clip_scale * g[i])"),
+    ("muon_scale_smaller_dim", "sqrt((double)(rows > cols ? rows : cols))",
+     "sqrt((double)(rows < cols ? rows : cols))"),
+    ("muon_decay_on_stash", "hp->lr * (s * O[i] + hp->weight_decay * xt)",
+     "hp->lr * (s * O[i] + hp->weight_decay * (hp->delay == 1 ? stash[i] : xt))"),
+    ("muon_stash_holds_new_weights", "stash[i] = oracle_round(x[i], hp->stash_store);",
+     "stash[i] = oracle_round(xn, hp->stash_store);"),
+    ("muon_ef_at_first_update", "const int ef_now = use_ef && t >= 2;",
+     "const int ef_now = use_ef && t >= 1;"),
 ]
 
 
@@ -73,7 +95,8 @@ def _build_mutant(tmp_path, name, old, new):
 def _run_pins(lib_path):
     env = dict(os.environ, DPO_ORACLE_LIB=lib_path, OMP_NUM_THREADS="1")
     r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
-                        os.path.join(ROOT, "tests", "test_oracle_pins.py")],
+                        os.path.join(ROOT, "tests", "test_oracle_pins.py"),
+                        os.path.join(ROOT, "tests", "test_oracle_muon.py")],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
     return r.returncode, r.stdout[-600:]
 
