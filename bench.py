@@ -36,6 +36,8 @@ if ROOT not in sys.path:
 METRIC = "params updated/sec and achieved HBM GB/s (% of GB300 peak), 7B-shaped step"
 UNIT = "params/s"
 FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS_SUSTAINED = 1700.0
+MUON_LR = 2e-3
 
 
 def parse_args(argv=None):
@@ -47,7 +49,11 @@ def parse_args(argv=None):
     p.add_argument("--workload", default="llama-7B")
     p.add_argument("--mode", choices=["ef", "std", "sapipe-same", "sapipe-updated"],
                    default="ef")
-    p.add_argument("--optimizer", choices=["adamw", "nadam", "lion", "adan"], default="adamw")
+    p.add_argument("--optimizer", choices=["adamw", "nadam", "lion", "adan", "muon"],
+                   default="adamw",
+                   help="muon: delayed Muon (Alg. 2) on the attention and MLP matrices, "
+                        "AdamW on the rest")
+    p.add_argument("--ns-steps", type=int, default=5, help="Newton-Schulz steps (muon)")
     p.add_argument("--dc-lambda", type=float, default=0.0,
                    help="DC-ASGD compensation strength (Sec. 3.1); 0: off")
     p.add_argument("--wpipe", action="store_true",
@@ -86,6 +92,17 @@ def aggregate(units_per_rank: float, seconds_per_rank: float, world: int, device
 
 
 # ----------------------------------------------------------------- peaks --
+
+def measured_bf16_peak():
+    """Sustained dense bf16 TFLOP/s (the Newton-Schulz GEMMs run back to back
+    for the whole step), measured on the GB300s."""
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["bf16_tflops_sustained"]), "measured"
+    except Exception:
+        return FALLBACK_BF16_TFLOPS_SUSTAINED, "fallback"
+
 
 def measured_hbm_peak():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
@@ -321,6 +338,131 @@ def run_gpu(args, w, world, rank, local):
                 device_name=props.name)
 
 
+def muon_split(w):
+    """(Muon matrix indices, AdamW tensor indices): the attention and MLP
+    projection matrices take Muon; embeddings, the LM head, norms and biases
+    keep AdamW, the usual division for Muon (Sec. 2.1 trains with it)."""
+    hidden = ("_proj", "c_attn.weight", "c_proj.weight", "c_fc.weight")
+    mu = [i for i, (name, shape) in enumerate(w.tensors)
+          if len(shape) == 2 and name.endswith(hidden)]
+    rest = [i for i in range(len(w.tensors)) if i not in set(mu)]
+    return mu, rest
+
+
+def run_muon(args, w, world, rank, local):
+    """Delayed Muon (Alg. 2, EF per --mode) on the set's hidden matrices plus
+    the fused AdamW step on the rest, one stream; a step is both calls."""
+    import numpy as np
+    import torch
+
+    from paper_2606_30634_gb300 import dpo, muon, synth
+    from paper_2606_30634_gb300.synth import workloads as W
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    ef = args.mode == "ef"
+    stream = torch.cuda.Stream(dev)
+    offs = np.concatenate([[0], np.cumsum(w.numels)]).astype(np.int64)
+    mi, ai = muon_split(w)
+    shapes = [w.tensors[i][1] for i in mi]
+    with torch.cuda.stream(stream):
+        mo = muon.DelayedMuon(shapes, stash_dtype=w.stash_dtype, grad_dtype=w.grad_dtype,
+                              lr=MUON_LR, ef=ef, ns_steps=args.ns_steps, delay=1, device=dev,
+                              init_mode=dpo.DPO_INIT_RESUME, stream=stream)
+        for j, i in enumerate(mi):
+            synth.dev_normal(w.seed, synth.STREAM_INIT, 0, int(offs[i]),
+                             mo.view(mo.master, j).view(-1), W.INIT_SIGMA)
+            synth.dev_normal(w.seed, synth.STREAM_GRAD, 1, int(offs[i]),
+                             mo.grads(j).view(-1), W.GRAD_SIGMA)
+        mo.stash.copy_(mo.master)   # Alg. 1 start: stash = param = x_0, m = U_prev = 0
+        mo.param.copy_(mo.master)
+        rest = [w.numels[i] for i in ai]
+        lay = dpo.Layout.of(rest)
+        x0 = torch.empty(lay.total, dtype=torch.float32, device=dev)
+        for j, i in enumerate(ai):
+            o, n = lay.offsets[j], lay.numels[j]
+            synth.dev_normal(w.seed, synth.STREAM_INIT, 0, int(offs[i]), x0[o:o + n],
+                             W.INIT_SIGMA)
+        ad = dpo.DelayedAdamW(rest, param_dtype=w.param_dtype, stash_dtype=w.stash_dtype,
+                              grad_dtype=w.grad_dtype, ef=ef, ef_lambda=1.0, delay=1,
+                              device=dev, x0=x0, stream=stream, lr=w.lr, beta1=w.beta1,
+                              beta2=w.beta2, eps=w.eps, weight_decay=w.weight_decay)
+        del x0
+        for j, i in enumerate(ai):
+            synth.dev_normal(w.seed, synth.STREAM_GRAD, 1, int(offs[i]), ad.grads(j),
+                             W.GRAD_SIGMA)
+    torch.cuda.synchronize(dev)
+    flops = mo.flops()
+    n_groups = len({(min(r, c), max(r, c)) for r, c in shapes})
+    launches_per_step = 1 + 3 + n_groups * (1 + 3 * args.ns_steps)
+
+    mo.set_timing(True)
+    for _ in range(args.warmup):
+        ad.step(stream=stream)
+        mo.step(stream=stream)
+    torch.cuda.synchronize(dev)
+    mo.gemm_time()   # start the count at the timed region
+
+    props = torch.cuda.get_device_properties(dev)
+    sampler = ClockSampler(getattr(props, "pci_bus_id", None))
+    K = args.steps
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize(dev)
+    sampler.start()
+    time.sleep(0.25)
+    ev[0].record(stream)
+    for _ in range(K):
+        ad.step(stream=stream)
+        mo.step(stream=stream)
+    ev[1].record(stream)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        torch.distributed.barrier()
+    clocks = sampler.stop()
+    gemm_ms, gemm_launches = mo.gemm_time()
+    status = mo.status()
+    total_s = ev[0].elapsed_time(ev[1]) / 1e3
+    value, t_max = aggregate(w.n_params * K, total_s, world, dev)
+    achieved = flops * K / (gemm_ms / 1e3) / 1e12
+    ws = mo.workspace_bytes()
+    mo.close()
+    ad.close()
+    if status != 0:
+        raise RuntimeError(f"tensor-core pipeline status {status}")
+    return dict(value=value, t_max=t_max, achieved=achieved, flops=flops, gemm_ms=gemm_ms / K,
+                gemm_launches=gemm_launches, clocks=clocks, launches=K * launches_per_step,
+                n_muon=sum(w.numels[i] for i in mi), n_matrices=len(mi), workspace=ws,
+                device_name=props.name)
+
+
+def oracle_muon_sample(seconds: float, rows: int = 1024, cols: int = 4096):
+    """The Muon oracle as it stands (Newton-Schulz with bf16 iterates, exact
+    accumulation) on one rows x cols matrix of the 7B set's width, steps
+    until ``seconds`` pass. Returns (params/s, cores, steps, params)."""
+    import numpy as np
+
+    import oracle
+    from oracle import muon as omuon
+    from paper_2606_30634_gb300 import synth
+
+    x0 = synth.host_normal(0xD0D0 + 5, synth.STREAM_INIT, 0, 0, rows * cols, 0.02)
+    opt = omuon.DelayedMuon([x0.reshape(rows, cols).astype(np.float64)],
+                            omuon.MuonHParams(lr=MUON_LR, ef_lambda=1.0).as_f32(), ef=True,
+                            x_store=oracle.F32, stash_store=oracle.BF16, param_store=oracle.BF16)
+    steps, spent = 0, 0.0
+    while spent < seconds or steps == 0:
+        g = synth.bf16_bits_to_f32(synth.host_normal(0xD0D0 + 5, synth.STREAM_GRAD, steps + 1, 0,
+                                                     rows * cols, 1e-3, synth.BF16))
+        g = g.astype(np.float64).reshape(rows, cols)
+        t0 = time.perf_counter()
+        opt.step([g])
+        spent += time.perf_counter() - t0
+        steps += 1
+    return rows * cols * steps / spent, oracle.num_threads(), steps, rows * cols
+
+
 def _host_avail_bytes():
     try:
         with open("/proc/meminfo") as f:
@@ -393,11 +535,78 @@ def run_e2e(args, opt, stream, dev, world, w):
 
 # ------------------------------------------------------------------ main --
 
+def main_muon(args, w, world, rank, local):
+    """--optimizer muon: delayed Muon on the hidden matrices, AdamW on the
+    rest; the roofline is the Newton-Schulz GEMMs against the sustained bf16
+    tensor peak."""
+    mi, ai = muon_split(w)
+    n_muon = sum(w.numels[i] for i in mi)
+    cfg = {"workload": f"{w.name}: {w.n_params} params; delayed Muon (Alg. 2, "
+                       f"{args.ns_steps} Newton-Schulz steps) on {len(mi)} attention/MLP "
+                       f"matrices ({n_muon} params), AdamW on the other {len(ai)} tensors, "
+                       f"{'EF' if args.mode == 'ef' else 'standard rule'}, one-step delay",
+           "mode": args.mode, "optimizer": "muon", "ns_steps": args.ns_steps,
+           "param_dtype": "bf16", "stash_dtype": "bf16" if w.stash_dtype else "f32",
+           "grad_dtype": "bf16" if w.grad_dtype else "f32",
+           "ns_dtype": "bf16 operands, fp32 accumulation (tcgen05)",
+           "l2": "inputs larger than L2 (no flush needed)"}
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        v, cores, steps, n = oracle_muon_sample(args.cpu_seconds)
+        line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT,
+                "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+                "ms_per_step": w.n_params / v * 1e3, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                "config": cfg,
+                "cpu_baseline": {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
+                                 "sample": f"one 1024 x 4096 matrix, {steps} Muon oracle steps "
+                                           "(plain C, fp64, bf16 Newton-Schulz iterates)"},
+                "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
+        print(json.dumps(line), flush=True)
+        return 0
+    import torch
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    r = run_muon(args, w, world, rank, local)
+    peak, peak_kind = measured_bf16_peak()
+    roof = {"bound": "tensor", "achieved": r["achieved"], "peak": peak, "unit": "TFLOP/s",
+            "frac": r["achieved"] / peak, "peak_kind": f"{peak_kind} (sustained)",
+            "traffic": None, "kernel": "ns_gemm_kernel",
+            "algorithmic_flops_per_step": r["flops"], "gemm_ms_per_step": r["gemm_ms"],
+            "gemm_launches_per_step": r["gemm_launches"] / max(1, args.steps),
+            "nominal_peak_tflops": 2250.0}
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        v, cores, steps, n = oracle_muon_sample(args.cpu_seconds)
+        cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
+               "sample": f"one 1024 x 4096 matrix, {steps} Muon oracle steps (plain C, fp64, "
+                         "bf16 Newton-Schulz iterates)"}
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    if rank != 0:
+        return 0
+    line = {"metric": METRIC, "value": r["value"], "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": r["t_max"] / args.steps * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16+f32", "data": "synthetic",
+            "config": cfg, "roofline": roof, "cpu_baseline": cpu, "e2e": None,
+            "gpu_launches": r["launches"], "clocks": r["clocks"],
+            "workspace_bytes": r["workspace"], "device": r["device_name"]}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main(argv=None):
     args = parse_args(argv)
     from paper_2606_30634_gb300.synth import workloads as W
     w = W.ALL[args.workload]
     world, rank, local = dist_env()
+    if args.optimizer == "muon":
+        return main_muon(args, w, world, rank, local)
     ef, _, what = MODES[args.mode]
     cfg = {"workload": f"{w.name}: {w.n_params} params in {len(w.tensors)} tensors, "
                        f"{what}, one-step delay",

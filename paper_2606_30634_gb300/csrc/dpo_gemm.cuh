@@ -1,0 +1,322 @@
+// dpo_gemm.cuh -- batched bf16 GEMM on the sm_103a tensor cores (tcgen05,
+// TMA, TMEM) with the epilogues of the Newton-Schulz iteration.
+//
+//   D[b] = alpha * A[b] B[b]^T + beta * C[b]      (optionally also D[b]^T)
+//
+// A[b] (M x K) and B[b] (N x K) are row-major bf16 ("K-major" operands), the
+// product accumulates in fp32 in tensor memory, and the epilogue rounds once
+// to bf16. Every dimension is a multiple of the tile (the Newton-Schulz
+// scratch is padded with zeros to multiples of 256), so no tile is partial.
+//
+// One CTA computes one 128 x 256 tile of one batch entry:
+//   warp 0      TMA producer: 128 x 64 and 256 x 64 bf16 boxes (128-byte
+//               swizzle) into a 4-stage shared-memory ring;
+//   warp 1      allocates 256 TMEM columns; one lane issues
+//               tcgen05.mma.cta_group::1.kind::f16 (M 128, N 256, K 16) four
+//               times per stage and commits each stage back to the producer;
+//   warps 2-5   epilogue: tcgen05.ld 32 lanes x 32 columns at a time, scale,
+//               add the addend, round to bf16, store row-major (16-byte
+//               stores) and, when asked, transposed (each warp writes 64
+//               contiguous bytes per column).
+// Every wait on an mbarrier gives up after kWaitNs, records an error code and
+// lets the CTA finish (draining its own TMA loads first), so a fault in the
+// pipeline surfaces as a status instead of a hang.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cstdint>
+
+namespace dpo {
+namespace gemm {
+
+constexpr int BM = 128, BN = 256, BK = 64, kStages = 4;
+constexpr int kThreads = 192;
+constexpr uint32_t kTmemCols = 256;
+constexpr int kABytes = BM * BK * 2;                 // 16 KiB
+constexpr int kBBytes = BN * BK * 2;                 // 32 KiB
+constexpr int kStageBytes = kABytes + kBBytes;       // 48 KiB
+constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256;
+constexpr unsigned long long kWaitNs = 1000000000ull;  // 1 s per wait
+
+// Error codes OR-ed into Params::err.
+constexpr unsigned int kErrWaitFull = 1u, kErrWaitEmpty = 2u, kErrWaitDone = 4u,
+                       kErrDrain = 8u;
+
+struct Params {
+    __nv_bfloat16 *d;             // M x N row-major output
+    int64_t ldd, d_bstride;       // elements
+    __nv_bfloat16 *dt;            // N x M row-major transposed output, or nullptr
+    int64_t ldt, dt_bstride;
+    const __nv_bfloat16 *c;       // M x N addend, or nullptr
+    int64_t ldc, c_bstride;
+    float alpha, beta;
+    int k_blocks;                 // K / BK
+    unsigned int *err;
+};
+
+__device__ __forceinline__ unsigned long long globaltimer()
+{
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Wait for the phase with the given parity to complete, for at most kWaitNs.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity)
+{
+    if (mbar_try(bar, parity))
+        return true;
+    const unsigned long long t0 = globaltimer();
+    while (!mbar_try(bar, parity))
+        if (globaltimer() - t0 > kWaitNs)
+            return false;
+    return true;
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, int x, int y,
+                                            int z, uint32_t bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
+        : "memory");
+}
+
+// Shared-memory matrix descriptor of a K-major operand tile stored as rows of
+// 64 bf16 (128 bytes) with the 128-byte swizzle, 8-row groups 1024 bytes
+// apart (the layout the TMA box above produces): start address, leading
+// byte offset 16 (unused by swizzled K-major layouts), stride byte offset
+// 1024, descriptor version 1, swizzle mode 2 (128-byte).
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr)
+{
+    return (uint64_t)((addr & 0x3FFFFu) >> 4) | ((uint64_t)(16 >> 4) << 16) |
+           ((uint64_t)(1024 >> 4) << 32) | (1ull << 46) | (2ull << 61);
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, both
+// K-major, N = BN, M = BM.
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
+                            ((uint32_t)(BM >> 4) << 24);
+
+__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t a_desc, uint64_t b_desc,
+                                         uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+        "l"(a_desc), "l"(b_desc), "r"(kIdesc), "r"(accumulate));
+}
+
+__device__ __forceinline__ void mma_commit(uint32_t bar)
+{
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32])
+{
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+        "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
+{
+    const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t *>(&h);
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    ns_gemm_kernel(const __grid_constant__ CUtensorMap tma_a,
+                   const __grid_constant__ CUtensorMap tma_b, const Params p)
+{
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ uint64_t bars[2 * kStages + 1];
+    __shared__ uint32_t tmem_slot;
+    __shared__ int aborted;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM, b = blockIdx.z;
+
+    // 1024-byte aligned operand ring (the 128-byte swizzle repeats every
+    // 1024 bytes and the descriptors assume that alignment).
+    const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
+    const uint32_t ring = (raw + 1023u) & ~1023u;
+    const uint32_t sa = ring, sb = ring + kStages * kABytes;
+    const uint32_t bar0 = (uint32_t)__cvta_generic_to_shared(bars);
+    auto full = [&](int s) { return bar0 + 8u * (uint32_t)s; };
+    auto empty = [&](int s) { return bar0 + 8u * (uint32_t)(kStages + s); };
+    const uint32_t done = bar0 + 8u * (uint32_t)(2 * kStages);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(full(s), 1);
+            mbar_init(empty(s), 1);
+        }
+        mbar_init(done, 1);
+        aborted = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         (uint32_t)__cvta_generic_to_shared(&tmem_slot)),
+                     "r"(kTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = tmem_slot;
+    const int kb_n = p.k_blocks;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tma_a))
+                         : "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tma_b))
+                         : "memory");
+            int issued = 0;
+            for (int kb = 0; kb < kb_n; ++kb) {
+                const int s = kb % kStages;
+                const uint32_t ph = (uint32_t)(kb / kStages) & 1u;
+                if (!mbar_wait(empty(s), ph ^ 1u) || *(volatile int *)&aborted) {
+                    atomicOr(p.err, kErrWaitEmpty);
+                    aborted = 1;
+                    break;
+                }
+                mbar_arrive_expect_tx(full(s), (uint32_t)kStageBytes);
+                tma_load_3d(sa + (uint32_t)(s * kABytes), &tma_a, kb * BK, m0, b, full(s));
+                tma_load_3d(sb + (uint32_t)(s * kBBytes), &tma_b, kb * BK, n0, b, full(s));
+                issued = kb + 1;
+            }
+            // Drain: every load this thread issued lands before the CTA ends
+            // (normally the MMA warp has consumed them all already).
+            for (int kb = issued - kStages < 0 ? 0 : issued - kStages; kb < issued; ++kb)
+                if (!mbar_wait(full(kb % kStages), (uint32_t)(kb / kStages) & 1u))
+                    atomicOr(p.err, kErrDrain);
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            for (int kb = 0; kb < kb_n; ++kb) {
+                const int s = kb % kStages;
+                const uint32_t ph = (uint32_t)(kb / kStages) & 1u;
+                if (!mbar_wait(full(s), ph) || *(volatile int *)&aborted) {
+                    atomicOr(p.err, kErrWaitFull);
+                    aborted = 1;
+                    break;
+                }
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+#pragma unroll
+                for (int k = 0; k < BK / 16; ++k) {
+                    const uint64_t ad = smem_desc(sa + (uint32_t)(s * kABytes + k * 32));
+                    const uint64_t bd = smem_desc(sb + (uint32_t)(s * kBBytes + k * 32));
+                    mma_bf16(tmem, ad, bd, (kb | k) != 0 ? 1u : 0u);
+                }
+                mma_commit(empty(s));
+            }
+            mma_commit(done);   // arrives when every MMA issued above has completed
+        }
+    } else {
+        // Epilogue: warp w reads TMEM lanes 32 (w % 4) .. +31 = tile rows.
+        const int q = warp & 3;
+        const bool seen = mbar_wait(done, 0u);
+        if (!seen)
+            atomicOr(p.err, kErrWaitDone);
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        // tcgen05.ld is warp-collective: the whole warp goes on, or none of it.
+        const bool ok = __all_sync(0xFFFFFFFFu, seen && !*(volatile int *)&aborted);
+        if (ok) {
+            const int64_t row = m0 + q * 32 + lane;
+            __nv_bfloat16 *drow = p.d + (int64_t)b * p.d_bstride + row * p.ldd + n0;
+            const __nv_bfloat16 *crow =
+                p.c != nullptr ? p.c + (int64_t)b * p.c_bstride + row * p.ldc + n0 : nullptr;
+#pragma unroll 1
+            for (int ch = 0; ch < BN / 32; ++ch) {
+                uint32_t r[32];
+                tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(ch * 32), r);
+                float v[32];
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                    v[j] = p.alpha * __uint_as_float(r[j]);
+                if (crow != nullptr) {
+#pragma unroll
+                    for (int j8 = 0; j8 < 4; ++j8) {
+                        const uint4 cv = *reinterpret_cast<const uint4 *>(crow + ch * 32 + j8 * 8);
+                        const __nv_bfloat162 *c2 = reinterpret_cast<const __nv_bfloat162 *>(&cv);
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const float2 f = __bfloat1622float2(c2[e]);
+                            v[j8 * 8 + 2 * e] = fmaf(p.beta, f.x, v[j8 * 8 + 2 * e]);
+                            v[j8 * 8 + 2 * e + 1] = fmaf(p.beta, f.y, v[j8 * 8 + 2 * e + 1]);
+                        }
+                    }
+                }
+#pragma unroll
+                for (int j8 = 0; j8 < 4; ++j8) {
+                    uint4 o;
+                    o.x = pack_bf16(v[j8 * 8 + 0], v[j8 * 8 + 1]);
+                    o.y = pack_bf16(v[j8 * 8 + 2], v[j8 * 8 + 3]);
+                    o.z = pack_bf16(v[j8 * 8 + 4], v[j8 * 8 + 5]);
+                    o.w = pack_bf16(v[j8 * 8 + 6], v[j8 * 8 + 7]);
+                    *reinterpret_cast<uint4 *>(drow + ch * 32 + j8 * 8) = o;
+                }
+                if (p.dt != nullptr) {
+                    __nv_bfloat16 *dcol = p.dt + (int64_t)b * p.dt_bstride +
+                                          (int64_t)(n0 + ch * 32) * p.ldt + row;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        dcol[(int64_t)j * p.ldt] = __float2bfloat16_rn(v[j]);
+                }
+            }
+        }
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    }
+    __syncthreads();
+    if (warp == 1) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                     "r"(kTmemCols)
+                     : "memory");
+    }
+}
+
+}  // namespace gemm
+}  // namespace dpo

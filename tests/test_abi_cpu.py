@@ -11,11 +11,11 @@ import re
 import pytest
 
 from paper_2606_30634_gb300 import build as pkg_build
-from paper_2606_30634_gb300 import dpo
+from paper_2606_30634_gb300 import dpo, muon
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
-HEADER_LIB = {"dpo.h": "libdpo.so", "dpo_synth.h": "libdpo_synth.so"}
+HEADER_LIB = {"dpo.h": "libdpo.so", "dpo_muon.h": "libdpo.so", "dpo_synth.h": "libdpo_synth.so"}
 
 
 def declared_functions(header: str):
@@ -53,6 +53,63 @@ def test_python_binding_wraps_every_dpo_entry_point():
     assert set(names) == set(dpo.EXPORTS)
     for n in names:
         assert callable(getattr(dpo, n))
+
+
+def test_python_binding_types_every_muon_entry_point():
+    names = declared_functions(os.path.join(ROOT, "include", "dpo_muon.h"))
+    assert set(names) == set(muon.EXPORTS)
+    L = muon.lib()
+    for n in names:
+        assert getattr(L, n).argtypes is not None
+
+
+# ---- dpo_muon_init host-side validation (returns before any CUDA call) ----
+
+def _m(i, rows=64, cols=96, **kw):
+    step = 1 << 20
+    b = BASE + (64 + i) * 16 * step
+    d = dict(param=b, master=b + step, mom=b + 2 * step, stash=b + 3 * step, ef=None,
+             grad=b + 4 * step, rows=rows, cols=cols, flags=dpo.DPO_WD_ON)
+    d.update(kw)
+    return muon.dpo_matrix(**d)
+
+
+def _muon_init(mats, hp=None, sdt=dpo.DPO_BF16, gdt=dpo.DPO_BF16, mode=0):
+    L = muon.lib()
+    arr = (muon.dpo_matrix * max(1, len(mats)))(*mats)
+    out = ctypes.c_void_p(123)
+    rc = L.dpo_muon_init(ctypes.byref(out), arr, len(mats), sdt, gdt,
+                         ctypes.byref(hp or muon.hparams()), mode, None)
+    return rc, out.value, L.dpo_muon_last_error(None).decode()
+
+
+@pytest.mark.parametrize("case,code", [
+    ("bad_dtype", dpo.DPO_EDTYPE), ("momentum_one", dpo.DPO_EINVAL),
+    ("ns_steps", dpo.DPO_EINVAL), ("negative_shape", dpo.DPO_EINVAL),
+    ("no_stash", dpo.DPO_EINVAL), ("ef_mismatch", dpo.DPO_EINVAL),
+    ("misaligned", dpo.DPO_EALIGN), ("no_master", dpo.DPO_EINVAL), ("bad_mode", dpo.DPO_EINVAL)])
+def test_muon_init_rejects(case, code):
+    mats, hp, kw = [_m(0), _m(1, rows=300, cols=20)], muon.hparams(), {}
+    if case == "bad_dtype":
+        kw["gdt"] = 7
+    elif case == "momentum_one":
+        hp = muon.hparams(momentum=1.0)
+    elif case == "ns_steps":
+        hp = muon.hparams(ns_steps=17)
+    elif case == "negative_shape":
+        mats[1] = _m(1, rows=-1)
+    elif case == "no_stash":
+        mats[0] = _m(0, stash=None)
+    elif case == "ef_mismatch":
+        mats[0] = _m(0, ef=BASE + (1 << 30))
+    elif case == "misaligned":
+        mats[1] = _m(1, master=BASE + (1 << 31) + 16)
+    elif case == "no_master":
+        mats[1] = _m(1, master=None)
+    elif case == "bad_mode":
+        kw["mode"] = 5
+    rc, out, msg = _muon_init(mats, hp, **kw)
+    assert rc == code and out is None and msg
 
 
 # ---- host-side validation (returns before any CUDA call) -----------------

@@ -1,0 +1,241 @@
+"""GPU parity of delayed Muon (Alg. 2): momentum, Newton-Schulz on the
+tcgen05 tensor cores, the delayed / EF update, stash and weights, through the
+C ABI (include/dpo_muon.h), against the oracle (oracle/muon.py).
+
+Newton-Schulz in bf16 is sensitive to its own rounding decisions: a product
+that lands within an fp32 accumulation error of a bf16 rounding boundary
+rounds the other way, and from the third step on such flips cascade. The
+oracle accumulates exactly and rounds every iterate to bf16 once; the kernels
+accumulate in fp32. The bars below come from running the two arithmetics side
+by side on the CPU (an fp32-accumulation emulation against the oracle, same
+inputs), with about 3x margin:
+  steps 0: identical except rare one-ulp flips of X_0
+  steps 1 / 2: normwise <= 2e-4 / 5e-4, differing elements <= 0.2% / 1%
+  steps 5: normwise <= 1.5e-2 (measured 4.7e-3 to 5.8e-3), singular values
+           within 5e-3 (measured <= 1.3e-3)
+The momentum does not depend on Newton-Schulz and is held to the one-step
+bar of the elementwise path.
+"""
+from __future__ import annotations
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from oracle.muon import DelayedMuon as OracleMuon, MuonHParams
+from paper_2606_30634_gb300 import dpo, muon, synth
+from parity_util import TOL_ONE_STEP, TOL_RUN, bf16_ulps, rel_err
+
+pytestmark = pytest.mark.gpu
+
+F, B = dpo.DPO_F32, dpo.DPO_BF16
+# wide, tall, ragged (padded to 256 inside), several tiles, tiny, empty
+SHAPES = [(256, 512), (512, 256), (300, 700), (64, 96), (1, 7), (0, 5), (768, 2304)]
+NS_BARS = {1: (2e-4, 2e-3), 2: (5e-4, 1e-2)}
+
+
+def inputs(shapes, seed, k):
+    """x_0 ~ N(0, 0.02^2) (fp32) and the k-th gradient ~ N(0, 1e-3^2) (bf16
+    bits), per matrix, from the seeded generator."""
+    xs, gs, off = [], [], 0
+    for r, c in shapes:
+        n = r * c
+        xs.append(synth.host_normal(seed, synth.STREAM_INIT, 0, off, n, 0.02).reshape(r, c))
+        gs.append(synth.host_normal(seed, synth.STREAM_GRAD, k, off, n, 1e-3,
+                                    synth.BF16).reshape(r, c))
+        off += n
+    return xs, gs
+
+
+def bf16_to_f64(bits):
+    return synth.bf16_bits_to_f32(np.asarray(bits)).astype(np.float64)
+
+
+class Pair:
+    """The GPU context and the oracle on the same seeded inputs."""
+
+    def __init__(self, shapes, device, seed=0x3A0, ns_steps=5, ef=True, delay=1, sdt=B,
+                 lr=2e-3, momentum=0.95, wd=0.1, max_grad_norm=0.0, rms_scale=0.2):
+        self.shapes, self.seed, self.lr = shapes, seed, lr
+        xs, _ = inputs(shapes, seed, 1)
+        self.gpu = muon.DelayedMuon(shapes, stash_dtype=sdt, grad_dtype=B, lr=lr,
+                                    momentum=momentum, weight_decay=wd, ef=ef,
+                                    max_grad_norm=max_grad_norm, rms_scale=rms_scale,
+                                    ns_steps=ns_steps, delay=delay, device=device,
+                                    x0=[torch.from_numpy(x) for x in xs])
+        hp = MuonHParams(lr=lr, momentum=momentum, weight_decay=wd, ef_lambda=1.0,
+                         ns_steps=ns_steps, rms_scale=rms_scale, ns_store=oracle.BF16,
+                         max_grad_norm=max_grad_norm, delay=delay).as_f32()
+        self.ref = OracleMuon([x.astype(np.float64) for x in xs], hp, ef=ef, x_store=oracle.F32,
+                              stash_store=oracle.BF16 if sdt == B else oracle.F32,
+                              param_store=oracle.BF16)
+        self.k = 0
+
+    def step(self):
+        self.k += 1
+        _, gs = inputs(self.shapes, self.seed, self.k + 1)
+        for i, g in enumerate(gs):
+            if g.size:
+                self.gpu.grads(i).copy_(torch.from_numpy(g.view(np.int16)).view(torch.bfloat16)
+                                        .reshape(g.shape))
+        self.gpu.step()
+        self.ref.step([bf16_to_f64(g) for g in gs])
+        torch.cuda.synchronize()
+
+    def cat(self, arena):
+        return np.concatenate([self.gpu.view(arena, i).float().cpu().numpy().ravel()
+                               for i in range(len(self.shapes))])
+
+    def o_pairs(self):
+        got = [self.gpu.last_update(i).float().cpu().numpy().astype(np.float64)
+               for i in range(len(self.shapes))]
+        return got, list(self.ref.o)
+
+    def close(self):
+        assert self.gpu.status() == 0, "a tensor-core pipeline wait gave up"
+        self.gpu.close()
+
+
+def _flat(a):
+    return np.concatenate([x.ravel() for x in a]) if a else np.zeros(0)
+
+
+def _ulp(v):
+    return np.exp2(np.floor(np.log2(np.maximum(np.abs(v), 2.0 ** -126))) - 7)
+
+
+@pytest.mark.parametrize("steps", [0, 1, 2, 5])
+def test_newton_schulz_parity(cuda_device, steps):
+    p = Pair(SHAPES, cuda_device, ns_steps=steps)
+    try:
+        p.step()
+        got, ref = p.o_pairs()
+        g, r = _flat(got), _flat(ref)
+        d = np.abs(g - r)
+        norm = np.linalg.norm(g - r) / np.linalg.norm(r)
+        frac = float(np.mean(d > 0))
+        print(f"steps {steps}: normwise {norm:.3e}, differing {frac:.4%}, "
+              f"max {d.max() / np.abs(r).max():.3e}")
+        if steps == 0:
+            assert frac <= 1e-3
+            assert np.all(d <= _ulp(r))
+        elif steps in NS_BARS:
+            assert norm <= NS_BARS[steps][0] and frac <= NS_BARS[steps][1]
+        else:
+            assert norm <= 1.5e-2
+            for gi, ri in zip(got, ref):
+                if gi.size:
+                    sg = np.linalg.svd(gi, compute_uv=False)
+                    sr = np.linalg.svd(ri, compute_uv=False)
+                    assert np.max(np.abs(sg - sr)) <= 5e-3
+        # the padding of every matrix stays out of the result: O has the
+        # matrix's shape and the momentum is the same as the oracle's
+        assert rel_err(p.cat(p.gpu.mom), _flat(p.ref.mom)) <= TOL_ONE_STEP
+    finally:
+        p.close()
+
+
+def close_with_flips(gpu, ref, tol, flip, max_frac):
+    """Elementwise at the floored bar ``tol`` except where a flipped bf16
+    rounding of O moved an element: at most ``max_frac`` of the elements may
+    miss the bar, and none by more than ``flip`` (absolute)."""
+    gpu, ref = np.asarray(gpu, np.float64), np.asarray(ref, np.float64)
+    d = np.abs(gpu - ref)
+    den = np.maximum(np.abs(ref), 1e-2 * np.sqrt(np.mean(ref * ref)))
+    bad = d > tol * den
+    assert np.mean(bad) <= max_frac, f"{np.mean(bad):.2e} of the elements off the bar"
+    assert np.all(d[bad] <= flip + tol * den[bad]), f"max miss {d[bad].max():.3e} > {flip:.3e}"
+
+
+@pytest.mark.parametrize("steps,sdt,ef,delay", [(0, B, True, 1), (1, F, True, 1), (1, B, False, 1),
+                                                (0, B, False, 0)])
+def test_muon_step_parity(cuda_device, steps, sdt, ef, delay):
+    """Four calls of Alg. 2 (EF from the second), every buffer checked after
+    each. The momentum does not depend on O: one-step bar, then the run bar
+    (the EMA rounds twice where the oracle rounds once). The weights, stash,
+    bf16 weights and update history are held elementwise to the run / one-ulp
+    bars except where a bf16 rounding of O flipped (see the module note):
+    such a flip moves U by at most lr r ulp(O) <= lr r 2^-7 (|O| < 2), and
+    the weights by that much per call so far."""
+    p = Pair(SHAPES, cuda_device, ns_steps=steps, ef=ef, delay=delay, sdt=sdt)
+    r_max = 0.2 * np.sqrt(max(max(sh) for sh in SHAPES))
+    du = p.lr * r_max * 2.0 ** -7
+    try:
+        for k in range(4):
+            p.step()
+            assert rel_err(p.cat(p.gpu.mom), _flat(p.ref.mom)) <= (TOL_ONE_STEP if k == 0
+                                                                    else TOL_RUN)
+            close_with_flips(p.cat(p.gpu.master), _flat(p.ref.x), TOL_RUN, (k + 1) * du, 1e-3)
+            vals = lambda a: p.cat(a).astype(np.float64)
+            ref_p = _flat(p.ref.param)
+            close_with_flips(vals(p.gpu.param), ref_p, 2.0 ** -7, (k + 1) * du, 1e-3)
+            if delay == 1:
+                close_with_flips(vals(p.gpu.stash), _flat(p.ref.stash),
+                                 2.0 ** -7 if sdt == B else TOL_RUN, k * du, 1e-3)
+            if ef and delay == 1:
+                close_with_flips(p.cat(p.gpu.ef), _flat(p.ref.u_prev), 1e-5, du, 2e-3)
+    finally:
+        p.close()
+
+
+def test_muon_clipping(cuda_device):
+    """Global clipping over all matrices scales the gradient before the
+    momentum (the norm of these gradients is ~1.3)."""
+    p = Pair(SHAPES, cuda_device, ns_steps=1, max_grad_norm=0.5)
+    try:
+        p.step()
+        assert p.ref.last_clip < 0.5
+        assert rel_err(p.cat(p.gpu.mom), _flat(p.ref.mom)) <= TOL_ONE_STEP
+    finally:
+        p.close()
+
+
+def test_muon_flops_and_workspace(cuda_device):
+    shapes = [(256, 512), (512, 256), (300, 700)]
+    m = muon.DelayedMuon(shapes, ns_steps=5, device=cuda_device)
+    try:
+        want = sum(2 * (2 * min(r, c) ** 2 * max(r, c) + min(r, c) ** 3) * 5 for r, c in shapes)
+        assert m.flops() == pytest.approx(want, rel=1e-12)
+        # (256, 512) and (512, 256) share the 256 x 512 group; (300, 700) pads to 512 x 768
+        ws = 2 * ((2 * (256 * 512 * 3 + 256 * 256 * 2)) + (512 * 768 * 3 + 512 * 512 * 2))
+        assert m.workspace_bytes() == ws
+    finally:
+        m.close()
+
+
+def test_muon_full_size_shapes(cuda_device):
+    """The Llama-7B matrix shapes (4096 x 4096, 11008 x 4096 tall, 4096 x
+    11008 wide): one call, then properties that hold at any size. The
+    momentum equals (1 - mu) g on sampled elements; O's singular values
+    follow the scalar quintic applied to those of M / ||M||_F (numpy-free:
+    torch.linalg.svdvals on the GPU in fp32) within 2e-2."""
+    shapes = [(4096, 4096), (11008, 4096), (4096, 11008)]
+    gpu = muon.DelayedMuon(shapes, ns_steps=5, ef=True, device=cuda_device)
+    try:
+        off = 0
+        for i, (r, c) in enumerate(shapes):
+            synth.dev_normal(0x7B, synth.STREAM_GRAD, 1, off, gpu.grads(i).view(-1), 1e-3)
+            off += r * c
+        gpu.step()
+        torch.cuda.synchronize()
+        assert gpu.status() == 0
+        a, b_, c_ = muon.NS_COEFFS
+        for i, (r, c) in enumerate(shapes):
+            m = gpu.view(gpu.mom, i)
+            g = gpu.grads(i).float()
+            idx = torch.randint(0, r * c, (4096,), generator=torch.Generator().manual_seed(i))
+            mg = m.reshape(-1)[idx.to(m.device)].double()
+            want = (g.reshape(-1)[idx.to(m.device)].double() *
+                    float(np.float32(1.0) - np.float32(0.95)))
+            assert torch.max(torch.abs(mg - want) / torch.abs(want).clamp_min(1e-12)) <= 1e-6
+            s = torch.linalg.svdvals(m.double() if r * c <= (1 << 24) else m).double()
+            x = s / (torch.linalg.norm(s) + 1e-7)
+            for _ in range(5):
+                x = a * x + b_ * x ** 3 + c_ * x ** 5
+            so = torch.linalg.svdvals(gpu.last_update(i).float()).double()
+            err = torch.max(torch.abs(torch.sort(so).values - torch.sort(x).values)).item()
+            print(f"{r}x{c}: singular values within {err:.3e}")
+            assert err <= 2e-2
+    finally:
+        gpu.close()
