@@ -124,9 +124,10 @@ int dpo_muon_get_step(const dpo_muon_ctx *ctx, int64_t *k);
 int dpo_muon_set_step(dpo_muon_ctx *ctx, int64_t k);
 
 /*
- * Tensor-core work of one step: 2 (2 r^2 w + r^3) ns_steps summed over the
- * matrices (r x w the orientation with r <= w), counting the multiply-adds
- * of the unpadded shapes as two flops.
+ * Tensor-core work of one step, summed over the matrices (r x w the
+ * orientation with r <= w, unpadded), two flops per multiply-add:
+ * ns_steps (r (r + 1) w + r (r + 1) r + 2 r^2 w), the first two terms being
+ * the unique entries of the symmetric products X X^T and A A.
  */
 int dpo_muon_flops(const dpo_muon_ctx *ctx, double *flops);
 

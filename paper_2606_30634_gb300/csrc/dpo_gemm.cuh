@@ -8,16 +8,22 @@
 // to bf16. Every dimension is a multiple of the tile (the Newton-Schulz
 // scratch is padded with zeros to multiples of 256), so no tile is partial.
 //
-// One CTA computes one 128 x 256 tile of one batch entry:
+// A persistent grid (one CTA per SM) walks the 128 x 256 output tiles:
 //   warp 0      TMA producer: 128 x 64 and 256 x 64 bf16 boxes (128-byte
 //               swizzle) into a 4-stage shared-memory ring;
-//   warp 1      allocates 256 TMEM columns; one lane issues
-//               tcgen05.mma.cta_group::1.kind::f16 (M 128, N 256, K 16) four
-//               times per stage and commits each stage back to the producer;
+//   warp 1      allocates 512 TMEM columns (two accumulators); one lane
+//               issues tcgen05.mma.cta_group::1.kind::f16 (M 128, N 256, K 16)
+//               four times per stage, commits each stage back to the
+//               producer and each finished tile to the epilogue;
 //   warps 2-5   epilogue: tcgen05.ld 32 lanes x 32 columns at a time, scale,
 //               add the addend, round to bf16, store row-major (16-byte
 //               stores) and, when asked, transposed (each warp writes 64
 //               contiguous bytes per column).
+// Symmetric products (Params::sym; X X^T and c A A + b A): only tiles that
+// reach the upper triangle (n0 + BN > m0) are computed; each of their
+// elements (i, j) is also stored at (j, i) when the tile holding (j, i) is
+// not computed. Every element is then written exactly once, by one thread,
+// and the result does not depend on scheduling.
 // Every wait on an mbarrier gives up after kWaitNs, records an error code and
 // lets the CTA finish (draining its own TMA loads first), so a fault in the
 // pipeline surfaces as a status instead of a hang.
@@ -39,7 +45,7 @@ constexpr int kStageBytes = kABytes + kBBytes;       // 48 KiB
 constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256;
 constexpr unsigned long long kWaitNs = 1000000000ull;  // 1 s per wait
 
-// Error codes OR-ed into Params::err.
+// Error codes OR-ed into Params::err (kErrWaitDone: an accumulator hand-off).
 constexpr unsigned int kErrWaitFull = 1u, kErrWaitEmpty = 2u, kErrWaitDone = 4u,
                        kErrDrain = 8u;
 
@@ -52,6 +58,7 @@ struct Params {
     int64_t ldc, c_bstride;
     float alpha, beta;
     int k_blocks;                 // K / BK
+    int sym;                      // D is symmetric (M == N): see ns_gemm_kernel
     unsigned int *err;
 };
 
@@ -163,41 +170,63 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
     return *reinterpret_cast<const uint32_t *>(&h);
 }
 
+// Tile t of a launch: batch entry, row block and column block, columns
+// fastest (consecutive CTAs share the A rows of a block row in L2).
+struct TileGrid {
+    int m_tiles, n_tiles, nb;
+    __device__ __forceinline__ int count() const { return m_tiles * n_tiles * nb; }
+    __device__ __forceinline__ void at(int t, int &b, int &m0, int &n0) const
+    {
+        n0 = (t % n_tiles) * BN;
+        t /= n_tiles;
+        m0 = (t % m_tiles) * BM;
+        b = t / m_tiles;
+    }
+};
+
+__device__ __forceinline__ bool tile_skipped(const Params &p, int m0, int n0)
+{
+    return p.sym && n0 + BN <= m0;   // strictly below the diagonal: mirrored
+}
+
+// Persistent: CTA c takes tiles c, c + gridDim.x, ... Two accumulators in
+// TMEM (columns 0-255 and 256-511) let the MMA lane fill one while the
+// epilogue warps drain the other.
 __global__ void __launch_bounds__(kThreads, 1)
     ns_gemm_kernel(const __grid_constant__ CUtensorMap tma_a,
-                   const __grid_constant__ CUtensorMap tma_b, const Params p)
+                   const __grid_constant__ CUtensorMap tma_b, const Params p, const TileGrid tg)
 {
     extern __shared__ uint8_t smem_raw[];
-    __shared__ uint64_t bars[2 * kStages + 1];
+    __shared__ uint64_t bars[2 * kStages + 4];
     __shared__ uint32_t tmem_slot;
     __shared__ int aborted;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM, b = blockIdx.z;
-
-    // 1024-byte aligned operand ring (the 128-byte swizzle repeats every
-    // 1024 bytes and the descriptors assume that alignment).
     const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
-    const uint32_t ring = (raw + 1023u) & ~1023u;
+    const uint32_t ring = (raw + 1023u) & ~1023u;   // the swizzle atoms repeat every 1024 B
     const uint32_t sa = ring, sb = ring + kStages * kABytes;
     const uint32_t bar0 = (uint32_t)__cvta_generic_to_shared(bars);
     auto full = [&](int s) { return bar0 + 8u * (uint32_t)s; };
     auto empty = [&](int s) { return bar0 + 8u * (uint32_t)(kStages + s); };
-    const uint32_t done = bar0 + 8u * (uint32_t)(2 * kStages);
+    auto acc_full = [&](int a) { return bar0 + 8u * (uint32_t)(2 * kStages + a); };
+    auto acc_empty = [&](int a) { return bar0 + 8u * (uint32_t)(2 * kStages + 2 + a); };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(full(s), 1);
             mbar_init(empty(s), 1);
         }
-        mbar_init(done, 1);
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(acc_full(a), 1);
+            mbar_init(acc_empty(a), 4);   // one arrival per epilogue warp
+        }
         aborted = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          (uint32_t)__cvta_generic_to_shared(&tmem_slot)),
-                     "r"(kTmemCols)
+                     "r"(2 * kTmemCols)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
@@ -206,6 +235,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = tmem_slot;
     const int kb_n = p.k_blocks;
+    const int n_tiles = tg.count();
 
     if (warp == 0) {
         if (lane == 0) {
@@ -213,65 +243,98 @@ __global__ void __launch_bounds__(kThreads, 1)
                          : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tma_b))
                          : "memory");
-            int issued = 0;
-            for (int kb = 0; kb < kb_n; ++kb) {
-                const int s = kb % kStages;
-                const uint32_t ph = (uint32_t)(kb / kStages) & 1u;
-                if (!mbar_wait(empty(s), ph ^ 1u) || *(volatile int *)&aborted) {
-                    atomicOr(p.err, kErrWaitEmpty);
-                    aborted = 1;
-                    break;
+            int it = 0;   // k-blocks issued by this CTA
+            for (int t = blockIdx.x; t < n_tiles && !*(volatile int *)&aborted; t += gridDim.x) {
+                int b, m0, n0;
+                tg.at(t, b, m0, n0);
+                if (tile_skipped(p, m0, n0))
+                    continue;
+                for (int kb = 0; kb < kb_n; ++kb, ++it) {
+                    const int s = it % kStages;
+                    const uint32_t ph = (uint32_t)(it / kStages) & 1u;
+                    if (!mbar_wait(empty(s), ph ^ 1u) || *(volatile int *)&aborted) {
+                        atomicOr(p.err, kErrWaitEmpty);
+                        aborted = 1;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(full(s), (uint32_t)kStageBytes);
+                    tma_load_3d(sa + (uint32_t)(s * kABytes), &tma_a, kb * BK, m0, b, full(s));
+                    tma_load_3d(sb + (uint32_t)(s * kBBytes), &tma_b, kb * BK, n0, b, full(s));
                 }
-                mbar_arrive_expect_tx(full(s), (uint32_t)kStageBytes);
-                tma_load_3d(sa + (uint32_t)(s * kABytes), &tma_a, kb * BK, m0, b, full(s));
-                tma_load_3d(sb + (uint32_t)(s * kBBytes), &tma_b, kb * BK, n0, b, full(s));
-                issued = kb + 1;
             }
-            // Drain: every load this thread issued lands before the CTA ends
-            // (normally the MMA warp has consumed them all already).
-            for (int kb = issued - kStages < 0 ? 0 : issued - kStages; kb < issued; ++kb)
-                if (!mbar_wait(full(kb % kStages), (uint32_t)(kb / kStages) & 1u))
+            // Drain: every load issued lands before the CTA ends.
+            for (int q = it - kStages < 0 ? 0 : it - kStages; q < it; ++q)
+                if (!mbar_wait(full(q % kStages), (uint32_t)(q / kStages) & 1u))
                     atomicOr(p.err, kErrDrain);
         }
     } else if (warp == 1) {
         if (lane == 0) {
-            for (int kb = 0; kb < kb_n; ++kb) {
-                const int s = kb % kStages;
-                const uint32_t ph = (uint32_t)(kb / kStages) & 1u;
-                if (!mbar_wait(full(s), ph) || *(volatile int *)&aborted) {
-                    atomicOr(p.err, kErrWaitFull);
+            int it = 0, lt = 0;   // k-blocks consumed, tiles accumulated
+            for (int t = blockIdx.x; t < n_tiles && !*(volatile int *)&aborted; t += gridDim.x) {
+                int b, m0, n0;
+                tg.at(t, b, m0, n0);
+                if (tile_skipped(p, m0, n0))
+                    continue;
+                const int a = lt & 1;
+                const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
+                if (!mbar_wait(acc_empty(a), aph ^ 1u)) {
+                    atomicOr(p.err, kErrWaitDone);
                     aborted = 1;
                     break;
                 }
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint32_t d = tmem + (uint32_t)(a * (int)kTmemCols);
+                bool ok = true;
+                for (int kb = 0; kb < kb_n; ++kb, ++it) {
+                    const int s = it % kStages;
+                    const uint32_t ph = (uint32_t)(it / kStages) & 1u;
+                    if (!mbar_wait(full(s), ph) || *(volatile int *)&aborted) {
+                        atomicOr(p.err, kErrWaitFull);
+                        aborted = 1;
+                        ok = false;
+                        break;
+                    }
+                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 #pragma unroll
-                for (int k = 0; k < BK / 16; ++k) {
-                    const uint64_t ad = smem_desc(sa + (uint32_t)(s * kABytes + k * 32));
-                    const uint64_t bd = smem_desc(sb + (uint32_t)(s * kBBytes + k * 32));
-                    mma_bf16(tmem, ad, bd, (kb | k) != 0 ? 1u : 0u);
+                    for (int k = 0; k < BK / 16; ++k) {
+                        const uint64_t ad = smem_desc(sa + (uint32_t)(s * kABytes + k * 32));
+                        const uint64_t bd = smem_desc(sb + (uint32_t)(s * kBBytes + k * 32));
+                        mma_bf16(d, ad, bd, (kb | k) != 0 ? 1u : 0u);
+                    }
+                    mma_commit(empty(s));
                 }
-                mma_commit(empty(s));
+                mma_commit(acc_full(a));   // arrives when this tile's MMAs have completed
+                ++lt;
+                if (!ok)
+                    break;
             }
-            mma_commit(done);   // arrives when every MMA issued above has completed
         }
     } else {
         // Epilogue: warp w reads TMEM lanes 32 (w % 4) .. +31 = tile rows.
         const int q = warp & 3;
-        const bool seen = mbar_wait(done, 0u);
-        if (!seen)
-            atomicOr(p.err, kErrWaitDone);
-        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        // tcgen05.ld is warp-collective: the whole warp goes on, or none of it.
-        const bool ok = __all_sync(0xFFFFFFFFu, seen && !*(volatile int *)&aborted);
-        if (ok) {
+        int lt = 0;
+        for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) {
+            int b, m0, n0;
+            tg.at(t, b, m0, n0);
+            if (tile_skipped(p, m0, n0))
+                continue;
+            const int a = lt & 1;
+            const bool seen = mbar_wait(acc_full(a), (uint32_t)(lt >> 1) & 1u);
+            if (!seen)
+                atomicOr(p.err, kErrWaitDone);
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            // tcgen05.ld is warp-collective: the whole warp goes on, or none of it.
+            if (!__all_sync(0xFFFFFFFFu, seen && !*(volatile int *)&aborted))
+                break;
             const int64_t row = m0 + q * 32 + lane;
             __nv_bfloat16 *drow = p.d + (int64_t)b * p.d_bstride + row * p.ldd + n0;
             const __nv_bfloat16 *crow =
                 p.c != nullptr ? p.c + (int64_t)b * p.c_bstride + row * p.ldc + n0 : nullptr;
+            const uint32_t acc = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(a * (int)kTmemCols);
 #pragma unroll 1
             for (int ch = 0; ch < BN / 32; ++ch) {
                 uint32_t r[32];
-                tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(ch * 32), r);
+                tmem_ld32(acc + (uint32_t)(ch * 32), r);
                 float v[32];
 #pragma unroll
                 for (int j = 0; j < 32; ++j)
@@ -305,7 +368,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int j = 0; j < 32; ++j)
                         dcol[(int64_t)j * p.ldt] = __float2bfloat16_rn(v[j]);
                 }
+                // Mirror of a symmetric product: (col, row) lies in the tile
+                // (col / BM, row / BN), skipped when row / BN * BN + BN <= col / BM * BM.
+                // Uniform over the warp (its rows share row / BN) and the
+                // 32-column chunk (its columns share col / BM).
+                if (p.sym && (int64_t)(row / BN) * BN + BN <= (int64_t)((n0 + ch * 32) / BM) * BM) {
+                    __nv_bfloat16 *dcol = p.d + (int64_t)b * p.d_bstride +
+                                          (int64_t)(n0 + ch * 32) * p.ldd + row;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        dcol[(int64_t)j * p.ldd] = __float2bfloat16_rn(v[j]);
+                }
             }
+            // this warp's rows of the accumulator are read: release it
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncwarp();
+            if (lane == 0)
+                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(acc_empty(a))
+                             : "memory");
+            ++lt;
         }
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     }
@@ -313,7 +394,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 1) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
-                     "r"(kTmemCols)
+                     "r"(2 * kTmemCols)
                      : "memory");
     }
 }

@@ -503,7 +503,10 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
             c->groups.push_back(g);
         }
         c->groups[gidx[key]].mats.push_back(i);
-        c->flops += 2.0 * (2.0 * (double)r * r * w + (double)r * r * r) * hp->ns_steps;
+        // unique entries of the symmetric products X X^T (r (r + 1) / 2, each
+        // w multiply-adds) and A A (r (r + 1) / 2, r each), all of B X
+        c->flops += (double)hp->ns_steps * ((double)r * (r + 1) * w + (double)r * (r + 1) * r +
+                                            2.0 * (double)r * r * w);
     }
     c->chunks = (int)std::max<int64_t>(1, (max_n + kChunk - 1) / kChunk);
 
@@ -696,8 +699,11 @@ namespace {
 int launch_gemm(dpo_muon_ctx *c, const CUtensorMap &ta, const CUtensorMap &tb,
                 const dpo::gemm::Params &p, int64_t M, int64_t N, int64_t nb, cudaStream_t s)
 {
-    const dim3 grid((unsigned)(N / dpo::gemm::BN), (unsigned)(M / dpo::gemm::BM), (unsigned)nb);
-    dpo::gemm::ns_gemm_kernel<<<grid, dpo::gemm::kThreads, dpo::gemm::kSmemBytes, s>>>(ta, tb, p);
+    dpo::gemm::TileGrid tg{(int)(M / dpo::gemm::BM), (int)(N / dpo::gemm::BN), (int)nb};
+    const int64_t tiles = (int64_t)tg.m_tiles * tg.n_tiles * tg.nb;
+    const int grid = (int)std::min<int64_t>(tiles, std::max(1, c->sms));   // one CTA per SM
+    dpo::gemm::ns_gemm_kernel<<<grid, dpo::gemm::kThreads, dpo::gemm::kSmemBytes, s>>>(ta, tb, p,
+                                                                                       tg);
     const cudaError_t e = cudaGetLastError();
     return e == cudaSuccess ? DPO_OK : mcuda(c, e, "Newton-Schulz GEMM launch");
 }
@@ -784,6 +790,7 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
             p.d_bstride = g.R * g.R;
             p.alpha = 1.0f;
             p.k_blocks = (int)(g.W / dpo::gemm::BK);
+            p.sym = 1;
             int rc = launch_gemm(c, g.x128, g.x256, p, g.R, g.R, nb, s);
             if (rc != DPO_OK)
                 return rc;
@@ -798,6 +805,7 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
             if ((rc = launch_gemm(c, g.a128, g.a256, p, g.R, g.R, nb, s)) != DPO_OK)
                 return rc;
             // X <- B X + a X, and X^T
+            p.sym = 0;
             p.d = g.x;
             p.ldd = g.W;
             p.d_bstride = g.R * g.W;

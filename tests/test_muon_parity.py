@@ -195,7 +195,8 @@ def test_muon_flops_and_workspace(cuda_device):
     shapes = [(256, 512), (512, 256), (300, 700)]
     m = muon.DelayedMuon(shapes, ns_steps=5, device=cuda_device)
     try:
-        want = sum(2 * (2 * min(r, c) ** 2 * max(r, c) + min(r, c) ** 3) * 5 for r, c in shapes)
+        want = sum(5 * (a * (a + 1) * b + a * (a + 1) * a + 2 * a * a * b)
+                   for a, b in ((min(r, c), max(r, c)) for r, c in shapes))
         assert m.flops() == pytest.approx(want, rel=1e-12)
         # (256, 512) and (512, 256) share the 256 x 512 group; (300, 700) pads to 512 x 768
         ws = 2 * ((2 * (256 * 512 * 3 + 256 * 256 * 2)) + (512 * 768 * 3 + 512 * 512 * 2))
