@@ -31,8 +31,8 @@
  * Layout and ownership. The caller owns every buffer of a dpo_matrix: device
  * memory of the current device, row-major, 32-byte aligned, no overlaps, kept
  * alive and in place until dpo_muon_destroy. The library allocates, in
- * dpo_muon_init, the Newton-Schulz workspace (bf16, for every matrix: the
- * iterate and its transpose twice, and two Gram-sized matrices, each
+ * dpo_muon_init, the Newton-Schulz workspace (bf16, for every matrix: two
+ * copies of the iterate, its transpose and two Gram-sized matrices, each
  * dimension padded to a multiple of 256) plus a small table; no other call
  * allocates or synchronizes the host. All launches go to the stream passed in.
  *

@@ -8,19 +8,25 @@
 // to bf16. Every dimension is a multiple of the tile (the Newton-Schulz
 // scratch is padded with zeros to multiples of 256), so no tile is partial.
 //
-// A persistent grid (one CTA per SM) walks the 128 x 256 output tiles:
-//   warp 0      TMA producer: 128 x 64 and 256 x 64 bf16 boxes (128-byte
-//               swizzle) into a 4-stage shared-memory ring;
-//   warp 1      allocates 512 TMEM columns (two accumulators); one lane
-//               issues tcgen05.mma.cta_group::1.kind::f16 (M 128, N 256, K 16)
-//               four times per stage, commits each stage back to the
-//               producer and each finished tile to the epilogue;
-//   warps 2-5   epilogue: tcgen05.ld 32 lanes x 32 columns at a time, scale,
-//               add the addend, round to bf16, store row-major (16-byte
-//               stores) and, when asked, transposed (each warp writes 64
-//               contiguous bytes per column).
+// A persistent grid of CTA pairs (clusters of 2, one CTA per SM) walks the
+// 256 x 256 output tiles with the 2-SM MMA. In each CTA:
+//   warp 0      TMA producer: this CTA's 128 x 64 half of the A block and
+//               128 x 64 half of the B block (bf16, 128-byte swizzle) into a
+//               6-stage ring, completing on the leader CTA's mbarrier;
+//   warp 1      allocates 512 TMEM columns (two accumulators) together with
+//               the peer; in the leader, one lane issues
+//               tcgen05.mma.cta_group::2.kind::f16 (M 256, N 256, K 16) four
+//               times per stage, reading both CTAs' halves, and commits each
+//               stage and each finished tile to both CTAs;
+//   warps 2-5   epilogue of this CTA's 128 rows: tcgen05.ld 32 lanes x 32
+//               columns at a time, scale, add the addend, round to bf16,
+//               store row-major (16-byte stores) and, when asked,
+//               transposed (each warp writes 64 contiguous bytes per column).
+// Per CTA a stage is 32 KiB for 4.2 MFLOP, a third less than one SM holding
+// a whole 128 x 256 operand pair, so six stages fit and keep the tensor pipe
+// fed across the L2 / DRAM round trip.
 // Symmetric products (Params::sym; X X^T and c A A + b A): only tiles that
-// reach the upper triangle (n0 + BN > m0) are computed; each of their
+// reach the upper triangle (n0 + TN > m0) are computed; each of their
 // elements (i, j) is also stored at (j, i) when the tile holding (j, i) is
 // not computed. Every element is then written exactly once, by one thread,
 // and the result does not depend on scheduling.
@@ -36,13 +42,17 @@
 namespace dpo {
 namespace gemm {
 
-constexpr int BM = 128, BN = 256, BK = 64, kStages = 4;
+// A CTA pair (a cluster of 2) computes one TM x TN output tile with the
+// 2-SM MMA: each CTA holds BM = TM / 2 rows of A and BH = TN / 2 rows of B
+// per stage, and its TMEM holds its BM rows of the accumulator.
+constexpr int TM = 256, TN = 256, BM = 128, BH = 128, BK = 64, kStages = 6;
 constexpr int kThreads = 192;
-constexpr uint32_t kTmemCols = 256;
+constexpr uint32_t kTmemCols = 256;                  // one accumulator (fp32, TN columns)
 constexpr int kABytes = BM * BK * 2;                 // 16 KiB
-constexpr int kBBytes = BN * BK * 2;                 // 32 KiB
-constexpr int kStageBytes = kABytes + kBBytes;       // 48 KiB
-constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256;
+constexpr int kBBytes = BH * BK * 2;                 // 16 KiB
+constexpr int kStageBytes = kABytes + kBBytes;       // 32 KiB per CTA
+// ring + 1024-byte alignment slack + 16 KiB kept free behind the ring
+constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 16384;
 constexpr unsigned long long kWaitNs = 1000000000ull;  // 1 s per wait
 
 // Error codes OR-ed into Params::err (kErrWaitDone: an accumulator hand-off).
@@ -105,14 +115,43 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t byt
                  : "memory");
 }
 
+// TMA tile load into this CTA's shared memory; the mbarrier (a shared::cluster
+// address) may belong to either CTA of the pair.
 __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, int x, int y,
-                                            int z, uint32_t bar)
+                                            int z, uint32_t bar_cluster)
 {
     asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
         " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar_cluster)
         : "memory");
+}
+
+__device__ __forceinline__ uint32_t cluster_rank()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// shared::cluster address of the same shared::cta offset in CTA `rank`
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank)
+{
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster)
+{
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster)
+                 : "memory");
+}
+
+__device__ __forceinline__ void cluster_sync()
+{
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
 // Shared-memory matrix descriptor of a K-major operand tile stored as rows of
@@ -126,25 +165,43 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t addr)
            ((uint64_t)(1024 >> 4) << 32) | (1ull << 46) | (2ull << 61);
 }
 
-// Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, both
-// K-major, N = BN, M = BM.
-constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
-                            ((uint32_t)(BM >> 4) << 24);
+// Shared-memory descriptor of an MN-major operand tile: rows of 64 bf16
+// (128 bytes) along N with the 128-byte swizzle, one row per K index, 8-row
+// K groups 1024 bytes apart (stride byte offset), and the second 64-column
+// N chunk 8192 bytes further (leading byte offset: one 64-row TMA box).
+__device__ __forceinline__ uint64_t smem_desc_mn(uint32_t addr)
+{
+    return (uint64_t)((addr & 0x3FFFFu) >> 4) | ((uint64_t)(8192 >> 4) << 16) |
+           ((uint64_t)(1024 >> 4) << 32) | (1ull << 46) | (2ull << 61);
+}
 
+// Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, A
+// K-major, N = TN, M = TM (the pair's 2-SM shape); B K-major, or MN-major
+// with bit 16 (B read as stored row-major along N).
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(TN >> 3) << 17) |
+                            ((uint32_t)(TM >> 4) << 24);
+constexpr uint32_t kIdescBmn = kIdesc | (1u << 16);
+
+// One TM x TN x 16 step of the pair, issued by the leader CTA: A rows from
+// both CTAs' shared memory at the descriptor's offset, B likewise, the
+// accumulator rows in each CTA's TMEM.
 __device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t a_desc, uint64_t b_desc,
-                                         uint32_t accumulate)
+                                         uint32_t idesc, uint32_t accumulate)
 {
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
-        "l"(a_desc), "l"(b_desc), "r"(kIdesc), "r"(accumulate));
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate));
 }
 
-__device__ __forceinline__ void mma_commit(uint32_t bar)
+// Arrive on the mbarrier at this shared::cta offset in both CTAs of the pair
+// once the leader's MMAs issued so far have completed.
+__device__ __forceinline__ void mma_commit_pair(uint32_t bar)
 {
     asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+        " [%0], %1;" ::"r"(bar), "h"((uint16_t)0x3)
         : "memory");
 }
 
@@ -171,28 +228,37 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
 }
 
 // Tile t of a launch: batch entry, row block and column block, columns
-// fastest (consecutive CTAs share the A rows of a block row in L2).
+// fastest (consecutive pairs share the A rows of a block row in L2).
 struct TileGrid {
     int m_tiles, n_tiles, nb;
     __device__ __forceinline__ int count() const { return m_tiles * n_tiles * nb; }
     __device__ __forceinline__ void at(int t, int &b, int &m0, int &n0) const
     {
-        n0 = (t % n_tiles) * BN;
+        n0 = (t % n_tiles) * TN;
         t /= n_tiles;
-        m0 = (t % m_tiles) * BM;
+        m0 = (t % m_tiles) * TM;
         b = t / m_tiles;
     }
 };
 
 __device__ __forceinline__ bool tile_skipped(const Params &p, int m0, int n0)
 {
-    return p.sym && n0 + BN <= m0;   // strictly below the diagonal: mirrored
+    return p.sym && n0 + TN <= m0;   // strictly below the diagonal: mirrored
 }
 
-// Persistent: CTA c takes tiles c, c + gridDim.x, ... Two accumulators in
-// TMEM (columns 0-255 and 256-511) let the MMA lane fill one while the
-// epilogue warps drain the other.
-__global__ void __launch_bounds__(kThreads, 1)
+// Persistent: the CTA pairs (clusters of 2) take tiles c, c + pairs, ...
+// Within a pair, rank 0 (the leader) issues the MMAs; both ranks load their
+// halves of A and B and drain their own accumulator rows. Two accumulators
+// in TMEM (columns 0-255 and 256-511) let the MMA fill one while the
+// epilogues drain the other.
+//   full[s]      (leader) both ranks' TMA bytes of stage s have landed
+//   empty[s]     (each)   the leader's MMAs have finished reading stage s
+//   acc_full[a]  (each)   accumulator a holds a finished tile
+//   acc_empty[a] (leader) all 8 epilogue warps of the pair have read it
+// BMN: the B operand is stored N-contiguous (a row-major K x N matrix) and
+// loaded as two 64 x 64 boxes per stage, read MN-major by the MMA.
+template <bool BMN>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     ns_gemm_kernel(const __grid_constant__ CUtensorMap tma_a,
                    const __grid_constant__ CUtensorMap tma_b, const Params p, const TileGrid tg)
 {
@@ -202,6 +268,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     __shared__ int aborted;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_rank();
+    const bool leader = rank == 0;
+    const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
     const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
     const uint32_t ring = (raw + 1023u) & ~1023u;   // the swizzle atoms repeat every 1024 B
     const uint32_t sa = ring, sb = ring + kStages * kABytes;
@@ -218,20 +287,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(acc_full(a), 1);
-            mbar_init(acc_empty(a), 4);   // one arrival per epilogue warp
+            mbar_init(acc_empty(a), 8);   // one arrival per epilogue warp of the pair
         }
         aborted = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    if (warp == 1) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+    if (warp == 1) {   // both CTAs of the pair allocate together
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          (uint32_t)__cvta_generic_to_shared(&tmem_slot)),
                      "r"(2 * kTmemCols)
                      : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-    __syncthreads();
+    cluster_sync();   // barriers of both CTAs initialised before any remote use
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = tmem_slot;
     const int kb_n = p.k_blocks;
@@ -244,11 +313,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tma_b))
                          : "memory");
             int it = 0;   // k-blocks issued by this CTA
-            for (int t = blockIdx.x; t < n_tiles && !*(volatile int *)&aborted; t += gridDim.x) {
+            for (int t = pair; t < n_tiles && !*(volatile int *)&aborted; t += n_pairs) {
                 int b, m0, n0;
                 tg.at(t, b, m0, n0);
                 if (tile_skipped(p, m0, n0))
                     continue;
+                const int ma = m0 + (int)rank * BM, nb_ = n0 + (int)rank * BH;
                 for (int kb = 0; kb < kb_n; ++kb, ++it) {
                     const int s = it % kStages;
                     const uint32_t ph = (uint32_t)(it / kStages) & 1u;
@@ -257,20 +327,31 @@ __global__ void __launch_bounds__(kThreads, 1)
                         aborted = 1;
                         break;
                     }
-                    mbar_arrive_expect_tx(full(s), (uint32_t)kStageBytes);
-                    tma_load_3d(sa + (uint32_t)(s * kABytes), &tma_a, kb * BK, m0, b, full(s));
-                    tma_load_3d(sb + (uint32_t)(s * kBBytes), &tma_b, kb * BK, n0, b, full(s));
+                    const uint32_t fbar = map_to_rank(full(s), 0);
+                    if (leader)   // the leader's barrier counts both CTAs' bytes
+                        mbar_arrive_expect_tx(full(s), (uint32_t)(2 * kStageBytes));
+                    tma_load_3d(sa + (uint32_t)(s * kABytes), &tma_a, kb * BK, ma, b, fbar);
+                    if (BMN) {
+                        tma_load_3d(sb + (uint32_t)(s * kBBytes), &tma_b, nb_, kb * BK, b, fbar);
+                        tma_load_3d(sb + (uint32_t)(s * kBBytes + kBBytes / 2), &tma_b, nb_ + 64,
+                                    kb * BK, b, fbar);
+                    } else {
+                        tma_load_3d(sb + (uint32_t)(s * kBBytes), &tma_b, kb * BK, nb_, b, fbar);
+                    }
                 }
             }
-            // Drain: every load issued lands before the CTA ends.
-            for (int q = it - kStages < 0 ? 0 : it - kStages; q < it; ++q)
-                if (!mbar_wait(full(q % kStages), (uint32_t)(q / kStages) & 1u))
-                    atomicOr(p.err, kErrDrain);
+            // Drain (leader): every stage issued by either CTA has landed
+            // before the pair leaves (the peer waits at the final cluster
+            // barrier for this).
+            if (leader)
+                for (int q = it - kStages < 0 ? 0 : it - kStages; q < it; ++q)
+                    if (!mbar_wait(full(q % kStages), (uint32_t)(q / kStages) & 1u))
+                        atomicOr(p.err, kErrDrain);
         }
     } else if (warp == 1) {
-        if (lane == 0) {
+        if (lane == 0 && leader) {
             int it = 0, lt = 0;   // k-blocks consumed, tiles accumulated
-            for (int t = blockIdx.x; t < n_tiles && !*(volatile int *)&aborted; t += gridDim.x) {
+            for (int t = pair; t < n_tiles && !*(volatile int *)&aborted; t += n_pairs) {
                 int b, m0, n0;
                 tg.at(t, b, m0, n0);
                 if (tile_skipped(p, m0, n0))
@@ -298,22 +379,25 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int k = 0; k < BK / 16; ++k) {
                         const uint64_t ad = smem_desc(sa + (uint32_t)(s * kABytes + k * 32));
-                        const uint64_t bd = smem_desc(sb + (uint32_t)(s * kBBytes + k * 32));
-                        mma_bf16(d, ad, bd, (kb | k) != 0 ? 1u : 0u);
+                        const uint64_t bd =
+                            BMN ? smem_desc_mn(sb + (uint32_t)(s * kBBytes + k * 16 * 128))
+                                : smem_desc(sb + (uint32_t)(s * kBBytes + k * 32));
+                        mma_bf16(d, ad, bd, BMN ? kIdescBmn : kIdesc, (kb | k) != 0 ? 1u : 0u);
                     }
-                    mma_commit(empty(s));
+                    mma_commit_pair(empty(s));
                 }
-                mma_commit(acc_full(a));   // arrives when this tile's MMAs have completed
+                mma_commit_pair(acc_full(a));   // when this tile's MMAs have completed
                 ++lt;
                 if (!ok)
                     break;
             }
         }
     } else {
-        // Epilogue: warp w reads TMEM lanes 32 (w % 4) .. +31 = tile rows.
+        // Epilogue: warp w reads TMEM lanes 32 (w % 4) .. +31 = this CTA's
+        // tile rows m0 + BM rank + 32 (w % 4) + lane.
         const int q = warp & 3;
         int lt = 0;
-        for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) {
+        for (int t = pair; t < n_tiles; t += n_pairs) {
             int b, m0, n0;
             tg.at(t, b, m0, n0);
             if (tile_skipped(p, m0, n0))
@@ -326,13 +410,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             // tcgen05.ld is warp-collective: the whole warp goes on, or none of it.
             if (!__all_sync(0xFFFFFFFFu, seen && !*(volatile int *)&aborted))
                 break;
-            const int64_t row = m0 + q * 32 + lane;
+            const int64_t row = m0 + (int)rank * BM + q * 32 + lane;
             __nv_bfloat16 *drow = p.d + (int64_t)b * p.d_bstride + row * p.ldd + n0;
             const __nv_bfloat16 *crow =
                 p.c != nullptr ? p.c + (int64_t)b * p.c_bstride + row * p.ldc + n0 : nullptr;
             const uint32_t acc = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(a * (int)kTmemCols);
 #pragma unroll 1
-            for (int ch = 0; ch < BN / 32; ++ch) {
+            for (int ch = 0; ch < TN / 32; ++ch) {
                 uint32_t r[32];
                 tmem_ld32(acc + (uint32_t)(ch * 32), r);
                 float v[32];
@@ -369,10 +453,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         dcol[(int64_t)j * p.ldt] = __float2bfloat16_rn(v[j]);
                 }
                 // Mirror of a symmetric product: (col, row) lies in the tile
-                // (col / BM, row / BN), skipped when row / BN * BN + BN <= col / BM * BM.
-                // Uniform over the warp (its rows share row / BN) and the
-                // 32-column chunk (its columns share col / BM).
-                if (p.sym && (int64_t)(row / BN) * BN + BN <= (int64_t)((n0 + ch * 32) / BM) * BM) {
+                // (col / TM, row / TN), skipped when row / TN < col / TM
+                // (TM == TN). Uniform over the warp (its rows share row / TN)
+                // and the 32-column chunk (its columns share col / TM).
+                if (p.sym && row / TN < (int64_t)((n0 + ch * 32) / TM)) {
                     __nv_bfloat16 *dcol = p.d + (int64_t)b * p.d_bstride +
                                           (int64_t)(n0 + ch * 32) * p.ldd + row;
 #pragma unroll
@@ -380,20 +464,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                         dcol[(int64_t)j * p.ldd] = __float2bfloat16_rn(v[j]);
                 }
             }
-            // this warp's rows of the accumulator are read: release it
+            // this warp's rows of the accumulator are read: release them to
+            // the leader's MMA lane
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             __syncwarp();
             if (lane == 0)
-                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(acc_empty(a))
-                             : "memory");
+                mbar_arrive_cluster(map_to_rank(acc_empty(a), 0));
             ++lt;
         }
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     }
     __syncthreads();
+    cluster_sync();   // no CTA leaves while its peer may still read its shared memory
     if (warp == 1) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                      "r"(2 * kTmemCols)
                      : "memory");
     }

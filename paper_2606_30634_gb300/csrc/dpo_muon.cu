@@ -9,13 +9,13 @@
 //                           sums of M^2 (fixed chunks: deterministic)
 //   muon_norm_kernel        ||M||_F per matrix from its partials, in order
 //   muon_normalize_kernel   X_0 = bf16(M / (||M||_F + eps)) into the padded
-//                           workspace, in the wide orientation, together with
-//                           X_0^T (64 x 64 tiles through shared memory)
+//                           workspace, in the wide orientation (64 x 64 tiles
+//                           through shared memory)
 //   ns_gemm_kernel x 3 per Newton-Schulz step and matrix shape, batched over
 //                           every matrix of that shape (dpo_gemm.cuh):
 //                             A = X X^T;  B = c A A + b A;  X <- B X + a X
-//                           (the last also writes X^T for the next step's
-//                           third product, whose second operand it is)
+//                           (the third reads X MN-major; at the last step it
+//                           also writes X^T, the output of tall matrices)
 //   muon_apply_kernel       U = lr (r O + wd X_t) and the delayed or EF
 //                           update, stash, history and bf16 weights
 #include "dpo_muon.h"
@@ -144,7 +144,7 @@ struct NormArgsM {
     const DevMat *mats;
     const int *group_mats;    // global matrix index of each batch entry
     const float *inv_norm;
-    __nv_bfloat16 *x, *xt;    // X (R x W) and X^T (W x R) of batch entry 0
+    __nv_bfloat16 *x, *xt;    // X (R x W) and X^T (W x R, or nullptr) of batch entry 0
     int64_t R, W;
     int64_t r, w;
 };
@@ -178,10 +178,12 @@ __global__ void __launch_bounds__(kThreads) muon_normalize_kernel(const NormArgs
     }
     __syncthreads();
     __nv_bfloat16 *x = a.x + (int64_t)bz * a.R * a.W;
-    __nv_bfloat16 *xt = a.xt + (int64_t)bz * a.W * a.R;
-    for (int rr = ty; rr < 64; rr += 4) {
+    for (int rr = ty; rr < 64; rr += 4)
         x[(i0 + rr) * a.W + j0 + tx] = __float2bfloat16_rn(tile[rr][tx]);
-        xt[(j0 + rr) * a.R + i0 + tx] = __float2bfloat16_rn(tile[tx][rr]);
+    if (a.xt != nullptr) {   // X_0^T: the output of tall matrices when there are no steps
+        __nv_bfloat16 *xt = a.xt + (int64_t)bz * a.W * a.R;
+        for (int rr = ty; rr < 64; rr += 4)
+            xt[(j0 + rr) * a.R + i0 + tx] = __float2bfloat16_rn(tile[tx][rr]);
     }
 }
 
@@ -324,8 +326,12 @@ struct Group {
     int64_t r, w, R, W;
     std::vector<int> mats;
     int *d_mats = nullptr;          // into the context's device block
-    __nv_bfloat16 *x = nullptr, *xt[2] = {nullptr, nullptr}, *a = nullptr, *b = nullptr;
-    CUtensorMap x128, x256, a128, a256, b128, xt256[2];
+    bool has_tall = false;
+    // X ping-pongs between x[0] and x[1]: every tile of X <- B X + a X reads
+    // all of the old X, so the new one goes to the other buffer.
+    __nv_bfloat16 *x[2] = {nullptr, nullptr}, *xt = nullptr, *a = nullptr, *b = nullptr;
+    CUtensorMap x128[2], a128, b128;   // 128-row K-major boxes: one CTA's half of a pair tile
+    CUtensorMap x_mn[2];               // 64 x 64 boxes of X read MN-major (B of B X)
 };
 
 }  // namespace
@@ -338,6 +344,7 @@ struct dpo_muon_ctx {
     bool ef = false;
     int64_t k = 0;
     int sms = 0;
+    int gemm_pairs = 0;   // clusters of 2 the GEMM kernel keeps resident at once
     std::vector<dpo_matrix> mats;
     std::vector<DevMat> host_mats;
     std::vector<Group> groups;
@@ -510,11 +517,13 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
     }
     c->chunks = (int)std::max<int64_t>(1, (max_n + kChunk - 1) / kChunk);
 
-    // Workspace: per group X, X^T twice, A, B (bf16).
+    // Workspace: per group X twice, X^T (the output of tall matrices), A, B (bf16).
     int64_t ws = 0;
     for (Group &g : c->groups) {
         const int64_t nb = (int64_t)g.mats.size();
         ws += nb * (g.R * g.W * 3 + g.R * g.R * 2) * 2;
+        for (int mi : g.mats)
+            g.has_tall = g.has_tall || mats[mi].rows > mats[mi].cols;
     }
     c->ws_bytes = ws;
     // Norm-pass table (the elementwise path's gradient-norm kernel).
@@ -607,38 +616,37 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
     for (size_t gi = 0; gi < c->groups.size(); ++gi) {
         Group &g = c->groups[gi];
         const int64_t nb = (int64_t)g.mats.size();
-        g.x = reinterpret_cast<__nv_bfloat16 *>(wp);
-        wp += nb * g.R * g.W * 2;
-        g.xt[0] = reinterpret_cast<__nv_bfloat16 *>(wp);
-        wp += nb * g.W * g.R * 2;
-        g.xt[1] = reinterpret_cast<__nv_bfloat16 *>(wp);
+        for (int q = 0; q < 2; ++q) {
+            g.x[q] = reinterpret_cast<__nv_bfloat16 *>(wp);
+            wp += nb * g.R * g.W * 2;
+        }
+        g.xt = reinterpret_cast<__nv_bfloat16 *>(wp);
         wp += nb * g.W * g.R * 2;
         g.a = reinterpret_cast<__nv_bfloat16 *>(wp);
         wp += nb * g.R * g.R * 2;
         g.b = reinterpret_cast<__nv_bfloat16 *>(wp);
         wp += nb * g.R * g.R * 2;
         g.d_mats = reinterpret_cast<int *>(blk + o_groups[gi]);
-        const bool ok = make_map(&g.x128, g.x, g.R, g.W, nb, dpo::gemm::BM) &&
-                        make_map(&g.x256, g.x, g.R, g.W, nb, dpo::gemm::BN) &&
+        const bool ok = make_map(&g.x128[0], g.x[0], g.R, g.W, nb, dpo::gemm::BM) &&
+                        make_map(&g.x128[1], g.x[1], g.R, g.W, nb, dpo::gemm::BM) &&
                         make_map(&g.a128, g.a, g.R, g.R, nb, dpo::gemm::BM) &&
-                        make_map(&g.a256, g.a, g.R, g.R, nb, dpo::gemm::BN) &&
                         make_map(&g.b128, g.b, g.R, g.R, nb, dpo::gemm::BM) &&
-                        make_map(&g.xt256[0], g.xt[0], g.W, g.R, nb, dpo::gemm::BN) &&
-                        make_map(&g.xt256[1], g.xt[1], g.W, g.R, nb, dpo::gemm::BN);
+                        make_map(&g.x_mn[0], g.x[0], g.R, g.W, nb, 64) &&
+                        make_map(&g.x_mn[1], g.x[1], g.R, g.W, nb, 64);
         if (!ok) {
             free_ctx(c);
             return mfail(nullptr, DPO_ECUDA, "tensor map encoding failed");
         }
-        // Newton-Schulz output: X (wide matrices) or the last X^T (tall
-        // ones), whose rows are the original matrix's rows.
-        const int last = hp->ns_steps % 2;
+        // Newton-Schulz output: X (wide matrices) or X^T (tall ones, whose
+        // rows are the original matrix's rows; written by the normalisation
+        // when there are no steps, else by the last step).
         for (size_t bi = 0; bi < g.mats.size(); ++bi) {
             DevMat &d = c->host_mats[g.mats[bi]];
             if (d.rows > d.cols) {
-                d.o = g.xt[last] + (int64_t)bi * g.W * g.R;
+                d.o = g.xt + (int64_t)bi * g.W * g.R;
                 d.o_ld = g.R;
-            } else {
-                d.o = g.x + (int64_t)bi * g.R * g.W;
+            } else {   // the buffer the last step wrote
+                d.o = g.x[hp->ns_steps % 2] + (int64_t)bi * g.R * g.W;
                 d.o_ld = g.W;
             }
         }
@@ -676,11 +684,27 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
         free_ctx(c);
         return mcuda(nullptr, e, "workspace clear");
     }
-    e = cudaFuncSetAttribute(dpo::gemm::ns_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             dpo::gemm::kSmemBytes);
-    if (e != cudaSuccess) {
+    c->gemm_pairs = 1 << 30;
+    for (const void *fn : {(const void *)dpo::gemm::ns_gemm_kernel<false>,
+                           (const void *)dpo::gemm::ns_gemm_kernel<true>}) {
+        e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 dpo::gemm::kSmemBytes);
+        int pairs = 0;
+        if (e == cudaSuccess) {
+            cudaLaunchConfig_t cfg = {};
+            cfg.gridDim = dim3(2 * std::max(1, c->sms / 2));
+            cfg.blockDim = dim3(dpo::gemm::kThreads);
+            cfg.dynamicSmemBytes = dpo::gemm::kSmemBytes;
+            e = cudaOccupancyMaxActiveClusters(&pairs, fn, &cfg);
+        }
+        if (e != cudaSuccess)
+            break;
+        c->gemm_pairs = std::min(c->gemm_pairs, pairs);
+    }
+    if (e != cudaSuccess || c->gemm_pairs < 1) {
         free_ctx(c);
-        return mcuda(nullptr, e, "GEMM shared-memory attribute");
+        return e != cudaSuccess ? mcuda(nullptr, e, "GEMM launch configuration")
+                                : mfail(nullptr, DPO_ECUDA, "GEMM kernel cannot be resident");
     }
     if (init_mode == DPO_INIT_FRESH) {
         const int rc = launch_init(c, s, 1);
@@ -697,13 +721,20 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
 namespace {
 
 int launch_gemm(dpo_muon_ctx *c, const CUtensorMap &ta, const CUtensorMap &tb,
-                const dpo::gemm::Params &p, int64_t M, int64_t N, int64_t nb, cudaStream_t s)
+                const dpo::gemm::Params &p, int64_t M, int64_t N, int64_t nb, bool b_mn,
+                cudaStream_t s)
 {
-    dpo::gemm::TileGrid tg{(int)(M / dpo::gemm::BM), (int)(N / dpo::gemm::BN), (int)nb};
+    dpo::gemm::TileGrid tg{(int)(M / dpo::gemm::TM), (int)(N / dpo::gemm::TN), (int)nb};
     const int64_t tiles = (int64_t)tg.m_tiles * tg.n_tiles * tg.nb;
-    const int grid = (int)std::min<int64_t>(tiles, std::max(1, c->sms));   // one CTA per SM
-    dpo::gemm::ns_gemm_kernel<<<grid, dpo::gemm::kThreads, dpo::gemm::kSmemBytes, s>>>(ta, tb, p,
-                                                                                       tg);
+    // one CTA pair per co-resident cluster slot (the tile walk assumes every
+    // pair runs at once)
+    const int grid = 2 * (int)std::min<int64_t>(tiles, std::max(1, c->gemm_pairs));
+    if (b_mn)
+        dpo::gemm::ns_gemm_kernel<true><<<grid, dpo::gemm::kThreads, dpo::gemm::kSmemBytes, s>>>(
+            ta, tb, p, tg);
+    else
+        dpo::gemm::ns_gemm_kernel<false><<<grid, dpo::gemm::kThreads, dpo::gemm::kSmemBytes, s>>>(
+            ta, tb, p, tg);
     const cudaError_t e = cudaGetLastError();
     return e == cudaSuccess ? DPO_OK : mcuda(c, e, "Newton-Schulz GEMM launch");
 }
@@ -759,7 +790,8 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
 
     for (Group &g : c->groups) {
         const int64_t nb = (int64_t)g.mats.size();
-        dpo::muon::NormArgsM na{c->d_mats, g.d_mats, c->d_inv_norm, g.x, g.xt[0], g.R, g.W, g.r, g.w};
+        dpo::muon::NormArgsM na{c->d_mats, g.d_mats, c->d_inv_norm, g.x[0],
+                                c->hp.ns_steps == 0 ? g.xt : nullptr, g.R, g.W, g.r, g.w};
         const dim3 ngrid((unsigned)(g.W / 64), (unsigned)(g.R / 64), (unsigned)nb);
         dpo::muon::muon_normalize_kernel<<<ngrid, kThreads, 0, s>>>(na);
         if ((e = cudaGetLastError()) != cudaSuccess)
@@ -781,6 +813,7 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
             c->gemm_launches += 3 * (int64_t)c->hp.ns_steps;
         }
         for (int it = 0; it < c->hp.ns_steps; ++it) {
+            const bool last = it + 1 == c->hp.ns_steps;
             const int cur = it % 2, nxt = cur ^ 1;
             dpo::gemm::Params p{};
             p.err = c->d_err;
@@ -791,7 +824,7 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
             p.alpha = 1.0f;
             p.k_blocks = (int)(g.W / dpo::gemm::BK);
             p.sym = 1;
-            int rc = launch_gemm(c, g.x128, g.x256, p, g.R, g.R, nb, s);
+            int rc = launch_gemm(c, g.x128[cur], g.x128[cur], p, g.R, g.R, nb, false, s);
             if (rc != DPO_OK)
                 return rc;
             // B = c A A + b A
@@ -802,23 +835,24 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
             p.alpha = c->hp.ns_c;
             p.beta = c->hp.ns_b;
             p.k_blocks = (int)(g.R / dpo::gemm::BK);
-            if ((rc = launch_gemm(c, g.a128, g.a256, p, g.R, g.R, nb, s)) != DPO_OK)
+            if ((rc = launch_gemm(c, g.a128, g.a128, p, g.R, g.R, nb, false, s)) != DPO_OK)
                 return rc;
-            // X <- B X + a X, and X^T
+            // X <- B X + a X (X read MN-major in place of X^T), and at the
+            // last step X^T for the tall matrices' output
             p.sym = 0;
-            p.d = g.x;
+            p.d = g.x[nxt];
             p.ldd = g.W;
             p.d_bstride = g.R * g.W;
-            p.dt = g.xt[nxt];
+            p.dt = last && g.has_tall ? g.xt : nullptr;
             p.ldt = g.R;
             p.dt_bstride = g.W * g.R;
-            p.c = g.x;
+            p.c = g.x[cur];
             p.ldc = g.W;
             p.c_bstride = g.R * g.W;
             p.alpha = 1.0f;
             p.beta = c->hp.ns_a;
             p.k_blocks = (int)(g.R / dpo::gemm::BK);
-            if ((rc = launch_gemm(c, g.b128, g.xt256[cur], p, g.R, g.W, nb, s)) != DPO_OK)
+            if ((rc = launch_gemm(c, g.b128, g.x_mn[cur], p, g.R, g.W, nb, true, s)) != DPO_OK)
                 return rc;
         }
         if (ev_end != nullptr && (e = cudaEventRecord(ev_end, s)) != cudaSuccess)

@@ -30,8 +30,11 @@ from parity_util import TOL_ONE_STEP, TOL_RUN, bf16_ulps, rel_err
 pytestmark = pytest.mark.gpu
 
 F, B = dpo.DPO_F32, dpo.DPO_BF16
-# wide, tall, ragged (padded to 256 inside), several tiles, tiny, empty
-SHAPES = [(256, 512), (512, 256), (300, 700), (64, 96), (1, 7), (0, 5), (768, 2304)]
+# wide, tall, ragged (padded to 256 inside), several tiles, tiny, empty, and
+# a shape whose 96 output tiles outnumber the CTA pairs (each pair then walks
+# several tiles, reading operands other pairs' tiles are being written next to)
+SHAPES = [(256, 512), (512, 256), (300, 700), (64, 96), (1, 7), (0, 5), (768, 2304),
+          (1024, 3072), (3072, 1024)]
 NS_BARS = {1: (2e-4, 2e-3), 2: (5e-4, 1e-2)}
 
 
@@ -198,7 +201,8 @@ def test_muon_flops_and_workspace(cuda_device):
         want = sum(5 * (a * (a + 1) * b + a * (a + 1) * a + 2 * a * a * b)
                    for a, b in ((min(r, c), max(r, c)) for r, c in shapes))
         assert m.flops() == pytest.approx(want, rel=1e-12)
-        # (256, 512) and (512, 256) share the 256 x 512 group; (300, 700) pads to 512 x 768
+        # (256, 512) and (512, 256) share the 256 x 512 group; (300, 700) pads to 512 x 768;
+        # per matrix X twice, X^T, A and B
         ws = 2 * ((2 * (256 * 512 * 3 + 256 * 256 * 2)) + (512 * 768 * 3 + 512 * 512 * 2))
         assert m.workspace_bytes() == ws
     finally:
