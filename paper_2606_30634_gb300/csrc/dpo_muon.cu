@@ -150,7 +150,10 @@ struct NormArgsM {
 };
 
 // One 64 x 64 tile of X (rows i over r, columns j over w) per CTA; padding
-// outside r x w is written as zero.
+// outside r x w is written as zero. M is read along its own rows (32-byte
+// fp32 vectors where the row pitch allows) and X written along its rows
+// (16-byte bf16 vectors), through a shared-memory tile that transposes the
+// tall matrices.
 __global__ void __launch_bounds__(kThreads) muon_normalize_kernel(const NormArgsM a)
 {
     __shared__ float tile[64][65];
@@ -160,30 +163,49 @@ __global__ void __launch_bounds__(kThreads) muon_normalize_kernel(const NormArgs
     const bool tall = d.rows > d.cols;
     const float s = a.inv_norm[gm];
     const int64_t i0 = (int64_t)blockIdx.y * 64, j0 = (int64_t)blockIdx.x * 64;
-    const int tx = threadIdx.x & 63, ty = threadIdx.x >> 6;   // 64 x 4
-    // load: X[i][j] = tall ? M[j][i] : M[i][j], read along M's rows
-    for (int rr = ty; rr < 64; rr += 4) {
-        float v = 0.0f;
-        if (!tall) {
-            const int64_t i = i0 + rr, j = j0 + tx;
-            if (i < a.r && j < a.w)
-                v = d.mom[i * d.cols + j] * s;
-            tile[rr][tx] = v;
+    // tile origin in M: (mr0, mc0), 64 x 64, clipped to rows x cols
+    const int64_t mr0 = tall ? j0 : i0, mc0 = tall ? i0 : j0;
+    const bool vec = (d.cols % kPacket) == 0 && mr0 + 64 <= d.rows && mc0 + 64 <= d.cols;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int v = (int)threadIdx.x + h * kThreads;   // 512 vectors of 8
+        const int row = v >> 3, c8 = (v & 7) * 8;         // within the tile, in M's layout
+        float x[8];
+        if (vec) {
+            ld8(d.mom + (mr0 + row) * d.cols + mc0 + c8, x);
         } else {
-            const int64_t j = j0 + rr, i = i0 + tx;   // M row j, column i
-            if (i < a.r && j < a.w)
-                v = d.mom[j * d.cols + i] * s;
-            tile[tx][rr] = v;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const int64_t mr = mr0 + row, mc = mc0 + c8 + e;
+                x[e] = (mr < d.rows && mc < d.cols) ? d.mom[mr * d.cols + mc] : 0.0f;
+            }
+        }
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            if (tall)
+                tile[c8 + e][row] = x[e] * s;   // X row = M column
+            else
+                tile[row][c8 + e] = x[e] * s;
         }
     }
     __syncthreads();
-    __nv_bfloat16 *x = a.x + (int64_t)bz * a.R * a.W;
-    for (int rr = ty; rr < 64; rr += 4)
-        x[(i0 + rr) * a.W + j0 + tx] = __float2bfloat16_rn(tile[rr][tx]);
-    if (a.xt != nullptr) {   // X_0^T: the output of tall matrices when there are no steps
-        __nv_bfloat16 *xt = a.xt + (int64_t)bz * a.W * a.R;
-        for (int rr = ty; rr < 64; rr += 4)
-            xt[(j0 + rr) * a.R + i0 + tx] = __float2bfloat16_rn(tile[tx][rr]);
+    __nv_bfloat16 *xb = a.x + (int64_t)bz * a.R * a.W;
+    __nv_bfloat16 *xt = a.xt != nullptr ? a.xt + (int64_t)bz * a.W * a.R : nullptr;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int v = (int)threadIdx.x + h * kThreads;
+        const int row = v >> 3, c8 = (v & 7) * 8;   // within the tile, in X's layout
+        float o[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e)
+            o[e] = tile[row][c8 + e];
+        st8(xb + (i0 + row) * a.W + j0 + c8, o);
+        if (xt != nullptr) {   // X_0^T: the output of tall matrices when there are no steps
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                o[e] = tile[c8 + e][row];
+            st8(xt + (j0 + row) * a.R + i0 + c8, o);
+        }
     }
 }
 
