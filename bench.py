@@ -113,23 +113,29 @@ def measured_hbm_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def kernel_source_sha() -> str:
-    """First 16 hex digits of the sha256 over the device sources (every .cu
-    and .cuh under csrc/, in name order): a summary taken on other sources
-    describes another kernel."""
+# The device sources each profiled kernel is compiled from.
+KERNEL_SOURCES = {
+    "fused_step": ("dpo_internal.h", "dpo_device.cuh", "dpo_step.cuh", "dpo_step_adamw.cu",
+                   "dpo_step_nadam.cu", "dpo_step_lion.cu", "dpo_step_adan.cu", "dpo_kernels.cu"),
+    "ns_gemm": ("dpo_internal.h", "dpo_device.cuh", "dpo_gemm.cuh", "dpo_muon.cu"),
+}
+
+
+def kernel_source_sha(kernel: str = "fused_step") -> str:
+    """First 16 hex digits of the sha256 over the kernel's device sources (in
+    name order): a summary taken on other sources describes another kernel."""
     csrc = os.path.join(ROOT, "paper_2606_30634_gb300", "csrc")
     h = hashlib.sha256()
-    for name in sorted(os.listdir(csrc)):
-        if name.endswith((".cu", ".cuh")):
-            h.update(name.encode() + b"\0")
-            h.update(open(os.path.join(csrc, name), "rb").read())
+    for name in sorted(KERNEL_SOURCES[kernel]):
+        h.update(name.encode() + b"\0")
+        h.update(open(os.path.join(csrc, name), "rb").read())
     return h.hexdigest()[:16]
 
 
 def committed_traffic(kernel_tag: str):
     """dram bytes per parameter from the committed ncu summary of the fused
     kernel, if that summary was taken on the kernel source as it is now."""
-    sha = kernel_source_sha()
+    sha = kernel_source_sha(kernel_tag.split(":")[0])
     for name in sorted(os.listdir(os.path.join(ROOT, "profiles"))) if os.path.isdir(
             os.path.join(ROOT, "profiles")) else []:
         if not name.endswith(".md"):
