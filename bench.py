@@ -135,7 +135,10 @@ def kernel_source_sha(kernel: str = "fused_step") -> str:
 def committed_traffic(kernel_tag: str):
     """dram bytes per parameter from the committed ncu summary of the fused
     kernel, if that summary was taken on the kernel source as it is now."""
-    sha = kernel_source_sha(kernel_tag.split(":")[0])
+    kernel = kernel_tag.split(":")[0]
+    if kernel not in KERNEL_SOURCES:
+        return None
+    sha = kernel_source_sha(kernel)
     for name in sorted(os.listdir(os.path.join(ROOT, "profiles"))) if os.path.isdir(
             os.path.join(ROOT, "profiles")) else []:
         if not name.endswith(".md"):
