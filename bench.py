@@ -5,8 +5,11 @@ Error Feedback) on a 6.74e9-parameter Llama-7B-shaped tensor set.
                     [--workload llama-7B] [--mode ef|std]
 
 A step is one dpo_step over the whole set: every parameter's stale gradient
-is consumed and master, m, v, the EF buffer, the bf16 stash and the bf16
-latest copy are rewritten (inputs already resident in HBM when timing
+is consumed and master, m, v, the EF buffer and the bf16 weights are
+rewritten; the stale version is the bf16 weights of the previous step, kept
+in the second of two weight buffers that swap roles (PipeDream-2BW's double
+buffering, --stash pingpong, the default where the layout allows it; --stash
+copy writes a separate stash instead) (inputs already resident in HBM when timing
 starts; the 148 GB working set is far larger than L2, so no flush is
 needed). Prints one JSON line: throughput in parameters updated per second,
 the fused kernel's achieved HBM bandwidth against the measured copy peak,
@@ -54,6 +57,10 @@ def parse_args(argv=None):
                    help="muon: delayed Muon (Alg. 2) on the attention and MLP matrices, "
                         "AdamW on the rest")
     p.add_argument("--ns-steps", type=int, default=5, help="Newton-Schulz steps (muon)")
+    p.add_argument("--stash", choices=["auto", "copy", "pingpong"], default="auto",
+                   help="pingpong: bf16 param and stash buffers swap roles (no stash store); "
+                        "auto: pingpong where the layout allows it (bf16 param and stash, "
+                        "standard rule or EF), else copy")
     p.add_argument("--dc-lambda", type=float, default=0.0,
                    help="DC-ASGD compensation strength (Sec. 3.1); 0: off")
     p.add_argument("--wpipe", action="store_true",
@@ -290,7 +297,9 @@ def run_gpu(args, w, world, rank, local):
         for i, (o, n) in enumerate(zip(lay.offsets, lay.numels)):
             synth.dev_normal(w.seed, synth.STREAM_INIT, 0, int(offs[i]), x0[o:o + n], W.INIT_SIGMA)
         kw = dict(lr=w.lr, beta1=w.beta1, beta2=w.beta2, eps=w.eps,
-                  weight_decay=w.weight_decay)
+                  weight_decay=w.weight_decay,
+                  stash_mode=(dpo.DPO_STASH_PINGPONG if args.stash == "pingpong"
+                              else dpo.DPO_STASH_COPY))
         kw.update(rule_settings(args))
         opt = dpo.DelayedAdamW(w.numels, param_dtype=w.param_dtype, stash_dtype=w.stash_dtype,
                                grad_dtype=w.grad_dtype, ef=ef, ef_lambda=1.0,
@@ -613,6 +622,10 @@ def main(argv=None):
     args = parse_args(argv)
     from paper_2606_30634_gb300.synth import workloads as W
     w = W.ALL[args.workload]
+    if args.stash == "auto":
+        ok = (w.param_dtype == W.BF16 and w.stash_dtype == W.BF16
+              and args.mode in ("ef", "std") and args.optimizer != "muon")
+        args.stash = "pingpong" if ok else "copy"
     world, rank, local = dist_env()
     if args.optimizer == "muon":
         return main_muon(args, w, world, rank, local)
@@ -625,7 +638,7 @@ def main(argv=None):
            "state": "fp32 master/m/v" + (" + fp32 update-history buffer" if ef else ""),
            "clip": w.max_grad_norm, "l2": "inputs larger than L2 (no flush needed)",
            "wpipe": bool(args.wpipe), "optimizer": args.optimizer,
-           "dc_lambda": args.dc_lambda}
+           "dc_lambda": args.dc_lambda, "stash": args.stash}
 
     if args.impl == "reference":
         if rank != 0:
@@ -653,7 +666,7 @@ def main(argv=None):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     r = run_gpu(args, w, world, rank, local)
     peak, peak_kind = measured_hbm_peak()
-    kernel_tag = f"fused_step:{w.name}:{args.mode}"
+    kernel_tag = f"fused_step:{w.name}:{args.mode}" + (":pingpong" if args.stash == "pingpong" else "")
     traffic = committed_traffic(kernel_tag)
     kernels = "fused_step_kernel" if w.max_grad_norm <= 0 else "grad_sqnorm_kernel+fused_step_kernel"
     roof = {"bound": "hbm", "achieved": r["achieved"], "peak": peak, "unit": "GB/s",

@@ -124,6 +124,25 @@ typedef enum { DPO_F32 = 0, DPO_BF16 = 1 } dpo_dtype;
  *                  u = lr ((m/(1-beta1^k) + beta2 v/(1-beta2^k)) / (sqrt(n/(1-beta3^k)) + eps)
  *                      + wd x_t); needs the n and grad_prev buffers.
  * DPO_CORR_SAPIPE_UPDATED is defined for AdamW only. */
+/* dpo_hparams.stash_mode. PipeDream-2BW keeps two weight versions (Sec. 2):
+ *   DPO_STASH_COPY      the step writes x_t into the stash buffer and
+ *                       x_{t+1} into the param buffer (every layout).
+ *   DPO_STASH_PINGPONG  with bf16 param and stash buffers, the stale version
+ *                       x_t is bitwise the bf16 weights the previous call
+ *                       wrote, so the two buffers of a delayed tensor swap
+ *                       roles instead: call k writes x_{k+1} into the buffer
+ *                       that held x_{k-1}, and no stash is written (2 bytes per
+ *                       parameter less). After call k the param buffer holds
+ *                       the latest weights when k is even and the stash buffer
+ *                       when k is odd; dpo_read_weights resolves the roles.
+ *                       Needs param_dtype = stash_dtype = DPO_BF16, device
+ *                       param buffers, and the standard rule or EF (the SAPipe
+ *                       corrections stash a prediction, not a previous version).
+ *                       Synchronously trained tensors (DPO_SYNC) keep their
+ *                       weights in the param buffer. */
+#define DPO_STASH_COPY 0
+#define DPO_STASH_PINGPONG 1
+
 #define DPO_OPT_ADAMW 0
 #define DPO_OPT_NADAM 1
 #define DPO_OPT_LION 2
@@ -145,6 +164,7 @@ typedef struct {
      * compensated, g~ = g + dc_lambda g^2 (x_t - stash), the stash holding the
      * weights the gradient was evaluated at (after clipping). */
     float dc_lambda;
+    int stash_mode;       /* DPO_STASH_* */
 } dpo_hparams;
 
 typedef struct {

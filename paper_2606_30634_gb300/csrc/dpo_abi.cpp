@@ -11,6 +11,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cstring>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -102,6 +103,19 @@ StashKind stash_kind(const dpo_ctx *c)
     return c->stash_dt == DPO_BF16 ? dpo::kStashBF16 : dpo::kStashF32;
 }
 
+// Ping-pong stash in use (delayed training).
+bool pingpong_on(const dpo_ctx *c)
+{
+    return c->hp.stash_mode == DPO_STASH_PINGPONG && c->hp.delay == 1;
+}
+
+// Ping-pong stash: the latest weights of delayed tensors sit in the stash
+// buffer after an odd number of calls of the current delayed phase.
+bool latest_in_stash(const dpo_ctx *c)
+{
+    return pingpong_on(c) && ((c->k - c->phase_k0) & 1) != 0;
+}
+
 // Stash kind of the stash kernel: the buffers' dtype whenever they exist.
 StashKind stash_buffer_kind(const dpo_ctx *c)
 {
@@ -167,7 +181,7 @@ int set_step_grid(dpo_ctx *c)
     int per_sm = 0;
     const cudaError_t e = dpo::step_ctas_per_sm(
         static_cast<dpo::Optimizer>(c->hp.optimizer), c->param_dt == DPO_BF16, stash_kind(c),
-        c->grad_dt == DPO_BF16, corr, dc_on(c), &per_sm);
+        c->grad_dt == DPO_BF16, corr, dc_on(c), pingpong_on(c), &per_sm);
     if (e != cudaSuccess)
         return cuda_fail(c, e, "occupancy query");
     int64_t hist_elems = 0;
@@ -236,6 +250,16 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
         return fail(nullptr, DPO_EINVAL, "momentum_decay must be >= 0");
     if (hp->correction == DPO_CORR_SAPIPE_UPDATED && hp->optimizer != DPO_OPT_ADAMW)
         return fail(nullptr, DPO_EINVAL, "the SAPipe updated-state prediction is defined for AdamW");
+    if (hp->stash_mode != DPO_STASH_COPY && hp->stash_mode != DPO_STASH_PINGPONG)
+        return fail(nullptr, DPO_EINVAL, "stash_mode must be one of DPO_STASH_*");
+    if (hp->stash_mode == DPO_STASH_PINGPONG) {
+        if (param_dtype != DPO_BF16 || stash_dtype != DPO_BF16)
+            return fail(nullptr, DPO_EDTYPE, "the ping-pong stash needs bf16 param and stash buffers");
+        if (hp->correction != DPO_CORR_EF)
+            return fail(nullptr, DPO_EINVAL,
+                        "the ping-pong stash needs the standard rule or EF (the SAPipe "
+                        "corrections stash a prediction)");
+    }
 
     // Table: NULL pointers, EF consistency, alignment, overlaps.
     const bool ef = table[0].ef != nullptr;
@@ -320,7 +344,7 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
         return cuda_fail(nullptr, e, "cudaGetDevice");
     int pageable_ok = 0;
     cudaDeviceGetAttribute(&pageable_ok, cudaDevAttrPageableMemoryAccess, device);
-    bool host_io = false;
+    bool host_io = false, host_param = false;
     for (const Span &s : spans) {
         cudaPointerAttributes attr{};
         const void *ptr = reinterpret_cast<const void *>(s.lo);
@@ -335,6 +359,7 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
             continue;
         if (s.host_ok && (host_mapped || host_pageable)) {
             host_io = true;
+            host_param = host_param || std::strcmp(s.name, "param") == 0;
             continue;
         }
         return fail(nullptr, DPO_EINVAL,
@@ -343,6 +368,9 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
                               : "tensor %d: %s is not device memory of the current device",
                     s.tensor, s.name);
     }
+
+    if (hp->stash_mode == DPO_STASH_PINGPONG && host_param)
+        return fail(nullptr, DPO_EINVAL, "the ping-pong stash needs device param buffers");
 
     dpo_ctx *c = new (std::nothrow) dpo_ctx;
     if (c == nullptr)
@@ -486,6 +514,14 @@ extern "C" int dpo_set_delay(dpo_ctx *c, int delay, void *cuda_stream)
                 return cuda_fail(c, e, "stash launch");
         }
         c->phase_k0 = c->k;
+    } else if (latest_in_stash(c) && c->total_pkts > 0) {
+        // Ping-pong: the latest weights sit in the stash buffer; synchronous
+        // training keeps them in the param buffer (param := bf16(master)).
+        dpo::StashArgs a{c->d_table, c->d_pkt_begin, c->n, c->total_pkts, 0, 0};
+        const cudaError_t e = dpo::launch_stash(true, stash_buffer_kind(c), c->stash_grid, a,
+                                                static_cast<cudaStream_t>(cuda_stream));
+        if (e != cudaSuccess)
+            return cuda_fail(c, e, "stash launch");
     }
     c->hp.delay = delay;
     const int rc = set_step_grid(c);
@@ -541,11 +577,15 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
         a.adan_c2 = (float)(lrd * b2 / bc2);
         a.first = k == 1;
         a.dc_lambda = c->hp.delay == 1 ? c->hp.dc_lambda : 0.0f;
+        // Ping-pong: call t of the delayed phase writes the new weights of
+        // delayed tensors into the buffer holding x_{t-1}: the stash buffer
+        // when t is odd, the param buffer when t is even.
+        a.swap = pingpong_on(c) && (t & 1) != 0;
         a.clip = c->clip ? &c->d_scalars->clip : nullptr;
         const cudaError_t e = dpo::launch_step(static_cast<dpo::Optimizer>(c->hp.optimizer),
                                                c->param_dt == DPO_BF16, stash_kind(c),
                                                c->grad_dt == DPO_BF16, corr, dc_on(c),
-                                               c->step_grid, a, s);
+                                               pingpong_on(c), c->step_grid, a, s);
         if (e != cudaSuccess)
             return cuda_fail(c, e, "fused step launch");
     }
@@ -562,12 +602,15 @@ extern "C" int dpo_read_weights(const dpo_ctx *c, int which, int tensor, const v
     if (tensor < 0 || tensor >= c->n || (which != DPO_STALE && which != DPO_LATEST))
         return DPO_EINVAL;
     const dpo_tensor &d = c->table[tensor];
+    // Ping-pong: after an odd number of delayed calls the two buffers of a
+    // delayed tensor hold each other's role.
+    const bool swapped = latest_in_stash(c) && !(d.flags & DPO_SYNC);
     if (which == DPO_STALE && c->hp.delay == 1 && !(d.flags & DPO_SYNC)) {
-        *ptr = d.stash;
+        *ptr = swapped ? d.param : d.stash;
         if (dtype)
             *dtype = c->stash_dt;
     } else if (c->param_dt == DPO_BF16) {
-        *ptr = d.param;
+        *ptr = swapped ? d.stash : d.param;
         if (dtype)
             *dtype = DPO_BF16;
     } else {
@@ -631,10 +674,13 @@ extern "C" int dpo_algorithmic_bytes(const dpo_ctx *c, int64_t *step_bytes, int6
     // correction reads and writes its update-history buffer.
     const int64_t base = 8 * (1 + rule_state_streams(c->hp.optimizer)) + dt_size(c->grad_dt) +
                          (c->param_dt == DPO_BF16 ? 2 : 0);
+    // (the ping-pong stash writes no stash; DC-ASGD reads it)
+    const int stash_writes = c->hp.stash_mode == DPO_STASH_PINGPONG ? 0 : 1;
     const int64_t delayed_extra =
-        c->hp.delay == 1 ? dt_size(c->stash_dt) * (c->hp.dc_lambda != 0.0f ? 2 : 1) +
-                               (c->ef ? 8 : 0)
-                         : 0;
+        c->hp.delay == 1
+            ? dt_size(c->stash_dt) * (stash_writes + (c->hp.dc_lambda != 0.0f ? 1 : 0)) +
+                  (c->ef ? 8 : 0)
+            : 0;
     int64_t total = 0;
     for (const dpo_tensor &d : c->table)
         total += d.numel * (base + ((d.flags & DPO_SYNC) ? 0 : delayed_extra));

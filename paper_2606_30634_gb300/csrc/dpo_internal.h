@@ -76,6 +76,8 @@ struct StepArgs {
     float adan_c2;              // Adan: lr beta2 / (1 - beta2^k)
     int first;                  // Adan: k == 1 (the gradient difference is 0)
     float dc_lambda;            // DC-ASGD strength (0: off)
+    int swap;                   // ping-pong stash: write delayed tensors' weights into
+                                // their stash buffer (else their param buffer)
     const float *clip;          // device clip coefficient, or nullptr
 };
 
@@ -112,24 +114,25 @@ struct StashArgs {
 // that combination is not provided.
 using StepFn = void (*)(StepArgs);
 StepFn pick_step_adamw(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr,
-                       bool dc);
+                       bool dc, bool pp);
 StepFn pick_step_nadam(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr,
-                       bool dc);
+                       bool dc, bool pp);
 StepFn pick_step_lion(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr,
-                      bool dc);
+                      bool dc, bool pp);
 StepFn pick_step_adan(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr,
-                      bool dc);
+                      bool dc, bool pp);
 
 // Launchers (dpo_kernels.cu). Each returns the launch's cudaError_t.
 cudaError_t launch_step(Optimizer opt, bool param_bf16, StashKind stash, bool grad_bf16,
-                        Correction corr, bool dc, int grid, const StepArgs &a, cudaStream_t s);
+                        Correction corr, bool dc, bool pp, int grid, const StepArgs &a,
+                        cudaStream_t s);
 cudaError_t launch_norm(bool grad_bf16, int grid, const NormArgs &a, cudaStream_t s);
 cudaError_t launch_stash(bool param_bf16, StashKind stash, int grid, const StashArgs &a,
                          cudaStream_t s);
 
 // Resident CTAs per SM of each kernel at its block size (occupancy query).
 cudaError_t step_ctas_per_sm(Optimizer opt, bool param_bf16, StashKind stash, bool grad_bf16,
-                             Correction corr, bool dc, int *n);
+                             Correction corr, bool dc, bool pp, int *n);
 cudaError_t norm_ctas_per_sm(bool grad_bf16, int *n);
 
 }  // namespace dpo

@@ -226,25 +226,25 @@ StashFn pick_stash_sk(StashKind sk)
 }  // namespace
 
 static StepFn pick_step_for(Optimizer opt, bool pb, StashKind sk, bool gb, Correction corr,
-                            bool dc)
+                            bool dc, bool pp)
 {
     switch (opt) {
     case kOptAdamW:
-        return pick_step_adamw(pb, sk, gb, corr, dc);
+        return pick_step_adamw(pb, sk, gb, corr, dc, pp);
     case kOptNAdam:
-        return pick_step_nadam(pb, sk, gb, corr, dc);
+        return pick_step_nadam(pb, sk, gb, corr, dc, pp);
     case kOptLion:
-        return pick_step_lion(pb, sk, gb, corr, dc);
+        return pick_step_lion(pb, sk, gb, corr, dc, pp);
     case kOptAdan:
-        return pick_step_adan(pb, sk, gb, corr, dc);
+        return pick_step_adan(pb, sk, gb, corr, dc, pp);
     }
     return nullptr;
 }
 
 cudaError_t launch_step(Optimizer opt, bool pb, StashKind sk, bool gb, Correction corr, bool dc,
-                        int grid, const StepArgs &a, cudaStream_t s)
+                        bool pp, int grid, const StepArgs &a, cudaStream_t s)
 {
-    StepFn f = pick_step_for(opt, pb, sk, gb, corr, dc);
+    StepFn f = pick_step_for(opt, pb, sk, gb, corr, dc, pp);
     if (f == nullptr)
         return cudaErrorInvalidValue;
     f<<<grid, kStepThreads, 0, s>>>(a);
@@ -268,9 +268,9 @@ cudaError_t launch_stash(bool pb, StashKind sk, int grid, const StashArgs &a, cu
 }
 
 cudaError_t step_ctas_per_sm(Optimizer opt, bool pb, StashKind sk, bool gb, Correction corr,
-                             bool dc, int *n)
+                             bool dc, bool pp, int *n)
 {
-    StepFn f = pick_step_for(opt, pb, sk, gb, corr, dc);
+    StepFn f = pick_step_for(opt, pb, sk, gb, corr, dc, pp);
     if (f == nullptr)
         return cudaErrorInvalidValue;
     return cudaOccupancyMaxActiveBlocksPerMultiprocessor(n, f, kStepThreads, 0);

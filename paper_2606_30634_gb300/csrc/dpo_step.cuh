@@ -107,7 +107,9 @@ __device__ __forceinline__ float dc_compensate(float lambda, float g, float x, f
 // point x_t - u_prev; the weights take the standard rule). OPT is the rule.
 // DC selects the DC-ASGD compensation of delayed tensors (instances with a
 // stash only); without it the kernel holds no registers for the stash read.
-template <int PB, int SK, int GB, int CORR, int OPT, int DC>
+// PP selects the ping-pong stash (bf16 param and stash, standard rule or EF):
+// the buffers of delayed tensors swap roles instead of the stash being stored.
+template <int PB, int SK, int GB, int CORR, int OPT, int DC, int PP>
 __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs a)
 {
     using GT = typename Elem<GB != 0>::T;
@@ -143,12 +145,16 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
         float *__restrict__ gpv = d.grad_prev;
         float *__restrict__ ef = d.ef;
         const GT *__restrict__ grad = static_cast<const GT *>(d.grad);
-        ST *__restrict__ stash = static_cast<ST *>(d.stash);
-        __nv_bfloat16 *__restrict__ param = static_cast<__nv_bfloat16 *>(d.param);
         const float wd_lr = (d.flags & kFlagWd) ? a.lr_wd : 0.0f;
         // A DPO_SYNC tensor takes the standard update with no stash and no
         // correction even while the run is delayed.
         const bool dly = SK != kStashNone && !(d.flags & kFlagSync);
+        // Ping-pong stash (bf16 param and stash): the new weights go into the
+        // buffer holding the stale version, which is then the one DC-ASGD
+        // reads, and no stash is stored.
+        const bool pp = PP && dly;
+        __nv_bfloat16 *param = static_cast<__nv_bfloat16 *>(pp && a.swap ? d.stash : d.param);
+        ST *stash = pp ? reinterpret_cast<ST *>(param) : static_cast<ST *>(d.stash);   // may alias param
         const bool prev_t = dly && use_prev;
         const bool efn_t = dly && ef_now;
         const bool dc_t = DC && dly;
@@ -169,7 +175,7 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
                 ld8(ef + e, up);
             if (dc_t)
                 ld8(stash + e, sw);   // the weights the gradient was evaluated at
-            if (dly) {
+            if (dly && !pp) {
                 if (kSapipe) {   // stash := the prediction point x_t - u_prev
                     float xp[8];
 #pragma unroll
@@ -213,7 +219,7 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
                 const float up = prev_t ? ef[i] : 0.0f;
                 if (dc_t)
                     g = dc_compensate(dc, g, x, ld1(stash + i));
-                if (dly)
+                if (dly && !pp)
                     st1(stash + i, kSapipe ? x - up : x);
                 float u = rule_update<OPT>(s, g, x, wd_lr, m, v, n, gp);
                 x -= efn_t ? ef_displacement(s.lam, u, up) : u;
@@ -239,44 +245,53 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
 // ------------------------------------------------------------ dispatch ----
 
 template <int PB, int SK, int GB, int OPT, int DC>
-StepFn pick_step_corr(Correction corr)
+StepFn pick_step_corr(Correction corr, bool pp)
 {
+    // the ping-pong stash: bf16 param and stash, standard rule or EF
+    constexpr bool kPP = PB == 1 && SK == kStashBF16;
     switch (corr) {
     case kCorrNone:
-        return fused_step_kernel<PB, SK, GB, kCorrNone, OPT, DC>;
+        if (pp)
+            return kPP ? fused_step_kernel<PB, SK, GB, kCorrNone, OPT, DC, kPP ? 1 : 0> : nullptr;
+        return fused_step_kernel<PB, SK, GB, kCorrNone, OPT, DC, 0>;
     case kCorrEF:
-        return fused_step_kernel<PB, SK, GB, kCorrEF, OPT, DC>;
+        if (pp)
+            return kPP ? fused_step_kernel<PB, SK, GB, kCorrEF, OPT, DC, kPP ? 1 : 0> : nullptr;
+        return fused_step_kernel<PB, SK, GB, kCorrEF, OPT, DC, 0>;
     case kCorrSapipeSame:
-        return fused_step_kernel<PB, SK, GB, kCorrSapipeSame, OPT, DC>;
+        return pp ? nullptr : fused_step_kernel<PB, SK, GB, kCorrSapipeSame, OPT, DC, 0>;
     case kCorrSapipeUpdated:   // the prediction step is defined for AdamW
-        return OPT != kOptAdamW ? nullptr
-                                : fused_step_kernel<PB, SK, GB, kCorrSapipeUpdated, OPT, DC>;
+        return pp || OPT != kOptAdamW
+                   ? nullptr
+                   : fused_step_kernel<PB, SK, GB, kCorrSapipeUpdated, OPT, DC, 0>;
     }
     return nullptr;
 }
 
 template <int PB, int GB, int OPT>
-StepFn pick_step_sk(StashKind sk, Correction corr, bool dc)
+StepFn pick_step_sk(StashKind sk, Correction corr, bool dc, bool pp)
 {
     switch (sk) {
     case kStashF32:
-        return dc ? pick_step_corr<PB, kStashF32, GB, OPT, 1>(corr)
-                  : pick_step_corr<PB, kStashF32, GB, OPT, 0>(corr);
+        return dc ? pick_step_corr<PB, kStashF32, GB, OPT, 1>(corr, pp)
+                  : pick_step_corr<PB, kStashF32, GB, OPT, 0>(corr, pp);
     case kStashBF16:
-        return dc ? pick_step_corr<PB, kStashBF16, GB, OPT, 1>(corr)
-                  : pick_step_corr<PB, kStashBF16, GB, OPT, 0>(corr);
+        return dc ? pick_step_corr<PB, kStashBF16, GB, OPT, 1>(corr, pp)
+                  : pick_step_corr<PB, kStashBF16, GB, OPT, 0>(corr, pp);
     default:   // synchronous: no stash, no correction, no compensation
-        return corr == kCorrNone && !dc ? fused_step_kernel<PB, kStashNone, GB, kCorrNone, OPT, 0>
-                                        : nullptr;
+        return corr == kCorrNone && !dc && !pp
+                   ? fused_step_kernel<PB, kStashNone, GB, kCorrNone, OPT, 0, 0>
+                   : nullptr;
     }
 }
 
 template <int OPT>
-StepFn pick_step(bool pb, StashKind sk, bool gb, Correction corr, bool dc)
+StepFn pick_step(bool pb, StashKind sk, bool gb, Correction corr, bool dc, bool pp)
 {
     if (pb)
-        return gb ? pick_step_sk<1, 1, OPT>(sk, corr, dc) : pick_step_sk<1, 0, OPT>(sk, corr, dc);
-    return gb ? pick_step_sk<0, 1, OPT>(sk, corr, dc) : pick_step_sk<0, 0, OPT>(sk, corr, dc);
+        return gb ? pick_step_sk<1, 1, OPT>(sk, corr, dc, pp)
+                  : pick_step_sk<1, 0, OPT>(sk, corr, dc, pp);
+    return gb ? pick_step_sk<0, 1, OPT>(sk, corr, dc, pp) : pick_step_sk<0, 0, OPT>(sk, corr, dc, pp);
 }
 
 }  // namespace

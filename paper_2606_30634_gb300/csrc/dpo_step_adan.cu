@@ -5,9 +5,9 @@
 namespace dpo {
 
 StepFn pick_step_adan(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr,
-                       bool dc)
+                       bool dc, bool pp)
 {
-    return pick_step<kOptAdan>(param_bf16, stash, grad_bf16, corr, dc);
+    return pick_step<kOptAdan>(param_bf16, stash, grad_bf16, corr, dc, pp);
 }
 
 }  // namespace dpo

@@ -28,6 +28,7 @@ DPO_INIT_FRESH, DPO_INIT_RESUME = 0, 1
 DPO_FLAG_NONFINITE = 1
 DPO_CORR_EF, DPO_CORR_SAPIPE_SAME, DPO_CORR_SAPIPE_UPDATED = 0, 1, 2
 DPO_OPT_ADAMW, DPO_OPT_NADAM, DPO_OPT_LION, DPO_OPT_ADAN = 0, 1, 2, 3
+DPO_STASH_COPY, DPO_STASH_PINGPONG = 0, 1
 
 EXPORTS = ("dpo_init", "dpo_stash", "dpo_step", "dpo_read_weights", "dpo_get_step",
            "dpo_set_step", "dpo_get_flags", "dpo_algorithmic_bytes", "dpo_launch_config",
@@ -50,7 +51,7 @@ class dpo_hparams(ctypes.Structure):
                 ("max_grad_norm", ctypes.c_float), ("delay", ctypes.c_int),
                 ("correction", ctypes.c_int), ("optimizer", ctypes.c_int),
                 ("beta3", ctypes.c_float), ("momentum_decay", ctypes.c_float),
-                ("dc_lambda", ctypes.c_float)]
+                ("dc_lambda", ctypes.c_float), ("stash_mode", ctypes.c_int)]
 
 
 class dpo_tensor(ctypes.Structure):
@@ -243,7 +244,7 @@ class DelayedAdamW:
                  init_mode=DPO_INIT_FRESH, stream=None, host_grad=False, host_param=False,
                  correction=DPO_CORR_EF, sync: Optional[Sequence[bool]] = None,
                  keep_stash: Optional[bool] = None, optimizer=DPO_OPT_ADAMW, beta3=0.99,
-                 momentum_decay=0.004, dc_lambda=0.0):
+                 momentum_decay=0.004, dc_lambda=0.0, stash_mode=DPO_STASH_COPY):
         import torch
         self.torch = torch
         self.device = torch.device(device or "cuda")
@@ -271,7 +272,7 @@ class DelayedAdamW:
             self.master.copy_(x0)
         self.hp = dpo_hparams(beta1, beta2, eps, weight_decay, ef_lambda if ef else 0.0,
                               max_grad_norm, delay, correction, optimizer, beta3,
-                              momentum_decay, dc_lambda)
+                              momentum_decay, dc_lambda, stash_mode)
         self.wd_on = list(wd_on) if wd_on is not None else [True] * len(numels)
         self.sync = list(sync) if sync is not None else [False] * len(numels)
         self.ctx = None
@@ -297,6 +298,14 @@ class DelayedAdamW:
         torch = self.torch
         k = self.k
         torch.cuda.synchronize(self.device)
+        if param and self.hp.stash_mode == DPO_STASH_PINGPONG:
+            # host weights take the copying stash: put both versions in their
+            # buffers' own roles first
+            latest, stale = self.role_arenas()
+            if latest is not self.param:
+                self.param.copy_(latest)
+                self.stash.copy_(stale)
+            self.hp.stash_mode = DPO_STASH_COPY
         dpo_destroy(self.ctx)
         self.ctx = None
         to_host = lambda t: torch.empty(t.shape, dtype=t.dtype, pin_memory=True).copy_(t)
@@ -314,11 +323,32 @@ class DelayedAdamW:
     def grads(self, i: int):
         return self.view(self.grad, i)
 
+    def _swapped(self, i: int) -> bool:
+        """Ping-pong stash: tensor i's param and stash buffers hold each
+        other's role (include/dpo.h, DPO_STASH_PINGPONG)."""
+        if self.hp.stash_mode != DPO_STASH_PINGPONG or self.delay != 1 or self.sync[i]:
+            return False
+        p, _ = dpo_read_weights(self.ctx, DPO_LATEST, i)
+        return p != self.table[i].param
+
     def stale(self, i: int):
         """What the next forward/backward reads (dpo_read_weights(DPO_STALE))."""
         if self.delay == 1 and not self.sync[i]:
-            return self.view(self.stash, i)
+            return self.view(self.param if self._swapped(i) else self.stash, i)
         return self.latest(i)
+
+    def role_arenas(self):
+        """(latest, stale) arenas, each tensor in its role: the param and stash
+        arenas, or (ping-pong stash, odd calls) copies with the delayed
+        tensors' slices exchanged."""
+        if self.stash is None or not any(self._swapped(i) for i in range(len(self.sync))):
+            return self.param, self.stash
+        latest, stale = self.param.clone(), self.stash.clone()
+        for i in range(len(self.sync)):
+            if self._swapped(i):
+                self.view(latest, i).copy_(self.view(self.stash, i))
+                self.view(stale, i).copy_(self.view(self.param, i))
+        return latest, stale
 
     def set_delay(self, delay: int, stream=None) -> None:
         """Switch between synchronous and delayed training (dpo_set_delay)."""
@@ -327,7 +357,9 @@ class DelayedAdamW:
         self.hp.delay = delay
 
     def latest(self, i: int):
-        return self.view(self.param if self.param is not None else self.master, i)
+        if self.param is None:
+            return self.view(self.master, i)
+        return self.view(self.stash if self._swapped(i) else self.param, i)
 
     def step(self, lr: Optional[float] = None, stream=None) -> None:
         dpo_step(self.ctx, self.lr if lr is None else lr, stream)

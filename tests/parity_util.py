@@ -134,6 +134,7 @@ class Case:
     schedule: Optional[dict] = None            # call k -> delay mode switched to before it
     host_grad: bool = False     # grad arena in pinned host memory
     host_param: bool = False    # bf16 param arena in pinned host memory
+    stash_mode: int = dpo.DPO_STASH_COPY   # or DPO_STASH_PINGPONG (bf16 param and stash)
 
 
 class Run:
@@ -154,7 +155,7 @@ class Run:
             host_grad=case.host_grad, host_param=case.host_param, correction=case.correction,
             sync=case.sync, keep_stash=True, optimizer=case.optimizer, beta1=case.beta1,
             beta2=case.beta2, beta3=case.beta3, momentum_decay=case.momentum_decay,
-            dc_lambda=case.dc_lambda)
+            dc_lambda=case.dc_lambda, stash_mode=case.stash_mode)
         # the oracle tracks every element, or only ``sample`` (global indices)
         self.sample = sample
         idx = np.arange(self.N) if sample is None else np.asarray(sample, np.int64)
@@ -254,8 +255,9 @@ class Run:
         GPU and the oracle (inputs of the next step)."""
         self.torch.cuda.synchronize()
         bad = self.gather(self.gpu.master).astype(np.float64) != self.ref.x
-        if self.gpu.stash is not None:
-            s = self.gather(self.gpu.stash)
+        _, stale = self.gpu.role_arenas()
+        if stale is not None:
+            s = self.gather(stale)
             if self.c.stash_dtype == dpo.DPO_BF16:
                 s = synth.bf16_bits_to_f32(s)
             bad |= s.astype(np.float64) != self.ref.stash
@@ -285,17 +287,22 @@ class Run:
             sync_sel = self.sync_mask & sel
             if sync_sel.any():
                 out["ef_sync_absdiff"] = float(np.max(np.abs(e[sync_sel] - r.u_prev[sync_sel])))
-        if g.stash is not None:
+        # the weight buffers in their roles (the ping-pong stash swaps them);
+        # under delay 0 the stale view is the latest weights and the stash
+        # buffer is not read (the ping-pong stash refreshes it on leaving
+        # delayed training, the copying stash leaves it as it was)
+        latest, stale = g.role_arenas()
+        if stale is not None and (g.delay == 1 or self.c.stash_mode == dpo.DPO_STASH_COPY):
             # the stash of a synchronously trained tensor is never read
             keep = ~self.sync_mask & sel
-            s, rs = self.gather(g.stash)[keep], r.stash[keep]
+            s, rs = self.gather(stale)[keep], r.stash[keep]
             if self.c.stash_dtype == dpo.DPO_BF16:
                 out["stash_ulp"] = bf16_ulps(s, rs)
                 out["stash_raw_ulp"] = bf16_raw_ulps(s, rs)
             else:
                 out["stash"] = rel_err(s, rs)
-        if g.param is not None:
-            p = self.gather(g.param)[sel]
+        if latest is not None:
+            p = self.gather(latest)[sel]
             out["param_ulp"] = bf16_ulps(p, r.param[sel])
             out["param_raw_ulp"] = bf16_raw_ulps(p, r.param[sel])
         return out

@@ -160,6 +160,9 @@ def _init(table, hp=None, pdt=dpo.DPO_BF16, sdt=dpo.DPO_F32, gdt=dpo.DPO_BF16, m
     ("empty_table", dpo.DPO_EINVAL),
     ("bad_flags", dpo.DPO_EINVAL),
     ("bad_mode", dpo.DPO_EINVAL),
+    ("bad_stash_mode", dpo.DPO_EINVAL),
+    ("pingpong_fp32_stash", dpo.DPO_EDTYPE),
+    ("pingpong_sapipe", dpo.DPO_EINVAL),
 ])
 def test_init_rejects(case, expect):
     tbl = [_t(0), _t(1, numel=7)]
@@ -198,6 +201,13 @@ def test_init_rejects(case, expect):
         tbl[0] = _t(0, flags=8)
     elif case == "bad_mode":
         kw = dict(mode=5)
+    elif case == "bad_stash_mode":
+        hp = _hp(stash_mode=2)
+    elif case == "pingpong_fp32_stash":
+        hp = _hp(stash_mode=dpo.DPO_STASH_PINGPONG)   # the helper's stash is fp32
+    elif case == "pingpong_sapipe":
+        hp = _hp(stash_mode=dpo.DPO_STASH_PINGPONG, correction=dpo.DPO_CORR_SAPIPE_SAME)
+        kw = dict(sdt=dpo.DPO_BF16)
     rc, out, msg = _init(tbl, hp, **kw)
     assert rc == expect, msg
     assert out is None

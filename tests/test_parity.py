@@ -369,6 +369,64 @@ def test_synchronous_start_then_delayed(cuda_device, ef, corr):
         run.close()
 
 
+# ---------------- ping-pong stash (PipeDream-2BW's two weight versions)
+
+PP = dpo.DPO_STASH_PINGPONG
+
+
+@pytest.mark.parametrize("ef,sync", [(True, False), (False, False), (True, True)])
+def test_pingpong_stash_parity(cuda_device, ef, sync):
+    """The bf16 param and stash buffers swap roles instead of the stash being
+    written: the latest and stale views, and all state, match the oracle over
+    odd and even calls (and with every other tensor trained synchronously)."""
+    sync_l = [i % 2 == 1 for i in range(len(RAGGED))] if sync else None
+    run = Run(Case(RAGGED, stash_dtype=B, ef=ef, sync=sync_l, stash_mode=PP), cuda_device)
+    try:
+        for k in range(1, 7):
+            run.step()
+            run.assert_close(TOL_ONE_STEP if k == 1 else TOL_RUN)
+    finally:
+        run.close()
+
+
+def test_pingpong_stash_switches(cuda_device):
+    """Synchronous start, delayed calls 3-5 (odd: the latest weights end in
+    the stash buffer), cooldown, and delayed again: the roles follow the
+    delayed phase and the synchronous calls find the latest weights."""
+    run = Run(Case(RAGGED, stash_dtype=B, ef=True, delay=0, schedule={3: 1, 6: 0, 8: 1},
+                   stash_mode=PP), cuda_device)
+    try:
+        for k in range(1, 11):
+            run.step()
+            run.assert_close(TOL_ONE_STEP if k == 1 else TOL_RUN)
+    finally:
+        run.close()
+
+
+@pytest.mark.parametrize("dc", [0.0, 1e4])
+def test_pingpong_equals_copy_stash_bitwise(cuda_device, dc):
+    """Same seeded run with the copying and the ping-pong stash: master, m, v,
+    EF buffer and the latest / stale weights bitwise equal after every call,
+    DC-ASGD included (it reads the stale buffer the new weights then overwrite)."""
+    runs = [Run(Case(RAGGED, stash_dtype=B, ef=True, dc_lambda=dc, stash_mode=m), cuda_device)
+            for m in (dpo.DPO_STASH_COPY, PP)]
+    try:
+        for k in range(1, 6):
+            for r in runs:
+                r.step()
+            torch.cuda.synchronize()
+            a, b = runs[0].gpu, runs[1].gpu
+            for name in ("master", "m", "v", "ef"):
+                assert torch.equal(getattr(a, name), getattr(b, name)), (k, name)
+            for ra, rb in zip(a.role_arenas(), b.role_arenas()):
+                assert torch.equal(ra.view(torch.int16), rb.view(torch.int16)), k
+            la, _ = dpo.dpo_read_weights(b.ctx, dpo.DPO_LATEST, 6)
+            assert la == (b.table[6].stash if k % 2 else b.table[6].param)
+    finally:
+        for r in runs:
+            r.close()
+
+
 def test_synchronous_cooldown(cuda_device):
     """App. A.10: delayed with EF for 5 calls, then synchronous."""
     run = Run(Case(RAGGED, ef=True, schedule={6: 0}), cuda_device)
