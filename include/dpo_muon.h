@@ -61,7 +61,9 @@ typedef struct {
     float *ef;          /* fp32 U_prev (Error Feedback history), or NULL (standard rule) */
     const void *grad;   /* gradient (grad dtype) */
     int64_t rows, cols; /* >= 0; a matrix with no elements is skipped */
-    uint32_t flags;     /* DPO_WD_ON */
+    uint32_t flags;     /* DPO_WD_ON; DPO_SYNC: trained synchronously even while the run
+                           is delayed (no stash, no correction; its gradient comes from
+                           the latest weights, as for dpo_tensor) */
 } dpo_matrix;
 
 typedef struct {
@@ -81,8 +83,8 @@ typedef struct dpo_muon_ctx dpo_muon_ctx;
 /*
  * Validate the matrices and settings, allocate the workspace and (init_mode
  * DPO_INIT_FRESH) enqueue the start state: mom = 0, ef = 0, stash and param
- * := master. Every matrix needs master, mom and grad; stash when delay = 1;
- * ef for all matrices or none. param_dtype is DPO_BF16; stash_dtype and
+ * := master. Every matrix needs master, mom and grad; a stash when delay = 1
+ * (unless DPO_SYNC); ef for all matrices or none. param_dtype is DPO_BF16; stash_dtype and
  * grad_dtype are DPO_F32 or DPO_BF16. Returns DPO_OK and *out, or DPO_EINVAL,
  * DPO_EALIGN, DPO_EDTYPE, DPO_ENOMEM or DPO_ECUDA and *out = NULL.
  */
@@ -97,6 +99,17 @@ int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n, dpo_dtype s
  * update pass. Returns DPO_OK, DPO_EINVAL or DPO_ECUDA.
  */
 int dpo_muon_step(dpo_muon_ctx *ctx, float lr, void *cuda_stream);
+
+/*
+ * Switch between synchronous (0) and one-step-delayed (1) training
+ * (synchronous start and cooldown, Sec. 3.1, App. A.10), as dpo_set_delay does
+ * for the elementwise path: entering delayed training stashes the current
+ * weights of every matrix without DPO_SYNC and zeroes the update history, so
+ * Alg. 1 restarts (its first delayed call takes the standard rule). Needs a
+ * stash for every such matrix (DPO_ESTATE otherwise). Returns DPO_OK,
+ * DPO_EINVAL, DPO_ESTATE or DPO_ECUDA.
+ */
+int dpo_muon_set_delay(dpo_muon_ctx *ctx, int delay, void *cuda_stream);
 
 /*
  * Newton-Schulz output O of the last step for matrix i, as a strided bf16

@@ -97,6 +97,13 @@ class DelayedMuon:
     stash holds X_0 and the master X_1 = X_0; with delay = 1 call k consumes
     the gradient evaluated at the stash and leaves the stash at X_k. Clipping
     takes the global norm over all matrices.
+
+    ``delayed`` marks per matrix whether it takes delayed updates (default
+    all; a synchronous matrix has no stash write and no correction, as WPipe
+    and the synchronous LM head train part of the model). ``set_delay``
+    switches the whole run between synchronous and delayed training
+    (synchronous start and cooldown, Sec. 3.1): entering delayed training
+    stashes the current weights and restarts Alg. 1.
     """
     x0: Sequence[np.ndarray]
     hp: MuonHParams = field(default_factory=MuonHParams)
@@ -105,6 +112,7 @@ class DelayedMuon:
     stash_store: int = F32
     param_store: Optional[int] = None
     lib: object = None
+    delayed: Optional[Sequence[bool]] = None
 
     def __post_init__(self):
         self.lib = self.lib or load()
@@ -118,26 +126,43 @@ class DelayedMuon:
         self.param = ([round_to(x, self.param_store, self.lib).reshape(x.shape) for x in self.x]
                       if self.param_store is not None else None)
         self.o = [np.zeros(s) for s in self.shapes]
+        self.delay = self.hp.delay
         self.k = 0
-        self.t = 0
+        self.t = 0   # Alg. 1 iteration within the current delayed phase
         self.last_clip = 1.0
+
+    def set_delay(self, delay: int) -> None:
+        """Switch between synchronous (0) and delayed (1) training; entering
+        delayed training stashes the current weights and zeroes the update
+        history (Alg. 1 restarts)."""
+        if delay == self.delay:
+            return
+        if delay == 1:
+            self.stash = [round_to(x, self.stash_store, self.lib).reshape(x.shape)
+                          for x in self.x]
+            if self.u_prev is not None:
+                for u in self.u_prev:
+                    u[...] = 0.0
+            self.t = 0
+        self.delay = delay
 
     def step(self, grads: Sequence[np.ndarray], lr: Optional[float] = None,
              sq: Optional[float] = None) -> None:
         grads = [_f64(g).reshape(s) for g, s in zip(grads, self.shapes)]
         self.k += 1
-        if self.hp.delay == 1:
+        if self.delay == 1:
             self.t += 1
         if sq is None:
             sq = sum(float(self.lib.oracle_sqnorm(g.size, _ptr(g))) for g in grads)
         clip = self.lib.oracle_clip_coef(sq, self.hp.max_grad_norm)
         self.last_clip = clip
         h = self.hp
-        hp = _MuonHParams(lr if lr is not None else h.lr, h.momentum, h.weight_decay,
-                          h.ef_lambda, h.ns_a, h.ns_b, h.ns_c, h.ns_steps, h.ns_eps,
-                          h.rms_scale, h.ns_store, h.delay, self.x_store, self.stash_store,
-                          self.param_store if self.param_store is not None else F64)
         for i, (rows, cols) in enumerate(self.shapes):
+            dly = self.delay if self.delayed is None or self.delayed[i] else 0
+            hp = _MuonHParams(lr if lr is not None else h.lr, h.momentum, h.weight_decay,
+                              h.ef_lambda, h.ns_a, h.ns_b, h.ns_c, h.ns_steps, h.ns_eps,
+                              h.rms_scale, h.ns_store, dly, self.x_store, self.stash_store,
+                              self.param_store if self.param_store is not None else F64)
             rc = self.lib.oracle_muon_step(
                 rows, cols, max(self.t, 1), ctypes.byref(hp), _ptr(grads[i]), clip,
                 _ptr(self.x[i]), _ptr(self.mom[i]),

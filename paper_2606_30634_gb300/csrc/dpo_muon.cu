@@ -54,6 +54,7 @@ struct DevMat {
     int64_t o_ld;
     float wd_lr_scale;        // 1 with DPO_WD_ON, else 0
     float r_scale;            // rms_scale sqrt(max(rows, cols)), or 1
+    int sync;                 // DPO_SYNC: trained synchronously (no stash, no history)
 };
 
 struct MomArgs {
@@ -230,23 +231,26 @@ __global__ void __launch_bounds__(kThreads) muon_apply_kernel(const ApplyArgs a)
     ST *stash = static_cast<ST *>(d.stash);
     __nv_bfloat16 *param = static_cast<__nv_bfloat16 *>(d.param);
     const bool vec_o = (d.cols % kPacket) == 0;
+    // a DPO_SYNC matrix takes the standard update with no stash and no history
+    const bool dly = a.delayed && !d.sync;
+    const bool hist = a.hist && dly, ef_now = a.ef_now && dly;
     for (int64_t e = lo + (int64_t)threadIdx.x * kPacket; e < hi; e += (int64_t)kThreads * kPacket) {
         if (e + kPacket <= hi && vec_o) {
             const int64_t i = e / d.cols, j = e - i * d.cols;
             float x[8], o[8], up[8], u[8];
             ld8(d.master + e, x);
             ld8(d.o + i * d.o_ld + j, o);
-            if (a.ef_now)
+            if (ef_now)
                 ld8(d.ef + e, up);
-            if (SK != kStashNone && a.delayed)
+            if (SK != kStashNone && dly)
                 st8(stash + e, x);
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
                 u[k] = fmaf(lr_r, o[k], lr_wd * x[k]);
-                x[k] -= a.ef_now ? fmaf(a.lam, u[k] - up[k], u[k]) : u[k];
+                x[k] -= ef_now ? fmaf(a.lam, u[k] - up[k], u[k]) : u[k];
             }
             st8(d.master + e, x);
-            if (a.hist)
+            if (hist)
                 st8(d.ef + e, u);
             if (param != nullptr)
                 st8(param + e, x);
@@ -256,12 +260,12 @@ __global__ void __launch_bounds__(kThreads) muon_apply_kernel(const ApplyArgs a)
                 const int64_t i = q / d.cols, j = q - i * d.cols;
                 float x = d.master[q];
                 const float o = __bfloat162float(d.o[i * d.o_ld + j]);
-                if (SK != kStashNone && a.delayed)
+                if (SK != kStashNone && dly)
                     st1(stash + q, x);
                 const float u = fmaf(lr_r, o, lr_wd * x);
-                x -= a.ef_now ? fmaf(a.lam, u - d.ef[q], u) : u;
+                x -= ef_now ? fmaf(a.lam, u - d.ef[q], u) : u;
                 d.master[q] = x;
-                if (a.hist)
+                if (hist)
                     d.ef[q] = u;
                 if (param != nullptr)
                     st1(param + q, x);
@@ -270,9 +274,12 @@ __global__ void __launch_bounds__(kThreads) muon_apply_kernel(const ApplyArgs a)
     }
 }
 
-// Start state: mom = 0, ef = 0, stash := master, param := master.
+// Start state (zero_mom, zero_ef: mom = 0, ef = 0) or the restart of Alg. 1
+// on entering delayed training (zero_ef only): stash := master for matrices
+// trained delayed, param := master.
 template <int SK>
-__global__ void __launch_bounds__(kThreads) muon_init_kernel(const DevMat *mats, int zero_ef)
+__global__ void __launch_bounds__(kThreads) muon_init_kernel(const DevMat *mats, int zero_mom,
+                                                             int zero_ef)
 {
     using ST = typename StashT<SK>::T;
     const DevMat &d = mats[blockIdx.y];
@@ -282,10 +289,11 @@ __global__ void __launch_bounds__(kThreads) muon_init_kernel(const DevMat *mats,
     for (int64_t q = (int64_t)blockIdx.x * kThreads + threadIdx.x; q < n;
          q += (int64_t)gridDim.x * kThreads) {
         const float x = d.master[q];
-        d.mom[q] = 0.0f;
+        if (zero_mom)
+            d.mom[q] = 0.0f;
         if (zero_ef && d.ef != nullptr)
             d.ef[q] = 0.0f;
-        if (SK != kStashNone && stash != nullptr)
+        if (SK != kStashNone && stash != nullptr && !d.sync)
             st1(stash + q, x);
         if (param != nullptr)
             st1(param + q, x);
@@ -364,7 +372,10 @@ struct dpo_muon_ctx {
     dpo_dtype stash_dt = DPO_F32, grad_dt = DPO_F32;
     dpo_muon_hparams hp{};
     bool ef = false;
+    bool has_stash = false;   // some matrix has a stash buffer
+    bool can_delay = true;    // every matrix without DPO_SYNC has one
     int64_t k = 0;
+    int64_t phase_k0 = 0;     // k when the current delayed phase began
     int sms = 0;
     int gemm_pairs = 0;   // clusters of 2 the GEMM kernel keeps resident at once
     std::vector<dpo_matrix> mats;
@@ -432,7 +443,7 @@ void free_ctx(dpo_muon_ctx *c)
     delete c;
 }
 
-int launch_init(dpo_muon_ctx *c, cudaStream_t s, int zero_ef)
+int launch_init(dpo_muon_ctx *c, cudaStream_t s, int zero_mom, int zero_ef)
 {
     int64_t max_n = 0;
     for (const dpo_matrix &m : c->mats)
@@ -441,13 +452,13 @@ int launch_init(dpo_muon_ctx *c, cudaStream_t s, int zero_ef)
         return DPO_OK;
     const dim3 grid((unsigned)std::min<int64_t>((max_n + kThreads - 1) / kThreads, 4096),
                     (unsigned)c->n);
-    const bool st = c->hp.delay == 1 || c->mats[0].stash != nullptr;
-    if (!st)
-        dpo::muon::muon_init_kernel<dpo::kStashNone><<<grid, kThreads, 0, s>>>(c->d_mats, zero_ef);
+    const DevMat *m = c->d_mats;
+    if (!c->has_stash)
+        dpo::muon::muon_init_kernel<dpo::kStashNone><<<grid, kThreads, 0, s>>>(m, zero_mom, zero_ef);
     else if (c->stash_dt == DPO_BF16)
-        dpo::muon::muon_init_kernel<dpo::kStashBF16><<<grid, kThreads, 0, s>>>(c->d_mats, zero_ef);
+        dpo::muon::muon_init_kernel<dpo::kStashBF16><<<grid, kThreads, 0, s>>>(m, zero_mom, zero_ef);
     else
-        dpo::muon::muon_init_kernel<dpo::kStashF32><<<grid, kThreads, 0, s>>>(c->d_mats, zero_ef);
+        dpo::muon::muon_init_kernel<dpo::kStashF32><<<grid, kThreads, 0, s>>>(m, zero_mom, zero_ef);
     const cudaError_t e = cudaGetLastError();
     return e == cudaSuccess ? DPO_OK : mcuda(c, e, "muon init launch");
 }
@@ -489,7 +500,9 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
             continue;
         if (m.master == nullptr || m.mom == nullptr || m.grad == nullptr)
             return mfail(nullptr, DPO_EINVAL, "matrix %d: master, mom and grad are required", i);
-        if (hp->delay == 1 && m.stash == nullptr)
+        if ((m.flags & ~(DPO_WD_ON | DPO_SYNC)) != 0)
+            return mfail(nullptr, DPO_EINVAL, "matrix %d: unknown flags", i);
+        if (hp->delay == 1 && m.stash == nullptr && !(m.flags & DPO_SYNC))
             return mfail(nullptr, DPO_EINVAL, "matrix %d: delay 1 needs a stash", i);
         if ((m.ef != nullptr) != ef)
             return mfail(nullptr, DPO_EINVAL, "ef buffers must be given for all matrices or none");
@@ -506,6 +519,12 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
     c->hp = *hp;
     c->ef = ef;
     c->mats.assign(mats, mats + n);
+    for (int i = 0; i < n; ++i) {
+        if (mats[i].rows * mats[i].cols == 0)
+            continue;
+        c->has_stash = c->has_stash || mats[i].stash != nullptr;
+        c->can_delay = c->can_delay && (mats[i].stash != nullptr || (mats[i].flags & DPO_SYNC));
+    }
     cudaGetDevice(&c->device);
     cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, c->device);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -634,6 +653,7 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
         d.r_scale = hp->rms_scale > 0.0f
                         ? (float)(hp->rms_scale * std::sqrt((double)std::max(m.rows, m.cols)))
                         : 1.0f;
+        d.sync = (m.flags & DPO_SYNC) ? 1 : 0;
     }
     for (size_t gi = 0; gi < c->groups.size(); ++gi) {
         Group &g = c->groups[gi];
@@ -729,7 +749,7 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
                                 : mfail(nullptr, DPO_ECUDA, "GEMM kernel cannot be resident");
     }
     if (init_mode == DPO_INIT_FRESH) {
-        const int rc = launch_init(c, s, 1);
+        const int rc = launch_init(c, s, 1, 1);
         if (rc != DPO_OK) {
             g_muon_init_err = c->err;
             free_ctx(c);
@@ -882,7 +902,7 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
     }
 
     // update, stash, history, weights
-    const int64_t t = k;   // Alg. 1 iteration (delayed from the start)
+    const int64_t t = k - c->phase_k0;   // Alg. 1 iteration within the delayed phase
     dpo::muon::ApplyArgs aa{};
     aa.mats = c->d_mats;
     aa.chunks = c->chunks;
@@ -902,6 +922,28 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
     if ((e = cudaGetLastError()) != cudaSuccess)
         return mcuda(c, e, "apply launch");
     c->k = k;
+    return DPO_OK;
+}
+
+extern "C" int dpo_muon_set_delay(dpo_muon_ctx *c, int delay, void *stream)
+{
+    if (c == nullptr)
+        return DPO_EINVAL;
+    if (delay != 0 && delay != 1)
+        return mfail(c, DPO_EINVAL, "delay must be 0 or 1");
+    if (delay == c->hp.delay)
+        return DPO_OK;
+    if (delay == 1) {
+        if (!c->can_delay)
+            return mfail(c, DPO_ESTATE,
+                         "delayed training needs a stash for every matrix without DPO_SYNC");
+        // stash := the current weights, update history := 0: Alg. 1 restarts
+        const int rc = launch_init(c, static_cast<cudaStream_t>(stream), 0, 1);
+        if (rc != DPO_OK)
+            return rc;
+        c->phase_k0 = c->k;
+    }
+    c->hp.delay = delay;
     return DPO_OK;
 }
 

@@ -10,8 +10,8 @@ from __future__ import annotations
 import ctypes
 from typing import List, Optional, Sequence, Tuple
 
-from .dpo import (DPO_BF16, DPO_F32, DPO_INIT_FRESH, DPO_OK, DPO_WD_ON, ALIGN_ELEMS, DpoError,
-                  _stream, load)
+from .dpo import (DPO_BF16, DPO_F32, DPO_INIT_FRESH, DPO_OK, DPO_SYNC, DPO_WD_ON, ALIGN_ELEMS,
+                  DpoError, _stream, load)
 
 NS_COEFFS = (3.4445, -4.7750, 2.0315)
 
@@ -31,7 +31,8 @@ class dpo_muon_hparams(ctypes.Structure):
                 ("ns_steps", ctypes.c_int), ("delay", ctypes.c_int)]
 
 
-EXPORTS = ("dpo_muon_init", "dpo_muon_step", "dpo_muon_last_update", "dpo_muon_copy_update",
+EXPORTS = ("dpo_muon_init", "dpo_muon_step", "dpo_muon_set_delay", "dpo_muon_last_update",
+           "dpo_muon_copy_update",
            "dpo_muon_get_status",
            "dpo_muon_get_step", "dpo_muon_set_step", "dpo_muon_flops",
            "dpo_muon_set_timing", "dpo_muon_get_gemm_time",
@@ -49,6 +50,7 @@ def lib() -> ctypes.CDLL:
             "dpo_muon_init": (I, [ctypes.POINTER(P), ctypes.POINTER(dpo_matrix), I, I, I,
                                   ctypes.POINTER(dpo_muon_hparams), I, P]),
             "dpo_muon_step": (I, [P, F, P]),
+            "dpo_muon_set_delay": (I, [P, I, P]),
             "dpo_muon_last_update": (I, [P, I, ctypes.POINTER(P),
                                          ctypes.POINTER(ctypes.c_int64)]),
             "dpo_muon_copy_update": (I, [P, I, P, P]),
@@ -93,7 +95,8 @@ class DelayedMuon:
                  grad_dtype=DPO_BF16, lr=2e-3, momentum=0.95, weight_decay=0.1, ef=False,
                  ef_lambda=1.0, max_grad_norm=0.0, coeffs=NS_COEFFS, ns_eps=1e-7,
                  rms_scale=0.2, ns_steps=5, delay=1, wd_on: Optional[Sequence[bool]] = None,
-                 device=None, x0=None, init_mode=DPO_INIT_FRESH, stream=None):
+                 device=None, x0=None, init_mode=DPO_INIT_FRESH, stream=None,
+                 sync: Optional[Sequence[bool]] = None, keep_stash: Optional[bool] = None):
         import torch
         self.torch = torch
         self.device = torch.device(device or "cuda")
@@ -111,7 +114,8 @@ class DelayedMuon:
         self.ef = alloc(torch.float32) if ef else None
         self.grad = alloc(tdt[grad_dtype])
         self.param = alloc(torch.bfloat16)
-        self.stash = alloc(tdt[stash_dtype]) if delay == 1 else None
+        keep_stash = delay == 1 if keep_stash is None else keep_stash
+        self.stash = alloc(tdt[stash_dtype]) if keep_stash else None
         self.lr, self.delay = lr, delay
         if isinstance(x0, (list, tuple)):   # one array per matrix
             for i, xi in enumerate(x0):
@@ -122,12 +126,14 @@ class DelayedMuon:
         self.hp = hparams(momentum, weight_decay, ef_lambda if ef else 0.0, max_grad_norm,
                           coeffs, ns_eps, rms_scale, ns_steps, delay)
         wd_on = list(wd_on) if wd_on is not None else [True] * len(self.shapes)
+        self.sync = list(sync) if sync is not None else [False] * len(self.shapes)
         ptr = lambda t, off: (t.data_ptr() + off * t.element_size()) if t is not None else None
         mats = []
-        for (r, c), off, wd in zip(self.shapes, self.offsets, wd_on):
+        for (r, c), off, wd, sy in zip(self.shapes, self.offsets, wd_on, self.sync):
             mats.append(dpo_matrix(ptr(self.param, off), ptr(self.master, off),
                                    ptr(self.mom, off), ptr(self.stash, off), ptr(self.ef, off),
-                                   ptr(self.grad, off), r, c, DPO_WD_ON if wd else 0))
+                                   ptr(self.grad, off), r, c,
+                                   (DPO_WD_ON if wd else 0) | (DPO_SYNC if sy else 0)))
         self.table = mats
         L = lib()
         arr = (dpo_matrix * len(mats))(*mats)
@@ -144,7 +150,14 @@ class DelayedMuon:
         return self.view(self.grad, i)
 
     def stale(self, i: int):
-        return self.view(self.stash if self.delay == 1 else self.param, i)
+        """What the next forward/backward reads for matrix i."""
+        return self.view(self.stash if self.delay == 1 and not self.sync[i] else self.param, i)
+
+    def set_delay(self, delay: int, stream=None) -> None:
+        """Switch between synchronous and delayed training (dpo_muon_set_delay)."""
+        _check(lib().dpo_muon_set_delay(self.ctx, delay, _stream(stream)), self.ctx)
+        self.delay = delay
+        self.hp.delay = delay
 
     def step(self, lr: Optional[float] = None, stream=None) -> None:
         _check(lib().dpo_muon_step(self.ctx, self.lr if lr is None else lr, _stream(stream)),

@@ -59,23 +59,31 @@ class Pair:
     """The GPU context and the oracle on the same seeded inputs."""
 
     def __init__(self, shapes, device, seed=0x3A0, ns_steps=5, ef=True, delay=1, sdt=B,
-                 lr=2e-3, momentum=0.95, wd=0.1, max_grad_norm=0.0, rms_scale=0.2):
+                 lr=2e-3, momentum=0.95, wd=0.1, max_grad_norm=0.0, rms_scale=0.2, sync=None,
+                 schedule=None):
         self.shapes, self.seed, self.lr = shapes, seed, lr
+        self.schedule = schedule or {}
         xs, _ = inputs(shapes, seed, 1)
         self.gpu = muon.DelayedMuon(shapes, stash_dtype=sdt, grad_dtype=B, lr=lr,
                                     momentum=momentum, weight_decay=wd, ef=ef,
                                     max_grad_norm=max_grad_norm, rms_scale=rms_scale,
                                     ns_steps=ns_steps, delay=delay, device=device,
-                                    x0=[torch.from_numpy(x) for x in xs])
+                                    x0=[torch.from_numpy(x) for x in xs], sync=sync,
+                                    keep_stash=True)
         hp = MuonHParams(lr=lr, momentum=momentum, weight_decay=wd, ef_lambda=1.0,
                          ns_steps=ns_steps, rms_scale=rms_scale, ns_store=oracle.BF16,
                          max_grad_norm=max_grad_norm, delay=delay).as_f32()
         self.ref = OracleMuon([x.astype(np.float64) for x in xs], hp, ef=ef, x_store=oracle.F32,
                               stash_store=oracle.BF16 if sdt == B else oracle.F32,
-                              param_store=oracle.BF16)
+                              param_store=oracle.BF16,
+                              delayed=None if sync is None else [not q for q in sync])
+        self.sync = sync or [False] * len(shapes)
         self.k = 0
 
     def step(self):
+        if self.k + 1 in self.schedule:
+            self.gpu.set_delay(self.schedule[self.k + 1])
+            self.ref.set_delay(self.schedule[self.k + 1])
         self.k += 1
         _, gs = inputs(self.shapes, self.seed, self.k + 1)
         for i, g in enumerate(gs):
@@ -178,6 +186,34 @@ def test_muon_step_parity(cuda_device, steps, sdt, ef, delay):
                                  2.0 ** -7 if sdt == B else TOL_RUN, k * du, 1e-3)
             if ef and delay == 1:
                 close_with_flips(p.cat(p.gpu.ef), _flat(p.ref.u_prev), 1e-5, du, 2e-3)
+    finally:
+        p.close()
+
+
+@pytest.mark.parametrize("sync,schedule", [(True, None), (False, {1: 0, 3: 1, 5: 0}),
+                                           (True, {1: 0, 2: 1})])
+def test_muon_sync_matrices_and_mode_switches(cuda_device, sync, schedule):
+    """Per-matrix synchronous training (every other matrix) and synchronous
+    start / cooldown: Alg. 1 restarts at each switch into delayed training.
+    One Newton-Schulz step, so O agrees up to rare flips (module note)."""
+    sync_l = [i % 2 == 1 for i in range(len(SHAPES))] if sync else None
+    p = Pair(SHAPES, cuda_device, ns_steps=1, ef=True, sync=sync_l, schedule=schedule,
+             delay=0 if schedule else 1)
+    r_max = 0.2 * np.sqrt(max(max(sh) for sh in SHAPES))
+    du = p.lr * r_max * 2.0 ** -7
+    try:
+        for k in range(6):
+            p.step()
+            assert rel_err(p.cat(p.gpu.mom), _flat(p.ref.mom)) <= (TOL_ONE_STEP if k == 0
+                                                                    else TOL_RUN)
+            close_with_flips(p.cat(p.gpu.master), _flat(p.ref.x), TOL_RUN, (k + 1) * du, 1e-3)
+            u, ur = p.cat(p.gpu.ef), _flat(p.ref.u_prev)
+            close_with_flips(u, ur, 1e-5, du, 2e-3)
+            if p.gpu.delay == 1:
+                keep = np.concatenate([np.full(r * c, not p.sync[i]) for i, (r, c)
+                                       in enumerate(SHAPES)])
+                st = p.cat(p.gpu.stash).astype(np.float64)[keep]
+                close_with_flips(st, _flat(p.ref.stash)[keep], 2.0 ** -7, k * du, 1e-3)
     finally:
         p.close()
 

@@ -206,3 +206,59 @@ def test_muon_empty_and_clip(lib):
     opt.step([np.zeros((0, 4)), g])
     assert opt.last_clip == pytest.approx(1.0 / (6.0 + 1e-6), rel=1e-15)
     np.testing.assert_allclose(opt.mom[1], 0.05 * g * opt.last_clip, rtol=1e-15)
+
+
+def test_muon_per_matrix_delay_is_independent(lib):
+    """A table mixing a delayed and a synchronous matrix gives, matrix by
+    matrix, bitwise the runs of each matrix alone in its mode; the
+    synchronous one never writes its stash or history."""
+    rng = np.random.default_rng(10)
+    x0 = [rng.normal(size=(4, 6)), rng.normal(size=(7, 3))]
+    grads = [[rng.normal(size=(4, 6)), rng.normal(size=(7, 3))] for _ in range(4)]
+    mixed = DelayedMuon(x0, _hp(ef_lambda=1.0), ef=True, x_store=F64, stash_store=F64,
+                        delayed=[True, False], lib=lib)
+    alone = [DelayedMuon([x0[0]], _hp(ef_lambda=1.0), ef=True, x_store=F64, stash_store=F64,
+                         lib=lib),
+             DelayedMuon([x0[1]], _hp(ef_lambda=1.0, delay=0), ef=True, x_store=F64,
+                         stash_store=F64, lib=lib)]
+    for g in grads:
+        mixed.step(g)
+        alone[0].step([g[0]])
+        alone[1].step([g[1]])
+    assert np.array_equal(mixed.x[0], alone[0].x[0])
+    assert np.array_equal(mixed.x[1], alone[1].x[0])
+    assert np.array_equal(mixed.stash[1], x0[1]) and not np.any(mixed.u_prev[1])
+
+
+def test_muon_synchronous_start_restarts_alg1(lib):
+    """Two synchronous calls, then delayed: the switch stashes the current
+    weights and zeroes the history; the first delayed call takes the
+    standard rule, the next ones Alg. 2's EF line; the stash lags by one."""
+    rng = np.random.default_rng(11)
+    x0 = rng.normal(size=(5, 8))
+    opt = DelayedMuon([x0], _hp(ef_lambda=1.0, delay=0), ef=True, x_store=F64,
+                      stash_store=F64, lib=lib)
+    scale = 0.2 * math.sqrt(8)
+    for _ in range(2):
+        xt = opt.x[0].copy()
+        opt.step([rng.normal(size=(5, 8))])
+        np.testing.assert_allclose(opt.x[0], xt - 0.01 * (scale * opt.o[0] + 0.1 * xt),
+                                   rtol=1e-13)
+    assert not np.any(opt.u_prev[0])
+    opt.set_delay(1)
+    assert np.array_equal(opt.stash[0], opt.x[0])
+    us = []
+    for k in range(3):
+        xt = opt.x[0].copy()
+        opt.step([rng.normal(size=(5, 8))])
+        us.append(0.01 * (scale * opt.o[0] + 0.1 * xt))
+        assert np.array_equal(opt.stash[0], xt)
+        want = xt - us[0] if k == 0 else xt - 2 * us[k] + us[k - 1]
+        np.testing.assert_allclose(opt.x[0], want, rtol=1e-13)
+    # cooldown: the standard rule again, stash and history left as they were
+    opt.set_delay(0)
+    stash, hist = opt.stash[0].copy(), opt.u_prev[0].copy()
+    xt = opt.x[0].copy()
+    opt.step([rng.normal(size=(5, 8))])
+    np.testing.assert_allclose(opt.x[0], xt - 0.01 * (scale * opt.o[0] + 0.1 * xt), rtol=1e-13)
+    assert np.array_equal(opt.stash[0], stash) and np.array_equal(opt.u_prev[0], hist)
