@@ -229,6 +229,18 @@ def rule_settings(args) -> dict:
     return dict(base, dc_lambda=args.dc_lambda)
 
 
+def resolve_stash(args, w) -> str:
+    """--stash auto: the ping-pong stash where the layout allows it (bf16
+    param and stash buffers, the standard rule or EF, the elementwise path),
+    else the copying stash."""
+    from paper_2606_30634_gb300.synth import workloads as W
+    if args.stash != "auto":
+        return args.stash
+    ok = (w.param_dtype == W.BF16 and w.stash_dtype == W.BF16
+          and args.mode in ("ef", "std") and args.optimizer != "muon")
+    return "pingpong" if ok else "copy"
+
+
 def wpipe_sync(w, args):
     """Per-tensor DPO_SYNC flags: the second half of the tensor list under
     --wpipe (WPipe trains the second half of the model without delay)."""
@@ -622,10 +634,7 @@ def main(argv=None):
     args = parse_args(argv)
     from paper_2606_30634_gb300.synth import workloads as W
     w = W.ALL[args.workload]
-    if args.stash == "auto":
-        ok = (w.param_dtype == W.BF16 and w.stash_dtype == W.BF16
-              and args.mode in ("ef", "std") and args.optimizer != "muon")
-        args.stash = "pingpong" if ok else "copy"
+    args.stash = resolve_stash(args, w)
     world, rank, local = dist_env()
     if args.optimizer == "muon":
         return main_muon(args, w, world, rank, local)

@@ -1,6 +1,7 @@
 """Host-side logic of bench.py: the max-over-ranks timing and whole-job
 aggregation across processes (gloo, world size 2, CPU only), the JSON of the
-reference arm, and the committed-traffic lookup."""
+reference arm, the committed-traffic lookup, the choice of stash mode and the
+division of a set between Muon and AdamW."""
 from __future__ import annotations
 
 import json
@@ -69,3 +70,28 @@ def test_reference_arm_json_line():
 
 def test_traffic_lookup_ignores_stale_summaries(tmp_path, monkeypatch):
     assert bench.committed_traffic("no-such-kernel") is None
+
+
+@pytest.mark.parametrize("argv,want", [
+    ([], "pingpong"),                                  # llama-7B: bf16 param and stash, EF
+    (["--mode", "std"], "pingpong"),
+    (["--mode", "sapipe-same"], "copy"),               # the stash holds a prediction
+    (["--workload", "gpt2-small-124M"], "copy"),       # fp32 stash
+    (["--optimizer", "muon"], "copy"),
+    (["--stash", "copy"], "copy"),
+])
+def test_stash_mode_resolution(argv, want):
+    from paper_2606_30634_gb300.synth import workloads as W
+    args = bench.parse_args(argv)
+    assert bench.resolve_stash(args, W.ALL[args.workload]) == want
+
+
+def test_muon_takes_the_attention_and_mlp_matrices():
+    from paper_2606_30634_gb300.synth import workloads as W
+    mi, ai = bench.muon_split(W.LLAMA_7B)
+    assert len(mi) == 32 * 7 and len(ai) == len(W.LLAMA_7B.tensors) - 32 * 7
+    assert sum(W.LLAMA_7B.numels[i] for i in mi) == 32 * (4 * 4096 * 4096 + 3 * 4096 * 11008)
+    names = [W.LLAMA_7B.tensors[i][0] for i in ai]
+    assert "embed_tokens" in names and "lm_head" in names and "norm" in names
+    mi, _ = bench.muon_split(W.GPT2_SMALL)
+    assert len(mi) == 12 * 4 and all(len(W.GPT2_SMALL.tensors[i][1]) == 2 for i in mi)
