@@ -57,6 +57,8 @@ def parse_args(argv=None):
                    help="muon: delayed Muon (Alg. 2) on the attention and MLP matrices, "
                         "AdamW on the rest")
     p.add_argument("--ns-steps", type=int, default=5, help="Newton-Schulz steps (muon)")
+    p.add_argument("--no-library-ns", action="store_true",
+                   help="muon: skip timing the cuBLAS Newton-Schulz chain for context")
     p.add_argument("--stash", choices=["auto", "copy", "pingpong"], default="auto",
                    help="pingpong: bf16 param and stash buffers swap roles (no stash store); "
                         "auto: pingpong where the layout allows it (bf16 param and stash, "
@@ -461,10 +463,51 @@ def run_muon(args, w, world, rank, local):
     ad.close()
     if status != 0:
         raise RuntimeError(f"tensor-core pipeline status {status}")
+    library = None if args.no_library_ns else library_ns(shapes, args.ns_steps, dev)
     return dict(value=value, t_max=t_max, achieved=achieved, flops=flops, gemm_ms=gemm_ms / K,
                 gemm_launches=gemm_launches, clocks=clocks, launches=K * launches_per_step,
                 n_muon=sum(w.numels[i] for i in mi), n_matrices=len(mi), workspace=ws,
-                device_name=props.name)
+                device_name=props.name, library=library)
+
+
+def library_ns(shapes, steps: int, dev, reps: int = 3):
+    """Context for the Newton-Schulz roofline: the same iteration on the same
+    matrix shapes with cuBLAS (torch.matmul / baddbmm in bf16, full
+    products), one batched chain per shape as the library runs it, timed
+    with CUDA events. Not part of the measured step."""
+    import torch
+    a_, b_, c_ = 3.4445, -4.7750, 2.0315
+    groups = {}
+    for r, c in shapes:
+        key = (min(r, c), max(r, c))
+        groups[key] = groups.get(key, 0) + 1
+
+    def chain(X):
+        for _ in range(steps):
+            A = torch.bmm(X, X.transpose(1, 2))
+            B = torch.baddbmm(A, A, A, beta=b_, alpha=c_)
+            X = torch.baddbmm(X, B, X, beta=a_, alpha=1.0)
+        return X
+
+    gen = torch.Generator(device=dev).manual_seed(0)
+    Xs = [torch.randn(nb, r, w, device=dev, dtype=torch.bfloat16, generator=gen) * 0.01
+          for (r, w), nb in groups.items()]
+    full = sum(steps * nb * (4.0 * r * r * w + 2.0 * r * r * r) for (r, w), nb in groups.items())
+    for X in Xs:
+        chain(X)
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        for X in Xs:
+            chain(X)
+    e1.record()
+    torch.cuda.synchronize(dev)
+    ms = e0.elapsed_time(e1) / reps
+    del Xs
+    torch.cuda.empty_cache()
+    return {"what": "cuBLAS bf16 Newton-Schulz chain (torch bmm/baddbmm, full products) on the "
+                    "same matrix shapes", "ms_per_step": ms, "tflops_full_products": full / ms / 1e9}
 
 
 def oracle_muon_sample(seconds: float, rows: int = 1024, cols: int = 4096):
@@ -608,7 +651,7 @@ def main_muon(args, w, world, rank, local):
             "traffic": None, "kernel": "ns_gemm_kernel",
             "algorithmic_flops_per_step": r["flops"], "gemm_ms_per_step": r["gemm_ms"],
             "gemm_launches_per_step": r["gemm_launches"] / max(1, args.steps),
-            "nominal_peak_tflops": 2250.0}
+            "nominal_peak_tflops": 2250.0, "library_newton_schulz": r["library"]}
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         v, cores, steps, n = oracle_muon_sample(args.cpu_seconds)
