@@ -194,6 +194,7 @@ class Run:
             self.ref.delay_mask = (~self.sync_mask).astype(np.uint8)
         # arena index of every tracked element
         t_of = np.searchsorted(self.offs, idx, side="right") - 1
+        self._t_of = t_of
         arena_off = np.asarray(self.gpu.layout.offsets, np.int64)
         self.arena_idx = arena_off[t_of] + (idx - self.offs[t_of])
         self._arena_idx_cpu = torch.from_numpy(self.arena_idx)
@@ -250,14 +251,27 @@ class Run:
             return t.view(self.torch.int16).cpu().numpy().view(np.uint16)
         return t.cpu().numpy()
 
+    def role_values(self):
+        """(latest, stale) weights of the tracked elements, each tensor's two
+        weight buffers read in their roles (the ping-pong stash swaps them on
+        odd calls; include/dpo.h, DPO_STASH_PINGPONG)."""
+        g = self.gpu
+        p = self.gather(g.param) if g.param is not None else None
+        st = self.gather(g.stash) if g.stash is not None else None
+        if p is None or st is None or self.c.stash_mode != dpo.DPO_STASH_PINGPONG:
+            return p, st
+        swapped = np.array([g._swapped(i) for i in range(len(self.c.numels))], bool)
+        m = swapped[self._t_of]
+        return np.where(m, st, p), np.where(m, p, st)
+
     def input_mismatch(self) -> np.ndarray:
         """Tracked elements whose master or stash differ bitwise between the
         GPU and the oracle (inputs of the next step)."""
         self.torch.cuda.synchronize()
         bad = self.gather(self.gpu.master).astype(np.float64) != self.ref.x
-        _, stale = self.gpu.role_arenas()
+        _, stale = self.role_values()
         if stale is not None:
-            s = self.gather(stale)
+            s = stale
             if self.c.stash_dtype == dpo.DPO_BF16:
                 s = synth.bf16_bits_to_f32(s)
             bad |= s.astype(np.float64) != self.ref.stash
@@ -291,18 +305,18 @@ class Run:
         # under delay 0 the stale view is the latest weights and the stash
         # buffer is not read (the ping-pong stash refreshes it on leaving
         # delayed training, the copying stash leaves it as it was)
-        latest, stale = g.role_arenas()
+        latest, stale = self.role_values()
         if stale is not None and (g.delay == 1 or self.c.stash_mode == dpo.DPO_STASH_COPY):
             # the stash of a synchronously trained tensor is never read
             keep = ~self.sync_mask & sel
-            s, rs = self.gather(stale)[keep], r.stash[keep]
+            s, rs = stale[keep], r.stash[keep]
             if self.c.stash_dtype == dpo.DPO_BF16:
                 out["stash_ulp"] = bf16_ulps(s, rs)
                 out["stash_raw_ulp"] = bf16_raw_ulps(s, rs)
             else:
                 out["stash"] = rel_err(s, rs)
         if latest is not None:
-            p = self.gather(latest)[sel]
+            p = latest[sel]
             out["param_ulp"] = bf16_ulps(p, r.param[sel])
             out["param_raw_ulp"] = bf16_raw_ulps(p, r.param[sel])
         return out

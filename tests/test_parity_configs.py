@@ -34,11 +34,18 @@ pytestmark = pytest.mark.gpu
 FULL = os.environ.get("DPO_FULL_RUNS", "0") == "1"
 
 
-def _case(w: W.Workload, ef: bool, correction: int = dpo.DPO_CORR_EF) -> Case:
+def _case(w: W.Workload, ef: bool, correction: int = dpo.DPO_CORR_EF,
+          stash_mode: int = None) -> Case:
+    """The workload as the benchmark runs it: the ping-pong stash where the
+    layout allows it (bf16 param and stash, the standard rule or EF)."""
+    if stash_mode is None:
+        pp = (w.param_dtype == W.BF16 and w.stash_dtype == W.BF16
+              and correction == dpo.DPO_CORR_EF)
+        stash_mode = dpo.DPO_STASH_PINGPONG if pp else dpo.DPO_STASH_COPY
     return Case(w.numels, param_dtype=w.param_dtype, stash_dtype=w.stash_dtype,
                 grad_dtype=w.grad_dtype, ef=ef, max_grad_norm=w.max_grad_norm, lr=w.lr,
                 weight_decay=w.weight_decay, seed=w.seed, grad_sigma=W.GRAD_SIGMA,
-                init_sigma=W.INIT_SIGMA, correction=correction)
+                init_sigma=W.INIT_SIGMA, correction=correction, stash_mode=stash_mode)
 
 
 def _free():
@@ -143,12 +150,15 @@ def test_llama_1b_clipped(cuda_device):
         _free()
 
 
-@pytest.mark.parametrize("ef", [True, False])
-def test_llama_7b(cuda_device, ef):
+@pytest.mark.parametrize("ef,stash", [(True, None), (False, None),
+                                      (True, dpo.DPO_STASH_COPY)])
+def test_llama_7b(cuda_device, ef, stash):
     """The 6.74e9-parameter set: bf16 params, stash and grads, fp32
-    master/m/v (and EF buffer): ~148 GB resident with EF."""
+    master/m/v (and EF buffer): ~148 GB resident with EF. As the benchmark
+    runs it (the ping-pong stash), and with the copying stash."""
     w = W.LLAMA_7B
-    run = Run(_case(w, ef), cuda_device, sample=sample_indices(w.numels, 1_000_000))
+    run = Run(_case(w, ef, stash_mode=stash), cuda_device,
+              sample=sample_indices(w.numels, 1_000_000))
     try:
         _run_steps(run, w.steps, check_every=5)
     finally:
