@@ -400,14 +400,21 @@ int oracle_muon_step(int64_t rows, int64_t cols, int64_t t, const oracle_muon_hp
     const double s = hp->rms_scale > 0.0
                          ? hp->rms_scale * sqrt((double)(rows > cols ? rows : cols))
                          : 1.0;
+    if (hp->correction != ORACLE_CORR_EF && hp->correction != ORACLE_CORR_SAPIPE_SAME) {
+        free(O);
+        return -1;
+    }
     const int use_ef = hp->delay == 1 && u_prev != NULL;
+    const int sapipe = use_ef && hp->correction == ORACLE_CORR_SAPIPE_SAME;
     /* Alg. 1 / Alg. 2: the standard rule at t <= 1, EF from t = 2. */
-    const int ef_now = use_ef && t >= 2;
+    const int ef_now = use_ef && !sapipe && t >= 2;
     for (int64_t i = 0; i < n; ++i) {
         const double xt = x[i];
         const double u = hp->lr * (s * O[i] + hp->weight_decay * xt);
         const double xn = ef_now ? xt - u - hp->ef_lambda * (u - u_prev[i]) : xt - u;
-        if (hp->delay == 1)   /* the weights the next gradient is evaluated at */
+        if (sapipe)   /* SAPipe-WP: the next gradient is taken at x_t - U_prev */
+            stash[i] = oracle_round(oracle_round(x[i] - u_prev[i], hp->x_store), hp->stash_store);
+        else if (hp->delay == 1)   /* the weights the next gradient is evaluated at */
             stash[i] = oracle_round(x[i], hp->stash_store);
         if (use_ef)
             u_prev[i] = oracle_round(u, hp->x_store);

@@ -202,6 +202,9 @@ typedef struct {
     double rms_scale;      /* see above; 0 = no scaling */
     int ns_store;          /* storage of every Newton-Schulz matrix: F64 or BF16 */
     int delay;             /* 1 = one-step-delayed, 0 = synchronous */
+    int correction;        /* ORACLE_CORR_EF or ORACLE_CORR_SAPIPE_SAME (App. B.1: the
+                              weights take the standard rule, the stash receives the
+                              prediction point X_t - U_prev, the history U) */
     int x_store;           /* storage of X, M and U_prev (F64 or F32) */
     int stash_store;       /* storage of the stash */
     int param_store;       /* storage of the latest-weights copy */

@@ -44,6 +44,7 @@ class _MuonHParams(ctypes.Structure):
         ("rms_scale", ctypes.c_double),
         ("ns_store", ctypes.c_int),
         ("delay", ctypes.c_int),
+        ("correction", ctypes.c_int),
         ("x_store", ctypes.c_int),
         ("stash_store", ctypes.c_int),
         ("param_store", ctypes.c_int),
@@ -65,6 +66,7 @@ class MuonHParams:
     ns_store: int = BF16
     max_grad_norm: float = 0.0
     delay: int = 1
+    correction: int = 0   # CORR_EF, or CORR_SAPIPE_SAME (App. B.1)
 
     def as_f32(self) -> "MuonHParams":
         """Every real rounded to fp32, as a device taking fp32 settings sees them."""
@@ -72,7 +74,7 @@ class MuonHParams:
         return MuonHParams(r(self.lr), r(self.momentum), r(self.weight_decay),
                            r(self.ef_lambda), r(self.ns_a), r(self.ns_b), r(self.ns_c),
                            self.ns_steps, r(self.ns_eps), r(self.rms_scale), self.ns_store,
-                           r(self.max_grad_norm), self.delay)
+                           r(self.max_grad_norm), self.delay, self.correction)
 
 
 def newton_schulz(M, steps: int = 5, store: int = F64, eps: float = 1e-7,
@@ -161,7 +163,8 @@ class DelayedMuon:
             dly = self.delay if self.delayed is None or self.delayed[i] else 0
             hp = _MuonHParams(lr if lr is not None else h.lr, h.momentum, h.weight_decay,
                               h.ef_lambda, h.ns_a, h.ns_b, h.ns_c, h.ns_steps, h.ns_eps,
-                              h.rms_scale, h.ns_store, dly, self.x_store, self.stash_store,
+                              h.rms_scale, h.ns_store, dly, h.correction, self.x_store,
+                              self.stash_store,
                               self.param_store if self.param_store is not None else F64)
             rc = self.lib.oracle_muon_step(
                 rows, cols, max(self.t, 1), ctypes.byref(hp), _ptr(grads[i]), clip,

@@ -262,3 +262,33 @@ def test_muon_synchronous_start_restarts_alg1(lib):
     opt.step([rng.normal(size=(5, 8))])
     np.testing.assert_allclose(opt.x[0], xt - 0.01 * (scale * opt.o[0] + 0.1 * xt), rtol=1e-13)
     assert np.array_equal(opt.stash[0], stash) and np.array_equal(opt.u_prev[0], hist)
+
+
+def test_muon_sapipe_same_state(lib):
+    """SAPipe-WP with the same state (App. B.1): the weights are bitwise the
+    standard rule's; the stash holds the prediction point X_t - U_prev, so
+    consecutive prediction points move by Eq. (1)'s displacement -2U + U_prev,
+    which an independent EF run's weights show (zero decay: the updates of
+    the two runs are the same)."""
+    rng = np.random.default_rng(12)
+    x0 = rng.normal(size=(4, 6))
+    grads = [rng.normal(size=(4, 6)) for _ in range(6)]
+    sp = DelayedMuon([x0], _hp(weight_decay=0.0, correction=oracle.CORR_SAPIPE_SAME), ef=True,
+                     x_store=F64, stash_store=F64, lib=lib)
+    std = DelayedMuon([x0], _hp(weight_decay=0.0), x_store=F64, stash_store=F64, lib=lib)
+    ef = DelayedMuon([x0], _hp(weight_decay=0.0, ef_lambda=1.0), ef=True, x_store=F64,
+                     stash_store=F64, lib=lib)
+    stash, efx = [], [x0.copy()]
+    for g in grads:
+        xt = sp.x[0].copy()
+        hist = sp.u_prev[0].copy()
+        for o in (sp, std, ef):
+            o.step([g])
+        assert np.array_equal(sp.x[0], std.x[0])
+        assert np.array_equal(sp.stash[0], xt - hist)
+        stash.append(sp.stash[0].copy())
+        efx.append(ef.x[0].copy())
+    # stash after call k+1 minus after call k == EF weights after call k minus after call k-1
+    for k in range(2, len(grads)):
+        np.testing.assert_allclose(stash[k] - stash[k - 1], efx[k] - efx[k - 1],
+                                   rtol=1e-9, atol=1e-15)

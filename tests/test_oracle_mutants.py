@@ -78,8 +78,11 @@ MUTANTS = [
      "hp->lr * (s * O[i] + hp->weight_decay * (hp->delay == 1 ? stash[i] : xt))"),
     ("muon_stash_holds_new_weights", "stash[i] = oracle_round(x[i], hp->stash_store);",
      "stash[i] = oracle_round(xn, hp->stash_store);"),
-    ("muon_ef_at_first_update", "const int ef_now = use_ef && t >= 2;",
-     "const int ef_now = use_ef && t >= 1;"),
+    ("muon_sapipe_predicts_with_current_update",
+     "oracle_round(oracle_round(x[i] - u_prev[i], hp->x_store), hp->stash_store)",
+     "oracle_round(oracle_round(x[i] - u, hp->x_store), hp->stash_store)"),
+    ("muon_ef_at_first_update", "const int ef_now = use_ef && !sapipe && t >= 2;",
+     "const int ef_now = use_ef && !sapipe && t >= 1;"),
 ]
 
 
