@@ -23,6 +23,8 @@
  *   X_{t+1} = X_t - U - lambda (U - U_prev)     Error Feedback (Eq. (1);
  *        Alg. 2 is lambda = 1: X_t - 2 U_{t-1} + U_{t-2})
  *   stash := X_t,  U_prev := U,  param := bf16(X_{t+1})
+ *   With correction DPO_CORR_SAPIPE_SAME (SAPipe-WP, App. B.1) the weights take
+ *   the standard rule and the stash receives the predicted point X_t - U_prev.
  *
  * The k-th dpo_muon_step is Alg. 1's iteration t = k (t = 0 only sets
  * X_1 = X_0). With delay = 0 the same update runs on gradients of the latest
@@ -76,6 +78,10 @@ typedef struct {
     float rms_scale;      /* 0.2: match the update RMS; 0: no scaling */
     int ns_steps;         /* iterations, 0..16 (5) */
     int delay;            /* 1: one-step-delayed (Alg. 1 / 2); 0: synchronous */
+    int correction;       /* with ef buffers: DPO_CORR_EF (lambda-scaled Error Feedback) or
+                             DPO_CORR_SAPIPE_SAME (SAPipe-WP with the same state, App. B.1:
+                             the weights take the standard rule, the stash receives the
+                             prediction point X_t - U_prev, the history U) */
 } dpo_muon_hparams;
 
 typedef struct dpo_muon_ctx dpo_muon_ctx;

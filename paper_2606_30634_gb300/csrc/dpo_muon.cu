@@ -215,6 +215,7 @@ struct ApplyArgs {
     int chunks;
     float lr, lr_wd, lam;
     int ef_now, hist, delayed;
+    int sapipe;               // SAPipe-WP same state: stash := x_t - U_prev, standard rule
 };
 
 template <int SK>
@@ -234,16 +235,26 @@ __global__ void __launch_bounds__(kThreads) muon_apply_kernel(const ApplyArgs a)
     // a DPO_SYNC matrix takes the standard update with no stash and no history
     const bool dly = a.delayed && !d.sync;
     const bool hist = a.hist && dly, ef_now = a.ef_now && dly;
+    const bool sapipe = a.sapipe && hist;
     for (int64_t e = lo + (int64_t)threadIdx.x * kPacket; e < hi; e += (int64_t)kThreads * kPacket) {
         if (e + kPacket <= hi && vec_o) {
             const int64_t i = e / d.cols, j = e - i * d.cols;
             float x[8], o[8], up[8], u[8];
             ld8(d.master + e, x);
             ld8(d.o + i * d.o_ld + j, o);
-            if (ef_now)
+            if (ef_now || sapipe)
                 ld8(d.ef + e, up);
-            if (SK != kStashNone && dly)
-                st8(stash + e, x);
+            if (SK != kStashNone && dly) {
+                if (sapipe) {   // the prediction point x_t - U_prev
+                    float xp[8];
+#pragma unroll
+                    for (int k = 0; k < 8; ++k)
+                        xp[k] = x[k] - up[k];
+                    st8(stash + e, xp);
+                } else {
+                    st8(stash + e, x);
+                }
+            }
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
                 u[k] = fmaf(lr_r, o[k], lr_wd * x[k]);
@@ -261,7 +272,7 @@ __global__ void __launch_bounds__(kThreads) muon_apply_kernel(const ApplyArgs a)
                 float x = d.master[q];
                 const float o = __bfloat162float(d.o[i * d.o_ld + j]);
                 if (SK != kStashNone && dly)
-                    st1(stash + q, x);
+                    st1(stash + q, sapipe ? x - d.ef[q] : x);
                 const float u = fmaf(lr_r, o, lr_wd * x);
                 x -= ef_now ? fmaf(a.lam, u - d.ef[q], u) : u;
                 d.master[q] = x;
@@ -489,6 +500,10 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
         !(hp->ns_eps >= 0.0f) || !(hp->rms_scale >= 0.0f) || (hp->delay != 0 && hp->delay != 1) ||
         !std::isfinite(hp->ns_a) || !std::isfinite(hp->ns_b) || !std::isfinite(hp->ns_c))
         return mfail(nullptr, DPO_EINVAL, "hyperparameter out of range");
+    if (hp->correction != DPO_CORR_EF && hp->correction != DPO_CORR_SAPIPE_SAME)
+        return mfail(nullptr, DPO_EINVAL,
+                     "correction must be DPO_CORR_EF or DPO_CORR_SAPIPE_SAME (the updated-state "
+                     "prediction would need a second Newton-Schulz iteration)");
     if (init_mode != DPO_INIT_FRESH && init_mode != DPO_INIT_RESUME)
         return mfail(nullptr, DPO_EINVAL, "bad init_mode");
     const bool ef = n > 0 && mats[0].ef != nullptr;
@@ -910,7 +925,8 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
     aa.lr_wd = (float)((double)lr * (double)c->hp.weight_decay);
     aa.delayed = c->hp.delay == 1;
     aa.hist = c->ef && c->hp.delay == 1;
-    aa.ef_now = aa.hist && t >= 2 && c->hp.ef_lambda != 0.0f;
+    aa.sapipe = c->hp.correction == DPO_CORR_SAPIPE_SAME;
+    aa.ef_now = aa.hist && !aa.sapipe && t >= 2 && c->hp.ef_lambda != 0.0f;
     aa.lam = c->hp.ef_lambda;
     const bool st = c->hp.delay == 1;
     if (!st)

@@ -28,7 +28,8 @@ class dpo_muon_hparams(ctypes.Structure):
                 ("ef_lambda", ctypes.c_float), ("max_grad_norm", ctypes.c_float),
                 ("ns_a", ctypes.c_float), ("ns_b", ctypes.c_float), ("ns_c", ctypes.c_float),
                 ("ns_eps", ctypes.c_float), ("rms_scale", ctypes.c_float),
-                ("ns_steps", ctypes.c_int), ("delay", ctypes.c_int)]
+                ("ns_steps", ctypes.c_int), ("delay", ctypes.c_int),
+                ("correction", ctypes.c_int)]
 
 
 EXPORTS = ("dpo_muon_init", "dpo_muon_step", "dpo_muon_set_delay", "dpo_muon_last_update",
@@ -80,9 +81,10 @@ def _check(rc: int, ctx) -> None:
 
 def hparams(momentum=0.95, weight_decay=0.1, ef_lambda=1.0, max_grad_norm=0.0,
             coeffs=NS_COEFFS, ns_eps=1e-7, rms_scale=0.2, ns_steps=5,
-            delay=1) -> dpo_muon_hparams:
+            delay=1, correction=0) -> dpo_muon_hparams:
     return dpo_muon_hparams(momentum, weight_decay, ef_lambda, max_grad_norm, coeffs[0],
-                            coeffs[1], coeffs[2], ns_eps, rms_scale, ns_steps, delay)
+                            coeffs[1], coeffs[2], ns_eps, rms_scale, ns_steps, delay,
+                            correction)
 
 
 class DelayedMuon:
@@ -96,7 +98,8 @@ class DelayedMuon:
                  ef_lambda=1.0, max_grad_norm=0.0, coeffs=NS_COEFFS, ns_eps=1e-7,
                  rms_scale=0.2, ns_steps=5, delay=1, wd_on: Optional[Sequence[bool]] = None,
                  device=None, x0=None, init_mode=DPO_INIT_FRESH, stream=None,
-                 sync: Optional[Sequence[bool]] = None, keep_stash: Optional[bool] = None):
+                 sync: Optional[Sequence[bool]] = None, keep_stash: Optional[bool] = None,
+                 correction: int = 0):
         import torch
         self.torch = torch
         self.device = torch.device(device or "cuda")
@@ -124,7 +127,7 @@ class DelayedMuon:
             self.master.copy_(x0)
         self.stash_dtype, self.grad_dtype = stash_dtype, grad_dtype
         self.hp = hparams(momentum, weight_decay, ef_lambda if ef else 0.0, max_grad_norm,
-                          coeffs, ns_eps, rms_scale, ns_steps, delay)
+                          coeffs, ns_eps, rms_scale, ns_steps, delay, correction)
         wd_on = list(wd_on) if wd_on is not None else [True] * len(self.shapes)
         self.sync = list(sync) if sync is not None else [False] * len(self.shapes)
         ptr = lambda t, off: (t.data_ptr() + off * t.element_size()) if t is not None else None

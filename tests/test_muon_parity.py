@@ -60,7 +60,7 @@ class Pair:
 
     def __init__(self, shapes, device, seed=0x3A0, ns_steps=5, ef=True, delay=1, sdt=B,
                  lr=2e-3, momentum=0.95, wd=0.1, max_grad_norm=0.0, rms_scale=0.2, sync=None,
-                 schedule=None):
+                 schedule=None, correction=0):
         self.shapes, self.seed, self.lr = shapes, seed, lr
         self.schedule = schedule or {}
         xs, _ = inputs(shapes, seed, 1)
@@ -69,10 +69,11 @@ class Pair:
                                     max_grad_norm=max_grad_norm, rms_scale=rms_scale,
                                     ns_steps=ns_steps, delay=delay, device=device,
                                     x0=[torch.from_numpy(x) for x in xs], sync=sync,
-                                    keep_stash=True)
+                                    keep_stash=True, correction=correction)
         hp = MuonHParams(lr=lr, momentum=momentum, weight_decay=wd, ef_lambda=1.0,
                          ns_steps=ns_steps, rms_scale=rms_scale, ns_store=oracle.BF16,
-                         max_grad_norm=max_grad_norm, delay=delay).as_f32()
+                         max_grad_norm=max_grad_norm, delay=delay,
+                         correction=correction).as_f32()
         self.ref = OracleMuon([x.astype(np.float64) for x in xs], hp, ef=ef, x_store=oracle.F32,
                               stash_store=oracle.BF16 if sdt == B else oracle.F32,
                               param_store=oracle.BF16,
@@ -214,6 +215,25 @@ def test_muon_sync_matrices_and_mode_switches(cuda_device, sync, schedule):
                                        in enumerate(SHAPES)])
                 st = p.cat(p.gpu.stash).astype(np.float64)[keep]
                 close_with_flips(st, _flat(p.ref.stash)[keep], 2.0 ** -7, k * du, 1e-3)
+    finally:
+        p.close()
+
+
+def test_muon_sapipe_same_state(cuda_device):
+    """SAPipe-WP with the same state (App. B.1): the stash receives the
+    prediction point X_t - U_prev, the weights take the standard rule."""
+    p = Pair(SHAPES, cuda_device, ns_steps=1, ef=True, correction=1)
+    r_max = 0.2 * np.sqrt(max(max(sh) for sh in SHAPES))
+    du = p.lr * r_max * 2.0 ** -7
+    try:
+        for k in range(5):
+            p.step()
+            assert rel_err(p.cat(p.gpu.mom), _flat(p.ref.mom)) <= (TOL_ONE_STEP if k == 0
+                                                                    else TOL_RUN)
+            close_with_flips(p.cat(p.gpu.master), _flat(p.ref.x), TOL_RUN, (k + 1) * du, 1e-3)
+            close_with_flips(p.cat(p.gpu.ef), _flat(p.ref.u_prev), 1e-5, du, 2e-3)
+            close_with_flips(p.cat(p.gpu.stash).astype(np.float64), _flat(p.ref.stash), 2.0 ** -7,
+                             (k + 1) * du, 1e-3)
     finally:
         p.close()
 
