@@ -222,10 +222,39 @@ int dpo_stash(dpo_ctx *ctx, void *cuda_stream);
  * consumes every tensor's grad, updates master, m, v (and the EF buffer),
  * writes stash := x_t (delay == 1) and param := x_{t+1}, then k += 1.
  * With clipping, first computes the global gradient norm over all tensors
- * (deterministic, fixed reduction order). Asynchronous on cuda_stream, no
+ * (deterministic, fixed reduction order), or takes it from the clip source
+ * set by dpo_set_clip_source. Asynchronous on cuda_stream, no
  * host synchronization, no allocation. lr must be finite and >= 0.
  */
 int dpo_step(dpo_ctx *ctx, float lr, void *cuda_stream);
+
+/*
+ * One global gradient norm across contexts and ranks. Clipping scales every
+ * gradient by one coefficient from the norm over all parameters (App. E.1);
+ * when those parameters are split over several contexts (an AdamW context
+ * for the vectors and embeddings beside a dpo_muon context for the
+ * matrices, or one shard per rank of a partitioned set), each context adds
+ * its share and all of them clip from the total:
+ *
+ *   dpo_grad_sqnorm: enqueue on cuda_stream  *d_sumsq += sum of g^2  over
+ *     this context's gradients (fp64; the same fixed-order reduction as
+ *     dpo_step's own norm pass, whatever max_grad_norm is). d_sumsq is
+ *     caller-owned device memory, 8-byte aligned; contributions to it must
+ *     be ordered (one stream, or events), and the caller zeroes it before
+ *     the first. A context with no elements adds nothing.
+ *   dpo_set_clip_source: with d_sumsq != NULL, every later dpo_step clips
+ *     from sqrt(*d_sumsq) (read on the device when the step runs) instead of
+ *     computing its own norm: coefficient min(1, max_grad_norm /
+ *     (sqrt(*d_sumsq) + 1e-6)). NULL goes back to the context's own norm.
+ *     Needs max_grad_norm > 0 (DPO_ESTATE otherwise). The pointer must stay
+ *     valid while it is set.
+ *
+ * Summing the per-rank values of *d_sumsq (an all-reduce) between the two
+ * calls is the one exchange a partitioned step needs. Both return DPO_OK,
+ * DPO_EINVAL, DPO_ESTATE or DPO_ECUDA.
+ */
+int dpo_grad_sqnorm(dpo_ctx *ctx, double *d_sumsq, void *cuda_stream);
+int dpo_set_clip_source(dpo_ctx *ctx, const double *d_sumsq);
 
 /*
  * Switch the run between synchronous (delay = 0) and one-step-delayed
@@ -266,7 +295,8 @@ int dpo_get_flags(dpo_ctx *ctx, uint32_t *flags, double *grad_norm,
 /*
  * Bytes one dpo_step must move through memory by the layout of the context
  * (algorithmic, not measured): *step_bytes for the fused step over all
- * tensors, *norm_bytes for the gradient-norm pass (0 without clipping).
+ * tensors, *norm_bytes for the gradient-norm pass (0 without clipping, or
+ * with a clip source: dpo_grad_sqnorm then reads the gradients once more).
  */
 int dpo_algorithmic_bytes(const dpo_ctx *ctx, int64_t *step_bytes,
                           int64_t *norm_bytes);

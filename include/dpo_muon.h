@@ -6,7 +6,8 @@
  * its stale gradient G_{t-1} (evaluated at the stashed weights):
  *
  *   G^ = s G,  s = min(1, max_norm / (||G||_2 + 1e-6))   global clipping over
- *        all matrices of the context (App. E.1), 1 when max_grad_norm <= 0
+ *        all matrices of the context, or over every parameter through a
+ *        shared clip source (App. E.1), 1 when max_grad_norm <= 0
  *   M  = mu M + (1 - mu) G^          momentum as an exponential moving average
  *        (Sec. 2.2's convention for the momentum decay mu; Alg. 2 prints the
  *        two weights the other way round)
@@ -137,6 +138,15 @@ int dpo_muon_copy_update(const dpo_muon_ctx *ctx, int i, void *dst, void *cuda_s
  * context's last work. Returns DPO_OK or DPO_ECUDA.
  */
 int dpo_muon_get_status(dpo_muon_ctx *ctx, uint32_t *bits);
+
+/*
+ * The global gradient norm shared with other contexts (see dpo_grad_sqnorm
+ * and dpo_set_clip_source in dpo.h, which these follow): add this context's
+ * sum of G^2 over all its matrices to *d_sumsq, and clip later steps from
+ * the total. Returns DPO_OK, DPO_EINVAL, DPO_ESTATE or DPO_ECUDA.
+ */
+int dpo_muon_grad_sqnorm(dpo_muon_ctx *ctx, double *d_sumsq, void *cuda_stream);
+int dpo_muon_set_clip_source(dpo_muon_ctx *ctx, const double *d_sumsq);
 
 /* Calls consumed so far (k), and restore after loading a checkpoint. */
 int dpo_muon_get_step(const dpo_muon_ctx *ctx, int64_t *k);

@@ -11,6 +11,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cstdint>
 #include <cstring>
 #include <cmath>
 #include <cstdarg>
@@ -46,6 +47,7 @@ struct dpo_ctx {
     int64_t *d_pkt_begin = nullptr;
     double *d_partials = nullptr;
     dpo::NormScalars *d_scalars = nullptr;
+    const double *clip_src = nullptr;   // external sum of squares (dpo_set_clip_source)
     std::string err;
 };
 
@@ -538,7 +540,12 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
     const int64_t t = k - c->phase_k0; // Alg. 1 iteration within the delayed phase
     cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
     if (c->total_pkts > 0) {
-        if (c->clip) {
+        if (c->clip && c->clip_src != nullptr) {
+            const cudaError_t e = dpo::launch_clip_from_sumsq(
+                c->clip_src, (double)c->hp.max_grad_norm, c->d_scalars, s);
+            if (e != cudaSuccess)
+                return cuda_fail(c, e, "clip-coefficient launch");
+        } else if (c->clip) {
             dpo::NormArgs na{c->d_table, c->d_pkt_begin, c->n, c->total_pkts,
                              (double)c->hp.max_grad_norm, c->d_partials, c->d_scalars};
             const cudaError_t e = dpo::launch_norm(c->grad_dt == DPO_BF16, c->norm_grid, na, s);
@@ -591,6 +598,35 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
     }
     c->mu_prod *= nadam_mu(c->hp, k);
     c->k = k;
+    return DPO_OK;
+}
+
+extern "C" int dpo_grad_sqnorm(dpo_ctx *c, double *d_sumsq, void *cuda_stream)
+{
+    if (c == nullptr)
+        return fail(nullptr, DPO_EINVAL, "ctx is NULL");
+    if (d_sumsq == nullptr || reinterpret_cast<uintptr_t>(d_sumsq) % alignof(double) != 0)
+        return fail(c, DPO_EINVAL, "d_sumsq must be an 8-byte aligned device pointer");
+    if (c->total_pkts == 0)
+        return DPO_OK;
+    dpo::NormArgs na{c->d_table, c->d_pkt_begin, c->n, c->total_pkts, 0.0, c->d_partials,
+                     c->d_scalars, d_sumsq};
+    const cudaError_t e = dpo::launch_norm(c->grad_dt == DPO_BF16, c->norm_grid, na,
+                                           static_cast<cudaStream_t>(cuda_stream));
+    if (e != cudaSuccess)
+        return cuda_fail(c, e, "gradient-norm launch");
+    return DPO_OK;
+}
+
+extern "C" int dpo_set_clip_source(dpo_ctx *c, const double *d_sumsq)
+{
+    if (c == nullptr)
+        return fail(nullptr, DPO_EINVAL, "ctx is NULL");
+    if (d_sumsq != nullptr && reinterpret_cast<uintptr_t>(d_sumsq) % alignof(double) != 0)
+        return fail(c, DPO_EINVAL, "d_sumsq must be 8-byte aligned");
+    if (d_sumsq != nullptr && !c->clip)
+        return fail(c, DPO_ESTATE, "a clip source needs max_grad_norm > 0");
+    c->clip_src = d_sumsq;
     return DPO_OK;
 }
 
@@ -687,7 +723,8 @@ extern "C" int dpo_algorithmic_bytes(const dpo_ctx *c, int64_t *step_bytes, int6
     if (step_bytes)
         *step_bytes = total;
     if (norm_bytes)
-        *norm_bytes = c->clip ? dt_size(c->grad_dt) * c->total_elems : 0;
+        *norm_bytes = c->clip && c->clip_src == nullptr ? dt_size(c->grad_dt) * c->total_elems
+                                                        : 0;
     return DPO_OK;
 }
 

@@ -98,6 +98,7 @@ struct NormArgs {
     double max_norm;            // clip threshold (> 0)
     double *partials;           // one per CTA (scratch)
     NormScalars *out;           // norm, clip coefficient, ticket, flags
+    double *accum;              // non-null: add ||g||^2 to *accum, form no coefficient
 };
 
 struct StashArgs {
@@ -127,6 +128,9 @@ cudaError_t launch_step(Optimizer opt, bool param_bf16, StashKind stash, bool gr
                         Correction corr, bool dc, bool pp, int grid, const StepArgs &a,
                         cudaStream_t s);
 cudaError_t launch_norm(bool grad_bf16, int grid, const NormArgs &a, cudaStream_t s);
+// Clip coefficient and norm from an external sum of squares (one thread).
+cudaError_t launch_clip_from_sumsq(const double *sumsq, double max_norm, NormScalars *out,
+                                   cudaStream_t s);
 cudaError_t launch_stash(bool param_bf16, StashKind stash, int grid, const StashArgs &a,
                          cudaStream_t s);
 

@@ -75,6 +75,24 @@ __device__ __forceinline__ float packet_sqsum(const GT *grad, int64_t e, int64_t
     return s;
 }
 
+// Norm and clip coefficient min(1, max_norm / (norm + 1e-6)) from a sum of
+// squares; a NaN norm stays NaN and reaches every element.
+__device__ void finish_clip(double total, double max_norm, NormScalars *out)
+{
+    const double norm = sqrt(total);
+    double coef = max_norm / (norm + 1e-6);
+    coef = coef > 1.0 ? 1.0 : coef;
+    if (!isfinite(total))
+        out->flags |= 1u;
+    out->clip = (float)coef;
+    out->norm = norm;
+}
+
+__global__ void clip_from_sumsq_kernel(const double *sumsq, double max_norm, NormScalars *out)
+{
+    finish_clip(*sumsq, max_norm, out);
+}
+
 template <int GB>
 __global__ void __launch_bounds__(kNormThreads) grad_sqnorm_kernel(const NormArgs a)
 {
@@ -132,13 +150,13 @@ __global__ void __launch_bounds__(kNormThreads) grad_sqnorm_kernel(const NormArg
         acc += __ldcg(a.partials + b);
     const double total = block_sum<kNormThreads>(acc, red);
     if (threadIdx.x == 0) {
-        const double norm = sqrt(total);
-        double coef = a.max_norm / (norm + 1e-6);
-        coef = coef > 1.0 ? 1.0 : coef;   // a NaN norm stays NaN and reaches every element
-        if (!isfinite(total))
-            a.out->flags |= 1u;
-        a.out->clip = (float)coef;
-        a.out->norm = norm;
+        if (a.accum != nullptr) {   // one share of a norm over several contexts
+            if (!isfinite(total))
+                a.out->flags |= 1u;
+            *a.accum += total;
+        } else {
+            finish_clip(total, a.max_norm, a.out);
+        }
         a.out->ticket = 0u;   // ready for the next launch
     }
 }
@@ -257,6 +275,13 @@ cudaError_t launch_norm(bool gb, int grid, const NormArgs &a, cudaStream_t s)
         grad_sqnorm_kernel<1><<<grid, kNormThreads, 0, s>>>(a);
     else
         grad_sqnorm_kernel<0><<<grid, kNormThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_clip_from_sumsq(const double *sumsq, double max_norm, NormScalars *out,
+                                   cudaStream_t s)
+{
+    clip_from_sumsq_kernel<<<1, 1, 0, s>>>(sumsq, max_norm, out);
     return cudaGetLastError();
 }
 

@@ -408,6 +408,7 @@ struct dpo_muon_ctx {
     int64_t *d_pkt_begin = nullptr;
     double *d_norm_partials = nullptr;
     dpo::NormScalars *d_norm_scalars = nullptr;
+    const double *clip_src = nullptr;   // external sum of squares (dpo_muon_set_clip_source)
     int64_t total_pkts = 0;
     int norm_grid = 0;
     // GEMM timing (dpo_muon_set_timing): event pairs recorded since the last read
@@ -811,7 +812,12 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
         return DPO_OK;
     }
     const bool clip = c->hp.max_grad_norm > 0.0f;
-    if (clip) {
+    if (clip && c->clip_src != nullptr) {
+        const cudaError_t e = dpo::launch_clip_from_sumsq(c->clip_src, c->hp.max_grad_norm,
+                                                          c->d_norm_scalars, s);
+        if (e != cudaSuccess)
+            return mcuda(c, e, "clip-coefficient launch");
+    } else if (clip) {
         dpo::NormArgs na{};
         na.table = c->d_norm_table;
         na.pkt_begin = c->d_pkt_begin;
@@ -995,6 +1001,41 @@ extern "C" int dpo_muon_get_status(dpo_muon_ctx *c, uint32_t *bits)
     if (e != cudaSuccess)
         return mcuda(c, e, "status read");
     *bits = v;
+    return DPO_OK;
+}
+
+extern "C" int dpo_muon_grad_sqnorm(dpo_muon_ctx *c, double *d_sumsq, void *stream)
+{
+    if (c == nullptr)
+        return mfail(nullptr, DPO_EINVAL, "ctx is NULL");
+    if (d_sumsq == nullptr || reinterpret_cast<uintptr_t>(d_sumsq) % alignof(double) != 0)
+        return mfail(c, DPO_EINVAL, "d_sumsq must be an 8-byte aligned device pointer");
+    if (c->total_pkts == 0)
+        return DPO_OK;
+    dpo::NormArgs na{};
+    na.table = c->d_norm_table;
+    na.pkt_begin = c->d_pkt_begin;
+    na.n_tensors = c->n;
+    na.total_pkts = c->total_pkts;
+    na.partials = c->d_norm_partials;
+    na.out = c->d_norm_scalars;
+    na.accum = d_sumsq;
+    const cudaError_t e = dpo::launch_norm(c->grad_dt == DPO_BF16, c->norm_grid, na,
+                                           static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess)
+        return mcuda(c, e, "norm launch");
+    return DPO_OK;
+}
+
+extern "C" int dpo_muon_set_clip_source(dpo_muon_ctx *c, const double *d_sumsq)
+{
+    if (c == nullptr)
+        return mfail(nullptr, DPO_EINVAL, "ctx is NULL");
+    if (d_sumsq != nullptr && reinterpret_cast<uintptr_t>(d_sumsq) % alignof(double) != 0)
+        return mfail(c, DPO_EINVAL, "d_sumsq must be 8-byte aligned");
+    if (d_sumsq != nullptr && !(c->hp.max_grad_norm > 0.0f))
+        return mfail(c, DPO_ESTATE, "a clip source needs max_grad_norm > 0");
+    c->clip_src = d_sumsq;
     return DPO_OK;
 }
 

@@ -32,7 +32,8 @@ DPO_STASH_COPY, DPO_STASH_PINGPONG = 0, 1
 
 EXPORTS = ("dpo_init", "dpo_stash", "dpo_step", "dpo_read_weights", "dpo_get_step",
            "dpo_set_step", "dpo_get_flags", "dpo_algorithmic_bytes", "dpo_launch_config",
-           "dpo_last_error", "dpo_destroy", "dpo_grad_norm_noalloc", "dpo_set_delay")
+           "dpo_last_error", "dpo_destroy", "dpo_grad_norm_noalloc", "dpo_set_delay",
+           "dpo_grad_sqnorm", "dpo_set_clip_source")
 
 DPO_NOALLOC_CHUNK_ELEMS = 1 << 20
 DPO_NOALLOC_MAX_CHUNKS = 16384
@@ -97,6 +98,8 @@ def load() -> ctypes.CDLL:
         "dpo_last_error": (ctypes.c_char_p, [P]),
         "dpo_destroy": (V, [P]),
         "dpo_grad_norm_noalloc": (I, [P, ctypes.c_int64, I, F, P, P, P]),
+        "dpo_grad_sqnorm": (I, [P, P, P]),
+        "dpo_set_clip_source": (I, [P, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -146,6 +149,44 @@ def dpo_set_delay(ctx, delay: int, stream=None) -> None:
 
 def dpo_step(ctx, lr: float, stream=None) -> None:
     _check(load().dpo_step(ctx, lr, _stream(stream)), ctx)
+
+
+def _dptr(t) -> Optional[int]:
+    return t if isinstance(t, int) or t is None else t.data_ptr()
+
+
+def dpo_grad_sqnorm(ctx, acc, stream=None) -> None:
+    """Add the context's sum of g^2 to ``acc`` (a float64 device scalar)."""
+    _check(load().dpo_grad_sqnorm(ctx, _dptr(acc), _stream(stream)), ctx)
+
+
+def dpo_set_clip_source(ctx, acc) -> None:
+    """Clip later steps from the sum of squares in ``acc`` (None: own norm)."""
+    _check(load().dpo_set_clip_source(ctx, _dptr(acc)), ctx)
+
+
+def allreduce_sqnorm(acc, group=None) -> None:
+    """Sum ``acc`` over the ranks of ``group`` (torch.distributed), each rank
+    holding one shard of the parameter set: the one exchange of a
+    partitioned step. Nothing to do without an initialised process group."""
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size(group) > 1:
+        dist.all_reduce(acc, op=dist.ReduceOp.SUM, group=group)
+
+
+def global_sqnorm(optimizers, acc, stream=None, group=None) -> None:
+    """||g||^2 over every parameter that ``optimizers`` (DelayedAdamW,
+    DelayedMuon) hold, into ``acc`` (a one-element float64 device tensor):
+    zeroed, each context's share added in list order on ``stream``, then
+    summed over ``group``'s ranks. Optimizers whose clip source is ``acc``
+    then clip from the norm over all of them (App. E.1)."""
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream(acc.device)
+    with torch.cuda.stream(s):
+        acc.zero_()
+        for o in optimizers:
+            o.grad_sqnorm(acc, s)
+        allreduce_sqnorm(acc, group)
 
 
 def dpo_read_weights(ctx, which: int, tensor: int):
@@ -276,6 +317,7 @@ class DelayedAdamW:
         self.wd_on = list(wd_on) if wd_on is not None else [True] * len(numels)
         self.sync = list(sync) if sync is not None else [False] * len(numels)
         self.ctx = None
+        self._clip_src = None
         self._init(init_mode, stream)
 
     def _init(self, init_mode, stream) -> None:
@@ -289,6 +331,8 @@ class DelayedAdamW:
         self.table = table
         self.ctx = dpo_init(table, self.param_dtype, self.stash_dtype, self.grad_dtype, self.hp,
                             init_mode, stream)
+        if self._clip_src is not None:
+            dpo_set_clip_source(self.ctx, self._clip_src)
 
     def use_host_io(self, grad: bool = True, param: bool = True, stream=None) -> None:
         """Move the grad and/or bf16 param arenas to pinned host memory (their
@@ -363,6 +407,16 @@ class DelayedAdamW:
 
     def step(self, lr: Optional[float] = None, stream=None) -> None:
         dpo_step(self.ctx, self.lr if lr is None else lr, stream)
+
+    def grad_sqnorm(self, acc, stream=None) -> None:
+        """Add this context's sum of g^2 to ``acc`` (dpo_grad_sqnorm)."""
+        dpo_grad_sqnorm(self.ctx, acc, stream)
+
+    def set_clip_source(self, acc=None) -> None:
+        """Clip from the sum of squares in ``acc`` (a float64 device tensor
+        kept alive here), or from this context's own norm when None."""
+        dpo_set_clip_source(self.ctx, acc)
+        self._clip_src = acc
 
     def restash(self, stream=None) -> None:
         dpo_stash(self.ctx, stream)

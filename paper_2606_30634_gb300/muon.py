@@ -37,7 +37,8 @@ EXPORTS = ("dpo_muon_init", "dpo_muon_step", "dpo_muon_set_delay", "dpo_muon_las
            "dpo_muon_get_status",
            "dpo_muon_get_step", "dpo_muon_set_step", "dpo_muon_flops",
            "dpo_muon_set_timing", "dpo_muon_get_gemm_time",
-           "dpo_muon_workspace_bytes", "dpo_muon_last_error", "dpo_muon_destroy")
+           "dpo_muon_workspace_bytes", "dpo_muon_last_error", "dpo_muon_destroy",
+           "dpo_muon_grad_sqnorm", "dpo_muon_set_clip_source")
 
 _typed = False
 
@@ -65,6 +66,8 @@ def lib() -> ctypes.CDLL:
             "dpo_muon_workspace_bytes": (I, [P, ctypes.POINTER(ctypes.c_int64)]),
             "dpo_muon_last_error": (ctypes.c_char_p, [P]),
             "dpo_muon_destroy": (None, [P]),
+            "dpo_muon_grad_sqnorm": (I, [P, P, P]),
+            "dpo_muon_set_clip_source": (I, [P, P]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -206,6 +209,18 @@ class DelayedMuon:
         _check(lib().dpo_muon_get_gemm_time(self.ctx, ctypes.byref(ms), ctypes.byref(n)),
                self.ctx)
         return float(ms.value), int(n.value)
+
+    def grad_sqnorm(self, acc, stream=None) -> None:
+        """Add the sum of G^2 over all matrices to ``acc`` (a float64 device
+        scalar; dpo_muon_grad_sqnorm)."""
+        _check(lib().dpo_muon_grad_sqnorm(self.ctx, acc.data_ptr(), _stream(stream)), self.ctx)
+
+    def set_clip_source(self, acc=None) -> None:
+        """Clip from the sum of squares in ``acc`` (kept alive here), or from
+        this context's own norm when None."""
+        _check(lib().dpo_muon_set_clip_source(self.ctx, acc.data_ptr() if acc is not None
+                                              else None), self.ctx)
+        self._clip_src = acc
 
     def workspace_bytes(self) -> int:
         v = ctypes.c_int64()

@@ -211,26 +211,36 @@ class Run:
                                  x0[o:o + n], self.c.init_sigma)
         return x0
 
-    def step(self, lr: Optional[float] = None):
-        """Draw gradient k+1 on both sides and take one step on each."""
+    def draw(self, k: int) -> np.ndarray:
+        """Gradient k on both sides: drawn into the GPU's grad arena, and
+        returned (tracked elements, fp64) for the oracle."""
+        c = self.c
+        for i, n in enumerate(c.numels):
+            if n:
+                synth.dev_normal(c.seed, synth.STREAM_GRAD, k, int(self.offs[i]),
+                                 self.gpu.grads(i), c.grad_sigma)
+        gdt = synth.BF16 if c.grad_dtype == dpo.DPO_BF16 else synth.F32
+        g = synth.host_normal_at(c.seed, synth.STREAM_GRAD, k, self.idx, c.grad_sigma, gdt)
+        g = synth.bf16_bits_to_f32(g) if gdt == synth.BF16 else g
+        return g.astype(np.float64)
+
+    def step(self, lr: Optional[float] = None, sq: Optional[float] = None, before=None):
+        """Draw gradient k+1 on both sides and take one step on each. ``sq``:
+        the squared norm the oracle clips from (default: its own gradient's);
+        ``before``: called after the draw, before the GPU step."""
         c = self.c
         k = self.k + 1
         if c.schedule and k in c.schedule:
             self.gpu.set_delay(c.schedule[k])
             self.ref.set_delay(c.schedule[k])
-        for i, n in enumerate(c.numels):
-            if n:
-                synth.dev_normal(c.seed, synth.STREAM_GRAD, k, int(self.offs[i]),
-                                 self.gpu.grads(i), c.grad_sigma)
+        g = self.draw(k)
+        if before is not None:
+            before(g)
         self.gpu.step(lr)
-        gdt = synth.BF16 if c.grad_dtype == dpo.DPO_BF16 else synth.F32
-        g = synth.host_normal_at(c.seed, synth.STREAM_GRAD, k, self.idx, c.grad_sigma, gdt)
-        g = synth.bf16_bits_to_f32(g) if gdt == synth.BF16 else g
-        sq = None
-        if c.max_grad_norm > 0 and self.sample is not None:
+        if sq is None and c.max_grad_norm > 0 and self.sample is not None:
             sq = self.full_sqnorm(k)
         lr32 = None if lr is None else float(np.float32(lr))
-        self.ref.step(g.astype(np.float64), tag=self.ref.read_weights("stale")[1], lr=lr32, sq=sq)
+        self.ref.step(g, tag=self.ref.read_weights("stale")[1], lr=lr32, sq=sq)
         self.k = k
 
     def full_sqnorm(self, k: int) -> float:

@@ -81,18 +81,27 @@ class Pair:
         self.sync = sync or [False] * len(shapes)
         self.k = 0
 
-    def step(self):
-        if self.k + 1 in self.schedule:
-            self.gpu.set_delay(self.schedule[self.k + 1])
-            self.ref.set_delay(self.schedule[self.k + 1])
-        self.k += 1
-        _, gs = inputs(self.shapes, self.seed, self.k + 1)
+    def draw(self, k: int):
+        """Gradient k (the seeded draw numbered k + 1) into the GPU's grad
+        arena; returned as fp64 matrices for the oracle."""
+        _, gs = inputs(self.shapes, self.seed, k + 1)
         for i, g in enumerate(gs):
             if g.size:
                 self.gpu.grads(i).copy_(torch.from_numpy(g.view(np.int16)).view(torch.bfloat16)
                                         .reshape(g.shape))
+        return [bf16_to_f64(g) for g in gs]
+
+    def step(self, sq=None, before=None):
+        """One call on both sides; ``sq`` and ``before`` as in Run.step."""
+        if self.k + 1 in self.schedule:
+            self.gpu.set_delay(self.schedule[self.k + 1])
+            self.ref.set_delay(self.schedule[self.k + 1])
+        self.k += 1
+        gs = self.draw(self.k)
+        if before is not None:
+            before(gs)
         self.gpu.step()
-        self.ref.step([bf16_to_f64(g) for g in gs])
+        self.ref.step(gs, sq=sq)
         torch.cuda.synchronize()
 
     def cat(self, arena):
