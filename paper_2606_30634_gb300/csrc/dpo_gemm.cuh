@@ -25,8 +25,8 @@
 // Per CTA a stage is 32 KiB for 4.2 MFLOP, a third less than one SM holding
 // a whole 128 x 256 operand pair, so six stages fit and keep the tensor pipe
 // fed across the L2 / DRAM round trip.
-// Symmetric products (Params::sym; X X^T and c A A + b A): only tiles that
-// reach the upper triangle (n0 + TN > m0) are computed; each of their
+// Symmetric products (Params::sym; X X^T and c A A + b A): only tiles on or
+// above the diagonal block (n0 >= m0) are computed; each of their
 // elements (i, j) is also stored at (j, i) when the tile holding (j, i) is
 // not computed. Every element is then written exactly once, by one thread,
 // and the result does not depend on scheduling.
@@ -228,23 +228,36 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
 }
 
 // Tile t of a launch: batch entry, row block and column block, columns
-// fastest (consecutive pairs share the A rows of a block row in L2).
+// fastest (consecutive pairs share the A rows of a block row in L2). A
+// symmetric product (sym, m_tiles == n_tiles) enumerates only the tiles on
+// or above the diagonal, row m holding m_tiles - m of them, so the pairs'
+// shares of its work differ by at most one tile.
 struct TileGrid {
-    int m_tiles, n_tiles, nb;
-    __device__ __forceinline__ int count() const { return m_tiles * n_tiles * nb; }
+    int m_tiles, n_tiles, nb, sym;
+    __host__ __device__ __forceinline__ int per_batch() const
+    {
+        return sym ? m_tiles * (m_tiles + 1) / 2 : m_tiles * n_tiles;
+    }
+    __host__ __device__ __forceinline__ int count() const { return per_batch() * nb; }
     __device__ __forceinline__ void at(int t, int &b, int &m0, int &n0) const
     {
-        n0 = (t % n_tiles) * TN;
-        t /= n_tiles;
-        m0 = (t % m_tiles) * TM;
-        b = t / m_tiles;
+        const int per = per_batch();
+        b = t / per;
+        int u = t - b * per;
+        if (sym) {
+            int m = 0;
+            while (u >= m_tiles - m) {   // u < per, so m stays below m_tiles
+                u -= m_tiles - m;
+                ++m;
+            }
+            m0 = m * TM;
+            n0 = (m + u) * TN;
+        } else {
+            n0 = (u % n_tiles) * TN;
+            m0 = (u / n_tiles) * TM;
+        }
     }
 };
-
-__device__ __forceinline__ bool tile_skipped(const Params &p, int m0, int n0)
-{
-    return p.sym && n0 + TN <= m0;   // strictly below the diagonal: mirrored
-}
 
 // Persistent: the CTA pairs (clusters of 2) take tiles c, c + pairs, ...
 // Within a pair, rank 0 (the leader) issues the MMAs; both ranks load their
@@ -316,8 +329,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             for (int t = pair; t < n_tiles && !*(volatile int *)&aborted; t += n_pairs) {
                 int b, m0, n0;
                 tg.at(t, b, m0, n0);
-                if (tile_skipped(p, m0, n0))
-                    continue;
                 const int ma = m0 + (int)rank * BM, nb_ = n0 + (int)rank * BH;
                 for (int kb = 0; kb < kb_n; ++kb, ++it) {
                     const int s = it % kStages;
@@ -354,8 +365,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             for (int t = pair; t < n_tiles && !*(volatile int *)&aborted; t += n_pairs) {
                 int b, m0, n0;
                 tg.at(t, b, m0, n0);
-                if (tile_skipped(p, m0, n0))
-                    continue;
                 const int a = lt & 1;
                 const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
                 if (!mbar_wait(acc_empty(a), aph ^ 1u)) {
@@ -400,8 +409,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         for (int t = pair; t < n_tiles; t += n_pairs) {
             int b, m0, n0;
             tg.at(t, b, m0, n0);
-            if (tile_skipped(p, m0, n0))
-                continue;
             const int a = lt & 1;
             const bool seen = mbar_wait(acc_full(a), (uint32_t)(lt >> 1) & 1u);
             if (!seen)

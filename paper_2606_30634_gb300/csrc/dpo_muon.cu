@@ -782,8 +782,10 @@ int launch_gemm(dpo_muon_ctx *c, const CUtensorMap &ta, const CUtensorMap &tb,
                 const dpo::gemm::Params &p, int64_t M, int64_t N, int64_t nb, bool b_mn,
                 cudaStream_t s)
 {
-    dpo::gemm::TileGrid tg{(int)(M / dpo::gemm::TM), (int)(N / dpo::gemm::TN), (int)nb};
-    const int64_t tiles = (int64_t)tg.m_tiles * tg.n_tiles * tg.nb;
+    dpo::gemm::TileGrid tg{(int)(M / dpo::gemm::TM), (int)(N / dpo::gemm::TN), (int)nb, p.sym};
+    if (p.sym && M != N)
+        return mfail(c, DPO_EINVAL, "symmetric product of a non-square shape");
+    const int64_t tiles = tg.count();
     // one CTA pair per co-resident cluster slot (the tile walk assumes every
     // pair runs at once)
     const int grid = 2 * (int)std::min<int64_t>(tiles, std::max(1, c->gemm_pairs));
