@@ -353,7 +353,7 @@ bool make_map(CUtensorMap *m, void *base, int64_t rows, int64_t cols, int64_t nb
         return false;
     const cuuint64_t dims[3] = {(cuuint64_t)cols, (cuuint64_t)rows, (cuuint64_t)nb};
     const cuuint64_t strides[2] = {(cuuint64_t)cols * 2, (cuuint64_t)(rows * cols) * 2};
-    const cuuint32_t box[3] = {(cuuint32_t)dpo::gemm::BK, (cuuint32_t)box_rows, 1};
+    const cuuint32_t box[3] = {(cuuint32_t)dpo::gemm::kBoxK, (cuuint32_t)box_rows, 1};
     const cuuint32_t es[3] = {1, 1, 1};
     return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, base, dims, strides, box, es,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
