@@ -21,8 +21,8 @@
 //               stage and each finished tile to both CTAs;
 //   warps 2-5   epilogue of this CTA's 128 rows: tcgen05.ld 32 lanes x 32
 //               columns at a time, scale, add the addend, round to bf16,
-//               store row-major (16-byte stores) and, when asked,
-//               transposed (each warp writes 64 contiguous bytes per column).
+//               stage the 32 x 32 chunk (and, when asked, its transpose) in
+//               shared memory and write it with a TMA store.
 // Per CTA a stage is 64 KiB for 8.4 MFLOP, a third less than one SM holding
 // a whole 128 x 256 operand pair, so three stages fit and keep the tensor
 // pipe fed across the L2 / DRAM round trip.
@@ -55,24 +55,28 @@ constexpr uint32_t kTmemCols = 256;                  // one accumulator (fp32, T
 constexpr int kABytes = BM * BK * 2;                 // 32 KiB
 constexpr int kBBytes = BH * BK * 2;                 // 32 KiB
 constexpr int kStageBytes = kABytes + kBBytes;       // 64 KiB per CTA
-// ring + 1024-byte alignment slack + 16 KiB kept free behind the ring
-constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 16384;
+// Epilogue staging behind the ring: per epilogue warp two buffers for its
+// 32 x 32 chunk of D and two for the chunk's transpose, 2 KiB each, in the
+// 64-byte-swizzled layout the TMA store reads.
+constexpr int kChunkBytes = 32 * 32 * 2;
+constexpr int kEpiBytes = 4 * 4 * kChunkBytes;              // 32 KiB
+// ring + 1024-byte alignment slack + staging
+constexpr int kSmemBytes = kStages * kStageBytes + 1024 + kEpiBytes;
 constexpr unsigned long long kWaitNs = 1000000000ull;  // 1 s per wait
 
 // Error codes OR-ed into Params::err (kErrWaitDone: an accumulator hand-off).
 constexpr unsigned int kErrWaitFull = 1u, kErrWaitEmpty = 2u, kErrWaitDone = 4u,
                        kErrDrain = 8u;
 
+// D is written through the store map tma_d (boxes of 32 x 32, 64-byte
+// swizzle) and, with trans, D^T through tma_dt.
 struct Params {
-    __nv_bfloat16 *d;             // M x N row-major output
-    int64_t ldd, d_bstride;       // elements
-    __nv_bfloat16 *dt;            // N x M row-major transposed output, or nullptr
-    int64_t ldt, dt_bstride;
     const __nv_bfloat16 *c;       // M x N addend, or nullptr
     int64_t ldc, c_bstride;
     float alpha, beta;
     int k_blocks;                 // K / BK
     int sym;                      // D is symmetric (M == N): see ns_gemm_kernel
+    int trans;                    // also write D^T (N x M) through tma_dt
     unsigned int *err;
 };
 
@@ -129,6 +133,24 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map
         " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar_cluster)
         : "memory");
+}
+
+// TMA store of a 32 x 32 bf16 box from this CTA's shared memory to global
+// coordinates (x = column, y = row, z = batch entry), in this thread's bulk
+// async-group.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap *map, uint32_t src, int x, int y,
+                                             int z)
+{
+    asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];"
+                 ::"l"(reinterpret_cast<uint64_t>(map)), "r"(src), "r"(x), "r"(y), "r"(z)
+                 : "memory");
+}
+
+// Byte offset of 16-byte granule g of row r in a tile of 64-byte rows with
+// the 64-byte swizzle (granule index XOR bits 1-2 of the row).
+__device__ __forceinline__ uint32_t swz64(int r, int g)
+{
+    return (uint32_t)(r * 64 + ((g ^ ((r >> 1) & 3)) << 4));
 }
 
 __device__ __forceinline__ uint32_t cluster_rank()
@@ -277,7 +299,9 @@ struct TileGrid {
 template <bool BMN>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     ns_gemm_kernel(const __grid_constant__ CUtensorMap tma_a,
-                   const __grid_constant__ CUtensorMap tma_b, const Params p, const TileGrid tg)
+                   const __grid_constant__ CUtensorMap tma_b,
+                   const __grid_constant__ CUtensorMap tma_d,
+                   const __grid_constant__ CUtensorMap tma_dt, const Params p, const TileGrid tg)
 {
     extern __shared__ uint8_t smem_raw[];
     __shared__ uint64_t bars[2 * kStages + 4];
@@ -414,9 +438,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
     } else {
         // Epilogue: warp w reads TMEM lanes 32 (w % 4) .. +31 = this CTA's
-        // tile rows m0 + BM rank + 32 (w % 4) + lane.
+        // tile rows m0 + BM rank + 32 (w % 4) + lane. Each 32 x 32 chunk is
+        // staged in shared memory (and its transpose, for a mirrored or a
+        // transposed output) and written by one TMA store per box from lane
+        // 0; direct stores from 32 rows at a time cost the MMAs a fifth of
+        // their rate on GB300. Two buffers per kind alternate, so lane 0
+        // waits for the group of two chunks back before they are rewritten.
         const int q = warp & 3;
-        int lt = 0;
+        const uint32_t wbuf = ring + (uint32_t)(kStages * kStageBytes + q * 4 * kChunkBytes);
+        int lt = 0, staged = 0;
         for (int t = pair; t < n_tiles; t += n_pairs) {
             int b, m0, n0;
             tg.at(t, b, m0, n0);
@@ -428,8 +458,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             // tcgen05.ld is warp-collective: the whole warp goes on, or none of it.
             if (!__all_sync(0xFFFFFFFFu, seen && !*(volatile int *)&aborted))
                 break;
-            const int64_t row = m0 + (int)rank * BM + q * 32 + lane;
-            __nv_bfloat16 *drow = p.d + (int64_t)b * p.d_bstride + row * p.ldd + n0;
+            const int row0 = m0 + (int)rank * BM + q * 32;
+            const int64_t row = row0 + lane;
             const __nv_bfloat16 *crow =
                 p.c != nullptr ? p.c + (int64_t)b * p.c_bstride + row * p.ldc + n0 : nullptr;
             const uint32_t acc = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(a * (int)kTmemCols);
@@ -454,33 +484,47 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         }
                     }
                 }
-#pragma unroll
-                for (int j8 = 0; j8 < 4; ++j8) {
-                    uint4 o;
-                    o.x = pack_bf16(v[j8 * 8 + 0], v[j8 * 8 + 1]);
-                    o.y = pack_bf16(v[j8 * 8 + 2], v[j8 * 8 + 3]);
-                    o.z = pack_bf16(v[j8 * 8 + 4], v[j8 * 8 + 5]);
-                    o.w = pack_bf16(v[j8 * 8 + 6], v[j8 * 8 + 7]);
-                    *reinterpret_cast<uint4 *>(drow + ch * 32 + j8 * 8) = o;
-                }
-                if (p.dt != nullptr) {
-                    __nv_bfloat16 *dcol = p.dt + (int64_t)b * p.dt_bstride +
-                                          (int64_t)(n0 + ch * 32) * p.ldt + row;
-#pragma unroll
-                    for (int j = 0; j < 32; ++j)
-                        dcol[(int64_t)j * p.ldt] = __float2bfloat16_rn(v[j]);
-                }
+                const int col0 = n0 + ch * 32;
                 // Mirror of a symmetric product: (col, row) lies in the tile
-                // (col / TM, row / TN), skipped when row / TN < col / TM
+                // (col / TM, row / TN), not computed when row / TN < col / TM
                 // (TM == TN). Uniform over the warp (its rows share row / TN)
-                // and the 32-column chunk (its columns share col / TM).
-                if (p.sym && row / TN < (int64_t)((n0 + ch * 32) / TM)) {
-                    __nv_bfloat16 *dcol = p.d + (int64_t)b * p.d_bstride +
-                                          (int64_t)(n0 + ch * 32) * p.ldd + row;
+                // and the chunk (its columns share col / TM).
+                const bool mirror = p.sym && row0 / TN < col0 / TM;
+                const bool trans = mirror || p.trans != 0;
+                const uint32_t rb = wbuf + (uint32_t)((staged & 1) * kChunkBytes);
+                const uint32_t tb = rb + (uint32_t)(2 * kChunkBytes);
+                if (lane == 0)   // the buffers' previous group has been read
+                    asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+                __syncwarp();
 #pragma unroll
-                    for (int j = 0; j < 32; ++j)
-                        dcol[(int64_t)j * p.ldd] = __float2bfloat16_rn(v[j]);
+                for (int g = 0; g < 4; ++g) {
+                    const uint32_t w0 = pack_bf16(v[g * 8 + 0], v[g * 8 + 1]);
+                    const uint32_t w1 = pack_bf16(v[g * 8 + 2], v[g * 8 + 3]);
+                    const uint32_t w2 = pack_bf16(v[g * 8 + 4], v[g * 8 + 5]);
+                    const uint32_t w3 = pack_bf16(v[g * 8 + 6], v[g * 8 + 7]);
+                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(rb + swz64(lane, g)),
+                                 "r"(w0), "r"(w1), "r"(w2), "r"(w3)
+                                 : "memory");
                 }
+                if (trans) {   // element (row, col0 + j) at row j, column lane of the transpose
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const __nv_bfloat16 h = __float2bfloat16_rn(v[j]);
+                        asm volatile("st.shared.b16 [%0], %1;" ::"r"(tb + swz64(j, lane >> 3) +
+                                                                      (uint32_t)((lane & 7) * 2)),
+                                     "h"(*reinterpret_cast<const uint16_t *>(&h))
+                                     : "memory");
+                    }
+                }
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                __syncwarp();
+                if (lane == 0) {
+                    tma_store_3d(&tma_d, rb, col0, row0, b);
+                    if (trans)
+                        tma_store_3d(mirror ? &tma_d : &tma_dt, tb, row0, col0, b);
+                    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+                }
+                ++staged;
             }
             // this warp's rows of the accumulator are read: release them to
             // the leader's MMA lane
@@ -490,6 +534,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 mbar_arrive_cluster(map_to_rank(acc_empty(a), 0));
             ++lt;
         }
+        if (lane == 0)   // every store has been written before the CTA ends
+            asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+        __syncwarp();
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     }
     __syncthreads();

@@ -361,6 +361,22 @@ bool make_map(CUtensorMap *m, void *base, int64_t rows, int64_t cols, int64_t nb
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The same over rows x cols with 32 x 32 boxes and the 64-byte swizzle: the
+// epilogue's TMA stores.
+bool make_store_map(CUtensorMap *m, void *base, int64_t rows, int64_t cols, int64_t nb)
+{
+    EncodeTiled enc = encode_fn();
+    if (enc == nullptr)
+        return false;
+    const cuuint64_t dims[3] = {(cuuint64_t)cols, (cuuint64_t)rows, (cuuint64_t)nb};
+    const cuuint64_t strides[2] = {(cuuint64_t)cols * 2, (cuuint64_t)(rows * cols) * 2};
+    const cuuint32_t box[3] = {32, 32, 1};
+    const cuuint32_t es[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, base, dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
+               CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 int64_t pad_up(int64_t v) { return (v + kPad - 1) / kPad * kPad; }
 
 struct Group {
@@ -373,6 +389,7 @@ struct Group {
     __nv_bfloat16 *x[2] = {nullptr, nullptr}, *xt = nullptr, *a = nullptr, *b = nullptr;
     CUtensorMap x128[2], a128, b128;   // 128-row K-major boxes: one CTA's half of a pair tile
     CUtensorMap x_mn[2];               // 64 x 64 boxes of X read MN-major (B of B X)
+    CUtensorMap st_x[2], st_xt, st_a, st_b;   // 32 x 32 store boxes of X, X^T, A, B
 };
 
 }  // namespace
@@ -690,7 +707,12 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
                         make_map(&g.a128, g.a, g.R, g.R, nb, dpo::gemm::BM) &&
                         make_map(&g.b128, g.b, g.R, g.R, nb, dpo::gemm::BM) &&
                         make_map(&g.x_mn[0], g.x[0], g.R, g.W, nb, 64) &&
-                        make_map(&g.x_mn[1], g.x[1], g.R, g.W, nb, 64);
+                        make_map(&g.x_mn[1], g.x[1], g.R, g.W, nb, 64) &&
+                        make_store_map(&g.st_x[0], g.x[0], g.R, g.W, nb) &&
+                        make_store_map(&g.st_x[1], g.x[1], g.R, g.W, nb) &&
+                        make_store_map(&g.st_xt, g.xt, g.W, g.R, nb) &&
+                        make_store_map(&g.st_a, g.a, g.R, g.R, nb) &&
+                        make_store_map(&g.st_b, g.b, g.R, g.R, nb);
         if (!ok) {
             free_ctx(c);
             return mfail(nullptr, DPO_ECUDA, "tensor map encoding failed");
@@ -779,8 +801,8 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
 namespace {
 
 int launch_gemm(dpo_muon_ctx *c, const CUtensorMap &ta, const CUtensorMap &tb,
-                const dpo::gemm::Params &p, int64_t M, int64_t N, int64_t nb, bool b_mn,
-                cudaStream_t s)
+                const CUtensorMap &td, const CUtensorMap &tdt, const dpo::gemm::Params &p,
+                int64_t M, int64_t N, int64_t nb, bool b_mn, cudaStream_t s)
 {
     dpo::gemm::TileGrid tg{(int)(M / dpo::gemm::TM), (int)(N / dpo::gemm::TN), (int)nb, p.sym};
     if (p.sym && M != N)
@@ -791,10 +813,10 @@ int launch_gemm(dpo_muon_ctx *c, const CUtensorMap &ta, const CUtensorMap &tb,
     const int grid = 2 * (int)std::min<int64_t>(tiles, std::max(1, c->gemm_pairs));
     if (b_mn)
         dpo::gemm::ns_gemm_kernel<true><<<grid, dpo::gemm::kThreads, dpo::gemm::kSmemBytes, s>>>(
-            ta, tb, p, tg);
+            ta, tb, td, tdt, p, tg);
     else
         dpo::gemm::ns_gemm_kernel<false><<<grid, dpo::gemm::kThreads, dpo::gemm::kSmemBytes, s>>>(
-            ta, tb, p, tg);
+            ta, tb, td, tdt, p, tg);
     const cudaError_t e = cudaGetLastError();
     return e == cudaSuccess ? DPO_OK : mcuda(c, e, "Newton-Schulz GEMM launch");
 }
@@ -883,41 +905,35 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
             dpo::gemm::Params p{};
             p.err = c->d_err;
             // A = X X^T
-            p.d = g.a;
-            p.ldd = g.R;
-            p.d_bstride = g.R * g.R;
             p.alpha = 1.0f;
             p.k_blocks = (int)(g.W / dpo::gemm::BK);
             p.sym = 1;
-            int rc = launch_gemm(c, g.x128[cur], g.x128[cur], p, g.R, g.R, nb, false, s);
+            int rc = launch_gemm(c, g.x128[cur], g.x128[cur], g.st_a, g.st_a, p, g.R, g.R, nb,
+                                 false, s);
             if (rc != DPO_OK)
                 return rc;
             // B = c A A + b A
-            p.d = g.b;
             p.c = g.a;
             p.ldc = g.R;
             p.c_bstride = g.R * g.R;
             p.alpha = c->hp.ns_c;
             p.beta = c->hp.ns_b;
             p.k_blocks = (int)(g.R / dpo::gemm::BK);
-            if ((rc = launch_gemm(c, g.a128, g.a128, p, g.R, g.R, nb, false, s)) != DPO_OK)
+            if ((rc = launch_gemm(c, g.a128, g.a128, g.st_b, g.st_b, p, g.R, g.R, nb, false, s)) !=
+                DPO_OK)
                 return rc;
             // X <- B X + a X (X read MN-major in place of X^T), and at the
             // last step X^T for the tall matrices' output
             p.sym = 0;
-            p.d = g.x[nxt];
-            p.ldd = g.W;
-            p.d_bstride = g.R * g.W;
-            p.dt = last && g.has_tall ? g.xt : nullptr;
-            p.ldt = g.R;
-            p.dt_bstride = g.W * g.R;
+            p.trans = last && g.has_tall ? 1 : 0;
             p.c = g.x[cur];
             p.ldc = g.W;
             p.c_bstride = g.R * g.W;
             p.alpha = 1.0f;
             p.beta = c->hp.ns_a;
             p.k_blocks = (int)(g.R / dpo::gemm::BK);
-            if ((rc = launch_gemm(c, g.b128, g.x_mn[cur], p, g.R, g.W, nb, true, s)) != DPO_OK)
+            if ((rc = launch_gemm(c, g.b128, g.x_mn[cur], g.st_x[nxt], g.st_xt, p, g.R, g.W, nb,
+                                  true, s)) != DPO_OK)
                 return rc;
         }
         if (ev_end != nullptr && (e = cudaEventRecord(ev_end, s)) != cudaSuccess)
