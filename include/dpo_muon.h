@@ -148,6 +148,22 @@ int dpo_muon_get_status(dpo_muon_ctx *ctx, uint32_t *bits);
 int dpo_muon_grad_sqnorm(dpo_muon_ctx *ctx, double *d_sumsq, void *cuda_stream);
 int dpo_muon_set_clip_source(dpo_muon_ctx *ctx, const double *d_sumsq);
 
+/*
+ * Clear the error bits that dpo_muon_get_status reports (enqueued on
+ * cuda_stream). Returns DPO_OK, DPO_EINVAL or DPO_ECUDA.
+ */
+int dpo_muon_clear_status(dpo_muon_ctx *ctx, void *cuda_stream);
+
+/*
+ * Test hook for the failure path: in each of the next `launches` Newton-Schulz
+ * GEMM launches, the MMA lane's first accumulator wait targets a phase that
+ * no arrival completes. The wait gives up after its one-second limit, every
+ * role of the kernel leaves through its own bounded wait, and the launch ends
+ * with error bits set (its output is not computed); later launches run
+ * normally. Returns DPO_OK or DPO_EINVAL (launches < 0).
+ */
+int dpo_muon_test_stall(dpo_muon_ctx *ctx, int launches);
+
 /* Calls consumed so far (k), and restore after loading a checkpoint. */
 int dpo_muon_get_step(const dpo_muon_ctx *ctx, int64_t *k);
 int dpo_muon_set_step(dpo_muon_ctx *ctx, int64_t k);

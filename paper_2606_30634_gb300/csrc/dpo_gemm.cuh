@@ -77,6 +77,8 @@ struct Params {
     int k_blocks;                 // K / BK
     int sym;                      // D is symmetric (M == N): see ns_gemm_kernel
     int trans;                    // also write D^T (N x M) through tma_dt
+    int stall;                    // test hook: the MMA lane's first accumulator wait
+                                  // targets a phase no arrival completes, so it gives up
     unsigned int *err;
 };
 
@@ -400,7 +402,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 tg.at(t, b, m0, n0);
                 const int a = lt & 1;
                 const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
-                if (!mbar_wait(acc_empty(a), aph ^ 1u)) {
+                if (!mbar_wait(acc_empty(a), p.stall && lt == 0 ? aph : aph ^ 1u)) {
                     atomicOr(p.err, kErrWaitDone);
                     aborted = 1;
                     break;
@@ -432,8 +434,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 }
                 mma_commit_pair(acc_full(a));   // when this tile's MMAs have completed
                 ++lt;
-                if (!ok)
+                if (!ok) {
+                    // the MMAs issued for this tile finish before the pair
+                    // leaves and its TMEM is released
+                    if (!mbar_wait(acc_full(a), aph))
+                        atomicOr(p.err, kErrDrain);
                     break;
+                }
             }
         }
     } else {

@@ -406,6 +406,7 @@ struct dpo_muon_ctx {
     int64_t phase_k0 = 0;     // k when the current delayed phase began
     int sms = 0;
     int gemm_pairs = 0;   // clusters of 2 the GEMM kernel keeps resident at once
+    int stall_launches = 0;   // dpo_muon_test_stall: GEMM launches left to stall
     std::vector<dpo_matrix> mats;
     std::vector<DevMat> host_mats;
     std::vector<Group> groups;
@@ -904,10 +905,17 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
             const int cur = it % 2, nxt = cur ^ 1;
             dpo::gemm::Params p{};
             p.err = c->d_err;
+            auto stall_next = [c]() {
+                if (c->stall_launches <= 0)
+                    return 0;
+                --c->stall_launches;
+                return 1;
+            };
             // A = X X^T
             p.alpha = 1.0f;
             p.k_blocks = (int)(g.W / dpo::gemm::BK);
             p.sym = 1;
+            p.stall = stall_next();
             int rc = launch_gemm(c, g.x128[cur], g.x128[cur], g.st_a, g.st_a, p, g.R, g.R, nb,
                                  false, s);
             if (rc != DPO_OK)
@@ -919,6 +927,7 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
             p.alpha = c->hp.ns_c;
             p.beta = c->hp.ns_b;
             p.k_blocks = (int)(g.R / dpo::gemm::BK);
+            p.stall = stall_next();
             if ((rc = launch_gemm(c, g.a128, g.a128, g.st_b, g.st_b, p, g.R, g.R, nb, false, s)) !=
                 DPO_OK)
                 return rc;
@@ -932,6 +941,7 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
             p.alpha = 1.0f;
             p.beta = c->hp.ns_a;
             p.k_blocks = (int)(g.R / dpo::gemm::BK);
+            p.stall = stall_next();
             if ((rc = launch_gemm(c, g.b128, g.x_mn[cur], g.st_x[nxt], g.st_xt, p, g.R, g.W, nb,
                                   true, s)) != DPO_OK)
                 return rc;
@@ -1019,6 +1029,25 @@ extern "C" int dpo_muon_get_status(dpo_muon_ctx *c, uint32_t *bits)
     if (e != cudaSuccess)
         return mcuda(c, e, "status read");
     *bits = v;
+    return DPO_OK;
+}
+
+extern "C" int dpo_muon_clear_status(dpo_muon_ctx *c, void *stream)
+{
+    if (c == nullptr)
+        return DPO_EINVAL;
+    const cudaError_t e = cudaMemsetAsync(c->d_err, 0, sizeof(unsigned int),
+                                          static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? DPO_OK : mcuda(c, e, "status reset");
+}
+
+extern "C" int dpo_muon_test_stall(dpo_muon_ctx *c, int launches)
+{
+    if (c == nullptr)
+        return DPO_EINVAL;
+    if (launches < 0)
+        return mfail(c, DPO_EINVAL, "launches must be >= 0");
+    c->stall_launches = launches;
     return DPO_OK;
 }
 

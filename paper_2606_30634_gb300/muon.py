@@ -38,7 +38,8 @@ EXPORTS = ("dpo_muon_init", "dpo_muon_step", "dpo_muon_set_delay", "dpo_muon_las
            "dpo_muon_get_step", "dpo_muon_set_step", "dpo_muon_flops",
            "dpo_muon_set_timing", "dpo_muon_get_gemm_time",
            "dpo_muon_workspace_bytes", "dpo_muon_last_error", "dpo_muon_destroy",
-           "dpo_muon_grad_sqnorm", "dpo_muon_set_clip_source")
+           "dpo_muon_grad_sqnorm", "dpo_muon_set_clip_source", "dpo_muon_clear_status",
+           "dpo_muon_test_stall")
 
 _typed = False
 
@@ -68,6 +69,8 @@ def lib() -> ctypes.CDLL:
             "dpo_muon_destroy": (None, [P]),
             "dpo_muon_grad_sqnorm": (I, [P, P, P]),
             "dpo_muon_set_clip_source": (I, [P, P]),
+            "dpo_muon_clear_status": (I, [P, P]),
+            "dpo_muon_test_stall": (I, [P, I]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -184,6 +187,13 @@ class DelayedMuon:
         v = ctypes.c_uint32()
         _check(lib().dpo_muon_get_status(self.ctx, ctypes.byref(v)), self.ctx)
         return int(v.value)
+
+    def clear_status(self, stream=None) -> None:
+        _check(lib().dpo_muon_clear_status(self.ctx, _stream(stream)), self.ctx)
+
+    def test_stall(self, launches: int) -> None:
+        """Make the next ``launches`` GEMM launches give up a wait (include/dpo_muon.h)."""
+        _check(lib().dpo_muon_test_stall(self.ctx, launches), self.ctx)
 
     @property
     def k(self) -> int:

@@ -309,3 +309,46 @@ def test_muon_full_size_shapes(cuda_device):
             assert err <= 2e-2
     finally:
         gpu.close()
+
+
+def test_gemm_wait_timeout_reports_status(cuda_device):
+    """The failure path of the tensor-core pipeline, without a GPU fault: one
+    GEMM launch whose MMA lane waits on a phase nothing completes gives up
+    after its one-second limit, every role leaves through its own bounded
+    wait, the step returns and the status says which waits gave up
+    (4: accumulator hand-off, 2: free stage; not 1 or 8, since every TMA
+    stage issued has landed). After clearing, the context and the GPU work
+    on: the next call reports nothing, and a fresh context holds parity."""
+    import time
+    shapes = [(256, 512), (512, 768)]
+    m = muon.DelayedMuon(shapes, ns_steps=1, device=cuda_device)
+    try:
+        off = 0
+        for i, (r, c) in enumerate(shapes):
+            synth.dev_normal(0x57A1, synth.STREAM_GRAD, 1, off, m.grads(i).view(-1), 1e-3)
+            off += r * c
+        m.step()
+        torch.cuda.synchronize()
+        assert m.status() == 0
+        m.test_stall(1)
+        t0 = time.monotonic()
+        m.step()
+        torch.cuda.synchronize()
+        took = time.monotonic() - t0
+        bits = m.status()
+        assert bits & 4 and bits & ~(2 | 4) == 0, bits
+        assert 0.9 < took < 10.0, took
+        m.clear_status()
+        m.step()
+        torch.cuda.synchronize()
+        assert m.status() == 0
+    finally:
+        m.close()
+    p = Pair([(256, 512), (300, 700)], cuda_device, ns_steps=1)
+    try:
+        p.step()
+        got, ref = p.o_pairs()
+        g, r = _flat(got), _flat(ref)
+        assert np.linalg.norm(g - r) / np.linalg.norm(r) <= NS_BARS[1][0]
+    finally:
+        p.close()
