@@ -349,6 +349,16 @@ int dpo_grad_norm_noalloc(const void *grad, int64_t numel, dpo_dtype grad_dtype,
 
 /* Message of the last failing call on ctx (NULL ctx: last dpo_init failure of
  * the calling thread). Never NULL; owned by the library. */
+/*
+ * Test hook for the allocation-failure paths, process-wide: of the library's
+ * next device allocations (dpo_init makes one, dpo_muon_init one or two: its
+ * table, then its workspace), let `after` succeed and make the following
+ * `count` fail as if the device were out of memory (the call then returns
+ * DPO_ENOMEM and frees what it had allocated). count = 0 turns the hook off.
+ * Returns DPO_OK or DPO_EINVAL (a negative argument).
+ */
+int dpo_test_fail_allocs(int after, int count);
+
 const char *dpo_last_error(const dpo_ctx *ctx);
 
 /* Free the context and its device scratch (after the work enqueued on it has

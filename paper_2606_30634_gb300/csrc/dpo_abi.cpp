@@ -16,6 +16,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <mutex>
 #include <new>
 #include <string>
 #include <vector>
@@ -54,6 +55,10 @@ struct dpo_ctx {
 namespace {
 
 thread_local std::string g_init_err;
+
+// dpo_test_fail_allocs: allocations to let through, then allocations to fail.
+std::mutex g_alloc_mu;
+int g_alloc_after = 0, g_alloc_fail = 0;
 
 int fail(dpo_ctx *c, int code, const char *fmt, ...)
 {
@@ -417,7 +422,7 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
     const size_t off_part = align_up(off_pkt + sizeof(int64_t) * (n_tensors + 1), 256);
     const size_t off_scal = align_up(off_part + sizeof(double) * c->norm_grid, 256);
     const size_t bytes = off_scal + sizeof(dpo::NormScalars);
-    e = cudaMalloc(&c->dev_block, bytes);
+    e = dpo::device_alloc(&c->dev_block, bytes);
     if (e != cudaSuccess) {
         cudaGetLastError();
         fail(nullptr, DPO_ENOMEM, "cudaMalloc of %zu bytes: %s", bytes, cudaGetErrorString(e));
@@ -598,6 +603,33 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
     }
     c->mu_prod *= nadam_mu(c->hp, k);
     c->k = k;
+    return DPO_OK;
+}
+
+cudaError_t dpo::device_alloc(void **p, size_t bytes)
+{
+    {
+        std::lock_guard<std::mutex> lock(g_alloc_mu);
+        if (g_alloc_fail > 0) {
+            if (g_alloc_after > 0) {
+                --g_alloc_after;
+            } else {
+                --g_alloc_fail;
+                *p = nullptr;
+                return cudaErrorMemoryAllocation;
+            }
+        }
+    }
+    return cudaMalloc(p, bytes);
+}
+
+extern "C" int dpo_test_fail_allocs(int after, int count)
+{
+    if (after < 0 || count < 0)
+        return DPO_EINVAL;
+    std::lock_guard<std::mutex> lock(g_alloc_mu);
+    g_alloc_after = after;
+    g_alloc_fail = count;
     return DPO_OK;
 }
 

@@ -123,6 +123,10 @@ StepFn pick_step_lion(bool param_bf16, StashKind stash, bool grad_bf16, Correcti
 StepFn pick_step_adan(bool param_bf16, StashKind stash, bool grad_bf16, Correction corr,
                       bool dc, bool pp);
 
+// Device allocation of the library's own blocks (dpo_init, dpo_muon_init),
+// through the hook of dpo_test_fail_allocs (dpo_abi.cpp).
+cudaError_t device_alloc(void **p, size_t bytes);
+
 // Launchers (dpo_kernels.cu). Each returns the launch's cudaError_t.
 cudaError_t launch_step(Optimizer opt, bool param_bf16, StashKind stash, bool grad_bf16,
                         Correction corr, bool dc, bool pp, int grid, const StepArgs &a,

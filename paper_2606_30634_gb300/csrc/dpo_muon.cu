@@ -644,13 +644,13 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
     const int64_t o_nsc = off;
     off += al(sizeof(dpo::NormScalars));
 
-    cudaError_t e = cudaMalloc(&c->dev_block, (size_t)off);
+    cudaError_t e = dpo::device_alloc(&c->dev_block, (size_t)off);
     if (e != cudaSuccess) {
         free_ctx(c);
         return mfail(nullptr, DPO_ENOMEM, "device table allocation failed");
     }
     if (ws > 0) {
-        e = cudaMalloc(&c->ws, (size_t)ws);
+        e = dpo::device_alloc(&c->ws, (size_t)ws);
         if (e != cudaSuccess) {
             free_ctx(c);
             return mfail(nullptr, DPO_ENOMEM, "Newton-Schulz workspace (%lld bytes) allocation failed",

@@ -33,7 +33,7 @@ DPO_STASH_COPY, DPO_STASH_PINGPONG = 0, 1
 EXPORTS = ("dpo_init", "dpo_stash", "dpo_step", "dpo_read_weights", "dpo_get_step",
            "dpo_set_step", "dpo_get_flags", "dpo_algorithmic_bytes", "dpo_launch_config",
            "dpo_last_error", "dpo_destroy", "dpo_grad_norm_noalloc", "dpo_set_delay",
-           "dpo_grad_sqnorm", "dpo_set_clip_source")
+           "dpo_grad_sqnorm", "dpo_set_clip_source", "dpo_test_fail_allocs")
 
 DPO_NOALLOC_CHUNK_ELEMS = 1 << 20
 DPO_NOALLOC_MAX_CHUNKS = 16384
@@ -100,6 +100,7 @@ def load() -> ctypes.CDLL:
         "dpo_grad_norm_noalloc": (I, [P, ctypes.c_int64, I, F, P, P, P]),
         "dpo_grad_sqnorm": (I, [P, P, P]),
         "dpo_set_clip_source": (I, [P, P]),
+        "dpo_test_fail_allocs": (I, [I, I]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -163,6 +164,12 @@ def dpo_grad_sqnorm(ctx, acc, stream=None) -> None:
 def dpo_set_clip_source(ctx, acc) -> None:
     """Clip later steps from the sum of squares in ``acc`` (None: own norm)."""
     _check(load().dpo_set_clip_source(ctx, _dptr(acc)), ctx)
+
+
+def dpo_test_fail_allocs(after: int, count: int) -> None:
+    """Make the library's device allocations after the next ``after`` fail,
+    ``count`` of them (include/dpo.h); (0, 0) turns the hook off."""
+    _check(load().dpo_test_fail_allocs(after, count), None)
 
 
 def allreduce_sqnorm(acc, group=None) -> None:
