@@ -38,15 +38,16 @@ SHAPES = [(256, 512), (512, 256), (300, 700), (64, 96), (1, 7), (0, 5), (768, 23
 NS_BARS = {1: (2e-4, 2e-3), 2: (5e-4, 1e-2)}
 
 
-def inputs(shapes, seed, k):
+def inputs(shapes, seed, k, gdt=None):
     """x_0 ~ N(0, 0.02^2) (fp32) and the k-th gradient ~ N(0, 1e-3^2) (bf16
-    bits), per matrix, from the seeded generator."""
+    bits, or fp32 with gdt = synth.F32), per matrix, from the seeded
+    generator."""
     xs, gs, off = [], [], 0
     for r, c in shapes:
         n = r * c
         xs.append(synth.host_normal(seed, synth.STREAM_INIT, 0, off, n, 0.02).reshape(r, c))
         gs.append(synth.host_normal(seed, synth.STREAM_GRAD, k, off, n, 1e-3,
-                                    synth.BF16).reshape(r, c))
+                                    synth.BF16 if gdt is None else gdt).reshape(r, c))
         off += n
     return xs, gs
 
@@ -60,11 +61,12 @@ class Pair:
 
     def __init__(self, shapes, device, seed=0x3A0, ns_steps=5, ef=True, delay=1, sdt=B,
                  lr=2e-3, momentum=0.95, wd=0.1, max_grad_norm=0.0, rms_scale=0.2, sync=None,
-                 schedule=None, correction=0):
+                 schedule=None, correction=0, gdt=B):
         self.shapes, self.seed, self.lr = shapes, seed, lr
         self.schedule = schedule or {}
         xs, _ = inputs(shapes, seed, 1)
-        self.gpu = muon.DelayedMuon(shapes, stash_dtype=sdt, grad_dtype=B, lr=lr,
+        self.gdt = gdt
+        self.gpu = muon.DelayedMuon(shapes, stash_dtype=sdt, grad_dtype=gdt, lr=lr,
                                     momentum=momentum, weight_decay=wd, ef=ef,
                                     max_grad_norm=max_grad_norm, rms_scale=rms_scale,
                                     ns_steps=ns_steps, delay=delay, device=device,
@@ -84,6 +86,12 @@ class Pair:
     def draw(self, k: int):
         """Gradient k (the seeded draw numbered k + 1) into the GPU's grad
         arena; returned as fp64 matrices for the oracle."""
+        if self.gdt == F:
+            _, gs = inputs(self.shapes, self.seed, k + 1, synth.F32)
+            for i, g in enumerate(gs):
+                if g.size:
+                    self.gpu.grads(i).copy_(torch.from_numpy(g))
+            return [g.astype(np.float64) for g in gs]
         _, gs = inputs(self.shapes, self.seed, k + 1)
         for i, g in enumerate(gs):
             if g.size:
@@ -169,9 +177,10 @@ def close_with_flips(gpu, ref, tol, flip, max_frac):
     assert np.all(d[bad] <= flip + tol * den[bad]), f"max miss {d[bad].max():.3e} > {flip:.3e}"
 
 
-@pytest.mark.parametrize("steps,sdt,ef,delay", [(0, B, True, 1), (1, F, True, 1), (1, B, False, 1),
-                                                (0, B, False, 0)])
-def test_muon_step_parity(cuda_device, steps, sdt, ef, delay):
+@pytest.mark.parametrize("steps,sdt,ef,delay,gdt", [(0, B, True, 1, B), (1, F, True, 1, B),
+                                                    (1, B, False, 1, B), (0, B, False, 0, B),
+                                                    (1, F, True, 1, F)])
+def test_muon_step_parity(cuda_device, steps, sdt, ef, delay, gdt):
     """Four calls of Alg. 2 (EF from the second), every buffer checked after
     each. The momentum does not depend on O: one-step bar, then the run bar
     (the EMA rounds twice where the oracle rounds once). The weights, stash,
@@ -179,7 +188,7 @@ def test_muon_step_parity(cuda_device, steps, sdt, ef, delay):
     bars except where a bf16 rounding of O flipped (see the module note):
     such a flip moves U by at most lr r ulp(O) <= lr r 2^-7 (|O| < 2), and
     the weights by that much per call so far."""
-    p = Pair(SHAPES, cuda_device, ns_steps=steps, ef=ef, delay=delay, sdt=sdt)
+    p = Pair(SHAPES, cuda_device, ns_steps=steps, ef=ef, delay=delay, sdt=sdt, gdt=gdt)
     r_max = 0.2 * np.sqrt(max(max(sh) for sh in SHAPES))
     du = p.lr * r_max * 2.0 ** -7
     try:
