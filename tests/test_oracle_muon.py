@@ -292,3 +292,40 @@ def test_muon_sapipe_same_state(lib):
     for k in range(2, len(grads)):
         np.testing.assert_allclose(stash[k] - stash[k - 1], efx[k] - efx[k - 1],
                                    rtol=1e-9, atol=1e-15)
+
+
+def test_muon_ef_lambda_scales_the_correction(lib):
+    """Eq. (1) for Muon's update: X_{t+1} = X_t - U - lambda (U - U_prev).
+    At lambda = 0 the EF run is bitwise the standard one; at lambda = 1/2 the
+    weights sit halfway between the standard and lambda = 1 runs (the same
+    U_t in all three while no correction has changed X_t: first two calls)."""
+    rng = np.random.default_rng(23)
+    x0 = rng.normal(size=(4, 6))
+    grads = [rng.normal(size=(4, 6)) for _ in range(4)]
+    runs = {}
+    for lam in (None, 0.0, 0.5, 1.0):
+        opt = DelayedMuon([x0], _hp(ef_lambda=lam or 0.0), ef=lam is not None, x_store=F64,
+                          stash_store=F64, lib=lib)
+        xs = []
+        for g in grads:
+            opt.step([g])
+            xs.append(opt.x[0].copy())
+        runs[lam] = xs
+    for a, b in zip(runs[None], runs[0.0]):
+        assert np.array_equal(a, b)
+    # second call: the first EF correction, on identical X_2 and U
+    half = 0.5 * (runs[None][1] + runs[1.0][1])
+    assert np.max(np.abs(runs[0.5][1] - half)) < 1e-14
+    assert np.max(np.abs(runs[1.0][1] - runs[None][1])) > 1e-6
+
+
+def test_muon_sapipe_prediction_rounds_through_the_master(lib):
+    """As for the elementwise rules: the SAPipe-WP stash is X_t - U_prev in
+    the master's format (fp32), then the stash's (bf16); 1 + 2^-8 - (-2^-30)
+    lands on the bf16 tie and rounds to even, 1.0."""
+    x0 = np.full((2, 2), 1.0 + 2.0 ** -8)
+    opt = DelayedMuon([x0], _hp(lr=0.0, weight_decay=0.0, correction=1), ef=True,
+                      x_store=F32, stash_store=BF16, lib=lib)
+    opt.u_prev[0][...] = -(2.0 ** -30)
+    opt.step([np.ones((2, 2))])
+    assert np.all(opt.stash[0] == 1.0)

@@ -83,6 +83,20 @@ MUTANTS = [
      "oracle_round(oracle_round(x[i] - u, hp->x_store), hp->stash_store)"),
     ("muon_ef_at_first_update", "const int ef_now = use_ef && !sapipe && t >= 2;",
      "const int ef_now = use_ef && !sapipe && t >= 1;"),
+    ("lion_sign_of_zero_positive", "(c < 0.0 ? -1.0 : 0.0)", "(c < 0.0 ? -1.0 : 1.0)"),
+    ("dc_abs_gradient", "hp->dc_lambda * gi * gi * (xt - stash[i])",
+     "hp->dc_lambda * fabs(gi) * (xt - stash[i])"),
+    ("dc_on_synchronous_tensors", "if (hp->dc_lambda != 0.0 && delayed)",
+     "if (hp->dc_lambda != 0.0)"),
+    ("sapipe_prediction_rounded_once",
+     "stash[i] = oracle_round(oracle_round(xt - u_prev[i], hp->x_store),\n"
+     "                                        hp->stash_store);",
+     "stash[i] = oracle_round(xt - u_prev[i], hp->stash_store);"),
+    ("muon_ef_lambda_ignored", "xt - u - hp->ef_lambda * (u - u_prev[i])",
+     "xt - u - (u - u_prev[i])"),
+    ("muon_sapipe_prediction_rounded_once",
+     "oracle_round(oracle_round(x[i] - u_prev[i], hp->x_store), hp->stash_store)",
+     "oracle_round(x[i] - u_prev[i], hp->stash_store)"),
 ]
 
 

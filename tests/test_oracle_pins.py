@@ -785,6 +785,12 @@ def test_dc_asgd_compensation(lib):
     o.step(np.array([1.0]), tag=o.read_weights()[1])
     assert o.m[0] == pytest.approx(1.0 + lam * 1.0 * (x2 - x1), rel=1e-14)
     assert x1 == 1.0 and x2 < 1.0
+    # a gradient of magnitude other than 1, and negative: the term is g^2,
+    # not |g| or g |g|
+    x3, x2s = o.x[0], o.stash[0]
+    o.step(np.array([-3.0]), tag=o.read_weights()[1])
+    assert o.m[0] == pytest.approx(-3.0 + lam * 9.0 * (x3 - x2s), rel=1e-14)
+    assert x3 != x2s
     # lambda = 0: identical to the plain rule
     rng = np.random.default_rng(15)
     x0, grads = rng.normal(0, 1, 30), [rng.normal(0, 1, 30) for _ in range(5)]
@@ -796,3 +802,56 @@ def test_dc_asgd_compensation(lib):
             o.step(g)
         runs.append(o.x.copy())
     assert np.array_equal(runs[0], runs[1])
+
+
+def test_dc_asgd_leaves_synchronous_tensors_alone(lib):
+    """DC-ASGD compensates for the staleness of a delayed tensor's gradient
+    (Sec. 3.1). A tensor trained synchronously (WPipe, App. B.2) has a fresh
+    gradient and no stash, so in a mixed table it follows the plain
+    synchronous rule bitwise, whatever lambda_dc."""
+    rng = np.random.default_rng(21)
+    xa, xb = rng.normal(0, 1, 9), rng.normal(0, 1, 6)
+    grads = [rng.normal(0, 1, 15) for _ in range(5)]
+    hp = HParams(lr=0.05, dc_lambda=30.0)
+    mixed = oracle.DelayedOptimizer([xa, xb], hp, x_store=F32, stash_store=F32,
+                                    delayed=[True, False], lib=lib)
+    plain = oracle.DelayedOptimizer([xb], HParams(lr=0.05, delay=0), x_store=F32,
+                                    stash_store=F32, lib=lib)
+    for g in grads:
+        mixed.step(g)
+        plain.step(g[9:])
+    assert np.array_equal(mixed.x[9:], plain.x)
+    # the delayed tensor is compensated: it differs from the lambda_dc = 0 run
+    nodc = oracle.DelayedOptimizer([xa, xb], HParams(lr=0.05), x_store=F32, stash_store=F32,
+                                   delayed=[True, False], lib=lib)
+    for g in grads:
+        nodc.step(g)
+    assert np.max(np.abs(mixed.x[:9] - nodc.x[:9])) > 1e-6
+
+
+def test_lion_sign_of_zero_is_zero(lib):
+    """Lion's update is the sign of the interpolation c, and sign(0) = 0: a
+    zero gradient from the zero start state moves no weight without decay,
+    and only by the decay lr wd x_t with it."""
+    for wd in (0.0, 0.1):
+        hp = HParams(lr=0.1, beta1=0.9, beta2=0.99, weight_decay=wd, rule=oracle.RULE_LION)
+        o = oracle.DelayedOptimizer([np.array([1.0, -2.0])], hp, x_store=F64, stash_store=F64,
+                                    lib=lib)
+        o.step(np.zeros(2), tag=o.read_weights()[1])
+        assert o.x.tolist() == pytest.approx([1.0 - 0.1 * wd, -2.0 * (1.0 - 0.1 * wd)],
+                                             abs=1e-16)
+
+
+def test_sapipe_prediction_is_a_master_weight_rounded_to_the_stash(lib):
+    """SAPipe-WP's stash (App. B.1) is the predicted weight x_t - u_prev, a
+    weight in the master's format (fp32) then stored in the stash's (bf16):
+    two roundings. x_t = 1 + 2^-8 and u_prev = -2^-30 give 1 + 2^-8 + 2^-30,
+    which fp32 rounds to the bf16 tie 1 + 2^-8 and bf16 then rounds to even,
+    1.0; rounded once it would be 1 + 2^-7."""
+    hp = HParams(lr=0.0, weight_decay=0.0, correction=oracle.CORR_SAPIPE_SAME)
+    o = oracle.DelayedOptimizer([np.array([1.0 + 2.0 ** -8])], hp, ef=True, x_store=F32,
+                                stash_store=BF16, lib=lib)
+    o.u_prev[:] = -(2.0 ** -30)
+    o.step(np.array([0.5]), tag=o.read_weights()[1])
+    assert o.stash[0] == 1.0
+    assert o.x[0] == 1.0 + 2.0 ** -8
