@@ -23,3 +23,14 @@ def cuda_device():
     if not torch.cuda.is_available():
         pytest.fail("GPU test collected on a machine without CUDA")
     return torch.device("cuda:0")
+
+
+def pytest_collection_modifyitems(config, items):
+    """Every GPU test runs under a wall-clock limit (pytest-timeout, where it
+    is installed): a test that stops making progress ends its process instead
+    of holding the GPU. The kernels' own waits are bounded well below it."""
+    if not config.pluginmanager.hasplugin("timeout"):
+        return
+    for item in items:
+        if item.get_closest_marker("gpu") is not None and item.get_closest_marker("timeout") is None:
+            item.add_marker(pytest.mark.timeout(1200, method="thread"))
