@@ -141,9 +141,11 @@ def kernel_source_sha(kernel: str = "fused_step") -> str:
     return h.hexdigest()[:16]
 
 
-def committed_traffic(kernel_tag: str):
-    """dram bytes per parameter from the committed ncu summary of the fused
-    kernel, if that summary was taken on the kernel source as it is now."""
+def committed_traffic(kernel_tag: str, key: str = "dram_bytes_per_param"):
+    """A DRAM-traffic figure (``key``: bytes per parameter of the fused
+    kernel, or bytes per step of the Newton-Schulz GEMMs) from the committed
+    ncu summary with this kernel tag, if that summary was taken on the kernel
+    source as it is now."""
     kernel = kernel_tag.split(":")[0]
     if kernel not in KERNEL_SOURCES:
         return None
@@ -155,7 +157,7 @@ def committed_traffic(kernel_tag: str):
         text = open(os.path.join(ROOT, "profiles", name)).read()
         m_tag = re.search(r"^kernel_tag:\s*(\S+)", text, re.M)
         m_sha = re.search(r"^kernel_source_sha256_16:\s*(\S+)", text, re.M)
-        m_b = re.search(r"^dram_bytes_per_param:\s*([0-9.eE+-]+)", text, re.M)
+        m_b = re.search(r"^" + re.escape(key) + r":\s*([0-9.eE+-]+)", text, re.M)
         if m_tag and m_sha and m_b and m_tag.group(1) == kernel_tag and m_sha.group(1) == sha:
             return float(m_b.group(1))
     return None
@@ -648,7 +650,9 @@ def main_muon(args, w, world, rank, local):
     peak, peak_kind = measured_bf16_peak()
     roof = {"bound": "tensor", "achieved": r["achieved"], "peak": peak, "unit": "TFLOP/s",
             "frac": r["achieved"] / peak, "peak_kind": f"{peak_kind} (sustained)",
-            "traffic": None, "kernel": "ns_gemm_kernel",
+            "traffic": committed_traffic(f"ns_gemm:{w.name}:muon-{args.mode}",
+                                         "dram_bytes_per_step"),
+            "kernel": "ns_gemm_kernel",
             "algorithmic_flops_per_step": r["flops"], "gemm_ms_per_step": r["gemm_ms"],
             "gemm_launches_per_step": r["gemm_launches"] / max(1, args.steps),
             "nominal_peak_tflops": 2250.0, "library_newton_schulz": r["library"]}
