@@ -186,7 +186,9 @@ def global_sqnorm(optimizers, acc, stream=None, group=None) -> None:
     DelayedMuon) hold, into ``acc`` (a one-element float64 device tensor):
     zeroed, each context's share added in list order on ``stream``, then
     summed over ``group``'s ranks. Optimizers whose clip source is ``acc``
-    then clip from the norm over all of them (App. E.1)."""
+    then clip from the norm over all of them (App. E.1): step them on the
+    same stream (the default, torch's current one) or after an event on it,
+    since the step reads ``acc`` on the device when it runs."""
     import torch
     s = stream if stream is not None else torch.cuda.current_stream(acc.device)
     with torch.cuda.stream(s):
