@@ -549,6 +549,13 @@ def _host_avail_bytes():
     return 0
 
 
+def e2e_fits(avail: int, io_bytes: int, local_world: int) -> bool:
+    """Whether every rank on the node can pin its staged copies and its
+    host-I/O arenas (twice the step's input and output bytes each), with
+    16 GiB left for the rest of the host."""
+    return avail >= local_world * 2 * io_bytes + (16 << 30)
+
+
 def run_e2e(args, opt, stream, dev, world, w):
     """End to end through the public API with the step's inputs (gradients)
     in pinned host memory and its result (the new bf16 weights) delivered to
@@ -559,8 +566,17 @@ def run_e2e(args, opt, stream, dev, world, w):
     import torch
     gbytes = opt.grad.numel() * opt.grad.element_size()
     pbytes = opt.param.numel() * opt.param.element_size()
-    if _host_avail_bytes() < 2 * (gbytes + pbytes) + (16 << 30):
-        return {"skipped": f"host memory: {(gbytes + pbytes) / 1e9:.1f} GB pinned needed"}
+    # every rank on this node pins its own copies, and all ranks must agree
+    # (the timed region has barriers)
+    local_world = int(os.environ.get("LOCAL_WORLD_SIZE", "1"))
+    ok = e2e_fits(_host_avail_bytes(), gbytes + pbytes, local_world)
+    if world > 1:
+        t = torch.tensor([1 if ok else 0], dtype=torch.int32, device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MIN)
+        ok = bool(t.item())
+    if not ok:
+        return {"skipped": f"host memory: {(gbytes + pbytes) / 1e9:.1f} GB pinned needed per rank, "
+                           f"{local_world} rank(s) on this node"}
     K = max(1, args.e2e_steps)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
 

@@ -95,3 +95,10 @@ def test_muon_takes_the_attention_and_mlp_matrices():
     assert "embed_tokens" in names and "lm_head" in names and "norm" in names
     mi, _ = bench.muon_split(W.GPT2_SMALL)
     assert len(mi) == 12 * 4 and all(len(W.GPT2_SMALL.tensors[i][1]) == 2 for i in mi)
+
+
+def test_e2e_host_memory_check_counts_every_rank_on_the_node():
+    io = 27 << 30
+    assert bench.e2e_fits(2 * io + (16 << 30), io, 1)
+    assert not bench.e2e_fits(2 * io + (16 << 30), io, 2)
+    assert bench.e2e_fits(8 * 2 * io + (16 << 30), io, 8)
