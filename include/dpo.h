@@ -284,6 +284,18 @@ int dpo_get_step(const dpo_ctx *ctx, int64_t *k);
 int dpo_set_step(dpo_ctx *ctx, int64_t k);
 
 /*
+ * The value of k at which the current delayed phase began (0 for a run that
+ * is delayed from the start; dpo_set_delay(1) sets it to the current k).
+ * Alg. 1's iteration index is t = k - k0: it decides where EF starts (t >= 2)
+ * and, with the ping-pong stash, which buffer holds which weights (the parity
+ * of t). A checkpoint saves it with k and the delay mode, and a resumed
+ * context restores it after dpo_set_step; 0 <= k0 <= k. Returns DPO_OK or
+ * DPO_EINVAL.
+ */
+int dpo_get_phase_start(const dpo_ctx *ctx, int64_t *k0);
+int dpo_set_phase_start(dpo_ctx *ctx, int64_t k0);
+
+/*
  * Diagnostics of the last clipped step: the DPO_FLAG_* bits raised since the
  * previous dpo_get_flags (reading clears them), the global gradient norm and
  * the clip coefficient used. Synchronizes cuda_stream (not for the hot

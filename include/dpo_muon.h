@@ -169,6 +169,15 @@ int dpo_muon_get_step(const dpo_muon_ctx *ctx, int64_t *k);
 int dpo_muon_set_step(dpo_muon_ctx *ctx, int64_t k);
 
 /*
+ * k at the start of the current delayed phase, as dpo_get_phase_start /
+ * dpo_set_phase_start (dpo.h): Alg. 1's t = k - k0 decides where EF starts.
+ * Save it with k; restore it after dpo_muon_set_step. Returns DPO_OK or
+ * DPO_EINVAL.
+ */
+int dpo_muon_get_phase_start(const dpo_muon_ctx *ctx, int64_t *k0);
+int dpo_muon_set_phase_start(dpo_muon_ctx *ctx, int64_t k0);
+
+/*
  * Tensor-core work of one step, summed over the matrices (r x w the
  * orientation with r <= w, unpadded), two flops per multiply-add:
  * ns_steps (r (r + 1) w + r (r + 1) r + 2 r^2 w), the first two terms being

@@ -710,6 +710,24 @@ extern "C" int dpo_set_step(dpo_ctx *c, int64_t k)
     return DPO_OK;
 }
 
+extern "C" int dpo_get_phase_start(const dpo_ctx *c, int64_t *k0)
+{
+    if (c == nullptr || k0 == nullptr)
+        return DPO_EINVAL;
+    *k0 = c->phase_k0;
+    return DPO_OK;
+}
+
+extern "C" int dpo_set_phase_start(dpo_ctx *c, int64_t k0)
+{
+    if (c == nullptr)
+        return DPO_EINVAL;
+    if (k0 < 0 || k0 > c->k)
+        return fail(c, DPO_EINVAL, "phase start must lie in [0, k]");
+    c->phase_k0 = k0;
+    return DPO_OK;
+}
+
 extern "C" int dpo_get_flags(dpo_ctx *c, uint32_t *flags, double *grad_norm, float *clip_scale,
                              void *cuda_stream)
 {

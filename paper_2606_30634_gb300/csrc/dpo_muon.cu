@@ -1086,6 +1086,24 @@ extern "C" int dpo_muon_set_clip_source(dpo_muon_ctx *c, const double *d_sumsq)
     return DPO_OK;
 }
 
+extern "C" int dpo_muon_get_phase_start(const dpo_muon_ctx *c, int64_t *k0)
+{
+    if (c == nullptr || k0 == nullptr)
+        return DPO_EINVAL;
+    *k0 = c->phase_k0;
+    return DPO_OK;
+}
+
+extern "C" int dpo_muon_set_phase_start(dpo_muon_ctx *c, int64_t k0)
+{
+    if (c == nullptr)
+        return DPO_EINVAL;
+    if (k0 < 0 || k0 > c->k)
+        return mfail(c, DPO_EINVAL, "phase start must lie in [0, k]");
+    c->phase_k0 = k0;
+    return DPO_OK;
+}
+
 extern "C" int dpo_muon_get_step(const dpo_muon_ctx *c, int64_t *k)
 {
     if (c == nullptr || k == nullptr)

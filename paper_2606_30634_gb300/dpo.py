@@ -33,7 +33,8 @@ DPO_STASH_COPY, DPO_STASH_PINGPONG = 0, 1
 EXPORTS = ("dpo_init", "dpo_stash", "dpo_step", "dpo_read_weights", "dpo_get_step",
            "dpo_set_step", "dpo_get_flags", "dpo_algorithmic_bytes", "dpo_launch_config",
            "dpo_last_error", "dpo_destroy", "dpo_grad_norm_noalloc", "dpo_set_delay",
-           "dpo_grad_sqnorm", "dpo_set_clip_source", "dpo_test_fail_allocs")
+           "dpo_grad_sqnorm", "dpo_set_clip_source", "dpo_test_fail_allocs",
+           "dpo_get_phase_start", "dpo_set_phase_start")
 
 DPO_NOALLOC_CHUNK_ELEMS = 1 << 20
 DPO_NOALLOC_MAX_CHUNKS = 16384
@@ -101,6 +102,8 @@ def load() -> ctypes.CDLL:
         "dpo_grad_sqnorm": (I, [P, P, P]),
         "dpo_set_clip_source": (I, [P, P]),
         "dpo_test_fail_allocs": (I, [I, I]),
+        "dpo_get_phase_start": (I, [P, ctypes.POINTER(ctypes.c_int64)]),
+        "dpo_set_phase_start": (I, [P, ctypes.c_int64]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -212,6 +215,16 @@ def dpo_get_step(ctx) -> int:
 
 def dpo_set_step(ctx, k: int) -> None:
     _check(load().dpo_set_step(ctx, k), ctx)
+
+
+def dpo_get_phase_start(ctx) -> int:
+    k0 = ctypes.c_int64()
+    _check(load().dpo_get_phase_start(ctx, ctypes.byref(k0)), ctx)
+    return k0.value
+
+
+def dpo_set_phase_start(ctx, k0: int) -> None:
+    _check(load().dpo_set_phase_start(ctx, k0), ctx)
 
 
 def dpo_get_flags(ctx, stream=None):
@@ -435,14 +448,22 @@ class DelayedAdamW:
         return dpo_get_step(self.ctx)
 
     def state_dict(self) -> dict:
+        """Every state arena, the step counter k, the start of the current
+        delayed phase (Alg. 1's t = k - k0) and the delay mode."""
         bufs = {n: getattr(self, n) for n in STATE_BUFFERS}
-        return {"k": self.k, **{n: b.clone() for n, b in bufs.items() if b is not None}}
+        return {"k": self.k, "phase_start": dpo_get_phase_start(self.ctx), "delay": self.delay,
+                **{n: b.clone() for n, b in bufs.items() if b is not None}}
 
     def load_state(self, sd: dict) -> None:
+        """Restore a state_dict into a context built with init_mode
+        DPO_INIT_RESUME and the same delay mode."""
+        if "delay" in sd and int(sd["delay"]) != self.delay:
+            raise ValueError(f"checkpoint taken with delay {sd['delay']}, context has {self.delay}")
         for n in STATE_BUFFERS:
             if getattr(self, n) is not None:
                 getattr(self, n).copy_(sd[n])
         dpo_set_step(self.ctx, int(sd["k"]))
+        dpo_set_phase_start(self.ctx, int(sd.get("phase_start", 0)))
 
     def close(self) -> None:
         if getattr(self, "ctx", None):

@@ -39,7 +39,7 @@ EXPORTS = ("dpo_muon_init", "dpo_muon_step", "dpo_muon_set_delay", "dpo_muon_las
            "dpo_muon_set_timing", "dpo_muon_get_gemm_time",
            "dpo_muon_workspace_bytes", "dpo_muon_last_error", "dpo_muon_destroy",
            "dpo_muon_grad_sqnorm", "dpo_muon_set_clip_source", "dpo_muon_clear_status",
-           "dpo_muon_test_stall")
+           "dpo_muon_test_stall", "dpo_muon_get_phase_start", "dpo_muon_set_phase_start")
 
 _typed = False
 
@@ -71,6 +71,8 @@ def lib() -> ctypes.CDLL:
             "dpo_muon_set_clip_source": (I, [P, P]),
             "dpo_muon_clear_status": (I, [P, P]),
             "dpo_muon_test_stall": (I, [P, I]),
+            "dpo_muon_get_phase_start": (I, [P, ctypes.POINTER(ctypes.c_int64)]),
+            "dpo_muon_set_phase_start": (I, [P, ctypes.c_int64]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -203,6 +205,32 @@ class DelayedMuon:
 
     def set_step(self, k: int) -> None:
         _check(lib().dpo_muon_set_step(self.ctx, k), self.ctx)
+
+    @property
+    def phase_start(self) -> int:
+        v = ctypes.c_int64()
+        _check(lib().dpo_muon_get_phase_start(self.ctx, ctypes.byref(v)), self.ctx)
+        return int(v.value)
+
+    STATE = ("master", "mom", "ef", "param", "stash")
+
+    def state_dict(self) -> dict:
+        """Every arena, k, the start of the current delayed phase and the
+        delay mode."""
+        return {"k": self.k, "phase_start": self.phase_start, "delay": self.delay,
+                **{n: getattr(self, n).clone() for n in self.STATE
+                   if getattr(self, n) is not None}}
+
+    def load_state(self, sd: dict) -> None:
+        """Restore a state_dict into a context built with init_mode
+        DPO_INIT_RESUME, the same shapes and the same delay mode."""
+        if int(sd["delay"]) != self.delay:
+            raise ValueError(f"checkpoint taken with delay {sd['delay']}, context has {self.delay}")
+        for n in self.STATE:
+            if getattr(self, n) is not None:
+                getattr(self, n).copy_(sd[n])
+        self.set_step(int(sd["k"]))
+        _check(lib().dpo_muon_set_phase_start(self.ctx, int(sd["phase_start"])), self.ctx)
 
     def flops(self) -> float:
         v = ctypes.c_double()

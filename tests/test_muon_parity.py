@@ -361,3 +361,51 @@ def test_gemm_wait_timeout_reports_status(cuda_device):
         assert np.linalg.norm(g - r) / np.linalg.norm(r) <= NS_BARS[1][0]
     finally:
         p.close()
+
+
+def test_muon_checkpoint_resume_after_synchronous_start(cuda_device):
+    """Synchronous start of 3 calls, delayed training with EF from call 4,
+    a checkpoint after call 5 restored into a new context (INIT_RESUME), 3
+    more calls: bitwise equal to 8 straight calls (k and the phase start
+    restored, so EF starts at the same call)."""
+    shapes = [(256, 512), (300, 700)]
+    kw = dict(ns_steps=1, ef=True, keep_stash=True, device=cuda_device)
+
+    def grads(m, k):
+        off = 0
+        for i, (r, c) in enumerate(shapes):
+            synth.dev_normal(0xC4E, synth.STREAM_GRAD, k, off, m.grads(i).view(-1), 1e-3)
+            off += r * c
+
+    x0 = [torch.from_numpy(x) for x in inputs(shapes, 0xC4E, 1)[0]]
+    straight = muon.DelayedMuon(shapes, x0=x0, **kw)
+    split = muon.DelayedMuon(shapes, x0=x0, **kw)
+    fresh = None
+    try:
+        for m in (straight, split):
+            m.set_delay(0)
+        for k in range(1, 9):
+            if k == 4:
+                straight.set_delay(1)
+            grads(straight, k)
+            straight.step()
+        for k in range(1, 6):
+            if k == 4:
+                split.set_delay(1)
+            grads(split, k)
+            split.step()
+        sd = split.state_dict()
+        assert sd["phase_start"] == 3 and sd["k"] == 5 and sd["delay"] == 1
+        fresh = muon.DelayedMuon(shapes, init_mode=dpo.DPO_INIT_RESUME, **kw)
+        fresh.load_state(sd)
+        for k in range(6, 9):
+            grads(fresh, k)
+            fresh.step()
+        torch.cuda.synchronize()
+        for name in muon.DelayedMuon.STATE:
+            assert torch.equal(getattr(straight, name), getattr(fresh, name)), name
+        assert straight.status() == 0 and fresh.status() == 0
+    finally:
+        for m in (straight, split, fresh):
+            if m is not None:
+                m.close()

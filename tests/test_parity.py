@@ -182,6 +182,42 @@ def test_checkpoint_resume_bitwise(cuda_device):
         split.close()
 
 
+def test_checkpoint_resume_after_synchronous_start(cuda_device):
+    """Synchronous start of 3 calls (odd), delayed training with EF and the
+    ping-pong stash, a checkpoint after call 5, restored into a new
+    context, 3 more calls: bitwise equal to 8 straight calls. The restored
+    phase start keeps Alg. 1's t = k - k0, which decides both where EF
+    starts and which of the two weight buffers holds which version."""
+    case = Case(RAGGED, stash_dtype=B, ef=True, stash_mode=dpo.DPO_STASH_PINGPONG,
+                schedule={1: 0, 4: 1})
+    straight = Run(case, cuda_device)
+    split = Run(case, cuda_device)
+    try:
+        for _ in range(8):
+            straight.step()
+        for _ in range(5):
+            split.step()
+        sd = split.gpu.state_dict()
+        assert sd["phase_start"] == 3 and sd["k"] == 5 and sd["delay"] == 1
+        split.gpu.close()
+        fresh = dpo.DelayedAdamW(case.numels, param_dtype=case.param_dtype,
+                                 stash_dtype=case.stash_dtype, grad_dtype=case.grad_dtype,
+                                 ef=True, device=cuda_device, init_mode=dpo.DPO_INIT_RESUME,
+                                 keep_stash=True, stash_mode=dpo.DPO_STASH_PINGPONG)
+        fresh.load_state(sd)
+        split.gpu = fresh
+        for _ in range(3):
+            split.step()
+        torch.cuda.synchronize()
+        for name in ("master", "m", "v", "ef"):
+            assert torch.equal(getattr(straight.gpu, name), getattr(split.gpu, name)), name
+        for a, b in zip(straight.gpu.role_arenas(), split.gpu.role_arenas()):
+            assert torch.equal(a, b)
+    finally:
+        straight.close()
+        split.close()
+
+
 def test_nonfinite_gradient_flag(cuda_device):
     run = Run(Case([1000, 17], max_grad_norm=1.0), cuda_device)
     try:
