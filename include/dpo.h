@@ -229,6 +229,28 @@ int dpo_stash(dpo_ctx *ctx, void *cuda_stream);
 int dpo_step(dpo_ctx *ctx, float lr, void *cuda_stream);
 
 /*
+ * Capturable mode, for CUDA graphs. A dpo_step captured into a graph and
+ * replayed must not reuse the scalars of the call it was captured at (the
+ * bias corrections and NAdam/Adan factors depend on k, EF's lambda on
+ * t = k - k0, the ping-pong roles on the parity of t). With on != 0 the
+ * counters (k, the phase start, NAdam's running product) move to device
+ * memory and every dpo_step enqueues a one-thread kernel that forms that
+ * call's scalars from them, in the same double arithmetic as the host path,
+ * and advances them; the fused kernel reads the scalars from there. The
+ * learning rate is read from lr_source (a device float, 4-byte aligned, kept
+ * alive while set; write it between replays for a schedule) or, when
+ * lr_source is NULL, is dpo_step's lr argument (fixed in a captured graph).
+ * dpo_step then enqueues launches only and can be captured; the calls that
+ * report or change the counters (dpo_get_step, dpo_set_step, dpo_get/
+ * set_phase_start, dpo_set_delay, dpo_read_weights with the ping-pong stash)
+ * synchronize the device first, so they do not belong inside a capture.
+ * on = 0 brings the counters back to the host (synchronizing). The hyper-
+ * parameters and the delay mode are fixed in a captured graph: change them
+ * outside it and capture again. Returns DPO_OK, DPO_EINVAL or DPO_ECUDA.
+ */
+int dpo_set_capturable(dpo_ctx *ctx, int on, const float *lr_source, void *cuda_stream);
+
+/*
  * One global gradient norm across contexts and ranks. Clipping scales every
  * gradient by one coefficient from the norm over all parameters (App. E.1);
  * when those parameters are split over several contexts (an AdamW context

@@ -34,9 +34,13 @@ struct dpo_ctx {
     bool host_io = false;   // grad or param in host memory
     bool has_stash = false; // some tensor has a stash buffer
     bool can_delay = false; // every tensor without DPO_SYNC has one
-    int64_t k = 0;
-    int64_t phase_k0 = 0;   // k when the current delayed phase began
-    double mu_prod = 1.0;   // NAdam: prod_{i<=k} mu_i
+    // step counters; a capturable context keeps the authoritative copy on
+    // the device (d_cnt) and refreshes these from it when the host needs them
+    mutable int64_t k = 0;
+    mutable int64_t phase_k0 = 0;   // k when the current delayed phase began
+    mutable double mu_prod = 1.0;   // NAdam: prod_{i<=k} mu_i
+    bool capturable = false;        // dpo_set_capturable
+    const float *lr_src = nullptr;  // capturable: device learning rate, or nullptr
     int64_t total_pkts = 0;
     int64_t total_elems = 0;
     std::vector<dpo_tensor> table;
@@ -48,6 +52,8 @@ struct dpo_ctx {
     int64_t *d_pkt_begin = nullptr;
     double *d_partials = nullptr;
     dpo::NormScalars *d_scalars = nullptr;
+    dpo::StepCounters *d_cnt = nullptr;   // capturable mode's counters
+    dpo::StepScalars *d_sc = nullptr;     // capturable mode's per-call scalars
     const double *clip_src = nullptr;   // external sum of squares (dpo_set_clip_source)
     std::string err;
 };
@@ -118,6 +124,32 @@ bool pingpong_on(const dpo_ctx *c)
 
 // Ping-pong stash: the latest weights of delayed tensors sit in the stash
 // buffer after an odd number of calls of the current delayed phase.
+// A capturable context's counters live on the device: refresh the host copy
+// (after all work on the device so far), or write the host copy back.
+int pull_counters(const dpo_ctx *c)
+{
+    if (!c->capturable)
+        return DPO_OK;
+    dpo::StepCounters h{};
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e == cudaSuccess)
+        e = cudaMemcpy(&h, c->d_cnt, sizeof h, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess)
+        return DPO_ECUDA;
+    c->k = h.k;
+    c->phase_k0 = h.phase_k0;
+    c->mu_prod = h.mu_prod;
+    return DPO_OK;
+}
+
+int push_counters(const dpo_ctx *c, cudaStream_t s)
+{
+    const dpo::StepCounters h{c->k, c->phase_k0, c->mu_prod};
+    // pageable source: the call returns once the bytes are staged
+    const cudaError_t e = cudaMemcpyAsync(c->d_cnt, &h, sizeof h, cudaMemcpyHostToDevice, s);
+    return e == cudaSuccess ? DPO_OK : DPO_ECUDA;
+}
+
 bool latest_in_stash(const dpo_ctx *c)
 {
     return pingpong_on(c) && ((c->k - c->phase_k0) & 1) != 0;
@@ -421,7 +453,9 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
     const size_t off_pkt = align_up(off_table + sizeof(DevTensor) * n_tensors, 256);
     const size_t off_part = align_up(off_pkt + sizeof(int64_t) * (n_tensors + 1), 256);
     const size_t off_scal = align_up(off_part + sizeof(double) * c->norm_grid, 256);
-    const size_t bytes = off_scal + sizeof(dpo::NormScalars);
+    const size_t off_cnt = align_up(off_scal + sizeof(dpo::NormScalars), 256);
+    const size_t off_sc = align_up(off_cnt + sizeof(dpo::StepCounters), 256);
+    const size_t bytes = off_sc + sizeof(dpo::StepScalars);
     e = dpo::device_alloc(&c->dev_block, bytes);
     if (e != cudaSuccess) {
         cudaGetLastError();
@@ -434,6 +468,8 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
     c->d_pkt_begin = reinterpret_cast<int64_t *>(base + off_pkt);
     c->d_partials = reinterpret_cast<double *>(base + off_part);
     c->d_scalars = reinterpret_cast<dpo::NormScalars *>(base + off_scal);
+    c->d_cnt = reinterpret_cast<dpo::StepCounters *>(base + off_cnt);
+    c->d_sc = reinterpret_cast<dpo::StepScalars *>(base + off_sc);
 
     std::vector<DevTensor> dt(n_tensors);
     std::vector<int64_t> pkt(n_tensors + 1, 0);
@@ -507,6 +543,8 @@ extern "C" int dpo_set_delay(dpo_ctx *c, int delay, void *cuda_stream)
         return fail(c, DPO_EINVAL, "delay must be 0 or 1");
     if (delay == c->hp.delay)
         return DPO_OK;
+    if (pull_counters(c) != DPO_OK)
+        return fail(c, DPO_ECUDA, "reading the device step counters failed");
     if (delay == 1) {
         if (!c->can_delay)
             return fail(c, DPO_ESTATE,
@@ -521,6 +559,8 @@ extern "C" int dpo_set_delay(dpo_ctx *c, int delay, void *cuda_stream)
                 return cuda_fail(c, e, "stash launch");
         }
         c->phase_k0 = c->k;
+        if (c->capturable && push_counters(c, static_cast<cudaStream_t>(cuda_stream)) != DPO_OK)
+            return fail(c, DPO_ECUDA, "writing the device step counters failed");
     } else if (latest_in_stash(c) && c->total_pkts > 0) {
         // Ping-pong: the latest weights sit in the stash buffer; synchronous
         // training keeps them in the param buffer (param := bf16(master)).
@@ -594,6 +634,15 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
         // when t is odd, the param buffer when t is even.
         a.swap = pingpong_on(c) && (t & 1) != 0;
         a.clip = c->clip ? &c->d_scalars->clip : nullptr;
+        if (c->capturable) {   // the per-call scalars come from the device counters
+            const dpo::ScalarConsts kc{c->hp.beta1, c->hp.beta2, c->hp.beta3, c->hp.weight_decay,
+                                       c->hp.momentum_decay, c->hp.ef_lambda,
+                                       corr == dpo::kCorrEF ? 1 : 0, pingpong_on(c) ? 1 : 0};
+            const cudaError_t es = dpo::launch_step_scalars(c->d_cnt, c->lr_src, lr, kc, c->d_sc, s);
+            if (es != cudaSuccess)
+                return cuda_fail(c, es, "step-scalars launch");
+            a.dev = c->d_sc;
+        }
         const cudaError_t e = dpo::launch_step(static_cast<dpo::Optimizer>(c->hp.optimizer),
                                                c->param_dt == DPO_BF16, stash_kind(c),
                                                c->grad_dt == DPO_BF16, corr, dc_on(c),
@@ -601,8 +650,39 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
         if (e != cudaSuccess)
             return cuda_fail(c, e, "fused step launch");
     }
+    if (c->capturable) {
+        if (c->total_pkts == 0) {   // nothing launched: keep the device counter in step
+            const dpo::ScalarConsts kc{c->hp.beta1, c->hp.beta2, c->hp.beta3, c->hp.weight_decay,
+                                       c->hp.momentum_decay, c->hp.ef_lambda, 0, 0};
+            const cudaError_t es = dpo::launch_step_scalars(c->d_cnt, c->lr_src, lr, kc, c->d_sc, s);
+            if (es != cudaSuccess)
+                return cuda_fail(c, es, "step-scalars launch");
+        }
+        return DPO_OK;   // the device counters advanced
+    }
     c->mu_prod *= nadam_mu(c->hp, k);
     c->k = k;
+    return DPO_OK;
+}
+
+extern "C" int dpo_set_capturable(dpo_ctx *c, int on, const float *lr_source, void *cuda_stream)
+{
+    if (c == nullptr)
+        return fail(nullptr, DPO_EINVAL, "ctx is NULL");
+    if (lr_source != nullptr && reinterpret_cast<uintptr_t>(lr_source) % alignof(float) != 0)
+        return fail(c, DPO_EINVAL, "lr_source must be 4-byte aligned");
+    cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+    if (on) {
+        if (!c->capturable && push_counters(c, s) != DPO_OK)
+            return fail(c, DPO_ECUDA, "writing the device step counters failed");
+        c->capturable = true;
+        c->lr_src = lr_source;
+    } else {
+        if (c->capturable && pull_counters(c) != DPO_OK)
+            return fail(c, DPO_ECUDA, "reading the device step counters failed");
+        c->capturable = false;
+        c->lr_src = nullptr;
+    }
     return DPO_OK;
 }
 
@@ -670,6 +750,8 @@ extern "C" int dpo_read_weights(const dpo_ctx *c, int which, int tensor, const v
     if (tensor < 0 || tensor >= c->n || (which != DPO_STALE && which != DPO_LATEST))
         return DPO_EINVAL;
     const dpo_tensor &d = c->table[tensor];
+    if (pingpong_on(c) && pull_counters(c) != DPO_OK)
+        return DPO_ECUDA;
     // Ping-pong: after an odd number of delayed calls the two buffers of a
     // delayed tensor hold each other's role.
     const bool swapped = latest_in_stash(c) && !(d.flags & DPO_SYNC);
@@ -693,6 +775,8 @@ extern "C" int dpo_get_step(const dpo_ctx *c, int64_t *k)
 {
     if (c == nullptr || k == nullptr)
         return DPO_EINVAL;
+    if (pull_counters(c) != DPO_OK)
+        return DPO_ECUDA;
     *k = c->k;
     return DPO_OK;
 }
@@ -703,10 +787,17 @@ extern "C" int dpo_set_step(dpo_ctx *c, int64_t k)
         return DPO_EINVAL;
     if (k < 0)
         return fail(c, DPO_EINVAL, "step counter must be >= 0");
+    if (pull_counters(c) != DPO_OK)   // the phase start stays as it is
+        return fail(c, DPO_ECUDA, "reading the device step counters failed");
     c->k = k;
     c->mu_prod = 1.0;   // NAdam's running product, rebuilt for the restored counter
     for (int64_t i = 1; i <= k; ++i)
         c->mu_prod *= nadam_mu(c->hp, i);
+    if (c->phase_k0 > k)
+        c->phase_k0 = k;
+    if (c->capturable && (push_counters(c, nullptr) != DPO_OK ||
+                          cudaDeviceSynchronize() != cudaSuccess))
+        return fail(c, DPO_ECUDA, "writing the device step counters failed");
     return DPO_OK;
 }
 
@@ -714,6 +805,8 @@ extern "C" int dpo_get_phase_start(const dpo_ctx *c, int64_t *k0)
 {
     if (c == nullptr || k0 == nullptr)
         return DPO_EINVAL;
+    if (pull_counters(c) != DPO_OK)
+        return DPO_ECUDA;
     *k0 = c->phase_k0;
     return DPO_OK;
 }
@@ -722,9 +815,14 @@ extern "C" int dpo_set_phase_start(dpo_ctx *c, int64_t k0)
 {
     if (c == nullptr)
         return DPO_EINVAL;
+    if (pull_counters(c) != DPO_OK)
+        return fail(c, DPO_ECUDA, "reading the device step counters failed");
     if (k0 < 0 || k0 > c->k)
         return fail(c, DPO_EINVAL, "phase start must lie in [0, k]");
     c->phase_k0 = k0;
+    if (c->capturable && (push_counters(c, nullptr) != DPO_OK ||
+                          cudaDeviceSynchronize() != cudaSuccess))
+        return fail(c, DPO_ECUDA, "writing the device step counters failed");
     return DPO_OK;
 }
 

@@ -53,8 +53,32 @@ enum Correction { kCorrNone = 0, kCorrEF = 1, kCorrSapipeSame = 2, kCorrSapipeUp
 // Update rule (the DPO_OPT_* of include/dpo.h).
 enum Optimizer { kOptAdamW = 0, kOptNAdam = 1, kOptLion = 2, kOptAdan = 3 };
 
+// The scalars of one fused step that change from call to call, formed in
+// double and rounded once to fp32: on the host (the fields of StepArgs) or,
+// for a capturable context, on the device by step_scalars_kernel.
+struct StepScalars {
+    float step_size, inv_sqrt_bc2, lr_wd, lam, step_size_next, inv_sqrt_bc2_next, lr;
+    float nadam_cg, nadam_cm, inv_sqrt_bc3, adan_c2;
+    int first, swap;
+};
+
+// Device-resident step counters of a capturable context.
+struct StepCounters {
+    int64_t k;          // gradients consumed so far
+    int64_t phase_k0;   // k at the start of the current delayed phase
+    double mu_prod;     // NAdam: prod_{i<=k} mu_i
+};
+
+// The step's constants, for step_scalars_kernel.
+struct ScalarConsts {
+    double beta1, beta2, beta3, weight_decay, momentum_decay;
+    float ef_lambda;
+    int ef_corr;        // the correction is EF (lambda applies from t = 2)
+    int pingpong;       // ping-pong stash in delayed training
+};
+
 // Scalars of one fused step, precomputed on the host in double and rounded
-// once to fp32.
+// once to fp32 (the per-call ones come from `dev` instead when it is set).
 struct StepArgs {
     const DevTensor *table;
     const int64_t *pkt_begin;   // n_tensors + 1 prefix offsets
@@ -79,6 +103,7 @@ struct StepArgs {
     int swap;                   // ping-pong stash: write delayed tensors' weights into
                                 // their stash buffer (else their param buffer)
     const float *clip;          // device clip coefficient, or nullptr
+    const StepScalars *dev;     // capturable context: the per-call scalars, or nullptr
 };
 
 // Device scalars written by the norm pass (one per context).
@@ -132,6 +157,10 @@ cudaError_t launch_step(Optimizer opt, bool param_bf16, StashKind stash, bool gr
                         Correction corr, bool dc, bool pp, int grid, const StepArgs &a,
                         cudaStream_t s);
 cudaError_t launch_norm(bool grad_bf16, int grid, const NormArgs &a, cudaStream_t s);
+// The per-call scalars of the next step from the device counters, which it
+// advances (one thread; lr from *lr_src when set, else lr).
+cudaError_t launch_step_scalars(StepCounters *cnt, const float *lr_src, float lr,
+                                const ScalarConsts &k, StepScalars *out, cudaStream_t s);
 // Clip coefficient and norm from an external sum of squares (one thread).
 cudaError_t launch_clip_from_sumsq(const double *sumsq, double max_norm, NormScalars *out,
                                    cudaStream_t s);

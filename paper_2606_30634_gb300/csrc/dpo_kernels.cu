@@ -278,6 +278,50 @@ cudaError_t launch_norm(bool gb, int grid, const NormArgs &a, cudaStream_t s)
     return cudaGetLastError();
 }
 
+// NAdam's momentum schedule mu_i = beta1 (1 - 0.5 * 0.96^(i psi)).
+__device__ double nadam_mu_dev(const ScalarConsts &k, int64_t i)
+{
+    return k.beta1 * (1.0 - 0.5 * pow(0.96, (double)i * k.momentum_decay));
+}
+
+// The host's per-call arithmetic of dpo_step, on the device counters.
+__global__ void step_scalars_kernel(StepCounters *cnt, const float *lr_src, float lr_host,
+                                    const ScalarConsts k, StepScalars *out)
+{
+    const int64_t kk = cnt->k + 1;            // this call consumes the kk-th gradient
+    const int64_t t = kk - cnt->phase_k0;     // Alg. 1 iteration within the delayed phase
+    const float lr = lr_src != nullptr ? *lr_src : lr_host;
+    const double lrd = lr;
+    const double bc1 = 1.0 - pow(k.beta1, (double)kk);
+    const double bc2 = 1.0 - pow(k.beta2, (double)kk);
+    StepScalars sc;
+    sc.step_size = (float)(lrd / bc1);
+    sc.inv_sqrt_bc2 = (float)(1.0 / sqrt(bc2));
+    sc.lr_wd = (float)(lrd * k.weight_decay);
+    sc.lam = (k.ef_corr && t >= 2) ? k.ef_lambda : 0.0f;   // Alg. 1: standard rule at t <= 1
+    sc.step_size_next = (float)(lrd / (1.0 - pow(k.beta1, (double)(kk + 1))));
+    sc.inv_sqrt_bc2_next = (float)(1.0 / sqrt(1.0 - pow(k.beta2, (double)(kk + 1))));
+    sc.lr = lr;
+    const double mu_k = nadam_mu_dev(k, kk), mu_next = nadam_mu_dev(k, kk + 1);
+    const double mu_prod = cnt->mu_prod * mu_k;
+    sc.nadam_cg = (float)(lrd * (1.0 - mu_k) / (1.0 - mu_prod));
+    sc.nadam_cm = (float)(lrd * mu_next / (1.0 - mu_prod * mu_next));
+    sc.inv_sqrt_bc3 = (float)(1.0 / sqrt(1.0 - pow(k.beta3, (double)kk)));
+    sc.adan_c2 = (float)(lrd * k.beta2 / bc2);
+    sc.first = kk == 1;
+    sc.swap = k.pingpong && (t & 1) != 0;
+    *out = sc;
+    cnt->k = kk;
+    cnt->mu_prod = mu_prod;
+}
+
+cudaError_t launch_step_scalars(StepCounters *cnt, const float *lr_src, float lr,
+                                const ScalarConsts &k, StepScalars *out, cudaStream_t s)
+{
+    step_scalars_kernel<<<1, 1, 0, s>>>(cnt, lr_src, lr, k, out);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_clip_from_sumsq(const double *sumsq, double max_norm, NormScalars *out,
                                    cudaStream_t s)
 {

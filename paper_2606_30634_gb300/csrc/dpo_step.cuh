@@ -124,12 +124,19 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
     if (p >= a.total_pkts)
         return;
 
-    const Scalars s{a.beta1, a.omb1, a.beta2, a.omb2, a.step_size, a.inv_sqrt_bc2, a.eps, a.lam,
-                    a.step_size_next, a.inv_sqrt_bc2_next, a.lr, a.nadam_cg, a.nadam_cm,
-                    a.beta3, a.omb3, a.inv_sqrt_bc3, a.adan_c2, a.first != 0};
+    // The per-call scalars: kernel parameters, or (capturable context) the
+    // values step_scalars_kernel left in device memory for this call.
+    StepScalars sc{a.step_size, a.inv_sqrt_bc2, a.lr_wd, a.lam, a.step_size_next,
+                   a.inv_sqrt_bc2_next, a.lr, a.nadam_cg, a.nadam_cm, a.inv_sqrt_bc3, a.adan_c2,
+                   a.first, a.swap};
+    if (a.dev != nullptr)
+        sc = *a.dev;
+    const Scalars s{a.beta1, a.omb1, a.beta2, a.omb2, sc.step_size, sc.inv_sqrt_bc2, a.eps, sc.lam,
+                    sc.step_size_next, sc.inv_sqrt_bc2_next, sc.lr, sc.nadam_cg, sc.nadam_cm,
+                    a.beta3, a.omb3, sc.inv_sqrt_bc3, sc.adan_c2, sc.first != 0};
     const float clip = a.clip != nullptr ? __ldg(a.clip) : 1.0f;
-    const bool use_prev = kSapipe || (CORR == kCorrEF && a.lam != 0.0f);
-    const bool ef_now = CORR == kCorrEF && a.lam != 0.0f;
+    const bool use_prev = kSapipe || (CORR == kCorrEF && sc.lam != 0.0f);
+    const bool ef_now = CORR == kCorrEF && sc.lam != 0.0f;
     const float dc = a.dc_lambda;
 
     Cursor c;
@@ -145,7 +152,7 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
         float *__restrict__ gpv = d.grad_prev;
         float *__restrict__ ef = d.ef;
         const GT *__restrict__ grad = static_cast<const GT *>(d.grad);
-        const float wd_lr = (d.flags & kFlagWd) ? a.lr_wd : 0.0f;
+        const float wd_lr = (d.flags & kFlagWd) ? sc.lr_wd : 0.0f;
         // A DPO_SYNC tensor takes the standard update with no stash and no
         // correction even while the run is delayed.
         const bool dly = SK != kStashNone && !(d.flags & kFlagSync);
@@ -153,7 +160,7 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
         // buffer holding the stale version, which is then the one DC-ASGD
         // reads, and no stash is stored.
         const bool pp = PP && dly;
-        __nv_bfloat16 *param = static_cast<__nv_bfloat16 *>(pp && a.swap ? d.stash : d.param);
+        __nv_bfloat16 *param = static_cast<__nv_bfloat16 *>(pp && sc.swap ? d.stash : d.param);
         ST *stash = pp ? reinterpret_cast<ST *>(param) : static_cast<ST *>(d.stash);   // may alias param
         const bool prev_t = dly && use_prev;
         const bool efn_t = dly && ef_now;

@@ -34,7 +34,7 @@ EXPORTS = ("dpo_init", "dpo_stash", "dpo_step", "dpo_read_weights", "dpo_get_ste
            "dpo_set_step", "dpo_get_flags", "dpo_algorithmic_bytes", "dpo_launch_config",
            "dpo_last_error", "dpo_destroy", "dpo_grad_norm_noalloc", "dpo_set_delay",
            "dpo_grad_sqnorm", "dpo_set_clip_source", "dpo_test_fail_allocs",
-           "dpo_get_phase_start", "dpo_set_phase_start")
+           "dpo_get_phase_start", "dpo_set_phase_start", "dpo_set_capturable")
 
 DPO_NOALLOC_CHUNK_ELEMS = 1 << 20
 DPO_NOALLOC_MAX_CHUNKS = 16384
@@ -104,6 +104,7 @@ def load() -> ctypes.CDLL:
         "dpo_test_fail_allocs": (I, [I, I]),
         "dpo_get_phase_start": (I, [P, ctypes.POINTER(ctypes.c_int64)]),
         "dpo_set_phase_start": (I, [P, ctypes.c_int64]),
+        "dpo_set_capturable": (I, [P, I, P, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -215,6 +216,11 @@ def dpo_get_step(ctx) -> int:
 
 def dpo_set_step(ctx, k: int) -> None:
     _check(load().dpo_set_step(ctx, k), ctx)
+
+
+def dpo_set_capturable(ctx, on: bool, lr_source=None, stream=None) -> None:
+    """Capturable mode (include/dpo.h): step counters on the device."""
+    _check(load().dpo_set_capturable(ctx, 1 if on else 0, _dptr(lr_source), _stream(stream)), ctx)
 
 
 def dpo_get_phase_start(ctx) -> int:
@@ -429,6 +435,14 @@ class DelayedAdamW:
 
     def step(self, lr: Optional[float] = None, stream=None) -> None:
         dpo_step(self.ctx, self.lr if lr is None else lr, stream)
+
+    def set_capturable(self, on: bool = True, lr_source=None, stream=None) -> None:
+        """Capturable mode (dpo_set_capturable): the step counters live on
+        the device, so a step captured in a CUDA graph can be replayed.
+        ``lr_source``: a one-element float32 device tensor read at every
+        step (kept alive here), or None for the lr passed to step()."""
+        dpo_set_capturable(self.ctx, on, lr_source, stream)
+        self._lr_src = lr_source if on else None
 
     def grad_sqnorm(self, acc, stream=None) -> None:
         """Add this context's sum of g^2 to ``acc`` (dpo_grad_sqnorm)."""

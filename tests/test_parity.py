@@ -11,7 +11,7 @@ import torch
 
 from paper_2606_30634_gb300 import dpo, synth
 import oracle
-from parity_util import TOL_ONE_STEP, TOL_RUN, Case, Run, bf16_ulps, rel_err
+from parity_util import TOL_ONE_STEP, TOL_RUN, Case, Run, bf16_ord, bf16_ulps, rel_err
 
 pytestmark = pytest.mark.gpu
 
@@ -584,3 +584,64 @@ def test_sapipe_updated_state_needs_adamw(cuda_device):
         dpo.DelayedAdamW([100], ef=True, correction=SP_UPD, optimizer=dpo.DPO_OPT_LION,
                          device=cuda_device)
     assert e.value.code == dpo.DPO_EINVAL
+
+
+@pytest.mark.parametrize("name,case,n_sync", [
+    ("adamw_ef_pingpong", Case(RAGGED, stash_dtype=B, ef=True,
+                               stash_mode=dpo.DPO_STASH_PINGPONG), 0),
+    ("nadam_ef_after_sync_start", Case(RAGGED, ef=True, optimizer=dpo.DPO_OPT_NADAM), 3),
+    ("adan_clipped", Case(RAGGED, optimizer=dpo.DPO_OPT_ADAN, max_grad_norm=0.05), 0),
+])
+def test_capturable_step_replays_in_a_cuda_graph(cuda_device, name, case, n_sync):
+    """One dpo_step captured in a CUDA graph (capturable mode) and replayed
+    six times with fresh gradients and a learning rate written to device
+    memory between replays, beside an eager run: the device-formed scalars
+    follow k (bias corrections, NAdam's products, Adan's first step), t = k -
+    k0 (EF from t = 2, the ping-pong roles) and the schedule, so both runs
+    agree at every call (fp32 state to 1e-6, bf16 weights to one ulp)."""
+    eager, cap = Run(case, cuda_device), Run(case, cuda_device)
+    lrs = [None] + [3e-4 * (1.0 - 0.07 * i) for i in range(1, 1 + n_sync + 6)]
+    lr_t = torch.empty(1, dtype=torch.float32, device=cuda_device)
+    try:
+        k = 0
+        if n_sync:
+            for r in (eager, cap):
+                r.gpu.set_delay(0)
+        for _ in range(n_sync):
+            k += 1
+            for r in (eager, cap):
+                r.draw(k)
+                r.gpu.step(lrs[k])
+        if n_sync:
+            for r in (eager, cap):
+                r.gpu.set_delay(1)
+        cap.gpu.set_capturable(True, lr_source=lr_t)
+        torch.cuda.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            cap.gpu.step()
+        for _ in range(6):
+            k += 1
+            eager.draw(k)
+            cap.draw(k)
+            lr_t.fill_(lrs[k])
+            eager.gpu.step(lrs[k])
+            graph.replay()
+            torch.cuda.synchronize()
+            for buf in ("master", "m", "v", "n", "grad_prev", "ef"):
+                a, b = getattr(eager.gpu, buf), getattr(cap.gpu, buf)
+                if a is not None:
+                    assert rel_err(b.cpu().numpy(), a.cpu().numpy().astype(np.float64)) <= 1e-6, \
+                        (name, k, buf)
+            la, _ = eager.gpu.role_arenas()
+            lb, _ = cap.gpu.role_arenas()
+            if la is not None:
+                d = bf16_ord(lb.view(torch.int16).cpu().numpy().view(np.uint16)).astype(np.int64) - \
+                    bf16_ord(la.view(torch.int16).cpu().numpy().view(np.uint16)).astype(np.int64)
+                assert np.max(np.abs(d)) <= 1, (name, k)
+        assert cap.gpu.k == eager.gpu.k == k
+        cap.gpu.set_capturable(False)
+        assert cap.gpu.k == k
+    finally:
+        eager.close()
+        cap.close()
