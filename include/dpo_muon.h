@@ -164,6 +164,20 @@ int dpo_muon_clear_status(dpo_muon_ctx *ctx, void *cuda_stream);
  */
 int dpo_muon_test_stall(dpo_muon_ctx *ctx, int launches);
 
+/*
+ * Capturable mode for CUDA graphs, as dpo_set_capturable (dpo.h): the step
+ * counters move to device memory, and each dpo_muon_step forms its update's
+ * lr, lr wd and EF start (t >= 2) on the device, so a step captured in a
+ * graph replays correctly; lr from lr_source (a device float) when set, else
+ * dpo_muon_step's argument. The counter calls and dpo_muon_set_delay
+ * synchronize the device and do not belong inside a capture; with
+ * dpo_muon_set_timing on, the step records events whose host bookkeeping a
+ * replay does not repeat, so leave timing off while capturing. Returns
+ * DPO_OK, DPO_EINVAL or DPO_ECUDA.
+ */
+int dpo_muon_set_capturable(dpo_muon_ctx *ctx, int on, const float *lr_source,
+                            void *cuda_stream);
+
 /* Calls consumed so far (k), and restore after loading a checkpoint. */
 int dpo_muon_get_step(const dpo_muon_ctx *ctx, int64_t *k);
 int dpo_muon_set_step(dpo_muon_ctx *ctx, int64_t k);

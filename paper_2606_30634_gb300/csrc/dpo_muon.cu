@@ -210,13 +210,42 @@ __global__ void __launch_bounds__(kThreads) muon_normalize_kernel(const NormArgs
     }
 }
 
+// The update's per-call scalars (host-formed, or device-formed for a
+// capturable context by muon_scalars_kernel).
+struct ApplyScalars {
+    float lr, lr_wd;
+    int ef_now;
+};
+
+// Device-resident counters of a capturable context.
+struct MuonCounters {
+    int64_t k, phase_k0;
+};
+
 struct ApplyArgs {
     const DevMat *mats;
     int chunks;
     float lr, lr_wd, lam;
     int ef_now, hist, delayed;
     int sapipe;               // SAPipe-WP same state: stash := x_t - U_prev, standard rule
+    const ApplyScalars *dev;  // capturable context: lr, lr_wd, ef_now of this call
 };
+
+// One thread: the next call's lr (from *lr_src when set), lr wd and whether
+// EF applies (Alg. 1: from t = 2 of the delayed phase); advances k.
+__global__ void muon_scalars_kernel(MuonCounters *cnt, const float *lr_src, float lr_host,
+                                    double weight_decay, int ef_possible, ApplyScalars *out)
+{
+    const int64_t k = cnt->k + 1;
+    const int64_t t = k - cnt->phase_k0;
+    const float lr = lr_src != nullptr ? *lr_src : lr_host;
+    ApplyScalars sc;
+    sc.lr = lr;
+    sc.lr_wd = (float)((double)lr * weight_decay);
+    sc.ef_now = ef_possible && t >= 2;
+    *out = sc;
+    cnt->k = k;
+}
 
 template <int SK>
 __global__ void __launch_bounds__(kThreads) muon_apply_kernel(const ApplyArgs a)
@@ -228,13 +257,14 @@ __global__ void __launch_bounds__(kThreads) muon_apply_kernel(const ApplyArgs a)
     if (lo >= n)
         return;
     const int64_t hi = lo + kChunk < n ? lo + kChunk : n;
-    const float lr_r = a.lr * d.r_scale, lr_wd = a.lr_wd * d.wd_lr_scale;
+    const ApplyScalars sc = a.dev != nullptr ? *a.dev : ApplyScalars{a.lr, a.lr_wd, a.ef_now};
+    const float lr_r = sc.lr * d.r_scale, lr_wd = sc.lr_wd * d.wd_lr_scale;
     ST *stash = static_cast<ST *>(d.stash);
     __nv_bfloat16 *param = static_cast<__nv_bfloat16 *>(d.param);
     const bool vec_o = (d.cols % kPacket) == 0;
     // a DPO_SYNC matrix takes the standard update with no stash and no history
     const bool dly = a.delayed && !d.sync;
-    const bool hist = a.hist && dly, ef_now = a.ef_now && dly;
+    const bool hist = a.hist && dly, ef_now = sc.ef_now && dly;
     const bool sapipe = a.sapipe && hist;
     for (int64_t e = lo + (int64_t)threadIdx.x * kPacket; e < hi; e += (int64_t)kThreads * kPacket) {
         if (e + kPacket <= hi && vec_o) {
@@ -402,8 +432,14 @@ struct dpo_muon_ctx {
     bool ef = false;
     bool has_stash = false;   // some matrix has a stash buffer
     bool can_delay = true;    // every matrix without DPO_SYNC has one
-    int64_t k = 0;
-    int64_t phase_k0 = 0;     // k when the current delayed phase began
+    // step counters; a capturable context keeps the authoritative copy on
+    // the device (d_cnt) and refreshes these from it when the host needs them
+    mutable int64_t k = 0;
+    mutable int64_t phase_k0 = 0;     // k when the current delayed phase began
+    bool capturable = false;          // dpo_muon_set_capturable
+    const float *lr_src = nullptr;    // capturable: device learning rate, or nullptr
+    dpo::muon::MuonCounters *d_cnt = nullptr;
+    dpo::muon::ApplyScalars *d_asc = nullptr;
     int sms = 0;
     int gemm_pairs = 0;   // clusters of 2 the GEMM kernel keeps resident at once
     int stall_launches = 0;   // dpo_muon_test_stall: GEMM launches left to stall
@@ -643,6 +679,10 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
     off += al((int64_t)sizeof(double) * c->norm_grid);
     const int64_t o_nsc = off;
     off += al(sizeof(dpo::NormScalars));
+    const int64_t o_cnt = off;
+    off += al(sizeof(dpo::muon::MuonCounters));
+    const int64_t o_asc = off;
+    off += al(sizeof(dpo::muon::ApplyScalars));
 
     cudaError_t e = dpo::device_alloc(&c->dev_block, (size_t)off);
     if (e != cudaSuccess) {
@@ -666,6 +706,8 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
     c->d_pkt_begin = reinterpret_cast<int64_t *>(blk + o_pkt);
     c->d_norm_partials = reinterpret_cast<double *>(blk + o_npart);
     c->d_norm_scalars = reinterpret_cast<dpo::NormScalars *>(blk + o_nsc);
+    c->d_cnt = reinterpret_cast<dpo::muon::MuonCounters *>(blk + o_cnt);
+    c->d_asc = reinterpret_cast<dpo::muon::ApplyScalars *>(blk + o_asc);
 
     // Carve the workspace and build the tensor maps.
     char *wp = static_cast<char *>(c->ws);
@@ -833,6 +875,12 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const int64_t k = c->k + 1;
     if (c->n == 0 || c->total_elems == 0) {
+        if (c->capturable) {   // keep the device counter in step
+            dpo::muon::muon_scalars_kernel<<<1, 1, 0, s>>>(c->d_cnt, c->lr_src, lr, 0.0, 0,
+                                                           c->d_asc);
+            const cudaError_t e = cudaGetLastError();
+            return e == cudaSuccess ? DPO_OK : mcuda(c, e, "scalars launch");
+        }
         c->k = k;
         return DPO_OK;
     }
@@ -962,6 +1010,14 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
     aa.sapipe = c->hp.correction == DPO_CORR_SAPIPE_SAME;
     aa.ef_now = aa.hist && !aa.sapipe && t >= 2 && c->hp.ef_lambda != 0.0f;
     aa.lam = c->hp.ef_lambda;
+    if (c->capturable) {   // lr and EF's start from the device counters
+        dpo::muon::muon_scalars_kernel<<<1, 1, 0, s>>>(
+            c->d_cnt, c->lr_src, lr, (double)c->hp.weight_decay,
+            aa.hist && !aa.sapipe && c->hp.ef_lambda != 0.0f ? 1 : 0, c->d_asc);
+        if ((e = cudaGetLastError()) != cudaSuccess)
+            return mcuda(c, e, "scalars launch");
+        aa.dev = c->d_asc;
+    }
     const bool st = c->hp.delay == 1;
     if (!st)
         dpo::muon::muon_apply_kernel<dpo::kStashNone><<<mgrid, kThreads, 0, s>>>(aa);
@@ -971,7 +1027,59 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
         dpo::muon::muon_apply_kernel<dpo::kStashF32><<<mgrid, kThreads, 0, s>>>(aa);
     if ((e = cudaGetLastError()) != cudaSuccess)
         return mcuda(c, e, "apply launch");
-    c->k = k;
+    if (!c->capturable)
+        c->k = k;
+    return DPO_OK;
+}
+
+namespace {
+
+// A capturable context's counters live on the device: refresh the host copy
+// (after all work so far), or write the host copy back.
+int mpull(const dpo_muon_ctx *c)
+{
+    if (!c->capturable)
+        return DPO_OK;
+    dpo::muon::MuonCounters h{};
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e == cudaSuccess)
+        e = cudaMemcpy(&h, c->d_cnt, sizeof h, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess)
+        return DPO_ECUDA;
+    c->k = h.k;
+    c->phase_k0 = h.phase_k0;
+    return DPO_OK;
+}
+
+int mpush(const dpo_muon_ctx *c, cudaStream_t s)
+{
+    const dpo::muon::MuonCounters h{c->k, c->phase_k0};
+    // pageable source: the call returns once the bytes are staged
+    return cudaMemcpyAsync(c->d_cnt, &h, sizeof h, cudaMemcpyHostToDevice, s) == cudaSuccess
+               ? DPO_OK
+               : DPO_ECUDA;
+}
+
+}  // namespace
+
+extern "C" int dpo_muon_set_capturable(dpo_muon_ctx *c, int on, const float *lr_source,
+                                       void *stream)
+{
+    if (c == nullptr)
+        return DPO_EINVAL;
+    if (lr_source != nullptr && reinterpret_cast<uintptr_t>(lr_source) % alignof(float) != 0)
+        return mfail(c, DPO_EINVAL, "lr_source must be 4-byte aligned");
+    if (on) {
+        if (!c->capturable && mpush(c, static_cast<cudaStream_t>(stream)) != DPO_OK)
+            return mfail(c, DPO_ECUDA, "writing the device step counters failed");
+        c->capturable = true;
+        c->lr_src = lr_source;
+    } else {
+        if (c->capturable && mpull(c) != DPO_OK)
+            return mfail(c, DPO_ECUDA, "reading the device step counters failed");
+        c->capturable = false;
+        c->lr_src = nullptr;
+    }
     return DPO_OK;
 }
 
@@ -991,7 +1099,11 @@ extern "C" int dpo_muon_set_delay(dpo_muon_ctx *c, int delay, void *stream)
         const int rc = launch_init(c, static_cast<cudaStream_t>(stream), 0, 1);
         if (rc != DPO_OK)
             return rc;
+        if (mpull(c) != DPO_OK)
+            return mfail(c, DPO_ECUDA, "reading the device step counters failed");
         c->phase_k0 = c->k;
+        if (c->capturable && mpush(c, static_cast<cudaStream_t>(stream)) != DPO_OK)
+            return mfail(c, DPO_ECUDA, "writing the device step counters failed");
     }
     c->hp.delay = delay;
     return DPO_OK;
@@ -1090,6 +1202,8 @@ extern "C" int dpo_muon_get_phase_start(const dpo_muon_ctx *c, int64_t *k0)
 {
     if (c == nullptr || k0 == nullptr)
         return DPO_EINVAL;
+    if (mpull(c) != DPO_OK)
+        return DPO_ECUDA;
     *k0 = c->phase_k0;
     return DPO_OK;
 }
@@ -1098,9 +1212,13 @@ extern "C" int dpo_muon_set_phase_start(dpo_muon_ctx *c, int64_t k0)
 {
     if (c == nullptr)
         return DPO_EINVAL;
+    if (mpull(c) != DPO_OK)
+        return mfail(c, DPO_ECUDA, "reading the device step counters failed");
     if (k0 < 0 || k0 > c->k)
         return mfail(c, DPO_EINVAL, "phase start must lie in [0, k]");
     c->phase_k0 = k0;
+    if (c->capturable && (mpush(c, nullptr) != DPO_OK || cudaDeviceSynchronize() != cudaSuccess))
+        return mfail(c, DPO_ECUDA, "writing the device step counters failed");
     return DPO_OK;
 }
 
@@ -1108,6 +1226,8 @@ extern "C" int dpo_muon_get_step(const dpo_muon_ctx *c, int64_t *k)
 {
     if (c == nullptr || k == nullptr)
         return DPO_EINVAL;
+    if (mpull(c) != DPO_OK)
+        return DPO_ECUDA;
     *k = c->k;
     return DPO_OK;
 }
@@ -1116,7 +1236,13 @@ extern "C" int dpo_muon_set_step(dpo_muon_ctx *c, int64_t k)
 {
     if (c == nullptr || k < 0)
         return DPO_EINVAL;
+    if (mpull(c) != DPO_OK)
+        return mfail(c, DPO_ECUDA, "reading the device step counters failed");
     c->k = k;
+    if (c->phase_k0 > k)
+        c->phase_k0 = k;
+    if (c->capturable && (mpush(c, nullptr) != DPO_OK || cudaDeviceSynchronize() != cudaSuccess))
+        return mfail(c, DPO_ECUDA, "writing the device step counters failed");
     return DPO_OK;
 }
 

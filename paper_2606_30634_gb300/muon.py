@@ -39,7 +39,8 @@ EXPORTS = ("dpo_muon_init", "dpo_muon_step", "dpo_muon_set_delay", "dpo_muon_las
            "dpo_muon_set_timing", "dpo_muon_get_gemm_time",
            "dpo_muon_workspace_bytes", "dpo_muon_last_error", "dpo_muon_destroy",
            "dpo_muon_grad_sqnorm", "dpo_muon_set_clip_source", "dpo_muon_clear_status",
-           "dpo_muon_test_stall", "dpo_muon_get_phase_start", "dpo_muon_set_phase_start")
+           "dpo_muon_test_stall", "dpo_muon_get_phase_start", "dpo_muon_set_phase_start",
+           "dpo_muon_set_capturable")
 
 _typed = False
 
@@ -73,6 +74,7 @@ def lib() -> ctypes.CDLL:
             "dpo_muon_test_stall": (I, [P, I]),
             "dpo_muon_get_phase_start": (I, [P, ctypes.POINTER(ctypes.c_int64)]),
             "dpo_muon_set_phase_start": (I, [P, ctypes.c_int64]),
+            "dpo_muon_set_capturable": (I, [P, I, P, P]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -189,6 +191,14 @@ class DelayedMuon:
         v = ctypes.c_uint32()
         _check(lib().dpo_muon_get_status(self.ctx, ctypes.byref(v)), self.ctx)
         return int(v.value)
+
+    def set_capturable(self, on: bool = True, lr_source=None, stream=None) -> None:
+        """Capturable mode (dpo_muon_set_capturable); ``lr_source`` a
+        one-element float32 device tensor, kept alive here, or None."""
+        _check(lib().dpo_muon_set_capturable(self.ctx, 1 if on else 0,
+                                             lr_source.data_ptr() if lr_source is not None
+                                             else None, _stream(stream)), self.ctx)
+        self._lr_src = lr_source if on else None
 
     def clear_status(self, stream=None) -> None:
         _check(lib().dpo_muon_clear_status(self.ctx, _stream(stream)), self.ctx)

@@ -409,3 +409,54 @@ def test_muon_checkpoint_resume_after_synchronous_start(cuda_device):
         for m in (straight, split, fresh):
             if m is not None:
                 m.close()
+
+
+def test_muon_capturable_step_replays_in_a_cuda_graph(cuda_device):
+    """Capturable mode: after a 2-call synchronous start, one dpo_muon_step
+    (clipped, EF) captured in a CUDA graph and replayed five times with fresh
+    gradients and a learning rate written between replays equals an eager
+    run bitwise at every call (the device forms the same lr, lr wd and EF
+    start as the host; the Newton-Schulz chain is deterministic)."""
+    shapes = [(256, 512), (300, 700)]
+    kw = dict(ns_steps=1, ef=True, keep_stash=True, max_grad_norm=0.5, device=cuda_device)
+    x0 = [torch.from_numpy(x) for x in inputs(shapes, 0x6A, 1)[0]]
+    eager, cap = muon.DelayedMuon(shapes, x0=x0, **kw), muon.DelayedMuon(shapes, x0=x0, **kw)
+    lr_t = torch.empty(1, dtype=torch.float32, device=cuda_device)
+    lrs = [None] + [2e-3 * (1.0 - 0.05 * i) for i in range(1, 8)]
+
+    def grads(m, k):
+        off = 0
+        for i, (r, c) in enumerate(shapes):
+            synth.dev_normal(0x6A, synth.STREAM_GRAD, k, off, m.grads(i).view(-1), 1e-3)
+            off += r * c
+
+    try:
+        for m in (eager, cap):
+            m.set_delay(0)
+        for k in (1, 2):
+            for m in (eager, cap):
+                grads(m, k)
+                m.step(lrs[k])
+        for m in (eager, cap):
+            m.set_delay(1)
+        cap.set_capturable(True, lr_source=lr_t)
+        torch.cuda.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            cap.step()
+        for k in range(3, 8):
+            grads(eager, k)
+            grads(cap, k)
+            lr_t.fill_(lrs[k])
+            eager.step(lrs[k])
+            graph.replay()
+            torch.cuda.synchronize()
+            for name in muon.DelayedMuon.STATE:
+                assert torch.equal(getattr(eager, name), getattr(cap, name)), (k, name)
+        assert cap.k == eager.k == 7 and cap.phase_start == 2
+        cap.set_capturable(False)
+        assert cap.k == 7
+        assert eager.status() == 0 and cap.status() == 0
+    finally:
+        eager.close()
+        cap.close()
