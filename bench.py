@@ -57,6 +57,9 @@ def parse_args(argv=None):
                    help="muon: delayed Muon (Alg. 2) on the attention and MLP matrices, "
                         "AdamW on the rest")
     p.add_argument("--ns-steps", type=int, default=5, help="Newton-Schulz steps (muon)")
+    p.add_argument("--graph", action="store_true",
+                   help="muon: also time the step captured once in a CUDA graph and replayed "
+                        "(capturable mode)")
     p.add_argument("--no-library-ns", action="store_true",
                    help="muon: skip timing the cuBLAS Newton-Schulz chain for context")
     p.add_argument("--stash", choices=["auto", "copy", "pingpong"], default="auto",
@@ -458,6 +461,29 @@ def run_muon(args, w, world, rank, local):
     gemm_ms, gemm_launches = mo.gemm_time()
     status = mo.status()
     total_s = ev[0].elapsed_time(ev[1]) / 1e3
+    graph = None
+    if args.graph:   # the same step captured once and replayed K times
+        mo.set_timing(False)
+        for o in (ad, mo):
+            o.set_capturable(True, stream=stream)
+        torch.cuda.synchronize(dev)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            ad.step(stream=stream)
+            mo.step(stream=stream)
+        with torch.cuda.stream(stream):
+            for _ in range(2):
+                g.replay()
+            torch.cuda.synchronize(dev)
+            ev[0].record(stream)
+            for _ in range(K):
+                g.replay()
+            ev[1].record(stream)
+        torch.cuda.synchronize(dev)
+        graph = {"ms_per_step": ev[0].elapsed_time(ev[1]) / K,
+                 "what": "the same step (AdamW call + Muon call) captured once in a CUDA graph "
+                         "in capturable mode and replayed"}
+        status |= mo.status()
     value, t_max = aggregate(w.n_params * K, total_s, world, dev)
     achieved = flops * K / (gemm_ms / 1e3) / 1e12
     ws = mo.workspace_bytes()
@@ -469,7 +495,7 @@ def run_muon(args, w, world, rank, local):
     return dict(value=value, t_max=t_max, achieved=achieved, flops=flops, gemm_ms=gemm_ms / K,
                 gemm_launches=gemm_launches, clocks=clocks, launches=K * launches_per_step,
                 n_muon=sum(w.numels[i] for i in mi), n_matrices=len(mi), workspace=ws,
-                device_name=props.name, library=library)
+                device_name=props.name, library=library, graph=graph)
 
 
 def library_ns(shapes, steps: int, dev, reps: int = 3):
@@ -689,6 +715,8 @@ def main_muon(args, w, world, rank, local):
             "config": cfg, "roofline": roof, "cpu_baseline": cpu, "e2e": None,
             "gpu_launches": r["launches"], "clocks": r["clocks"],
             "workspace_bytes": r["workspace"], "device": r["device_name"]}
+    if r["graph"] is not None:
+        line["graph"] = r["graph"]
     print(json.dumps(line), flush=True)
     return 0
 
