@@ -346,6 +346,8 @@ class DelayedAdamW:
         self.sync = list(sync) if sync is not None else [False] * len(numels)
         self.ctx = None
         self._clip_src = None
+        self._capturable = False
+        self._lr_src = None
         self._init(init_mode, stream)
 
     def _init(self, init_mode, stream) -> None:
@@ -361,6 +363,8 @@ class DelayedAdamW:
                             init_mode, stream)
         if self._clip_src is not None:
             dpo_set_clip_source(self.ctx, self._clip_src)
+        if self._capturable:   # a rebuilt context (use_host_io) keeps the mode
+            dpo_set_capturable(self.ctx, True, self._lr_src, stream)
 
     def use_host_io(self, grad: bool = True, param: bool = True, stream=None) -> None:
         """Move the grad and/or bf16 param arenas to pinned host memory (their
@@ -368,7 +372,7 @@ class DelayedAdamW:
         counter and all device state: from then on each step reads its
         gradients from and writes its new weights to host memory directly."""
         torch = self.torch
-        k = self.k
+        k, k0 = self.k, dpo_get_phase_start(self.ctx)
         torch.cuda.synchronize(self.device)
         if param and self.hp.stash_mode == DPO_STASH_PINGPONG:
             # host weights take the copying stash: put both versions in their
@@ -387,6 +391,7 @@ class DelayedAdamW:
             self.param = to_host(self.param)
         self._init(DPO_INIT_RESUME, stream)
         dpo_set_step(self.ctx, k)
+        dpo_set_phase_start(self.ctx, k0)
 
     def view(self, arena, i: int):
         off, cnt = self.layout.offsets[i], self.layout.numels[i]
@@ -442,6 +447,7 @@ class DelayedAdamW:
         ``lr_source``: a one-element float32 device tensor read at every
         step (kept alive here), or None for the lr passed to step()."""
         dpo_set_capturable(self.ctx, on, lr_source, stream)
+        self._capturable = bool(on)
         self._lr_src = lr_source if on else None
 
     def grad_sqnorm(self, acc, stream=None) -> None:

@@ -218,6 +218,26 @@ def test_checkpoint_resume_after_synchronous_start(cuda_device):
         split.close()
 
 
+def test_host_io_switch_keeps_the_delayed_phase(cuda_device):
+    """use_host_io rebuilds the context: the step counter and the start of
+    the delayed phase carry over. Switching right after entering delayed
+    training (synchronous start of two calls) leaves the next call Alg. 1's
+    first delayed iteration: standard rule, EF from the call after."""
+    run = Run(Case(RAGGED, stash_dtype=B, ef=True, schedule={1: 0}), cuda_device)
+    try:
+        for _ in range(2):
+            run.step()
+        run.gpu.set_delay(1)
+        run.ref.set_delay(1)
+        run.gpu.use_host_io()
+        assert run.gpu.k == 2 and dpo.dpo_get_phase_start(run.gpu.ctx) == 2
+        for _ in range(4):
+            run.step()
+            run.assert_close(TOL_RUN)
+    finally:
+        run.close()
+
+
 def test_nonfinite_gradient_flag(cuda_device):
     run = Run(Case([1000, 17], max_grad_norm=1.0), cuda_device)
     try:
