@@ -258,10 +258,10 @@ def wpipe_sync(w, args):
 # ------------------------------------------------------------ CPU oracle --
 
 def oracle_sample_run(w, mode: str, seconds: float, max_steps: int = 1000, n: int = 1 << 22,
-                      rule: dict = None):
+                      rule: dict = None, threads: int = 0):
     """Time the oracle as it stands on the first n parameters of the set
-    (input draws excluded from the timing). Returns (params/s, cores, steps,
-    n)."""
+    (input draws excluded from the timing), on all host cores or on
+    ``threads`` of them. Returns (params/s, cores, steps, n)."""
     import numpy as np
 
     import oracle
@@ -284,16 +284,23 @@ def oracle_sample_run(w, mode: str, seconds: float, max_steps: int = 1000, n: in
                                 stash_store=STORE[w.stash_dtype],
                                 param_store=oracle.BF16 if w.param_dtype == 1 else None)
     gdt = synth.BF16 if w.grad_dtype == 1 else synth.F32
-    spent, steps = 0.0, 0
-    while steps < max_steps and (spent < seconds or steps < 2):
-        g = synth.host_normal(w.seed, synth.STREAM_GRAD, steps + 1, 0, n, W.GRAD_SIGMA, gdt)
-        g = (synth.bf16_bits_to_f32(g) if gdt == synth.BF16 else g).astype(np.float64)
-        sq = oracle.sqnorm(g) if w.max_grad_norm > 0 else None
-        t0 = time.perf_counter()
-        o.step(g, sq=sq)
-        spent += time.perf_counter() - t0
-        steps += 1
-    return n * steps / spent, oracle.num_threads(), steps, n
+    all_cores = oracle.num_threads()
+    if threads:
+        oracle.set_num_threads(threads)
+    try:
+        cores = oracle.num_threads()
+        spent, steps = 0.0, 0
+        while steps < max_steps and (spent < seconds or steps < 2):
+            g = synth.host_normal(w.seed, synth.STREAM_GRAD, steps + 1, 0, n, W.GRAD_SIGMA, gdt)
+            g = (synth.bf16_bits_to_f32(g) if gdt == synth.BF16 else g).astype(np.float64)
+            sq = oracle.sqnorm(g) if w.max_grad_norm > 0 else None
+            t0 = time.perf_counter()
+            o.step(g, sq=sq)
+            spent += time.perf_counter() - t0
+            steps += 1
+    finally:
+        oracle.set_num_threads(all_cores)
+    return n * steps / spent, cores, steps, n
 
 
 # ------------------------------------------------------------------- GPU --
@@ -780,8 +787,12 @@ def main(argv=None):
     if rank == 0 and not args.no_cpu_baseline:
         v, cores, steps, n = oracle_sample_run(w, args.mode, args.cpu_seconds,
                                                rule=rule_settings(args))
+        v1, _, steps1, n1 = oracle_sample_run(w, args.mode, args.cpu_seconds / 3,
+                                              rule=rule_settings(args), n=1 << 20, threads=1)
         cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
-               "sample": f"first {n} params of the set, {steps} oracle steps (plain C, fp64)"}
+               "sample": f"first {n} params of the set, {steps} oracle steps (plain C, fp64)",
+               "single_thread": {"value": v1, "unit": UNIT, "cores": 1,
+                                 "sample": f"first {n1} params, {steps1} oracle steps"}}
     if world > 1:
         torch.distributed.destroy_process_group()
     if rank != 0:

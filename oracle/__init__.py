@@ -99,6 +99,8 @@ def load(path: Optional[str] = None):
     lib.oracle_round_n.argtypes = [ctypes.c_int64, _dp, _dp, ctypes.c_int]
     lib.oracle_num_threads.restype = ctypes.c_int
     lib.oracle_num_threads.argtypes = []
+    lib.oracle_set_num_threads.restype = None
+    lib.oracle_set_num_threads.argtypes = [ctypes.c_int]
     lib.oracle_quadratic.restype = ctypes.c_double
     lib.oracle_quadratic.argtypes = [ctypes.c_int64, _dp, _dp, _dp, _dp,
                                      ctypes.c_int, _dp]
@@ -128,6 +130,10 @@ def _f64(a) -> np.ndarray:
 
 def num_threads(lib=None) -> int:
     return int((lib or load()).oracle_num_threads())
+
+
+def set_num_threads(n: int, lib=None) -> None:
+    (lib or load()).oracle_set_num_threads(int(n))
 
 
 def round_to(x, store: int, lib=None) -> np.ndarray:

@@ -31,6 +31,16 @@ int oracle_num_threads(void)
 #endif
 }
 
+void oracle_set_num_threads(int n)
+{
+#ifdef _OPENMP
+    if (n > 0)
+        omp_set_num_threads(n);
+#else
+    (void)n;
+#endif
+}
+
 /* bf16: 8 significant bits, the exponent range of fp32. Round half to even
  * on the value's own ulp; below 2^-126 the ulp is fixed at 2^-133. */
 static double round_bf16(double x)

@@ -160,6 +160,9 @@ double oracle_clip_coef(double sqnorm, double max_norm);
 
 /* Number of threads the element loops use (OpenMP), 1 without OpenMP. */
 int oracle_num_threads(void);
+/* Set it (n > 0; no effect without OpenMP). Results do not depend on it:
+ * the element loops are independent and the sums run in fixed blocks. */
+void oracle_set_num_threads(int n);
 
 /* Round a value to a storage format (ORACLE_F64 / F32 / BF16). */
 double oracle_round(double x, int store);

@@ -102,3 +102,14 @@ def test_e2e_host_memory_check_counts_every_rank_on_the_node():
     assert bench.e2e_fits(2 * io + (16 << 30), io, 1)
     assert not bench.e2e_fits(2 * io + (16 << 30), io, 2)
     assert bench.e2e_fits(8 * 2 * io + (16 << 30), io, 8)
+
+
+def test_oracle_thread_count_is_settable():
+    import oracle
+    n = oracle.num_threads()
+    oracle.set_num_threads(1)
+    try:
+        assert oracle.num_threads() == 1
+    finally:
+        oracle.set_num_threads(n)
+    assert oracle.num_threads() == n
