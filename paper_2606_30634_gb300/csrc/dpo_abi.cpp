@@ -207,6 +207,11 @@ bool dc_on(const dpo_ctx *c)
 //   AdamW, NAdam, Lion       4                     3
 //   Adan                     3                     3
 //   SAPipe updated state     -                     4
+//   Lion, ping-pong stash    4                     5
+// the same with the copying and the ping-pong stash, except Lion with an
+// update history: without the stash store its packets carry too few bytes
+// for three CTAs to fill the memory system (ping-pong: 3 CTAs 85.2%, 4 95.0%,
+// 5 99.0%, 6 96.6% of the copy peak; copying stash: 3 CTAs 98.0%).
 // Three CTAs where packets also carry the history buffer keep about 55 KiB
 // of loads in flight per SM; the standard rule loads less per packet and
 // wants a fourth; Adan's two extra state streams make three enough; the
@@ -234,6 +239,8 @@ int set_step_grid(dpo_ctx *c)
         want = 4;
     else if (c->hp.optimizer == DPO_OPT_ADAN)
         want = 3;
+    else if (c->hp.optimizer == DPO_OPT_LION && pingpong_on(c) && mostly_hist)
+        want = 5;
     else
         want = mostly_hist ? 3 : 4;
     c->step_grid = grid_of(c, std::min(per_sm, want), dpo::kStepThreads);
