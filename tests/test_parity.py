@@ -301,6 +301,20 @@ def test_launch_geometry_is_persistent(cuda_device):
         run.close()
 
 
+@pytest.mark.parametrize("stash_mode,per_sm", [(dpo.DPO_STASH_PINGPONG, 5), (dpo.DPO_STASH_COPY, 3)])
+def test_launch_geometry_lion_with_history(cuda_device, stash_mode, per_sm):
+    """The measured grid table: Lion with an update history takes five CTAs
+    per SM under the ping-pong stash, three with the copying stash."""
+    run = Run(Case([5_000_000, 123], stash_dtype=B, ef=True, optimizer=dpo.DPO_OPT_LION,
+                   stash_mode=stash_mode), cuda_device)
+    try:
+        steps, _, _ = dpo.dpo_launch_config(run.gpu.ctx)
+        sms = torch.cuda.get_device_properties(cuda_device).multi_processor_count
+        assert steps == per_sm * sms
+    finally:
+        run.close()
+
+
 @pytest.mark.parametrize("host_grad,host_param", [(True, True), (True, False), (False, True)])
 def test_host_io_parity(cuda_device, host_grad, host_param):
     """Gradients read from and/or bf16 weights written to pinned host memory
