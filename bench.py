@@ -773,7 +773,12 @@ def main(argv=None):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     r = run_gpu(args, w, world, rank, local)
     peak, peak_kind = measured_hbm_peak()
-    kernel_tag = f"fused_step:{w.name}:{args.mode}" + (":pingpong" if args.stash == "pingpong" else "")
+    # the tag names every setting that changes the kernel's traffic; the
+    # headline keeps "fused_step:<set>:<mode>[:pingpong]"
+    variant = [x for x in (args.optimizer if args.optimizer != "adamw" else None,
+                           "dc" if args.dc_lambda else None, "wpipe" if args.wpipe else None) if x]
+    kernel_tag = (f"fused_step:{w.name}:{args.mode}" + "".join(":" + v for v in variant) +
+                  (":pingpong" if args.stash == "pingpong" else ""))
     traffic = committed_traffic(kernel_tag)
     kernels = "fused_step_kernel" if w.max_grad_norm <= 0 else "grad_sqnorm_kernel+fused_step_kernel"
     roof = {"bound": "hbm", "achieved": r["achieved"], "peak": peak, "unit": "GB/s",

@@ -113,3 +113,11 @@ def test_oracle_thread_count_is_settable():
     finally:
         oracle.set_num_threads(n)
     assert oracle.num_threads() == n
+
+
+def test_committed_traffic_is_per_kernel_variant():
+    """The committed headline summary's figure serves the headline only, not
+    another rule or mode that runs a different kernel instance."""
+    import bench
+    assert bench.committed_traffic("fused_step:llama-7B:ef:lion:pingpong") is None
+    assert bench.committed_traffic("fused_step:llama-7B:ef:dc:pingpong") is None
