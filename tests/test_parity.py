@@ -238,6 +238,29 @@ def test_host_io_switch_keeps_the_delayed_phase(cuda_device):
         run.close()
 
 
+def test_lion_zero_gradient_moves_only_by_decay(cuda_device):
+    """Lion's sign(0) = 0 on the GPU as in the oracle: a zero gradient from
+    the zero start state leaves the update at the decay term alone, so every
+    weight matches the oracle's x (1 - lr wd) path, decayed and undecayed
+    tensors alike."""
+    case = Case([4096, 77, 300_001], optimizer=dpo.DPO_OPT_LION, stash_dtype=B,
+                wd_on=[True, False, True])
+    run = Run(case, cuda_device)
+    try:
+        x0 = run.gather(run.gpu.master).astype(np.float64)
+        run.gpu.grad.zero_()
+        run.gpu.step()
+        run.ref.step(np.zeros(run.idx.size), tag=run.ref.read_weights("stale")[1])
+        torch.cuda.synchronize()
+        run.assert_close(TOL_ONE_STEP)
+        got = run.gather(run.gpu.master).astype(np.float64)
+        moved = got != x0
+        assert not moved[4096:4096 + 77].any()        # no decay: untouched
+        assert moved[:4096].mean() > 0.99             # decay: x (1 - lr wd)
+    finally:
+        run.close()
+
+
 def test_nonfinite_gradient_flag(cuda_device):
     run = Run(Case([1000, 17], max_grad_norm=1.0), cuda_device)
     try:
