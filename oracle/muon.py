@@ -100,7 +100,9 @@ class DelayedMuon:
     the gradient evaluated at the stash and leaves the stash at X_k. Clipping
     takes the global norm over all matrices.
 
-    ``delayed`` marks per matrix whether it takes delayed updates (default
+    ``wd_on`` marks per matrix whether its update decays X_t (default all;
+    embeddings and norms commonly go without). ``delayed`` marks per matrix
+    whether it takes delayed updates (default
     all; a synchronous matrix has no stash write and no correction, as WPipe
     and the synchronous LM head train part of the model). ``set_delay``
     switches the whole run between synchronous and delayed training
@@ -115,6 +117,7 @@ class DelayedMuon:
     param_store: Optional[int] = None
     lib: object = None
     delayed: Optional[Sequence[bool]] = None
+    wd_on: Optional[Sequence[bool]] = None
 
     def __post_init__(self):
         self.lib = self.lib or load()
@@ -161,7 +164,8 @@ class DelayedMuon:
         h = self.hp
         for i, (rows, cols) in enumerate(self.shapes):
             dly = self.delay if self.delayed is None or self.delayed[i] else 0
-            hp = _MuonHParams(lr if lr is not None else h.lr, h.momentum, h.weight_decay,
+            wd = h.weight_decay if self.wd_on is None or self.wd_on[i] else 0.0
+            hp = _MuonHParams(lr if lr is not None else h.lr, h.momentum, wd,
                               h.ef_lambda, h.ns_a, h.ns_b, h.ns_c, h.ns_steps, h.ns_eps,
                               h.rms_scale, h.ns_store, dly, h.correction, self.x_store,
                               self.stash_store,

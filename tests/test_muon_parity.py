@@ -61,7 +61,7 @@ class Pair:
 
     def __init__(self, shapes, device, seed=0x3A0, ns_steps=5, ef=True, delay=1, sdt=B,
                  lr=2e-3, momentum=0.95, wd=0.1, max_grad_norm=0.0, rms_scale=0.2, sync=None,
-                 schedule=None, correction=0, gdt=B):
+                 schedule=None, correction=0, gdt=B, wd_on=None):
         self.shapes, self.seed, self.lr = shapes, seed, lr
         self.schedule = schedule or {}
         xs, _ = inputs(shapes, seed, 1)
@@ -71,7 +71,7 @@ class Pair:
                                     max_grad_norm=max_grad_norm, rms_scale=rms_scale,
                                     ns_steps=ns_steps, delay=delay, device=device,
                                     x0=[torch.from_numpy(x) for x in xs], sync=sync,
-                                    keep_stash=True, correction=correction)
+                                    keep_stash=True, correction=correction, wd_on=wd_on)
         hp = MuonHParams(lr=lr, momentum=momentum, weight_decay=wd, ef_lambda=1.0,
                          ns_steps=ns_steps, rms_scale=rms_scale, ns_store=oracle.BF16,
                          max_grad_norm=max_grad_norm, delay=delay,
@@ -79,7 +79,8 @@ class Pair:
         self.ref = OracleMuon([x.astype(np.float64) for x in xs], hp, ef=ef, x_store=oracle.F32,
                               stash_store=oracle.BF16 if sdt == B else oracle.F32,
                               param_store=oracle.BF16,
-                              delayed=None if sync is None else [not q for q in sync])
+                              delayed=None if sync is None else [not q for q in sync],
+                              wd_on=wd_on)
         self.sync = sync or [False] * len(shapes)
         self.k = 0
 
@@ -460,3 +461,19 @@ def test_muon_capturable_step_replays_in_a_cuda_graph(cuda_device):
     finally:
         eager.close()
         cap.close()
+
+
+def test_muon_weight_decay_mask_parity(cuda_device):
+    """Per-matrix decay (DPO_WD_ON): matrices without it take U = lr r O
+    only; three calls against the oracle with the same mask."""
+    wd_on = [i % 2 == 0 for i in range(len(SHAPES))]
+    p = Pair(SHAPES, cuda_device, ns_steps=1, ef=True, wd_on=wd_on)
+    r_max = 0.2 * np.sqrt(max(max(sh) for sh in SHAPES))
+    du = p.lr * r_max * 2.0 ** -7
+    try:
+        for k in range(3):
+            p.step()
+            close_with_flips(p.cat(p.gpu.master), _flat(p.ref.x), TOL_RUN, (k + 1) * du, 1e-3)
+            close_with_flips(p.cat(p.gpu.ef), _flat(p.ref.u_prev), 1e-5, du, 2e-3)
+    finally:
+        p.close()

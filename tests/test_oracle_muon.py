@@ -329,3 +329,22 @@ def test_muon_sapipe_prediction_rounds_through_the_master(lib):
     opt.u_prev[0][...] = -(2.0 ** -30)
     opt.step([np.ones((2, 2))])
     assert np.all(opt.stash[0] == 1.0)
+
+
+def test_muon_weight_decay_mask(lib):
+    """A matrix without decay is the same run as a context whose decay is
+    zero, bitwise; the decayed matrix beside it is unchanged by the mask."""
+    rng = np.random.default_rng(31)
+    xa, xb = rng.normal(size=(4, 6)), rng.normal(size=(5, 3))
+    grads = [[rng.normal(size=(4, 6)), rng.normal(size=(5, 3))] for _ in range(3)]
+    mixed = DelayedMuon([xa, xb], _hp(), ef=True, x_store=F64, stash_store=F64, lib=lib,
+                        wd_on=[True, False])
+    decayed = DelayedMuon([xa], _hp(), ef=True, x_store=F64, stash_store=F64, lib=lib)
+    plain = DelayedMuon([xb], _hp(weight_decay=0.0), ef=True, x_store=F64, stash_store=F64,
+                        lib=lib)
+    for ga, gb in grads:
+        mixed.step([ga, gb])
+        decayed.step([ga])
+        plain.step([gb])
+    assert np.array_equal(mixed.x[0], decayed.x[0])
+    assert np.array_equal(mixed.x[1], plain.x[0])
