@@ -269,6 +269,20 @@ def test_muon_clipping(cuda_device):
         p.close()
 
 
+def test_muon_without_rms_scaling(cuda_device):
+    """rms_scale = 0: Alg. 2 as printed, U = lr (O + wd X_t), no
+    0.2 sqrt(max(r, c)) factor; two calls against the oracle."""
+    p = Pair(SHAPES, cuda_device, ns_steps=1, ef=True, rms_scale=0.0)
+    du = p.lr * 2.0 ** -7
+    try:
+        for k in range(2):
+            p.step()
+            close_with_flips(p.cat(p.gpu.master), _flat(p.ref.x), TOL_RUN, (k + 1) * du, 1e-3)
+            close_with_flips(p.cat(p.gpu.ef), _flat(p.ref.u_prev), 1e-5, du, 2e-3)
+    finally:
+        p.close()
+
+
 def test_muon_flops_and_workspace(cuda_device):
     shapes = [(256, 512), (512, 256), (300, 700)]
     m = muon.DelayedMuon(shapes, ns_steps=5, device=cuda_device)
