@@ -348,3 +348,33 @@ def test_muon_weight_decay_mask(lib):
         plain.step([gb])
     assert np.array_equal(mixed.x[0], decayed.x[0])
     assert np.array_equal(mixed.x[1], plain.x[0])
+
+
+def test_muon_stored_state_is_in_its_storage_format(lib):
+    """Muon's buffers hold values of their storage formats after each call:
+    master, momentum and the EF history in fp32, stash and weights in
+    bf16."""
+    rng = np.random.default_rng(43)
+    x0 = rng.normal(0, 0.02, (6, 10))
+    opt = DelayedMuon([x0], _hp(ef_lambda=1.0, ns_store=BF16), ef=True, x_store=F32,
+                      stash_store=BF16, param_store=BF16, lib=lib)
+    f32 = lambda a: np.array_equal(np.asarray(a).astype(np.float32).astype(np.float64), a)
+    bf16 = lambda a: f32(a) and not np.any(np.asarray(a, np.float32).view(np.uint32) & 0xFFFF)
+    for _ in range(3):
+        opt.step([rng.normal(0, 1e-3, (6, 10))])
+        assert f32(opt.x[0]) and f32(opt.mom[0]) and f32(opt.u_prev[0])
+        assert bf16(opt.stash[0]) and bf16(opt.param[0])
+
+
+def test_muon_weights_round_the_stored_master(lib):
+    """As for the elementwise rules: a 1 x 1 matrix, no Newton-Schulz steps
+    and eps 0 give O = sign(M) = -1, so with lr = 2^-30, no decay and no RMS
+    scaling X_1 = 1 + 2^-8 + 2^-30, stored in fp32 as the bf16 tie 1 + 2^-8;
+    the bf16 weights are then 1.0, not 1 + 2^-7."""
+    opt = DelayedMuon([np.array([[1.0 + 2.0 ** -8]])],
+                      _hp(lr=2.0 ** -30, weight_decay=0.0, rms_scale=0.0, ns_steps=0,
+                          ns_eps=0.0, ns_store=F64), x_store=F32, stash_store=F32,
+                      param_store=BF16, lib=lib)
+    opt.step([np.array([[-1.0]])])
+    assert opt.x[0][0, 0] == 1.0 + 2.0 ** -8
+    assert opt.param[0][0, 0] == 1.0

@@ -97,6 +97,27 @@ MUTANTS = [
     ("muon_sapipe_prediction_rounded_once",
      "oracle_round(oracle_round(x[i] - u_prev[i], hp->x_store), hp->stash_store)",
      "oracle_round(x[i] - u_prev[i], hp->stash_store)"),
+    ("bf16_weights_from_unrounded_update",
+     "        x[i] = oracle_round(xn, hp->x_store);\n        if (param != NULL)\n"
+     "            param[i] = oracle_round(x[i], hp->param_store);\n    }\n    return 0;\n}",
+     "        x[i] = oracle_round(xn, hp->x_store);\n        if (param != NULL)\n"
+     "            param[i] = oracle_round(xn, hp->param_store);\n    }\n    return 0;\n}"),
+    ("history_not_stored_in_fp32", "            u_prev[i] = oracle_round(hist, hp->x_store);",
+     "            u_prev[i] = hist;"),
+    ("muon_master_not_stored_in_fp32",
+     "        x[i] = oracle_round(xn, hp->x_store);\n        if (param != NULL)\n"
+     "            param[i] = oracle_round(x[i], hp->param_store);\n    }\n    if (o_out",
+     "        x[i] = xn;\n        if (param != NULL)\n"
+     "            param[i] = oracle_round(x[i], hp->param_store);\n    }\n    if (o_out"),
+    ("muon_momentum_not_stored_in_fp32",
+     "        mom[i] = oracle_round(hp->momentum * mom[i] + (1.0 - hp->momentum) * (clip_scale * g[i]),"
+     "\n                              hp->x_store);",
+     "        mom[i] = hp->momentum * mom[i] + (1.0 - hp->momentum) * (clip_scale * g[i]);"),
+    ("muon_bf16_weights_from_unrounded_update",
+     "        x[i] = oracle_round(xn, hp->x_store);\n        if (param != NULL)\n"
+     "            param[i] = oracle_round(x[i], hp->param_store);\n    }\n    if (o_out",
+     "        x[i] = oracle_round(xn, hp->x_store);\n        if (param != NULL)\n"
+     "            param[i] = oracle_round(xn, hp->param_store);\n    }\n    if (o_out"),
 ]
 
 

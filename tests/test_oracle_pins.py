@@ -855,3 +855,44 @@ def test_sapipe_prediction_is_a_master_weight_rounded_to_the_stash(lib):
     o.step(np.array([0.5]), tag=o.read_weights()[1])
     assert o.stash[0] == 1.0
     assert o.x[0] == 1.0 + 2.0 ** -8
+
+
+def _fp32_exact(a):
+    a = np.asarray(a, dtype=np.float64)
+    return np.array_equal(a.astype(np.float32).astype(np.float64), a)
+
+
+def _bf16_exact(a):
+    a = np.asarray(a, dtype=np.float64)
+    bits = a.astype(np.float32).view(np.uint32)
+    return _fp32_exact(a) and not np.any(bits & 0xFFFF)
+
+
+def test_stored_state_is_in_its_storage_format(lib):
+    """Every buffer holds values of its own storage format after each call
+    (the oracle rounds each stored quantity once, as the device stores it):
+    master, m, v and the EF history in fp32, the stash and the bf16 weights
+    in bf16."""
+    rng = np.random.default_rng(41)
+    x0 = rng.normal(0, 0.02, 300)
+    o = oracle.DelayedOptimizer([x0], HParams(lr=1e-3, ef_lambda=1.0).as_f32(), ef=True,
+                                x_store=F32, stash_store=BF16, param_store=BF16, lib=lib)
+    for _ in range(4):
+        o.step(rng.normal(0, 1e-3, 300), tag=o.read_weights()[1])
+        assert _fp32_exact(o.x) and _fp32_exact(o.m) and _fp32_exact(o.v)
+        assert _fp32_exact(o.u_prev)
+        assert _bf16_exact(o.stash) and _bf16_exact(o.param)
+
+
+def test_bf16_weights_round_the_stored_master(lib):
+    """The bf16 weights are the stored fp32 master rounded to bf16 (a5): two
+    roundings from the update's exact result. x_0 = 1 + 2^-8, SGD rule with
+    u = -2^-30: x_1 = 1 + 2^-8 + 2^-30, stored in fp32 as 1 + 2^-8 (a bf16
+    tie), so the bf16 copy is 1.0; rounding the exact result once would give
+    1 + 2^-7."""
+    hp = HParams(lr=1.0, weight_decay=0.0, rule=oracle.RULE_SGD, delay=0)
+    o = oracle.DelayedOptimizer([np.array([1.0 + 2.0 ** -8])], hp, x_store=F32,
+                                stash_store=F32, param_store=BF16, lib=lib)
+    o.step(np.array([-(2.0 ** -30)]), tag=o.read_weights()[1])
+    assert o.x[0] == 1.0 + 2.0 ** -8
+    assert o.param[0] == 1.0
