@@ -113,12 +113,46 @@ MUTANTS = [
      "        mom[i] = oracle_round(hp->momentum * mom[i] + (1.0 - hp->momentum) * (clip_scale * g[i]),"
      "\n                              hp->x_store);",
      "        mom[i] = hp->momentum * mom[i] + (1.0 - hp->momentum) * (clip_scale * g[i]);"),
+    ("adan_previous_gradient_unclipped", "g_prev[i] = oracle_round(gi, hp->x_store);",
+     "g_prev[i] = oracle_round(g[i], hp->x_store);"),
+    ("nadam_gradient_term_unclipped", "(1.0 - mu_k) / (1.0 - mu_prod) * gi / d",
+     "(1.0 - mu_k) / (1.0 - mu_prod) * g[i] / d"),
+    ("lion_blend_unclipped", "const double c = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;",
+     "const double c = hp->beta1 * m[i] + (1.0 - hp->beta1) * g[i];"),
+    ("sapipe_updated_blend_unclipped", "const double m2 = hp->beta1 * mi + (1.0 - hp->beta1) * gi;",
+     "const double m2 = hp->beta1 * mi + (1.0 - hp->beta1) * g[i];"),
+    ("synchronous_tensor_stash_written", "        if (delayed) {\n            if (corr == ORACLE_CORR_EF)",
+     "        if (hp->delay == 1) {\n            if (corr == ORACLE_CORR_EF)"),
+    ("lion_sign_after_momentum_update",
+     "            const double c = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;\n"
+     "            const double sgn = c > 0.0 ? 1.0 : (c < 0.0 ? -1.0 : 0.0);\n"
+     "            u = hp->lr * (sgn + wd * xt);\n"
+     "            m[i] = oracle_round(hp->beta2 * m[i] + (1.0 - hp->beta2) * gi, hp->x_store);",
+     "            m[i] = oracle_round(hp->beta2 * m[i] + (1.0 - hp->beta2) * gi, hp->x_store);\n"
+     "            const double c = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;\n"
+     "            const double sgn = c > 0.0 ? 1.0 : (c < 0.0 ? -1.0 : 0.0);\n"
+     "            u = hp->lr * (sgn + wd * xt);"),
     ("muon_bf16_weights_from_unrounded_update",
      "        x[i] = oracle_round(xn, hp->x_store);\n        if (param != NULL)\n"
      "            param[i] = oracle_round(x[i], hp->param_store);\n    }\n    if (o_out",
      "        x[i] = oracle_round(xn, hp->x_store);\n        if (param != NULL)\n"
      "            param[i] = oracle_round(xn, hp->param_store);\n    }\n    if (o_out"),
 ]
+
+
+def _dc_before_clip():
+    """The DC-ASGD compensation applied to the raw gradient, then clipped."""
+    src = open(oracle_build.SRC).read()
+    i = src.index("        double gi = clip_scale * g[i];\n")
+    tail = "gi = gi + hp->dc_lambda * gi * gi * (xt - stash[i]);"
+    j = src.index(tail) + len(tail)
+    old = src[i:j]
+    new = old.replace("double gi = clip_scale * g[i];", "double gi = g[i];") + \
+        "\n        gi = clip_scale * gi;"
+    return ("dc_compensates_the_raw_gradient", old, new)
+
+
+MUTANTS.append(_dc_before_clip())
 
 
 def _build_mutant(tmp_path, name, old, new):

@@ -459,12 +459,12 @@ def test_quadratic_gradient_is_loss_derivative(lib):
 # ------------------------------------------------------- SAPipe-WP (App. B.1)
 
 def _fixed_grad_run(lib, correction, steps=8, wd=0.1, ef=True, lam=1.0, beta=(0.9, 0.95),
-                    eps=1e-8, n=64, seed=21):
+                    eps=1e-8, n=64, seed=21, max_norm=0.0):
     rng = np.random.default_rng(seed)
     x0 = rng.normal(0, 0.5, n)
     grads = [rng.normal(0, 1.0, n) for _ in range(steps)]
     hp = HParams(lr=0.01, beta1=beta[0], beta2=beta[1], eps=eps, weight_decay=wd,
-                 ef_lambda=lam, correction=correction)
+                 ef_lambda=lam, correction=correction, max_grad_norm=max_norm)
     o = oracle.DelayedOptimizer([x0], hp, ef=ef, x_store=F64, stash_store=F64, lib=lib)
     hist = []
     for g in grads:
@@ -500,11 +500,16 @@ def test_sapipe_same_prediction_points_move_like_ef(lib):
             np.testing.assert_allclose(d_stash, d_ef, rtol=1e-11, atol=1e-15)
 
 
-def test_sapipe_updated_prediction_is_adamw_stepped_again(lib):
+@pytest.mark.parametrize("max_norm", [0.0, 3.0])
+def test_sapipe_updated_prediction_is_adamw_stepped_again(lib, max_norm):
     """The updated-state prediction update is what torch.optim.AdamW applies
     when stepped once more on the same gradient from the state its real step
-    left (then discarded)."""
-    hist, grads, x0, hp = _fixed_grad_run(lib, oracle.CORR_SAPIPE_UPDATED)
+    left (then discarded); with clipping (norms about 8 against 3), on the
+    same clipped gradient the real step consumed."""
+    hist, grads, x0, hp = _fixed_grad_run(lib, oracle.CORR_SAPIPE_UPDATED, max_norm=max_norm)
+    clip = lambda g: g * (min(1.0, max_norm / (np.sqrt(np.sum(g * g)) + 1e-6))
+                          if max_norm > 0 else 1.0)
+    grads = [clip(g) for g in grads]
     p = torch.nn.Parameter(torch.tensor(x0))
     opt = torch.optim.AdamW([p], lr=hp.lr, betas=(hp.beta1, hp.beta2), eps=hp.eps,
                             weight_decay=hp.weight_decay, foreach=False, fused=False)
@@ -674,8 +679,8 @@ def f64_default():
 
 
 @pytest.mark.parametrize("delay", [0, 1])
-@pytest.mark.parametrize("psi", [0.004, 0.02])
-def test_nadam_matches_torch(lib, f64_default, delay, psi):
+@pytest.mark.parametrize("psi,max_norm", [(0.004, 0.0), (0.02, 0.0), (0.004, 1.5)])
+def test_nadam_matches_torch(lib, f64_default, delay, psi, max_norm):
     """NAdam = torch.optim.NAdam with decoupled weight decay, including its
     momentum schedule mu_k = beta1 (1 - 0.5 * 0.96^(k psi)), changing lr."""
     rng = np.random.default_rng(12)
@@ -687,11 +692,13 @@ def test_nadam_matches_torch(lib, f64_default, delay, psi):
     opt = torch.optim.NAdam(ps, lr=lrs[0], betas=(0.9, 0.95), eps=1e-8, weight_decay=0.1,
                             momentum_decay=psi, decoupled_weight_decay=True, foreach=False)
     hp = HParams(lr=lrs[0], weight_decay=0.1, delay=delay, rule=oracle.RULE_NADAM,
-                 momentum_decay=psi)
+                 momentum_decay=psi, max_grad_norm=max_norm)
     o = oracle.DelayedOptimizer(x0s, hp, x_store=F64, stash_store=F64, lib=lib)
     for gs, lr in zip(grads, lrs):
         for p, g in zip(ps, gs):
             p.grad = torch.tensor(g)
+        if max_norm > 0:   # the clipped gradient enters every term
+            torch.nn.utils.clip_grad_norm_(ps, max_norm)
         for group in opt.param_groups:
             group["lr"] = lr
         opt.step()
@@ -896,3 +903,74 @@ def test_bf16_weights_round_the_stored_master(lib):
     o.step(np.array([-(2.0 ** -30)]), tag=o.read_weights()[1])
     assert o.x[0] == 1.0 + 2.0 ** -8
     assert o.param[0] == 1.0
+
+
+def test_dc_asgd_compensates_the_clipped_gradient(lib):
+    """Reading 20: the clip coefficient scales the gradient that arrived and
+    the compensation corrects the consumed one, so g~ = s g + lambda (s g)^2
+    (x_t - stash). beta1 = 0 makes the first moment exactly g~."""
+    lam = 50.0
+    hp = HParams(lr=0.1, beta1=0.0, beta2=0.95, eps=1e-8, weight_decay=0.0, dc_lambda=lam,
+                 max_grad_norm=1.0)
+    o = oracle.DelayedOptimizer([np.array([1.0])], hp, x_store=F64, stash_store=F64, lib=lib)
+    o.step(np.array([2.0]), tag=o.read_weights()[1])
+    x2, x1 = o.x[0], o.stash[0]
+    o.step(np.array([3.0]), tag=o.read_weights()[1])
+    gh = 3.0 / (3.0 + 1e-6)
+    assert o.m[0] == pytest.approx(gh + lam * gh * gh * (x2 - x1), rel=1e-13)
+
+
+def test_adan_previous_gradient_is_the_consumed_one(lib):
+    """Reading 19: Adan's stored previous gradient is the one consumed,
+    clipped; its difference at the next call is taken between consumed
+    gradients."""
+    hp = HParams(lr=0.01, rule=oracle.RULE_ADAN, max_grad_norm=1.0)
+    g = np.array([3.0, -4.0])
+    o = oracle.DelayedOptimizer([np.array([0.5, 0.25])], hp, x_store=F64, stash_store=F64,
+                                lib=lib)
+    o.step(g, tag=o.read_weights()[1])
+    np.testing.assert_allclose(o.g_prev, g * (1.0 / (5.0 + 1e-6)), rtol=1e-15)
+
+
+def test_lion_blends_the_clipped_gradient(lib):
+    """Lion's sign takes the interpolation of m and the consumed (clipped)
+    gradient. beta = (0.99, 0.5), clip at 1, gradients 1 then -100: the
+    clipped second gradient is -1, so c = 0.99 * 0.5 - 0.01 > 0 and the
+    weight keeps moving down (1 -> 0.9 -> 0.8); the raw -100 would flip the
+    sign and move it back up."""
+    hp = HParams(lr=0.1, beta1=0.99, beta2=0.5, weight_decay=0.0, rule=oracle.RULE_LION,
+                 max_grad_norm=1.0)
+    o = oracle.DelayedOptimizer([np.array([1.0])], hp, x_store=F64, stash_store=F64, lib=lib)
+    xs = []
+    for g in (1.0, -100.0):
+        o.step(np.array([g]), tag=o.read_weights()[1])
+        xs.append(o.x[0])
+    assert xs == pytest.approx([0.9, 0.8], abs=1e-15)
+
+
+def test_lion_sign_before_the_momentum_update(lib):
+    """Lion takes the sign of beta1 m_{t-1} + (1 - beta1) g before m moves to
+    its beta2 average. beta = (0.5, 0): after g = 1 (m = 1), g = -0.5 gives
+    c = 0.5 - 0.25 > 0 (down again, 0.9 -> 0.8); the updated m (-0.5) would
+    give c < 0."""
+    hp = HParams(lr=0.1, beta1=0.5, beta2=0.0, weight_decay=0.0, rule=oracle.RULE_LION)
+    o = oracle.DelayedOptimizer([np.array([1.0])], hp, x_store=F64, stash_store=F64, lib=lib)
+    xs = []
+    for g in (1.0, -0.5):
+        o.step(np.array([g]), tag=o.read_weights()[1])
+        xs.append(o.x[0])
+    assert xs == pytest.approx([0.9, 0.8], abs=1e-15)
+
+
+def test_synchronous_tensor_stash_untouched(lib):
+    """A tensor trained synchronously (App. B.2) has no stale version: its
+    stash is never written while the delayed tensor beside it rotates."""
+    rng = np.random.default_rng(51)
+    xa, xb = rng.normal(0, 1, 5), rng.normal(0, 1, 4)
+    o = oracle.DelayedOptimizer([xa, xb], HParams(lr=0.05, ef_lambda=1.0), ef=True,
+                                x_store=F64, stash_store=F64, delayed=[True, False], lib=lib)
+    s0 = o.stash.copy()
+    for _ in range(3):
+        o.step(rng.normal(0, 1, 9))
+    assert np.array_equal(o.stash[5:], s0[5:])
+    assert not np.array_equal(o.stash[:5], s0[:5])

@@ -566,14 +566,17 @@ def test_rule_parity(cuda_device, rule, ef, corr, pdt, sdt, gdt):
         run.close()
 
 
-def test_dc_asgd_parity_multistep(cuda_device):
+@pytest.mark.parametrize("clip", [0.0, 0.3])
+def test_dc_asgd_parity_multistep(cuda_device, clip):
     """DC-ASGD's Taylor compensation (Sec. 3.1) with EF over six steps, at
-    lambda = 1e4 with an fp32 stash. The term multiplies x_t - stash by
-    lambda g^2, so at larger lambda (the paper sweeps up to 1e8) a one-rounding
-    difference between the two sides' master or stash, allowed by the fp32
-    and bf16 bars, is amplified into the gradient: there the step is checked
-    on identical inputs instead (next test)."""
-    run = Run(Case(RAGGED, stash_dtype=F, ef=True, dc_lambda=1e4), cuda_device)
+    lambda = 1e4 with an fp32 stash, with and without clipping (the
+    compensation then corrects the clipped gradient). The term multiplies
+    x_t - stash by lambda g^2, so at larger lambda (the paper sweeps up to
+    1e8) a one-rounding difference between the two sides' master or stash,
+    allowed by the fp32 and bf16 bars, is amplified into the gradient: there
+    the step is checked on identical inputs instead (next test)."""
+    run = Run(Case(RAGGED, stash_dtype=F, ef=True, dc_lambda=1e4, max_grad_norm=clip),
+              cuda_device)
     try:
         for k in range(1, 7):
             run.step()
