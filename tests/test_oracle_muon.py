@@ -378,3 +378,28 @@ def test_muon_weights_round_the_stored_master(lib):
     opt.step([np.array([[-1.0]])])
     assert opt.x[0][0, 0] == 1.0 + 2.0 ** -8
     assert opt.param[0][0, 0] == 1.0
+
+
+@pytest.mark.parametrize("steps", [1, 2, 3])
+@pytest.mark.parametrize("tall", [False, True])
+def test_newton_schulz_bf16_restated_exactly(lib, steps, tall):
+    """An independent restatement of the bf16 iteration (numpy products,
+    torch's bf16 rounding) on inputs where every fp64 operation is exact: a
+    2 x 8 matrix of +-1 entries (||M||_F = 4, X_0 = M / 4 exact with eps 0,
+    each product a sum of few short-mantissa terms). The iteration runs on
+    the orientation with the smaller Gram matrix (2 x 2), for the matrix and
+    for its 8 x 2 transpose; the oracle must agree bitwise."""
+    import torch
+    rng = np.random.default_rng(61)
+    Mw = rng.choice([-1.0, 1.0], size=(2, 8))
+    M = Mw.T.copy() if tall else Mw
+    bf = lambda x: torch.tensor(x, dtype=torch.float64).to(torch.bfloat16).double().numpy()
+    a, b, c = NS_COEFFS
+    X = bf(Mw / 4.0)
+    for _ in range(steps):
+        A = bf(X @ X.T)
+        B = bf(b * A + c * (A @ A))
+        X = bf(a * X + B @ X)
+    want = X.T if tall else X
+    got = newton_schulz(M, steps=steps, store=BF16, eps=0.0, lib=lib)
+    assert np.array_equal(got, want)

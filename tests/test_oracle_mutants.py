@@ -132,6 +132,14 @@ MUTANTS = [
      "            const double c = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;\n"
      "            const double sgn = c > 0.0 ? 1.0 : (c < 0.0 ? -1.0 : 0.0);\n"
      "            u = hp->lr * (sgn + wd * xt);"),
+    ("ns_on_the_larger_gram_matrix", "const int tall = rows > cols;",
+     "const int tall = rows < cols;"),
+    ("quadratic_gradient_unrounded",
+     "grad_out[i] = oracle_round(a[i] * d + (noise ? noise[i] : 0.0), store);",
+     "grad_out[i] = a[i] * d + (noise ? noise[i] : 0.0);"),
+    ("quadratic_noise_dropped",
+     "grad_out[i] = oracle_round(a[i] * d + (noise ? noise[i] : 0.0), store);",
+     "grad_out[i] = oracle_round(a[i] * d, store);"),
     ("muon_bf16_weights_from_unrounded_update",
      "        x[i] = oracle_round(xn, hp->x_store);\n        if (param != NULL)\n"
      "            param[i] = oracle_round(x[i], hp->param_store);\n    }\n    if (o_out",

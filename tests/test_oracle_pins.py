@@ -456,6 +456,38 @@ def test_quadratic_gradient_is_loss_derivative(lib):
     assert loss == pytest.approx(0.5 * np.sum(a * (w - ws) ** 2), rel=1e-14)
 
 
+def test_quadratic_noise_enters_the_gradient(lib):
+    """With a noise sample, the harness's gradient is the loss derivative
+    (central differences, the noise is not part of the loss) plus that
+    sample: the stale-gradient noise of the quadratic workload."""
+    rng = np.random.default_rng(16)
+    n = 12
+    a = np.exp(rng.uniform(np.log(1e-3), 0, n))
+    ws, w, noise = rng.normal(0, 1, n), rng.normal(0, 1, n), rng.normal(0, 1e-2, n)
+    g, _ = oracle.quadratic(a, ws, w, noise, F64, lib=lib)
+    h = 1e-6
+    for i in range(n):
+        e = np.zeros(n)
+        e[i] = h
+        lp = oracle.quadratic(a, ws, w + e, None, F64, lib=lib)[1]
+        lm = oracle.quadratic(a, ws, w - e, None, F64, lib=lib)[1]
+        assert g[i] - (lp - lm) / (2 * h) == pytest.approx(noise[i], abs=1e-8)
+
+
+@pytest.mark.parametrize("store", [F32, BF16])
+def test_quadratic_gradient_in_its_storage_format(lib, store):
+    """The harness's gradient is delivered in the gradient's storage format
+    (the dtype the step consumes)."""
+    rng = np.random.default_rng(17)
+    n = 200
+    a = np.exp(rng.uniform(np.log(1e-3), 0, n))
+    g, _ = oracle.quadratic(a, rng.normal(0, 1, n), rng.normal(0, 1, n),
+                            rng.normal(0, 1e-2, n), store, lib=lib)
+    assert _fp32_exact(g)
+    if store == BF16:
+        assert _bf16_exact(g)
+
+
 # ------------------------------------------------------- SAPipe-WP (App. B.1)
 
 def _fixed_grad_run(lib, correction, steps=8, wd=0.1, ef=True, lam=1.0, beta=(0.9, 0.95),
