@@ -403,3 +403,28 @@ def test_newton_schulz_bf16_restated_exactly(lib, steps, tall):
     want = X.T if tall else X
     got = newton_schulz(M, steps=steps, store=BF16, eps=0.0, lib=lib)
     assert np.array_equal(got, want)
+
+
+@pytest.mark.parametrize("correction", [0, 1])
+def test_muon_reentering_delayed_training_restarts(lib, correction):
+    """Delayed, synchronous, delayed again: from the re-entry on, the run is a
+    fresh Alg. 1 run (stash at X, history zero, standard rule first, then EF
+    or SAPipe's prediction) started at the weights and momentum reached
+    there."""
+    rng = np.random.default_rng(73)
+    x0 = rng.normal(size=(4, 6))
+    grads = [rng.normal(size=(4, 6)) for _ in range(10)]
+    hp = _hp(ef_lambda=1.0, correction=correction)
+    o = DelayedMuon([x0], hp, ef=True, x_store=F64, stash_store=F64, lib=lib)
+    for k, g in enumerate(grads[:7], start=1):
+        if k == 4:
+            o.set_delay(0)
+        o.step([g])
+    o.set_delay(1)
+    fresh = DelayedMuon([o.x[0].copy()], hp, ef=True, x_store=F64, stash_store=F64, lib=lib)
+    fresh.mom[0][...] = o.mom[0]
+    for g in grads[7:]:
+        o.step([g])
+        fresh.step([g])
+        assert np.array_equal(o.x[0], fresh.x[0])
+        assert np.array_equal(o.stash[0], fresh.stash[0])

@@ -191,6 +191,67 @@ def test_every_planted_mistake_fails_a_pin(tmp_path):
     assert all(rc == 1 for _, rc, _ in results), results
 
 
+# Single mistakes in the oracle's Python drivers (oracle/__init__.py and
+# oracle/muon.py): the mode switches and Alg. 1's phase counter live there.
+PY_MUTANTS = [
+    ("__init__.py", "set_delay_keeps_history", "                self.u_prev[:] = 0.0\n",
+     "                pass\n"),
+    ("__init__.py", "set_delay_no_restash",
+     "            self.stash = round_to(self.x, self.stash_store, self.lib)\n", "            pass\n"),
+    ("__init__.py", "set_delay_no_phase_reset", "            self.t = 0\n            self.stash_tag",
+     "            self.stash_tag"),
+    ("__init__.py", "ef_timing_from_global_k", "g.size, self.k, max(self.t, 1)",
+     "g.size, self.k, max(self.k, 1)"),
+    ("muon.py", "muon_set_delay_keeps_history", "                    u[...] = 0.0\n",
+     "                    pass\n"),
+    ("muon.py", "muon_set_delay_no_restash",
+     "            self.stash = [round_to(x, self.stash_store, self.lib).reshape(x.shape)\n"
+     "                          for x in self.x]\n", "            pass\n"),
+    ("muon.py", "muon_set_delay_no_phase_reset",
+     "                    u[...] = 0.0\n            self.t = 0\n", "                    u[...] = 0.0\n"),
+    ("muon.py", "muon_ef_timing_from_global_k", "rows, cols, max(self.t, 1),",
+     "rows, cols, max(self.k, 1),"),
+    ("muon.py", "muon_sync_matrix_delayed",
+     "dly = self.delay if self.delayed is None or self.delayed[i] else 0", "dly = self.delay"),
+    ("muon.py", "muon_clip_per_matrix",
+     "            sq = sum(float(self.lib.oracle_sqnorm(g.size, _ptr(g))) for g in grads)",
+     "            sq = float(self.lib.oracle_sqnorm(grads[0].size, _ptr(grads[0])))"),
+]
+
+
+def _run_py_mutant(root, fname, old, new):
+    """The pins against a copy of the oracle package with one driver line
+    changed (the copy's tests directory puts the copy first on the path)."""
+    import shutil
+    shutil.copytree(os.path.join(ROOT, "oracle"), os.path.join(root, "oracle"),
+                    ignore=shutil.ignore_patterns("__pycache__"))
+    os.makedirs(os.path.join(root, "tests"))
+    for f in ("conftest.py", "test_oracle_pins.py", "test_oracle_muon.py"):
+        shutil.copy(os.path.join(ROOT, "tests", f), os.path.join(root, "tests", f))
+    path = os.path.join(root, "oracle", fname)
+    src = open(path).read()
+    assert src.count(old) == 1, f"mutation site in {fname} not unique"
+    open(path, "w").write(src.replace(old, new))
+    env = dict(os.environ, OMP_NUM_THREADS="1")
+    env.pop("DPO_ORACLE_LIB", None)
+    r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
+                        "tests/test_oracle_pins.py", "tests/test_oracle_muon.py"],
+                       cwd=root, env=env, capture_output=True, text=True, timeout=600)
+    return r.returncode
+
+
+def test_every_planted_driver_mistake_fails_a_pin(tmp_path):
+    jobs = [(str(tmp_path / name), f, old, new) for f, name, old, new in PY_MUTANTS]
+    with ThreadPoolExecutor(max_workers=min(8, os.cpu_count() or 1)) as ex:
+        rcs = list(ex.map(lambda j: _run_py_mutant(*j), jobs))
+    survivors = [m[1] for m, rc in zip(PY_MUTANTS, rcs) if rc == 0]
+    assert not survivors, f"driver mistakes no pin caught: {survivors}"
+    assert all(rc == 1 for rc in rcs), rcs
+    # the harness itself: an unchanged copy passes
+    assert _run_py_mutant(str(tmp_path / "identity"), "__init__.py",
+                          "class DelayedOptimizer:", "class DelayedOptimizer:") == 0
+
+
 def test_unmutated_copy_passes(tmp_path):
     lib = _build_mutant(tmp_path, "identity", "int oracle_step(", "int oracle_step(")
     rc, out = _run_pins(lib)

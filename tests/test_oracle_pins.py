@@ -1006,3 +1006,34 @@ def test_synchronous_tensor_stash_untouched(lib):
         o.step(rng.normal(0, 1, 9))
     assert np.array_equal(o.stash[5:], s0[5:])
     assert not np.array_equal(o.stash[:5], s0[:5])
+
+
+@pytest.mark.parametrize("corr", [oracle.CORR_EF, oracle.CORR_SAPIPE_SAME])
+def test_reentering_delayed_training_restarts_alg1(lib, corr):
+    """Delayed, synchronous, then delayed again (Sec. 3.1, App. A.10): from the
+    re-entry on, the run is a fresh Alg. 1 run started at the weights reached
+    there (SGD rule: no optimizer state besides the stash and the history):
+    the stash restarts at x, the history at zero, the first call takes the
+    standard rule and EF (or SAPipe's prediction) starts from there."""
+    rng = np.random.default_rng(71)
+    a = np.exp(rng.uniform(np.log(0.05), 0, 6))
+    x0 = rng.normal(0, 1, 6)
+    hp = HParams(lr=0.3, weight_decay=0.0, rule=oracle.RULE_SGD, ef_lambda=1.0, correction=corr)
+
+    def drive(o, n, switch=None):
+        xs = []
+        for c in range(1, n + 1):
+            if switch and c in switch:
+                o.set_delay(switch[c])
+            w, tag = o.read_weights("stale")
+            g, _ = oracle.quadratic(a, np.zeros(6), w, None, F64, lib=lib)
+            o.step(g, tag=tag)
+            xs.append(o.x.copy())
+        return xs
+
+    o = oracle.DelayedOptimizer([x0], hp, ef=True, x_store=F64, stash_store=F64, lib=lib)
+    xs = drive(o, 11, {5: 0, 8: 1})      # delayed 1-4, synchronous 5-7, delayed 8-11
+    fresh = oracle.DelayedOptimizer([xs[6]], hp, ef=True, x_store=F64, stash_store=F64, lib=lib)
+    ys = drive(fresh, 4)
+    for got, want in zip(xs[7:], ys):
+        assert np.array_equal(got, want)
