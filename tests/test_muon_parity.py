@@ -491,3 +491,23 @@ def test_muon_weight_decay_mask_parity(cuda_device):
             close_with_flips(p.cat(p.gpu.ef), _flat(p.ref.u_prev), 1e-5, du, 2e-3)
     finally:
         p.close()
+
+
+@pytest.mark.parametrize("correction", [0, 1])
+def test_muon_reentering_delayed_training_parity(cuda_device, correction):
+    """Delayed calls 1-2, synchronous 3-4, delayed again from 5 (EF or SAPipe
+    same state): Alg. 1 restarts at the re-entry on the device as in the
+    oracle."""
+    p = Pair(SHAPES, cuda_device, ns_steps=1, ef=True, schedule={3: 0, 5: 1},
+             correction=correction)
+    r_max = 0.2 * np.sqrt(max(max(sh) for sh in SHAPES))
+    du = p.lr * r_max * 2.0 ** -7
+    try:
+        for k in range(7):
+            p.step()
+            close_with_flips(p.cat(p.gpu.master), _flat(p.ref.x), TOL_RUN, (k + 1) * du, 1e-3)
+            if p.gpu.delay == 1:
+                close_with_flips(p.cat(p.gpu.stash).astype(np.float64), _flat(p.ref.stash),
+                                 2.0 ** -7, (k + 1) * du, 1e-3)
+    finally:
+        p.close()

@@ -496,6 +496,21 @@ def test_pingpong_stash_switches(cuda_device):
         run.close()
 
 
+@pytest.mark.parametrize("corr", [dpo.DPO_CORR_EF, SP_SAME])
+def test_reentering_delayed_training_parity(cuda_device, corr):
+    """Delayed calls 1-2, synchronous 3-4, delayed again from 5: the device
+    restarts Alg. 1 there as the oracle does (history zeroed, so SAPipe's
+    first prediction is x itself, EF from the second call)."""
+    run = Run(Case(RAGGED, stash_dtype=B, ef=True, correction=corr, schedule={3: 0, 5: 1}),
+              cuda_device)
+    try:
+        for k in range(1, 9):
+            run.step()
+            run.assert_close(TOL_ONE_STEP if k == 1 else TOL_RUN)
+    finally:
+        run.close()
+
+
 @pytest.mark.parametrize("dc", [0.0, 1e4])
 def test_pingpong_equals_copy_stash_bitwise(cuda_device, dc):
     """Same seeded run with the copying and the ping-pong stash: master, m, v,
