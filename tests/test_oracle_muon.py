@@ -428,3 +428,21 @@ def test_muon_reentering_delayed_training_restarts(lib, correction):
         fresh.step([g])
         assert np.array_equal(o.x[0], fresh.x[0])
         assert np.array_equal(o.stash[0], fresh.stash[0])
+
+
+def test_muon_momentum_depends_only_on_consumed_gradients(lib):
+    """Muon's momentum takes each consumed gradient whatever the delay mode:
+    a run with a synchronous start, a cooldown and a re-entry holds the same
+    momentum as a run delayed throughout, given the same gradients."""
+    rng = np.random.default_rng(83)
+    x0 = rng.normal(size=(3, 5))
+    grads = [rng.normal(size=(3, 5)) for _ in range(8)]
+    runs = []
+    for schedule in ({}, {1: 0, 3: 1, 5: 0, 7: 1}):
+        o = DelayedMuon([x0], _hp(ef_lambda=1.0), ef=True, x_store=F64, stash_store=F64, lib=lib)
+        for c, g in enumerate(grads, start=1):
+            if c in schedule:
+                o.set_delay(schedule[c])
+            o.step([g])
+        runs.append(o.mom[0].copy())
+    assert np.array_equal(runs[0], runs[1])

@@ -132,6 +132,8 @@ MUTANTS = [
      "            const double c = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;\n"
      "            const double sgn = c > 0.0 ? 1.0 : (c < 0.0 ? -1.0 : 0.0);\n"
      "            u = hp->lr * (sgn + wd * xt);"),
+    ("adan_first_step_per_delayed_phase", "const double diff = k == 1 ? 0.0 : gi - g_prev[i];",
+     "const double diff = t == 1 ? 0.0 : gi - g_prev[i];"),
     ("ns_on_the_larger_gram_matrix", "const int tall = rows > cols;",
      "const int tall = rows < cols;"),
     ("quadratic_gradient_unrounded",

@@ -1037,3 +1037,29 @@ def test_reentering_delayed_training_restarts_alg1(lib, corr):
     ys = drive(fresh, 4)
     for got, want in zip(xs[7:], ys):
         assert np.array_equal(got, want)
+
+
+@pytest.mark.parametrize("rule", [oracle.RULE_ADAMW, oracle.RULE_NADAM, oracle.RULE_ADAN])
+def test_statistics_depend_only_on_consumed_gradients(lib, rule):
+    """The optimizer statistics (m, v; Adan's n and previous gradient) are
+    updated with the gradient each call consumes (Alg. 1), whatever the
+    delay mode: with the same gradient sequence, a run with a synchronous
+    start, a cooldown and a re-entry holds the same statistics as a run
+    delayed throughout. (Adan's first-step rule, a zero difference, belongs
+    to the first gradient of the run, not of a delayed phase.)"""
+    rng = np.random.default_rng(81)
+    x0 = rng.normal(0, 0.5, 20)
+    grads = [rng.normal(0, 1, 20) for _ in range(9)]
+    hp = HParams(lr=0.01, ef_lambda=1.0, rule=rule)
+    runs = []
+    for schedule in ({}, {1: 0, 3: 1, 6: 0, 8: 1}):
+        o = oracle.DelayedOptimizer([x0], hp, ef=True, x_store=F64, stash_store=F64, lib=lib)
+        for c, g in enumerate(grads, start=1):
+            if c in schedule:
+                o.set_delay(schedule[c])
+            o.step(g)
+        runs.append(o)
+    a, b = runs
+    for name in ("m", "v", "n3", "g_prev"):
+        if getattr(a, name) is not None:
+            assert np.array_equal(getattr(a, name), getattr(b, name)), name
