@@ -511,6 +511,21 @@ def test_reentering_delayed_training_parity(cuda_device, corr):
         run.close()
 
 
+@pytest.mark.parametrize("rule", ["nadam", "adan"])
+def test_rules_across_mode_switches_parity(cuda_device, rule):
+    """NAdam's and Adan's statistics continue across a synchronous start, a
+    cooldown and a re-entry (Adan's zero first difference only at the run's
+    first gradient), on the device as in the oracle."""
+    run = Run(Case(RAGGED, stash_dtype=B, ef=True, schedule={1: 0, 3: 1, 6: 0, 8: 1},
+                   **RULES[rule]), cuda_device)
+    try:
+        for k in range(1, 11):
+            run.step()
+            run.assert_close(TOL_ONE_STEP if k == 1 else TOL_RUN)
+    finally:
+        run.close()
+
+
 @pytest.mark.parametrize("dc", [0.0, 1e4])
 def test_pingpong_equals_copy_stash_bitwise(cuda_device, dc):
     """Same seeded run with the copying and the ping-pong stash: master, m, v,
