@@ -117,7 +117,14 @@ def test_oracle_thread_count_is_settable():
 
 def test_committed_traffic_is_per_kernel_variant():
     """The committed headline summary's figure serves the headline only, not
-    another rule or mode that runs a different kernel instance."""
+    another rule or mode that runs a different kernel instance: each of those
+    takes its own summary's figure, or none."""
     import bench
-    assert bench.committed_traffic("fused_step:llama-7B:ef:lion:pingpong") is None
+    head = bench.committed_traffic("fused_step:llama-7B:ef:pingpong")
+    assert head is not None
+    for tag in ("fused_step:llama-7B:ef:lion:pingpong", "fused_step:llama-7B:std:pingpong",
+                "fused_step:llama-7B:ef"):
+        got = bench.committed_traffic(tag)
+        assert got is None or got != head
     assert bench.committed_traffic("fused_step:llama-7B:ef:dc:pingpong") is None
+    assert bench.committed_traffic("fused_step:llama-7B:ef:pingpong:extra") is None
