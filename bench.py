@@ -166,6 +166,13 @@ def committed_traffic(kernel_tag: str, key: str = "dram_bytes_per_param"):
     return None
 
 
+def ns_gemm_tag(workload: str, ns_steps: int) -> str:
+    """Kernel tag of the Newton-Schulz GEMM chain's per-step traffic: it
+    depends on the matrix set and the number of Newton-Schulz steps, not on
+    the delayed rule (which changes only the elementwise apply pass)."""
+    return f"ns_gemm:{workload}:ns{ns_steps}"
+
+
 # ---------------------------------------------------------------- clocks --
 
 class ClockSampler:
@@ -699,7 +706,7 @@ def main_muon(args, w, world, rank, local):
     peak, peak_kind = measured_bf16_peak()
     roof = {"bound": "tensor", "achieved": r["achieved"], "peak": peak, "unit": "TFLOP/s",
             "frac": r["achieved"] / peak, "peak_kind": f"{peak_kind} (sustained)",
-            "traffic": committed_traffic(f"ns_gemm:{w.name}:muon-{args.mode}",
+            "traffic": committed_traffic(ns_gemm_tag(w.name, args.ns_steps),
                                          "dram_bytes_per_step"),
             "kernel": "ns_gemm_kernel",
             "algorithmic_flops_per_step": r["flops"], "gemm_ms_per_step": r["gemm_ms"],

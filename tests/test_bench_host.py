@@ -123,8 +123,21 @@ def test_committed_traffic_is_per_kernel_variant():
     head = bench.committed_traffic("fused_step:llama-7B:ef:pingpong")
     assert head is not None
     for tag in ("fused_step:llama-7B:ef:lion:pingpong", "fused_step:llama-7B:std:pingpong",
-                "fused_step:llama-7B:ef"):
+                "fused_step:llama-7B:ef", "fused_step:llama-7B:ef:dc:pingpong",
+                "fused_step:llama-7B:ef:adan:pingpong"):
         got = bench.committed_traffic(tag)
         assert got is None or got != head
-    assert bench.committed_traffic("fused_step:llama-7B:ef:dc:pingpong") is None
+    # WPipe's traffic does not scale from one layer to the set: no figure
+    assert bench.committed_traffic("fused_step:llama-7B:ef:wpipe:pingpong") is None
     assert bench.committed_traffic("fused_step:llama-7B:ef:pingpong:extra") is None
+
+
+def test_ns_gemm_traffic_follows_the_newton_schulz_steps():
+    """The GEMM chain's committed traffic serves the Newton-Schulz step count
+    it was taken with, under any delayed rule, and no other step count."""
+    import bench
+    got = bench.committed_traffic(bench.ns_gemm_tag("llama-7B", 5), "dram_bytes_per_step")
+    assert got is not None and got > 0
+    assert bench.committed_traffic(bench.ns_gemm_tag("llama-7B", 3), "dram_bytes_per_step") is None
+    assert bench.committed_traffic(bench.ns_gemm_tag("llama-1B", 5), "dram_bytes_per_step") is None
+    assert bench.ns_gemm_tag("llama-7B", 5) == "ns_gemm:llama-7B:ns5"
