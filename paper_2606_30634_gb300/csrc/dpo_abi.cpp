@@ -599,7 +599,8 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
                 return cuda_fail(c, e, "clip-coefficient launch");
         } else if (c->clip) {
             dpo::NormArgs na{c->d_table, c->d_pkt_begin, c->n, c->total_pkts,
-                             (double)c->hp.max_grad_norm, c->d_partials, c->d_scalars};
+                             (double)c->hp.max_grad_norm, c->d_partials, c->d_scalars,
+                             nullptr};
             const cudaError_t e = dpo::launch_norm(c->grad_dt == DPO_BF16, c->norm_grid, na, s);
             if (e != cudaSuccess)
                 return cuda_fail(c, e, "gradient-norm launch");
