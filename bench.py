@@ -713,7 +713,7 @@ def main_muon(args, w, world, rank, local):
             "gemm_launches_per_step": r["gemm_launches"] / max(1, args.steps),
             "nominal_peak_tflops": 2250.0, "library_newton_schulz": r["library"]}
     cpu = None
-    if rank == 0 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:   # the oracle at N=1 only
         v, cores, steps, n = oracle_muon_sample(args.cpu_seconds)
         cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
                "sample": f"one 1024 x 4096 matrix, {steps} Muon oracle steps (plain C, fp64, "
@@ -796,7 +796,7 @@ def main(argv=None):
             "avg_launch_ms": r["kernel_ms"], "nominal_peak_gbs": 8000.0,
             "frac_of_nominal": r["achieved"] / 8000.0}
     cpu = None
-    if rank == 0 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:   # the oracle at N=1 only
         v, cores, steps, n = oracle_sample_run(w, args.mode, args.cpu_seconds,
                                                rule=rule_settings(args))
         v1, _, steps1, n1 = oracle_sample_run(w, args.mode, args.cpu_seconds / 3,
