@@ -255,11 +255,16 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
     return *reinterpret_cast<const uint32_t *>(&h);
 }
 
-// Tile t of a launch: batch entry, row block and column block, columns
-// fastest (consecutive pairs share the A rows of a block row in L2). A
-// symmetric product (sym, m_tiles == n_tiles) enumerates only the tiles on
-// or above the diagonal, row m holding m_tiles - m of them, so the pairs'
-// shares of its work differ by at most one tile.
+// Tile t of a launch: batch entry, row block and column block. A full
+// product walks bands of kBandRows block rows, each band column by column,
+// so the tiles in flight at once (one per CTA pair) share a few A row blocks
+// and a few B column blocks in L2: on a 4096 x 11008 operand, walking whole
+// block rows instead had the pairs stream all 43 B column blocks every
+// wave. A symmetric product (sym, m_tiles == n_tiles) enumerates only the
+// tiles on or above the diagonal, row m holding m_tiles - m of them, so the
+// pairs' shares of its work differ by at most one tile.
+constexpr int kBandRows = 8;   // block rows per band of a full product's walk
+
 struct TileGrid {
     int m_tiles, n_tiles, nb, sym;
     __host__ __device__ __forceinline__ int per_batch() const
@@ -281,8 +286,12 @@ struct TileGrid {
             m0 = m * TM;
             n0 = (m + u) * TN;
         } else {
-            n0 = (u % n_tiles) * TN;
-            m0 = (u / n_tiles) * TM;
+            const int band = u / (kBandRows * n_tiles);
+            const int first = band * kBandRows;
+            const int rows = min(kBandRows, m_tiles - first);
+            const int r = u - first * n_tiles;   // 0 <= r < rows * n_tiles
+            m0 = (first + r % rows) * TM;
+            n0 = (r / rows) * TN;
         }
     }
 };
