@@ -256,14 +256,15 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
 }
 
 // Tile t of a launch: batch entry, row block and column block. A full
-// product walks bands of kBandRows block rows, each band column by column,
-// so the tiles in flight at once (one per CTA pair) share a few A row blocks
-// and a few B column blocks in L2: on a 4096 x 11008 operand, walking whole
-// block rows instead had the pairs stream all 43 B column blocks every
-// wave. A symmetric product (sym, m_tiles == n_tiles) enumerates only the
+// product walks bands of kBandRows block rows (all of them, up to 4096 rows),
+// each band column by column, so the tiles in flight at once (one per CTA
+// pair) share the band's A row blocks and a few B column blocks in L2, and
+// each B column block comes from DRAM about once per band. On a 4096 x 11008
+// operand, walking whole block rows instead had the pairs stream all 43 B
+// column blocks every round. A symmetric product (sym, m_tiles == n_tiles) enumerates only the
 // tiles on or above the diagonal, row m holding m_tiles - m of them, so the
 // pairs' shares of its work differ by at most one tile.
-constexpr int kBandRows = 8;   // block rows per band of a full product's walk
+constexpr int kBandRows = 16;   // block rows per band of a full product's walk
 
 struct TileGrid {
     int m_tiles, n_tiles, nb, sym;
