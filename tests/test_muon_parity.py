@@ -166,6 +166,29 @@ def test_newton_schulz_parity(cuda_device, steps):
         p.close()
 
 
+def test_newton_schulz_parity_past_one_band(cuda_device):
+    """A matrix with more block rows (18, ragged) than one band of the full
+    product's tile walk (16) and more block columns (19) than rows: one
+    Newton-Schulz step against the oracle at the one-step bars, and every
+    256 x 256 output tile on its own, so a tile the walk skipped or visited
+    twice would stand out."""
+    shape = (4353, 4700)
+    p = Pair([shape], cuda_device, ns_steps=1, seed=0xB4D)
+    try:
+        p.step()
+        (g,), (r,) = p.o_pairs()
+        d = np.abs(g - r)
+        norm = np.linalg.norm(g - r) / np.linalg.norm(r)
+        frac = float(np.mean(d > 0))
+        print(f"{shape}: normwise {norm:.3e}, differing {frac:.4%}")
+        assert norm <= NS_BARS[1][0] and frac <= NS_BARS[1][1]
+        worst = max(np.linalg.norm(d[i:i + 256, j:j + 256]) /
+                    np.linalg.norm(r[i:i + 256, j:j + 256])
+                    for i in range(0, shape[0], 256) for j in range(0, shape[1], 256))
+        assert worst <= 10 * NS_BARS[1][0], f"tile normwise {worst:.3e}"
+    finally:
+        p.close()
+
 def close_with_flips(gpu, ref, tol, flip, max_frac):
     """Elementwise at the floored bar ``tol`` except where a flipped bf16
     rounding of O moved an element: at most ``max_frac`` of the elements may
