@@ -261,9 +261,11 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
 // pair) share the band's A row blocks and a few B column blocks in L2, and
 // each B column block comes from DRAM about once per band. On a 4096 x 11008
 // operand, walking whole block rows instead had the pairs stream all 43 B
-// column blocks every round. A symmetric product (sym, m_tiles == n_tiles) enumerates only the
-// tiles on or above the diagonal, row m holding m_tiles - m of them, so the
-// pairs' shares of its work differ by at most one tile.
+// column blocks every round. A symmetric product (sym, m_tiles == n_tiles)
+// enumerates only the tiles on or above the diagonal, column by column
+// (column n holds n + 1 of them), so the pairs' shares of its work differ by
+// at most one tile, and the tiles in flight at once read the first block rows
+// of the operand before the pairs move on to the last ones.
 constexpr int kBandRows = 16;   // block rows per band of a full product's walk
 
 struct TileGrid {
@@ -279,13 +281,13 @@ struct TileGrid {
         b = t / per;
         int u = t - b * per;
         if (sym) {
-            int m = 0;
-            while (u >= m_tiles - m) {   // u < per, so m stays below m_tiles
-                u -= m_tiles - m;
-                ++m;
+            int n = 0;
+            while (u > n) {   // u < per, so n stays below m_tiles
+                u -= n + 1;
+                ++n;
             }
-            m0 = m * TM;
-            n0 = (m + u) * TN;
+            m0 = u * TM;
+            n0 = n * TN;
         } else {
             const int band = u / (kBandRows * n_tiles);
             const int first = band * kBandRows;
