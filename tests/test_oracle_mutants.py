@@ -218,6 +218,14 @@ PY_MUTANTS = [
     ("muon.py", "muon_clip_per_matrix",
      "            sq = sum(float(self.lib.oracle_sqnorm(g.size, _ptr(g))) for g in grads)",
      "            sq = float(self.lib.oracle_sqnorm(grads[0].size, _ptr(grads[0])))"),
+    ("muon.py", "muon_decay_mask_ignored",
+     "wd = h.weight_decay if self.wd_on is None or self.wd_on[i] else 0.0",
+     "wd = h.weight_decay"),
+    ("__init__.py", "decay_mask_ignored", "        self.mask = self._tensor_mask(self.wd_on, n)\n",
+     "        self.mask = self._tensor_mask(None, n)\n"),
+    ("__init__.py", "delay_mask_ignored",
+     "        self.delay_mask = self._tensor_mask(self.delayed, n)\n",
+     "        self.delay_mask = self._tensor_mask(None, n)\n"),
 ]
 
 
