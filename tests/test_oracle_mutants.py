@@ -226,6 +226,17 @@ PY_MUTANTS = [
     ("__init__.py", "delay_mask_ignored",
      "        self.delay_mask = self._tensor_mask(self.delayed, n)\n",
      "        self.delay_mask = self._tensor_mask(None, n)\n"),
+    ("__init__.py", "supplied_norm_ignored", "        if sq is None:\n            sq = float(",
+     "        if True:\n            sq = float("),
+    ("__init__.py", "stale_view_ignores_sync_tensors",
+     "            return np.where(self.delay_mask == 1, self.stash, latest), self.stash_tag\n",
+     "            return self.stash, self.stash_tag\n"),
+    ("__init__.py", "stale_view_in_synchronous_training",
+     "        if which == \"stale\" and self.delay == 1:\n",
+     "        if which == \"stale\":\n"),
+    ("__init__.py", "stash_tag_not_advanced",
+     "        if self.delay == 1:\n            self.stash_tag = self.latest_tag\n        self.latest_tag += 1\n",
+     "        self.latest_tag += 1\n"),
 ]
 
 

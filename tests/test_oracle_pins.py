@@ -439,6 +439,33 @@ def test_clip_nonfinite_norm_like_torch(lib):
         np.testing.assert_array_equal(coef * g, p.grad.numpy())
 
 
+
+def test_clip_from_a_supplied_norm(lib):
+    """Global clipping (App. E.1): two oracles over the halves of a set, each
+    given the squared norm over the whole gradient, take torch's
+    clip_grad_norm_ coefficient over the whole set and step exactly as one
+    oracle over the set, bitwise."""
+    rng = np.random.default_rng(12)
+    x0 = [rng.normal(0, 1, 300), rng.normal(0, 1, 217)]
+    hp = HParams(lr=0.01, weight_decay=0.1, max_grad_norm=1.0, ef_lambda=1.0)
+    full = oracle.DelayedOptimizer(x0, hp, ef=True, x_store=F64, stash_store=F64, lib=lib)
+    halves = [oracle.DelayedOptimizer([x], hp, ef=True, x_store=F64, stash_store=F64, lib=lib)
+              for x in x0]
+    for _ in range(4):
+        g = rng.normal(0, 0.2, 517)
+        params = [torch.nn.Parameter(torch.zeros(n, dtype=torch.float64)) for n in (300, 217)]
+        params[0].grad, params[1].grad = torch.tensor(g[:300]), torch.tensor(g[300:])
+        torch.nn.utils.clip_grad_norm_(params, 1.0)
+        coef = float(params[0].grad[0] / g[0])
+        assert coef < 0.5   # clipping is active
+        sq = oracle.sqnorm(g, lib=lib)
+        full.step(g)
+        halves[0].step(g[:300], sq=sq)
+        halves[1].step(g[300:], sq=sq)
+        for o in [full] + halves:
+            assert o.last_clip == pytest.approx(coef, rel=1e-13)
+        assert np.array_equal(np.concatenate([h.x for h in halves]), full.x)
+
 def test_quadratic_gradient_is_loss_derivative(lib):
     """grad = d loss / dw (central differences) when the noise is zero."""
     rng = np.random.default_rng(6)
