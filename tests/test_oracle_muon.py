@@ -17,6 +17,7 @@ import os
 
 import numpy as np
 import pytest
+import torch
 
 import oracle
 from oracle import muon
@@ -330,6 +331,34 @@ def test_muon_sapipe_prediction_rounds_through_the_master(lib):
     opt.step([np.ones((2, 2))])
     assert np.all(opt.stash[0] == 1.0)
 
+
+
+def test_muon_clip_from_a_supplied_norm(lib):
+    """Global clipping (App. E.1) across contexts: two Muon oracles, one per
+    matrix, each given the squared norm over both gradients, take torch's
+    clip_grad_norm_ coefficient over the pair and step exactly as one oracle
+    over both matrices, bitwise."""
+    rng = np.random.default_rng(37)
+    xs = [rng.normal(size=(4, 6)), rng.normal(size=(5, 3))]
+    hp = _hp(max_grad_norm=1.0, ef_lambda=1.0)
+    both = DelayedMuon(xs, hp, ef=True, x_store=F64, stash_store=F64, lib=lib)
+    one = [DelayedMuon([x], hp, ef=True, x_store=F64, stash_store=F64, lib=lib) for x in xs]
+    for _ in range(3):
+        gs = [rng.normal(0, 0.5, x.shape) for x in xs]
+        params = [torch.nn.Parameter(torch.zeros(x.shape, dtype=torch.float64)) for x in xs]
+        for p_, g in zip(params, gs):
+            p_.grad = torch.tensor(g)
+        torch.nn.utils.clip_grad_norm_(params, 1.0)
+        coef = float(params[0].grad[0, 0] / gs[0][0, 0])
+        assert coef < 0.5   # clipping is active
+        sq = sum(oracle.sqnorm(g, lib=lib) for g in gs)
+        both.step(gs)
+        for o, g in zip(one, gs):
+            o.step([g], sq=sq)
+        for o in [both] + one:
+            assert o.last_clip == pytest.approx(coef, rel=1e-13)
+        for i in range(2):
+            assert np.array_equal(one[i].x[0], both.x[i])
 
 def test_muon_weight_decay_mask(lib):
     """A matrix without decay is the same run as a context whose decay is

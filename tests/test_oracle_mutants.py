@@ -234,6 +234,8 @@ PY_MUTANTS = [
     ("__init__.py", "stale_view_in_synchronous_training",
      "        if which == \"stale\" and self.delay == 1:\n",
      "        if which == \"stale\":\n"),
+    ("muon.py", "muon_supplied_norm_ignored", "        if sq is None:\n            sq = sum(",
+     "        if True:\n            sq = sum("),
     ("__init__.py", "stash_tag_not_advanced",
      "        if self.delay == 1:\n            self.stash_tag = self.latest_tag\n        self.latest_tag += 1\n",
      "        self.latest_tag += 1\n"),
