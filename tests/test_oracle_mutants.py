@@ -147,6 +147,22 @@ MUTANTS = [
      "            param[i] = oracle_round(x[i], hp->param_store);\n    }\n    if (o_out",
      "        x[i] = oracle_round(xn, hp->x_store);\n        if (param != NULL)\n"
      "            param[i] = oracle_round(xn, hp->param_store);\n    }\n    if (o_out"),
+    ("adan_n_bias_by_bc2", "const double d = sqrt(ni / bc3) + hp->eps;",
+     "const double d = sqrt(ni / bc2) + hp->eps;"),
+    ("adan_update_drops_difference",
+     "u = hp->lr * ((mi / bc1 + hp->beta2 * vi / bc2) / d + wd * xt);",
+     "u = hp->lr * ((mi / bc1) / d + wd * xt);"),
+    ("adan_n_of_gradient_only", "const double w = gi + hp->beta2 * diff;",
+     "const double w = gi;"),
+    ("nadam_product_excludes_current", "    for (int64_t i = 1; i <= k; ++i)\n        mu_prod",
+     "    for (int64_t i = 1; i < k; ++i)\n        mu_prod"),
+    ("nadam_momentum_term_uses_mu_k", "mu_next / (1.0 - mu_prod_next) * mi / d",
+     "mu_k / (1.0 - mu_prod_next) * mi / d"),
+    ("lion_decay_not_scaled_by_lr", "u = hp->lr * (sgn + wd * xt);",
+     "u = hp->lr * sgn + wd * xt;"),
+    ("adamw_decay_not_scaled_by_lr",
+     "u = hp->lr * (m_hat / (sqrt(v_hat) + hp->eps) + wd * xt);",
+     "u = hp->lr * (m_hat / (sqrt(v_hat) + hp->eps)) + wd * xt;"),
 ]
 
 
