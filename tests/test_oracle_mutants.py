@@ -163,6 +163,24 @@ MUTANTS = [
     ("adamw_decay_not_scaled_by_lr",
      "u = hp->lr * (m_hat / (sqrt(v_hat) + hp->eps) + wd * xt);",
      "u = hp->lr * (m_hat / (sqrt(v_hat) + hp->eps)) + wd * xt;"),
+    ("ef_lambda_ignored", "xn = xt - u - lam * (u - u_prev[i]);", "xn = xt - u - (u - u_prev[i]);"),
+    ("sapipe_updated_without_decay",
+     "                                 wd * oracle_round(xn, hp->x_store));",
+     "                                 0.0 * oracle_round(xn, hp->x_store));"),
+    ("synchronous_tensor_history_written", "        if (hist_i) {\n            double hist = u;",
+     "        if (use_ef) {\n            double hist = u;"),
+    ("param_holds_old_weights",
+     "            param[i] = oracle_round(x[i], hp->param_store);\n    }\n    return 0;",
+     "            param[i] = oracle_round(xt, hp->param_store);\n    }\n    return 0;"),
+    ("muon_rms_scale_ignored", "? hp->rms_scale * sqrt((double)(rows > cols ? rows : cols))",
+     "? sqrt((double)(rows > cols ? rows : cols))"),
+    ("muon_clip_not_applied", "(1.0 - hp->momentum) * (clip_scale * g[i])",
+     "(1.0 - hp->momentum) * g[i]"),
+    ("muon_decay_not_scaled_by_lr",
+     "const double u = hp->lr * (s * O[i] + hp->weight_decay * xt);",
+     "const double u = hp->lr * s * O[i] + hp->weight_decay * xt;"),
+    ("ns_eps_inside_sqrt", "const double scale = 1.0 / (sqrt(ss) + eps);",
+     "const double scale = 1.0 / sqrt(ss + eps);"),
 ]
 
 
