@@ -379,6 +379,21 @@ def test_muon_weight_decay_mask(lib):
     assert np.array_equal(mixed.x[1], plain.x[0])
 
 
+
+def test_muon_initial_state_is_x0_in_its_storage_formats(lib):
+    """The start state holds each matrix's X_0 as the device stores it: the
+    master cast to fp32, the stash and the weights that value cast to bf16
+    (torch's casts), before any call."""
+    rng = np.random.default_rng(45)
+    xs = [rng.normal(0, 0.02, (6, 10)), rng.normal(0, 0.02, (3, 4))]
+    opt = DelayedMuon(xs, _hp(ef_lambda=1.0), ef=True, x_store=F32, stash_store=BF16,
+                      param_store=BF16, lib=lib)
+    for i, x in enumerate(xs):
+        x32 = torch.tensor(x).float()
+        np.testing.assert_array_equal(opt.x[i], x32.double().numpy())
+        np.testing.assert_array_equal(opt.stash[i], x32.bfloat16().double().numpy())
+        np.testing.assert_array_equal(opt.param[i], x32.bfloat16().double().numpy())
+
 def test_muon_stored_state_is_in_its_storage_format(lib):
     """Muon's buffers hold values of their storage formats after each call:
     master, momentum and the EF history in fp32, stash and weights in

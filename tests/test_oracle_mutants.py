@@ -270,6 +270,14 @@ PY_MUTANTS = [
      "        if which == \"stale\":\n"),
     ("muon.py", "muon_supplied_norm_ignored", "        if sq is None:\n            sq = sum(",
      "        if True:\n            sq = sum("),
+    ("__init__.py", "initial_weights_not_rounded",
+     "        self.x = round_to(flat, self.x_store, self.lib)\n", "        self.x = flat.copy()\n"),
+    ("__init__.py", "initial_param_not_rounded",
+     "        self.param = (round_to(self.x, self.param_store, self.lib)\n",
+     "        self.param = (self.x.copy()\n"),
+    ("muon.py", "muon_initial_weights_not_rounded",
+     "        self.x = [round_to(_f64(t), self.x_store, self.lib).reshape(s)\n",
+     "        self.x = [_f64(t).copy().reshape(s)\n"),
     ("__init__.py", "stash_tag_not_advanced",
      "        if self.delay == 1:\n            self.stash_tag = self.latest_tag\n        self.latest_tag += 1\n",
      "        self.latest_tag += 1\n"),

@@ -950,6 +950,21 @@ def test_stored_state_is_in_its_storage_format(lib):
         assert _bf16_exact(o.stash) and _bf16_exact(o.param)
 
 
+
+def test_initial_state_is_x0_in_its_storage_formats(lib):
+    """Alg. 1's start state holds x_0 as the device stores it: the master is
+    x_0 cast to fp32, the stash and the weights that fp32 value cast to bf16
+    (torch's casts, round to nearest even), before any call."""
+    rng = np.random.default_rng(44)
+    x0 = rng.normal(0, 0.02, 513)
+    o = oracle.DelayedOptimizer([x0[:300], x0[300:]], HParams(ef_lambda=1.0), ef=True,
+                                x_store=F32, stash_store=BF16, param_store=BF16, lib=lib)
+    x32 = torch.tensor(x0).float()
+    np.testing.assert_array_equal(o.x, x32.double().numpy())
+    xb = x32.bfloat16().double().numpy()
+    np.testing.assert_array_equal(o.stash, xb)
+    np.testing.assert_array_equal(o.param, xb)
+
 def test_bf16_weights_round_the_stored_master(lib):
     """The bf16 weights are the stored fp32 master rounded to bf16 (a5): two
     roundings from the update's exact result. x_0 = 1 + 2^-8, SGD rule with
