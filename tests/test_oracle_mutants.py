@@ -278,6 +278,10 @@ PY_MUTANTS = [
     ("muon.py", "muon_initial_weights_not_rounded",
      "        self.x = [round_to(_f64(t), self.x_store, self.lib).reshape(s)\n",
      "        self.x = [_f64(t).copy().reshape(s)\n"),
+    ("__init__.py", "fp32_settings_keep_lr", "        return HParams(r(self.lr), r(self.beta1)",
+     "        return HParams(self.lr, r(self.beta1)"),
+    ("muon.py", "muon_fp32_settings_keep_lr", "        return MuonHParams(r(self.lr), r(self.momentum)",
+     "        return MuonHParams(self.lr, r(self.momentum)"),
     ("__init__.py", "stash_tag_not_advanced",
      "        if self.delay == 1:\n            self.stash_tag = self.latest_tag\n        self.latest_tag += 1\n",
      "        self.latest_tag += 1\n"),

@@ -965,6 +965,26 @@ def test_initial_state_is_x0_in_its_storage_formats(lib):
     np.testing.assert_array_equal(o.stash, xb)
     np.testing.assert_array_equal(o.param, xb)
 
+
+def test_fp32_settings_are_torch_casts():
+    """HParams.as_f32 (and the Muon twin) hand the oracle the numbers a
+    device given fp32 settings computes with: every real is torch's fp32 cast
+    of the setting, every integer setting unchanged."""
+    from oracle.muon import MuonHParams
+    hp = HParams(lr=3e-4, beta1=0.9, beta2=0.95, eps=1e-8, weight_decay=0.1, ef_lambda=0.7,
+                 max_grad_norm=1.3, delay=1, rule=oracle.RULE_ADAN, correction=0,
+                 beta3=0.99, momentum_decay=4e-3, dc_lambda=0.04)
+    mh = MuonHParams(lr=2e-3, momentum=0.95, weight_decay=0.1, ef_lambda=0.7, ns_eps=1e-7,
+                     rms_scale=0.2, max_grad_norm=1.3)
+    for src in (hp, mh):
+        got = src.as_f32()
+        for name, v in vars(src).items():
+            w = getattr(got, name)
+            if isinstance(v, float):
+                assert w == torch.tensor(v, dtype=torch.float32).item(), name
+            else:
+                assert w == v, name
+
 def test_bf16_weights_round_the_stored_master(lib):
     """The bf16 weights are the stored fp32 master rounded to bf16 (a5): two
     roundings from the update's exact result. x_0 = 1 + 2^-8, SGD rule with
