@@ -181,6 +181,11 @@ MUTANTS = [
      "const double u = hp->lr * s * O[i] + hp->weight_decay * xt;"),
     ("ns_eps_inside_sqrt", "const double scale = 1.0 / (sqrt(ss) + eps);",
      "const double scale = 1.0 / sqrt(ss + eps);"),
+    ("clip_not_clamped_at_one", "    return coef > 1.0 ? 1.0 : coef;", "    return coef;"),
+    ("clip_nan_norm_passes", "    return coef > 1.0 ? 1.0 : coef;",
+     "    return coef <= 1.0 ? coef : 1.0;"),
+    ("sqnorm_drops_last_block", "        for (int64_t b = 0; b < nb; ++b)" + " " * 36 + "\\\n",
+     "        for (int64_t b = 0; b < nb - 1; ++b)" + " " * 32 + "\\\n"),
 ]
 
 
