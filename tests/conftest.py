@@ -34,3 +34,22 @@ def pytest_collection_modifyitems(config, items):
     for item in items:
         if item.get_closest_marker("gpu") is not None and item.get_closest_marker("timeout") is None:
             item.add_marker(pytest.mark.timeout(1200, method="thread"))
+
+
+def pytest_terminal_summary(terminalreporter):
+    """The worst parity figure of every buffer, per test that compared the
+    CUDA path with the oracle: printed every run, so a drift shows before it
+    crosses a bar. Floored metrics are asserted; ``*_raw_ulp_all`` (bf16
+    code points over all elements), ``*_under_floor`` (elements under the
+    floor) and ``*_norm`` (normwise) are reported beside them."""
+    pu = sys.modules.get("parity_util")
+    if pu is None or not getattr(pu, "WORST", None):
+        return
+    tr = terminalreporter
+    tr.section("parity (worst over each test's comparisons)")
+    for test, errs in sorted(pu.WORST.items()):
+        cells = []
+        for key in sorted(errs):
+            v = errs[key]
+            cells.append(f"{key}={v}" if isinstance(v, int) else f"{key}={v:.2e}")
+        tr.write_line(f"{test.split('::', 1)[-1]}: " + " ".join(cells))
