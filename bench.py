@@ -24,6 +24,7 @@ collective on the data path); timing is the maximum over ranks.
 from __future__ import annotations
 
 import argparse
+import gc
 import hashlib
 import json
 import os
@@ -72,6 +73,11 @@ def parse_args(argv=None):
                    help="train the second half of the tensor list synchronously (App. B.2)")
     p.add_argument("--e2e-steps", type=int, default=4)
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-link-peak", action="store_true",
+                   help="skip timing plain pinned-host copies (the e2e path's bound)")
+    p.add_argument("--no-secondary", action="store_true",
+                   help="skip the clipped Llama-1B step (norm pass and fused step timed apart)")
+    p.add_argument("--secondary-steps", type=int, default=10)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     return p.parse_args(argv)
@@ -127,8 +133,10 @@ def measured_hbm_peak():
 
 # The device sources each profiled kernel is compiled from.
 KERNEL_SOURCES = {
-    "fused_step": ("dpo_internal.h", "dpo_device.cuh", "dpo_step.cuh", "dpo_step_adamw.cu",
-                   "dpo_step_nadam.cu", "dpo_step_lion.cu", "dpo_step_adan.cu", "dpo_kernels.cu"),
+    "fused_step": ("dpo_internal.h", "dpo_device.cuh", "dpo_reduce.cuh", "dpo_step.cuh",
+                   "dpo_step_adamw.cu", "dpo_step_nadam.cu", "dpo_step_lion.cu",
+                   "dpo_step_adan.cu", "dpo_kernels.cu"),
+    "grad_sqnorm": ("dpo_internal.h", "dpo_device.cuh", "dpo_reduce.cuh", "dpo_kernels.cu"),
     "ns_gemm": ("dpo_internal.h", "dpo_device.cuh", "dpo_gemm.cuh", "dpo_muon.cu"),
 }
 
@@ -264,6 +272,16 @@ def wpipe_sync(w, args):
 
 # ------------------------------------------------------------ CPU oracle --
 
+def extrapolation(n_params: int, timed_params: int, timed_steps: int, timed_s: float,
+                  wall_s: float) -> dict:
+    """Labels of a CPU figure measured on a sample: its ms_per_step is the
+    sample's per-parameter rate scaled to the whole set, not a timed step."""
+    return {"extrapolated": timed_params < n_params, "timed_params": timed_params,
+            "timed_steps": timed_steps, "timed_s": timed_s, "wall_s": wall_s,
+            "ms_per_step_basis": f"{n_params} params / the rate measured on {timed_params} "
+                                 f"params over {timed_steps} steps"}
+
+
 def oracle_sample_run(w, mode: str, seconds: float, max_steps: int = 1000, n: int = 1 << 22,
                       rule: dict = None, threads: int = 0):
     """Time the oracle as it stands on the first n parameters of the set
@@ -387,6 +405,87 @@ def run_gpu(args, w, world, rank, local):
                 achieved=achieved, step_bytes=step_bytes, norm_bytes=norm_bytes, clocks=clocks,
                 launches=K * launches_per_step, step_ctas=step_ctas, threads=threads, e2e=e2e,
                 device_name=props.name)
+
+
+def run_secondary(args, dev, world):
+    """The clipped Llama-1B step (global-norm clipping at 1.0 over all 146
+    tensors, EF, fp32 stash, one-step delay): the norm pass and the fused
+    step each timed by the library's CUDA events on the launch stream
+    (dpo_set_timing), and the whole step by events around it."""
+    import numpy as np
+    import torch
+
+    from paper_2606_30634_gb300 import dpo, synth
+    from paper_2606_30634_gb300.synth import workloads as W
+
+    w = W.LLAMA_1B
+    gc.collect()
+    torch.cuda.empty_cache()   # the headline set's arenas
+    stream = torch.cuda.Stream(dev)
+    offs = np.concatenate([[0], np.cumsum(w.numels)]).astype(np.int64)
+    with torch.cuda.stream(stream):
+        lay = dpo.Layout.of(w.numels)
+        x0 = torch.empty(lay.total, dtype=torch.float32, device=dev)
+        for i, (o, n) in enumerate(zip(lay.offsets, lay.numels)):
+            synth.dev_normal(w.seed, synth.STREAM_INIT, 0, int(offs[i]), x0[o:o + n], W.INIT_SIGMA)
+        opt = dpo.DelayedAdamW(w.numels, param_dtype=w.param_dtype, stash_dtype=w.stash_dtype,
+                               grad_dtype=w.grad_dtype, ef=True, ef_lambda=1.0,
+                               max_grad_norm=w.max_grad_norm, delay=1, device=dev, x0=x0,
+                               stream=stream, lr=w.lr, beta1=w.beta1, beta2=w.beta2, eps=w.eps,
+                               weight_decay=w.weight_decay)
+        del x0
+        for i, (o, n) in enumerate(zip(lay.offsets, lay.numels)):
+            synth.dev_normal(w.seed, synth.STREAM_GRAD, 1, int(offs[i]), opt.grads(i),
+                             W.GRAD_SIGMA)
+    torch.cuda.synchronize(dev)
+    step_bytes, norm_bytes = dpo.dpo_algorithmic_bytes(opt.ctx)
+    _, norm_ctas, _ = dpo.dpo_launch_config(opt.ctx)
+    for _ in range(args.warmup):
+        opt.step(stream=stream)
+    torch.cuda.synchronize(dev)
+    K = max(1, args.secondary_steps)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    opt.set_timing(True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize(dev)
+    e0.record(stream)
+    for _ in range(K):
+        opt.step(stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    norm_ms, fused_ms, calls = opt.kernel_times()
+    opt.set_timing(False)
+    _, gnorm, coef = dpo.dpo_get_flags(opt.ctx, stream)
+    total_ms = e0.elapsed_time(e1)
+    opt.close()
+    del opt
+    torch.cuda.empty_cache()
+    total_ms = max_over_ranks(total_ms, world, dev)
+    norm_ms = max_over_ranks(norm_ms / calls, world, dev)
+    fused_ms = max_over_ranks(fused_ms / calls, world, dev)
+    peak, peak_kind = measured_hbm_peak()
+    n = w.n_params
+
+    def kern(bytes_, ms, tag):
+        t = committed_traffic(tag)
+        return {"avg_launch_ms": ms, "algorithmic_bytes_per_launch": bytes_,
+                "bytes_per_param": bytes_ / n, "achieved_gbs": bytes_ / (ms / 1e3) / 1e9,
+                "frac": bytes_ / (ms / 1e3) / 1e9 / peak,
+                "traffic": None if t is None else t * n, "traffic_tag": tag}
+
+    pair_ms = norm_ms + fused_ms
+    return {"workload": f"{w.name}: {n} params in {len(w.tensors)} tensors, EF (lambda=1), "
+                        f"global-norm clip at {w.max_grad_norm}, fp32 stash, one-step delay",
+            "value": n * K / (total_ms / 1e3) * world, "unit": UNIT, "steps": K,
+            "ms_per_step": total_ms / K, "grad_norm": gnorm, "clip_coef": coef,
+            "peak": peak, "peak_kind": peak_kind, "norm_ctas": norm_ctas,
+            "grad_sqnorm_kernel": kern(norm_bytes, norm_ms, f"grad_sqnorm:{w.name}"),
+            "fused_step_kernel": kern(step_bytes, fused_ms, f"fused_step:{w.name}:ef"),
+            "pair": {"bytes_per_param": (norm_bytes + step_bytes) / n,
+                     "achieved_gbs": (norm_bytes + step_bytes) / (pair_ms / 1e3) / 1e9,
+                     "frac": (norm_bytes + step_bytes) / (pair_ms / 1e3) / 1e9 / peak,
+                     "kernel_ms": pair_ms}}
 
 
 def muon_split(w):
@@ -646,6 +745,7 @@ def run_e2e(args, opt, stream, dev, world, w):
             h_param.copy_(opt.param, non_blocking=True)
 
     staged_s = timed(staged_step)
+    link = None if args.no_link_peak else link_peak(opt, h_grad, h_param, stream, dev)
     del h_grad, h_param
 
     # host I/O: the fused kernel reads the gradients from and writes the new
@@ -659,9 +759,60 @@ def run_e2e(args, opt, stream, dev, world, w):
             "path": "dpo_step with grad and bf16 param arenas in pinned host memory: the "
                     "fused kernel reads gradients and writes weights across the host link",
             "host_link_gbs": (gbytes + pbytes) / (secs / K) / 1e9,
+            "link_peak": link,
+            "link_frac": (None if link is None else
+                          (gbytes + pbytes) / (secs / K) / 1e9 / link["both_gbs"]),
             "staged": {"value": staged_value, "ms_per_step": staged_s / K * 1e3,
                        "path": "cudaMemcpy grad in, device-resident dpo_step, cudaMemcpy "
                                "weights out, on one stream"}}
+
+
+def link_peak(opt, h_grad, h_param, stream, dev, reps: int = 2) -> dict:
+    """The host link's own rates for the e2e step's transfers, by CUDA
+    events: the gradients' bytes host -> device alone, the weights' bytes
+    device -> host alone, and both at once on two streams (what the host-I/O
+    step needs every step). Plain cudaMemcpyAsync from and to the same pinned
+    buffers."""
+    import torch
+    other = torch.cuda.Stream(dev)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+
+    def h2d(s):
+        with torch.cuda.stream(s):
+            opt.grad.copy_(h_grad, non_blocking=True)
+
+    def d2h(s):
+        with torch.cuda.stream(s):
+            h_param.copy_(opt.param, non_blocking=True)
+
+    def best(fn):
+        ms = []
+        for _ in range(reps):
+            torch.cuda.synchronize(dev)
+            ev[0].record(stream)
+            fn()
+            ev[1].record(stream)
+            torch.cuda.synchronize(dev)
+            ms.append(ev[0].elapsed_time(ev[1]))
+        return min(ms)
+
+    def both():
+        # the second stream starts after the first's start event and the
+        # first waits for it at the end, so the interval spans both copies
+        other.wait_event(ev[0])
+        h2d(stream)
+        d2h(other)
+        ev[2].record(other)
+        stream.wait_event(ev[2])
+
+    gb, pb = opt.grad.numel() * opt.grad.element_size(), opt.param.numel() * opt.param.element_size()
+    t_in, t_out, t_both = best(lambda: h2d(stream)), best(lambda: d2h(stream)), best(both)
+    torch.cuda.synchronize(dev)
+    return {"h2d_gbs": gb / t_in / 1e6, "d2h_gbs": pb / t_out / 1e6,
+            "both_gbs": (gb + pb) / t_both / 1e6, "h2d_bytes": gb, "d2h_bytes": pb,
+            "what": "best of %d: pinned host -> device copy of the gradients alone, device -> "
+                    "pinned host copy of the bf16 weights alone, and both at once on two "
+                    "streams (combined bytes / elapsed)" % reps}
 
 
 # ------------------------------------------------------------------ main --
@@ -684,10 +835,14 @@ def main_muon(args, w, world, rank, local):
     if args.impl == "reference":
         if rank != 0:
             return 0
+        t0 = time.perf_counter()
         v, cores, steps, n = oracle_muon_sample(args.cpu_seconds)
+        wall = time.perf_counter() - t0
         line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT,
                 "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-                "ms_per_step": w.n_params / v * 1e3, "higher_is_better": True,
+                "ms_per_step": w.n_params / v * 1e3,
+                **extrapolation(w.n_params, n, steps, n * steps / v, wall),
+                "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
                 "config": cfg,
                 "cpu_baseline": {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
@@ -757,13 +912,17 @@ def main(argv=None):
     if args.impl == "reference":
         if rank != 0:
             return 0
+        t0 = time.perf_counter()
         v, cores, steps, n = oracle_sample_run(w, args.mode, args.cpu_seconds,
                                                max_steps=max(1, args.steps + args.warmup),
                                                rule=rule_settings(args))
+        wall = time.perf_counter() - t0
         sample = f"first {n} params of the set, {steps} oracle steps (plain C, fp64)"
         line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT,
                 "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-                "ms_per_step": w.n_params / v * 1e3, "higher_is_better": True,
+                "ms_per_step": w.n_params / v * 1e3,
+                **extrapolation(w.n_params, n, steps, n * steps / v, wall),
+                "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
                 "config": cfg,
                 "cpu_baseline": {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
@@ -779,6 +938,9 @@ def main(argv=None):
         torch.cuda.set_device(local)
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     r = run_gpu(args, w, world, rank, local)
+    secondary = None
+    if not args.no_secondary and w.name == "llama-7B":
+        secondary = run_secondary(args, torch.device("cuda", local), world)
     peak, peak_kind = measured_hbm_peak()
     # the tag names every setting that changes the kernel's traffic; the
     # headline keeps "fused_step:<set>:<mode>[:pingpong]"
@@ -816,6 +978,8 @@ def main(argv=None):
             "e2e": r["e2e"], "gpu_launches": r["launches"], "clocks": r["clocks"],
             "launch": {"ctas": r["step_ctas"], "threads": r["threads"]},
             "hbm_gbs_achieved": r["achieved"], "device": r["device_name"]}
+    if secondary is not None:
+        line["secondary"] = secondary
     print(json.dumps(line), flush=True)
     return 0
 

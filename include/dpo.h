@@ -342,6 +342,20 @@ int dpo_launch_config(const dpo_ctx *ctx, int *step_ctas, int *norm_ctas,
                       int *threads);
 
 /*
+ * Per-kernel timing, for measurement. With timing on, every dpo_step that
+ * launches work records three CUDA events on its stream: before the
+ * gradient-norm pass (or the clip-coefficient kernel of a clip source), before
+ * the fused step, and after it. dpo_get_timing waits for the recorded events,
+ * returns the summed milliseconds of the norm interval (*norm_ms, 0 without
+ * clipping) and of the fused-step interval (*step_ms) over the *calls timed
+ * calls since the last read, and starts a new count. The events' host
+ * bookkeeping is not repeated by a CUDA-graph replay: leave timing off while
+ * capturing. Returns DPO_OK, DPO_EINVAL or DPO_ECUDA.
+ */
+int dpo_set_timing(dpo_ctx *ctx, int on);
+int dpo_get_timing(dpo_ctx *ctx, double *norm_ms, double *step_ms, int64_t *calls);
+
+/*
  * Gradient norm without device allocation.
  *
  * The paper has no counterpart to this entry point; it serves callers that
@@ -351,26 +365,32 @@ int dpo_launch_config(const dpo_ctx *ctx, int *step_ctas, int *norm_ctas,
  * synchronization cudaMalloc and cudaFree may imply; dpo_init allocates a
  * small device block, so such callers use this instead. It computes what
  * the clipped dpo_step computes before its update, for one contiguous
- * gradient buffer: the global L2 norm (deterministic: fixed chunking and
- * summation order) and the clip coefficient min(1, max_grad_norm /
- * (norm + 1e-6)) (1 when max_grad_norm <= 0; NaN when the norm is NaN).
+ * gradient buffer: the global L2 norm (deterministic for a given numel:
+ * fixed chunking and summation order) and the clip coefficient
+ * min(1, max_grad_norm / (norm + 1e-6)): 1 when max_grad_norm <= 0, 1 for
+ * numel == 0 (norm 0), NaN when the norm is NaN (as the clipped dpo_step).
  *
  *   grad          device buffer of numel gradients (grad_dtype F32 or BF16),
  *                 32-byte aligned; 0 <= numel <= DPO_NOALLOC_MAX_NUMEL.
+ *   max_grad_norm finite (dpo_init's rule for its hyperparameters); a
+ *                 non-finite value gives DPO_EINVAL.
  *   norm_out      device pointer, receives the norm (double, 8-byte aligned).
  *   clip_out      device pointer, receives the coefficient (float).
  *
  * Its scratch is a fixed file-scope device array of
- * DPO_NOALLOC_MAX_CHUNKS partial sums (128 KiB), one per chunk of
- * DPO_NOALLOC_CHUNK_ELEMS elements; every GPU that loads the library holds
+ * DPO_NOALLOC_MAX_CHUNKS partial sums (128 KiB), one per chunk of at most
+ * DPO_NOALLOC_CHUNK_ELEMS elements (smaller chunks for smaller buffers, so
+ * they still spread over the SMs); every GPU that loads the library holds
  * it until the process exits. Larger inputs are rejected with DPO_EINVAL.
  * The call allocates nothing: it enqueues one small memset (clearing the
  * scratch's counter, which must start at zero) and one kernel on
  * cuda_stream. The first call on each device looks up the scratch array's
- * device address (cudaGetSymbolAddress) with that device current; make that
- * first call before any stream capture. All calls share the scratch array,
- * which keeps the last call's contents, so calls whose kernels overlap on the
- * GPU (different streams or host threads on one device) race on it.
+ * device address (cudaGetSymbolAddress) with that device current and keeps
+ * it until the process exits, which assumes the device's primary context
+ * lives that long (no cudaDeviceReset in between); make that first call
+ * before any stream capture. All calls share the scratch array, which keeps
+ * the last call's contents, so calls whose kernels overlap on the GPU
+ * (different streams or host threads on one device) race on it.
  * Returns DPO_OK, DPO_EINVAL, DPO_EALIGN, DPO_EDTYPE or DPO_ECUDA.
  */
 #define DPO_NOALLOC_CHUNK_ELEMS (1 << 20)
@@ -381,8 +401,6 @@ int dpo_grad_norm_noalloc(const void *grad, int64_t numel, dpo_dtype grad_dtype,
                           float max_grad_norm, double *norm_out, float *clip_out,
                           void *cuda_stream);
 
-/* Message of the last failing call on ctx (NULL ctx: last dpo_init failure of
- * the calling thread). Never NULL; owned by the library. */
 /*
  * Test hook for the allocation-failure paths, process-wide: of the library's
  * next device allocations (dpo_init makes one, dpo_muon_init one or two: its
@@ -393,6 +411,8 @@ int dpo_grad_norm_noalloc(const void *grad, int64_t numel, dpo_dtype grad_dtype,
  */
 int dpo_test_fail_allocs(int after, int count);
 
+/* Message of the last failing call on ctx (NULL ctx: last dpo_init failure of
+ * the calling thread). Never NULL; owned by the library. */
 const char *dpo_last_error(const dpo_ctx *ctx);
 
 /* Free the context and its device scratch (after the work enqueued on it has

@@ -32,7 +32,8 @@ LIBS = {
         "sources": ["csrc/dpo_kernels.cu", "csrc/dpo_step_adamw.cu", "csrc/dpo_step_nadam.cu",
                     "csrc/dpo_step_lion.cu", "csrc/dpo_step_adan.cu", "csrc/dpo_abi.cpp",
                     "csrc/dpo_noalloc.cu", "csrc/dpo_muon.cu"],
-        "headers": ["csrc/dpo_internal.h", "csrc/dpo_device.cuh", "csrc/dpo_step.cuh",
+        "headers": ["csrc/dpo_internal.h", "csrc/dpo_device.cuh", "csrc/dpo_reduce.cuh",
+                    "csrc/dpo_step.cuh",
                     "csrc/dpo_gemm.cuh", "../include/dpo.h", "../include/dpo_muon.h"],
         "includes": ["csrc"],
         "ptxas_v": ["csrc/dpo_step_adamw.cu", "csrc/dpo_muon.cu"],

@@ -55,6 +55,11 @@ struct dpo_ctx {
     dpo::StepCounters *d_cnt = nullptr;   // capturable mode's counters
     dpo::StepScalars *d_sc = nullptr;     // capturable mode's per-call scalars
     const double *clip_src = nullptr;   // external sum of squares (dpo_set_clip_source)
+    // dpo_set_timing: three events per timed call (before the norm pass,
+    // before the fused step, after it), recorded since the last read
+    bool timing = false;
+    std::vector<cudaEvent_t> ev_pool;
+    size_t ev_used = 0;
     std::string err;
 };
 
@@ -591,6 +596,22 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
     const int64_t k = c->k + 1;        // this call consumes the k-th gradient
     const int64_t t = k - c->phase_k0; // Alg. 1 iteration within the delayed phase
     cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+    cudaEvent_t ev_mid = nullptr, ev_end = nullptr;
+    if (c->timing && c->total_pkts > 0) {
+        while (c->ev_used + 3 > c->ev_pool.size()) {
+            cudaEvent_t ev;
+            const cudaError_t e = cudaEventCreate(&ev);
+            if (e != cudaSuccess)
+                return cuda_fail(c, e, "timing event");
+            c->ev_pool.push_back(ev);
+        }
+        const cudaError_t e = cudaEventRecord(c->ev_pool[c->ev_used], s);
+        if (e != cudaSuccess)
+            return cuda_fail(c, e, "timing event record");
+        ev_mid = c->ev_pool[c->ev_used + 1];
+        ev_end = c->ev_pool[c->ev_used + 2];
+        c->ev_used += 3;
+    }
     if (c->total_pkts > 0) {
         if (c->clip && c->clip_src != nullptr) {
             const cudaError_t e = dpo::launch_clip_from_sumsq(
@@ -651,12 +672,22 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
                 return cuda_fail(c, es, "step-scalars launch");
             a.dev = c->d_sc;
         }
+        if (ev_mid != nullptr) {
+            const cudaError_t et = cudaEventRecord(ev_mid, s);
+            if (et != cudaSuccess)
+                return cuda_fail(c, et, "timing event record");
+        }
         const cudaError_t e = dpo::launch_step(static_cast<dpo::Optimizer>(c->hp.optimizer),
                                                c->param_dt == DPO_BF16, stash_kind(c),
                                                c->grad_dt == DPO_BF16, corr, dc_on(c),
                                                pingpong_on(c), c->step_grid, a, s);
         if (e != cudaSuccess)
             return cuda_fail(c, e, "fused step launch");
+        if (ev_end != nullptr) {
+            const cudaError_t et = cudaEventRecord(ev_end, s);
+            if (et != cudaSuccess)
+                return cuda_fail(c, et, "timing event record");
+        }
     }
     if (c->capturable) {
         if (c->total_pkts == 0) {   // nothing launched: keep the device counter in step
@@ -897,10 +928,44 @@ extern "C" int dpo_launch_config(const dpo_ctx *c, int *step_ctas, int *norm_cta
     return DPO_OK;
 }
 
+extern "C" int dpo_set_timing(dpo_ctx *c, int on)
+{
+    if (c == nullptr)
+        return DPO_EINVAL;
+    c->timing = on != 0;
+    return DPO_OK;
+}
+
+extern "C" int dpo_get_timing(dpo_ctx *c, double *norm_ms, double *step_ms, int64_t *calls)
+{
+    if (c == nullptr || norm_ms == nullptr || step_ms == nullptr || calls == nullptr)
+        return DPO_EINVAL;
+    double tn = 0.0, ts = 0.0;
+    for (size_t q = 0; q + 3 <= c->ev_used; q += 3) {
+        float a = 0.0f, b = 0.0f;
+        cudaError_t e = cudaEventSynchronize(c->ev_pool[q + 2]);
+        if (e == cudaSuccess)
+            e = cudaEventElapsedTime(&a, c->ev_pool[q], c->ev_pool[q + 1]);
+        if (e == cudaSuccess)
+            e = cudaEventElapsedTime(&b, c->ev_pool[q + 1], c->ev_pool[q + 2]);
+        if (e != cudaSuccess)
+            return cuda_fail(c, e, "timing event read");
+        tn += a;
+        ts += b;
+    }
+    *norm_ms = tn;
+    *step_ms = ts;
+    *calls = (int64_t)(c->ev_used / 3);
+    c->ev_used = 0;
+    return DPO_OK;
+}
+
 extern "C" void dpo_destroy(dpo_ctx *c)
 {
     if (c == nullptr)
         return;
+    for (cudaEvent_t e : c->ev_pool)
+        cudaEventDestroy(e);
     if (c->dev_block != nullptr)
         cudaFree(c->dev_block);
     delete c;

@@ -19,61 +19,12 @@
 // packets as 128-bit ones, all with streaming (evict-first) cache hints: no
 // element is touched twice in a step. The step is elementwise and HBM-bound;
 // there is no tensor-core work in it.
-#include "dpo_device.cuh"
+#include "dpo_reduce.cuh"
 
 namespace dpo {
 namespace {
 
 // ------------------------------------------------------ gradient norm ----
-
-template <int NT>
-__device__ __forceinline__ double block_sum(double x, double *red)
-{
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1)
-        x += __shfl_down_sync(0xFFFFFFFFu, x, off);
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (lane == 0)
-        red[warp] = x;
-    __syncthreads();
-    double r = 0.0;
-    if (warp == 0) {
-        r = lane < NT / 32 ? red[lane] : 0.0;
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1)
-            r += __shfl_down_sync(0xFFFFFFFFu, r, off);
-    }
-    __syncthreads();
-    return r;   // valid in thread 0
-}
-
-// Kahan-compensated fp32 accumulation of per-packet sums of squares (the
-// compensation keeps the per-thread error near one rounding however many
-// packets a thread visits), fp64 from the block reduction on.
-__device__ __forceinline__ void kahan_add(float &sum, float &c, float x)
-{
-    const float y = x - c;
-    const float t = sum + y;
-    c = (t - sum) - y;
-    sum = t;
-}
-
-template <class GT>
-__device__ __forceinline__ float packet_sqsum(const GT *grad, int64_t e, int64_t numel)
-{
-    if (e + kPacket <= numel) {
-        float g[8];
-        ld8(grad + e, g);
-        return ((g[0] * g[0] + g[1] * g[1]) + (g[2] * g[2] + g[3] * g[3])) +
-               ((g[4] * g[4] + g[5] * g[5]) + (g[6] * g[6] + g[7] * g[7]));
-    }
-    float s = 0.0f;
-    for (int64_t i = e; i < numel; ++i) {
-        const float g = ld1(grad + i);
-        s += g * g;
-    }
-    return s;
-}
 
 // Norm and clip coefficient min(1, max_norm / (norm + 1e-6)) from a sum of
 // squares; a NaN norm stays NaN and reaches every element.

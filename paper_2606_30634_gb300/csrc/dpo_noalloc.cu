@@ -11,15 +11,24 @@
 // dpo_step computes, over one contiguous gradient buffer, with its scratch in
 // a fixed file-scope device array instead.
 //
-// Scratch: g_noalloc_scratch holds one fp64 partial sum per chunk of
-// kChunkElems elements (at most kMaxChunks chunks, so at most
+// Scratch: g_noalloc_scratch holds one fp64 partial sum per chunk (at most
+// kMaxChunks chunks of at most kChunkElems elements, so at most
 // DPO_NOALLOC_MAX_NUMEL elements per call) and the arrival ticket of the
 // last-CTA-finishes reduction. Every GPU that loads the library holds it until
 // the process exits. All calls share it and it keeps the last call's
 // contents: each call clears the ticket before its launch, and calls whose
 // kernels overlap on the GPU (different streams, or different host threads,
 // on one device) race on it.
+//
+// Chunking: a buffer is cut into equal chunks, one CTA each, of
+// chunk_elems(numel) elements: about numel / kTargetCtas rounded up to a
+// multiple of kMinChunk (one full round of the CTA's loads), between
+// kMinChunk and kChunkElems. So a gradient of a few million elements still
+// spreads over several CTAs per SM, and the largest ones use at most
+// kMaxChunks partials. The chunking, and with it the summation order,
+// depends only on numel: the result is deterministic.
 #include "dpo.h"
+#include "dpo_reduce.cuh"
 
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -29,17 +38,36 @@
 
 namespace {
 
+using dpo::block_sum;
+using dpo::kahan_add;
+using dpo::packet_sqsum;
+
 constexpr int kThreads = 256;
 constexpr int kUnroll = 4;
 constexpr int64_t kChunkElems = DPO_NOALLOC_CHUNK_ELEMS;
 constexpr int kMaxChunks = DPO_NOALLOC_MAX_CHUNKS;
+constexpr int64_t kMinChunk = (int64_t)kThreads * kUnroll * dpo::kPacket;   // 8192
+constexpr int64_t kTargetCtas = 1216;   // 8 per SM on a 152-SM GB300
 constexpr size_t kTicketOffset = sizeof(double) * kMaxChunks;
 constexpr size_t kScratchBytes = kTicketOffset + 256;
 
+static_assert(kChunkElems % kMinChunk == 0, "chunks are whole rounds of loads");
+
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kScratchBytes];
 
-// Device address of g_noalloc_scratch per device, looked up once per device
-// (host code cannot use the symbol's name as a device address).
+// Elements per chunk for a buffer of numel elements (see the file comment).
+int64_t chunk_elems(int64_t numel)
+{
+    int64_t c = (numel + kTargetCtas - 1) / kTargetCtas;
+    c = (c + kMinChunk - 1) / kMinChunk * kMinChunk;
+    return c < kMinChunk ? kMinChunk : (c > kChunkElems ? kChunkElems : c);
+}
+
+// Device address of g_noalloc_scratch per device, looked up by the first
+// call on each device and kept for the life of the process (host code cannot
+// use the symbol's name as a device address). This assumes the device's
+// primary context lives until exit: after cudaDeviceReset the module may be
+// loaded at another address, and the kept one would be stale.
 constexpr int kMaxDevices = 64;
 std::mutex g_mu;
 void *g_addr[kMaxDevices] = {};
@@ -58,103 +86,39 @@ cudaError_t scratch_address(int device, void **out)
     return cudaSuccess;
 }
 
-// ------------------------------------------------------- device helpers ----
-
-__device__ __forceinline__ void ld8(const float *p, float (&r)[8])
-{
-    asm volatile("ld.global.cs.v8.f32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
-                 : "=f"(r[0]), "=f"(r[1]), "=f"(r[2]), "=f"(r[3]), "=f"(r[4]), "=f"(r[5]),
-                   "=f"(r[6]), "=f"(r[7])
-                 : "l"(p));
-}
-
-__device__ __forceinline__ void ld8(const __nv_bfloat16 *p, float (&r)[8])
-{
-    const uint4 q = __ldcs(reinterpret_cast<const uint4 *>(p));
-    const uint32_t w[4] = {q.x, q.y, q.z, q.w};
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        r[2 * j] = __uint_as_float(w[j] << 16);
-        r[2 * j + 1] = __uint_as_float(w[j] & 0xFFFF0000u);
-    }
-}
-
-__device__ __forceinline__ float ld1(const float *p) { return __ldcs(p); }
-__device__ __forceinline__ float ld1(const __nv_bfloat16 *p) { return __bfloat162float(*p); }
-
-__device__ __forceinline__ void kahan_add(float &sum, float &c, float x)
-{
-    const float y = x - c;
-    const float t = sum + y;
-    c = (t - sum) - y;
-    sum = t;
-}
-
-__device__ __forceinline__ double block_sum(double x, double *red)
-{
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1)
-        x += __shfl_down_sync(0xFFFFFFFFu, x, off);
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (lane == 0)
-        red[warp] = x;
-    __syncthreads();
-    double r = 0.0;
-    if (warp == 0) {
-        r = lane < kThreads / 32 ? red[lane] : 0.0;
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1)
-            r += __shfl_down_sync(0xFFFFFFFFu, r, off);
-    }
-    __syncthreads();
-    return r;   // valid in thread 0
-}
-
-// CTA c sums the squares of chunk c, elements [c kChunkElems, (c+1) kChunkElems)
-// (8-element packets, kUnroll packets in flight per thread, Kahan fp32 per
-// thread, fp64 block tree), stores the partial in the scratch array, and the
-// last CTA to arrive adds the partials in chunk order and writes the norm and
-// the clip coefficient min(1, max_norm / (norm + 1e-6)). Deterministic.
+// CTA c sums the squares of chunk c, elements [c chunk, min((c+1) chunk,
+// numel)) (8-element packets, kUnroll packets in flight per thread, Kahan
+// fp32 per thread, fp64 block tree), stores the partial in the scratch array,
+// and the last CTA to arrive adds the partials in chunk order and writes the
+// norm and the clip coefficient min(1, max_norm / (norm + 1e-6)).
+// Deterministic for a given numel.
 template <class GT>
 __global__ void __launch_bounds__(kThreads)
-noalloc_sqnorm_kernel(const GT *__restrict__ grad, int64_t numel, double max_norm,
-                      unsigned char *scratch, double *norm_out, float *clip_out)
+noalloc_sqnorm_kernel(const GT *__restrict__ grad, int64_t numel, int64_t chunk,
+                      double max_norm, unsigned char *scratch, double *norm_out,
+                      float *clip_out)
 {
     __shared__ double red[kThreads / 32];
     __shared__ bool last;
     double *partials = reinterpret_cast<double *>(scratch);
     unsigned int *ticket = reinterpret_cast<unsigned int *>(scratch + kTicketOffset);
 
-    const int64_t lo = (int64_t)blockIdx.x * kChunkElems;
-    const int64_t hi = lo + kChunkElems < numel ? lo + kChunkElems : numel;
-    const int64_t pkts = (hi - lo + 7) / 8;
+    const int64_t lo = (int64_t)blockIdx.x * chunk;
+    const int64_t hi = lo + chunk < numel ? lo + chunk : numel;
+    const int64_t pkts = hi > lo ? (hi - lo + dpo::kPacket - 1) / dpo::kPacket : 0;
     float sum = 0.0f, comp = 0.0f;
     for (int64_t base = threadIdx.x; base < pkts; base += (int64_t)kThreads * kUnroll) {
         float part[kUnroll];
 #pragma unroll
         for (int u = 0; u < kUnroll; ++u) {
             const int64_t q = base + (int64_t)u * kThreads;
-            const int64_t e = lo + q * 8;
-            part[u] = 0.0f;
-            if (q < pkts) {
-                if (e + 8 <= hi) {
-                    float g[8];
-                    ld8(grad + e, g);
-                    part[u] = ((g[0] * g[0] + g[1] * g[1]) + (g[2] * g[2] + g[3] * g[3])) +
-                              ((g[4] * g[4] + g[5] * g[5]) + (g[6] * g[6] + g[7] * g[7]));
-                } else {
-                    for (int64_t i = e; i < hi; ++i) {
-                        const float g = ld1(grad + i);
-                        part[u] += g * g;
-                    }
-                }
-            }
+            part[u] = q < pkts ? packet_sqsum(grad, lo + q * dpo::kPacket, hi) : 0.0f;
         }
 #pragma unroll
         for (int u = 0; u < kUnroll; ++u)
             kahan_add(sum, comp, part[u]);
     }
-    const double cta = block_sum((double)sum - (double)comp, red);
+    const double cta = block_sum<kThreads>((double)sum - (double)comp, red);
     if (threadIdx.x == 0) {
         partials[blockIdx.x] = cta;
         __threadfence();
@@ -167,7 +131,7 @@ noalloc_sqnorm_kernel(const GT *__restrict__ grad, int64_t numel, double max_nor
     double acc = 0.0;
     for (int b = threadIdx.x; b < (int)gridDim.x; b += kThreads)
         acc += __ldcg(partials + b);
-    const double total = block_sum(acc, red);
+    const double total = block_sum<kThreads>(acc, red);
     if (threadIdx.x == 0) {
         const double norm = sqrt(total);
         double coef = max_norm > 0.0 ? max_norm / (norm + 1e-6) : 1.0;
@@ -207,14 +171,15 @@ extern "C" int dpo_grad_norm_noalloc(const void *grad, int64_t numel, dpo_dtype 
     // the ticket must start at zero (a previous call may have been cut short)
     if (cudaMemsetAsync(base + kTicketOffset, 0, sizeof(unsigned int), s) != cudaSuccess)
         return DPO_ECUDA;
-    const int grid = numel > 0 ? (int)((numel + kChunkElems - 1) / kChunkElems) : 1;
+    const int64_t chunk = chunk_elems(numel);
+    const int grid = numel > 0 ? (int)((numel + chunk - 1) / chunk) : 1;
     if (grad_dtype == DPO_BF16)
         noalloc_sqnorm_kernel<__nv_bfloat16><<<grid, kThreads, 0, s>>>(
-            static_cast<const __nv_bfloat16 *>(grad), numel, (double)max_grad_norm, base,
-            norm_out, clip_out);
+            static_cast<const __nv_bfloat16 *>(grad), numel, chunk, (double)max_grad_norm,
+            base, norm_out, clip_out);
     else
         noalloc_sqnorm_kernel<float><<<grid, kThreads, 0, s>>>(
-            static_cast<const float *>(grad), numel, (double)max_grad_norm, base, norm_out,
-            clip_out);
+            static_cast<const float *>(grad), numel, chunk, (double)max_grad_norm, base,
+            norm_out, clip_out);
     return cudaGetLastError() == cudaSuccess ? DPO_OK : DPO_ECUDA;
 }

@@ -34,7 +34,8 @@ EXPORTS = ("dpo_init", "dpo_stash", "dpo_step", "dpo_read_weights", "dpo_get_ste
            "dpo_set_step", "dpo_get_flags", "dpo_algorithmic_bytes", "dpo_launch_config",
            "dpo_last_error", "dpo_destroy", "dpo_grad_norm_noalloc", "dpo_set_delay",
            "dpo_grad_sqnorm", "dpo_set_clip_source", "dpo_test_fail_allocs",
-           "dpo_get_phase_start", "dpo_set_phase_start", "dpo_set_capturable")
+           "dpo_get_phase_start", "dpo_set_phase_start", "dpo_set_capturable",
+           "dpo_set_timing", "dpo_get_timing")
 
 DPO_NOALLOC_CHUNK_ELEMS = 1 << 20
 DPO_NOALLOC_MAX_CHUNKS = 16384
@@ -105,6 +106,9 @@ def load() -> ctypes.CDLL:
         "dpo_get_phase_start": (I, [P, ctypes.POINTER(ctypes.c_int64)]),
         "dpo_set_phase_start": (I, [P, ctypes.c_int64]),
         "dpo_set_capturable": (I, [P, I, P, P]),
+        "dpo_set_timing": (I, [P, I]),
+        "dpo_get_timing": (I, [P, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double),
+                               ctypes.POINTER(ctypes.c_int64)]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -200,6 +204,17 @@ def global_sqnorm(optimizers, acc, stream=None, group=None) -> None:
         for o in optimizers:
             o.grad_sqnorm(acc, s)
         allreduce_sqnorm(acc, group)
+
+
+def dpo_set_timing(ctx, on: bool) -> None:
+    _check(load().dpo_set_timing(ctx, 1 if on else 0), ctx)
+
+
+def dpo_get_timing(ctx):
+    """(norm-pass ms, fused-step ms, calls) since the last read."""
+    tn, ts, n = ctypes.c_double(), ctypes.c_double(), ctypes.c_int64()
+    _check(load().dpo_get_timing(ctx, ctypes.byref(tn), ctypes.byref(ts), ctypes.byref(n)), ctx)
+    return tn.value, ts.value, n.value
 
 
 def dpo_read_weights(ctx, which: int, tensor: int):
@@ -449,6 +464,16 @@ class DelayedAdamW:
         dpo_set_capturable(self.ctx, on, lr_source, stream)
         self._capturable = bool(on)
         self._lr_src = lr_source if on else None
+
+    def set_timing(self, on: bool = True) -> None:
+        """Record CUDA events around the norm pass and the fused step of
+        every step (dpo_set_timing); read them with kernel_times()."""
+        dpo_set_timing(self.ctx, on)
+
+    def kernel_times(self):
+        """(norm-pass ms, fused-step ms, calls) summed over the steps timed
+        since the last read (dpo_get_timing); waits for those steps."""
+        return dpo_get_timing(self.ctx)
 
     def grad_sqnorm(self, acc, stream=None) -> None:
         """Add this context's sum of g^2 to ``acc`` (dpo_grad_sqnorm)."""

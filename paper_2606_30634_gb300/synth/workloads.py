@@ -93,7 +93,15 @@ LLAMA_7B = Workload("llama-7B", _llama(4096, 11008, 32000, 32, 32, 32, tied=Fals
 LLAMA_7B_LAYER = Workload("llama-7B-layer", LLAMA_7B.tensors[1:10], BF16, BF16, BF16, steps=20,
                           seed=0xD0D0 + 5)
 
-ALL = {w.name: w for w in (FLAT, QUADRATIC, GPT2_SMALL, LLAMA_1B, LLAMA_7B, LLAMA_7B_LAYER)}
+# Four decoder layers of the 1B shapes with the 1B dtypes and clipping: the
+# same two kernel instances as the clipped 1B step (norm pass, fused step) on
+# 243M parameters, whose 486 MB of bf16 gradients exceed the 129 MB L2
+# (profiler captures).
+LLAMA_1B_4LAYERS = Workload("llama-1B-4layers", LLAMA_1B.tensors[1:37], BF16, F32, BF16,
+                            steps=50, max_grad_norm=1.0, seed=0xD0D0 + 4)
+
+ALL = {w.name: w for w in (FLAT, QUADRATIC, GPT2_SMALL, LLAMA_1B, LLAMA_7B, LLAMA_7B_LAYER,
+                           LLAMA_1B_4LAYERS)}
 
 # the quadratic's noise and curvature
 QUAD_NOISE_SIGMA = 1e-2
