@@ -106,8 +106,6 @@ int oracle_step(int64_t n, int64_t k, int64_t t, const oracle_hparams *hp,
     if (corr != ORACLE_CORR_EF && corr != ORACLE_CORR_SAPIPE_SAME &&
         corr != ORACLE_CORR_SAPIPE_UPDATED)
         return -1;
-    if (corr == ORACLE_CORR_SAPIPE_UPDATED && hp->rule != ORACLE_RULE_ADAMW)
-        return -1;
     /* Alg. 1: the standard rule is used for t <= 1 even under EF. */
     const int ef_now = use_ef && corr == ORACLE_CORR_EF && t >= 2;
     const double lam = hp->ef_lambda;
@@ -119,6 +117,7 @@ int oracle_step(int64_t n, int64_t k, int64_t t, const oracle_hparams *hp,
     const double bc1_next = 1.0 - pow(hp->beta1, (double)(k + 1));
     const double bc2_next = 1.0 - pow(hp->beta2, (double)(k + 1));
     const double bc3 = 1.0 - pow(hp->beta3, (double)k);
+    const double bc3_next = 1.0 - pow(hp->beta3, (double)(k + 1));
 
     /* NAdam's momentum schedule mu_i = beta1 (1 - 0.5 * 0.96^(i psi)) and its
      * running products up to k and k + 1. */
@@ -129,6 +128,12 @@ int oracle_step(int64_t n, int64_t k, int64_t t, const oracle_hparams *hp,
     const double mu_next =
         hp->beta1 * (1.0 - 0.5 * pow(0.96, (double)(k + 1) * hp->momentum_decay));
     const double mu_prod_next = mu_prod * mu_next;
+    /* ... and one index further, for the SAPipe updated-state prediction
+     * (NAdam's step at index k + 1 uses mu_{k+1}, mu_{k+2} and the products
+     * up to them). */
+    const double mu_next2 =
+        hp->beta1 * (1.0 - 0.5 * pow(0.96, (double)(k + 2) * hp->momentum_decay));
+    const double mu_prod_next2 = mu_prod_next * mu_next2;
 
 #pragma omp parallel for schedule(static)
     for (int64_t i = 0; i < n; ++i) {
@@ -204,13 +209,45 @@ int oracle_step(int64_t n, int64_t k, int64_t t, const oracle_hparams *hp,
         }
         if (hist_i) {
             double hist = u;
-            if (corr == ORACLE_CORR_SAPIPE_UPDATED) {
+            if (corr == ORACLE_CORR_SAPIPE_UPDATED && rule == ORACLE_RULE_ADAMW) {
                 /* The optimizer step once more on g_{t-1}, from the state the
-                 * real update left, at the next time index, decaying x_{t+1}. */
-                const double m2 = hp->beta1 * mi + (1.0 - hp->beta1) * gi;
-                const double v2 = hp->beta2 * vi + (1.0 - hp->beta2) * gi * gi;
+                 * real update left (the statistics as stored), at the next
+                 * time index, decaying x_{t+1}. */
+                const double m2 = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;
+                const double v2 = hp->beta2 * v[i] + (1.0 - hp->beta2) * gi * gi;
                 hist = hp->lr * ((m2 / bc1_next) / (sqrt(v2 / bc2_next) + hp->eps) +
                                  wd * oracle_round(xn, hp->x_store));
+            } else if (corr == ORACLE_CORR_SAPIPE_UPDATED) {
+                /* The same for the other rules: each rule's own step at index
+                 * k + 1 on g_{t-1}, from the statistics this call stored, with
+                 * decay on x_{t+1}. */
+                const double x_next = oracle_round(xn, hp->x_store);
+                if (rule == ORACLE_RULE_NADAM) {
+                    const double nm = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;
+                    const double nv = hp->beta2 * v[i] + (1.0 - hp->beta2) * gi * gi;
+                    const double d2 = sqrt(nv / bc2_next) + hp->eps;
+                    hist = hp->lr * ((1.0 - mu_next) / (1.0 - mu_prod_next) * gi / d2 +
+                                     mu_next2 / (1.0 - mu_prod_next2) * nm / d2 + wd * x_next);
+                } else if (rule == ORACLE_RULE_LION) {
+                    /* the sign of the beta1 blend of the updated momentum */
+                    const double c2 = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;
+                    const double s2 = c2 > 0.0 ? 1.0 : (c2 < 0.0 ? -1.0 : 0.0);
+                    hist = hp->lr * (s2 + wd * x_next);
+                } else if (rule == ORACLE_RULE_ADAN) {
+                    /* the stored previous gradient is now g_{t-1} itself, so
+                     * the next step's gradient difference is zero (up to that
+                     * store's rounding) */
+                    const double ad = gi - g_prev[i];
+                    const double am = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;
+                    const double av = hp->beta2 * v[i] + (1.0 - hp->beta2) * ad;
+                    const double aw = gi + hp->beta2 * ad;
+                    const double an = hp->beta3 * n3[i] + (1.0 - hp->beta3) * aw * aw;
+                    const double d2 = sqrt(an / bc3_next) + hp->eps;
+                    hist = hp->lr * ((am / bc1_next + hp->beta2 * av / bc2_next) / d2 +
+                                     wd * x_next);
+                } else {   /* SGD: no statistics */
+                    hist = hp->lr * (gi + wd * x_next);
+                }
             }
             u_prev[i] = oracle_round(hist, hp->x_store);
         }
@@ -410,12 +447,14 @@ int oracle_muon_step(int64_t rows, int64_t cols, int64_t t, const oracle_muon_hp
     const double s = hp->rms_scale > 0.0
                          ? hp->rms_scale * sqrt((double)(rows > cols ? rows : cols))
                          : 1.0;
-    if (hp->correction != ORACLE_CORR_EF && hp->correction != ORACLE_CORR_SAPIPE_SAME) {
+    if (hp->correction != ORACLE_CORR_EF && hp->correction != ORACLE_CORR_SAPIPE_SAME &&
+        hp->correction != ORACLE_CORR_SAPIPE_UPDATED) {
         free(O);
         return -1;
     }
     const int use_ef = hp->delay == 1 && u_prev != NULL;
-    const int sapipe = use_ef && hp->correction == ORACLE_CORR_SAPIPE_SAME;
+    const int updated = use_ef && hp->correction == ORACLE_CORR_SAPIPE_UPDATED;
+    const int sapipe = use_ef && (hp->correction == ORACLE_CORR_SAPIPE_SAME || updated);
     /* Alg. 1 / Alg. 2: the standard rule at t <= 1, EF from t = 2. */
     const int ef_now = use_ef && !sapipe && t >= 2;
     for (int64_t i = 0; i < n; ++i) {
@@ -426,7 +465,7 @@ int oracle_muon_step(int64_t rows, int64_t cols, int64_t t, const oracle_muon_hp
             stash[i] = oracle_round(oracle_round(x[i] - u_prev[i], hp->x_store), hp->stash_store);
         else if (hp->delay == 1)   /* the weights the next gradient is evaluated at */
             stash[i] = oracle_round(x[i], hp->stash_store);
-        if (use_ef)
+        if (use_ef && !updated)
             u_prev[i] = oracle_round(u, hp->x_store);
         x[i] = oracle_round(xn, hp->x_store);
         if (param != NULL)
@@ -434,6 +473,30 @@ int oracle_muon_step(int64_t rows, int64_t cols, int64_t t, const oracle_muon_hp
     }
     if (o_out != NULL)
         memcpy(o_out, O, sizeof(double) * (size_t)n);
+    if (updated) {
+        /* SAPipe-WP with the updated state (App. B.1): Alg. 2's step once
+         * more on G_{t-1} from the momentum the real step left, that momentum
+         * formed as the real step forms it (in its storage format), through
+         * a second Newton-Schulz, with decay on X_{t+1}. The history holds
+         * this prediction update; the momentum keeps the real step's. */
+        double *M2 = (double *)malloc(sizeof(double) * (size_t)n);
+        if (M2 == NULL) {
+            free(O);
+            return -1;
+        }
+        for (int64_t i = 0; i < n; ++i)
+            M2[i] = oracle_round(hp->momentum * mom[i] + (1.0 - hp->momentum) *
+                                 (clip_scale * g[i]), hp->x_store);
+        if (oracle_newton_schulz(rows, cols, M2, hp->ns_eps, hp->ns_a, hp->ns_b, hp->ns_c,
+                                 hp->ns_steps, hp->ns_store, O) != 0) {
+            free(M2);
+            free(O);
+            return -1;
+        }
+        for (int64_t i = 0; i < n; ++i)
+            u_prev[i] = oracle_round(hp->lr * (s * O[i] + hp->weight_decay * x[i]), hp->x_store);
+        free(M2);
+    }
     free(O);
     return 0;
 }

@@ -76,11 +76,14 @@ enum {
  *                  previous step, x~_t = x_t - u_{t-2} (the stash). u_prev
  *                  then holds u.
  *   SAPIPE_UPDATED App. B.1, SAPipe-WP with the updated state: as SAPIPE_SAME,
- *                  but the prediction update is the AdamW step at the next
+ *                  but the prediction update is the rule's step at the next
  *                  time index on the same gradient, from the state after the
- *                  real update (a temporary second blend of g into m and v,
- *                  bias corrections at k + 1, decay on x_{t+1}); u_prev holds
- *                  that prediction update. */
+ *                  real update (for AdamW a temporary second blend of g into m
+ *                  and v, bias corrections at k + 1, decay on x_{t+1}; NAdam
+ *                  also takes its momentum schedule at k + 1; Lion the sign of
+ *                  the beta1 blend of its updated momentum; Adan a zero
+ *                  gradient difference, its previous gradient being g itself);
+ *                  u_prev holds that prediction update. */
 enum { ORACLE_CORR_EF = 0, ORACLE_CORR_SAPIPE_SAME = 1, ORACLE_CORR_SAPIPE_UPDATED = 2 };
 
 typedef struct {
@@ -205,9 +208,13 @@ typedef struct {
     double rms_scale;      /* see above; 0 = no scaling */
     int ns_store;          /* storage of every Newton-Schulz matrix: F64 or BF16 */
     int delay;             /* 1 = one-step-delayed, 0 = synchronous */
-    int correction;        /* ORACLE_CORR_EF or ORACLE_CORR_SAPIPE_SAME (App. B.1: the
+    int correction;        /* ORACLE_CORR_EF, ORACLE_CORR_SAPIPE_SAME (App. B.1: the
                               weights take the standard rule, the stash receives the
-                              prediction point X_t - U_prev, the history U) */
+                              prediction point X_t - U_prev, the history U) or
+                              ORACLE_CORR_SAPIPE_UPDATED (the same, but the history
+                              receives the prediction update: Alg. 2's step once more
+                              on G_{t-1} from the updated momentum, with a second
+                              Newton-Schulz and decay on X_{t+1}) */
     int x_store;           /* storage of X, M and U_prev (F64 or F32) */
     int stash_store;       /* storage of the stash */
     int param_store;       /* storage of the latest-weights copy */
@@ -233,7 +240,8 @@ int oracle_newton_schulz(int64_t rows, int64_t cols, const double *M, double eps
  * iteration within the current delayed phase (>= 1). x, mom are updated in
  * place; u_prev (history, or NULL for the standard rule), stash (needed when
  * delay == 1) and param (or NULL) as in oracle_step. o_out, when not NULL,
- * receives the Newton-Schulz output O. Returns 0, or -1 on bad arguments.
+ * receives the Newton-Schulz output O of the real step. Returns 0, or -1 on
+ * bad arguments or no memory.
  */
 int oracle_muon_step(int64_t rows, int64_t cols, int64_t t, const oracle_muon_hparams *hp,
                      const double *g, double clip_scale, double *x, double *mom,

@@ -66,7 +66,7 @@ class MuonHParams:
     ns_store: int = BF16
     max_grad_norm: float = 0.0
     delay: int = 1
-    correction: int = 0   # CORR_EF, or CORR_SAPIPE_SAME (App. B.1)
+    correction: int = 0   # CORR_EF, CORR_SAPIPE_SAME or CORR_SAPIPE_UPDATED (App. B.1)
 
     def as_f32(self) -> "MuonHParams":
         """Every real rounded to fp32, as a device taking fp32 settings sees them."""

@@ -295,6 +295,57 @@ def test_muon_sapipe_same_state(lib):
                                    rtol=1e-9, atol=1e-15)
 
 
+@pytest.mark.parametrize("x_store,ns_store", [(F64, F64), (F32, BF16)])
+def test_muon_sapipe_updated_is_the_next_step_on_a_repeated_gradient(lib, x_store, ns_store):
+    """SAPipe-WP with the updated state (App. B.1) for Muon: the prediction
+    update stored after call k is, bitwise, the update that call k + 1 of a
+    run whose gradient k + 1 repeats gradient k stores (EF at lambda = 0:
+    the standard rule, keeping each update in its history): the same momentum
+    formed once more, the same Newton-Schulz, decay on X_{t+1}. Also with
+    fp32 state and bf16 Newton-Schulz iterates. The weights follow the
+    standard rule and the stash holds X_t - U_prev with U_prev the previous
+    prediction update."""
+    rng = np.random.default_rng(14)
+    x0 = rng.normal(size=(5, 8))
+    grads = [rng.normal(size=(5, 8)) for _ in range(5)]
+    kw = dict(x_store=x_store, stash_store=x_store, lib=lib)
+    sp = DelayedMuon([x0], _hp(correction=oracle.CORR_SAPIPE_UPDATED, ns_store=ns_store),
+                     ef=True, **kw)
+    std = DelayedMuon([x0], _hp(ns_store=ns_store), **kw)
+    for k in range(1, len(grads) + 1):
+        xt, hist = sp.x[0].copy(), sp.u_prev[0].copy()
+        sp.step([grads[k - 1]])
+        std.step([grads[k - 1]])
+        assert np.array_equal(sp.x[0], std.x[0])
+        assert np.array_equal(sp.stash[0], oracle.round_to(xt - hist, x_store, lib))
+        rep = DelayedMuon([x0], _hp(ef_lambda=0.0, ns_store=ns_store), ef=True, **kw)
+        for g in grads[:k] + [grads[k - 1]]:
+            rep.step([g])
+        assert np.array_equal(sp.u_prev[0], rep.u_prev[0])
+
+
+def test_muon_sapipe_updated_by_hand(lib):
+    """1 x 2 matrix, mu = 0.5, lr = 0.1, wd = 0, no RMS scaling, no
+    Newton-Schulz steps (O = M / ||M||), eps 0; gradients (3, 4), (4, -3).
+    Call 1: M = (1.5, 2), U = 0.1 (0.6, 0.8); prediction M' = (2.25, 3), the
+    same direction. Call 2: M = (2.75, -0.5), U = 0.1 M / sqrt(7.8125);
+    prediction M' = 0.5 M + 0.5 (4, -3) = (3.375, -1.75), so
+    U' = 0.1 M' / sqrt(14.453125), a direction the same state would miss.
+    Call 2 reads the stash X_1 - U'_1 = (0.88, 0.84)."""
+    hp = _hp(lr=0.1, momentum=0.5, weight_decay=0.0, rms_scale=0.0, ns_steps=0, ns_eps=0.0,
+             correction=oracle.CORR_SAPIPE_UPDATED)
+    o = DelayedMuon([np.array([[1.0, 1.0]])], hp, ef=True, x_store=F64, stash_store=F64, lib=lib)
+    o.step([np.array([[3.0, 4.0]])])
+    np.testing.assert_allclose(o.x[0], [[0.94, 0.92]], rtol=1e-15)
+    np.testing.assert_allclose(o.u_prev[0], [[0.06, 0.08]], rtol=1e-15)
+    o.step([np.array([[4.0, -3.0]])])
+    np.testing.assert_allclose(o.stash[0], [[0.88, 0.84]], rtol=1e-15)
+    u2 = 0.1 * np.array([2.75, -0.5]) / math.sqrt(7.8125)
+    np.testing.assert_allclose(o.x[0], [[0.94 - u2[0], 0.92 - u2[1]]], rtol=1e-15)
+    np.testing.assert_allclose(o.u_prev[0], [0.1 * np.array([3.375, -1.75]) /
+                                             math.sqrt(14.453125)], rtol=1e-15)
+
+
 def test_muon_ef_lambda_scales_the_correction(lib):
     """Eq. (1) for Muon's update: X_{t+1} = X_t - U - lambda (U - U_prev).
     At lambda = 0 the EF run is bitwise the standard one; at lambda = 1/2 the

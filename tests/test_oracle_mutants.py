@@ -46,8 +46,8 @@ MUTANTS = [
     ("sapipe_updated_bias_index", "bc1_next = 1.0 - pow(hp->beta1, (double)(k + 1))",
      "bc1_next = 1.0 - pow(hp->beta1, (double)k)"),
     ("sapipe_updated_decays_old_weights", "wd * oracle_round(xn, hp->x_store)", "wd * xt"),
-    ("sapipe_updated_no_second_blend", "hp->beta1 * mi + (1.0 - hp->beta1) * gi;",
-     "mi;"),
+    ("sapipe_updated_no_second_blend",
+     "const double m2 = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;", "const double m2 = m[i];"),
     ("delay_mask_ignored", "(delay_on == NULL || delay_on[i])", "(1)"),
     ("ef_restart_counts_all_steps", "corr == ORACLE_CORR_EF && t >= 2",
      "corr == ORACLE_CORR_EF && k >= 2"),
@@ -55,9 +55,30 @@ MUTANTS = [
      "pow(0.96, (double)k * hp->momentum_decay)"),
     ("lion_roles_swapped", "oracle_round(hp->beta2 * m[i] + (1.0 - hp->beta2) * gi, hp->x_store)",
      "oracle_round(hp->beta1 * m[i] + (1.0 - hp->beta1) * gi, hp->x_store)"),
-    ("adan_diff_sign", "gi - g_prev[i]", "g_prev[i] - gi"),
+    ("adan_diff_sign", "const double diff = k == 1 ? 0.0 : gi - g_prev[i];",
+     "const double diff = k == 1 ? 0.0 : g_prev[i] - gi;"),
     ("adan_no_lookahead", "gi + hp->beta2 * diff", "gi"),
     ("dc_sign", "(xt - stash[i])", "(stash[i] - xt)"),
+    # the updated-state prediction of the rules besides AdamW (App. B.1)
+    ("nadam_prediction_gradient_weight_at_k", "(1.0 - mu_next) / (1.0 - mu_prod_next) * gi / d2",
+     "(1.0 - mu_k) / (1.0 - mu_prod) * gi / d2"),
+    ("nadam_prediction_momentum_weight_at_k", "mu_next2 / (1.0 - mu_prod_next2) * nm / d2",
+     "mu_next / (1.0 - mu_prod_next) * nm / d2"),
+    ("nadam_prediction_bias_at_k", "sqrt(nv / bc2_next)", "sqrt(nv / bc2)"),
+    ("nadam_prediction_no_second_blend",
+     "const double nm = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;", "const double nm = m[i];"),
+    ("lion_prediction_is_the_current_update", "hist = hp->lr * (s2 + wd * x_next);",
+     "hist = u;"),
+    ("lion_prediction_roles_swapped",
+     "const double c2 = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;",
+     "const double c2 = hp->beta2 * m[i] + (1.0 - hp->beta2) * gi;"),
+    ("adan_prediction_difference_not_decayed",
+     "const double av = hp->beta2 * v[i] + (1.0 - hp->beta2) * ad;", "const double av = v[i];"),
+    ("adan_prediction_momentum_unblended",
+     "const double am = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;", "const double am = m[i];"),
+    ("adan_prediction_bias_at_k", "sqrt(an / bc3_next)", "sqrt(an / bc3)"),
+    ("prediction_decays_old_weights_other_rules",
+     "const double x_next = oracle_round(xn, hp->x_store);", "const double x_next = xt;"),
     # delayed Muon (Alg. 2) and its Newton-Schulz iteration
     ("ns_coefficient_roles", "AA[i] = oracle_round(b * A[i] + c * AA[i], store);",
      "AA[i] = oracle_round(c * A[i] + b * AA[i], store);"),
@@ -72,6 +93,13 @@ MUTANTS = [
     ("muon_momentum_roles",
      "hp->momentum * mom[i] + (1.0 - hp->momentum) * (clip_scale * g[i])",
      "(1.0 - hp->momentum) * mom[i] + hp->momentum * (clip_scale * g[i])"),
+    ("muon_sapipe_updated_no_second_blend",
+     "M2[i] = oracle_round(hp->momentum * mom[i] + (1.0 - hp->momentum) *\n"
+     "                                 (clip_scale * g[i]), hp->x_store);",
+     "M2[i] = mom[i];"),
+    ("muon_sapipe_updated_decays_the_stash",
+     "hp->weight_decay * x[i]), hp->x_store);", "hp->weight_decay * stash[i]), hp->x_store);"),
+    ("muon_sapipe_updated_keeps_the_real_update", "    if (updated) {", "    if (0) {"),
     ("muon_scale_smaller_dim", "sqrt((double)(rows > cols ? rows : cols))",
      "sqrt((double)(rows < cols ? rows : cols))"),
     ("muon_decay_on_stash", "hp->lr * (s * O[i] + hp->weight_decay * xt)",
@@ -119,8 +147,9 @@ MUTANTS = [
      "(1.0 - mu_k) / (1.0 - mu_prod) * g[i] / d"),
     ("lion_blend_unclipped", "const double c = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;",
      "const double c = hp->beta1 * m[i] + (1.0 - hp->beta1) * g[i];"),
-    ("sapipe_updated_blend_unclipped", "const double m2 = hp->beta1 * mi + (1.0 - hp->beta1) * gi;",
-     "const double m2 = hp->beta1 * mi + (1.0 - hp->beta1) * g[i];"),
+    ("sapipe_updated_blend_unclipped",
+     "const double m2 = hp->beta1 * m[i] + (1.0 - hp->beta1) * gi;",
+     "const double m2 = hp->beta1 * m[i] + (1.0 - hp->beta1) * g[i];"),
     ("synchronous_tensor_stash_written", "        if (delayed) {\n            if (corr == ORACLE_CORR_EF)",
      "        if (hp->delay == 1) {\n            if (corr == ORACLE_CORR_EF)"),
     ("lion_sign_after_momentum_update",

@@ -625,6 +625,119 @@ def test_sapipe_updated_hand_steps(lib):
                                         rel=1e-14)
 
 
+def _rule_run(lib, rule, correction, grads, x0, ef=True, max_norm=0.0, store=F64, **kw):
+    hp = HParams(lr=kw.pop("lr", 0.01), weight_decay=kw.pop("wd", 0.1), rule=rule,
+                 correction=correction, max_grad_norm=max_norm, **kw)
+    o = oracle.DelayedOptimizer([x0], hp, ef=ef, x_store=store, stash_store=store, lib=lib)
+    hist = []
+    for g in grads:
+        o.step(g, tag=o.read_weights()[1])
+        hist.append(dict(x=o.x.copy(), stash=o.stash.copy(),
+                         u=o.u_prev.copy() if ef else None))
+    return hist
+
+
+RULE_KW = {oracle.RULE_ADAMW: {}, oracle.RULE_NADAM: dict(momentum_decay=0.004),
+           oracle.RULE_LION: dict(beta1=0.9, beta2=0.99),
+           oracle.RULE_ADAN: dict(beta1=0.98, beta2=0.92, beta3=0.99),
+           oracle.RULE_SGD: {}}
+
+
+@pytest.mark.parametrize("rule", sorted(RULE_KW))
+@pytest.mark.parametrize("max_norm,store", [(0.0, F64), (3.0, F64), (0.0, F32)])
+def test_sapipe_updated_prediction_is_the_next_step_on_a_repeated_gradient(lib, rule, max_norm,
+                                                                          store):
+    """App. B.1's updated-state prediction is the optimizer's own step taken
+    once more on the same gradient from the state the real step left: for
+    every rule, the prediction update stored after call k equals, bitwise,
+    the update stored by call k + 1 of a run whose gradient k + 1 repeats
+    gradient k. That run is EF at lambda = 0, which is the standard rule
+    bitwise and keeps each update in its history buffer; the SAPipe run's
+    weights follow the standard rule too, so both runs start call k + 1 from
+    the same stored state. With clipping (norms about 8 against 3) the
+    repeated gradient takes the same coefficient; with fp32 storage the
+    prediction reads the statistics as stored."""
+    rng = np.random.default_rng(31)
+    n, steps = 48, 6
+    x0 = rng.normal(0, 0.5, n)
+    grads = [rng.normal(0, 1.0, n) for _ in range(steps)]
+    sp = _rule_run(lib, rule, oracle.CORR_SAPIPE_UPDATED, grads, x0, max_norm=max_norm,
+                   store=store, **RULE_KW[rule])
+    for k in range(1, steps + 1):
+        rep = _rule_run(lib, rule, oracle.CORR_EF, grads[:k] + [grads[k - 1]], x0,
+                        max_norm=max_norm, store=store, ef_lambda=0.0, **RULE_KW[rule])
+        np.testing.assert_array_equal(sp[k - 1]["x"], rep[k - 1]["x"])
+        np.testing.assert_array_equal(sp[k - 1]["u"], rep[k]["u"])
+
+
+@pytest.mark.parametrize("max_norm", [0.0, 1.5])
+def test_sapipe_updated_nadam_is_torch_nadam_stepped_again(lib, f64_default, max_norm):
+    """NAdam's prediction update is what torch.optim.NAdam (decoupled decay)
+    applies when stepped once more on the same (clipped) gradient from a copy
+    of the state its real step left: moments, step count and the running
+    product of its momentum schedule."""
+    rng = np.random.default_rng(33)
+    x0 = rng.normal(0, 0.5, 40)
+    grads = [rng.normal(0, 0.7, 40) for _ in range(7)]
+    hist = _rule_run(lib, oracle.RULE_NADAM, oracle.CORR_SAPIPE_UPDATED, grads, x0,
+                     max_norm=max_norm, lr=2e-2, momentum_decay=0.004)
+    kw = dict(lr=2e-2, betas=(0.9, 0.95), eps=1e-8, weight_decay=0.1, momentum_decay=0.004,
+              decoupled_weight_decay=True, foreach=False)
+    p = torch.nn.Parameter(torch.tensor(x0))
+    opt = torch.optim.NAdam([p], **kw)
+    for k, g in enumerate(grads):
+        p.grad = torch.tensor(g)
+        if max_norm > 0:
+            torch.nn.utils.clip_grad_norm_([p], max_norm)
+        gc = p.grad.clone()
+        opt.step()
+        np.testing.assert_allclose(p.detach().numpy(), hist[k]["x"], rtol=1e-12)
+        q = torch.nn.Parameter(p.detach().clone())
+        opt2 = torch.optim.NAdam([q], **kw)
+        opt2.state[q] = {key: val.clone() for key, val in opt.state[p].items()}
+        q.grad = gc
+        opt2.step()
+        np.testing.assert_allclose(hist[k]["u"], p.detach().numpy() - q.detach().numpy(),
+                                   rtol=1e-10, atol=1e-16)
+
+
+def test_sapipe_updated_lion_hand_steps(lib):
+    """Lion, beta = (0.5, 0.5), lr = 0.1, wd = 0, x0 = 1, gradients -2, 0.5, 0.5.
+    Call 1: c = -1 (u = -0.1, x = 1.1), m = -1; prediction c' = 0.5(-1) +
+    0.5(-2) = -1.5, so -0.1. Call 2: c = -0.25 (u = -0.1, x = 1.2), m = -0.25;
+    prediction c' = -0.125 + 0.25 = 0.125, so +0.1: the updated state flips
+    the sign the same state would keep. Call 3 reads the stash
+    x_3 - u'_2 = 1.2 - 0.1 = 1.1 (same state: 1.3)."""
+    hist = _rule_run(lib, oracle.RULE_LION, oracle.CORR_SAPIPE_UPDATED,
+                     [np.array([-2.0]), np.array([0.5]), np.array([0.5])], np.array([1.0]),
+                     lr=0.1, wd=0.0, beta1=0.5, beta2=0.5)
+    assert [h["x"][0] for h in hist[:2]] == pytest.approx([1.1, 1.2], abs=1e-15)
+    assert [h["u"][0] for h in hist[:2]] == pytest.approx([-0.1, 0.1], abs=1e-15)
+    assert hist[1]["stash"][0] == pytest.approx(1.2, abs=1e-15)
+    assert hist[2]["stash"][0] == pytest.approx(1.1, abs=1e-15)
+
+
+def test_sapipe_updated_adan_hand_steps(lib):
+    """Adan, beta = (0.98, 0.92, 0.99), lr = 0.1, eps = 0, wd = 0, x0 = 1,
+    gradients 2, then 1. Call 1: m = 0.04, v = 0 (no difference yet),
+    n = 0.04, u = 0.1; the prediction at k = 2 (difference 0: the stored
+    previous gradient is 2 itself) from m' = 0.0792, v' = 0, n' = 0.0796 is
+    0.1 (0.0792/0.0396) / sqrt(0.0796/0.0199) = 0.1. Call 2: diff = -1,
+    m = 0.0592, v = -0.08, n = 0.039664; prediction at k = 3 from
+    m' = 0.078016, v' = 0.92(-0.08) = -0.0736, n' = 0.04926736 with
+    1 - beta^3 = 0.058808, 0.221312, 0.029701."""
+    hist = _rule_run(lib, oracle.RULE_ADAN, oracle.CORR_SAPIPE_UPDATED,
+                     [np.array([2.0]), np.array([1.0])], np.array([1.0]), lr=0.1, wd=0.0,
+                     eps=0.0, beta1=0.98, beta2=0.92, beta3=0.99)
+    assert hist[0]["u"][0] == pytest.approx(0.1, rel=1e-14)
+    pred2 = 0.1 * ((0.078016 / 0.058808 + 0.92 * -0.0736 / 0.221312) /
+                   math.sqrt(0.04926736 / 0.029701))
+    assert hist[1]["u"][0] == pytest.approx(pred2, rel=1e-12)
+    # the real second update, for contrast (1 - beta^2 = 0.0396, 0.1536, 0.0199)
+    u2 = 0.1 * ((0.0592 / 0.0396 + 0.92 * -0.08 / 0.1536) / math.sqrt(0.039664 / 0.0199))
+    assert hist[1]["x"][0] == pytest.approx(0.9 - u2, rel=1e-13)
+
+
 # ------------------------------- per-tensor delay and mode switches (Sec. 3.1,
 # App. A.9 synchronous LM head, App. B.2 WPipe)
 
