@@ -97,11 +97,15 @@ typedef enum { DPO_F32 = 0, DPO_BF16 = 1 } dpo_dtype;
  *                            at the previous step, x_t - u_prev; the buffer then
  *                            holds u.
  *   DPO_CORR_SAPIPE_UPDATED  App. B.1 with the updated state: as above, but the
- *                            buffer holds the prediction update: the AdamW step
+ *                            buffer holds the prediction update: the rule's step
  *                            at the next time index on the same gradient, from
- *                            the state the real update left (moments blended
- *                            with g once more, bias corrections at k + 1, decay
- *                            on x_{t+1}), not kept in m and v. */
+ *                            the state the real update left (for AdamW the
+ *                            moments blended with g once more, bias corrections
+ *                            at k + 1, decay on x_{t+1}; NAdam also takes its
+ *                            momentum schedule at k + 1, Lion the sign of the
+ *                            beta1 blend of its updated momentum, Adan a zero
+ *                            gradient difference), not kept in the statistics.
+ *                            Every rule. */
 #define DPO_CORR_EF 0
 #define DPO_CORR_SAPIPE_SAME 1
 #define DPO_CORR_SAPIPE_UPDATED 2

@@ -299,8 +299,6 @@ extern "C" int dpo_init(dpo_ctx **out, const dpo_tensor *table, int n_tensors,
         return fail(nullptr, DPO_EINVAL, "beta3 must lie in [0, 1)");
     if (hp->optimizer == DPO_OPT_NADAM && hp->momentum_decay < 0.0f)
         return fail(nullptr, DPO_EINVAL, "momentum_decay must be >= 0");
-    if (hp->correction == DPO_CORR_SAPIPE_UPDATED && hp->optimizer != DPO_OPT_ADAMW)
-        return fail(nullptr, DPO_EINVAL, "the SAPipe updated-state prediction is defined for AdamW");
     if (hp->stash_mode != DPO_STASH_COPY && hp->stash_mode != DPO_STASH_PINGPONG)
         return fail(nullptr, DPO_EINVAL, "stash_mode must be one of DPO_STASH_*");
     if (hp->stash_mode == DPO_STASH_PINGPONG) {
@@ -656,6 +654,12 @@ extern "C" int dpo_step(dpo_ctx *c, float lr, void *cuda_stream)
         a.omb3 = (float)(1.0 - b3);
         a.inv_sqrt_bc3 = (float)(1.0 / std::sqrt(1.0 - std::pow(b3, (double)k)));
         a.adan_c2 = (float)(lrd * b2 / bc2);
+        // the same at the next index, for the SAPipe updated-state prediction
+        const double mu_next2 = nadam_mu(c->hp, k + 2);
+        a.nadam_cg_next = (float)(lrd * (1.0 - mu_next) / (1.0 - mu_prod * mu_next));
+        a.nadam_cm_next = (float)(lrd * mu_next2 / (1.0 - mu_prod * mu_next * mu_next2));
+        a.inv_sqrt_bc3_next = (float)(1.0 / std::sqrt(1.0 - std::pow(b3, (double)(k + 1))));
+        a.adan_c2_next = (float)(lrd * b2 / (1.0 - std::pow(b2, (double)(k + 1))));
         a.first = k == 1;
         a.dc_lambda = c->hp.delay == 1 ? c->hp.dc_lambda : 0.0f;
         // Ping-pong: call t of the delayed phase writes the new weights of

@@ -24,10 +24,10 @@ constexpr int kAlign = 32;      // buffer alignment: fp32 packets move as 256-bi
 // to keep HBM3e busy, not so many that DRAM efficiency drops.
 constexpr int kStepThreads = 128;
 
-// Gradient-norm kernel: one read stream, so each thread loads
-// kNormUnroll packets per iteration.
+// Gradient-norm kernel: one read stream, so each thread keeps up to
+// kNormUnroll packets (bf16; half as many fp32 ones) in flight per round.
 constexpr int kNormThreads = 256;
-constexpr int kNormUnroll = 4;
+constexpr int kNormUnroll = 8;
 
 // Device copy of one table entry.
 struct DevTensor {
@@ -59,6 +59,7 @@ enum Optimizer { kOptAdamW = 0, kOptNAdam = 1, kOptLion = 2, kOptAdan = 3 };
 struct StepScalars {
     float step_size, inv_sqrt_bc2, lr_wd, lam, step_size_next, inv_sqrt_bc2_next, lr;
     float nadam_cg, nadam_cm, inv_sqrt_bc3, adan_c2;
+    float nadam_cg_next, nadam_cm_next, inv_sqrt_bc3_next, adan_c2_next;
     int first, swap;
 };
 
@@ -98,6 +99,10 @@ struct StepArgs {
     float beta3, omb3;          // Adan: beta3, 1 - beta3
     float inv_sqrt_bc3;         // Adan: 1 / sqrt(1 - beta3^k)
     float adan_c2;              // Adan: lr beta2 / (1 - beta2^k)
+    // the same at the next index k + 1 (SAPipe updated state)
+    float nadam_cg_next, nadam_cm_next;   // lr (1-mu_{k+1})/(1-prod_{k+1}), lr mu_{k+2}/(1-prod_{k+2})
+    float inv_sqrt_bc3_next;    // Adan: 1 / sqrt(1 - beta3^(k+1))
+    float adan_c2_next;         // Adan: lr beta2 / (1 - beta2^(k+1))
     int first;                  // Adan: k == 1 (the gradient difference is 0)
     float dc_lambda;            // DC-ASGD strength (0: off)
     int swap;                   // ping-pong stash: write delayed tensors' weights into

@@ -48,38 +48,60 @@ template <int GB>
 __global__ void __launch_bounds__(kNormThreads) grad_sqnorm_kernel(const NormArgs a)
 {
     using GT = typename Elem<GB != 0>::T;
+    constexpr int U = NormUnroll<GT>::value;
     __shared__ double red[kNormThreads / 32];
     __shared__ bool last;
 
-    // Each thread takes kNormUnroll packets per round, kNormThreads apart, so
-    // their loads are in flight together; rounds are grid-stride, and each of
-    // the kNormUnroll packet streams keeps its own tensor cursor.
-    const int64_t round = (int64_t)gridDim.x * kNormThreads * kNormUnroll;
-    const int64_t first = (int64_t)blockIdx.x * kNormThreads * kNormUnroll + threadIdx.x;
+    // Each thread takes U packets per round, kNormThreads apart, and issues
+    // the loads of all of them before it sums any; rounds are grid-stride.
+    // The packets of a round and of the rounds after it have growing
+    // indices, so one forward-moving tensor cursor serves them all, and a
+    // tensor's gradient pointer and length are read only when the cursor
+    // enters it.
+    const int64_t round = (int64_t)gridDim.x * kNormThreads * U;
+    const int64_t first = (int64_t)blockIdx.x * kNormThreads * U + threadIdx.x;
     float sum = 0.0f, comp = 0.0f;
     if (first < a.total_pkts) {
-        Cursor c[kNormUnroll];
-#pragma unroll
-        for (int u = 0; u < kNormUnroll; ++u) {
-            const int64_t p = first + (int64_t)u * kNormThreads;
-            c[u].seek(a.pkt_begin, a.n_tensors, p < a.total_pkts ? p : a.total_pkts - 1);
-        }
+        Cursor c;
+        c.seek(a.pkt_begin, a.n_tensors, first);
+        const GT *grad = static_cast<const GT *>(a.table[c.t].grad);
+        int64_t numel = a.table[c.t].numel;
         for (int64_t base = first; base < a.total_pkts; base += round) {
-            float part[kNormUnroll];
+            const GT *ptr[U];
+            int cnt[U];   // elements of the packet: 8, 1..7 (a tensor's last), 0 (none)
 #pragma unroll
-            for (int u = 0; u < kNormUnroll; ++u) {
+            for (int u = 0; u < U; ++u) {
                 const int64_t p = base + (int64_t)u * kNormThreads;
-                part[u] = 0.0f;
+                ptr[u] = grad;
+                cnt[u] = 0;
                 if (p < a.total_pkts) {
-                    c[u].advance(a.pkt_begin, p);
-                    const DevTensor &d = a.table[c[u].t];
-                    part[u] = packet_sqsum(static_cast<const GT *>(d.grad),
-                                           (p - c[u].tb) * kPacket, d.numel);
+                    if (c.advance(a.pkt_begin, p)) {
+                        grad = static_cast<const GT *>(a.table[c.t].grad);
+                        numel = a.table[c.t].numel;
+                    }
+                    const int64_t e = (p - c.tb) * kPacket;
+                    ptr[u] = grad + e;
+                    cnt[u] = numel - e < kPacket ? (int)(numel - e) : kPacket;
                 }
             }
+            RawPacket<GT> raw[U];
 #pragma unroll
-            for (int u = 0; u < kNormUnroll; ++u)
-                kahan_add(sum, comp, part[u]);
+            for (int u = 0; u < U; ++u)
+                if (cnt[u] == kPacket)
+                    raw[u].load(ptr[u]);
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                float s = 0.0f;
+                if (cnt[u] == kPacket) {
+                    s = raw[u].sqsum();
+                } else {
+                    for (int i = 0; i < cnt[u]; ++i) {
+                        const float x = ld1(ptr[u] + i);
+                        s += x * x;
+                    }
+                }
+                kahan_add(sum, comp, s);
+            }
         }
     }
     const double cta = block_sum<kNormThreads>((double)sum - (double)comp, red);
@@ -259,6 +281,11 @@ __global__ void step_scalars_kernel(StepCounters *cnt, const float *lr_src, floa
     sc.nadam_cm = (float)(lrd * mu_next / (1.0 - mu_prod * mu_next));
     sc.inv_sqrt_bc3 = (float)(1.0 / sqrt(1.0 - pow(k.beta3, (double)kk)));
     sc.adan_c2 = (float)(lrd * k.beta2 / bc2);
+    const double mu_next2 = nadam_mu_dev(k, kk + 2);
+    sc.nadam_cg_next = (float)(lrd * (1.0 - mu_next) / (1.0 - mu_prod * mu_next));
+    sc.nadam_cm_next = (float)(lrd * mu_next2 / (1.0 - mu_prod * mu_next * mu_next2));
+    sc.inv_sqrt_bc3_next = (float)(1.0 / sqrt(1.0 - pow(k.beta3, (double)(kk + 1))));
+    sc.adan_c2_next = (float)(lrd * k.beta2 / (1.0 - pow(k.beta2, (double)(kk + 1))));
     sc.first = kk == 1;
     sc.swap = k.pingpong && (t & 1) != 0;
     *out = sc;

@@ -40,13 +40,15 @@ namespace {
 
 using dpo::block_sum;
 using dpo::kahan_add;
-using dpo::packet_sqsum;
+using dpo::NormUnroll;
+using dpo::RawPacket;
 
 constexpr int kThreads = 256;
-constexpr int kUnroll = 4;
 constexpr int64_t kChunkElems = DPO_NOALLOC_CHUNK_ELEMS;
 constexpr int kMaxChunks = DPO_NOALLOC_MAX_CHUNKS;
-constexpr int64_t kMinChunk = (int64_t)kThreads * kUnroll * dpo::kPacket;   // 8192
+// one round of a CTA's loads of bf16 packets (two of fp32 ones)
+constexpr int64_t kMinChunk =
+    (int64_t)kThreads * NormUnroll<__nv_bfloat16>::value * dpo::kPacket;   // 16384
 constexpr int64_t kTargetCtas = 1216;   // 8 per SM on a 152-SM GB300
 constexpr size_t kTicketOffset = sizeof(double) * kMaxChunks;
 constexpr size_t kScratchBytes = kTicketOffset + 256;
@@ -87,11 +89,11 @@ cudaError_t scratch_address(int device, void **out)
 }
 
 // CTA c sums the squares of chunk c, elements [c chunk, min((c+1) chunk,
-// numel)) (8-element packets, kUnroll packets in flight per thread, Kahan
-// fp32 per thread, fp64 block tree), stores the partial in the scratch array,
-// and the last CTA to arrive adds the partials in chunk order and writes the
-// norm and the clip coefficient min(1, max_norm / (norm + 1e-6)).
-// Deterministic for a given numel.
+// numel)) (8-element packets; each thread issues the loads of its U packets
+// of a round before summing them; Kahan fp32 per thread, fp64 block tree),
+// stores the partial in the scratch array, and the last CTA to arrive adds
+// the partials in chunk order and writes the norm and the clip coefficient
+// min(1, max_norm / (norm + 1e-6)). Deterministic for a given numel.
 template <class GT>
 __global__ void __launch_bounds__(kThreads)
 noalloc_sqnorm_kernel(const GT *__restrict__ grad, int64_t numel, int64_t chunk,
@@ -106,17 +108,34 @@ noalloc_sqnorm_kernel(const GT *__restrict__ grad, int64_t numel, int64_t chunk,
     const int64_t lo = (int64_t)blockIdx.x * chunk;
     const int64_t hi = lo + chunk < numel ? lo + chunk : numel;
     const int64_t pkts = hi > lo ? (hi - lo + dpo::kPacket - 1) / dpo::kPacket : 0;
+    constexpr int U = NormUnroll<GT>::value;
     float sum = 0.0f, comp = 0.0f;
-    for (int64_t base = threadIdx.x; base < pkts; base += (int64_t)kThreads * kUnroll) {
-        float part[kUnroll];
+    for (int64_t base = threadIdx.x; base < pkts; base += (int64_t)kThreads * U) {
+        int cnt[U];   // elements of the packet: 8, 1..7 (the buffer's last), 0 (none)
+        RawPacket<GT> raw[U];
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
-            const int64_t q = base + (int64_t)u * kThreads;
-            part[u] = q < pkts ? packet_sqsum(grad, lo + q * dpo::kPacket, hi) : 0.0f;
+        for (int u = 0; u < U; ++u) {
+            const int64_t e = lo + (base + (int64_t)u * kThreads) * dpo::kPacket;
+            cnt[u] = e < hi ? (hi - e < dpo::kPacket ? (int)(hi - e) : dpo::kPacket) : 0;
         }
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u)
-            kahan_add(sum, comp, part[u]);
+        for (int u = 0; u < U; ++u)
+            if (cnt[u] == dpo::kPacket)
+                raw[u].load(grad + lo + (base + (int64_t)u * kThreads) * dpo::kPacket);
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            float s = 0.0f;
+            if (cnt[u] == dpo::kPacket) {
+                s = raw[u].sqsum();
+            } else {
+                const GT *p = grad + lo + (base + (int64_t)u * kThreads) * dpo::kPacket;
+                for (int i = 0; i < cnt[u]; ++i) {
+                    const float x = dpo::ld1(p + i);
+                    s += x * x;
+                }
+            }
+            kahan_add(sum, comp, s);
+        }
     }
     const double cta = block_sum<kThreads>((double)sum - (double)comp, red);
     if (threadIdx.x == 0) {

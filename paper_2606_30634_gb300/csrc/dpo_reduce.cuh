@@ -30,6 +30,46 @@ __device__ __forceinline__ float packet_sqsum(const GT *grad, int64_t e, int64_t
     return s;
 }
 
+// One full packet held as loaded (bf16: 16 bytes, fp32: 32 bytes), so that a
+// thread can issue the loads of several packets before it sums any of them;
+// sqsum() is packet_sqsum's tree for a full packet.
+template <class GT> struct RawPacket;
+
+template <> struct RawPacket<__nv_bfloat16> {
+    uint4 q;
+    __device__ __forceinline__ void load(const __nv_bfloat16 *p)
+    {
+        q = __ldcs(reinterpret_cast<const uint4 *>(p));
+    }
+    __device__ __forceinline__ float sqsum() const
+    {
+        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+        float g[8];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            g[2 * j] = __uint_as_float(w[j] << 16);
+            g[2 * j + 1] = __uint_as_float(w[j] & 0xFFFF0000u);
+        }
+        return ((g[0] * g[0] + g[1] * g[1]) + (g[2] * g[2] + g[3] * g[3])) +
+               ((g[4] * g[4] + g[5] * g[5]) + (g[6] * g[6] + g[7] * g[7]));
+    }
+};
+
+template <> struct RawPacket<float> {
+    float g[8];
+    __device__ __forceinline__ void load(const float *p) { ld8(p, g); }
+    __device__ __forceinline__ float sqsum() const
+    {
+        return ((g[0] * g[0] + g[1] * g[1]) + (g[2] * g[2] + g[3] * g[3])) +
+               ((g[4] * g[4] + g[5] * g[5]) + (g[6] * g[6] + g[7] * g[7]));
+    }
+};
+
+// Packets a thread keeps in flight per round of a norm pass: 128 bytes of
+// gradient either way (eight bf16 packets, four fp32 packets).
+template <class GT> struct NormUnroll { static constexpr int value = 4; };
+template <> struct NormUnroll<__nv_bfloat16> { static constexpr int value = 8; };
+
 // Kahan-compensated fp32 accumulation of per-packet sums of squares: the
 // compensation keeps a thread's error near one rounding however many
 // packets it visits.

@@ -21,6 +21,7 @@ struct Scalars {
     float step_size_next, inv_sqrt_bc2_next;
     float lr, nadam_cg, nadam_cm;
     float beta3, omb3, inv_sqrt_bc3, adan_c2;
+    float nadam_cg_next, nadam_cm_next, inv_sqrt_bc3_next, adan_c2_next;
     bool first;
 };
 
@@ -74,16 +75,39 @@ __device__ __forceinline__ float rule_update(const Scalars &s, float g, float x,
     }
 }
 
-// SAPipe-WP with the updated state (App. B.1, AdamW): the AdamW update at the
-// next time index on the same gradient g, from the moments m, v the real
-// update left (blended with g once more into temporaries), decaying x_{t+1}.
-__device__ __forceinline__ float adamw_prediction(const Scalars &s, float g, float x_next,
-                                                  float wd_lr, float m, float v)
+// SAPipe-WP with the updated state (App. B.1): the rule's update at the next
+// time index k + 1 on the same gradient g, from the statistics m, v, n, gp
+// the real update left (blended with g once more into temporaries), decaying
+// x_{t+1}. Adan's stored previous gradient is g itself, so its difference is
+// zero.
+template <int OPT>
+__device__ __forceinline__ float rule_prediction(const Scalars &s, float g, float x_next,
+                                                 float wd_lr, float m, float v, float n,
+                                                 float gp)
 {
-    const float m2 = ema_exact(s.beta1, s.omb1, m, g);
-    const float v2 = fmaf(s.beta2, v, (s.omb2 * g) * g);
-    const float denom = fmaf(sqrtf(v2), s.inv_sqrt_bc2_next, s.eps);
-    return fmaf(s.step_size_next, m2 / denom, wd_lr * x_next);
+    if (OPT == kOptAdamW) {
+        const float m2 = ema_exact(s.beta1, s.omb1, m, g);
+        const float v2 = fmaf(s.beta2, v, (s.omb2 * g) * g);
+        const float denom = fmaf(sqrtf(v2), s.inv_sqrt_bc2_next, s.eps);
+        return fmaf(s.step_size_next, m2 / denom, wd_lr * x_next);
+    } else if (OPT == kOptNAdam) {
+        const float m2 = ema_exact(s.beta1, s.omb1, m, g);
+        const float v2 = fmaf(s.beta2, v, (s.omb2 * g) * g);
+        const float denom = fmaf(sqrtf(v2), s.inv_sqrt_bc2_next, s.eps);
+        return fmaf(s.nadam_cg_next, g, s.nadam_cm_next * m2) / denom + wd_lr * x_next;
+    } else if (OPT == kOptLion) {
+        const float c = ema_exact(s.beta1, s.omb1, m, g);
+        const float sgn = c > 0.0f ? 1.0f : (c < 0.0f ? -1.0f : 0.0f);
+        return fmaf(s.lr, sgn, wd_lr * x_next);
+    } else {   // Adan
+        const float diff = g - gp;
+        const float m2 = ema_exact(s.beta1, s.omb1, m, g);
+        const float v2 = ema_exact(s.beta2, s.omb2, v, diff);
+        const float w = fmaf(s.beta2, diff, g);
+        const float n2 = fmaf(s.beta3, n, (s.omb3 * w) * w);
+        const float denom = fmaf(sqrtf(n2), s.inv_sqrt_bc3_next, s.eps);
+        return fmaf(s.step_size_next, m2, s.adan_c2_next * v2) / denom + wd_lr * x_next;
+    }
 }
 
 // Displacement of the lambda-scaled EF rule, x_{t+1} = x_t - (u + lambda (u - u_prev)):
@@ -128,12 +152,14 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
     // values step_scalars_kernel left in device memory for this call.
     StepScalars sc{a.step_size, a.inv_sqrt_bc2, a.lr_wd, a.lam, a.step_size_next,
                    a.inv_sqrt_bc2_next, a.lr, a.nadam_cg, a.nadam_cm, a.inv_sqrt_bc3, a.adan_c2,
+                   a.nadam_cg_next, a.nadam_cm_next, a.inv_sqrt_bc3_next, a.adan_c2_next,
                    a.first, a.swap};
     if (a.dev != nullptr)
         sc = *a.dev;
     const Scalars s{a.beta1, a.omb1, a.beta2, a.omb2, sc.step_size, sc.inv_sqrt_bc2, a.eps, sc.lam,
                     sc.step_size_next, sc.inv_sqrt_bc2_next, sc.lr, sc.nadam_cg, sc.nadam_cm,
-                    a.beta3, a.omb3, sc.inv_sqrt_bc3, sc.adan_c2, sc.first != 0};
+                    a.beta3, a.omb3, sc.inv_sqrt_bc3, sc.adan_c2, sc.nadam_cg_next,
+                    sc.nadam_cm_next, sc.inv_sqrt_bc3_next, sc.adan_c2_next, sc.first != 0};
     const float clip = a.clip != nullptr ? __ldg(a.clip) : 1.0f;
     const bool use_prev = kSapipe || (CORR == kCorrEF && sc.lam != 0.0f);
     const bool ef_now = CORR == kCorrEF && sc.lam != 0.0f;
@@ -202,7 +228,7 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
                 u[j] = rule_update<OPT>(s, gc, x[j], wd_lr, m[j], v[j], n[j], gp[j]);
                 x[j] -= efn_t ? ef_displacement(s.lam, u[j], up[j]) : u[j];
                 if (CORR == kCorrSapipeUpdated)
-                    u[j] = adamw_prediction(s, gc, x[j], wd_lr, m[j], v[j]);
+                    u[j] = rule_prediction<OPT>(s, gc, x[j], wd_lr, m[j], v[j], n[j], gp[j]);
             }
             st8(master + e, x);
             st8(mm + e, m);
@@ -231,7 +257,7 @@ __global__ void __launch_bounds__(kStepThreads) fused_step_kernel(const StepArgs
                 float u = rule_update<OPT>(s, g, x, wd_lr, m, v, n, gp);
                 x -= efn_t ? ef_displacement(s.lam, u, up) : u;
                 if (CORR == kCorrSapipeUpdated)
-                    u = adamw_prediction(s, g, x, wd_lr, m, v);
+                    u = rule_prediction<OPT>(s, g, x, wd_lr, m, v, n, gp);
                 master[i] = x;
                 mm[i] = m;
                 if (kV)
@@ -267,10 +293,8 @@ StepFn pick_step_corr(Correction corr, bool pp)
         return fused_step_kernel<PB, SK, GB, kCorrEF, OPT, DC, 0>;
     case kCorrSapipeSame:
         return pp ? nullptr : fused_step_kernel<PB, SK, GB, kCorrSapipeSame, OPT, DC, 0>;
-    case kCorrSapipeUpdated:   // the prediction step is defined for AdamW
-        return pp || OPT != kOptAdamW
-                   ? nullptr
-                   : fused_step_kernel<PB, SK, GB, kCorrSapipeUpdated, OPT, DC, 0>;
+    case kCorrSapipeUpdated:
+        return pp ? nullptr : fused_step_kernel<PB, SK, GB, kCorrSapipeUpdated, OPT, DC, 0>;
     }
     return nullptr;
 }

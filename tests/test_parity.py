@@ -583,9 +583,12 @@ RULES = {
 
 @pytest.mark.parametrize("rule", sorted(RULES))
 @pytest.mark.parametrize("ef,corr", [(False, dpo.DPO_CORR_EF), (True, dpo.DPO_CORR_EF),
-                                     (True, SP_SAME)])
+                                     (True, SP_SAME), (True, SP_UPD)])
 @pytest.mark.parametrize("pdt,sdt,gdt", [(B, B, B), (B, F, B), (F, F, F)])
 def test_rule_parity(cuda_device, rule, ef, corr, pdt, sdt, gdt):
+    """NAdam, Lion and Adan under the standard rule, EF and both SAPipe-WP
+    predictions (the updated state: each rule's own step at k + 1), with
+    clipping, in every layout."""
     run = Run(Case(RAGGED, param_dtype=pdt, stash_dtype=sdt, grad_dtype=gdt, ef=ef,
                    correction=corr, max_grad_norm=0.3, **RULES[rule]), cuda_device)
     try:
@@ -669,18 +672,15 @@ def test_dc_asgd_step_on_identical_inputs(cuda_device, dc, sdt):
         opt.close()
 
 
-def test_sapipe_updated_state_needs_adamw(cuda_device):
-    with pytest.raises(dpo.DpoError) as e:
-        dpo.DelayedAdamW([100], ef=True, correction=SP_UPD, optimizer=dpo.DPO_OPT_LION,
-                         device=cuda_device)
-    assert e.value.code == dpo.DPO_EINVAL
-
-
 @pytest.mark.parametrize("name,case,n_sync", [
     ("adamw_ef_pingpong", Case(RAGGED, stash_dtype=B, ef=True,
                                stash_mode=dpo.DPO_STASH_PINGPONG), 0),
     ("nadam_ef_after_sync_start", Case(RAGGED, ef=True, optimizer=dpo.DPO_OPT_NADAM), 3),
     ("adan_clipped", Case(RAGGED, optimizer=dpo.DPO_OPT_ADAN, max_grad_norm=0.05), 0),
+    ("nadam_sapipe_updated", Case(RAGGED, ef=True, optimizer=dpo.DPO_OPT_NADAM,
+                                  correction=dpo.DPO_CORR_SAPIPE_UPDATED), 0),
+    ("adan_sapipe_updated", Case(RAGGED, ef=True, optimizer=dpo.DPO_OPT_ADAN,
+                                 correction=dpo.DPO_CORR_SAPIPE_UPDATED), 2),
 ])
 def test_capturable_step_replays_in_a_cuda_graph(cuda_device, name, case, n_sync):
     """One dpo_step captured in a CUDA graph (capturable mode) and replayed

@@ -205,3 +205,24 @@ def test_gpt2_small_other_rules_ef(cuda_device, rule, kw):
     finally:
         run.close()
         _free()
+
+
+@pytest.mark.parametrize("rule,kw", [
+    ("nadam", dict(optimizer=dpo.DPO_OPT_NADAM)),
+    ("lion", dict(optimizer=dpo.DPO_OPT_LION, beta1=0.9, beta2=0.99, lr=5e-4, weight_decay=0.5)),
+    ("adan", dict(optimizer=dpo.DPO_OPT_ADAN, beta1=0.98, beta2=0.92, beta3=0.99)),
+])
+def test_gpt2_small_other_rules_sapipe_updated(cuda_device, rule, kw):
+    """SAPipe-WP with the updated state (App. B.1) for NAdam, Lion and Adan
+    on the 124M set, 100 steps: each rule's own step at k + 1 predicts the
+    point the next gradient is taken at."""
+    w = W.GPT2_SMALL
+    case = _case(w, True, dpo.DPO_CORR_SAPIPE_UPDATED)
+    for key, val in kw.items():
+        setattr(case, key, val)
+    run = Run(case, cuda_device, sample=sample_indices(w.numels, 1_000_000))
+    try:
+        _run_steps(run, w.steps, check_every=10)
+    finally:
+        run.close()
+        _free()
