@@ -78,6 +78,11 @@ def parse_args(argv=None):
     p.add_argument("--no-secondary", action="store_true",
                    help="skip the clipped Llama-1B step (norm pass and fused step timed apart)")
     p.add_argument("--secondary-steps", type=int, default=10)
+    p.add_argument("--parallel", choices=["shard", "replica"], default="shard",
+                   help="N > 1: shard (each rank steps its contiguous share of the set, "
+                        "ZeRO-1 style; clipping takes one fp64 all-reduce of the squared "
+                        "norm; strong scaling) or replica (each rank its own full set; "
+                        "weak scaling). One GPU: the whole set either way")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     return p.parse_args(argv)
@@ -330,43 +335,77 @@ def oracle_sample_run(w, mode: str, seconds: float, max_steps: int = 1000, n: in
 
 # ------------------------------------------------------------------- GPU --
 
-def run_gpu(args, w, world, rank, local):
+def sharded(args, world: int) -> bool:
+    """Whether ranks split one set between them (else each steps its own)."""
+    return args.parallel == "shard" and world > 1
+
+
+def build_step(args, w, world, rank, dev, stream, sync=None, **kw):
+    """The rank's optimizer over its share of the set (the whole set on one
+    GPU or in replica mode) through the product's shard API, start weights
+    and the first gradient drawn for its pieces only, and the step function.
+    Sharded with clipping, each step sums the ranks' squared norms with one
+    fp64 all-reduce (dpo.global_sqnorm) and every rank clips from the total.
+    Returns (optimizer, its parameter count, step function)."""
     import numpy as np
     import torch
 
-    from paper_2606_30634_gb300 import dpo, synth
+    from paper_2606_30634_gb300 import dpo, shard, synth
+    from paper_2606_30634_gb300.synth import workloads as W
+
+    offs = np.concatenate([[0], np.cumsum(w.numels)]).astype(np.int64)
+    world_s, rank_s = (world, rank) if sharded(args, world) else (1, 0)
+    fill = lambda start, out: synth.dev_normal(w.seed, synth.STREAM_INIT, 0, int(start), out,
+                                               W.INIT_SIGMA)
+    with torch.cuda.stream(stream):
+        opt, pieces = shard.shard_optimizer(
+            w.numels, world_s, rank_s, x0=fill, sync=sync, device=dev,
+            stream=stream, param_dtype=w.param_dtype, stash_dtype=w.stash_dtype,
+            grad_dtype=w.grad_dtype, max_grad_norm=w.max_grad_norm, delay=1, **kw)
+        for j, (i, a, b) in enumerate(pieces):
+            synth.dev_normal(w.seed, synth.STREAM_GRAD, 1, int(offs[i]) + a, opt.grads(j),
+                             W.GRAD_SIGMA)
+    acc = None
+    if world_s > 1 and w.max_grad_norm > 0:
+        acc = torch.zeros(1, dtype=torch.float64, device=dev)
+        opt.set_clip_source(acc)
+
+    def step():
+        if acc is not None:
+            dpo.global_sqnorm([opt], acc, stream=stream)
+        opt.step(stream=stream)
+
+    return opt, sum(b - a for _, a, b in pieces), step
+
+
+def run_gpu(args, w, world, rank, local):
+    import torch
+
+    from paper_2606_30634_gb300 import dpo
     from paper_2606_30634_gb300.synth import workloads as W
 
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     ef, corr, _ = MODES[args.mode]
     stream = torch.cuda.Stream(dev)
-    offs = np.concatenate([[0], np.cumsum(w.numels)]).astype(np.int64)
-    with torch.cuda.stream(stream):
-        lay = dpo.Layout.of(w.numels)
-        x0 = torch.empty(lay.total, dtype=torch.float32, device=dev)
-        for i, (o, n) in enumerate(zip(lay.offsets, lay.numels)):
-            synth.dev_normal(w.seed, synth.STREAM_INIT, 0, int(offs[i]), x0[o:o + n], W.INIT_SIGMA)
-        kw = dict(lr=w.lr, beta1=w.beta1, beta2=w.beta2, eps=w.eps,
-                  weight_decay=w.weight_decay,
-                  stash_mode=(dpo.DPO_STASH_PINGPONG if args.stash == "pingpong"
-                              else dpo.DPO_STASH_COPY))
-        kw.update(rule_settings(args))
-        opt = dpo.DelayedAdamW(w.numels, param_dtype=w.param_dtype, stash_dtype=w.stash_dtype,
-                               grad_dtype=w.grad_dtype, ef=ef, ef_lambda=1.0,
-                               max_grad_norm=w.max_grad_norm, delay=1, device=dev, x0=x0,
-                               stream=stream, correction=corr, sync=wpipe_sync(w, args), **kw)
-        del x0
-        for i, (o, n) in enumerate(zip(lay.offsets, lay.numels)):
-            synth.dev_normal(w.seed, synth.STREAM_GRAD, 1, int(offs[i]), opt.grads(i),
-                             W.GRAD_SIGMA)
+    kw = dict(lr=w.lr, beta1=w.beta1, beta2=w.beta2, eps=w.eps, weight_decay=w.weight_decay,
+              stash_mode=(dpo.DPO_STASH_PINGPONG if args.stash == "pingpong"
+                          else dpo.DPO_STASH_COPY), ef=ef, ef_lambda=1.0, correction=corr)
+    kw.update(rule_settings(args))
+    opt, n_local, one_step = build_step(args, w, world, rank, dev, stream,
+                                        sync=wpipe_sync(w, args), **kw)
     torch.cuda.synchronize(dev)
     step_bytes, norm_bytes = dpo.dpo_algorithmic_bytes(opt.ctx)
     step_ctas, norm_ctas, threads = dpo.dpo_launch_config(opt.ctx)
     launches_per_step = 2 if w.max_grad_norm > 0 else 1
+    if sharded(args, world) and w.max_grad_norm > 0:
+        # the norm pass runs through dpo_grad_sqnorm (into the all-reduced
+        # scalar), then one thread forms the coefficient: 3 launches
+        norm_bytes = (2 if w.grad_dtype == W.BF16 else 4) * n_local
+        launches_per_step = 3
 
     for _ in range(args.warmup):
-        opt.step(stream=stream)
+        one_step()
     torch.cuda.synchronize(dev)
 
     props = torch.cuda.get_device_properties(dev)
@@ -380,7 +419,7 @@ def run_gpu(args, w, world, rank, local):
     time.sleep(0.25)
     ev[0].record(stream)
     for i in range(K):
-        opt.step(stream=stream)
+        one_step()
         ev[i + 1].record(stream)
     torch.cuda.synchronize(dev)
     if world > 1:
@@ -388,7 +427,10 @@ def run_gpu(args, w, world, rank, local):
     clocks = sampler.stop()
     per_step_ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(K)]
     total_s = ev[0].elapsed_time(ev[K]) / 1e3
-    value, t_max = aggregate(w.n_params * K, total_s, world, dev)
+    if sharded(args, world):   # all ranks together update the set once per step
+        value, t_max = aggregate(w.n_params * K / world, total_s, world, dev)
+    else:
+        value, t_max = aggregate(w.n_params * K, total_s, world, dev)
     # Without clipping a step is one fused-kernel launch; with clipping it is
     # the norm pass followed by the fused kernel, timed together.
     kernel_ms = sum(per_step_ms) / K
@@ -398,7 +440,7 @@ def run_gpu(args, w, world, rank, local):
     # to pinned host memory, copies inside the timed region.
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(args, opt, stream, dev, world, w)
+        e2e = run_e2e(args, opt, one_step, stream, dev, world, w)
 
     opt.close()
     return dict(value=value, t_max=t_max, per_step_ms=per_step_ms, kernel_ms=kernel_ms,
@@ -412,36 +454,25 @@ def run_secondary(args, dev, world):
     tensors, EF, fp32 stash, one-step delay): the norm pass and the fused
     step each timed by the library's CUDA events on the launch stream
     (dpo_set_timing), and the whole step by events around it."""
-    import numpy as np
     import torch
 
-    from paper_2606_30634_gb300 import dpo, synth
+    from paper_2606_30634_gb300 import dpo
     from paper_2606_30634_gb300.synth import workloads as W
 
     w = W.LLAMA_1B
     gc.collect()
     torch.cuda.empty_cache()   # the headline set's arenas
     stream = torch.cuda.Stream(dev)
-    offs = np.concatenate([[0], np.cumsum(w.numels)]).astype(np.int64)
-    with torch.cuda.stream(stream):
-        lay = dpo.Layout.of(w.numels)
-        x0 = torch.empty(lay.total, dtype=torch.float32, device=dev)
-        for i, (o, n) in enumerate(zip(lay.offsets, lay.numels)):
-            synth.dev_normal(w.seed, synth.STREAM_INIT, 0, int(offs[i]), x0[o:o + n], W.INIT_SIGMA)
-        opt = dpo.DelayedAdamW(w.numels, param_dtype=w.param_dtype, stash_dtype=w.stash_dtype,
-                               grad_dtype=w.grad_dtype, ef=True, ef_lambda=1.0,
-                               max_grad_norm=w.max_grad_norm, delay=1, device=dev, x0=x0,
-                               stream=stream, lr=w.lr, beta1=w.beta1, beta2=w.beta2, eps=w.eps,
-                               weight_decay=w.weight_decay)
-        del x0
-        for i, (o, n) in enumerate(zip(lay.offsets, lay.numels)):
-            synth.dev_normal(w.seed, synth.STREAM_GRAD, 1, int(offs[i]), opt.grads(i),
-                             W.GRAD_SIGMA)
+    opt, n_local, one_step = build_step(
+        args, w, world, int(os.environ.get("RANK", "0")), dev, stream, ef=True, ef_lambda=1.0,
+        lr=w.lr, beta1=w.beta1, beta2=w.beta2, eps=w.eps, weight_decay=w.weight_decay)
     torch.cuda.synchronize(dev)
     step_bytes, norm_bytes = dpo.dpo_algorithmic_bytes(opt.ctx)
     _, norm_ctas, _ = dpo.dpo_launch_config(opt.ctx)
+    if sharded(args, world):   # the norm pass runs outside dpo_step (dpo_grad_sqnorm)
+        norm_bytes = 2 * n_local
     for _ in range(args.warmup):
-        opt.step(stream=stream)
+        one_step()
     torch.cuda.synchronize(dev)
     K = max(1, args.secondary_steps)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -451,7 +482,7 @@ def run_secondary(args, dev, world):
     torch.cuda.synchronize(dev)
     e0.record(stream)
     for _ in range(K):
-        opt.step(stream=stream)
+        one_step()
     e1.record(stream)
     torch.cuda.synchronize(dev)
     norm_ms, fused_ms, calls = opt.kernel_times()
@@ -465,7 +496,7 @@ def run_secondary(args, dev, world):
     norm_ms = max_over_ranks(norm_ms / calls, world, dev)
     fused_ms = max_over_ranks(fused_ms / calls, world, dev)
     peak, peak_kind = measured_hbm_peak()
-    n = w.n_params
+    n = n_local
 
     def kern(bytes_, ms, tag):
         t = committed_traffic(tag)
@@ -475,9 +506,15 @@ def run_secondary(args, dev, world):
                 "traffic": None if t is None else t * n, "traffic_tag": tag}
 
     pair_ms = norm_ms + fused_ms
-    return {"workload": f"{w.name}: {n} params in {len(w.tensors)} tensors, EF (lambda=1), "
-                        f"global-norm clip at {w.max_grad_norm}, fp32 stash, one-step delay",
-            "value": n * K / (total_ms / 1e3) * world, "unit": UNIT, "steps": K,
+    units = w.n_params if sharded(args, world) else w.n_params * world
+    return {"workload": f"{w.name}: {w.n_params} params in {len(w.tensors)} tensors, EF "
+                        f"(lambda=1), global-norm clip at {w.max_grad_norm}, fp32 stash, "
+                        "one-step delay",
+            "value": units * K / (total_ms / 1e3), "unit": UNIT, "steps": K,
+            "params_per_rank": n_local,
+            "norm_timing": ("grad_sqnorm_kernel inside dpo_step" if not sharded(args, world)
+                            else "dpo_grad_sqnorm + fp64 all-reduce outside dpo_step; "
+                                 "grad_sqnorm_kernel's entry times only the coefficient kernel"),
             "ms_per_step": total_ms / K, "grad_norm": gnorm, "clip_coef": coef,
             "peak": peak, "peak_kind": peak_kind, "norm_ctas": norm_ctas,
             "grad_sqnorm_kernel": kern(norm_bytes, norm_ms, f"grad_sqnorm:{w.name}"),
@@ -510,7 +547,7 @@ def run_muon(args, w, world, rank, local):
 
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
-    ef = args.mode == "ef"
+    ef, corr, _ = MODES[args.mode]   # EF, standard rule, or a SAPipe-WP prediction
     stream = torch.cuda.Stream(dev)
     offs = np.concatenate([[0], np.cumsum(w.numels)]).astype(np.int64)
     mi, ai = muon_split(w)
@@ -518,7 +555,7 @@ def run_muon(args, w, world, rank, local):
     with torch.cuda.stream(stream):
         mo = muon.DelayedMuon(shapes, stash_dtype=w.stash_dtype, grad_dtype=w.grad_dtype,
                               lr=MUON_LR, ef=ef, ns_steps=args.ns_steps, delay=1, device=dev,
-                              init_mode=dpo.DPO_INIT_RESUME, stream=stream)
+                              init_mode=dpo.DPO_INIT_RESUME, stream=stream, correction=corr)
         for j, i in enumerate(mi):
             synth.dev_normal(w.seed, synth.STREAM_INIT, 0, int(offs[i]),
                              mo.view(mo.master, j).view(-1), W.INIT_SIGMA)
@@ -536,7 +573,8 @@ def run_muon(args, w, world, rank, local):
         ad = dpo.DelayedAdamW(rest, param_dtype=w.param_dtype, stash_dtype=w.stash_dtype,
                               grad_dtype=w.grad_dtype, ef=ef, ef_lambda=1.0, delay=1,
                               device=dev, x0=x0, stream=stream, lr=w.lr, beta1=w.beta1,
-                              beta2=w.beta2, eps=w.eps, weight_decay=w.weight_decay)
+                              beta2=w.beta2, eps=w.eps, weight_decay=w.weight_decay,
+                              correction=corr)
         del x0
         for j, i in enumerate(ai):
             synth.dev_normal(w.seed, synth.STREAM_GRAD, 1, int(offs[i]), ad.grads(j),
@@ -545,6 +583,8 @@ def run_muon(args, w, world, rank, local):
     flops = mo.flops()
     n_groups = len({(min(r, c), max(r, c)) for r, c in shapes})
     launches_per_step = 1 + 3 + n_groups * (1 + 3 * args.ns_steps)
+    if corr == 2:   # the updated-state prediction: momentum, norm, predict, a second chain
+        launches_per_step += 3 + n_groups * (1 + 3 * args.ns_steps)
 
     mo.set_timing(True)
     for _ in range(args.warmup):
@@ -695,7 +735,7 @@ def e2e_fits(avail: int, io_bytes: int, local_world: int) -> bool:
     return avail >= local_world * 2 * io_bytes + (16 << 30)
 
 
-def run_e2e(args, opt, stream, dev, world, w):
+def run_e2e(args, opt, one_step, stream, dev, world, w):
     """End to end through the public API with the step's inputs (gradients)
     in pinned host memory and its result (the new bf16 weights) delivered to
     pinned host memory, transfers inside the timed region. The library's
@@ -741,7 +781,7 @@ def run_e2e(args, opt, stream, dev, world, w):
     def staged_step():
         with torch.cuda.stream(stream):
             opt.grad.copy_(h_grad, non_blocking=True)
-            opt.step(stream=stream)
+            one_step()
             h_param.copy_(opt.param, non_blocking=True)
 
     staged_s = timed(staged_step)
@@ -751,17 +791,22 @@ def run_e2e(args, opt, stream, dev, world, w):
     # host I/O: the fused kernel reads the gradients from and writes the new
     # weights to pinned host memory itself
     opt.use_host_io(stream=stream)
-    secs = timed(lambda: opt.step(stream=stream))
-    value, _ = aggregate(w.n_params * K, secs, world, dev)
-    staged_value, _ = aggregate(w.n_params * K, staged_s, world, dev)
+    secs = timed(one_step)
+    units = w.n_params * K / (world if sharded(args, world) else 1)
+    value, _ = aggregate(units, secs, world, dev)
+    staged_value, _ = aggregate(units, staged_s, world, dev)
     return {"value": value, "unit": UNIT, "h2d_bytes_per_step": gbytes,
             "d2h_bytes_per_step": pbytes, "ms_per_step": secs / K * 1e3, "steps": K,
             "path": "dpo_step with grad and bf16 param arenas in pinned host memory: the "
                     "fused kernel reads gradients and writes weights across the host link",
             "host_link_gbs": (gbytes + pbytes) / (secs / K) / 1e9,
             "link_peak": link,
+            # the bound: each direction at its own measured rate, both at once
+            # (the host-I/O kernel overlaps them; two concurrent copy-engine
+            # copies do not, see link_peak.both_gbs)
+            "link_bound_ms": None if link is None else link["duplex_bound_ms"],
             "link_frac": (None if link is None else
-                          (gbytes + pbytes) / (secs / K) / 1e9 / link["both_gbs"]),
+                          link["duplex_bound_ms"] / (secs / K * 1e3)),
             "staged": {"value": staged_value, "ms_per_step": staged_s / K * 1e3,
                        "path": "cudaMemcpy grad in, device-resident dpo_step, cudaMemcpy "
                                "weights out, on one stream"}}
@@ -810,9 +855,12 @@ def link_peak(opt, h_grad, h_param, stream, dev, reps: int = 2) -> dict:
     torch.cuda.synchronize(dev)
     return {"h2d_gbs": gb / t_in / 1e6, "d2h_gbs": pb / t_out / 1e6,
             "both_gbs": (gb + pb) / t_both / 1e6, "h2d_bytes": gb, "d2h_bytes": pb,
+            "duplex_bound_ms": max(t_in, t_out),
             "what": "best of %d: pinned host -> device copy of the gradients alone, device -> "
                     "pinned host copy of the bf16 weights alone, and both at once on two "
-                    "streams (combined bytes / elapsed)" % reps}
+                    "streams (combined bytes / elapsed); duplex_bound_ms: the slower "
+                    "direction alone, the step's transfer time if both directions ran at "
+                    "their own rates at once" % reps}
 
 
 # ------------------------------------------------------------------ main --
@@ -826,7 +874,7 @@ def main_muon(args, w, world, rank, local):
     cfg = {"workload": f"{w.name}: {w.n_params} params; delayed Muon (Alg. 2, "
                        f"{args.ns_steps} Newton-Schulz steps) on {len(mi)} attention/MLP "
                        f"matrices ({n_muon} params), AdamW on the other {len(ai)} tensors, "
-                       f"{'EF' if args.mode == 'ef' else 'standard rule'}, one-step delay",
+                       f"{MODES[args.mode][2]}, one-step delay",
            "mode": args.mode, "optimizer": "muon", "ns_steps": args.ns_steps,
            "param_dtype": "bf16", "stash_dtype": "bf16" if w.stash_dtype else "f32",
            "grad_dtype": "bf16" if w.grad_dtype else "f32",
@@ -907,7 +955,12 @@ def main(argv=None):
            "state": "fp32 master/m/v" + (" + fp32 update-history buffer" if ef else ""),
            "clip": w.max_grad_norm, "l2": "inputs larger than L2 (no flush needed)",
            "wpipe": bool(args.wpipe), "optimizer": args.optimizer,
-           "dc_lambda": args.dc_lambda, "stash": args.stash}
+           "dc_lambda": args.dc_lambda, "stash": args.stash,
+           "parallelism": (f"shard{world}: each rank steps 1/{world} of the set (contiguous "
+                           "ranges of the flat concatenation), clip norm all-reduced"
+                           if sharded(args, world) else
+                           f"replica{world}: each rank steps its own full set"
+                           if world > 1 else "one GPU, the whole set")}
 
     if args.impl == "reference":
         if rank != 0:
@@ -923,7 +976,7 @@ def main(argv=None):
                 "ms_per_step": w.n_params / v * 1e3,
                 **extrapolation(w.n_params, n, steps, n * steps / v, wall),
                 "higher_is_better": True,
-                "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                "scaling": "strong" if args.parallel == "shard" else "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
                 "config": cfg,
                 "cpu_baseline": {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
                                  "sample": sample},
@@ -973,7 +1026,9 @@ def main(argv=None):
         return 0
     line = {"metric": METRIC, "value": r["value"], "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": r["t_max"] / args.steps * 1e3,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "higher_is_better": True,
+            "scaling": "strong" if args.parallel == "shard" else "weak",
+            "vs_baseline": None, "dtype": "f32",
             "data": "synthetic", "config": cfg, "roofline": roof, "cpu_baseline": cpu,
             "e2e": r["e2e"], "gpu_launches": r["launches"], "clocks": r["clocks"],
             "launch": {"ctas": r["step_ctas"], "threads": r["threads"]},

@@ -50,10 +50,12 @@ def shard_optimizer(numels: Sequence[int], world: int, rank: int, *,
                     sync: Optional[Sequence[bool]] = None, x0=None,
                     **kwargs) -> Tuple[DelayedAdamW, List[Piece]]:
     """A DelayedAdamW over rank's pieces. Each piece keeps the weight-decay
-    and synchronous flags of the tensor it comes from; ``x0`` (the full flat
-    fp32 weights, a torch tensor on any device) seeds the shard's master
-    copy. Pass ``max_grad_norm`` in ``kwargs`` and a clip source to clip
-    globally."""
+    and synchronous flags of the tensor it comes from. ``x0`` seeds the
+    shard's master copy: the full flat fp32 weights (a torch tensor on any
+    device), or a function ``x0(start, out)`` that writes the weights of flat
+    elements [start, start + out.numel()) into the fp32 device tensor ``out``
+    (so no rank holds the whole set). Pass ``max_grad_norm`` in ``kwargs``
+    and a clip source to clip globally."""
     pieces = partition(numels, world, rank)
     lay = Layout.of([b - a for _, a, b in pieces])
     buf = None
@@ -62,9 +64,14 @@ def shard_optimizer(numels: Sequence[int], world: int, rank: int, *,
         starts = [0]
         for n in numels:
             starts.append(starts[-1] + int(n))
-        buf = torch.zeros(lay.total, dtype=torch.float32, device=x0.device)
+        dev = kwargs.get("device") if callable(x0) else x0.device
+        buf = torch.zeros(lay.total, dtype=torch.float32, device=dev)
         for j, (i, a, b) in enumerate(pieces):
-            buf[lay.offsets[j]:lay.offsets[j] + b - a] = x0[starts[i] + a:starts[i] + b]
+            out = buf[lay.offsets[j]:lay.offsets[j] + b - a]
+            if callable(x0):
+                x0(starts[i] + a, out)
+            else:
+                out.copy_(x0[starts[i] + a:starts[i] + b])
     opt = DelayedAdamW(
         lay.numels,
         wd_on=[wd_on[i] for i, _, _ in pieces] if wd_on is not None else None,

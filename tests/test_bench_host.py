@@ -52,6 +52,42 @@ def test_aggregate_takes_slowest_rank_gloo():
         assert value == pytest.approx(1200.0 / 3.0)   # all ranks' units / slowest time
 
 
+def _shard_worker(rank, world, port, q):
+    """Partitioned mode: each rank updates its share of one set per step, so
+    the whole job's throughput is the set's size over the slowest rank."""
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    args = bench.parse_args(["--gpus", str(world)])
+    assert args.parallel == "shard" and bench.sharded(args, world)
+    assert not bench.sharded(bench.parse_args(["--parallel", "replica"]), world)
+    n_params, steps = 1000, 3
+    secs = [0.5, 0.75][rank]
+    value, t = bench.aggregate(n_params * steps / world, secs, world)
+    q.put((rank, value, t))
+    dist.destroy_process_group()
+
+
+def test_sharded_aggregate_counts_the_set_once_gloo():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_shard_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = sorted(q.get(timeout=120) for _ in procs)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    for rank, value, t in res:
+        assert t == 0.75
+        assert value == pytest.approx(3000 / 0.75)   # the set's 3 steps / slowest rank
+
+
+def test_one_gpu_is_never_sharded():
+    assert not bench.sharded(bench.parse_args([]), 1)
+
+
 def test_single_rank_aggregate():
     assert bench.aggregate(10.0, 2.0, 1) == (5.0, 2.0)
 

@@ -48,6 +48,38 @@ def test_bounds_rejects_bad_ranks():
     assert shard.partition([0, 0], 2, 1) == []
 
 
+@pytest.mark.parametrize("world,rank", [(1, 0), (2, 1), (3, 0), (3, 2)])
+def test_shard_optimizer_seeds_each_piece(monkeypatch, world, rank):
+    """A fill function (start, out) seeds the shard's master exactly as the
+    full flat weights would: each piece reads its own global range, into its
+    own offset of the shard's arena layout; flags follow their tensors."""
+    import torch
+    got = []
+
+    class Capture:   # stands in for the device context (no GPU here)
+        def __init__(self, numels, **kw):
+            got.append((list(numels), kw))
+
+    monkeypatch.setattr(shard, "DelayedAdamW", Capture)
+    full = torch.arange(sum(NUMELS), dtype=torch.float32) * 0.5 - 7.0
+    calls = []
+
+    def fill(start, out):
+        calls.append((start, out.numel()))
+        out.copy_(full[start:start + out.numel()])
+
+    wd = [True, False, True, True, False, True]
+    _, pieces = shard.shard_optimizer(NUMELS, world, rank, x0=fill, device="cpu", wd_on=wd)
+    _, pieces2 = shard.shard_optimizer(NUMELS, world, rank, x0=full, wd_on=wd)
+    assert pieces == pieces2
+    starts = np.concatenate([[0], np.cumsum(NUMELS)])
+    assert calls == [(int(starts[i]) + a, b - a) for i, a, b in pieces]
+    (n1, kw1), (n2, kw2) = got
+    assert n1 == n2 == [b - a for _, a, b in pieces]
+    assert torch.equal(kw1["x0"], kw2["x0"])
+    assert kw1["wd_on"] == [wd[i] for i, _, _ in pieces]
+
+
 def _free_port():
     s = socket.socket()
     s.bind(("127.0.0.1", 0))
