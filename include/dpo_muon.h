@@ -26,6 +26,12 @@
  *   stash := X_t,  U_prev := U,  param := bf16(X_{t+1})
  *   With correction DPO_CORR_SAPIPE_SAME (SAPipe-WP, App. B.1) the weights take
  *   the standard rule and the stash receives the predicted point X_t - U_prev.
+ *   With DPO_CORR_SAPIPE_UPDATED (App. B.1, updated state) the same, but
+ *   U_prev := U', the step taken once more on the same gradient from the
+ *   updated momentum: M' = mu M + (1 - mu) G^ (not kept in M),
+ *   O' = NewtonSchulz(M'), U' = lr (r O' + wd X_{t+1}). M' is formed in the
+ *   history buffer, so the prediction needs no extra memory; it doubles the
+ *   step's tensor-core work.
  *
  * The k-th dpo_muon_step is Alg. 1's iteration t = k (t = 0 only sets
  * X_1 = X_0). With delay = 0 the same update runs on gradients of the latest
@@ -79,10 +85,12 @@ typedef struct {
     float rms_scale;      /* 0.2: match the update RMS; 0: no scaling */
     int ns_steps;         /* iterations, 0..16 (5) */
     int delay;            /* 1: one-step-delayed (Alg. 1 / 2); 0: synchronous */
-    int correction;       /* with ef buffers: DPO_CORR_EF (lambda-scaled Error Feedback) or
+    int correction;       /* with ef buffers: DPO_CORR_EF (lambda-scaled Error Feedback),
                              DPO_CORR_SAPIPE_SAME (SAPipe-WP with the same state, App. B.1:
                              the weights take the standard rule, the stash receives the
-                             prediction point X_t - U_prev, the history U) */
+                             prediction point X_t - U_prev, the history U) or
+                             DPO_CORR_SAPIPE_UPDATED (the same with the history U', the
+                             updated-state prediction above) */
 } dpo_muon_hparams;
 
 typedef struct dpo_muon_ctx dpo_muon_ctx;
@@ -121,7 +129,8 @@ int dpo_muon_set_delay(dpo_muon_ctx *ctx, int delay, void *cuda_stream);
 /*
  * Newton-Schulz output O of the last step for matrix i, as a strided bf16
  * view into the workspace (valid until the next dpo_muon_step): element
- * (r, c) of O (rows x cols) is at (*ptr)[r * *ld + c].
+ * (r, c) of O (rows x cols) is at (*ptr)[r * *ld + c]. With the SAPipe-WP
+ * updated state in delayed training it is the prediction's output O'.
  */
 int dpo_muon_last_update(const dpo_muon_ctx *ctx, int i, const void **ptr, int64_t *ld);
 
@@ -195,7 +204,8 @@ int dpo_muon_set_phase_start(dpo_muon_ctx *ctx, int64_t k0);
  * Tensor-core work of one step, summed over the matrices (r x w the
  * orientation with r <= w, unpadded), two flops per multiply-add:
  * ns_steps (r (r + 1) w + r (r + 1) r + 2 r^2 w), the first two terms being
- * the unique entries of the symmetric products X X^T and A A.
+ * the unique entries of the symmetric products X X^T and A A; twice that
+ * with the SAPipe-WP updated state in delayed training.
  */
 int dpo_muon_flops(const dpo_muon_ctx *ctx, double *flops);
 

@@ -68,15 +68,15 @@ constexpr unsigned long long kWaitNs = 1000000000ull;  // 1 s per wait
 constexpr unsigned int kErrWaitFull = 1u, kErrWaitEmpty = 2u, kErrWaitDone = 4u,
                        kErrDrain = 8u;
 
-// D is written through the store map tma_d (boxes of 32 x 32, 64-byte
-// swizzle) and, with trans, D^T through tma_dt.
+// D is written through the group's store map d (boxes of 32 x 32, 64-byte
+// swizzle) and, with trans, D^T through dt.
 struct Params {
     const __nv_bfloat16 *c;       // M x N addend, or nullptr
     int64_t ldc, c_bstride;
     float alpha, beta;
     int k_blocks;                 // K / BK
     int sym;                      // D is symmetric (M == N): see ns_gemm_kernel
-    int trans;                    // also write D^T (N x M) through tma_dt
+    int trans;                    // also write D^T (N x M) through the map dt
     int stall;                    // test hook: the MMA lane's first accumulator wait
                                   // targets a phase no arrival completes, so it gives up
     unsigned int *err;
@@ -299,6 +299,38 @@ struct TileGrid {
     }
 };
 
+// One launch computes the same product for up to kMaxGroups batches of
+// different shapes (the shape groups of a Newton-Schulz step): each group
+// has its own operand and output maps, epilogue and tile grid, and its tiles
+// follow the previous group's in the launch's order. Small sets then fill
+// the CTA pairs with one launch per product instead of one per shape.
+constexpr int kMaxGroups = 4;
+
+struct GemmGroup {
+    CUtensorMap a, b, d, dt;   // A, B (operands), D and D^T (stores)
+    Params p;
+    TileGrid tg;
+    int tile0;                 // first tile of this group in the launch
+};
+
+struct GemmLaunch {
+    GemmGroup g[kMaxGroups];
+    int n_groups;
+    int n_tiles;               // over all groups
+};
+
+// Group, batch entry, row block and column block of tile t of a launch.
+__device__ __forceinline__ const GemmGroup &locate(const GemmLaunch &L, int t, int &b, int &m0,
+                                                   int &n0)
+{
+    int gi = L.n_groups - 1;
+    while (gi > 0 && t < L.g[gi].tile0)
+        --gi;
+    const GemmGroup &G = L.g[gi];
+    G.tg.at(t - G.tile0, b, m0, n0);
+    return G;
+}
+
 // Persistent: the CTA pairs (clusters of 2) take tiles c, c + pairs, ...
 // Within a pair, rank 0 (the leader) issues the MMAs; both ranks load their
 // halves of A and B and drain their own accumulator rows. Two accumulators
@@ -312,11 +344,9 @@ struct TileGrid {
 // loaded as two 64 x 64 boxes per stage, read MN-major by the MMA.
 template <bool BMN>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
-    ns_gemm_kernel(const __grid_constant__ CUtensorMap tma_a,
-                   const __grid_constant__ CUtensorMap tma_b,
-                   const __grid_constant__ CUtensorMap tma_d,
-                   const __grid_constant__ CUtensorMap tma_dt, const Params p, const TileGrid tg)
+    ns_gemm_kernel(const __grid_constant__ GemmLaunch L)
 {
+    const Params &p0 = L.g[0].p;   // err and stall are the launch's
     extern __shared__ uint8_t smem_raw[];
     __shared__ uint64_t bars[2 * kStages + 4];
     __shared__ uint32_t tmem_slot;
@@ -358,25 +388,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     cluster_sync();   // barriers of both CTAs initialised before any remote use
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = tmem_slot;
-    const int kb_n = p.k_blocks;
-    const int n_tiles = tg.count();
+    const int n_tiles = L.n_tiles;
 
     if (warp == 0) {
         if (lane == 0) {
-            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tma_a))
-                         : "memory");
-            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tma_b))
-                         : "memory");
+            for (int gi = 0; gi < L.n_groups; ++gi) {
+                asm volatile("prefetch.tensormap [%0];"
+                             ::"l"(reinterpret_cast<uint64_t>(&L.g[gi].a)) : "memory");
+                asm volatile("prefetch.tensormap [%0];"
+                             ::"l"(reinterpret_cast<uint64_t>(&L.g[gi].b)) : "memory");
+            }
             int it = 0;   // k-blocks issued by this CTA
             for (int t = pair; t < n_tiles && !*(volatile int *)&aborted; t += n_pairs) {
                 int b, m0, n0;
-                tg.at(t, b, m0, n0);
+                const GemmGroup &G = locate(L, t, b, m0, n0);
+                const CUtensorMap *tma_a = &G.a, *tma_b = &G.b;
+                const int kb_n = G.p.k_blocks;
                 const int ma = m0 + (int)rank * BM, nb_ = n0 + (int)rank * BH;
                 for (int kb = 0; kb < kb_n; ++kb, ++it) {
                     const int s = it % kStages;
                     const uint32_t ph = (uint32_t)(it / kStages) & 1u;
                     if (!mbar_wait(empty(s), ph ^ 1u) || *(volatile int *)&aborted) {
-                        atomicOr(p.err, kErrWaitEmpty);
+                        atomicOr(p0.err, kErrWaitEmpty);
                         aborted = 1;
                         break;
                     }
@@ -388,12 +421,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         const int k0 = kb * BK + h * kBoxK;
                         const uint32_t ah = sa + (uint32_t)(s * kABytes + h * (kABytes / 2));
                         const uint32_t bh = sb + (uint32_t)(s * kBBytes + h * (kBBytes / 2));
-                        tma_load_3d(ah, &tma_a, k0, ma, b, fbar);
+                        tma_load_3d(ah, tma_a, k0, ma, b, fbar);
                         if (BMN) {   // two 64 x 64 boxes: N columns nb_.. and nb_ + 64..
-                            tma_load_3d(bh, &tma_b, nb_, k0, b, fbar);
-                            tma_load_3d(bh + (uint32_t)(kBBytes / 4), &tma_b, nb_ + 64, k0, b, fbar);
+                            tma_load_3d(bh, tma_b, nb_, k0, b, fbar);
+                            tma_load_3d(bh + (uint32_t)(kBBytes / 4), tma_b, nb_ + 64, k0, b, fbar);
                         } else {
-                            tma_load_3d(bh, &tma_b, k0, nb_, b, fbar);
+                            tma_load_3d(bh, tma_b, k0, nb_, b, fbar);
                         }
                     }
                 }
@@ -404,18 +437,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             if (leader)
                 for (int q = it - kStages < 0 ? 0 : it - kStages; q < it; ++q)
                     if (!mbar_wait(full(q % kStages), (uint32_t)(q / kStages) & 1u))
-                        atomicOr(p.err, kErrDrain);
+                        atomicOr(p0.err, kErrDrain);
         }
     } else if (warp == 1) {
         if (lane == 0 && leader) {
             int it = 0, lt = 0;   // k-blocks consumed, tiles accumulated
             for (int t = pair; t < n_tiles && !*(volatile int *)&aborted; t += n_pairs) {
                 int b, m0, n0;
-                tg.at(t, b, m0, n0);
+                const int kb_n = locate(L, t, b, m0, n0).p.k_blocks;
                 const int a = lt & 1;
                 const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
-                if (!mbar_wait(acc_empty(a), p.stall && lt == 0 ? aph : aph ^ 1u)) {
-                    atomicOr(p.err, kErrWaitDone);
+                if (!mbar_wait(acc_empty(a), p0.stall && lt == 0 ? aph : aph ^ 1u)) {
+                    atomicOr(p0.err, kErrWaitDone);
                     aborted = 1;
                     break;
                 }
@@ -426,7 +459,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                     const int s = it % kStages;
                     const uint32_t ph = (uint32_t)(it / kStages) & 1u;
                     if (!mbar_wait(full(s), ph) || *(volatile int *)&aborted) {
-                        atomicOr(p.err, kErrWaitFull);
+                        atomicOr(p0.err, kErrWaitFull);
                         aborted = 1;
                         ok = false;
                         break;
@@ -450,7 +483,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                     // the MMAs issued for this tile finish before the pair
                     // leaves and its TMEM is released
                     if (!mbar_wait(acc_full(a), aph))
-                        atomicOr(p.err, kErrDrain);
+                        atomicOr(p0.err, kErrDrain);
                     break;
                 }
             }
@@ -465,24 +498,39 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         // waits for the group of two chunks back before they are rewritten.
         const int q = warp & 3;
         const uint32_t wbuf = ring + (uint32_t)(kStages * kStageBytes + q * 4 * kChunkBytes);
+        // The addend C (c A A + b A, B X + a X) is read 32 columns per lane per
+        // chunk, kCPre chunks ahead of their use, the first ones before the
+        // accumulator is ready: where K is short (768) the MMAs of a tile
+        // take a few microseconds, and one dependent global load per chunk
+        // made the epilogue the bottleneck. C is never the launch's output.
+        constexpr int kCPre = 4;
         int lt = 0, staged = 0;
         for (int t = pair; t < n_tiles; t += n_pairs) {
             int b, m0, n0;
-            tg.at(t, b, m0, n0);
+            const GemmGroup &G = locate(L, t, b, m0, n0);
+            const Params &p = G.p;
             const int a = lt & 1;
-            const bool seen = mbar_wait(acc_full(a), (uint32_t)(lt >> 1) & 1u);
-            if (!seen)
-                atomicOr(p.err, kErrWaitDone);
-            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            // tcgen05.ld is warp-collective: the whole warp goes on, or none of it.
-            if (!__all_sync(0xFFFFFFFFu, seen && !*(volatile int *)&aborted))
-                break;
             const int row0 = m0 + (int)rank * BM + q * 32;
             const int64_t row = row0 + lane;
             const __nv_bfloat16 *crow =
                 p.c != nullptr ? p.c + (int64_t)b * p.c_bstride + row * p.ldc + n0 : nullptr;
+            uint4 cpre[kCPre][4];
+            if (crow != nullptr) {
+#pragma unroll
+                for (int c = 0; c < kCPre; ++c)
+#pragma unroll
+                    for (int j8 = 0; j8 < 4; ++j8)
+                        cpre[c][j8] = __ldg(reinterpret_cast<const uint4 *>(crow + c * 32 + j8 * 8));
+            }
+            const bool seen = mbar_wait(acc_full(a), (uint32_t)(lt >> 1) & 1u);
+            if (!seen)
+                atomicOr(p0.err, kErrWaitDone);
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            // tcgen05.ld is warp-collective: the whole warp goes on, or none of it.
+            if (!__all_sync(0xFFFFFFFFu, seen && !*(volatile int *)&aborted))
+                break;
             const uint32_t acc = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(a * (int)kTmemCols);
-#pragma unroll 1
+#pragma unroll
             for (int ch = 0; ch < TN / 32; ++ch) {
                 uint32_t r[32];
                 tmem_ld32(acc + (uint32_t)(ch * 32), r);
@@ -493,7 +541,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 if (crow != nullptr) {
 #pragma unroll
                     for (int j8 = 0; j8 < 4; ++j8) {
-                        const uint4 cv = *reinterpret_cast<const uint4 *>(crow + ch * 32 + j8 * 8);
+                        const uint4 cv = cpre[ch % kCPre][j8];
+                        if (ch + kCPre < TN / 32)   // the slot's next chunk
+                            cpre[ch % kCPre][j8] = __ldg(
+                                reinterpret_cast<const uint4 *>(crow + (ch + kCPre) * 32 + j8 * 8));
                         const __nv_bfloat162 *c2 = reinterpret_cast<const __nv_bfloat162 *>(&cv);
 #pragma unroll
                         for (int e = 0; e < 4; ++e) {
@@ -538,9 +589,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 __syncwarp();
                 if (lane == 0) {
-                    tma_store_3d(&tma_d, rb, col0, row0, b);
+                    tma_store_3d(&G.d, rb, col0, row0, b);
                     if (trans)
-                        tma_store_3d(mirror ? &tma_d : &tma_dt, tb, row0, col0, b);
+                        tma_store_3d(mirror ? &G.d : &G.dt, tb, row0, col0, b);
                     asm volatile("cp.async.bulk.commit_group;" ::: "memory");
                 }
                 ++staged;

@@ -18,6 +18,11 @@
 //                           also writes X^T, the output of tall matrices)
 //   muon_apply_kernel       U = lr (r O + wd X_t) and the delayed or EF
 //                           update, stash, history and bf16 weights
+// With the SAPipe-WP updated-state prediction (App. B.1) the step then runs
+// the pipeline once more for the prediction update: the momentum kernel
+// forms M' = mu M + (1 - mu) G^ into the history buffer, M' is normalised and
+// put through a second Newton-Schulz chain, and muon_predict_kernel writes
+// U' = lr (r O' + wd X_{t+1}) into the history.
 #include "dpo_muon.h"
 
 #include <cuda.h>
@@ -63,6 +68,8 @@ struct MomArgs {
     float mu, omm;
     double *partials;         // [n_mats][chunks]
     int chunks;
+    int predict;              // M' = mu M + (1 - mu) G^ into the history buffer of each
+                              // delayed matrix; M keeps its value
 };
 
 template <class GT>
@@ -70,7 +77,10 @@ __global__ void __launch_bounds__(kThreads) muon_momentum_kernel(const MomArgs a
 {
     __shared__ double red[kThreads / 32];
     const DevMat &d = a.mats[blockIdx.y];
-    const int64_t n = d.rows * d.cols;
+    // the prediction pass leaves a synchronous matrix (and its history) alone
+    const bool skip = a.predict && (d.sync || d.ef == nullptr);
+    const int64_t n = skip ? 0 : d.rows * d.cols;
+    float *out = a.predict ? d.ef : d.mom;
     const int64_t lo = (int64_t)blockIdx.x * kChunk;
     float sum = 0.0f, comp = 0.0f;
     if (lo < n) {
@@ -90,7 +100,7 @@ __global__ void __launch_bounds__(kThreads) muon_momentum_kernel(const MomArgs a
                     m[j] = fmaf(a.mu, m[j], p) + fmaf(a.omm, gc, -p);
                     s = fmaf(m[j], m[j], s);
                 }
-                st8(d.mom + e, m);
+                st8(out + e, m);
                 const float y = s - comp, t = sum + y;   // Kahan
                 comp = (t - sum) - y;
                 sum = t;
@@ -99,7 +109,7 @@ __global__ void __launch_bounds__(kThreads) muon_momentum_kernel(const MomArgs a
                     const float gc = ld1(grad + i) * clip;
                     const float p = a.omm * gc;
                     const float m = fmaf(a.mu, d.mom[i], p) + fmaf(a.omm, gc, -p);
-                    d.mom[i] = m;
+                    out[i] = m;
                     const float y = m * m - comp, t = sum + y;
                     comp = (t - sum) - y;
                     sum = t;
@@ -148,6 +158,8 @@ struct NormArgsM {
     __nv_bfloat16 *x, *xt;    // X (R x W) and X^T (W x R, or nullptr) of batch entry 0
     int64_t R, W;
     int64_t r, w;
+    int predict;              // read M' from the history buffer (zeros for a
+                              // synchronous matrix) instead of M
 };
 
 // One 64 x 64 tile of X (rows i over r, columns j over w) per CTA; padding
@@ -163,6 +175,7 @@ __global__ void __launch_bounds__(kThreads) muon_normalize_kernel(const NormArgs
     const DevMat &d = a.mats[gm];
     const bool tall = d.rows > d.cols;
     const float s = a.inv_norm[gm];
+    const float *src = a.predict ? (d.sync ? nullptr : d.ef) : d.mom;
     const int64_t i0 = (int64_t)blockIdx.y * 64, j0 = (int64_t)blockIdx.x * 64;
     // tile origin in M: (mr0, mc0), 64 x 64, clipped to rows x cols
     const int64_t mr0 = tall ? j0 : i0, mc0 = tall ? i0 : j0;
@@ -172,13 +185,17 @@ __global__ void __launch_bounds__(kThreads) muon_normalize_kernel(const NormArgs
         const int v = (int)threadIdx.x + h * kThreads;   // 512 vectors of 8
         const int row = v >> 3, c8 = (v & 7) * 8;         // within the tile, in M's layout
         float x[8];
-        if (vec) {
-            ld8(d.mom + (mr0 + row) * d.cols + mc0 + c8, x);
+        if (src == nullptr) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                x[e] = 0.0f;
+        } else if (vec) {
+            ld8(src + (mr0 + row) * d.cols + mc0 + c8, x);
         } else {
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
                 const int64_t mr = mr0 + row, mc = mc0 + c8 + e;
-                x[e] = (mr < d.rows && mc < d.cols) ? d.mom[mr * d.cols + mc] : 0.0f;
+                x[e] = (mr < d.rows && mc < d.cols) ? src[mr * d.cols + mc] : 0.0f;
             }
         }
 #pragma unroll
@@ -227,7 +244,9 @@ struct ApplyArgs {
     int chunks;
     float lr, lr_wd, lam;
     int ef_now, hist, delayed;
-    int sapipe;               // SAPipe-WP same state: stash := x_t - U_prev, standard rule
+    int sapipe;               // SAPipe-WP: stash := x_t - U_prev, standard rule
+    int keep_hist;            // SAPipe-WP updated state: the history receives the
+                              // prediction update later (muon_predict_kernel)
     const ApplyScalars *dev;  // capturable context: lr, lr_wd, ef_now of this call
 };
 
@@ -266,6 +285,7 @@ __global__ void __launch_bounds__(kThreads) muon_apply_kernel(const ApplyArgs a)
     const bool dly = a.delayed && !d.sync;
     const bool hist = a.hist && dly, ef_now = sc.ef_now && dly;
     const bool sapipe = a.sapipe && hist;
+    const bool write_hist = hist && !a.keep_hist;
     for (int64_t e = lo + (int64_t)threadIdx.x * kPacket; e < hi; e += (int64_t)kThreads * kPacket) {
         if (e + kPacket <= hi && vec_o) {
             const int64_t i = e / d.cols, j = e - i * d.cols;
@@ -291,7 +311,7 @@ __global__ void __launch_bounds__(kThreads) muon_apply_kernel(const ApplyArgs a)
                 x[k] -= ef_now ? fmaf(a.lam, u[k] - up[k], u[k]) : u[k];
             }
             st8(d.master + e, x);
-            if (hist)
+            if (write_hist)
                 st8(d.ef + e, u);
             if (param != nullptr)
                 st8(param + e, x);
@@ -306,10 +326,46 @@ __global__ void __launch_bounds__(kThreads) muon_apply_kernel(const ApplyArgs a)
                 const float u = fmaf(lr_r, o, lr_wd * x);
                 x -= ef_now ? fmaf(a.lam, u - d.ef[q], u) : u;
                 d.master[q] = x;
-                if (hist)
+                if (write_hist)
                     d.ef[q] = u;
                 if (param != nullptr)
                     st1(param + q, x);
+            }
+        }
+    }
+}
+
+// SAPipe-WP updated state (App. B.1): the prediction update
+// U' = lr (r O' + wd X_{t+1}) of each delayed matrix into its history, O' the
+// Newton-Schulz output of M' and X_{t+1} the master the real update left.
+__global__ void __launch_bounds__(kThreads) muon_predict_kernel(const ApplyArgs a)
+{
+    const DevMat &d = a.mats[blockIdx.y];
+    if (d.sync || d.ef == nullptr)
+        return;
+    const int64_t n = d.rows * d.cols;
+    const int64_t lo = (int64_t)blockIdx.x * kChunk;
+    if (lo >= n)
+        return;
+    const int64_t hi = lo + kChunk < n ? lo + kChunk : n;
+    const ApplyScalars sc = a.dev != nullptr ? *a.dev : ApplyScalars{a.lr, a.lr_wd, a.ef_now};
+    const float lr_r = sc.lr * d.r_scale, lr_wd = sc.lr_wd * d.wd_lr_scale;
+    const bool vec_o = (d.cols % kPacket) == 0;
+    for (int64_t e = lo + (int64_t)threadIdx.x * kPacket; e < hi; e += (int64_t)kThreads * kPacket) {
+        if (e + kPacket <= hi && vec_o) {
+            const int64_t i = e / d.cols, j = e - i * d.cols;
+            float x[8], o[8], u[8];
+            ld8(d.master + e, x);
+            ld8(d.o + i * d.o_ld + j, o);
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+                u[k] = fmaf(lr_r, o[k], lr_wd * x[k]);
+            st8(d.ef + e, u);
+        } else {
+            const int64_t top = e + kPacket < hi ? e + kPacket : hi;
+            for (int64_t q = e; q < top; ++q) {
+                const int64_t i = q / d.cols, j = q - i * d.cols;
+                d.ef[q] = fmaf(lr_r, __bfloat162float(d.o[i * d.o_ld + j]), lr_wd * d.master[q]);
             }
         }
     }
@@ -469,11 +525,8 @@ struct dpo_muon_ctx {
     bool timing = false;
     std::vector<cudaEvent_t> ev_pool;
     size_t ev_used = 0;
-    // one stream per shape group for the Newton-Schulz chains (more than one
-    // group): fork after the normalisation, join before the update
-    std::vector<cudaStream_t> aux;
-    std::vector<cudaEvent_t> ev_join;
-    cudaEvent_t ev_fork = nullptr;
+    // short GEMM launches: one launch per product covers every shape group
+    bool grouped = false;
     int64_t gemm_launches = 0;
     std::string err;
 };
@@ -507,12 +560,6 @@ void free_ctx(dpo_muon_ctx *c)
         return;
     for (cudaEvent_t e : c->ev_pool)
         cudaEventDestroy(e);
-    for (cudaStream_t st : c->aux)
-        cudaStreamDestroy(st);
-    for (cudaEvent_t e : c->ev_join)
-        cudaEventDestroy(e);
-    if (c->ev_fork != nullptr)
-        cudaEventDestroy(c->ev_fork);
     if (c->ws != nullptr)
         cudaFree(c->ws);
     if (c->dev_block != nullptr)
@@ -566,10 +613,9 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
         !(hp->ns_eps >= 0.0f) || !(hp->rms_scale >= 0.0f) || (hp->delay != 0 && hp->delay != 1) ||
         !std::isfinite(hp->ns_a) || !std::isfinite(hp->ns_b) || !std::isfinite(hp->ns_c))
         return mfail(nullptr, DPO_EINVAL, "hyperparameter out of range");
-    if (hp->correction != DPO_CORR_EF && hp->correction != DPO_CORR_SAPIPE_SAME)
-        return mfail(nullptr, DPO_EINVAL,
-                     "correction must be DPO_CORR_EF or DPO_CORR_SAPIPE_SAME (the updated-state "
-                     "prediction would need a second Newton-Schulz iteration)");
+    if (hp->correction != DPO_CORR_EF && hp->correction != DPO_CORR_SAPIPE_SAME &&
+        hp->correction != DPO_CORR_SAPIPE_UPDATED)
+        return mfail(nullptr, DPO_EINVAL, "correction must be one of DPO_CORR_*");
     if (init_mode != DPO_INIT_FRESH && init_mode != DPO_INIT_RESUME)
         return mfail(nullptr, DPO_EINVAL, "bad init_mode");
     const bool ef = n > 0 && mats[0].ef != nullptr;
@@ -840,33 +886,18 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
         return e != cudaSuccess ? mcuda(nullptr, e, "GEMM launch configuration")
                                 : mfail(nullptr, DPO_ECUDA, "GEMM kernel cannot be resident");
     }
-    // Independent shape groups run their Newton-Schulz chains on streams of
-    // their own when every launch is short (at most 16 rounds of tiles over
-    // the CTA pairs): then one group's launches fill the pairs another
-    // leaves idle between launches (GPT-2-sized set: 2.28 -> 2.00 ms per
-    // step on GB300). Long launches keep one stream: two concurrent chains
-    // then mix their operands in L2 (7B set: 336 -> 410 ms).
+    // When every launch is short (at most 16 rounds of tiles over the CTA
+    // pairs), each product of a Newton-Schulz step covers all shape groups
+    // in one launch: one group's tiles fill the pairs another leaves idle,
+    // and a step takes 3 launches instead of 3 per group. Long launches keep
+    // one group per launch and run the groups' chains one after another:
+    // two chains at once mix their operands in L2 (7B set on two streams:
+    // 336 -> 410 ms per step on GB300).
     int64_t max_tiles = 0;
     for (const Group &g : c->groups)
         max_tiles = std::max<int64_t>(max_tiles, (int64_t)g.mats.size() *
                                                      (g.R / dpo::gemm::TM) * (g.W / dpo::gemm::TN));
-    if (c->groups.size() > 1 && max_tiles <= 16 * (int64_t)std::max(1, c->gemm_pairs)) {
-        bool ok = cudaEventCreateWithFlags(&c->ev_fork, cudaEventDisableTiming) == cudaSuccess;
-        for (size_t gi = 0; ok && gi < c->groups.size(); ++gi) {
-            cudaStream_t st = nullptr;
-            cudaEvent_t ev = nullptr;
-            ok = cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking) == cudaSuccess;
-            if (ok)
-                c->aux.push_back(st);
-            ok = ok && cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) == cudaSuccess;
-            if (ok)
-                c->ev_join.push_back(ev);
-        }
-        if (!ok) {
-            free_ctx(c);
-            return mfail(nullptr, DPO_ECUDA, "group streams");
-        }
-    }
+    c->grouped = c->groups.size() > 1 && max_tiles <= 16 * (int64_t)std::max(1, c->gemm_pairs);
     if (init_mode == DPO_INIT_FRESH) {
         const int rc = launch_init(c, s, 1, 1);
         if (rc != DPO_OK) {
@@ -881,25 +912,184 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
 
 namespace {
 
-int launch_gemm(dpo_muon_ctx *c, const CUtensorMap &ta, const CUtensorMap &tb,
-                const CUtensorMap &td, const CUtensorMap &tdt, const dpo::gemm::Params &p,
-                int64_t M, int64_t N, int64_t nb, bool b_mn, cudaStream_t s)
+// One product of a Newton-Schulz step for one shape group.
+struct GemmJob {
+    const CUtensorMap *ta, *tb, *td, *tdt;
+    dpo::gemm::Params p;
+    int64_t M, N, nb;
+};
+
+// One launch over up to kMaxGroups jobs of the same product (all read B
+// K-major, or all MN-major), the jobs with more K blocks first: the pairs
+// take tiles round-robin, so the longest tiles go out first and the short
+// ones fill the last round.
+int launch_gemm(dpo_muon_ctx *c, const GemmJob *jobs, int n_jobs, bool b_mn, cudaStream_t s)
 {
-    dpo::gemm::TileGrid tg{(int)(M / dpo::gemm::TM), (int)(N / dpo::gemm::TN), (int)nb, p.sym};
-    if (p.sym && M != N)
-        return mfail(c, DPO_EINVAL, "symmetric product of a non-square shape");
-    const int64_t tiles = tg.count();
+    if (n_jobs < 1 || n_jobs > dpo::gemm::kMaxGroups)
+        return mfail(c, DPO_EINVAL, "GEMM launch of %d groups", n_jobs);
+    int order[dpo::gemm::kMaxGroups];
+    for (int j = 0; j < n_jobs; ++j)
+        order[j] = j;
+    std::stable_sort(order, order + n_jobs, [&](int x, int y) {
+        return jobs[x].p.k_blocks > jobs[y].p.k_blocks;
+    });
+    dpo::gemm::GemmLaunch L;
+    std::memset(&L, 0, sizeof L);
+    int64_t tiles = 0;
+    for (int q = 0; q < n_jobs; ++q) {
+        const GemmJob &j = jobs[order[q]];
+        dpo::gemm::TileGrid tg{(int)(j.M / dpo::gemm::TM), (int)(j.N / dpo::gemm::TN), (int)j.nb,
+                               j.p.sym};
+        if (j.p.sym && j.M != j.N)
+            return mfail(c, DPO_EINVAL, "symmetric product of a non-square shape");
+        dpo::gemm::GemmGroup &G = L.g[q];
+        G.a = *j.ta;
+        G.b = *j.tb;
+        G.d = *j.td;
+        G.dt = *j.tdt;
+        G.p = j.p;
+        G.tg = tg;
+        G.tile0 = (int)tiles;
+        tiles += tg.count();
+    }
+    L.n_groups = n_jobs;
+    L.n_tiles = (int)tiles;
     // one CTA pair per co-resident cluster slot (the tile walk assumes every
     // pair runs at once)
     const int grid = 2 * (int)std::min<int64_t>(tiles, std::max(1, c->gemm_pairs));
     if (b_mn)
-        dpo::gemm::ns_gemm_kernel<true><<<grid, dpo::gemm::kThreads, dpo::gemm::kSmemBytes, s>>>(
-            ta, tb, td, tdt, p, tg);
+        dpo::gemm::ns_gemm_kernel<true><<<grid, dpo::gemm::kThreads, dpo::gemm::kSmemBytes, s>>>(L);
     else
-        dpo::gemm::ns_gemm_kernel<false><<<grid, dpo::gemm::kThreads, dpo::gemm::kSmemBytes, s>>>(
-            ta, tb, td, tdt, p, tg);
+        dpo::gemm::ns_gemm_kernel<false><<<grid, dpo::gemm::kThreads, dpo::gemm::kSmemBytes, s>>>(L);
+    if (c->timing)
+        ++c->gemm_launches;
     const cudaError_t e = cudaGetLastError();
     return e == cudaSuccess ? DPO_OK : mcuda(c, e, "Newton-Schulz GEMM launch");
+}
+
+}  // namespace
+
+namespace {
+
+// Momentum (M <- mu M + (1 - mu) G^, or with `predict` M' into the history
+// buffers), its Frobenius norms, the normalisation into the workspace and the
+// Newton-Schulz chains of every shape group: the Newton-Schulz output of each
+// matrix is then in the workspace (DevMat::o).
+int orthogonalize(dpo_muon_ctx *c, cudaStream_t s, bool predict)
+{
+    // momentum and its Frobenius norms
+    dpo::muon::MomArgs ma{};
+    ma.mats = c->d_mats;
+    ma.clip = c->hp.max_grad_norm > 0.0f ? &c->d_norm_scalars->clip : nullptr;
+    ma.mu = c->hp.momentum;
+    ma.omm = (float)(1.0 - (double)c->hp.momentum);
+    ma.partials = c->d_partials;
+    ma.chunks = c->chunks;
+    ma.predict = predict ? 1 : 0;
+    const dim3 mgrid((unsigned)c->chunks, (unsigned)c->n);
+    if (c->grad_dt == DPO_BF16)
+        dpo::muon::muon_momentum_kernel<__nv_bfloat16><<<mgrid, kThreads, 0, s>>>(ma);
+    else
+        dpo::muon::muon_momentum_kernel<float><<<mgrid, kThreads, 0, s>>>(ma);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess)
+        return mcuda(c, e, "momentum launch");
+    dpo::muon::muon_norm_kernel<<<(c->n + 7) / 8, 256, 0, s>>>(c->d_partials, c->chunks, c->n,
+                                                               c->hp.ns_eps, c->d_inv_norm);
+    if ((e = cudaGetLastError()) != cudaSuccess)
+        return mcuda(c, e, "norm launch");
+
+    for (Group &g : c->groups) {
+        const int64_t nb = (int64_t)g.mats.size();
+        dpo::muon::NormArgsM na{c->d_mats, g.d_mats, c->d_inv_norm, g.x[0],
+                                c->hp.ns_steps == 0 ? g.xt : nullptr, g.R, g.W, g.r, g.w,
+                                predict ? 1 : 0};
+        const dim3 ngrid((unsigned)(g.W / 64), (unsigned)(g.R / 64), (unsigned)nb);
+        dpo::muon::muon_normalize_kernel<<<ngrid, kThreads, 0, s>>>(na);
+        if ((e = cudaGetLastError()) != cudaSuccess)
+            return mcuda(c, e, "normalize launch");
+    }
+    cudaEvent_t ev_end = nullptr;
+    if (c->timing && c->hp.ns_steps > 0) {
+        if (c->ev_used + 2 > c->ev_pool.size()) {
+            for (int q = 0; q < 2; ++q) {
+                cudaEvent_t ev;
+                if ((e = cudaEventCreate(&ev)) != cudaSuccess)
+                    return mcuda(c, e, "timing event");
+                c->ev_pool.push_back(ev);
+            }
+        }
+        if ((e = cudaEventRecord(c->ev_pool[c->ev_used], s)) != cudaSuccess)
+            return mcuda(c, e, "timing event record");
+        ev_end = c->ev_pool[c->ev_used + 1];
+        c->ev_used += 2;
+    }
+    // Newton-Schulz, per step: A = X X^T, B = c A A + b A, X <- B X + a X.
+    // Short launches (c->grouped) take the same product of up to kMaxGroups
+    // shape groups in one launch, step by step; long ones run one group's
+    // chain after another, one launch per product.
+    auto stall_next = [c]() {
+        if (c->stall_launches <= 0)
+            return 0;
+        --c->stall_launches;
+        return 1;
+    };
+    const int n_groups = (int)c->groups.size();
+    const int per = c->grouped ? dpo::gemm::kMaxGroups : 1;
+    for (int g0 = 0; g0 < n_groups; g0 += per) {
+        const int n = std::min(per, n_groups - g0);
+        for (int it = 0; it < c->hp.ns_steps; ++it) {
+            const bool last = it + 1 == c->hp.ns_steps;
+            const int cur = it % 2, nxt = cur ^ 1;
+            GemmJob xx[dpo::gemm::kMaxGroups], aa[dpo::gemm::kMaxGroups],
+                bx[dpo::gemm::kMaxGroups];
+            const int st_xx = stall_next(), st_aa = stall_next(), st_bx = stall_next();
+            for (int q = 0; q < n; ++q) {
+                Group &g = c->groups[g0 + q];
+                const int64_t nb = (int64_t)g.mats.size();
+                dpo::gemm::Params p{};
+                p.err = c->d_err;
+                // A = X X^T
+                p.alpha = 1.0f;
+                p.k_blocks = (int)(g.W / dpo::gemm::BK);
+                p.sym = 1;
+                p.stall = st_xx;
+                xx[q] = GemmJob{&g.x128[cur], &g.x128[cur], &g.st_a, &g.st_a, p, g.R, g.R, nb};
+                // B = c A A + b A
+                p.c = g.a;
+                p.ldc = g.R;
+                p.c_bstride = g.R * g.R;
+                p.alpha = c->hp.ns_c;
+                p.beta = c->hp.ns_b;
+                p.k_blocks = (int)(g.R / dpo::gemm::BK);
+                p.stall = st_aa;
+                aa[q] = GemmJob{&g.a128, &g.a128, &g.st_b, &g.st_b, p, g.R, g.R, nb};
+                // X <- B X + a X (X read MN-major in place of X^T), and at the
+                // last step X^T for the tall matrices' output
+                p.sym = 0;
+                p.trans = last && g.has_tall ? 1 : 0;
+                p.c = g.x[cur];
+                p.ldc = g.W;
+                p.c_bstride = g.R * g.W;
+                p.alpha = 1.0f;
+                p.beta = c->hp.ns_a;
+                p.k_blocks = (int)(g.R / dpo::gemm::BK);
+                p.stall = st_bx;
+                bx[q] = GemmJob{&g.b128, &g.x_mn[cur], &g.st_x[nxt], &g.st_xt, p, g.R, g.W, nb};
+            }
+            int rc = launch_gemm(c, xx, n, false, s);
+            if (rc == DPO_OK)
+                rc = launch_gemm(c, aa, n, false, s);
+            if (rc == DPO_OK)
+                rc = launch_gemm(c, bx, n, true, s);
+            if (rc != DPO_OK)
+                return rc;
+        }
+    }
+    if (ev_end != nullptr && (e = cudaEventRecord(ev_end, s)) != cudaSuccess)
+        return mcuda(c, e, "timing event record");
+
+    return DPO_OK;
 }
 
 }  // namespace
@@ -941,115 +1131,11 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
         if (e != cudaSuccess)
             return mcuda(c, e, "norm launch");
     }
-    // momentum and its Frobenius norms
-    dpo::muon::MomArgs ma{};
-    ma.mats = c->d_mats;
-    ma.clip = clip ? &c->d_norm_scalars->clip : nullptr;
-    ma.mu = c->hp.momentum;
-    ma.omm = (float)(1.0 - (double)c->hp.momentum);
-    ma.partials = c->d_partials;
-    ma.chunks = c->chunks;
+    int rc = orthogonalize(c, s, false);
+    if (rc != DPO_OK)
+        return rc;
+    cudaError_t e;
     const dim3 mgrid((unsigned)c->chunks, (unsigned)c->n);
-    if (c->grad_dt == DPO_BF16)
-        dpo::muon::muon_momentum_kernel<__nv_bfloat16><<<mgrid, kThreads, 0, s>>>(ma);
-    else
-        dpo::muon::muon_momentum_kernel<float><<<mgrid, kThreads, 0, s>>>(ma);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess)
-        return mcuda(c, e, "momentum launch");
-    dpo::muon::muon_norm_kernel<<<(c->n + 7) / 8, 256, 0, s>>>(c->d_partials, c->chunks, c->n,
-                                                               c->hp.ns_eps, c->d_inv_norm);
-    if ((e = cudaGetLastError()) != cudaSuccess)
-        return mcuda(c, e, "norm launch");
-
-    for (Group &g : c->groups) {
-        const int64_t nb = (int64_t)g.mats.size();
-        dpo::muon::NormArgsM na{c->d_mats, g.d_mats, c->d_inv_norm, g.x[0],
-                                c->hp.ns_steps == 0 ? g.xt : nullptr, g.R, g.W, g.r, g.w};
-        const dim3 ngrid((unsigned)(g.W / 64), (unsigned)(g.R / 64), (unsigned)nb);
-        dpo::muon::muon_normalize_kernel<<<ngrid, kThreads, 0, s>>>(na);
-        if ((e = cudaGetLastError()) != cudaSuccess)
-            return mcuda(c, e, "normalize launch");
-    }
-    cudaEvent_t ev_end = nullptr;
-    if (c->timing && c->hp.ns_steps > 0) {
-        if (c->ev_used + 2 > c->ev_pool.size()) {
-            for (int q = 0; q < 2; ++q) {
-                cudaEvent_t ev;
-                if ((e = cudaEventCreate(&ev)) != cudaSuccess)
-                    return mcuda(c, e, "timing event");
-                c->ev_pool.push_back(ev);
-            }
-        }
-        if ((e = cudaEventRecord(c->ev_pool[c->ev_used], s)) != cudaSuccess)
-            return mcuda(c, e, "timing event record");
-        ev_end = c->ev_pool[c->ev_used + 1];
-        c->ev_used += 2;
-        c->gemm_launches += 3 * (int64_t)c->hp.ns_steps * (int64_t)c->groups.size();
-    }
-    const bool fork = !c->aux.empty() && c->hp.ns_steps > 0;
-    if (fork && (e = cudaEventRecord(c->ev_fork, s)) != cudaSuccess)
-        return mcuda(c, e, "fork event");
-    for (size_t gi = 0; gi < c->groups.size(); ++gi) {
-        Group &g = c->groups[gi];
-        const int64_t nb = (int64_t)g.mats.size();
-        cudaStream_t gs = fork ? c->aux[gi] : s;
-        if (fork && (e = cudaStreamWaitEvent(gs, c->ev_fork, 0)) != cudaSuccess)
-            return mcuda(c, e, "fork wait");
-        for (int it = 0; it < c->hp.ns_steps; ++it) {
-            const bool last = it + 1 == c->hp.ns_steps;
-            const int cur = it % 2, nxt = cur ^ 1;
-            dpo::gemm::Params p{};
-            p.err = c->d_err;
-            auto stall_next = [c]() {
-                if (c->stall_launches <= 0)
-                    return 0;
-                --c->stall_launches;
-                return 1;
-            };
-            // A = X X^T
-            p.alpha = 1.0f;
-            p.k_blocks = (int)(g.W / dpo::gemm::BK);
-            p.sym = 1;
-            p.stall = stall_next();
-            int rc = launch_gemm(c, g.x128[cur], g.x128[cur], g.st_a, g.st_a, p, g.R, g.R, nb,
-                                 false, gs);
-            if (rc != DPO_OK)
-                return rc;
-            // B = c A A + b A
-            p.c = g.a;
-            p.ldc = g.R;
-            p.c_bstride = g.R * g.R;
-            p.alpha = c->hp.ns_c;
-            p.beta = c->hp.ns_b;
-            p.k_blocks = (int)(g.R / dpo::gemm::BK);
-            p.stall = stall_next();
-            if ((rc = launch_gemm(c, g.a128, g.a128, g.st_b, g.st_b, p, g.R, g.R, nb, false, gs)) !=
-                DPO_OK)
-                return rc;
-            // X <- B X + a X (X read MN-major in place of X^T), and at the
-            // last step X^T for the tall matrices' output
-            p.sym = 0;
-            p.trans = last && g.has_tall ? 1 : 0;
-            p.c = g.x[cur];
-            p.ldc = g.W;
-            p.c_bstride = g.R * g.W;
-            p.alpha = 1.0f;
-            p.beta = c->hp.ns_a;
-            p.k_blocks = (int)(g.R / dpo::gemm::BK);
-            p.stall = stall_next();
-            if ((rc = launch_gemm(c, g.b128, g.x_mn[cur], g.st_x[nxt], g.st_xt, p, g.R, g.W, nb,
-                                  true, gs)) != DPO_OK)
-                return rc;
-        }
-        if (fork) {
-            if ((e = cudaEventRecord(c->ev_join[gi], gs)) != cudaSuccess ||
-                (e = cudaStreamWaitEvent(s, c->ev_join[gi], 0)) != cudaSuccess)
-                return mcuda(c, e, "join");
-        }
-    }
-    if (ev_end != nullptr && (e = cudaEventRecord(ev_end, s)) != cudaSuccess)
-        return mcuda(c, e, "timing event record");
 
     // update, stash, history, weights
     const int64_t t = k - c->phase_k0;   // Alg. 1 iteration within the delayed phase
@@ -1060,7 +1146,9 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
     aa.lr_wd = (float)((double)lr * (double)c->hp.weight_decay);
     aa.delayed = c->hp.delay == 1;
     aa.hist = c->ef && c->hp.delay == 1;
-    aa.sapipe = c->hp.correction == DPO_CORR_SAPIPE_SAME;
+    const bool updated = c->hp.correction == DPO_CORR_SAPIPE_UPDATED;
+    aa.sapipe = c->hp.correction == DPO_CORR_SAPIPE_SAME || updated;
+    aa.keep_hist = updated;
     aa.ef_now = aa.hist && !aa.sapipe && t >= 2 && c->hp.ef_lambda != 0.0f;
     aa.lam = c->hp.ef_lambda;
     if (c->capturable) {   // lr and EF's start from the device counters
@@ -1080,6 +1168,15 @@ extern "C" int dpo_muon_step(dpo_muon_ctx *c, float lr, void *stream)
         dpo::muon::muon_apply_kernel<dpo::kStashF32><<<mgrid, kThreads, 0, s>>>(aa);
     if ((e = cudaGetLastError()) != cudaSuccess)
         return mcuda(c, e, "apply launch");
+    if (updated && aa.hist) {
+        // SAPipe-WP updated state: the step once more on the same gradient
+        // from the momentum just stored, decaying X_{t+1}, into the history
+        if ((rc = orthogonalize(c, s, true)) != DPO_OK)
+            return rc;
+        dpo::muon::muon_predict_kernel<<<mgrid, kThreads, 0, s>>>(aa);
+        if ((e = cudaGetLastError()) != cudaSuccess)
+            return mcuda(c, e, "prediction launch");
+    }
     if (!c->capturable)
         c->k = k;
     return DPO_OK;
@@ -1303,7 +1400,10 @@ extern "C" int dpo_muon_flops(const dpo_muon_ctx *c, double *flops)
 {
     if (c == nullptr || flops == nullptr)
         return DPO_EINVAL;
-    *flops = c->flops;
+    // the updated-state prediction runs the Newton-Schulz chains a second
+    // time (delayed training with history buffers)
+    const bool twice = c->hp.correction == DPO_CORR_SAPIPE_UPDATED && c->ef && c->hp.delay == 1;
+    *flops = twice ? 2.0 * c->flops : c->flops;
     return DPO_OK;
 }
 

@@ -88,7 +88,7 @@ def _muon_init(mats, hp=None, sdt=dpo.DPO_BF16, gdt=dpo.DPO_BF16, mode=0):
     ("ns_steps", dpo.DPO_EINVAL), ("negative_shape", dpo.DPO_EINVAL),
     ("no_stash", dpo.DPO_EINVAL), ("ef_mismatch", dpo.DPO_EINVAL),
     ("misaligned", dpo.DPO_EALIGN), ("no_master", dpo.DPO_EINVAL), ("bad_mode", dpo.DPO_EINVAL),
-    ("sapipe_updated", dpo.DPO_EINVAL)])
+    ("bad_correction", dpo.DPO_EINVAL)])
 def test_muon_init_rejects(case, code):
     mats, hp, kw = [_m(0), _m(1, rows=300, cols=20)], muon.hparams(), {}
     if case == "bad_dtype":
@@ -109,8 +109,8 @@ def test_muon_init_rejects(case, code):
         mats[1] = _m(1, master=None)
     elif case == "bad_mode":
         kw["mode"] = 5
-    elif case == "sapipe_updated":
-        hp = muon.hparams(correction=dpo.DPO_CORR_SAPIPE_UPDATED)
+    elif case == "bad_correction":
+        hp = muon.hparams(correction=3)
     rc, out, msg = _muon_init(mats, hp, **kw)
     assert rc == code and out is None and msg
 

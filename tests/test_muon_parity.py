@@ -280,6 +280,44 @@ def test_muon_sapipe_same_state(cuda_device):
         p.close()
 
 
+@pytest.mark.parametrize("sync,clip,ns_steps", [(None, 0.0, 1), ([i % 3 == 1 for i in range(9)], 0.5, 1),
+                                           (None, 0.0, 5)])
+def test_muon_sapipe_updated_state(cuda_device, sync, clip, ns_steps):
+    """SAPipe-WP with the updated state (App. B.1): the history holds the
+    prediction update U' = lr (r NS(mu M + (1 - mu) G^) + wd X_{t+1}) from a
+    second Newton-Schulz chain, the stash X_t - U'_prev, the weights the
+    standard rule; a synchronous matrix (every third) keeps a zero history
+    and no stash; with clipping, the prediction consumes the clipped
+    gradient. U' carries the flip bound of one Newton-Schulz output (module
+    note) and the stash that of the previous call's U' and weights; with 5
+    Newton-Schulz steps, where the two bf16 iterations decorrelate, U' is
+    held to the 5-step output bar, normwise (Frobenius, over the delayed
+    matrices), as test_newton_schulz_parity holds O."""
+    p = Pair(SHAPES, cuda_device, ns_steps=ns_steps, ef=True, correction=2, sync=sync,
+             max_grad_norm=clip)
+    r_max = 0.2 * np.sqrt(max(max(sh) for sh in SHAPES))
+    du = p.lr * r_max * 2.0 ** -7
+    keep = np.concatenate([np.full(r * c, not p.sync[i]) for i, (r, c) in enumerate(SHAPES)])
+    try:
+        for k in range(5):
+            p.step()
+            assert rel_err(p.cat(p.gpu.mom), _flat(p.ref.mom)) <= (TOL_ONE_STEP if k == 0
+                                                                    else TOL_RUN)
+            u, ur = p.cat(p.gpu.ef), _flat(p.ref.u_prev)
+            assert np.all(u[~keep] == 0.0)
+            if ns_steps == 1:
+                close_with_flips(p.cat(p.gpu.master), _flat(p.ref.x), TOL_RUN, (k + 1) * du, 1e-3)
+                close_with_flips(u[keep], ur[keep], 1e-5, du, 2e-3)
+                close_with_flips(p.cat(p.gpu.stash).astype(np.float64)[keep],
+                                 _flat(p.ref.stash)[keep], 2.0 ** -7, (k + 1) * du, 1e-3)
+            else:
+                norm = np.linalg.norm(u[keep] - ur[keep]) / np.linalg.norm(ur[keep])
+                print(f"call {k + 1}: U' normwise {norm:.3e}")
+                assert norm <= 1.5e-2, (k, norm)
+    finally:
+        p.close()
+
+
 def test_muon_clipping(cuda_device):
     """Global clipping over all matrices scales the gradient before the
     momentum (the norm of these gradients is ~1.3)."""
