@@ -78,6 +78,10 @@ def parse_args(argv=None):
     p.add_argument("--no-secondary", action="store_true",
                    help="skip the clipped Llama-1B step (norm pass and fused step timed apart)")
     p.add_argument("--secondary-steps", type=int, default=10)
+    p.add_argument("--no-muon-secondary", action="store_true",
+                   help="skip the delayed-Muon step on the same set after the headline")
+    p.add_argument("--muon-steps", type=int, default=5,
+                   help="timed steps of the delayed-Muon entry of the default line")
     p.add_argument("--parallel", choices=["shard", "replica"], default="shard",
                    help="N > 1: shard (each rank steps its contiguous share of the set, "
                         "ZeRO-1 style; clipping takes one fp64 all-reduce of the squared "
@@ -523,6 +527,36 @@ def run_secondary(args, dev, world):
                      "achieved_gbs": (norm_bytes + step_bytes) / (pair_ms / 1e3) / 1e9,
                      "frac": (norm_bytes + step_bytes) / (pair_ms / 1e3) / 1e9 / peak,
                      "kernel_ms": pair_ms}}
+
+
+def run_muon_secondary(args, w, world, rank, local):
+    """Delayed Muon (Alg. 2, EF) on the headline set's attention and MLP
+    matrices with AdamW EF on the rest, as ``--optimizer muon`` times it: the
+    Newton-Schulz GEMM chains by the library's CUDA events against the
+    sustained bf16 tensor peak. Runs after the headline's arenas are freed."""
+    import torch
+
+    gc.collect()
+    torch.cuda.empty_cache()
+    a = argparse.Namespace(**vars(args))
+    a.mode, a.ns_steps, a.graph, a.no_library_ns = "ef", 5, False, True
+    a.steps, a.warmup = max(1, args.muon_steps), max(3, min(args.warmup, 3))
+    r = run_muon(a, w, world, rank, local)
+    torch.cuda.empty_cache()
+    peak, peak_kind = measured_bf16_peak()
+    mi, ai = muon_split(w)
+    return {"workload": f"{w.name}: {w.n_params} params; delayed Muon (Alg. 2, 5 Newton-Schulz "
+                        f"steps, EF) on {len(mi)} attention/MLP matrices ({r['n_muon']} params), "
+                        f"AdamW EF on the other {len(ai)} tensors, one-step delay",
+            "value": r["value"], "unit": UNIT, "steps": a.steps, "warmup": a.warmup,
+            "ms_per_step": r["t_max"] / a.steps * 1e3,
+            "gemm": {"kernel": "ns_gemm_kernel", "bound": "tensor",
+                     "gemm_ms_per_step": r["gemm_ms"],
+                     "algorithmic_flops_per_step": r["flops"],
+                     "achieved": r["achieved"], "unit": "TFLOP/s", "peak": peak,
+                     "peak_kind": f"{peak_kind} (sustained)", "frac": r["achieved"] / peak,
+                     "traffic": committed_traffic(ns_gemm_tag(w.name, 5), "dram_bytes_per_step")},
+            "gpu_launches": r["launches"], "clocks": r["clocks"]}
 
 
 def muon_split(w):
@@ -991,9 +1025,12 @@ def main(argv=None):
         torch.cuda.set_device(local)
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     r = run_gpu(args, w, world, rank, local)
-    secondary = None
+    secondary = muon_entry = None
     if not args.no_secondary and w.name == "llama-7B":
         secondary = run_secondary(args, torch.device("cuda", local), world)
+    if (not args.no_muon_secondary and w.name == "llama-7B" and args.optimizer == "adamw"
+            and not sharded(args, world)):
+        muon_entry = run_muon_secondary(args, w, world, rank, local)
     peak, peak_kind = measured_hbm_peak()
     # the tag names every setting that changes the kernel's traffic; the
     # headline keeps "fused_step:<set>:<mode>[:pingpong]"
@@ -1035,6 +1072,8 @@ def main(argv=None):
             "hbm_gbs_achieved": r["achieved"], "device": r["device_name"]}
     if secondary is not None:
         line["secondary"] = secondary
+    if muon_entry is not None:
+        line["muon"] = muon_entry
     print(json.dumps(line), flush=True)
     return 0
 

@@ -127,7 +127,7 @@ typedef enum { DPO_F32 = 0, DPO_BF16 = 1 } dpo_dtype;
  *                  v = beta2 v + (1-beta2) diff, n = beta3 n + (1-beta3)(g + beta2 diff)^2,
  *                  u = lr ((m/(1-beta1^k) + beta2 v/(1-beta2^k)) / (sqrt(n/(1-beta3^k)) + eps)
  *                      + wd x_t); needs the n and grad_prev buffers.
- * DPO_CORR_SAPIPE_UPDATED is defined for AdamW only. */
+ * Every rule takes every correction (DPO_CORR_*). */
 /* dpo_hparams.stash_mode. PipeDream-2BW keeps two weight versions (Sec. 2):
  *   DPO_STASH_COPY      the step writes x_t into the stash buffer and
  *                       x_{t+1} into the param buffer (every layout).
