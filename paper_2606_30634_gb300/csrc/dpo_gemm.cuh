@@ -498,12 +498,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         // waits for the group of two chunks back before they are rewritten.
         const int q = warp & 3;
         const uint32_t wbuf = ring + (uint32_t)(kStages * kStageBytes + q * 4 * kChunkBytes);
-        // The addend C (c A A + b A, B X + a X) is read 32 columns per lane per
-        // chunk, kCPre chunks ahead of their use, the first ones before the
-        // accumulator is ready: where K is short (768) the MMAs of a tile
-        // take a few microseconds, and one dependent global load per chunk
-        // made the epilogue the bottleneck. C is never the launch's output.
+        // The addend C (c A A + b A, B X + a X) is read kCPre chunks ahead of
+        // its use, the first ones before the accumulator is ready, coalesced:
+        // lane l loads granule l % 4 (8 columns) of rows l / 4 + 8 i of the
+        // warp's 32 x 32 chunk, 8 rows of 64 bytes per instruction; the chunk
+        // is then turned through its staging buffer so that each lane holds
+        // its own row. Loads of each lane's own row touched 32 lines per
+        // instruction, and where K is short (768) their L1 wavefronts, about
+        // two thirds of a tile's MMA time per SM, held the epilogue back.
+        // C is never the launch's output.
         constexpr int kCPre = 4;
+        const int crs = lane >> 2, cg = lane & 3;   // coalesced load: sub-row, granule
         int lt = 0, staged = 0;
         for (int t = pair; t < n_tiles; t += n_pairs) {
             int b, m0, n0;
@@ -511,16 +516,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             const Params &p = G.p;
             const int a = lt & 1;
             const int row0 = m0 + (int)rank * BM + q * 32;
-            const int64_t row = row0 + lane;
+            // C at (row0 + crs, n0 + 8 cg); rows 8 i further for i = 0..3
             const __nv_bfloat16 *crow =
-                p.c != nullptr ? p.c + (int64_t)b * p.c_bstride + row * p.ldc + n0 : nullptr;
+                p.c != nullptr ? p.c + (int64_t)b * p.c_bstride + (int64_t)(row0 + crs) * p.ldc +
+                                     n0 + cg * 8
+                               : nullptr;
+            const int64_t c8 = 8 * p.ldc;
             uint4 cpre[kCPre][4];
             if (crow != nullptr) {
 #pragma unroll
                 for (int c = 0; c < kCPre; ++c)
 #pragma unroll
-                    for (int j8 = 0; j8 < 4; ++j8)
-                        cpre[c][j8] = __ldg(reinterpret_cast<const uint4 *>(crow + c * 32 + j8 * 8));
+                    for (int i = 0; i < 4; ++i)
+                        cpre[c][i] = __ldg(reinterpret_cast<const uint4 *>(crow + i * c8 + c * 32));
             }
             const bool seen = mbar_wait(acc_full(a), (uint32_t)(lt >> 1) & 1u);
             if (!seen)
@@ -538,22 +546,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int j = 0; j < 32; ++j)
                     v[j] = p.alpha * __uint_as_float(r[j]);
-                if (crow != nullptr) {
-#pragma unroll
-                    for (int j8 = 0; j8 < 4; ++j8) {
-                        const uint4 cv = cpre[ch % kCPre][j8];
-                        if (ch + kCPre < TN / 32)   // the slot's next chunk
-                            cpre[ch % kCPre][j8] = __ldg(
-                                reinterpret_cast<const uint4 *>(crow + (ch + kCPre) * 32 + j8 * 8));
-                        const __nv_bfloat162 *c2 = reinterpret_cast<const __nv_bfloat162 *>(&cv);
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const float2 f = __bfloat1622float2(c2[e]);
-                            v[j8 * 8 + 2 * e] = fmaf(p.beta, f.x, v[j8 * 8 + 2 * e]);
-                            v[j8 * 8 + 2 * e + 1] = fmaf(p.beta, f.y, v[j8 * 8 + 2 * e + 1]);
-                        }
-                    }
-                }
                 const int col0 = n0 + ch * 32;
                 // Mirror of a symmetric product: (col, row) lies in the tile
                 // (col / TM, row / TN), not computed when row / TN < col / TM
@@ -566,6 +558,37 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 if (lane == 0)   // the buffers' previous group has been read
                     asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
                 __syncwarp();
+                if (crow != nullptr) {
+                    // the coalesced chunk of C into rb, then this lane's row out
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const uint4 cv = cpre[ch % kCPre][i];
+                        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};"
+                                     ::"r"(rb + swz64(crs + 8 * i, cg)), "r"(cv.x), "r"(cv.y),
+                                       "r"(cv.z), "r"(cv.w)
+                                     : "memory");
+                        if (ch + kCPre < TN / 32)   // the slot's next chunk
+                            cpre[ch % kCPre][i] = __ldg(
+                                reinterpret_cast<const uint4 *>(crow + i * c8 + (ch + kCPre) * 32));
+                    }
+                    __syncwarp();
+#pragma unroll
+                    for (int g = 0; g < 4; ++g) {
+                        uint4 cv;
+                        asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                                     : "=r"(cv.x), "=r"(cv.y), "=r"(cv.z), "=r"(cv.w)
+                                     : "r"(rb + swz64(lane, g))
+                                     : "memory");
+                        const __nv_bfloat162 *c2 = reinterpret_cast<const __nv_bfloat162 *>(&cv);
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const float2 f = __bfloat1622float2(c2[e]);
+                            v[g * 8 + 2 * e] = fmaf(p.beta, f.x, v[g * 8 + 2 * e]);
+                            v[g * 8 + 2 * e + 1] = fmaf(p.beta, f.y, v[g * 8 + 2 * e + 1]);
+                        }
+                    }
+                    // each lane rewrites only the row it has read
+                }
 #pragma unroll
                 for (int g = 0; g < 4; ++g) {
                     const uint32_t w0 = pack_bf16(v[g * 8 + 0], v[g * 8 + 1]);
