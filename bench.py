@@ -1026,11 +1026,19 @@ def main(argv=None):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     r = run_gpu(args, w, world, rank, local)
     secondary = muon_entry = None
+    # The extra entries never cost the headline its line: a failure is
+    # reported in the entry instead.
     if not args.no_secondary and w.name == "llama-7B":
-        secondary = run_secondary(args, torch.device("cuda", local), world)
+        try:
+            secondary = run_secondary(args, torch.device("cuda", local), world)
+        except Exception as e:   # noqa: BLE001
+            secondary = {"error": f"{type(e).__name__}: {e}"}
     if (not args.no_muon_secondary and w.name == "llama-7B" and args.optimizer == "adamw"
             and not sharded(args, world)):
-        muon_entry = run_muon_secondary(args, w, world, rank, local)
+        try:
+            muon_entry = run_muon_secondary(args, w, world, rank, local)
+        except Exception as e:   # noqa: BLE001
+            muon_entry = {"error": f"{type(e).__name__}: {e}"}
     peak, peak_kind = measured_hbm_peak()
     # the tag names every setting that changes the kernel's traffic; the
     # headline keeps "fused_step:<set>:<mode>[:pingpong]"
