@@ -886,18 +886,20 @@ extern "C" int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n,
         return e != cudaSuccess ? mcuda(nullptr, e, "GEMM launch configuration")
                                 : mfail(nullptr, DPO_ECUDA, "GEMM kernel cannot be resident");
     }
-    // When every launch is short (at most 16 rounds of tiles over the CTA
-    // pairs), each product of a Newton-Schulz step covers all shape groups
-    // in one launch: one group's tiles fill the pairs another leaves idle,
-    // and a step takes 3 launches instead of 3 per group. Long launches keep
-    // one group per launch and run the groups' chains one after another:
-    // two chains at once mix their operands in L2 (7B set on two streams:
-    // 336 -> 410 ms per step on GB300).
-    int64_t max_tiles = 0;
+    // When some shape group's launches are short (at most 16 rounds of tiles
+    // over the CTA pairs), each product of a Newton-Schulz step covers all
+    // shape groups in one launch: one group's tiles fill the pairs another
+    // leaves idle, and a step takes 3 launches instead of 3 per group (GPT-2:
+    // every group short; the Llama-1B set's 512 x 2048 group: 20.08 -> 19.80
+    // ms of GEMMs per step on GB300). Sets whose groups are all long keep one
+    // group per launch and run the groups' chains one after another (7B set:
+    // 0.3% slower grouped; two chains at once on two streams mixed their
+    // operands in L2, 336 -> 410 ms per step).
+    int64_t min_tiles = INT64_MAX;
     for (const Group &g : c->groups)
-        max_tiles = std::max<int64_t>(max_tiles, (int64_t)g.mats.size() *
+        min_tiles = std::min<int64_t>(min_tiles, (int64_t)g.mats.size() *
                                                      (g.R / dpo::gemm::TM) * (g.W / dpo::gemm::TN));
-    c->grouped = c->groups.size() > 1 && max_tiles <= 16 * (int64_t)std::max(1, c->gemm_pairs);
+    c->grouped = c->groups.size() > 1 && min_tiles <= 16 * (int64_t)std::max(1, c->gemm_pairs);
     if (init_mode == DPO_INIT_FRESH) {
         const int rc = launch_init(c, s, 1, 1);
         if (rc != DPO_OK) {
