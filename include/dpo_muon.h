@@ -110,8 +110,9 @@ int dpo_muon_init(dpo_muon_ctx **out, const dpo_matrix *mats, int n, dpo_dtype s
 /*
  * One iteration with learning rate lr (> 0) for every matrix, enqueued on
  * stream: the norm pass when clipping, the momentum pass, the
- * normalisation pass, 3 ns_steps GEMM launches per matrix shape and the
- * update pass. Returns DPO_OK, DPO_EINVAL or DPO_ECUDA.
+ * normalisation pass, 3 ns_steps GEMM launches per matrix shape (or, when
+ * some shape's launches are short, per set of up to four shapes sharing each
+ * launch) and the update pass. Returns DPO_OK, DPO_EINVAL or DPO_ECUDA.
  */
 int dpo_muon_step(dpo_muon_ctx *ctx, float lr, void *cuda_stream);
 
@@ -211,8 +212,8 @@ int dpo_muon_flops(const dpo_muon_ctx *ctx, double *flops);
 
 /*
  * Measurement of the tensor-core work: with on != 0, each later dpo_muon_step
- * brackets every matrix shape's chain of Newton-Schulz GEMM launches with a
- * pair of CUDA events recorded on its stream. dpo_muon_get_gemm_time waits
+ * brackets its Newton-Schulz GEMM launches (every shape's chain) with a pair
+ * of CUDA events recorded on its stream. dpo_muon_get_gemm_time waits
  * for those events, returns the summed milliseconds and the number of GEMM
  * launches since the previous read, and starts a new count. Returns DPO_OK,
  * DPO_EINVAL or DPO_ECUDA.
