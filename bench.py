@@ -616,9 +616,12 @@ def run_muon(args, w, world, rank, local):
     torch.cuda.synchronize(dev)
     flops = mo.flops()
     n_groups = len({(min(r, c), max(r, c)) for r, c in shapes})
-    launches_per_step = 1 + 3 + n_groups * (1 + 3 * args.ns_steps)
-    if corr == 2:   # the updated-state prediction: momentum, norm, predict, a second chain
-        launches_per_step += 3 + n_groups * (1 + 3 * args.ns_steps)
+    # AdamW's fused step; momentum, norm, apply; one normalisation per shape
+    # group (the GEMM launches are counted by the library: shape groups may
+    # share them)
+    other_launches_per_step = 1 + 3 + n_groups
+    if corr == 2:   # the updated-state prediction: momentum, norm, predict, normalisations
+        other_launches_per_step += 3 + n_groups
 
     mo.set_timing(True)
     for _ in range(args.warmup):
@@ -680,7 +683,8 @@ def run_muon(args, w, world, rank, local):
         raise RuntimeError(f"tensor-core pipeline status {status}")
     library = None if args.no_library_ns else library_ns(shapes, args.ns_steps, dev)
     return dict(value=value, t_max=t_max, achieved=achieved, flops=flops, gemm_ms=gemm_ms / K,
-                gemm_launches=gemm_launches, clocks=clocks, launches=K * launches_per_step,
+                gemm_launches=gemm_launches, clocks=clocks,
+                launches=K * other_launches_per_step + gemm_launches,
                 n_muon=sum(w.numels[i] for i in mi), n_matrices=len(mi), workspace=ws,
                 device_name=props.name, library=library, graph=graph)
 
