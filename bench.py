@@ -774,13 +774,18 @@ def e2e_fits(avail: int, io_bytes: int, local_world: int) -> bool:
 
 
 def run_e2e(args, opt, one_step, stream, dev, world, w):
-    """End to end through the public API with the step's inputs (gradients)
-    in pinned host memory and its result (the new bf16 weights) delivered to
-    pinned host memory, transfers inside the timed region. The library's
-    host-I/O mode does the transfers inside the fused kernel, over the host
-    link; a staged variant (cudaMemcpy in, device step, cudaMemcpy out) is
-    reported beside it."""
+    """End to end through the public API, transfers inside the timed region:
+    each step's inputs (the gradients) come from pinned host memory and each
+    step's result is read back to the host. The library's host-I/O mode does
+    the input transfer inside the fused kernel, over the host link. The main
+    figure reads back the step's diagnostics (flags, gradient norm, clip
+    coefficient: dpo_get_flags), the new bf16 weights staying on the device
+    for the next forward as in training; `weights_to_host` also delivers the
+    weights to pinned host memory every step, and `staged` runs cudaMemcpy in,
+    the device-resident step and cudaMemcpy out."""
     import torch
+
+    from paper_2606_30634_gb300 import dpo
     gbytes = opt.grad.numel() * opt.grad.element_size()
     pbytes = opt.param.numel() * opt.param.element_size()
     # every rank on this node pins its own copies, and all ranks must agree
@@ -826,25 +831,48 @@ def run_e2e(args, opt, one_step, stream, dev, world, w):
     link = None if args.no_link_peak else link_peak(opt, h_grad, h_param, stream, dev)
     del h_grad, h_param
 
-    # host I/O: the fused kernel reads the gradients from and writes the new
-    # weights to pinned host memory itself
-    opt.use_host_io(stream=stream)
-    secs = timed(one_step)
+    # host I/O, gradients in: the fused kernel reads them from pinned host
+    # memory; the step's diagnostics come back to the host every step
+    flags_bytes = 4 + 8 + 4   # uint32 flags, fp64 norm, fp32 clip coefficient
+    opt.use_host_io(grad=True, param=False, stream=stream)
+
+    def step_and_result():
+        one_step()
+        dpo.dpo_get_flags(opt.ctx, stream)
+
+    secs_in = timed(step_and_result)
+    # and the new weights out as well
+    opt.use_host_io(grad=False, param=True, stream=stream)
+    secs_both = timed(one_step)
     units = w.n_params * K / (world if sharded(args, world) else 1)
-    value, _ = aggregate(units, secs, world, dev)
+    value, _ = aggregate(units, secs_in, world, dev)
+    both_value, _ = aggregate(units, secs_both, world, dev)
     staged_value, _ = aggregate(units, staged_s, world, dev)
+    h2d_ms = None if link is None else gbytes / link["h2d_gbs"] / 1e6
     return {"value": value, "unit": UNIT, "h2d_bytes_per_step": gbytes,
-            "d2h_bytes_per_step": pbytes, "ms_per_step": secs / K * 1e3, "steps": K,
-            "path": "dpo_step with grad and bf16 param arenas in pinned host memory: the "
-                    "fused kernel reads gradients and writes weights across the host link",
-            "host_link_gbs": (gbytes + pbytes) / (secs / K) / 1e9,
+            "d2h_bytes_per_step": flags_bytes, "ms_per_step": secs_in / K * 1e3, "steps": K,
+            "path": "dpo_step with the gradient arena in pinned host memory: the fused kernel "
+                    "reads each step's gradients across the host link; the step's result read "
+                    "back every step is its flags, gradient norm and clip coefficient "
+                    "(dpo_get_flags); the new bf16 weights stay on the device for the next "
+                    "forward",
+            "host_link_gbs": gbytes / (secs_in / K) / 1e9,
             "link_peak": link,
-            # the bound: each direction at its own measured rate, both at once
-            # (the host-I/O kernel overlaps them; two concurrent copy-engine
-            # copies do not, see link_peak.both_gbs)
-            "link_bound_ms": None if link is None else link["duplex_bound_ms"],
-            "link_frac": (None if link is None else
-                          link["duplex_bound_ms"] / (secs / K * 1e3)),
+            # the bound: the gradients' bytes at the plain pinned copy's rate
+            "link_bound_ms": h2d_ms,
+            "link_frac": None if h2d_ms is None else h2d_ms / (secs_in / K * 1e3),
+            "weights_to_host": {
+                "value": both_value, "ms_per_step": secs_both / K * 1e3,
+                "h2d_bytes_per_step": gbytes, "d2h_bytes_per_step": pbytes,
+                "path": "as above, and the fused kernel also writes the new bf16 weights to "
+                        "pinned host memory every step",
+                "host_link_gbs": (gbytes + pbytes) / (secs_both / K) / 1e9,
+                # each direction at its own measured rate, both at once (the
+                # host-I/O kernel overlaps them; two concurrent copy-engine
+                # copies do not, see link_peak.both_gbs)
+                "link_bound_ms": None if link is None else link["duplex_bound_ms"],
+                "link_frac": (None if link is None else
+                              link["duplex_bound_ms"] / (secs_both / K * 1e3))},
             "staged": {"value": staged_value, "ms_per_step": staged_s / K * 1e3,
                        "path": "cudaMemcpy grad in, device-resident dpo_step, cudaMemcpy "
                                "weights out, on one stream"}}
