@@ -338,12 +338,16 @@ def test_launch_geometry_lion_with_history(cuda_device, stash_mode, per_sm):
         run.close()
 
 
-@pytest.mark.parametrize("host_grad,host_param", [(True, True), (True, False), (False, True)])
-def test_host_io_parity(cuda_device, host_grad, host_param):
+@pytest.mark.parametrize("host_grad,host_param,stash_mode", [
+    (True, True, dpo.DPO_STASH_COPY), (True, False, dpo.DPO_STASH_COPY),
+    (False, True, dpo.DPO_STASH_COPY), (True, False, dpo.DPO_STASH_PINGPONG)])
+def test_host_io_parity(cuda_device, host_grad, host_param, stash_mode):
     """Gradients read from and/or bf16 weights written to pinned host memory
-    by the fused kernel itself (no staging copy): same results."""
+    by the fused kernel itself (no staging copy): same results. Gradients in
+    host memory also with the ping-pong stash (the end-to-end benchmark's
+    configuration: the weights stay on the device)."""
     run = Run(Case(RAGGED, stash_dtype=B, ef=True, max_grad_norm=0.3, host_grad=host_grad,
-                   host_param=host_param), cuda_device)
+                   host_param=host_param, stash_mode=stash_mode), cuda_device)
     try:
         assert run.gpu.grad.is_cuda != host_grad and run.gpu.param.is_cuda != host_param
         for k in range(1, 5):
