@@ -232,3 +232,28 @@ def test_calls_on_null_context():
     assert L.dpo_get_step(None, ctypes.byref(k)) == dpo.DPO_EINVAL
     assert L.dpo_set_step(None, 3) == dpo.DPO_EINVAL
     L.dpo_destroy(None)
+
+
+@pytest.mark.parametrize("program", ["consumer", "muon_consumer"])
+def test_headers_serve_a_plain_c_program(program, tmp_path):
+    """include/dpo.h and include/dpo_muon.h compile as C11 (no C++), and a C
+    program using them links against libdpo.so: the GPU tests run the same
+    programs (tests/test_c_consumer.py)."""
+    import shutil
+    import subprocess
+    cc = os.environ.get("CC", "gcc")
+    nvcc = shutil.which("nvcc")
+    if shutil.which(cc) is None or nvcc is None:
+        pytest.skip("no C compiler or CUDA toolkit")
+    cuda = os.path.dirname(os.path.dirname(nvcc))
+    here = os.path.dirname(os.path.abspath(__file__))
+    lib = pkg_build.build()["libdpo.so"]
+    exe = str(tmp_path / program)
+    r = subprocess.run([cc, "-std=c11", "-O2", "-Wall", "-Wextra", "-Werror", "-pedantic",
+                        "-I", os.path.join(os.path.dirname(here), "include"),
+                        "-I", os.path.join(cuda, "include"),
+                        os.path.join(here, "c_abi", program + ".c"), "-o", exe, lib,
+                        "-L", os.path.join(cuda, "lib64"), "-lcudart"],
+                       capture_output=True, text=True)
+    assert r.returncode == 0, r.stdout + r.stderr
+    assert os.path.getsize(exe) > 0
