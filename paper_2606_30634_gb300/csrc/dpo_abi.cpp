@@ -211,7 +211,7 @@ bool dc_on(const dpo_ctx *c)
 //                      standard rule   with an update history (EF, SAPipe)
 //   AdamW, NAdam, Lion       4                     3
 //   Adan                     3                     3
-//   SAPipe updated state     -                     4
+//   SAPipe updated state     -                     4 (Lion, Adan: 3)
 //   Lion, ping-pong stash    4                     5
 // the same with the copying and the ping-pong stash, except Lion with an
 // update history: without the stash store its packets carry too few bytes
@@ -221,7 +221,10 @@ bool dc_on(const dpo_ctx *c)
 // of loads in flight per SM; the standard rule loads less per packet and
 // wants a fourth; Adan's two extra state streams make three enough; the
 // SAPipe prediction's second Adam evaluation spaces the loads out and wants
-// four. A table whose tensors mostly skip the history (DPO_SYNC, as WPipe's
+// four (AdamW: 4 CTAs 98.1%, 3 88.1%; NAdam: 4 97.5%, 3 89.9%), but not
+// Lion's, whose prediction is a sign, nor Adan's, whose packets already
+// carry the two extra streams (on one box, 3 CTAs against 4: Lion 98.3%
+// against 95.3%, Adan 97.6% against 94.0%). A table whose tensors mostly skip the history (DPO_SYNC, as WPipe's
 // synchronous half) takes the standard rule's figure (measured: 4 CTAs 96.2%,
 // 3 CTAs 93.7% of the copy peak with half the tensors synchronous).
 int set_step_grid(dpo_ctx *c)
@@ -241,7 +244,7 @@ int set_step_grid(dpo_ctx *c)
     const bool mostly_hist = 4 * hist_elems >= 3 * c->total_elems && hist_elems > 0;
     int want;
     if (corr == dpo::kCorrSapipeUpdated)
-        want = 4;
+        want = c->hp.optimizer == DPO_OPT_LION || c->hp.optimizer == DPO_OPT_ADAN ? 3 : 4;
     else if (c->hp.optimizer == DPO_OPT_ADAN)
         want = 3;
     else if (c->hp.optimizer == DPO_OPT_LION && pingpong_on(c) && mostly_hist)
