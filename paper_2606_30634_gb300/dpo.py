@@ -313,8 +313,12 @@ class DelayedAdamW:
 
     Arenas (torch tensors on the device): master, m, v (fp32), grad (grad
     dtype), param (bf16, only with param_dtype BF16), stash (stash dtype,
-    delay 1), ef (fp32, when ``ef`` is set). ``x0`` fills the master before
-    dpo_init(FRESH); pass ``init_mode=DPO_INIT_RESUME`` to start from arenas
+    delay 1), ef (fp32, when ``ef`` is set). Each tensor occupies a slice of
+    every arena (``layout.offsets``), padded to a multiple of ALIGN_ELEMS.
+    ``x0``, the fp32 start weights, fills the master before dpo_init(FRESH):
+    a sequence with one tensor per parameter tensor, their plain
+    concatenation (``sum(numels)`` elements), or a tensor in the arena layout
+    (``layout.total`` elements). Pass ``init_mode=DPO_INIT_RESUME`` to start from arenas
     restored by ``load_state``. ``ef`` allocates the update-history buffer the
     staleness ``correction`` (DPO_CORR_*) uses. With ``host_grad`` / ``host_param`` the grad /
     param arenas are pinned host memory instead, which the fused kernel reads
@@ -353,7 +357,7 @@ class DelayedAdamW:
         self.stash = alloc(tdt[stash_dtype]) if keep_stash else None
         self.ef = alloc(torch.float32) if ef else None
         if x0 is not None:
-            self.master.copy_(x0)
+            self._fill_master(x0)
         self.hp = dpo_hparams(beta1, beta2, eps, weight_decay, ef_lambda if ef else 0.0,
                               max_grad_norm, delay, correction, optimizer, beta3,
                               momentum_decay, dc_lambda, stash_mode)
@@ -411,6 +415,28 @@ class DelayedAdamW:
     def view(self, arena, i: int):
         off, cnt = self.layout.offsets[i], self.layout.numels[i]
         return arena[off:off + cnt]
+
+    def _fill_master(self, x0) -> None:
+        """Copy start weights into the master arena (see the class notes for
+        the forms ``x0`` may take)."""
+        lay = self.layout
+        if isinstance(x0, (list, tuple)):
+            if len(x0) != len(lay.numels):
+                raise ValueError(f"x0 has {len(x0)} tensors for {len(lay.numels)}")
+            for i, t in enumerate(x0):
+                self.view(self.master, i).copy_(t.reshape(-1))
+            return
+        flat = x0.reshape(-1)
+        if flat.numel() == lay.total:
+            self.master.copy_(flat)
+        elif flat.numel() == sum(lay.numels):
+            start = 0
+            for i, n in enumerate(lay.numels):
+                self.view(self.master, i).copy_(flat[start:start + n])
+                start += n
+        else:
+            raise ValueError(f"x0 has {flat.numel()} elements: expected {sum(lay.numels)} "
+                             f"(the tensors one after another) or {lay.total} (arena layout)")
 
     def grads(self, i: int):
         return self.view(self.grad, i)

@@ -739,3 +739,25 @@ def test_capturable_step_replays_in_a_cuda_graph(cuda_device, name, case, n_sync
     finally:
         eager.close()
         cap.close()
+
+
+def test_start_weights_in_every_form(cuda_device):
+    """x_0 given per tensor, as the tensors' plain concatenation, or in the
+    arena layout gives the same start state; any other length is refused."""
+    numels = [1000, 3, 517]
+    x = torch.randn(sum(numels), dtype=torch.float32, device=cuda_device)
+    parts = list(torch.split(x, numels))
+    built = [dpo.DelayedAdamW(numels, ef=True, stash_dtype=B, device=cuda_device, x0=x0)
+             for x0 in (parts, x)]
+    arena = built[1].master.clone()
+    built.append(dpo.DelayedAdamW(numels, ef=True, stash_dtype=B, device=cuda_device, x0=arena))
+    try:
+        for o in built:
+            for i in range(len(numels)):
+                assert torch.equal(o.view(o.master, i), parts[i])
+                assert torch.equal(o.view(o.param, i), parts[i].to(torch.bfloat16))
+        with pytest.raises(ValueError):
+            dpo.DelayedAdamW(numels, device=cuda_device, x0=x[:-1])
+    finally:
+        for o in built:
+            o.close()
