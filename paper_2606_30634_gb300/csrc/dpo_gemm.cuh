@@ -503,10 +503,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         // lane l loads granule l % 4 (8 columns) of rows l / 4 + 8 i of the
         // warp's 32 x 32 chunk, 8 rows of 64 bytes per instruction; the chunk
         // is then turned through its staging buffer so that each lane holds
-        // its own row. Loads of each lane's own row touched 32 lines per
-        // instruction, and where K is short (768) their L1 wavefronts, about
-        // two thirds of a tile's MMA time per SM, held the epilogue back.
-        // C is never the launch's output.
+        // its own row. Loading each lane's own row instead touched 32 lines
+        // per instruction; where K is short (768) that made the chain 6 %
+        // slower on GB300, and where K is long the epilogue is hidden behind
+        // the MMAs either way. C is never the launch's output.
         constexpr int kCPre = 4;
         const int crs = lane >> 2, cg = lane & 3;   // coalesced load: sub-row, granule
         int lt = 0, staged = 0;
