@@ -36,9 +36,9 @@
  * systems). The fused kernel then reads the gradients from and writes the new
  * weights to host memory itself, over the host link, with no staging copy;
  * the step is then bound by that link (2 B per parameter each way for bf16).
- * The host must not touch those buffers while a step is in flight. The library owns only its context: a device copy of the tensor
- * table and a few hundred bytes of device scratch per SM for the gradient
- * norm. All launches go to the stream passed in (a cudaStream_t, NULL for the
+ * The host must not touch those buffers while a step is in flight. The
+ * library owns only its context: a device copy of the tensor table and a few
+ * hundred bytes of device scratch per SM for the gradient norm. All launches go to the stream passed in (a cudaStream_t, NULL for the
  * legacy default stream); dpo_step never synchronizes the host.
  *
  * Errors. Every call returns DPO_OK (0) or a negative DPO_E* code; nothing
