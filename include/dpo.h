@@ -38,8 +38,9 @@
  * the step is then bound by that link (2 B per parameter each way for bf16).
  * The host must not touch those buffers while a step is in flight. The
  * library owns only its context: a device copy of the tensor table and a few
- * hundred bytes of device scratch per SM for the gradient norm. All launches go to the stream passed in (a cudaStream_t, NULL for the
- * legacy default stream); dpo_step never synchronizes the host.
+ * hundred bytes of device scratch per SM for the gradient norm. All launches
+ * go to the stream passed in (a cudaStream_t, NULL for the legacy default
+ * stream); dpo_step never synchronizes the host.
  *
  * Errors. Every call returns DPO_OK (0) or a negative DPO_E* code; nothing
  * aborts. dpo_last_error gives a message for the last failing call on a
